@@ -1,0 +1,307 @@
+"""CPU oracle for the batched ad hoc teamwork rollout path -- TEST INFRASTRUCTURE ONLY.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline and
+``--impl reference`` legs may import this package.  The product package
+(``paper_2609_13716_gb300``) never imports it and shares no code with it.
+
+The C++ source (``aht_oracle.cpp``) is compiled on first use into ``oracle/_build``
+with plain ``g++ -O2 -ffp-contract=off`` (no intrinsics, no fast-math), so fp32 reward
+arithmetic is IEEE single on x86-64 and aarch64 alike.  This module only marshals
+arguments; every step of the oracle's arithmetic lives in the C++ file.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_BUILD = os.path.join(_HERE, "_build")
+_SO = os.path.join(_BUILD, "liboracle.so")
+_SRC = [os.path.join(_HERE, "aht_oracle.cpp")]
+_HDR = os.path.join(_HERE, "aht_oracle.h")
+_lock = threading.Lock()
+_lib = None
+
+LBF, OVERCOOKED, HANABI = 0, 1, 2
+STREAM_ACT0, STREAM_ACT1, STREAM_RESET, STREAM_TEAMMATE = 0, 1, 2, 3
+STATE_BYTES = 768
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle shared library (g++, seconds).  Returns its path."""
+    os.makedirs(_BUILD, exist_ok=True)
+    newest = max(os.path.getmtime(p) for p in _SRC + [_HDR])
+    if not force and os.path.exists(_SO) and os.path.getmtime(_SO) >= newest:
+        return _SO
+    tmp = _SO + f".{os.getpid()}.tmp"
+    cmd = ["g++", "-std=c++17", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fPIC",
+           "-shared", "-pthread", "-Wall", "-o", tmp] + _SRC
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _SO)
+    return _SO
+
+
+class EnvDesc(C.Structure):
+    _fields_ = [("kind", C.c_int32), ("width", C.c_int32), ("height", C.c_int32),
+                ("n_food", C.c_int32), ("max_agent_level", C.c_int32),
+                ("episode_len", C.c_int32), ("cook_time", C.c_int32),
+                ("soup_reward", C.c_int32)]
+
+
+class LbfState(C.Structure):
+    _fields_ = [("ax", C.c_int32 * 2), ("ay", C.c_int32 * 2), ("al", C.c_int32 * 2),
+                ("fx", C.c_int32 * 3), ("fy", C.c_int32 * 3), ("fl", C.c_int32 * 3),
+                ("eaten", C.c_int32 * 3), ("F", C.c_int32), ("ep_t", C.c_int32),
+                ("done", C.c_int32), ("ret", C.c_float)]
+
+
+class OcState(C.Structure):
+    _fields_ = [("ax", C.c_int32 * 2), ("ay", C.c_int32 * 2), ("face", C.c_int32 * 2),
+                ("held", C.c_int32 * 2), ("pot_n", C.c_int32), ("pot_timer", C.c_int32),
+                ("counter_item", C.c_int32 * 20), ("ep_t", C.c_int32), ("done", C.c_int32),
+                ("ret", C.c_float)]
+
+
+class HanabiState(C.Structure):
+    _fields_ = [("deck", C.c_int32 * 50), ("ptr", C.c_int32),
+                ("hand", (C.c_int32 * 5) * 2), ("n_hand", C.c_int32 * 2),
+                ("know", (C.c_uint32 * 5) * 2), ("hint_col", (C.c_uint32 * 5) * 2),
+                ("hint_rank", (C.c_uint32 * 5) * 2), ("fw", C.c_int32 * 5),
+                ("info", C.c_int32), ("lives", C.c_int32), ("score", C.c_int32),
+                ("disc", C.c_int32 * 25), ("fr", C.c_int32), ("turn", C.c_int32),
+                ("la_valid", C.c_int32), ("la_actor", C.c_int32), ("la_type", C.c_int32),
+                ("la_colour", C.c_int32), ("la_rank", C.c_int32), ("la_slot", C.c_int32),
+                ("la_card", C.c_int32), ("la_hinted", C.c_int32), ("la_success", C.c_int32),
+                ("la_bomb", C.c_int32), ("done", C.c_int32), ("ret", C.c_float)]
+
+
+class Mlp(C.Structure):
+    _fields_ = [("obs_dim", C.c_int32), ("h0", C.c_int32), ("h1", C.c_int32),
+                ("n_out", C.c_int32),
+                ("W1", C.POINTER(C.c_double)), ("b1", C.POINTER(C.c_double)),
+                ("W2", C.POINTER(C.c_double)), ("b2", C.POINTER(C.c_double)),
+                ("W3", C.POINTER(C.c_double)), ("b3", C.POINTER(C.c_double))]
+
+
+_P = C.c_void_p
+
+
+class RolloutIO(C.Structure):
+    _fields_ = [("seed", C.c_uint64), ("n_envs", C.c_int64), ("step0", C.c_int64),
+                ("T", C.c_int32), ("ego_id", C.c_int32), ("pool", _P), ("pool_size", C.c_int32),
+                ("forced", _P), ("states", _P), ("n_threads", C.c_int32),
+                ("teammate", _P), ("obs", _P), ("obs_tm", _P), ("actions", _P),
+                ("own_actions", _P), ("margin", _P), ("logits", _P), ("logp", _P),
+                ("values", _P), ("rewards", _P), ("dones", _P), ("last_value", _P)]
+
+
+class XplayIO(C.Structure):
+    _fields_ = [("seed", C.c_uint64), ("step0", C.c_int64), ("ego_ids", _P),
+                ("n_ego", C.c_int32), ("tm_ids", _P), ("n_tm", C.c_int32),
+                ("envs_per_pair", C.c_int32), ("max_steps", C.c_int32), ("forced", _P),
+                ("n_threads", C.c_int32), ("returns", _P), ("steps", _P), ("actions", _P),
+                ("own_actions", _P), ("margin", _P), ("matrix", _P)]
+
+
+def lib() -> C.CDLL:
+    global _lib
+    with _lock:
+        if _lib is None:
+            L = C.CDLL(build())
+            L.orc_philox4x32_10.argtypes = [C.c_uint32, C.c_uint32, _P, _P]
+            L.orc_draw.argtypes = [C.c_uint64, C.c_uint32, C.c_uint32, C.c_uint32, C.c_uint32]
+            L.orc_draw.restype = C.c_uint32
+            L.orc_uniform_int.argtypes = [C.c_uint32, C.c_uint32]
+            L.orc_uniform_int.restype = C.c_uint32
+            L.orc_u01.argtypes = [C.c_uint32]
+            L.orc_u01.restype = C.c_double
+            for f in ("orc_obs_dim", "orc_n_actions", "orc_check_desc"):
+                getattr(L, f).argtypes = [C.POINTER(EnvDesc)]
+                getattr(L, f).restype = C.c_int32
+            L.orc_lbf_reset.argtypes = [C.POINTER(EnvDesc), C.c_uint64, C.c_uint32, C.c_uint32, C.POINTER(LbfState)]
+            L.orc_lbf_step.argtypes = [C.POINTER(EnvDesc), C.POINTER(LbfState), C.c_int32, C.c_int32, _P, _P]
+            L.orc_lbf_step.restype = C.c_int32
+            L.orc_lbf_obs.argtypes = [C.POINTER(EnvDesc), C.POINTER(LbfState), C.c_int32, _P]
+            L.orc_oc_cell.argtypes = [C.c_int32, C.c_int32]
+            L.orc_oc_cell.restype = C.c_int32
+            L.orc_oc_reset.argtypes = [C.POINTER(EnvDesc), C.POINTER(OcState)]
+            L.orc_oc_step.argtypes = [C.POINTER(EnvDesc), C.POINTER(OcState), C.c_int32, C.c_int32, _P, _P]
+            L.orc_oc_step.restype = C.c_int32
+            L.orc_oc_obs.argtypes = [C.POINTER(EnvDesc), C.POINTER(OcState), C.c_int32, _P]
+            L.orc_hanabi_reset.argtypes = [C.c_uint64, C.c_uint32, C.c_uint32, C.POINTER(HanabiState)]
+            L.orc_hanabi_legal.argtypes = [C.POINTER(HanabiState), _P]
+            L.orc_hanabi_step.argtypes = [C.POINTER(HanabiState), C.c_int32, _P]
+            L.orc_hanabi_step.restype = C.c_int32
+            L.orc_hanabi_obs.argtypes = [C.POINTER(HanabiState), C.c_int32, _P]
+            L.orc_mlp_forward.argtypes = [C.POINTER(Mlp), _P, _P]
+            L.orc_sample.argtypes = [_P, _P, C.c_int32, C.c_double, _P, _P, _P]
+            L.orc_logp.argtypes = [_P, _P, C.c_int32, C.c_int32]
+            L.orc_logp.restype = C.c_double
+            L.orc_gae.argtypes = [_P, _P, _P, _P, C.c_int64, C.c_int32, C.c_double, C.c_double, _P, _P]
+            L.orc_rollout.argtypes = [C.POINTER(EnvDesc), C.POINTER(Mlp), C.c_int32, C.POINTER(RolloutIO)]
+            L.orc_rollout.restype = C.c_int32
+            L.orc_reset_all.argtypes = [C.POINTER(EnvDesc), C.c_uint64, C.c_int64, C.c_int64, _P]
+            L.orc_reset_all.restype = C.c_int32
+            L.orc_step_forced.argtypes = [C.POINTER(EnvDesc), C.c_uint64, C.c_int64, C.c_int64, _P, _P, _P, _P, _P, _P]
+            L.orc_step_forced.restype = C.c_int32
+            L.orc_xplay.argtypes = [C.POINTER(EnvDesc), C.POINTER(Mlp), C.c_int32, C.POINTER(XplayIO)]
+            L.orc_xplay.restype = C.c_int32
+            L.orc_policy_outputs.argtypes = [C.POINTER(Mlp), _P, C.c_int64, _P]
+            _lib = L
+    return _lib
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(C.c_void_p)
+
+
+# ---------------------------------------------------------------------------------
+# Thin marshalling helpers.
+# ---------------------------------------------------------------------------------
+def env_desc(kind, width=0, height=0, n_food=0, max_agent_level=0, episode_len=0,
+             cook_time=0, soup_reward=0) -> EnvDesc:
+    return EnvDesc(kind, width, height, n_food, max_agent_level, episode_len, cook_time,
+                   soup_reward)
+
+
+def obs_dim(d: EnvDesc) -> int:
+    return lib().orc_obs_dim(C.byref(d))
+
+
+def n_actions(d: EnvDesc) -> int:
+    return lib().orc_n_actions(C.byref(d))
+
+
+def philox(key, ctr):
+    out = np.zeros(4, np.uint32)
+    c = np.asarray(ctr, np.uint32)
+    lib().orc_philox4x32_10(int(key[0]), int(key[1]), _ptr(c), _ptr(out))
+    return out
+
+
+def draw(seed, env, step, stream, n):
+    return lib().orc_draw(seed, env, step, stream, n)
+
+
+class Policies:
+    """fp64 copies of a population's weights (exact for fp32 and bf16 inputs)."""
+
+    def __init__(self, layers):
+        # layers: list per policy of [(W1, b1), (W2, b2), (W3, b3)], any float dtype.
+        self._keep = []
+        arr = (Mlp * len(layers))()
+        for p, pol in enumerate(layers):
+            ws = [np.ascontiguousarray(np.asarray(a, dtype=np.float64)) for wb in pol for a in wb]
+            self._keep.append(ws)
+            W1, b1, W2, b2, W3, b3 = ws
+            dp = C.POINTER(C.c_double)
+            arr[p] = Mlp(W1.shape[1], W1.shape[0], W2.shape[0], W3.shape[0],
+                         W1.ctypes.data_as(dp), b1.ctypes.data_as(dp),
+                         W2.ctypes.data_as(dp), b2.ctypes.data_as(dp),
+                         W3.ctypes.data_as(dp), b3.ctypes.data_as(dp))
+        self.arr = arr
+        self.n = len(layers)
+
+    def outputs(self, pid, obs_u8):
+        obs_u8 = np.ascontiguousarray(obs_u8, np.uint8)
+        n = obs_u8.shape[0]
+        out = np.zeros((n, self.arr[pid].n_out), np.float64)
+        lib().orc_policy_outputs(C.byref(self.arr[pid]), _ptr(obs_u8), n, _ptr(out))
+        return out
+
+
+def sample(z, legal, u):
+    z = np.ascontiguousarray(z, np.float64)
+    legal = np.ascontiguousarray(legal, np.uint8)
+    a = C.c_int32()
+    lp = C.c_double()
+    mg = C.c_double()
+    lib().orc_sample(_ptr(z), _ptr(legal), len(z), float(u), C.byref(a), C.byref(lp), C.byref(mg))
+    return a.value, lp.value, mg.value
+
+
+def gae(r, v, d, v_last, gamma, lam):
+    r = np.ascontiguousarray(r, np.float32)
+    v = np.ascontiguousarray(v, np.float32)
+    d = np.ascontiguousarray(d, np.uint8)
+    v_last = np.ascontiguousarray(v_last, np.float32)
+    T, N = r.shape
+    adv = np.zeros((T, N), np.float64)
+    tgt = np.zeros((T, N), np.float64)
+    lib().orc_gae(_ptr(r), _ptr(v), _ptr(d), _ptr(v_last), N, T, gamma, lam, _ptr(adv), _ptr(tgt))
+    return adv, tgt
+
+
+def new_states(n):
+    return np.zeros((n, STATE_BYTES), np.uint8)
+
+
+def reset_all(d, seed, n, step=0):
+    st = new_states(n)
+    rc = lib().orc_reset_all(C.byref(d), seed, n, step, _ptr(st))
+    assert rc == 0, rc
+    return st
+
+
+def step_forced(d, seed, step, states, actions):
+    n = states.shape[0]
+    od = obs_dim(d)
+    actions = np.ascontiguousarray(actions, np.uint8)
+    rew2 = np.zeros((n, 2), np.float32)
+    team = np.zeros(n, np.float32)
+    dones = np.zeros(n, np.uint8)
+    obs2 = np.zeros((n, 2, od), np.uint8)
+    rc = lib().orc_step_forced(C.byref(d), seed, n, step, _ptr(states), _ptr(actions),
+                               _ptr(rew2), _ptr(team), _ptr(dones), _ptr(obs2))
+    return rc, rew2, team, dones, obs2
+
+
+def rollout(d, pols: Policies, seed, states, step0, T, ego_id, pool, forced=None, n_threads=1):
+    """PPO collection.  Returns a dict of numpy arrays; states are updated in place."""
+    N = states.shape[0]
+    od = obs_dim(d)
+    K = n_actions(d)
+    n_out = pols.arr[ego_id].n_out
+    pool = np.ascontiguousarray(pool, np.int32)
+    out = dict(
+        teammate=np.zeros(N, np.int32), obs=np.zeros((T, N, od), np.uint8),
+        obs_tm=np.zeros((T, N, od), np.uint8), actions=np.zeros((T, N, 2), np.uint8),
+        own_actions=np.zeros((T, N, 2), np.uint8), margin=np.zeros((T, N, 2), np.float64),
+        logits=np.zeros((T, N, n_out), np.float64), logp=np.zeros((T, N), np.float64),
+        values=np.zeros((T, N), np.float64), rewards=np.zeros((T, N), np.float32),
+        dones=np.zeros((T, N), np.uint8), last_value=np.zeros(N, np.float64))
+    if forced is not None:
+        forced = np.ascontiguousarray(forced, np.uint8)
+        assert forced.shape == (T, N, 2)
+    io = RolloutIO(seed=seed, n_envs=N, step0=step0, T=T, ego_id=ego_id, pool=_ptr(pool),
+                   pool_size=len(pool), forced=_ptr(forced), states=_ptr(states),
+                   n_threads=n_threads, **{k: _ptr(v) for k, v in out.items()})
+    rc = lib().orc_rollout(C.byref(d), pols.arr, pols.n, C.byref(io))
+    out["rc"] = rc
+    return out
+
+
+def xplay(d, pols: Policies, seed, step0, ego_ids, tm_ids, P, max_steps, forced=None,
+          n_threads=1, record=True):
+    ego_ids = np.ascontiguousarray(ego_ids, np.int32)
+    tm_ids = np.ascontiguousarray(tm_ids, np.int32)
+    N = len(ego_ids) * len(tm_ids) * P
+    out = dict(returns=np.zeros(N, np.float32), steps=np.zeros(N, np.int32),
+               matrix=np.zeros((len(ego_ids), len(tm_ids)), np.float32))
+    if record:
+        out.update(actions=np.zeros((max_steps, N, 2), np.uint8),
+                   own_actions=np.zeros((max_steps, N, 2), np.uint8),
+                   margin=np.zeros((max_steps, N, 2), np.float64))
+    if forced is not None:
+        forced = np.ascontiguousarray(forced, np.uint8)
+    io = XplayIO(seed=seed, step0=step0, ego_ids=_ptr(ego_ids), n_ego=len(ego_ids),
+                 tm_ids=_ptr(tm_ids), n_tm=len(tm_ids), envs_per_pair=P, max_steps=max_steps,
+                 forced=_ptr(forced), n_threads=n_threads,
+                 **{k: _ptr(v) for k, v in out.items()})
+    rc = lib().orc_xplay(C.byref(d), pols.arr, pols.n, C.byref(io))
+    out["rc"] = rc
+    return out

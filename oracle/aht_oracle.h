@@ -1,0 +1,221 @@
+/*
+ * aht_oracle.h -- plain, slow CPU oracle for the batched ad hoc teamwork rollout path.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and bench.py's
+ * cpu_baseline / --impl reference legs may load this library.  The product path
+ * (paper_2609_13716_gb300/) never links, imports or calls it, and the two share no
+ * code: no headers, helpers, tables or constants.
+ *
+ * What it computes (the paper is JaxAHT, "A JAX-Based Library for Ad Hoc Teamwork"):
+ *   - the Dec-POMDP step of Sec. 3 (joint action -> next state, per-agent
+ *     observation, one shared team reward) for three games: Level-Based Foraging,
+ *     a 5x4 Overcooked-style kitchen and 2-player Hanabi (Sec. 4, Table
+ *     "JaxAHT Environments").  The paper gives no game rules; the rules here are
+ *     the readings listed in DESIGN.md ("Readings"), written from the workload
+ *     descriptions;
+ *   - the decentralised MLP policy pi_i(a | o_i) (Sec. 3) in fp64 from exact weights,
+ *     masked categorical sampling (App. B, masked categorical) in fp64;
+ *   - PPO's generalised advantage estimate (App. C, "PPO ego") in fp64;
+ *   - the ego-by-teammate cross-play return matrix (App. B, "Cross-play matrix
+ *     construction"; Sec. 3 J_AHT as its row mean).
+ * Randomness is Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11) keyed by the seed,
+ * with counter (env, step, stream, block).
+ *
+ * All functions are re-entrant.  Array arguments are caller-owned host memory.
+ */
+#ifndef AHT_ORACLE_H
+#define AHT_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- randomness --------------------------------------------------------------- */
+enum { ORC_STREAM_ACT0 = 0, ORC_STREAM_ACT1 = 1, ORC_STREAM_RESET = 2, ORC_STREAM_TEAMMATE = 3 };
+
+/* One Philox4x32-10 block: key (k0, k1), counter ctr[4] -> out[4]. */
+void orc_philox4x32_10(uint32_t k0, uint32_t k1, const uint32_t ctr[4], uint32_t out[4]);
+/* Draw n of the (env, step, stream) tuple: word n%4 of block n/4, key = (seed lo, seed hi),
+ * counter = (env, step, stream, n/4). */
+uint32_t orc_draw(uint64_t seed, uint32_t env, uint32_t step, uint32_t stream, uint32_t n);
+/* floor(x * n / 2^32): an integer in [0, n). */
+uint32_t orc_uniform_int(uint32_t x, uint32_t n);
+/* (x >> 8) * 2^-24: a double in [0, 1) exactly representable in fp32. */
+double orc_u01(uint32_t x);
+
+/* ---- environment description ------------------------------------------------------ */
+enum { ORC_LBF = 0, ORC_OVERCOOKED = 1, ORC_HANABI = 2 };
+typedef struct orc_env_desc {
+  int32_t kind;            /* ORC_LBF / ORC_OVERCOOKED / ORC_HANABI */
+  int32_t width, height;   /* LBF grid (3..12); Overcooked 5x4; Hanabi ignored */
+  int32_t n_food;          /* LBF 1..3 */
+  int32_t max_agent_level; /* LBF agent levels are uniform in 1..max_agent_level */
+  int32_t episode_len;     /* LBF / Overcooked step limit; Hanabi 0 = run to termination */
+  int32_t cook_time;       /* Overcooked steps a full pot cooks */
+  int32_t soup_reward;     /* Overcooked team reward per delivered soup */
+} orc_env_desc;
+
+int32_t orc_obs_dim(const orc_env_desc* d);
+int32_t orc_n_actions(const orc_env_desc* d);
+/* 0 if the description is valid, else a negative code. */
+int32_t orc_check_desc(const orc_env_desc* d);
+
+/* ---- Level-Based Foraging -------------------------------------------------------- */
+enum { ORC_LBF_MAX_FOOD = 3 };
+typedef struct orc_lbf_state {
+  int32_t ax[2], ay[2], al[2];         /* agent position and level */
+  int32_t fx[3], fy[3], fl[3], eaten[3];
+  int32_t F;                           /* sum of spawned food levels (reward normaliser) */
+  int32_t ep_t;                        /* steps taken in this episode */
+  int32_t done;                        /* the last step ended the episode */
+  float ret;                           /* team return of this episode */
+} orc_lbf_state;
+void orc_lbf_reset(const orc_env_desc* d, uint64_t seed, uint32_t env, uint32_t step,
+                   orc_lbf_state* s);
+/* r[2] = per-agent reward, *team = fp32(r0 + r1).  Returns done (0/1). */
+int32_t orc_lbf_step(const orc_env_desc* d, orc_lbf_state* s, int32_t a0, int32_t a1,
+                     float r[2], float* team);
+void orc_lbf_obs(const orc_env_desc* d, const orc_lbf_state* s, int32_t seat, uint8_t* out);
+
+/* ---- Overcooked-style kitchen (fixed 5x4 layout) -------------------------------- */
+enum { ORC_OC_NONE = 0, ORC_OC_ONION = 1, ORC_OC_DISH = 2, ORC_OC_SOUP = 3 };
+enum { ORC_OC_FLOOR = 0, ORC_OC_COUNTER = 1, ORC_OC_ONION_D = 2, ORC_OC_POT = 3,
+       ORC_OC_DISH_D = 4, ORC_OC_SERVE = 5 };
+typedef struct orc_oc_state {
+  int32_t ax[2], ay[2], face[2], held[2]; /* face 0 N, 1 S, 2 E, 3 W */
+  int32_t pot_n, pot_timer;
+  int32_t counter_item[20];               /* item on each cell (counters only) */
+  int32_t ep_t;
+  int32_t done;
+  float ret;
+} orc_oc_state;
+int32_t orc_oc_cell(int32_t x, int32_t y); /* layout cell type */
+void orc_oc_reset(const orc_env_desc* d, orc_oc_state* s);
+int32_t orc_oc_step(const orc_env_desc* d, orc_oc_state* s, int32_t a0, int32_t a1,
+                    float r[2], float* team);
+void orc_oc_obs(const orc_env_desc* d, const orc_oc_state* s, int32_t seat, uint8_t* out);
+
+/* ---- Hanabi, 2 players ------------------------------------------------------------ */
+typedef struct orc_hanabi_state {
+  int32_t deck[50];           /* card type c*5 + (rank-1) */
+  int32_t ptr;                /* next card to draw */
+  int32_t hand[2][5];         /* card type, -1 if empty */
+  int32_t n_hand[2];
+  uint32_t know[2][5];        /* 25-bit possible-card masks */
+  uint32_t hint_col[2][5];    /* explicit colour hints received, 5 bits */
+  uint32_t hint_rank[2][5];   /* explicit rank hints received, 5 bits */
+  int32_t fw[5];              /* fireworks height per colour */
+  int32_t info, lives, score;
+  int32_t disc[25];           /* discarded count per card type */
+  int32_t fr;                 /* final-round turns left; -1 while the deck has cards */
+  int32_t turn;               /* turns taken in this episode; acting seat = turn % 2 */
+  int32_t la_valid, la_actor, la_type, la_colour, la_rank, la_slot, la_card, la_hinted,
+          la_success, la_bomb; /* last action */
+  int32_t done;
+  float ret;
+} orc_hanabi_state;
+void orc_hanabi_reset(uint64_t seed, uint32_t env, uint32_t step, orc_hanabi_state* s);
+void orc_hanabi_legal(const orc_hanabi_state* s, uint8_t legal[20]); /* for the acting seat */
+/* Applies action a of the acting seat.  Returns done (0/1), or -1 (state untouched)
+ * if a is illegal. */
+int32_t orc_hanabi_step(orc_hanabi_state* s, int32_t a, float* team);
+void orc_hanabi_obs(const orc_hanabi_state* s, int32_t seat, uint8_t* out);
+
+/* ---- generic env state ------------------------------------------------------------ */
+enum { ORC_STATE_BYTES = 768 };   /* >= sizeof of every state struct above */
+typedef struct orc_state { uint8_t bytes[ORC_STATE_BYTES]; } orc_state;
+
+/* ---- policy MLP ------------------------------------------------------------------ */
+typedef struct orc_mlp {
+  int32_t obs_dim, h0, h1, n_out; /* n_out = n_actions, + 1 if a value row is present */
+  const double *W1, *b1;          /* [h0][obs_dim], [h0] */
+  const double *W2, *b2;          /* [h1][h0], [h1] */
+  const double *W3, *b3;          /* [n_out][h1], [n_out] */
+} orc_mlp;
+/* z = W3 tanh(W2 tanh(W1 x + b1) + b2) + b3, fp64. */
+void orc_mlp_forward(const orc_mlp* p, const double* x, double* z);
+/* Masked categorical inverse-CDF sample in fp64: a = min{k : u*Z < S_k}, with
+ * S_k = sum_{j<=k} exp(z_j - max) over legal j.  logp of a; margin = min_k |u - S_k/Z|. */
+void orc_sample(const double* z, const uint8_t* legal, int32_t K, double u,
+                int32_t* a, double* logp, double* margin);
+/* logp of a given action under the masked softmax of z. */
+double orc_logp(const double* z, const uint8_t* legal, int32_t K, int32_t a);
+
+/* ---- GAE (fp64) -------------------------------------------------------------------- */
+/* Time-major [T][N] inputs.  delta_t = r_t + g(1-d_t)V_{t+1} - V_t,
+ * A_t = delta_t + g l (1-d_t) A_{t+1}, V_T = v_last, A_T = 0; targets = A + V. */
+void orc_gae(const float* r, const float* v, const uint8_t* d, const float* v_last,
+             int64_t n_envs, int32_t T, double gamma, double lambda,
+             double* adv, double* targets);
+
+/* ---- PPO rollout collection (simultaneous-move envs) ---------------------------- */
+typedef struct orc_rollout_io {
+  /* inputs */
+  uint64_t seed;
+  int64_t n_envs;
+  int64_t step0;               /* global step counter at the start of the call */
+  int32_t T;
+  int32_t ego_id;
+  const int32_t* pool;         /* teammate policy ids */
+  int32_t pool_size;
+  const uint8_t* forced;       /* [T][N][2] actions to apply, or NULL to free-run */
+  orc_state* states;           /* [N] in/out */
+  int32_t n_threads;
+  /* outputs (each may be NULL) */
+  int32_t* teammate;           /* [N] */
+  uint8_t* obs;                /* [T][N][obs_dim] ego observation */
+  uint8_t* obs_tm;             /* [T][N][obs_dim] teammate observation */
+  uint8_t* actions;            /* [T][N][2] applied actions */
+  uint8_t* own_actions;        /* [T][N][2] the oracle's own samples */
+  double* margin;              /* [T][N][2] CDF margin of each own sample */
+  double* logits;              /* [T][N][n_out] ego outputs */
+  double* logp;                /* [T][N] ego logp of the applied action */
+  double* values;              /* [T][N] ego value (0 without a value row) */
+  float* rewards;              /* [T][N] team reward */
+  uint8_t* dones;              /* [T][N] */
+  double* last_value;          /* [N] value of the state after the last step */
+} orc_rollout_io;
+int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32_t n_pols,
+                    orc_rollout_io* io);
+
+/* Resets n_envs envs with env index 0..n-1 at the given step counter. */
+int32_t orc_reset_all(const orc_env_desc* d, uint64_t seed, int64_t n_envs, int64_t step,
+                      orc_state* states);
+/* One forced step of every env, PPO semantics (auto-reset with step+1).  Outputs the
+ * per-agent rewards [N][2], team rewards [N], dones [N] and both seats' observation of
+ * the resulting state [N][2][obs_dim]; each output may be NULL.  Hanabi applies the
+ * acting seat's action only. */
+int32_t orc_step_forced(const orc_env_desc* d, uint64_t seed, int64_t n_envs, int64_t step,
+                        orc_state* states, const uint8_t* actions, float* rewards2,
+                        float* team, uint8_t* dones, uint8_t* obs2);
+
+/* ---- cross-play evaluation ------------------------------------------------------- */
+typedef struct orc_xplay_io {
+  uint64_t seed;
+  int64_t step0;
+  const int32_t* ego_ids; int32_t n_ego;
+  const int32_t* tm_ids;  int32_t n_tm;
+  int32_t envs_per_pair;
+  int32_t max_steps;
+  const uint8_t* forced;   /* [max_steps][n_envs][2] or NULL */
+  int32_t n_threads;
+  /* outputs (each may be NULL) */
+  float* returns;          /* [n_ego][n_tm][P] team return of the first episode */
+  int32_t* steps;          /* [n_envs] active env-steps */
+  uint8_t* actions;        /* [max_steps][n_envs][2] applied actions (255 = none) */
+  uint8_t* own_actions;    /* [max_steps][n_envs][2] */
+  double* margin;          /* [max_steps][n_envs][2] (2 = no sample) */
+  float* matrix;           /* [n_ego][n_tm] mean return, fp64 sum */
+} orc_xplay_io;
+int32_t orc_xplay(const orc_env_desc* d, const orc_mlp* pols, int32_t n_pols,
+                  orc_xplay_io* io);
+
+/* Policy outputs z for n observations (u8 [n][obs_dim]) -> [n][n_out]. */
+void orc_policy_outputs(const orc_mlp* p, const uint8_t* obs, int64_t n, double* out);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

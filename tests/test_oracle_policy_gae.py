@@ -1,0 +1,176 @@
+"""Pins for the oracle's policy forward, masked categorical sampling, GAE and drivers."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_13716_gb300 import workloads as W
+
+
+def rand_policy(rng, dims, scale=0.1):
+    return [(rng.standard_normal((dims[i + 1], dims[i])) * scale,
+             rng.standard_normal(dims[i + 1]) * scale) for i in range(3)]
+
+
+def test_mlp_matches_torch_float64(orc):
+    rng = np.random.default_rng(0)
+    pol = rand_policy(rng, [196, 64, 64, 7])
+    P = orc.Policies([pol])
+    obs = rng.integers(0, 7, size=(50, 196)).astype(np.uint8)
+    got = P.outputs(0, obs)
+    x = torch.from_numpy(obs.astype(np.float64))
+    for W_, b in pol:
+        x = x @ torch.from_numpy(W_).T + torch.from_numpy(b)
+        if W_ is not pol[-1][0]:
+            x = torch.tanh(x)
+    assert np.allclose(got, x.numpy(), rtol=1e-13, atol=1e-13)
+
+
+def test_zero_weights_give_bias_and_uniform_policy(orc):
+    dims = [196, 64, 64, 6]
+    rng = np.random.default_rng(1)
+    pol = [(np.zeros((dims[i + 1], dims[i])), np.zeros(dims[i + 1])) for i in range(3)]
+    b3 = rng.standard_normal(6)
+    P = orc.Policies([pol[:2] + [(np.zeros((6, 64)), b3)]])
+    assert np.array_equal(P.outputs(0, np.ones((1, 196), np.uint8))[0], b3)
+    legal = np.ones(6, np.uint8)
+    for u in (0.0, 0.1, 0.49, 0.5, 0.83, 0.999):
+        a, lp, _ = orc.sample(np.zeros(6), legal, u)
+        assert a == int(np.floor(u * 6)) and abs(lp + np.log(6)) < 1e-15
+
+
+def test_sample_is_inverse_cdf_of_masked_softmax(orc):
+    rng = np.random.default_rng(2)
+    for _ in range(300):
+        K = int(rng.choice([6, 20]))
+        z = rng.standard_normal(K) * 3
+        legal = (rng.random(K) < 0.7).astype(np.uint8)
+        legal[rng.integers(K)] = 1
+        u = rng.random()
+        a, lp, mg = orc.sample(z, legal, u)
+        p = np.where(legal == 1, np.exp(z - z[legal == 1].max()), 0.0)
+        cdf = np.cumsum(p) / p.sum()
+        assert a == int(np.searchsorted(cdf, u, side="right"))
+        assert legal[a] == 1
+        logsm = torch.log_softmax(torch.from_numpy(np.where(legal == 1, z, -np.inf)), 0).numpy()
+        assert abs(lp - logsm[a]) < 1e-12
+        assert abs(mg - np.abs(u - cdf).min()) < 1e-12
+
+
+def test_onehot_last_layer_is_deterministic_argmax(orc):
+    dims = [196, 64, 64, 6]
+    pol = [(np.zeros((dims[i + 1], dims[i])), np.zeros(dims[i + 1])) for i in range(3)]
+    b3 = np.zeros(6)
+    b3[4] = 60.0   # a margin of e^60
+    P = orc.Policies([pol[:2] + [(np.zeros((6, 64)), b3)]])
+    z = P.outputs(0, np.zeros((1, 196), np.uint8))[0]
+    for u in np.linspace(1e-6, 0.999999, 17):   # u = 0 picks action 0 (S_0 = e^-60 > 0)
+        assert orc.sample(z, np.ones(6, np.uint8), u)[0] == 4
+
+
+def _gae_inputs(rng, T=40, N=7, p_done=0.1):
+    r = rng.standard_normal((T, N)).astype(np.float32)
+    v = rng.standard_normal((T, N)).astype(np.float32)
+    d = (rng.random((T, N)) < p_done).astype(np.uint8)
+    vl = rng.standard_normal(N).astype(np.float32)
+    return r, v, d, vl
+
+
+def test_gae_lambda_one_is_discounted_return_minus_value(orc):
+    rng = np.random.default_rng(3)
+    r, v, d, vl = _gae_inputs(rng, p_done=0.0)
+    g = 0.99
+    adv, tgt = orc.gae(r, v, d, vl, g, 1.0)
+    T = r.shape[0]
+    for t in range(T):
+        ret = sum(g ** (k - t) * r[k].astype(np.float64) for k in range(t, T)) + g ** (T - t) * vl.astype(np.float64)
+        assert np.allclose(adv[t], ret - v[t], atol=1e-11)
+        assert np.allclose(tgt[t], ret, atol=1e-11)
+
+
+def test_gae_lambda_zero_is_td_error(orc):
+    rng = np.random.default_rng(4)
+    r, v, d, vl = _gae_inputs(rng)
+    g = 0.99
+    adv, _ = orc.gae(r, v, d, vl, g, 0.0)
+    vnext = np.concatenate([v[1:], vl[None]], 0).astype(np.float64)
+    delta = r.astype(np.float64) + g * (1 - d) * vnext - v
+    assert np.allclose(adv, delta, atol=1e-13)
+
+
+def test_gae_geometric_closed_form(orc):
+    T, N, g, lam, c = 64, 3, 0.99, 0.95, 0.5
+    r = np.full((T, N), c, np.float32)
+    z = np.zeros((T, N), np.float32)
+    adv, _ = orc.gae(r, z, z.astype(np.uint8), np.zeros(N, np.float32), g, lam)
+    for t in range(T):
+        n = T - t
+        q = g * lam
+        assert np.allclose(adv[t], c * (1 - q ** n) / (1 - q), atol=1e-12)
+
+
+def test_gae_done_cuts_recursion(orc):
+    rng = np.random.default_rng(5)
+    r, v, d, vl = _gae_inputs(rng, p_done=0.0)
+    d[10] = 1
+    a1, _ = orc.gae(r, v, d, vl, 0.99, 0.95)
+    r2 = r.copy()
+    r2[11:] += 5.0   # changes after the cut must not reach t <= 10
+    v2 = v.copy()
+    v2[11:] -= 2.0
+    a2, _ = orc.gae(r2, v2, d, vl + 1, 0.99, 0.95)
+    assert np.array_equal(a1[:11], a2[:11])
+    assert not np.allclose(a1[11:], a2[11:])
+
+
+def test_rollout_matches_stepwise_replay(orc):
+    # The PPO driver = reset + per-step forced stepping with auto-reset at step t+1.
+    wl = W.WORKLOADS["lbf7x7_64x50_fp32"]
+    d = orc.env_desc(*wl.env.astuple())
+    pols = orc.Policies(W.population(wl))
+    N, T, seed = 16, 120, 9
+    st = orc.reset_all(d, seed, N)
+    out = orc.rollout(d, pols, seed, st, 0, T, 0, [1])
+    assert out["rc"] == 0
+    st2 = orc.reset_all(d, seed, N)
+    for t in range(T):
+        rc, _, team, dones, obs2 = orc.step_forced(d, seed, t, st2, out["actions"][t])
+        assert rc == 0
+        assert np.array_equal(team, out["rewards"][t]) and np.array_equal(dones, out["dones"][t])
+        if t + 1 < T:
+            assert np.array_equal(obs2[:, 0], out["obs"][t + 1])
+            assert np.array_equal(obs2[:, 1], out["obs_tm"][t + 1])
+    assert np.array_equal(st, st2)
+    assert out["dones"].sum() >= N   # 50-step episodes: every env resets at least once
+    # free running: applied actions are the oracle's own samples
+    assert np.array_equal(out["actions"], out["own_actions"])
+
+
+def test_rollout_teammate_draw_is_uniform(orc):
+    wl = W.WORKLOADS["lbf7x7_64x50_fp32"]
+    d = orc.env_desc(*wl.env.astuple())
+    pols = orc.Policies(W.population(wl) * 4)   # 8 policies
+    N = 4000
+    st = orc.reset_all(d, 1, N)
+    out = orc.rollout(d, pols, 1, st, 0, 1, 0, [1, 3, 5, 7])
+    c = np.bincount(out["teammate"], minlength=8)
+    assert c[[0, 2, 4, 6]].sum() == 0
+    assert np.abs(c[[1, 3, 5, 7]] - 1000).max() < 5 * np.sqrt(1000)
+
+
+def test_xplay_matrix_is_pair_mean(orc):
+    wl = W.WORKLOADS["hanabi_xplay_16x16x32"]
+    d = orc.env_desc(*wl.env.astuple())
+    pols = orc.Policies(W.population(wl)[:4])
+    out = orc.xplay(d, pols, 4, 0, [0, 1], [2, 3], 8, 100, n_threads=4)
+    assert out["rc"] == 0
+    R = out["returns"].reshape(2, 2, 8).astype(np.float64)
+    assert np.array_equal(out["matrix"], R.mean(-1).astype(np.float32))
+    assert (out["steps"] <= 97).all() and (out["steps"] > 0).all()
+    # Hanabi returns are integers in [0, 25]
+    assert np.array_equal(R, np.round(R)) and R.min() >= 0 and R.max() <= 25
+    # only the acting seat samples
+    acts = out["actions"]
+    for s in range(100):
+        live = acts[s, :, 0] != 255
+        assert (acts[s, :, 1 - s % 2] == 255).all()
+        assert ((acts[s, :, s % 2] != 255) == (out["steps"] > s)).all()
