@@ -1,0 +1,387 @@
+"""Benchmark: PPO rollout collection of 16384 LBF 7x7 envs x 128 steps with GAE, on GB300.
+
+One step = one aht_rollout call over the whole batch: per env-step, the ego (196-128-128-7
+actor-critic) and a teammate drawn from a 32-policy population (196-128-128-6) run,
+actions are sampled, the env steps, the trajectory (obs, actions, logp, values, rewards,
+dones) streams to HBM, then V_T and GAE advantages/targets are formed.  Weights are
+synthetic (N(0, 0.1), bf16); there are no trained policies in this build.
+
+Prints ONE JSON line (rank 0).  `--impl reference` times the CPU oracle instead, on a
+bounded sample of the same workload.  Multi-GPU (torchrun): every rank runs its own
+independent batch (weak scaling, no collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = "lbf7x7_ppo_16384x128"
+XPLAY_WORKLOAD = "lbf7x7_xplay_8x16x256"
+METRIC = "env-steps/sec (LBF 7x7 PPO rollout collection + GAE, ego vs 32-policy population)"
+UNIT = "env-steps/s"
+L2_BYTES = 129 * 2 ** 20
+
+
+def mlp_flops(dims):
+    return 2 * sum(dims[i] * dims[i + 1] for i in range(len(dims) - 1))
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-xplay", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=12.0)
+    return p.parse_args()
+
+
+def dist_env():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)),
+            int(os.environ.get("WORLD_SIZE", 1)))
+
+
+# ------------------------------------------------------------------------------------
+# CPU oracle timing (the reported baseline; never tuned)
+# ------------------------------------------------------------------------------------
+def oracle_rate(wl, target_s, seed_offset=0):
+    """Times the oracle's free-running PPO collection on a bounded env sample sized for
+    about target_s seconds on all host cores.  Returns (env-steps/s, threads, sample)."""
+    import numpy as np
+    import oracle as O
+    from paper_2609_13716_gb300 import workloads as W
+    threads = os.cpu_count() or 1
+    d = O.env_desc(*wl.env.astuple())
+    pols = O.Policies(W.population(wl))
+    n = max(threads, 2 * threads)
+    st = O.reset_all(d, wl.env_seed, n)
+    t0 = time.perf_counter()
+    O.rollout(d, pols, wl.env_seed, st, 0, wl.T, wl.ego_id, list(wl.pool), n_threads=threads)
+    rate = n * wl.T / (time.perf_counter() - t0)
+    n = int(min(wl.n_envs, max(threads, rate * target_s / wl.T)))
+    n = max(threads, n // threads * threads)
+    ids = np.arange(n, dtype=np.int64) * (wl.n_envs // n)   # spread over the batch
+    st = O.reset_envs(d, wl.env_seed, ids)
+    t0 = time.perf_counter()
+    out = O.rollout(d, pols, wl.env_seed, st, 0, wl.T, wl.ego_id, list(wl.pool),
+                    n_threads=threads, env_ids=ids)
+    adv = O.gae(out["rewards"], out["values"].astype(np.float32), out["dones"],
+                out["last_value"].astype(np.float32), wl.gamma, wl.lam)
+    dt = time.perf_counter() - t0
+    sample = f"{n} of {wl.n_envs} envs x {wl.T} steps (rollout + GAE), free-running fp64 oracle"
+    return n * wl.T / dt, threads, sample, dt
+
+
+def run_reference(args):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return
+    from paper_2609_13716_gb300 import workloads as W
+    wl = W.WORKLOADS[WORKLOAD]
+    import oracle as O
+    O.build()
+    per_step_s = max(2.0, 60.0 / max(1, args.steps + args.warmup))
+    for _ in range(args.warmup):
+        oracle_rate(wl, 0.5)
+    rates, dts = [], []
+    sample = ""
+    threads = 1
+    for _ in range(args.steps):
+        r, threads, sample, dt = oracle_rate(wl, per_step_s)
+        rates.append(r)
+        dts.append(dt)
+    value = statistics.median(rates)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": 0,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1000.0 * wl.n_envs * wl.T / value,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD, "n_envs": wl.n_envs, "T": wl.T, "pool": len(wl.pool)},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                         "sample": sample + "; each step is such a sample, ms_per_step is "
+                                   "scaled to the full batch"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------------------------
+# GPU arm
+# ------------------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ["clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
+              "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
+              "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + ",".join(self.FIELDS),
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx = float(parts[1])
+            except ValueError:
+                continue
+            for name, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def csrc_hash():
+    h = hashlib.sha256()
+    d = os.path.join(ROOT, "paper_2609_13716_gb300", "csrc")
+    for f in sorted(os.listdir(d)):
+        if f.endswith((".cu", ".cuh", ".h")):
+            h.update(open(os.path.join(d, f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel):
+    """Per-launch DRAM bytes from the committed ncu summary, if it still matches the source."""
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(path):
+        return None
+    want = csrc_hash()
+    for ln in open(path):
+        kv = dict(x.split("=", 1) for x in ln.split() if "=" in x)
+        if kv.get("kernel") == kernel and kv.get("csrc_sha") == want:
+            return float(kv["dram_bytes_per_launch"])
+    return None
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    rank, local, world = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    from paper_2609_13716_gb300 import aht, workloads as W
+    from paper_2609_13716_gb300 import build as B
+    B.build()
+    peaks = {}
+    pk = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(pk):
+        peaks = json.load(open(pk))
+    bf16_peak = peaks.get("bf16_tflops", 1900.0)
+    hbm_peak = peaks.get("hbm_gbs", 6800.0)
+    peak_src = "measured" if peaks else "fallback"
+
+    wl = W.WORKLOADS[WORKLOAD]
+    N, T = wl.n_envs, wl.T
+    pop_np = W.population(wl)
+    pop = [[(torch.from_numpy(Wt).to("cuda", torch.bfloat16), torch.from_numpy(b).to("cuda", torch.bfloat16))
+            for Wt, b in p] for p in pop_np]
+    ctx = aht.aht_create(wl.env, pop, N, wl.env_seed + 7919 * rank,
+                         has_value_head=list(wl.value_head), weight_dtype=aht.AHT_BF16)
+    traj = aht.traj_buffers(ctx, T)
+    scrub = torch.empty(256 * 2 ** 20, dtype=torch.uint8, device="cuda")   # > L2
+    stream = torch.cuda.current_stream()
+
+    def step():
+        aht.aht_rollout(ctx, wl.ego_id, wl.pool, T, traj, wl.gamma, wl.lam)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+
+    # ---- timed region: K rollouts, L2 scrubbed between them (outside the events) ----
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    stops = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    dev_index = local
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        dev_index = int(vis.split(",")[local])
+    aht.aht_get_timing(ctx)
+    aht.aht_set_timing(ctx, True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(dev_index) as clocks:
+        for k in range(args.steps):
+            scrub.fill_(k & 0xFF)
+            starts[k].record(stream)
+            step()
+            stops[k].record(stream)
+        torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    aht.aht_set_timing(ctx, False)
+    kernel_ms, kernel_launches = aht.aht_get_timing(ctx)
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, stops)]
+    ms = sum(step_ms) / len(step_ms)
+    ms_t = torch.tensor([ms], device="cuda")
+    if world > 1:
+        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)   # timing only, not the data path
+    ms_max = float(ms_t)
+    aht.aht_sync(ctx)
+
+    # ---- end to end: ego weights from pinned host memory in, whole trajectory out ------
+    ego_host = [(W_.to(torch.bfloat16).cpu().pin_memory(), b.to(torch.bfloat16).cpu().pin_memory())
+                for W_, b in [(torch.from_numpy(a), torch.from_numpy(c)) for a, c in pop_np[wl.ego_id]]]
+    host = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in traj.items() if v is not None}
+    h2d = sum(W_.numel() * 2 + b.numel() * 2 for W_, b in ego_host)
+    d2h = sum(v.numel() * v.element_size() for v in host.values())
+    e2e_s, e2e_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e2e_ms = []
+    for k in range(args.steps + 1):
+        torch.cuda.synchronize()
+        e2e_s.record(stream)
+        aht.aht_set_policy(ctx, wl.ego_id, ego_host, 1, aht.AHT_BF16)
+        step()
+        for key, hv in host.items():
+            hv.copy_(traj[key], non_blocking=True)
+        e2e_e.record(stream)
+        torch.cuda.synchronize()
+        if k > 0:
+            e2e_ms.append(e2e_s.elapsed_time(e2e_e))
+    aht.aht_sync(ctx)
+    e2e_ms_max = torch.tensor([sum(e2e_ms) / len(e2e_ms)], device="cuda")
+    if world > 1:
+        dist.all_reduce(e2e_ms_max, op=dist.ReduceOp.MAX)
+
+    # ---- roofline of the dominant kernel (the fused rollout) ----------------------------
+    env_steps = N * T
+    ego_dims = [wl.env.obs_dim, *wl.hidden, wl.env.n_actions + 1]
+    tm_dims = [wl.env.obs_dim, *wl.hidden, wl.env.n_actions]
+    flops_per_env_step = mlp_flops(ego_dims) + mlp_flops(tm_dims)          # 169,216
+    flops_launch = env_steps * flops_per_env_step + N * mlp_flops(ego_dims)  # + V_T forward
+    bytes_per_env_step = wl.env.obs_dim + 1 + 1 + 4 + 4 + 4 + 1              # obs, a, a_tm, logp, v, r, d
+    kern_ms = kernel_ms / max(1, kernel_launches)
+    achieved_tflops = flops_launch / (kern_ms * 1e-3) / 1e12
+    achieved_gbs = env_steps * bytes_per_env_step / (kern_ms * 1e-3) / 1e9
+    traffic = recorded_traffic("ppo_kernel")
+
+    line = None
+    if rank == 0:
+        value = world * env_steps / (ms_max * 1e-3)
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_max,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f32", "data": "synthetic (random-init N(0,0.1) bf16 weights, seeded envs)",
+            "config": {"workload": WORKLOAD, "n_envs": N, "T": T, "pool": len(wl.pool),
+                       "episode_len": wl.env.episode_len, "weights": "bf16",
+                       "l2": "scrubbed: 256 MB write between timed steps (outside the events); "
+                             "each step also writes a 449 MB trajectory",
+                       "parallelism": f"{world} independent replicas" if world > 1 else "1 GPU"},
+            "roofline": {"bound": "tensor", "achieved": achieved_tflops, "peak": bf16_peak,
+                         "unit": "TFLOP/s", "frac": achieved_tflops / bf16_peak,
+                         "traffic": traffic, "kernel": "ppo_kernel<EnvLbf>",
+                         "kernel_ms": kern_ms, "flops_per_launch": flops_launch,
+                         "peak_source": f"{peak_src} bf16 burst",
+                         "hbm": {"achieved_gbs": achieved_gbs, "peak_gbs": hbm_peak,
+                                 "frac": achieved_gbs / hbm_peak,
+                                 "bytes_per_launch": env_steps * bytes_per_env_step}},
+            "e2e": {"value": world * env_steps / (float(e2e_ms_max) * 1e-3), "unit": UNIT,
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": 3 * args.steps,
+            "clocks": clocks.summary(),
+        }
+    if not args.no_xplay:
+        xp = run_xplay(args, aht, W, torch)
+        if line is not None:
+            line["xplay"] = xp
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, cores, sample, _ = oracle_rate(wl, args.cpu_seconds)
+        line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
+                                "sample": sample}
+    if line is not None:
+        print(json.dumps(line), flush=True)
+    ctx.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_xplay(args, aht, W, torch):
+    """Cross-play cells/s on the 8x16 LBF matrix, 256 envs per pair, 128-step episodes."""
+    wl = W.WORKLOADS[XPLAY_WORKLOAD]
+    pop = [[(torch.from_numpy(Wt).cuda(), torch.from_numpy(b).cuda()) for Wt, b in p]
+           for p in W.population(wl)]
+    n = wl.xplay_envs
+    ctx = aht.aht_create(wl.env, pop, n, wl.env_seed, weight_dtype=aht.AHT_FP32)
+    ne, nt = len(wl.ego_ids), len(wl.tm_ids)
+    matrix = torch.empty(ne, nt, device="cuda")
+    steps = torch.empty(ne, nt, wl.envs_per_pair, dtype=torch.int32, device="cuda")
+    call = lambda: aht.aht_xplay_matrix(ctx, list(wl.ego_ids), list(wl.tm_ids),
+                                        wl.envs_per_pair, wl.max_steps, matrix, None, steps)
+    for _ in range(3):
+        call()
+    torch.cuda.synchronize()
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    K = max(3, args.steps)
+    s.record()
+    for _ in range(K):
+        call()
+    e.record()
+    torch.cuda.synchronize()
+    ms = s.elapsed_time(e) / K
+    active = int(steps.sum())
+    aht.aht_sync(ctx)
+    ctx.close()
+    return {"workload": XPLAY_WORKLOAD, "cells_per_s": ne * nt / (ms * 1e-3),
+            "ms_per_matrix": ms, "active_env_steps_per_s": active / (ms * 1e-3),
+            "dtype": "f32"}
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,223 @@
+/*
+ * aht.h -- C ABI of libaht.so, the GB300 (sm_103a) batched ad hoc teamwork rollout path.
+ *
+ * The operations follow the paper "JaxAHT: A JAX-Based Library for Ad Hoc Teamwork":
+ *   - the Dec-POMDP M = <S, {A_i}, P, {O_i}, Omega, r, rho, gamma> of Sec. 3 (joint
+ *     action -> next state, per-agent observation, one shared team reward), stepped for
+ *     thousands of independent envs at once (Sec. 5.1: the speedup comes from massive
+ *     env parallelism);
+ *   - an ego policy pi_e and teammates pi_{-e} drawn from a population (Sec. 3,
+ *     T_train / T_eval), both decentralised MLP policies pi_i(a | o_i);
+ *   - PPO rollout collection with GAE targets (App. C, "PPO ego");
+ *   - the ego-by-teammate cross-play (XP) return matrix (App. B, "Cross-play matrix
+ *     construction"); its row mean over held-out teammates is J_AHT of Sec. 3.
+ * The paper does not state the game rules; the rules implemented are the readings
+ * listed in the design doc.
+ *
+ * Conventions (all entry points):
+ *   - Bulk tensors are DEVICE pointers owned by the caller, laid out as documented,
+ *     and must stay valid until the work enqueued on the context's stream completes.
+ *     Small id lists (ego/teammate ids, teammate pools) are HOST arrays, passed by value
+ *     to the kernels.
+ *   - Calls are asynchronous on the CUDA stream given to aht_create (NULL = legacy
+ *     default stream), except aht_create, aht_destroy, aht_get_state, aht_set_state and
+ *     aht_sync, which synchronise that stream.
+ *   - Host-side argument errors are returned immediately (AHT_EINVAL) and nothing is
+ *     enqueued.  Errors detected on the device (an out-of-range id, an illegal forced
+ *     Hanabi action) are latched in a device status word and returned by aht_sync.
+ *   - Only aht_create allocates device memory.  Every other call allocates nothing.
+ *   - Seat 0 is the ego, seat 1 the teammate.  XP matrices are [ego][teammate]
+ *     (the transpose of the paper's figures, whose rows are teammates).
+ *   - Randomness is Philox4x32-10 (Salmon et al., SC'11), key = (seed lo, seed hi),
+ *     counter = (env, step, stream, block); streams 0/1 = action of seat 0/1, 2 = env
+ *     reset, 3 = teammate assignment.  "step" is the context's global step counter.
+ *   - aht_last_error returns a thread-local message for the last failing call.
+ */
+#ifndef AHT_H
+#define AHT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct aht_ctx aht_ctx; /* opaque, library-owned */
+
+typedef enum aht_status {
+  AHT_OK = 0,
+  AHT_EINVAL = 1,   /* invalid argument (host check) */
+  AHT_ENOMEM = 2,   /* device allocation failed in aht_create */
+  AHT_ECUDA = 3,    /* a CUDA runtime call failed */
+  AHT_ETIMEOUT = 4, /* reserved: a bounded device wait gave up */
+  AHT_EDEVICE = 5   /* the device status word recorded an error */
+} aht_status;
+
+enum { AHT_LBF = 0, AHT_OVERCOOKED = 1, AHT_HANABI = 2 };
+enum { AHT_FP32 = 0, AHT_BF16 = 1 };
+
+/* Environment (Sec. 4, Table "JaxAHT Environments"; the Dec-POMDP of Sec. 3).
+ *   LBF: width, height in 3..12; n_food 1..3; agent levels uniform in 1..max_agent_level
+ *        (1..9); episode_len >= 1.  Obs = width*height*4 u8, actions 6.
+ *   Overcooked: the fixed 5x4 kitchen (width 5, height 4); episode_len >= 1;
+ *        cook_time 0..255; soup_reward.  Obs = 520 u8, actions 6.
+ *   Hanabi: 2 players, full deck; episode_len must be 0 (run to termination; a game
+ *        lasts at most 97 turns, the library stops any game at 100).  Obs = 660 u8,
+ *        actions 20 with illegal-action masking. */
+typedef struct aht_env_desc {
+  int32_t kind;
+  int32_t width, height;
+  int32_t n_food;
+  int32_t max_agent_level;
+  int32_t episode_len;
+  int32_t cook_time, soup_reward;
+} aht_env_desc;
+
+/* Population of MLP policies (Sec. 3 pi_i; App. C: the ego and the teammates it meets).
+ * Every policy is z = W3 tanh(W2 tanh(W1 o + b1) + b2) + b3 with
+ *   W1 [hidden0][obs_dim], W2 [hidden1][hidden0], W3 [n_out_p][hidden1], row-major,
+ *   b1 [hidden0], b2 [hidden1], b3 [n_out_p],
+ * n_out_p = n_actions + has_value_head[p]: the optional last row is a value estimate.
+ * W[3*p + l] / b[3*p + l] point at layer l of policy p, host or device memory, of
+ * weight_dtype (fp32 or bf16).  aht_create copies and packs them; the caller may free
+ * them afterwards.  has_value_head may be NULL (no value rows).
+ * Limits: n_policies 1..1024, obs_dim must equal the env's, hidden0/hidden1 multiples
+ * of 16 in 16..512. */
+typedef struct aht_pop_desc {
+  int32_t n_policies;
+  int32_t obs_dim, hidden0, hidden1, n_actions;
+  const int32_t* has_value_head; /* host [n_policies] of 0/1, or NULL */
+  int32_t weight_dtype;          /* AHT_FP32 or AHT_BF16 */
+  const void* const* W;          /* host array of 3*n_policies pointers */
+  const void* const* b;          /* host array of 3*n_policies pointers */
+} aht_pop_desc;
+
+/* Creates a context for up to n_envs concurrent envs (PPO state and cross-play batch
+ * capacity), packs the population and resets every env with `seed` (step counter 0).
+ * cuda_stream is a cudaStream_t (NULL = default stream).  Allocates all device memory
+ * the context will ever use.  Returns AHT_EINVAL, AHT_ENOMEM or AHT_ECUDA on failure
+ * (*out is then NULL). */
+aht_status aht_create(const aht_env_desc* env, const aht_pop_desc* pop, int64_t n_envs,
+                      uint64_t seed, void* cuda_stream, aht_ctx** out);
+void aht_destroy(aht_ctx* ctx);
+
+/* rho of Sec. 3: re-draws the initial state of all n_envs envs with a new seed and
+ * sets the global step counter to 0.  Env e uses counter (e, 0, stream 2). */
+aht_status aht_reset(aht_ctx* ctx, uint64_t seed);
+
+/* Trajectory buffers of aht_rollout: caller-owned device memory, time-major [T][N]
+ * (N = the context's n_envs).  NULL members are not written. */
+typedef struct aht_traj {
+  uint8_t* obs;         /* [T][N][obs_dim] ego observation before each step */
+  uint8_t* actions;     /* [T][N] ego action */
+  uint8_t* tm_actions;  /* [T][N] teammate action */
+  float* logp;          /* [T][N] log pi_e(a | o) of the ego action */
+  float* values;        /* [T][N] ego value (0 if the ego has no value row) */
+  float* rewards;       /* [T][N] shared team reward r_t */
+  uint8_t* dones;       /* [T][N] 1 if step t ended the episode (auto-reset follows) */
+  float* advantages;    /* [T][N] GAE advantage */
+  float* targets;       /* [T][N] advantage + value */
+  float* last_value;    /* [N] value of the state after step T-1 (the bootstrap V_T) */
+  int32_t* teammate;    /* [N] teammate policy id used by each env in this call */
+  float gamma, lambda;  /* GAE discount and trace parameters, in [0, 1] */
+} aht_traj;
+
+/* PPO rollout collection (App. C "PPO ego"; Sec. 3 ego vs teammates from T_train).
+ * Each env draws its teammate once per call: pool[floor(x * pool_size / 2^32)] with x
+ * the first draw of counter (env, step0, stream 3).  Then for t in 0..T-1 (step
+ * step0+t): both seats observe, the ego and the teammate MLPs run, actions are
+ * sampled by inverse CDF with u from stream 0/1, the env steps, and an env whose
+ * episode ended is reset at step step0+t+1 (stream 2).  Finally V_T is computed and
+ * GAE (advantages, targets) is formed when `advantages` is non-NULL.  The step counter
+ * advances by T.  Simultaneous-move envs only (LBF, Overcooked): AHT_EINVAL for Hanabi.
+ * pool: host [pool_size] policy ids, 1 <= pool_size <= 256.  T >= 1. */
+aht_status aht_rollout(aht_ctx* ctx, int32_t ego_id, const int32_t* pool, int32_t pool_size,
+                       int32_t T, const aht_traj* out);
+
+/* Outputs of aht_xplay_matrix (caller-owned device memory; NULL members not written). */
+typedef struct aht_xplay_out {
+  float* matrix;        /* [n_ego][n_tm] mean team return over the pair's envs */
+  float* returns;       /* [n_ego][n_tm][P] team return of each env's first episode */
+  int32_t* steps;       /* [n_ego][n_tm][P] env-steps the episode took */
+  uint8_t* actions;     /* [max_steps][n_ego*n_tm*P][2] applied actions, 255 = none */
+} aht_xplay_out;
+
+/* Cross-play evaluation (App. B; J_AHT of Sec. 3 is a row mean).  Pair (i, j) plays
+ * P = envs_per_pair fresh episodes of ego_ids[i] (seat 0) with tm_ids[j] (seat 1); env
+ * index e = (i*n_tm + j)*P + k is reset at counter (e, step0, stream 2) and steps at
+ * step0 + s.  An env stops after its first episode.  matrix[i][j] = (sum of the P fp32
+ * returns, added exactly in fp64) / P.  Uses the context's scratch, not its PPO env
+ * state; the step counter advances by max_steps.  Requires n_ego*n_tm*P <= n_envs,
+ * 1 <= n_ego, n_tm <= 64, max_steps >= 1.  ego_ids / tm_ids are host arrays. */
+aht_status aht_xplay_matrix(aht_ctx* ctx, const int32_t* ego_ids, int32_t n_ego,
+                            const int32_t* tm_ids, int32_t n_tm, int32_t envs_per_pair,
+                            int32_t max_steps, const aht_xplay_out* out);
+
+/* Stateless GAE (App. C "PPO ego"), time-major [T][n_envs] device arrays:
+ *   delta_t = r_t + gamma (1 - d_t) V_{t+1} - V_t,
+ *   A_t = delta_t + gamma lambda (1 - d_t) A_{t+1},  V_T = v_last,  A_T = 0,
+ *   targets = A + V (targets may be NULL).  fp32 arithmetic; one reverse scan per env.
+ * Enqueued on cuda_stream (a cudaStream_t, NULL = default). */
+aht_status aht_gae(const float* rewards, const float* values, const uint8_t* dones,
+                   const float* v_last, int64_t n_envs, int32_t T, float gamma, float lambda,
+                   float* advantages, float* targets, void* cuda_stream);
+
+/* Replaces the weights of one policy (App. C: PPO updates the ego between rollout
+ * collections).  W[l] / b[l] (l = 0..2) have the shapes of aht_pop_desc for this policy,
+ * in host or device memory of weight_dtype; has_value_head as in aht_pop_desc.  The
+ * library packs them on the host into a staging buffer pinned at aht_create and
+ * enqueues the upload on the context's stream; it first waits for the context's
+ * previous upload.  Allocates nothing. */
+aht_status aht_set_policy(aht_ctx* ctx, int32_t policy, const void* const* W,
+                          const void* const* b, int32_t weight_dtype, int32_t has_value_head);
+
+/* Kernel timing.  While enabled, the library brackets each launch of its main kernel
+ * (the fused rollout of aht_rollout, the cross-play kernel of aht_xplay_matrix) with
+ * CUDA events on the context's stream.  aht_get_timing synchronises the stream and
+ * returns the summed kernel time in milliseconds and the number of timed launches
+ * since the previous aht_get_timing (then resets both). */
+aht_status aht_set_timing(aht_ctx* ctx, int32_t enable);
+aht_status aht_get_timing(aht_ctx* ctx, double* kernel_ms, int64_t* launches);
+
+/* ---- test and checkpoint hooks ------------------------------------------------ */
+
+/* Outputs of aht_step_forced (device memory; NULL members not written). */
+typedef struct aht_step_out {
+  float* rewards;   /* [N][2] per-agent reward */
+  float* team;      /* [N] team reward */
+  uint8_t* dones;   /* [N] */
+  uint8_t* obs;     /* [N][2][obs_dim] both seats' observation of the resulting state */
+} aht_step_out;
+
+/* One env step of every PPO env with the given actions (device u8 [N][2]; Hanabi uses
+ * the acting seat's entry), auto-reset at step+1 as in aht_rollout, then the step
+ * counter advances by 1.  An illegal Hanabi action leaves that env unchanged and
+ * latches AHT_EDEVICE. */
+aht_status aht_step_forced(aht_ctx* ctx, const uint8_t* actions, const aht_step_out* out);
+
+/* Policy outputs z = MLP_p(o) for n observations: obs device u8 [n][obs_dim] ->
+ * out device f32 [n][n_actions + 1] (the last column is the value row, 0 if absent). */
+aht_status aht_policy_forward(aht_ctx* ctx, int32_t policy, const uint8_t* obs, int64_t n,
+                              float* out);
+
+/* Checkpoint of the PPO env state, the seed and the step counter into a host buffer.
+ * Call with buf == NULL to get the size in *bytes.  Resuming from it is bit-exact:
+ * every draw is a function of (seed, env, step, stream). */
+aht_status aht_get_state(aht_ctx* ctx, void* buf, size_t* bytes);
+aht_status aht_set_state(aht_ctx* ctx, const void* buf, size_t bytes);
+
+/* Global step counter (the next step index). */
+int64_t aht_step_counter(const aht_ctx* ctx);
+
+/* Synchronises the context's stream and returns AHT_EDEVICE if the device status word
+ * recorded an error since the last aht_sync (the word is then cleared). */
+aht_status aht_sync(aht_ctx* ctx);
+
+const char* aht_last_error(void);
+const char* aht_status_string(aht_status s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -93,7 +93,7 @@ _P = C.c_void_p
 class RolloutIO(C.Structure):
     _fields_ = [("seed", C.c_uint64), ("n_envs", C.c_int64), ("step0", C.c_int64),
                 ("T", C.c_int32), ("ego_id", C.c_int32), ("pool", _P), ("pool_size", C.c_int32),
-                ("forced", _P), ("states", _P), ("n_threads", C.c_int32),
+                ("forced", _P), ("env_ids", _P), ("states", _P), ("n_threads", C.c_int32),
                 ("teammate", _P), ("obs", _P), ("obs_tm", _P), ("actions", _P),
                 ("own_actions", _P), ("margin", _P), ("logits", _P), ("logp", _P),
                 ("values", _P), ("rewards", _P), ("dones", _P), ("last_value", _P)]
@@ -103,7 +103,7 @@ class XplayIO(C.Structure):
     _fields_ = [("seed", C.c_uint64), ("step0", C.c_int64), ("ego_ids", _P),
                 ("n_ego", C.c_int32), ("tm_ids", _P), ("n_tm", C.c_int32),
                 ("envs_per_pair", C.c_int32), ("max_steps", C.c_int32), ("forced", _P),
-                ("n_threads", C.c_int32), ("returns", _P), ("steps", _P), ("actions", _P),
+                ("env_ids", _P), ("n_sel", C.c_int64), ("n_threads", C.c_int32), ("returns", _P), ("steps", _P), ("actions", _P),
                 ("own_actions", _P), ("margin", _P), ("matrix", _P)]
 
 
@@ -146,6 +146,8 @@ def lib() -> C.CDLL:
             L.orc_rollout.restype = C.c_int32
             L.orc_reset_all.argtypes = [C.POINTER(EnvDesc), C.c_uint64, C.c_int64, C.c_int64, _P]
             L.orc_reset_all.restype = C.c_int32
+            L.orc_reset_envs.argtypes = [C.POINTER(EnvDesc), C.c_uint64, _P, C.c_int64, C.c_int64, _P]
+            L.orc_reset_envs.restype = C.c_int32
             L.orc_step_forced.argtypes = [C.POINTER(EnvDesc), C.c_uint64, C.c_int64, C.c_int64, _P, _P, _P, _P, _P, _P]
             L.orc_step_forced.restype = C.c_int32
             L.orc_xplay.argtypes = [C.POINTER(EnvDesc), C.POINTER(Mlp), C.c_int32, C.POINTER(XplayIO)]
@@ -247,6 +249,14 @@ def reset_all(d, seed, n, step=0):
     return st
 
 
+def reset_envs(d, seed, ids, step=0):
+    ids = np.ascontiguousarray(ids, np.int64)
+    st = new_states(len(ids))
+    rc = lib().orc_reset_envs(C.byref(d), seed, _ptr(ids), len(ids), step, _ptr(st))
+    assert rc == 0, rc
+    return st
+
+
 def step_forced(d, seed, step, states, actions):
     n = states.shape[0]
     od = obs_dim(d)
@@ -260,9 +270,14 @@ def step_forced(d, seed, step, states, actions):
     return rc, rew2, team, dones, obs2
 
 
-def rollout(d, pols: Policies, seed, states, step0, T, ego_id, pool, forced=None, n_threads=1):
-    """PPO collection.  Returns a dict of numpy arrays; states are updated in place."""
+def rollout(d, pols: Policies, seed, states, step0, T, ego_id, pool, forced=None, n_threads=1,
+            env_ids=None):
+    """PPO collection.  Returns a dict of numpy arrays; states are updated in place.
+    env_ids: global env index of each state row (default 0..N-1)."""
     N = states.shape[0]
+    if env_ids is not None:
+        env_ids = np.ascontiguousarray(env_ids, np.int64)
+        assert env_ids.shape == (N,)
     od = obs_dim(d)
     K = n_actions(d)
     n_out = pols.arr[ego_id].n_out
@@ -278,7 +293,8 @@ def rollout(d, pols: Policies, seed, states, step0, T, ego_id, pool, forced=None
         forced = np.ascontiguousarray(forced, np.uint8)
         assert forced.shape == (T, N, 2)
     io = RolloutIO(seed=seed, n_envs=N, step0=step0, T=T, ego_id=ego_id, pool=_ptr(pool),
-                   pool_size=len(pool), forced=_ptr(forced), states=_ptr(states),
+                   pool_size=len(pool), forced=_ptr(forced), env_ids=_ptr(env_ids),
+                   states=_ptr(states),
                    n_threads=n_threads, **{k: _ptr(v) for k, v in out.items()})
     rc = lib().orc_rollout(C.byref(d), pols.arr, pols.n, C.byref(io))
     out["rc"] = rc
@@ -286,10 +302,14 @@ def rollout(d, pols: Policies, seed, states, step0, T, ego_id, pool, forced=None
 
 
 def xplay(d, pols: Policies, seed, step0, ego_ids, tm_ids, P, max_steps, forced=None,
-          n_threads=1, record=True):
+          n_threads=1, record=True, env_ids=None):
+    """Cross-play.  env_ids: run only these global env indices (rows of the outputs)."""
     ego_ids = np.ascontiguousarray(ego_ids, np.int32)
     tm_ids = np.ascontiguousarray(tm_ids, np.int32)
     N = len(ego_ids) * len(tm_ids) * P
+    if env_ids is not None:
+        env_ids = np.ascontiguousarray(env_ids, np.int64)
+        N = len(env_ids)
     out = dict(returns=np.zeros(N, np.float32), steps=np.zeros(N, np.int32),
                matrix=np.zeros((len(ego_ids), len(tm_ids)), np.float32))
     if record:
@@ -300,7 +320,8 @@ def xplay(d, pols: Policies, seed, step0, ego_ids, tm_ids, P, max_steps, forced=
         forced = np.ascontiguousarray(forced, np.uint8)
     io = XplayIO(seed=seed, step0=step0, ego_ids=_ptr(ego_ids), n_ego=len(ego_ids),
                  tm_ids=_ptr(tm_ids), n_tm=len(tm_ids), envs_per_pair=P, max_steps=max_steps,
-                 forced=_ptr(forced), n_threads=n_threads,
+                 forced=_ptr(forced), env_ids=_ptr(env_ids),
+                 n_sel=0 if env_ids is None else len(env_ids), n_threads=n_threads,
                  **{k: _ptr(v) for k, v in out.items()})
     rc = lib().orc_xplay(C.byref(d), pols.arr, pols.n, C.byref(io))
     out["rc"] = rc

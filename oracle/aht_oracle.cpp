@@ -723,6 +723,13 @@ extern "C" int32_t orc_reset_all(const orc_env_desc* d, uint64_t seed, int64_t n
   return 0;
 }
 
+extern "C" int32_t orc_reset_envs(const orc_env_desc* d, uint64_t seed, const int64_t* ids,
+                                  int64_t n, int64_t step, orc_state* states) {
+  if (orc_check_desc(d) != 0) return -1;
+  for (int64_t i = 0; i < n; ++i) env_reset(d, seed, (uint32_t)ids[i], (uint32_t)step, &states[i]);
+  return 0;
+}
+
 extern "C" int32_t orc_step_forced(const orc_env_desc* d, uint64_t seed, int64_t n_envs,
                                    int64_t step, orc_state* states, const uint8_t* actions,
                                    float* rewards2, float* team, uint8_t* dones, uint8_t* obs2) {
@@ -866,7 +873,7 @@ extern "C" int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32
   const bool has_value = ego->n_out > K;
   std::vector<int> status(N, 0);
   parallel_for(N, io->n_threads, [&](int64_t e) {
-    const uint32_t env = (uint32_t)e;
+    const uint32_t env = (uint32_t)(io->env_ids ? io->env_ids[e] : e);
     const uint32_t x = orc_draw(io->seed, env, (uint32_t)io->step0, ORC_STREAM_TEAMMATE, 0);
     const int tm_id = io->pool[orc_uniform_int(x, (uint32_t)io->pool_size)];
     if (io->teammate) io->teammate[e] = tm_id;
@@ -927,12 +934,16 @@ extern "C" int32_t orc_xplay(const orc_env_desc* d, const orc_mlp* pols, int32_t
     if (io->tm_ids[j] < 0 || io->tm_ids[j] >= n_pols) return -4;
   const int od = orc_obs_dim(d), K = orc_n_actions(d);
   const int P = io->envs_per_pair;
-  const int64_t N = (int64_t)io->n_ego * io->n_tm * P;
+  const int64_t n_all = (int64_t)io->n_ego * io->n_tm * P;
+  const int64_t N = io->env_ids ? io->n_sel : n_all;  // rows
+  for (int64_t r = 0; io->env_ids && r < N; ++r)
+    if (io->env_ids[r] < 0 || io->env_ids[r] >= n_all) return -4;
   std::vector<float> returns(N, 0.0f);
   std::vector<int> status(N, 0);
   parallel_for(N, io->n_threads, [&](int64_t e) {
-    const uint32_t env = (uint32_t)e;
-    const int64_t pair = e / P;
+    const int64_t g = io->env_ids ? io->env_ids[e] : e;  // global env index
+    const uint32_t env = (uint32_t)g;
+    const int64_t pair = g / P;
     const orc_mlp* pol[2] = {&pols[io->ego_ids[pair / io->n_tm]], &pols[io->tm_ids[pair % io->n_tm]]};
     orc_state st;
     env_reset(d, io->seed, env, (uint32_t)io->step0, &st);
@@ -978,7 +989,7 @@ extern "C" int32_t orc_xplay(const orc_env_desc* d, const orc_mlp* pols, int32_t
     if (io->returns) io->returns[e] = ret;
     if (io->steps) io->steps[e] = steps;
   });
-  if (io->matrix) {
+  if (io->matrix && !io->env_ids) {
     for (int64_t pair = 0; pair < (int64_t)io->n_ego * io->n_tm; ++pair) {
       double acc = 0.0;
       for (int k = 0; k < P; ++k) acc += (double)returns[pair * P + k];

@@ -161,6 +161,7 @@ typedef struct orc_rollout_io {
   const int32_t* pool;         /* teammate policy ids */
   int32_t pool_size;
   const uint8_t* forced;       /* [T][N][2] actions to apply, or NULL to free-run */
+  const int64_t* env_ids;      /* [N] global env index of each row, or NULL for 0..N-1 */
   orc_state* states;           /* [N] in/out */
   int32_t n_threads;
   /* outputs (each may be NULL) */
@@ -183,6 +184,9 @@ int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32_t n_pols,
 /* Resets n_envs envs with env index 0..n-1 at the given step counter. */
 int32_t orc_reset_all(const orc_env_desc* d, uint64_t seed, int64_t n_envs, int64_t step,
                       orc_state* states);
+/* Resets the envs with the given global indices (row i gets env ids[i]). */
+int32_t orc_reset_envs(const orc_env_desc* d, uint64_t seed, const int64_t* ids, int64_t n,
+                       int64_t step, orc_state* states);
 /* One forced step of every env, PPO semantics (auto-reset with step+1).  Outputs the
  * per-agent rewards [N][2], team rewards [N], dones [N] and both seats' observation of
  * the resulting state [N][2][obs_dim]; each output may be NULL.  Hanabi applies the
@@ -200,6 +204,9 @@ typedef struct orc_xplay_io {
   int32_t envs_per_pair;
   int32_t max_steps;
   const uint8_t* forced;   /* [max_steps][n_envs][2] or NULL */
+  const int64_t* env_ids;  /* [n_sel] global env indices to run, or NULL for all envs;
+                              outputs are then indexed by selection row */
+  int64_t n_sel;
   int32_t n_threads;
   /* outputs (each may be NULL) */
   float* returns;          /* [n_ego][n_tm][P] team return of the first episode */
@@ -207,7 +214,7 @@ typedef struct orc_xplay_io {
   uint8_t* actions;        /* [max_steps][n_envs][2] applied actions (255 = none) */
   uint8_t* own_actions;    /* [max_steps][n_envs][2] */
   double* margin;          /* [max_steps][n_envs][2] (2 = no sample) */
-  float* matrix;           /* [n_ego][n_tm] mean return, fp64 sum */
+  float* matrix;           /* [n_ego][n_tm] mean return, fp64 sum (all envs only) */
 } orc_xplay_io;
 int32_t orc_xplay(const orc_env_desc* d, const orc_mlp* pols, int32_t n_pols,
                   orc_xplay_io* io);

@@ -1,0 +1,304 @@
+"""Python binding of libaht.so (include/aht.h): argument marshalling only.
+
+Every step of the rollout path runs in the CUDA kernels behind the C ABI; this module
+converts torch tensors to device pointers, checks shapes and dtypes, and raises
+``AhtError`` for a non-OK status.  There is no CPU fallback: if the library has not
+been built (``paper_2609_13716_gb300.build.build()``), importing the functions raises.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+AHT_OK, AHT_EINVAL, AHT_ENOMEM, AHT_ECUDA, AHT_ETIMEOUT, AHT_EDEVICE = range(6)
+AHT_LBF, AHT_OVERCOOKED, AHT_HANABI = range(3)
+AHT_FP32, AHT_BF16 = 0, 1
+
+EXPORTED = ["aht_create", "aht_destroy", "aht_reset", "aht_rollout", "aht_xplay_matrix",
+            "aht_gae", "aht_step_forced", "aht_policy_forward", "aht_get_state",
+            "aht_set_state", "aht_step_counter", "aht_sync", "aht_last_error",
+            "aht_status_string", "aht_set_policy", "aht_set_timing", "aht_get_timing"]
+
+
+class AhtError(RuntimeError):
+    def __init__(self, status, msg):
+        super().__init__(f"aht status {status}: {msg}")
+        self.status = status
+
+
+class EnvDesc(C.Structure):
+    _fields_ = [("kind", C.c_int32), ("width", C.c_int32), ("height", C.c_int32),
+                ("n_food", C.c_int32), ("max_agent_level", C.c_int32),
+                ("episode_len", C.c_int32), ("cook_time", C.c_int32),
+                ("soup_reward", C.c_int32)]
+
+
+class PopDesc(C.Structure):
+    _fields_ = [("n_policies", C.c_int32), ("obs_dim", C.c_int32), ("hidden0", C.c_int32),
+                ("hidden1", C.c_int32), ("n_actions", C.c_int32),
+                ("has_value_head", C.POINTER(C.c_int32)), ("weight_dtype", C.c_int32),
+                ("W", C.POINTER(C.c_void_p)), ("b", C.POINTER(C.c_void_p))]
+
+
+class Traj(C.Structure):
+    _fields_ = [("obs", C.c_void_p), ("actions", C.c_void_p), ("tm_actions", C.c_void_p),
+                ("logp", C.c_void_p), ("values", C.c_void_p), ("rewards", C.c_void_p),
+                ("dones", C.c_void_p), ("advantages", C.c_void_p), ("targets", C.c_void_p),
+                ("last_value", C.c_void_p), ("teammate", C.c_void_p), ("gamma", C.c_float),
+                ("lambda_", C.c_float)]
+
+
+class XplayOut(C.Structure):
+    _fields_ = [("matrix", C.c_void_p), ("returns", C.c_void_p), ("steps", C.c_void_p),
+                ("actions", C.c_void_p)]
+
+
+class StepOut(C.Structure):
+    _fields_ = [("rewards", C.c_void_p), ("team", C.c_void_p), ("dones", C.c_void_p),
+                ("obs", C.c_void_p)]
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load() -> C.CDLL:
+    """Loads libaht.so (built in-tree).  Raises if it is missing: no fallback exists."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            path = library_path()
+            if not os.path.exists(path):
+                raise ImportError(f"libaht.so not built ({path}); run "
+                                  "paper_2609_13716_gb300.build.build() first")
+            L = C.CDLL(path)
+            vp, i32, i64, u64 = C.c_void_p, C.c_int32, C.c_int64, C.c_uint64
+            L.aht_create.argtypes = [C.POINTER(EnvDesc), C.POINTER(PopDesc), i64, u64, vp, C.POINTER(vp)]
+            L.aht_destroy.argtypes = [vp]
+            L.aht_destroy.restype = None
+            L.aht_reset.argtypes = [vp, u64]
+            L.aht_rollout.argtypes = [vp, i32, C.POINTER(i32), i32, i32, C.POINTER(Traj)]
+            L.aht_xplay_matrix.argtypes = [vp, C.POINTER(i32), i32, C.POINTER(i32), i32, i32, i32, C.POINTER(XplayOut)]
+            L.aht_gae.argtypes = [vp, vp, vp, vp, i64, i32, C.c_float, C.c_float, vp, vp, vp]
+            L.aht_step_forced.argtypes = [vp, vp, C.POINTER(StepOut)]
+            L.aht_policy_forward.argtypes = [vp, i32, vp, i64, vp]
+            L.aht_get_state.argtypes = [vp, vp, C.POINTER(C.c_size_t)]
+            L.aht_set_state.argtypes = [vp, vp, C.c_size_t]
+            L.aht_set_policy.argtypes = [vp, i32, C.POINTER(vp), C.POINTER(vp), i32, i32]
+            L.aht_set_timing.argtypes = [vp, i32]
+            L.aht_get_timing.argtypes = [vp, C.POINTER(C.c_double), C.POINTER(i64)]
+            L.aht_step_counter.argtypes = [vp]
+            L.aht_step_counter.restype = i64
+            L.aht_sync.argtypes = [vp]
+            L.aht_last_error.argtypes = []
+            L.aht_last_error.restype = C.c_char_p
+            L.aht_status_string.argtypes = [C.c_int]
+            L.aht_status_string.restype = C.c_char_p
+            for f in ("aht_create", "aht_reset", "aht_rollout", "aht_xplay_matrix", "aht_gae",
+                      "aht_step_forced", "aht_policy_forward", "aht_get_state", "aht_set_state",
+                      "aht_sync", "aht_set_policy", "aht_set_timing", "aht_get_timing"):
+                getattr(L, f).restype = C.c_int
+            _lib = L
+    return _lib
+
+
+def _check(status):
+    if status != AHT_OK:
+        raise AhtError(status, load().aht_last_error().decode())
+
+
+def _ptr(t, dtype=None, shape=None, name="tensor"):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    return getattr(stream, "cuda_stream", stream)
+
+
+class Context:
+    """Owns an aht_ctx handle (aht_destroy on close / garbage collection)."""
+
+    def __init__(self, handle, env, n_envs, obs_dim, n_actions, stream):
+        self.handle = handle
+        self.env = env
+        self.n_envs = n_envs
+        self.obs_dim = obs_dim
+        self.n_actions = n_actions
+        self.stream = stream
+
+    def close(self):
+        if self.handle:
+            load().aht_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def aht_create(env, population, n_envs, seed, has_value_head=None, weight_dtype=AHT_BF16,
+               stream=None) -> Context:
+    """env: workloads.EnvSpec; population: per policy [(W1, b1), (W2, b2), (W3, b3)] torch
+    tensors (CUDA or CPU, fp32 or bf16 matching weight_dtype), row-major [out][in]."""
+    L = load()
+    dt = torch.float32 if weight_dtype == AHT_FP32 else torch.bfloat16
+    keep, Ws, bs = [], [], []
+    for pol in population:
+        for W, b in pol:
+            W = W.to(dt).contiguous()
+            b = b.to(dt).contiguous()
+            keep += [W, b]
+            Ws.append(W.data_ptr())
+            bs.append(b.data_ptr())
+    n = len(population)
+    hv = (C.c_int32 * n)(*(has_value_head or [0] * n))
+    Warr = (C.c_void_p * len(Ws))(*Ws)
+    barr = (C.c_void_p * len(bs))(*bs)
+    h0 = population[0][0][0].shape[0]
+    h1 = population[0][1][0].shape[0]
+    pop = PopDesc(n, env.obs_dim, h0, h1, env.n_actions, hv, weight_dtype, Warr, barr)
+    desc = EnvDesc(*env.astuple())
+    handle = C.c_void_p()
+    s = _stream(stream)
+    _check(L.aht_create(C.byref(desc), C.byref(pop), n_envs, seed, s, C.byref(handle)))
+    del keep
+    return Context(handle, env, n_envs, env.obs_dim, env.n_actions, s)
+
+
+def aht_reset(ctx: Context, seed: int):
+    _check(load().aht_reset(ctx.handle, seed))
+
+
+def traj_buffers(ctx: Context, T: int, device="cuda", obs=True):
+    """Allocates (with torch) the caller-owned trajectory tensors of aht_rollout."""
+    N = ctx.n_envs
+    z = lambda shape, dt: torch.empty(shape, dtype=dt, device=device)
+    return dict(obs=z((T, N, ctx.obs_dim), torch.uint8) if obs else None,
+                actions=z((T, N), torch.uint8), tm_actions=z((T, N), torch.uint8),
+                logp=z((T, N), torch.float32), values=z((T, N), torch.float32),
+                rewards=z((T, N), torch.float32), dones=z((T, N), torch.uint8),
+                advantages=z((T, N), torch.float32), targets=z((T, N), torch.float32),
+                last_value=z((N,), torch.float32), teammate=z((N,), torch.int32))
+
+
+def aht_rollout(ctx: Context, ego_id, pool, T, traj: dict, gamma=0.99, lam=0.95):
+    N = ctx.n_envs
+    f32, u8 = torch.float32, torch.uint8
+    g = traj.get
+    t = Traj(_ptr(g("obs"), u8, (T, N, ctx.obs_dim), "obs"),
+             _ptr(g("actions"), u8, (T, N), "actions"),
+             _ptr(g("tm_actions"), u8, (T, N), "tm_actions"),
+             _ptr(g("logp"), f32, (T, N), "logp"), _ptr(g("values"), f32, (T, N), "values"),
+             _ptr(g("rewards"), f32, (T, N), "rewards"), _ptr(g("dones"), u8, (T, N), "dones"),
+             _ptr(g("advantages"), f32, (T, N), "advantages"),
+             _ptr(g("targets"), f32, (T, N), "targets"),
+             _ptr(g("last_value"), f32, (N,), "last_value"),
+             _ptr(g("teammate"), torch.int32, (N,), "teammate"), gamma, lam)
+    pool = list(pool)
+    parr = (C.c_int32 * len(pool))(*pool)
+    _check(load().aht_rollout(ctx.handle, ego_id, parr, len(pool), T, C.byref(t)))
+
+
+def aht_xplay_matrix(ctx: Context, ego_ids, tm_ids, envs_per_pair, max_steps, matrix,
+                     returns=None, steps=None, actions=None):
+    ne, nt, P = len(ego_ids), len(tm_ids), envs_per_pair
+    out = XplayOut(_ptr(matrix, torch.float32, (ne, nt), "matrix"),
+                   _ptr(returns, torch.float32, (ne, nt, P), "returns"),
+                   _ptr(steps, torch.int32, (ne, nt, P), "steps"),
+                   _ptr(actions, torch.uint8, (max_steps, ne * nt * P, 2), "actions"))
+    ea = (C.c_int32 * ne)(*ego_ids)
+    ta = (C.c_int32 * nt)(*tm_ids)
+    _check(load().aht_xplay_matrix(ctx.handle, ea, ne, ta, nt, P, max_steps, C.byref(out)))
+
+
+def aht_gae(rewards, values, dones, v_last, gamma, lam, advantages, targets=None, stream=None):
+    T, N = rewards.shape
+    f32 = torch.float32
+    _check(load().aht_gae(_ptr(rewards, f32, (T, N), "rewards"), _ptr(values, f32, (T, N), "values"),
+                          _ptr(dones, torch.uint8, (T, N), "dones"), _ptr(v_last, f32, (N,), "v_last"),
+                          N, T, gamma, lam, _ptr(advantages, f32, (T, N), "advantages"),
+                          _ptr(targets, f32, (T, N), "targets"), _stream(stream)))
+
+
+def aht_step_forced(ctx: Context, actions, rewards=None, team=None, dones=None, obs=None):
+    N = ctx.n_envs
+    out = StepOut(_ptr(rewards, torch.float32, (N, 2), "rewards"),
+                  _ptr(team, torch.float32, (N,), "team"), _ptr(dones, torch.uint8, (N,), "dones"),
+                  _ptr(obs, torch.uint8, (N, 2, ctx.obs_dim), "obs"))
+    _check(load().aht_step_forced(ctx.handle, _ptr(actions, torch.uint8, (N, 2), "actions"),
+                                  C.byref(out)))
+
+
+def aht_policy_forward(ctx: Context, policy, obs, out):
+    n = obs.shape[0]
+    _check(load().aht_policy_forward(ctx.handle, policy,
+                                     _ptr(obs, torch.uint8, (n, ctx.obs_dim), "obs"), n,
+                                     _ptr(out, torch.float32, (n, ctx.n_actions + 1), "out")))
+
+
+def aht_get_state(ctx: Context) -> bytes:
+    L = load()
+    n = C.c_size_t(0)
+    _check(L.aht_get_state(ctx.handle, None, C.byref(n)))
+    buf = C.create_string_buffer(n.value)
+    _check(L.aht_get_state(ctx.handle, buf, C.byref(n)))
+    return buf.raw[:n.value]
+
+
+def aht_set_state(ctx: Context, state: bytes):
+    buf = C.create_string_buffer(state, len(state))
+    _check(load().aht_set_state(ctx.handle, buf, len(state)))
+
+
+def aht_set_policy(ctx: Context, policy, layers, has_value_head=0, weight_dtype=AHT_BF16):
+    """layers: [(W1, b1), (W2, b2), (W3, b3)] tensors (pinned/pageable host or CUDA)."""
+    dt = torch.float32 if weight_dtype == AHT_FP32 else torch.bfloat16
+    for W, b in layers:
+        if W.dtype != dt or b.dtype != dt or not W.is_contiguous() or not b.is_contiguous():
+            raise TypeError(f"weights must be contiguous {dt}")
+    Ws = (C.c_void_p * 3)(*[W.data_ptr() for W, _ in layers])
+    bs = (C.c_void_p * 3)(*[b.data_ptr() for _, b in layers])
+    _check(load().aht_set_policy(ctx.handle, policy, Ws, bs, weight_dtype, has_value_head))
+
+
+def aht_set_timing(ctx: Context, enable: bool):
+    _check(load().aht_set_timing(ctx.handle, int(enable)))
+
+
+def aht_get_timing(ctx: Context):
+    """(summed kernel milliseconds, number of timed launches) since the previous call."""
+    ms = C.c_double(0)
+    n = C.c_int64(0)
+    _check(load().aht_get_timing(ctx.handle, C.byref(ms), C.byref(n)))
+    return ms.value, n.value
+
+
+def aht_step_counter(ctx: Context) -> int:
+    return load().aht_step_counter(ctx.handle)
+
+
+def aht_sync(ctx: Context):
+    _check(load().aht_sync(ctx.handle))

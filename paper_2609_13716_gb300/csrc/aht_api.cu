@@ -1,0 +1,610 @@
+// aht_api.cu -- the C ABI of libaht.so (declared in include/aht.h): argument checks,
+// context memory, weight packing and kernel launches.  No compute happens on the host
+// except packing the population once in aht_create.
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "kernels.h"
+#include "rollout_impl.cuh"
+
+using namespace aht;
+
+namespace {
+
+thread_local std::string g_err;
+
+aht_status fail(aht_status s, const std::string& msg) {
+  g_err = msg;
+  return s;
+}
+
+#define AHT_CUDA(call)                                                                   \
+  do {                                                                                   \
+    cudaError_t e_ = (call);                                                             \
+    if (e_ != cudaSuccess)                                                               \
+      return fail(AHT_ECUDA, std::string(#call) + ": " + cudaGetErrorString(e_));        \
+  } while (0)
+
+struct DeviceGuard {
+  int prev = -1;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) cudaSetDevice(dev);
+    else prev = -1;
+  }
+  ~DeviceGuard() {
+    if (prev >= 0) cudaSetDevice(prev);
+  }
+};
+
+struct EnvOps {
+  cudaError_t (*ppo)(const PpoArgs&, int, size_t, cudaStream_t);
+  cudaError_t (*xplay)(const XpArgs&, int, size_t, cudaStream_t);
+  cudaError_t (*forced)(const ForcedArgs&, cudaStream_t);
+  cudaError_t (*reset)(const ResetArgs&, cudaStream_t);
+  int (*words)();
+  int (*bytes)();
+  cudaError_t (*smem_limit)(size_t);
+  int max_rows;  // largest tile that fits the hidden activations of typical sizes
+};
+
+EnvOps ops_for(int kind) {
+  switch (kind) {
+    case AHT_LBF:
+      return {lbf_ppo, lbf_xplay, lbf_forced, lbf_reset, lbf_state_words, lbf_state_bytes, lbf_set_smem_limit, 128};
+    case AHT_OVERCOOKED:
+      return {overcooked_ppo, overcooked_xplay, overcooked_forced, overcooked_reset,
+              overcooked_state_words, overcooked_state_bytes, overcooked_set_smem_limit, 64};
+    default:
+      return {hanabi_ppo, hanabi_xplay, hanabi_forced, hanabi_reset, hanabi_state_words,
+              hanabi_state_bytes, hanabi_set_smem_limit, 32};
+  }
+}
+
+constexpr uint32_t kStateMagic = 0x31544841u;  // "AHT1"
+
+struct StateHeader {
+  uint32_t magic, kind, n_words, pad;
+  int64_t n_envs;
+  uint64_t seed;
+  int64_t step;
+};
+
+}  // namespace
+
+struct aht_ctx {
+  int device = 0;
+  cudaStream_t stream = nullptr;
+  aht_env_desc desc{};
+  DevEnv env{};
+  MlpDims mlp{};
+  EnvOps ops{};
+  int32_t n_policies = 0;
+  int64_t n_envs = 0;
+  uint64_t seed = 0;
+  int64_t step = 0;
+  size_t smem_optin = 0;
+  int64_t max_tiles = 0;
+  // device memory, all allocated in aht_create
+  uint32_t* state = nullptr;
+  float* weights = nullptr;
+  int32_t* perm = nullptr;
+  int4* tiles = nullptr;
+  float* xp_returns = nullptr;
+  float* last_value = nullptr;
+  uint32_t* status = nullptr;
+  // pinned host staging for aht_set_policy, and the event pool of the kernel timer
+  float* staging = nullptr;
+  cudaEvent_t upload_done = nullptr;
+  static constexpr int kTimerPairs = 256;
+  cudaEvent_t ev[2 * kTimerPairs] = {};
+  bool timing = false;
+  int n_pending = 0;
+  double timed_ms = 0.0;
+  int64_t timed_launches = 0;
+};
+
+namespace {
+
+Batch batch_of(const aht_ctx* c) {
+  Batch b;
+  b.env = c->env;
+  b.mlp = c->mlp;
+  b.weights = c->weights;
+  b.key = Key{(uint32_t)(c->seed & 0xFFFFFFFFu), (uint32_t)(c->seed >> 32)};
+  b.status = c->status;
+  return b;
+}
+
+aht_status check_env(const aht_env_desc* d, DevEnv* out) {
+  if (!d) return fail(AHT_EINVAL, "env desc is NULL");
+  DevEnv e{};
+  e.kind = d->kind;
+  e.width = d->width;
+  e.height = d->height;
+  e.n_food = d->n_food;
+  e.max_level = d->max_agent_level;
+  e.episode_len = d->episode_len;
+  e.cook_time = d->cook_time;
+  e.soup_reward = d->soup_reward;
+  if (d->kind == AHT_LBF) {
+    if (d->width < 3 || d->width > 12 || d->height < 3 || d->height > 12)
+      return fail(AHT_EINVAL, "LBF width/height must be in 3..12");
+    if (d->n_food < 1 || d->n_food > 3) return fail(AHT_EINVAL, "LBF n_food must be in 1..3");
+    if (d->max_agent_level < 1 || d->max_agent_level > 9)
+      return fail(AHT_EINVAL, "LBF max_agent_level must be in 1..9");
+    if (d->episode_len < 1) return fail(AHT_EINVAL, "LBF episode_len must be >= 1");
+    e.obs_dim = d->width * d->height * 4;
+    e.n_actions = 6;
+  } else if (d->kind == AHT_OVERCOOKED) {
+    if (d->width != 5 || d->height != 4) return fail(AHT_EINVAL, "Overcooked kitchen is 5x4");
+    if (d->episode_len < 1) return fail(AHT_EINVAL, "Overcooked episode_len must be >= 1");
+    if (d->cook_time < 0 || d->cook_time > 255) return fail(AHT_EINVAL, "cook_time must be in 0..255");
+    e.obs_dim = 520;
+    e.n_actions = 6;
+  } else if (d->kind == AHT_HANABI) {
+    if (d->episode_len != 0) return fail(AHT_EINVAL, "Hanabi episode_len must be 0 (to termination)");
+    e.obs_dim = 660;
+    e.n_actions = 20;
+  } else {
+    return fail(AHT_EINVAL, "unknown env kind");
+  }
+  *out = e;
+  return AHT_OK;
+}
+
+MlpDims make_dims(int K, int H0, int H1, int NA) {
+  MlpDims m{};
+  m.K = K;
+  m.KP = (int)align_up(K, 16);
+  m.H0 = H0;
+  m.H1 = H1;
+  m.NA = NA;
+  m.NOP = (int)align_up(NA + 1, 4);
+  int64_t o = 0;
+  m.oW1 = o; o += (int64_t)K * H0;
+  m.ob1 = o; o += H0;
+  m.oW2 = o; o += (int64_t)H0 * H1;
+  m.ob2 = o; o += H1;
+  m.oW3 = o; o += (int64_t)H1 * m.NOP;
+  m.ob3 = o; o += m.NOP;
+  m.stride = align_up(o, 4);
+  return m;
+}
+
+float to_f32(const void* p, int64_t i, int dtype) {
+  if (dtype == AHT_FP32) return static_cast<const float*>(p)[i];
+  uint32_t bits = (uint32_t) static_cast<const uint16_t*>(p)[i] << 16;
+  float f;
+  std::memcpy(&f, &bits, 4);
+  return f;
+}
+
+// Packs one policy into dst (m.stride floats): fp32, transposed [in][out], the last layer
+// padded to NOP columns (column n_actions is the value row when present, else zero).
+aht_status pack_policy(const MlpDims& m, const void* const* W, const void* const* b, int dtype,
+                       int vh, float* dst) {
+  if (vh != 0 && vh != 1) return fail(AHT_EINVAL, "has_value_head entries must be 0 or 1");
+  if (dtype != AHT_FP32 && dtype != AHT_BF16) return fail(AHT_EINVAL, "weight_dtype must be AHT_FP32 or AHT_BF16");
+  const int esz = dtype == AHT_FP32 ? 4 : 2;
+  const int ins[3] = {m.K, m.H0, m.H1};
+  const int outs[3] = {m.H0, m.H1, m.NA + vh};
+  const int64_t oW[3] = {m.oW1, m.oW2, m.oW3}, ob[3] = {m.ob1, m.ob2, m.ob3};
+  const int cols[3] = {m.H0, m.H1, m.NOP};
+  std::fill(dst, dst + m.stride, 0.0f);
+  std::vector<uint8_t> tmp;
+  // Host memory (pageable or pinned) is read in place; device memory is copied first.
+  auto host_view = [&](const void* p, size_t bytes, const void** out) -> bool {
+    cudaPointerAttributes at{};
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) cudaGetLastError();
+    if (at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged) {
+      tmp.resize(bytes);
+      if (cudaMemcpy(tmp.data(), p, bytes, cudaMemcpyDeviceToHost) != cudaSuccess) return false;
+      *out = tmp.data();
+    } else {
+      *out = p;
+    }
+    return true;
+  };
+  for (int l = 0; l < 3; ++l) {
+    if (!W[l] || !b[l]) return fail(AHT_EINVAL, "NULL weight pointer");
+    const void* src = nullptr;
+    if (!host_view(W[l], (size_t)outs[l] * ins[l] * esz, &src)) return fail(AHT_ECUDA, "copying weights failed");
+    for (int n = 0; n < outs[l]; ++n)
+      for (int k = 0; k < ins[l]; ++k)
+        dst[oW[l] + (int64_t)k * cols[l] + n] = to_f32(src, (int64_t)n * ins[l] + k, dtype);
+    if (!host_view(b[l], (size_t)outs[l] * esz, &src)) return fail(AHT_ECUDA, "copying biases failed");
+    for (int n = 0; n < outs[l]; ++n) dst[ob[l] + n] = to_f32(src, n, dtype);
+  }
+  return AHT_OK;
+}
+
+// Kernel timer: events around the main kernel of a call (see aht_set_timing).
+void timer_fold(aht_ctx* c) {
+  for (int i = 0; i < c->n_pending; ++i) {
+    float ms = 0.0f;
+    if (cudaEventSynchronize(c->ev[2 * i + 1]) == cudaSuccess &&
+        cudaEventElapsedTime(&ms, c->ev[2 * i], c->ev[2 * i + 1]) == cudaSuccess) {
+      c->timed_ms += ms;
+      c->timed_launches += 1;
+    }
+  }
+  c->n_pending = 0;
+}
+
+int timer_begin(aht_ctx* c) {
+  if (!c->timing) return -1;
+  if (c->n_pending == aht_ctx::kTimerPairs) timer_fold(c);
+  const int i = c->n_pending++;
+  cudaEventRecord(c->ev[2 * i], c->stream);
+  return i;
+}
+
+void timer_end(aht_ctx* c, int i) {
+  if (i >= 0) cudaEventRecord(c->ev[2 * i + 1], c->stream);
+}
+
+// Tile rows for an M-row launch that fits in shared memory (M multiple of 4).
+int fit_rows(const aht_ctx* c, int want) {
+  int M = (int)align_up(want, 4);
+  while (M > 4 && (size_t)smem_layout(M, c->mlp, c->ops.bytes()).total > c->smem_optin) M = (int)align_up(M / 2, 4);
+  return M;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* aht_last_error(void) { return g_err.c_str(); }
+
+const char* aht_status_string(aht_status s) {
+  switch (s) {
+    case AHT_OK: return "ok";
+    case AHT_EINVAL: return "invalid argument";
+    case AHT_ENOMEM: return "out of device memory";
+    case AHT_ECUDA: return "CUDA error";
+    case AHT_ETIMEOUT: return "device wait timed out";
+    case AHT_EDEVICE: return "device-side error";
+  }
+  return "unknown status";
+}
+
+void aht_destroy(aht_ctx* c) {
+  if (!c) return;
+  DeviceGuard g(c->device);
+  cudaStreamSynchronize(c->stream);
+  cudaFree(c->state);
+  cudaFree(c->weights);
+  cudaFree(c->perm);
+  cudaFree(c->tiles);
+  cudaFree(c->xp_returns);
+  cudaFree(c->last_value);
+  cudaFree(c->status);
+  if (c->staging) cudaFreeHost(c->staging);
+  if (c->upload_done) cudaEventDestroy(c->upload_done);
+  for (auto& e : c->ev)
+    if (e) cudaEventDestroy(e);
+  delete c;
+}
+
+aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t n_envs,
+                      uint64_t seed, void* cuda_stream, aht_ctx** out) {
+  if (!out) return fail(AHT_EINVAL, "out is NULL");
+  *out = nullptr;
+  DevEnv env;
+  aht_status st = check_env(envd, &env);
+  if (st != AHT_OK) return st;
+  if (!pop || !pop->W || !pop->b) return fail(AHT_EINVAL, "population desc or weight arrays are NULL");
+  if (pop->n_policies < 1 || pop->n_policies > 1024) return fail(AHT_EINVAL, "n_policies must be in 1..1024");
+  if (pop->obs_dim != env.obs_dim) return fail(AHT_EINVAL, "obs_dim does not match the env (" + std::to_string(env.obs_dim) + ")");
+  if (pop->n_actions != env.n_actions) return fail(AHT_EINVAL, "n_actions does not match the env (" + std::to_string(env.n_actions) + ")");
+  for (int h : {pop->hidden0, pop->hidden1})
+    if (h < 16 || h > 512 || h % 16) return fail(AHT_EINVAL, "hidden sizes must be multiples of 16 in 16..512");
+  if (pop->weight_dtype != AHT_FP32 && pop->weight_dtype != AHT_BF16) return fail(AHT_EINVAL, "weight_dtype must be AHT_FP32 or AHT_BF16");
+  if (n_envs < 1 || n_envs > (int64_t)1 << 30) return fail(AHT_EINVAL, "n_envs must be in 1..2^30");
+
+  aht_ctx* c = new aht_ctx();
+  c->desc = *envd;
+  c->env = env;
+  c->ops = ops_for(env.kind);
+  c->n_policies = pop->n_policies;
+  c->n_envs = n_envs;
+  c->seed = seed;
+  c->step = 0;
+  c->stream = (cudaStream_t)cuda_stream;
+  c->mlp = make_dims(env.obs_dim, pop->hidden0, pop->hidden1, env.n_actions);
+  auto bail = [&](aht_status s, const std::string& m) {
+    aht_destroy(c);
+    return fail(s, m);
+  };
+  if (cudaGetDevice(&c->device) != cudaSuccess) return bail(AHT_ECUDA, "no CUDA device");
+  int optin = 0;
+  cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, c->device);
+  c->smem_optin = (size_t)optin;
+
+  const MlpDims& m = c->mlp;
+  std::vector<float> packed((size_t)m.stride * pop->n_policies, 0.0f);
+  for (int p = 0; p < pop->n_policies; ++p) {
+    const int vh = pop->has_value_head ? pop->has_value_head[p] : 0;
+    aht_status ps = pack_policy(m, pop->W + 3 * p, pop->b + 3 * p, pop->weight_dtype, vh,
+                                packed.data() + (size_t)p * m.stride);
+    if (ps != AHT_OK) {
+      std::string msg = g_err;
+      return bail(ps, msg);
+    }
+  }
+
+  const int words = c->ops.words();
+  c->max_tiles = (n_envs + 3) / 4 + kMaxPool;
+  struct Alloc { void** p; size_t bytes; };
+  Alloc allocs[] = {
+      {(void**)&c->state, (size_t)words * n_envs * 4},
+      {(void**)&c->weights, packed.size() * 4},
+      {(void**)&c->perm, (size_t)n_envs * 4},
+      {(void**)&c->tiles, (size_t)c->max_tiles * sizeof(int4)},
+      {(void**)&c->xp_returns, (size_t)n_envs * 4},
+      {(void**)&c->last_value, (size_t)n_envs * 4},
+      {(void**)&c->status, 4},
+  };
+  for (auto& a : allocs)
+    if (cudaMalloc(a.p, a.bytes) != cudaSuccess) {
+      cudaGetLastError();
+      return bail(AHT_ENOMEM, "cudaMalloc of " + std::to_string(a.bytes) + " bytes failed");
+    }
+  if (cudaMemcpy(c->weights, packed.data(), packed.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
+      cudaMemset(c->status, 0, 4) != cudaSuccess)
+    return bail(AHT_ECUDA, "uploading the population failed");
+  if (c->ops.smem_limit(c->smem_optin) != cudaSuccess || policy_set_smem_limit(c->smem_optin) != cudaSuccess)
+    return bail(AHT_ECUDA, "setting the shared-memory limit failed");
+  if (cudaMallocHost((void**)&c->staging, (size_t)m.stride * 4) != cudaSuccess)
+    return bail(AHT_ENOMEM, "pinned staging allocation failed");
+  if (cudaEventCreateWithFlags(&c->upload_done, cudaEventDisableTiming) != cudaSuccess)
+    return bail(AHT_ECUDA, "cudaEventCreate failed");
+  for (auto& e : c->ev)
+    if (cudaEventCreate(&e) != cudaSuccess) return bail(AHT_ECUDA, "cudaEventCreate failed");
+  *out = c;
+  aht_status r = aht_reset(c, seed);
+  if (r != AHT_OK) {
+    *out = nullptr;
+    std::string msg = g_err;
+    aht_destroy(c);
+    return fail(r, msg);
+  }
+  if (cudaStreamSynchronize(c->stream) != cudaSuccess) {
+    *out = nullptr;
+    aht_destroy(c);
+    return fail(AHT_ECUDA, "reset kernel failed");
+  }
+  return AHT_OK;
+}
+
+aht_status aht_reset(aht_ctx* c, uint64_t seed) {
+  if (!c) return fail(AHT_EINVAL, "ctx is NULL");
+  DeviceGuard g(c->device);
+  c->seed = seed;
+  c->step = 0;
+  ResetArgs a{batch_of(c), c->state, c->n_envs, 0u};
+  AHT_CUDA(c->ops.reset(a, c->stream));
+  return AHT_OK;
+}
+
+aht_status aht_rollout(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t pool_size,
+                       int32_t T, const aht_traj* out) {
+  if (!c || !out) return fail(AHT_EINVAL, "ctx or out is NULL");
+  if (c->env.kind == AHT_HANABI) return fail(AHT_EINVAL, "PPO collection needs a simultaneous-move env (LBF, Overcooked)");
+  if (ego_id < 0 || ego_id >= c->n_policies) return fail(AHT_EINVAL, "ego_id out of range");
+  if (!pool || pool_size < 1 || pool_size > kMaxPool) return fail(AHT_EINVAL, "pool_size must be in 1..256");
+  for (int k = 0; k < pool_size; ++k)
+    if (pool[k] < 0 || pool[k] >= c->n_policies) return fail(AHT_EINVAL, "pool id out of range");
+  if (T < 1) return fail(AHT_EINVAL, "T must be >= 1");
+  if (c->step + T + 1 > (int64_t)UINT32_MAX) return fail(AHT_EINVAL, "step counter would exceed 2^32");
+  if (out->advantages && (!out->rewards || !out->values || !out->dones))
+    return fail(AHT_EINVAL, "advantages need rewards, values and dones");
+  if (out->gamma < 0.f || out->gamma > 1.f || out->lambda < 0.f || out->lambda > 1.f)
+    return fail(AHT_EINVAL, "gamma and lambda must be in [0, 1]");
+  DeviceGuard g(c->device);
+  const int M = fit_rows(c, 128);
+
+  GroupArgs ga{};
+  ga.key = batch_of(c).key;
+  ga.n_envs = c->n_envs;
+  ga.step0 = (uint32_t)c->step;
+  ga.pool_size = pool_size;
+  for (int k = 0; k < pool_size; ++k) ga.pool[k] = pool[k];
+  ga.M = M;
+  ga.max_tiles = (int)((c->n_envs + M - 1) / M + pool_size);
+  ga.perm = c->perm;
+  ga.tiles = c->tiles;
+  ga.teammate = out->teammate;
+  AHT_CUDA(launch_group(ga, c->stream));
+
+  PpoArgs a{};
+  a.b = batch_of(c);
+  a.state = c->state;
+  a.n_envs = c->n_envs;
+  a.perm = c->perm;
+  a.tiles = c->tiles;
+  a.M = M;
+  a.ego = ego_id;
+  a.step0 = (uint32_t)c->step;
+  a.T = T;
+  a.traj = TrajPtrs{out->obs, out->actions, out->tm_actions, out->logp, out->values,
+                    out->rewards, out->dones,
+                    out->last_value ? out->last_value : (out->advantages ? c->last_value : nullptr)};
+  const size_t smem = smem_layout(M, c->mlp, c->ops.bytes()).total;
+  const int tk = timer_begin(c);
+  AHT_CUDA(c->ops.ppo(a, ga.max_tiles, smem, c->stream));
+  timer_end(c, tk);
+  if (out->advantages)
+    AHT_CUDA(launch_gae(out->rewards, out->values, out->dones, a.traj.last_value, c->n_envs, T,
+                        out->gamma, out->lambda, out->advantages, out->targets, c->stream));
+  c->step += T;
+  return AHT_OK;
+}
+
+aht_status aht_xplay_matrix(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego,
+                            const int32_t* tm_ids, int32_t n_tm, int32_t envs_per_pair,
+                            int32_t max_steps, const aht_xplay_out* out) {
+  if (!c || !out) return fail(AHT_EINVAL, "ctx or out is NULL");
+  if (!ego_ids || !tm_ids || n_ego < 1 || n_tm < 1 || n_ego > kMaxXpIds || n_tm > kMaxXpIds)
+    return fail(AHT_EINVAL, "n_ego and n_tm must be in 1..64");
+  for (int i = 0; i < n_ego; ++i)
+    if (ego_ids[i] < 0 || ego_ids[i] >= c->n_policies) return fail(AHT_EINVAL, "ego id out of range");
+  for (int j = 0; j < n_tm; ++j)
+    if (tm_ids[j] < 0 || tm_ids[j] >= c->n_policies) return fail(AHT_EINVAL, "teammate id out of range");
+  if (envs_per_pair < 1 || envs_per_pair > (1 << 14)) return fail(AHT_EINVAL, "envs_per_pair must be in 1..16384");
+  if (max_steps < 1) return fail(AHT_EINVAL, "max_steps must be >= 1");
+  const int64_t n_pairs = (int64_t)n_ego * n_tm;
+  const int64_t n_total = n_pairs * envs_per_pair;
+  if (n_total > c->n_envs) return fail(AHT_EINVAL, "n_ego*n_tm*envs_per_pair exceeds the context's n_envs");
+  if (c->step + max_steps + 1 > (int64_t)UINT32_MAX) return fail(AHT_EINVAL, "step counter would exceed 2^32");
+  DeviceGuard g(c->device);
+  const int M = fit_rows(c, std::min(c->ops.max_rows, envs_per_pair));
+  XpArgs a{};
+  a.b = batch_of(c);
+  a.n_ego = n_ego;
+  a.n_tm = n_tm;
+  a.P = envs_per_pair;
+  a.max_steps = max_steps;
+  for (int i = 0; i < n_ego; ++i) a.ego_ids[i] = ego_ids[i];
+  for (int j = 0; j < n_tm; ++j) a.tm_ids[j] = tm_ids[j];
+  a.M = M;
+  a.tiles_per_pair = (envs_per_pair + M - 1) / M;
+  a.step0 = (uint32_t)c->step;
+  a.returns = out->returns ? out->returns : c->xp_returns;
+  a.steps = out->steps;
+  a.actions = out->actions;
+  if (out->actions) AHT_CUDA(cudaMemsetAsync(out->actions, 255, (size_t)max_steps * n_total * 2, c->stream));
+  const size_t smem = smem_layout(M, c->mlp, c->ops.bytes()).total;
+  const int64_t grid = n_pairs * a.tiles_per_pair;
+  if (grid > INT32_MAX) return fail(AHT_EINVAL, "too many tiles");
+  const int tk = timer_begin(c);
+  AHT_CUDA(c->ops.xplay(a, (int)grid, smem, c->stream));
+  timer_end(c, tk);
+  if (out->matrix) AHT_CUDA(launch_xp_reduce(a.returns, n_pairs, envs_per_pair, out->matrix, c->stream));
+  c->step += max_steps;
+  return AHT_OK;
+}
+
+aht_status aht_gae(const float* r, const float* v, const uint8_t* d, const float* v_last,
+                   int64_t n_envs, int32_t T, float gamma, float lambda, float* adv,
+                   float* tgt, void* cuda_stream) {
+  if (!r || !v || !d || !v_last || !adv) return fail(AHT_EINVAL, "NULL input or output");
+  if (n_envs < 1 || T < 1) return fail(AHT_EINVAL, "n_envs and T must be >= 1");
+  if (gamma < 0.f || gamma > 1.f || lambda < 0.f || lambda > 1.f)
+    return fail(AHT_EINVAL, "gamma and lambda must be in [0, 1]");
+  AHT_CUDA(launch_gae(r, v, d, v_last, n_envs, T, gamma, lambda, adv, tgt, (cudaStream_t)cuda_stream));
+  return AHT_OK;
+}
+
+aht_status aht_step_forced(aht_ctx* c, const uint8_t* actions, const aht_step_out* out) {
+  if (!c || !actions || !out) return fail(AHT_EINVAL, "NULL argument");
+  if (c->step + 2 > (int64_t)UINT32_MAX) return fail(AHT_EINVAL, "step counter would exceed 2^32");
+  DeviceGuard g(c->device);
+  ForcedArgs a{batch_of(c), c->state, c->n_envs, (uint32_t)c->step, actions, out->rewards,
+               out->team, out->dones, out->obs};
+  AHT_CUDA(c->ops.forced(a, c->stream));
+  c->step += 1;
+  return AHT_OK;
+}
+
+aht_status aht_policy_forward(aht_ctx* c, int32_t policy, const uint8_t* obs, int64_t n,
+                              float* out) {
+  if (!c || !obs || !out) return fail(AHT_EINVAL, "NULL argument");
+  if (policy < 0 || policy >= c->n_policies) return fail(AHT_EINVAL, "policy out of range");
+  if (n < 1) return fail(AHT_EINVAL, "n must be >= 1");
+  DeviceGuard g(c->device);
+  PolicyArgs a{batch_of(c), policy, obs, n, out, 0};
+  a.M = fit_rows(c, 64);
+  const size_t smem = smem_layout(a.M, c->mlp, 0).total;
+  const int64_t grid = (n + a.M - 1) / a.M;
+  if (grid > INT32_MAX) return fail(AHT_EINVAL, "n too large");
+  AHT_CUDA(launch_policy(a, (int)grid, smem, c->stream));
+  return AHT_OK;
+}
+
+aht_status aht_get_state(aht_ctx* c, void* buf, size_t* bytes) {
+  if (!c || !bytes) return fail(AHT_EINVAL, "NULL argument");
+  const size_t body = (size_t)c->ops.words() * c->n_envs * 4;
+  const size_t need = sizeof(StateHeader) + body;
+  if (!buf) {
+    *bytes = need;
+    return AHT_OK;
+  }
+  if (*bytes < need) return fail(AHT_EINVAL, "state buffer too small");
+  DeviceGuard g(c->device);
+  StateHeader h{kStateMagic, (uint32_t)c->env.kind, (uint32_t)c->ops.words(), 0, c->n_envs, c->seed, c->step};
+  std::memcpy(buf, &h, sizeof(h));
+  AHT_CUDA(cudaMemcpyAsync(static_cast<uint8_t*>(buf) + sizeof(h), c->state, body, cudaMemcpyDeviceToHost, c->stream));
+  AHT_CUDA(cudaStreamSynchronize(c->stream));
+  *bytes = need;
+  return AHT_OK;
+}
+
+aht_status aht_set_state(aht_ctx* c, const void* buf, size_t bytes) {
+  if (!c || !buf || bytes < sizeof(StateHeader)) return fail(AHT_EINVAL, "NULL or short buffer");
+  StateHeader h;
+  std::memcpy(&h, buf, sizeof(h));
+  const size_t body = (size_t)c->ops.words() * c->n_envs * 4;
+  if (h.magic != kStateMagic || h.kind != (uint32_t)c->env.kind || h.n_words != (uint32_t)c->ops.words() ||
+      h.n_envs != c->n_envs || bytes != sizeof(h) + body)
+    return fail(AHT_EINVAL, "state buffer does not match this context");
+  DeviceGuard g(c->device);
+  AHT_CUDA(cudaMemcpyAsync(c->state, static_cast<const uint8_t*>(buf) + sizeof(h), body, cudaMemcpyHostToDevice, c->stream));
+  AHT_CUDA(cudaStreamSynchronize(c->stream));
+  c->seed = h.seed;
+  c->step = h.step;
+  return AHT_OK;
+}
+
+aht_status aht_set_policy(aht_ctx* c, int32_t policy, const void* const* W, const void* const* b,
+                          int32_t weight_dtype, int32_t has_value_head) {
+  if (!c || !W || !b) return fail(AHT_EINVAL, "NULL argument");
+  if (policy < 0 || policy >= c->n_policies) return fail(AHT_EINVAL, "policy out of range");
+  DeviceGuard g(c->device);
+  AHT_CUDA(cudaEventSynchronize(c->upload_done));  // the staging buffer is free again
+  aht_status ps = pack_policy(c->mlp, W, b, weight_dtype, has_value_head, c->staging);
+  if (ps != AHT_OK) return ps;
+  AHT_CUDA(cudaMemcpyAsync(c->weights + (int64_t)policy * c->mlp.stride, c->staging,
+                           (size_t)c->mlp.stride * 4, cudaMemcpyHostToDevice, c->stream));
+  AHT_CUDA(cudaEventRecord(c->upload_done, c->stream));
+  return AHT_OK;
+}
+
+aht_status aht_set_timing(aht_ctx* c, int32_t enable) {
+  if (!c) return fail(AHT_EINVAL, "ctx is NULL");
+  c->timing = enable != 0;
+  return AHT_OK;
+}
+
+aht_status aht_get_timing(aht_ctx* c, double* kernel_ms, int64_t* launches) {
+  if (!c || !kernel_ms || !launches) return fail(AHT_EINVAL, "NULL argument");
+  DeviceGuard g(c->device);
+  AHT_CUDA(cudaStreamSynchronize(c->stream));
+  timer_fold(c);
+  *kernel_ms = c->timed_ms;
+  *launches = c->timed_launches;
+  c->timed_ms = 0.0;
+  c->timed_launches = 0;
+  return AHT_OK;
+}
+
+int64_t aht_step_counter(const aht_ctx* c) { return c ? c->step : -1; }
+
+aht_status aht_sync(aht_ctx* c) {
+  if (!c) return fail(AHT_EINVAL, "ctx is NULL");
+  DeviceGuard g(c->device);
+  AHT_CUDA(cudaStreamSynchronize(c->stream));
+  uint32_t s = 0;
+  AHT_CUDA(cudaMemcpy(&s, c->status, 4, cudaMemcpyDeviceToHost));
+  if (s != 0) {
+    AHT_CUDA(cudaMemset(c->status, 0, 4));
+    return fail(AHT_EDEVICE, "device status word 0x" + [&] { char b[16]; std::snprintf(b, sizeof b, "%x", s); return std::string(b); }() +
+                                 " (1 illegal action, 2 actor mismatch, 4 bad policy)");
+  }
+  return AHT_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,88 @@
+// aht_common.cuh -- types and device helpers shared by the libaht kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/aht.h"
+
+namespace aht {
+
+constexpr int kThreads = 256;       // threads per CTA of the rollout kernels
+constexpr int kMaxPool = 256;       // teammate pool entries passed by value
+constexpr int kMaxXpIds = 64;       // ego / teammate ids per cross-play call
+constexpr int kGroupThreads = 128;  // threads of the teammate-grouping kernel
+
+// Device status word bits (latched with atomicOr, read by aht_sync).
+enum : uint32_t {
+  kStatusIllegalAction = 1u,
+  kStatusActorMismatch = 2u,
+  kStatusBadPolicy = 4u,
+};
+
+// Philox streams (counter word 2).
+enum : uint32_t { kStreamAct0 = 0, kStreamAct1 = 1, kStreamReset = 2, kStreamTeammate = 3 };
+
+struct DevEnv {
+  int32_t kind, width, height, n_food, max_level, episode_len, cook_time, soup_reward;
+  int32_t obs_dim, n_actions;
+};
+
+// Packed fp32 policy: Wt1 [K][H0], b1 [H0], Wt2 [H0][H1], b2 [H1], Wt3 [H1][NOP], b3 [NOP]
+// (transposed, so a warp reading one k row of W reads consecutive outputs).
+struct MlpDims {
+  int32_t K, KP, H0, H1, NA, NOP;
+  int64_t stride;  // floats per policy
+  int64_t oW1, ob1, oW2, ob2, oW3, ob3;
+};
+
+struct Key {
+  uint32_t k0, k1;
+};
+
+// ---- Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11) -------------------------------
+__device__ __forceinline__ uint4 philox(uint4 c, Key key) {
+  uint32_t k0 = key.k0, k1 = key.k1;
+#pragma unroll
+  for (int i = 0; i < 10; ++i) {
+    const uint32_t hi0 = __umulhi(0xD2511F53u, c.x), lo0 = 0xD2511F53u * c.x;
+    const uint32_t hi1 = __umulhi(0xCD9E8D57u, c.z), lo1 = 0xCD9E8D57u * c.z;
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+    k0 += 0x9E3779B9u;
+    k1 += 0xBB67AE85u;
+  }
+  return c;
+}
+
+// First word of block 0 of (env, step, stream): one draw per action / teammate choice.
+__device__ __forceinline__ uint32_t draw0(Key key, uint32_t env, uint32_t step, uint32_t stream) {
+  return philox(make_uint4(env, step, stream, 0u), key).x;
+}
+
+// Successive draws of one (env, step, stream): draw n is word n % 4 of block n / 4.
+struct DrawSeq {
+  Key key;
+  uint32_t env, step, stream, n;
+  uint4 blk;
+  __device__ DrawSeq(Key k, uint32_t e, uint32_t t, uint32_t s)
+      : key(k), env(e), step(t), stream(s), n(0) {}
+  __device__ uint32_t next() {
+    const uint32_t w = n & 3u;
+    if (w == 0) blk = philox(make_uint4(env, step, stream, n >> 2), key);
+    ++n;
+    return w == 0 ? blk.x : (w == 1 ? blk.y : (w == 2 ? blk.z : blk.w));
+  }
+};
+
+// floor(x * n / 2^32)
+__device__ __forceinline__ uint32_t uniform_int(uint32_t x, uint32_t n) { return __umulhi(x, n); }
+// (x >> 8) * 2^-24, exact in fp32
+__device__ __forceinline__ float u01(uint32_t x) {
+  return __uint2float_rn(x >> 8) * (1.0f / 16777216.0f);
+}
+
+__host__ __device__ constexpr inline int64_t align_up(int64_t x, int64_t a) {
+  return (x + a - 1) / a * a;
+}
+
+}  // namespace aht

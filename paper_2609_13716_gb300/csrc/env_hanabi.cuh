@@ -1,0 +1,246 @@
+// env_hanabi.cuh -- 2-player Hanabi on the device (one thread per env).
+//
+// 50-card deck (5 colours x ranks 1,1,1,2,2,3,3,4,4,5), 5-card hands, 8 info and 3 life
+// tokens, 20 actions (play slot 0-4, discard slot 0-4, hint colour 0-4, hint rank 1-5),
+// seat 0 first.  Card type = colour*5 + rank-1.  Rules and the 660-bit observation as
+// read in DESIGN.md "Readings".
+#pragma once
+#include "aht_common.cuh"
+
+namespace aht {
+
+struct EnvHanabi {
+  static constexpr bool kTurnBased = true;
+  static constexpr int kTurnCap = 100;
+  struct State {
+    uint8_t deck[52];
+    uint8_t hand[2][5];
+    uint8_t n_hand[2];
+    uint32_t know[2][5];    // possible card types, 25 bits
+    uint16_t hints[2][5];   // explicit hints received: bits 0-4 colour, 5-9 rank
+    uint8_t fw[5], info, lives, score;
+    uint8_t disc[25], ptr, turn;
+    int8_t fr;              // final-round turns left, -1 while the deck has cards
+    uint8_t la_flags;       // bit0 valid, bit1 actor seat, bit2 play success, bit3 bomb
+    uint8_t la_type, la_colour, la_rank, la_slot, la_card, la_hinted, la_pad;
+    float ret;
+  };
+  static constexpr int kWords = sizeof(State) / 4;
+
+  __device__ static uint32_t colour_bits(int c) { return 0x1Fu << (5 * c); }
+  __device__ static uint32_t rank_bits(int r0) { return 0x108421u << r0; }  // rank index 0..4
+
+  __device__ static void reset(const DevEnv&, Key key, uint32_t env, uint32_t step, State& s) {
+    // canonical order: colour c, copies of ranks 1,1,1,2,2,3,3,4,4,5
+    for (int c = 0; c < 5; ++c) {
+      uint8_t* p = s.deck + c * 10;
+      const uint8_t b = (uint8_t)(c * 5);
+      p[0] = p[1] = p[2] = b;
+      p[3] = p[4] = b + 1;
+      p[5] = p[6] = b + 2;
+      p[7] = p[8] = b + 3;
+      p[9] = b + 4;
+    }
+    s.deck[50] = s.deck[51] = 0;
+    DrawSeq r(key, env, step, kStreamReset);
+    for (int i = 49; i >= 1; --i) {
+      const int j = (int)uniform_int(r.next(), (uint32_t)(i + 1));
+      const uint8_t t = s.deck[i];
+      s.deck[i] = s.deck[j];
+      s.deck[j] = t;
+    }
+    for (int p = 0; p < 2; ++p) {
+      for (int k = 0; k < 5; ++k) {
+        s.hand[p][k] = s.deck[p * 5 + k];
+        s.know[p][k] = 0x1FFFFFFu;
+        s.hints[p][k] = 0;
+      }
+      s.n_hand[p] = 5;
+    }
+    for (int c = 0; c < 5; ++c) s.fw[c] = 0;
+    for (int t = 0; t < 25; ++t) s.disc[t] = 0;
+    s.info = 8;
+    s.lives = 3;
+    s.score = 0;
+    s.ptr = 10;
+    s.turn = 0;
+    s.fr = -1;
+    s.la_flags = 0;
+    s.la_type = s.la_colour = s.la_rank = s.la_slot = s.la_card = s.la_hinted = s.la_pad = 0;
+    s.ret = 0.0f;
+  }
+
+  __device__ static int actor(const State& s) { return s.turn & 1; }
+
+  __device__ static uint32_t legal(const State& s) {
+    const int me = s.turn & 1, pa = me ^ 1;
+    uint32_t m = 0;
+    for (int k = 0; k < s.n_hand[me]; ++k) {
+      m |= 1u << k;
+      if (s.info < 8) m |= 1u << (5 + k);
+    }
+    if (s.info > 0) {
+      for (int k = 0; k < s.n_hand[pa]; ++k) {
+        const int card = s.hand[pa][k];
+        m |= 1u << (10 + card / 5);
+        m |= 1u << (15 + card % 5);
+      }
+    }
+    return m;
+  }
+
+  __device__ static void remove_slot(State& s, int p, int slot) {
+    const int n = s.n_hand[p];
+    for (int k = slot; k < n - 1; ++k) {
+      s.hand[p][k] = s.hand[p][k + 1];
+      s.know[p][k] = s.know[p][k + 1];
+      s.hints[p][k] = s.hints[p][k + 1];
+    }
+    s.hand[p][n - 1] = 0;
+    s.know[p][n - 1] = 0;
+    s.hints[p][n - 1] = 0;
+    s.n_hand[p] = (uint8_t)(n - 1);
+  }
+
+  // Applies the acting seat's action (a0 for seat 0, a1 for seat 1).  Returns done,
+  // or -1 (state untouched) for an illegal action.
+  __device__ static int step(const DevEnv&, State& s, int a0, int a1, float& r0, float& r1,
+                             float& team) {
+    const int me = s.turn & 1, pa = me ^ 1;
+    const int a = me == 0 ? a0 : a1;
+    if (a < 0 || a >= 20 || !((legal(s) >> a) & 1u)) {
+      r0 = r1 = team = 0.0f;
+      return -1;
+    }
+    const int fr_start = s.fr;
+    const int score_before = s.score;
+    float reward = 0.0f;
+    uint8_t flags = (uint8_t)(1u | (me << 1));
+    s.la_colour = 255;
+    s.la_rank = 0;
+    s.la_slot = 255;
+    s.la_card = 255;
+    s.la_hinted = 0;
+    if (a < 10) {
+      const int slot = a % 5;
+      const int card = s.hand[me][slot];
+      const int c = card / 5, rank = card % 5 + 1;
+      s.la_type = a < 5 ? 0 : 1;
+      s.la_colour = (uint8_t)c;
+      s.la_rank = (uint8_t)rank;
+      s.la_slot = (uint8_t)slot;
+      s.la_card = (uint8_t)card;
+      remove_slot(s, me, slot);
+      if (a < 5) {
+        if (s.fw[c] == rank - 1) {
+          s.fw[c] = (uint8_t)rank;
+          s.score += 1;
+          reward = 1.0f;
+          if (rank == 5 && s.info < 8) s.info += 1;
+          flags |= 4u;
+        } else {
+          s.lives -= 1;
+          s.disc[card] += 1;
+          flags |= 8u;
+        }
+      } else {
+        s.disc[card] += 1;
+        s.info += 1;
+      }
+      if (s.ptr < 50) {
+        const int k = s.n_hand[me];
+        s.hand[me][k] = s.deck[s.ptr];
+        s.know[me][k] = 0x1FFFFFFu;
+        s.hints[me][k] = 0;
+        s.n_hand[me] = (uint8_t)(k + 1);
+        s.ptr += 1;
+        if (s.ptr == 50) s.fr = 2;
+      }
+    } else {
+      const bool by_colour = a < 15;
+      const int v = (a - 10) % 5;
+      const uint32_t bits = by_colour ? colour_bits(v) : rank_bits(v);
+      s.info -= 1;
+      s.la_type = by_colour ? 2 : 3;
+      if (by_colour) s.la_colour = (uint8_t)v;
+      else s.la_rank = (uint8_t)(v + 1);
+      uint8_t hinted = 0;
+      for (int k = 0; k < s.n_hand[pa]; ++k) {
+        const int card = s.hand[pa][k];
+        if (by_colour ? (card / 5 == v) : (card % 5 == v)) {
+          s.know[pa][k] &= bits;
+          s.hints[pa][k] |= (uint16_t)(1u << (by_colour ? v : 5 + v));
+          hinted |= (uint8_t)(1u << k);
+        } else {
+          s.know[pa][k] &= ~bits;
+        }
+      }
+      s.la_hinted = hinted;
+    }
+    s.la_flags = flags;
+    s.turn += 1;
+    int done = 0;
+    if (s.lives == 0) {
+      done = 1;
+      reward = -(float)score_before;
+    } else if (s.score == 25) {
+      done = 1;
+    } else if (fr_start >= 1) {
+      s.fr = (int8_t)(fr_start - 1);
+      done = s.fr == 0;
+    }
+    if (!done && s.turn >= kTurnCap) done = 1;
+    r0 = r1 = team = reward;
+    s.ret = __fadd_rn(s.ret, reward);
+    return done;
+  }
+
+  // 660 binary features for `seat` (see the section offsets below).
+  __device__ static void obs(const DevEnv&, const State& s, int seat, uint8_t* row) {
+    uint32_t* w = reinterpret_cast<uint32_t*>(row);
+    for (int i = 0; i < 165; ++i) w[i] = 0u;
+    const int me = seat, pa = seat ^ 1;
+    for (int k = 0; k < s.n_hand[pa]; ++k) row[k * 25 + s.hand[pa][k]] = 1;       // [0,125)
+    for (int q = 0; q < 2; ++q) {                                                // [125,375)
+      const int who = q == 0 ? me : pa;
+      uint8_t* o = row + 125 + q * 125;
+      for (int k = 0; k < s.n_hand[who]; ++k) {
+        const uint32_t m = s.know[who][k];
+        for (int b = 0; b < 25; ++b) o[k * 25 + b] = (uint8_t)((m >> b) & 1u);
+      }
+    }
+    for (int c = 0; c < 5; ++c)                                                  // [375,400)
+      if (s.fw[c]) row[375 + c * 5 + s.fw[c] - 1] = 1;
+    for (int i = 0; i < s.info; ++i) row[400 + i] = 1;                           // [400,408)
+    for (int i = 0; i < s.lives; ++i) row[408 + i] = 1;                          // [408,411)
+    for (int i = 0; i < 50 - s.ptr; ++i) row[411 + i] = 1;                       // [411,451)
+    const uint8_t base[5] = {0, 3, 5, 7, 9};
+    for (int t = 0; t < 25; ++t)                                                 // [451,501)
+      for (int i = 0; i < s.disc[t]; ++i) row[451 + (t / 5) * 10 + base[t % 5] + i] = 1;
+    if (s.la_flags & 1u) {                                                       // [501,554)
+      uint8_t* o = row + 501;
+      o[((s.la_flags >> 1) & 1u) == (uint32_t)me ? 0 : 1] = 1;
+      o[2 + s.la_type] = 1;
+      if (s.la_colour != 255) o[6 + s.la_colour] = 1;
+      if (s.la_rank) o[11 + s.la_rank - 1] = 1;
+      if (s.la_slot != 255) o[16 + s.la_slot] = 1;
+      if (s.la_card != 255) o[21 + s.la_card] = 1;
+      for (int k = 0; k < 5; ++k)
+        if ((s.la_hinted >> k) & 1u) o[46 + k] = 1;
+      if (s.la_flags & 4u) o[51] = 1;
+      if (s.la_flags & 8u) o[52] = 1;
+    }
+    for (int q = 0; q < 2; ++q) {                                                // [554,654)
+      const int who = q == 0 ? me : pa;
+      uint8_t* o = row + 554 + q * 50;
+      for (int k = 0; k < 5; ++k)
+        for (int b = 0; b < 10; ++b) o[k * 10 + b] = (uint8_t)((s.hints[who][k] >> b) & 1u);
+    }
+    for (int k = 0; k < s.n_hand[me]; ++k) row[654 + k] = 1;                     // [654,659)
+    if (s.fr >= 0) row[659] = 1;                                                 // [659]
+  }
+
+  __device__ static float ret(const State& s) { return s.ret; }
+};
+
+}  // namespace aht

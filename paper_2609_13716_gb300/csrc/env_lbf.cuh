@@ -1,0 +1,138 @@
+// env_lbf.cuh -- Level-Based Foraging on the device (one thread per env).
+//
+// Rules (the workload's statement): two agents with levels in
+// 1..max_level, n_food foods with levels in 1..(sum of agent levels); actions
+// {noop, N, S, W, E, load}; a food is eaten when the summed levels of the 4-adjacent
+// loading agents reach its level, each loader receiving food_level*agent_level /
+// (loader_level_sum * total_food_level).  Moves resolve on the pre-step state.
+#pragma once
+#include "aht_common.cuh"
+
+namespace aht {
+
+struct EnvLbf {
+  static constexpr bool kTurnBased = false;
+  struct State {
+    uint8_t ax[2], ay[2];
+    uint8_t al[2], F, eaten;  // eaten: bit k set when food k is gone (absent foods too)
+    uint8_t fx[4], fy[4], fl[4];
+    uint32_t ep_t;
+    float ret;
+  };
+  static constexpr int kWords = sizeof(State) / 4;
+
+  __device__ static void reset(const DevEnv& d, Key key, uint32_t env, uint32_t step, State& s) {
+    DrawSeq r(key, env, step, kStreamReset);
+    s.al[0] = (uint8_t)(1 + uniform_int(r.next(), (uint32_t)d.max_level));
+    s.al[1] = (uint8_t)(1 + uniform_int(r.next(), (uint32_t)d.max_level));
+    const uint32_t lsum = s.al[0] + s.al[1];
+    uint32_t F = 0;
+    for (int k = 0; k < d.n_food; ++k) {
+      s.fl[k] = (uint8_t)(1 + uniform_int(r.next(), lsum));
+      F += s.fl[k];
+    }
+    s.F = (uint8_t)F;
+    // n_food + 2 steps of a Fisher-Yates shuffle of the cell indices, with the touched
+    // entries of the permutation kept in a small map (untouched entry p holds p).
+    const int cells = d.width * d.height;
+    int key_[10], val_[10], nmap = 0;
+    auto get = [&](int p) {
+      for (int m = 0; m < nmap; ++m)
+        if (key_[m] == p) return val_[m];
+      return p;
+    };
+    auto set = [&](int p, int v) {
+      for (int m = 0; m < nmap; ++m)
+        if (key_[m] == p) { val_[m] = v; return; }
+      key_[nmap] = p; val_[nmap] = v; ++nmap;
+    };
+    int placed[5];
+    const int n_obj = d.n_food + 2;
+    for (int i = 0; i < n_obj; ++i) {
+      const int j = i + (int)uniform_int(r.next(), (uint32_t)(cells - i));
+      const int vi = get(i), vj = get(j);
+      set(i, vj);
+      set(j, vi);
+      placed[i] = vj;
+    }
+    s.eaten = 0;
+    for (int k = 0; k < 3; ++k) {
+      if (k < d.n_food) {
+        s.fx[k] = (uint8_t)(placed[k] % d.width);
+        s.fy[k] = (uint8_t)(placed[k] / d.width);
+      } else {
+        s.fx[k] = s.fy[k] = s.fl[k] = 0;
+        s.eaten |= (uint8_t)(1u << k);
+      }
+    }
+    s.fx[3] = s.fy[3] = s.fl[3] = 0;
+    for (int i = 0; i < 2; ++i) {
+      s.ax[i] = (uint8_t)(placed[d.n_food + i] % d.width);
+      s.ay[i] = (uint8_t)(placed[d.n_food + i] / d.width);
+    }
+    s.ep_t = 0;
+    s.ret = 0.0f;
+  }
+
+  __device__ static int step(const DevEnv& d, State& s, int a0, int a1, float& r0, float& r1,
+                             float& team) {
+    r0 = 0.0f;
+    r1 = 0.0f;
+    uint32_t newly = 0;
+    for (int k = 0; k < d.n_food; ++k) {
+      if ((s.eaten >> k) & 1u) continue;
+      const bool l0 = a0 == 5 && abs((int)s.ax[0] - s.fx[k]) + abs((int)s.ay[0] - s.fy[k]) == 1;
+      const bool l1 = a1 == 5 && abs((int)s.ax[1] - s.fx[k]) + abs((int)s.ay[1] - s.fy[k]) == 1;
+      const int lsum = (l0 ? s.al[0] : 0) + (l1 ? s.al[1] : 0);
+      if (lsum > 0 && lsum >= s.fl[k]) {
+        newly |= 1u << k;
+        const float den = (float)(lsum * (int)s.F);
+        if (l0) r0 = __fadd_rn(r0, __fdiv_rn((float)(s.fl[k] * s.al[0]), den));
+        if (l1) r1 = __fadd_rn(r1, __fdiv_rn((float)(s.fl[k] * s.al[1]), den));
+      }
+    }
+    int tx[2], ty[2];
+    const int act[2] = {a0, a1};
+    for (int i = 0; i < 2; ++i) {
+      const int a = act[i];
+      const int dx = (a == 4) - (a == 3), dy = (a == 2) - (a == 1);
+      int x = s.ax[i] + dx, y = s.ay[i] + dy;
+      bool ok = (dx | dy) != 0 && x >= 0 && x < d.width && y >= 0 && y < d.height;
+      for (int k = 0; k < d.n_food && ok; ++k)
+        if (!((s.eaten >> k) & 1u) && s.fx[k] == x && s.fy[k] == y) ok = false;
+      if (ok && ((s.ax[0] == x && s.ay[0] == y) || (s.ax[1] == x && s.ay[1] == y))) ok = false;
+      tx[i] = ok ? x : s.ax[i];
+      ty[i] = ok ? y : s.ay[i];
+    }
+    if (!(tx[0] == tx[1] && ty[0] == ty[1])) {
+      for (int i = 0; i < 2; ++i) {
+        s.ax[i] = (uint8_t)tx[i];
+        s.ay[i] = (uint8_t)ty[i];
+      }
+    }
+    s.eaten |= (uint8_t)newly;
+    s.ep_t += 1;
+    team = __fadd_rn(r0, r1);
+    s.ret = __fadd_rn(s.ret, team);
+    return (s.eaten == 7u || (int)s.ep_t == d.episode_len) ? 1 : 0;
+  }
+
+  // Level-scaled one-hot per cell: channel 0 own level, 1 other's level, 2 food level,
+  // 3 = 1 for an empty cell.  One 32-bit word per cell (channel c in byte c).
+  __device__ static void obs(const DevEnv& d, const State& s, int seat, uint8_t* row) {
+    uint32_t* w = reinterpret_cast<uint32_t*>(row);
+    const int cells = d.width * d.height;
+    for (int c = 0; c < cells; ++c) w[c] = 0x01000000u;
+    for (int k = 0; k < d.n_food; ++k)
+      if (!((s.eaten >> k) & 1u)) w[s.fy[k] * d.width + s.fx[k]] = (uint32_t)s.fl[k] << 16;
+    const int o = 1 - seat;
+    w[s.ay[o] * d.width + s.ax[o]] = (uint32_t)s.al[o] << 8;
+    w[s.ay[seat] * d.width + s.ax[seat]] = (uint32_t)s.al[seat];
+  }
+
+  __device__ static uint32_t legal(const State&) { return 0x3Fu; }
+  __device__ static int actor(const State&) { return -1; }
+  __device__ static float ret(const State& s) { return s.ret; }
+};
+
+}  // namespace aht

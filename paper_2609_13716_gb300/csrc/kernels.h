@@ -1,0 +1,118 @@
+// kernels.h -- launch interface between the C-ABI layer (aht_api.cu) and the kernels.
+#pragma once
+#include "aht_common.cuh"
+
+namespace aht {
+
+struct TrajPtrs {
+  uint8_t* obs;
+  uint8_t* actions;
+  uint8_t* tm_actions;
+  float* logp;
+  float* values;
+  float* rewards;
+  uint8_t* dones;
+  float* last_value;
+};
+
+// Common per-launch description of the env batch and the population.
+struct Batch {
+  DevEnv env;
+  MlpDims mlp;
+  const float* weights;  // packed population
+  Key key;
+  uint32_t* status;      // device status word
+};
+
+struct PpoArgs {
+  Batch b;
+  uint32_t* state;       // SoA env state [kWords][n_envs]
+  int64_t n_envs;
+  const int32_t* perm;   // env ids grouped by teammate
+  const int4* tiles;     // (perm offset, count, teammate policy, -)
+  int32_t M;             // rows per tile
+  int32_t ego;
+  uint32_t step0;
+  int32_t T;
+  TrajPtrs traj;
+};
+
+struct GroupArgs {
+  Key key;
+  int64_t n_envs;
+  uint32_t step0;
+  int32_t pool_size;
+  int32_t pool[kMaxPool];
+  int32_t M;
+  int32_t max_tiles;
+  int32_t* perm;
+  int4* tiles;
+  int32_t* teammate;     // optional [n_envs]
+};
+
+struct XpArgs {
+  Batch b;
+  int32_t n_ego, n_tm, P, max_steps;
+  int32_t ego_ids[kMaxXpIds];
+  int32_t tm_ids[kMaxXpIds];
+  int32_t M, tiles_per_pair;
+  uint32_t step0;
+  float* returns;        // [n_pairs * P]
+  int32_t* steps;        // optional
+  uint8_t* actions;      // optional [max_steps][n][2]
+};
+
+struct ForcedArgs {
+  Batch b;
+  uint32_t* state;
+  int64_t n_envs;
+  uint32_t step;
+  const uint8_t* actions;  // [N][2]
+  float* rewards;          // [N][2]
+  float* team;
+  uint8_t* dones;
+  uint8_t* obs;            // [N][2][obs_dim]
+};
+
+struct ResetArgs {
+  Batch b;
+  uint32_t* state;
+  int64_t n_envs;
+  uint32_t step;
+};
+
+struct PolicyArgs {
+  Batch b;
+  int32_t policy;
+  const uint8_t* obs;
+  int64_t n;
+  float* out;              // [n][NA+1]
+  int32_t M;
+};
+
+// Per-env launchers (defined in rollout_<env>.cu).
+#define AHT_DECLARE_ENV_LAUNCHERS(name)                                          \
+  cudaError_t name##_ppo(const PpoArgs&, int grid, size_t smem, cudaStream_t);    \
+  cudaError_t name##_xplay(const XpArgs&, int grid, size_t smem, cudaStream_t);   \
+  cudaError_t name##_forced(const ForcedArgs&, cudaStream_t);                     \
+  cudaError_t name##_reset(const ResetArgs&, cudaStream_t);                       \
+  int name##_state_words();                                                      \
+  int name##_state_bytes();                                                      \
+  cudaError_t name##_set_smem_limit(size_t bytes);
+
+AHT_DECLARE_ENV_LAUNCHERS(lbf)
+AHT_DECLARE_ENV_LAUNCHERS(overcooked)
+AHT_DECLARE_ENV_LAUNCHERS(hanabi)
+
+// misc.cu
+cudaError_t launch_group(const GroupArgs&, cudaStream_t);
+cudaError_t launch_policy(const PolicyArgs&, int grid, size_t smem, cudaStream_t);
+cudaError_t policy_set_smem_limit(size_t bytes);
+size_t group_smem_bytes(int pool_size);
+cudaError_t launch_gae(const float* r, const float* v, const uint8_t* d, const float* v_last,
+                       int64_t n, int32_t T, float gamma, float lambda, float* adv, float* tgt,
+                       cudaStream_t);
+cudaError_t launch_xp_reduce(const float* returns, int64_t n_pairs, int32_t P, float* matrix,
+                             cudaStream_t);
+
+}  // namespace aht

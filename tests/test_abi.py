@@ -1,0 +1,56 @@
+"""The C-ABI library builds for sm_103a, loads, and exports every symbol include/aht.h declares."""
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_symbols():
+    src = open(os.path.join(ROOT, "include", "aht.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(aht_[a-z_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_13716_gb300 import build
+    path = build.build()
+    return path
+
+
+def test_header_declares_the_boundary():
+    syms = declared_symbols()
+    for name in ("aht_create", "aht_reset", "aht_rollout", "aht_xplay_matrix", "aht_gae"):
+        assert name in syms
+
+
+def test_library_exports_every_declared_symbol(lib):
+    out = subprocess.run(["nm", "-D", "--defined-only", lib], capture_output=True, text=True, check=True).stdout
+    exported = set(re.findall(r"\b[TtWw] (aht_\w+)", out))
+    missing = [s for s in declared_symbols() if s not in exported]
+    assert not missing, missing
+
+
+def test_library_loads_and_binding_matches(lib):
+    from paper_2609_13716_gb300 import aht
+    L = aht.load()
+    for s in declared_symbols():
+        assert hasattr(L, s), s
+    assert set(aht.EXPORTED) <= set(declared_symbols())
+    assert L.aht_status_string(1) == b"invalid argument"
+
+
+def test_host_validation_needs_no_gpu(lib):
+    # Argument checks happen before any CUDA call.
+    import ctypes as C
+    from paper_2609_13716_gb300 import aht
+    L = aht.load()
+    bad = aht.EnvDesc(0, 2, 7, 3, 3, 50, 0, 0)   # LBF width 2 is invalid
+    h = C.c_void_p()
+    assert L.aht_create(C.byref(bad), None, 4, 0, None, C.byref(h)) == aht.AHT_EINVAL
+    assert b"width" in L.aht_last_error()
+    assert L.aht_gae(None, None, None, None, 1, 1, 0.9, 0.9, None, None, None) == aht.AHT_EINVAL
+

@@ -1,0 +1,74 @@
+"""GPU policy forward and GAE vs the fp64 oracle."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2609_13716_gb300 import aht
+from paper_2609_13716_gb300 import workloads as W
+
+from gpu_util import GAE_REL, close, make_ctx, np_, oracle_of, require_gpu
+
+pytestmark = pytest.mark.gpu
+
+
+def _obs_samples(wl, n, seed):
+    """Realistic observations (env resets and forced random steps) plus random u8 rows."""
+    d = O.env_desc(*wl.env.astuple())
+    st = O.reset_all(d, seed, n)
+    rng = np.random.default_rng(seed)
+    rows = []
+    for t in range(3):
+        if wl.env.kind == W.HANABI:
+            acts = np.zeros((n, 2), np.uint8)   # play slot 0 is always legal
+        else:
+            acts = rng.integers(0, 6, size=(n, 2)).astype(np.uint8)
+        rc, _, _, _, ob = O.step_forced(d, seed, t, st, acts)
+        rows.append(ob[:, t % 2])
+    obs = np.concatenate(rows)
+    noise = rng.integers(0, 2 if wl.env.kind != W.LBF else 10, size=(n, wl.env.obs_dim)).astype(np.uint8)
+    return np.concatenate([obs, noise])
+
+
+@pytest.mark.parametrize("name,policies", [("lbf7x7_64x50_fp32", [0, 1]),
+                                           ("lbf7x7_ppo_16384x128", [0, 5]),
+                                           ("overcooked5x4_xplay_8x8x64", [3]),
+                                           ("hanabi_xplay_16x16x32", [0, 31])])
+def test_policy_outputs_match_fp64(name, policies):
+    require_gpu()
+    wl = W.WORKLOADS[name]
+    ctx, pop_np = make_ctx(wl, 8)
+    _, pols = oracle_of(wl.env, pop_np)
+    obs = _obs_samples(wl, 300, 7)   # 1200 rows: several tiles and a ragged tail
+    K = wl.env.n_actions
+    for p in policies:
+        out = torch.empty(obs.shape[0], K + 1, device="cuda")
+        aht.aht_policy_forward(ctx, p, torch.from_numpy(obs).cuda(), out)
+        ref = pols.outputs(p, obs)
+        got = np_(out)
+        ok, worst = close(got[:, :K], ref[:, :K])
+        assert ok, f"logits of policy {p}: worst error / bound = {worst:.3g}"
+        if wl.value_head[p]:
+            ok, worst = close(got[:, K], ref[:, K])
+            assert ok, f"values of policy {p}: {worst:.3g}"
+        else:
+            assert (got[:, K] == 0).all()
+
+
+@pytest.mark.parametrize("T,N,p_done", [(128, 5000, 0.02), (1, 1, 0.0), (7, 33, 0.5)])
+def test_gae_kernel(T, N, p_done):
+    require_gpu()
+    rng = np.random.default_rng(T + N)
+    r = rng.standard_normal((T, N)).astype(np.float32)
+    v = rng.standard_normal((T, N)).astype(np.float32)
+    d = (rng.random((T, N)) < p_done).astype(np.uint8)
+    vl = rng.standard_normal(N).astype(np.float32)
+    cu = lambda a: torch.from_numpy(a).cuda()
+    adv = torch.empty(T, N, device="cuda")
+    tgt = torch.empty(T, N, device="cuda")
+    aht.aht_gae(cu(r), cu(v), cu(d), cu(vl), 0.99, 0.95, adv, tgt)
+    torch.cuda.synchronize()
+    a_ref, t_ref = O.gae(r, v, d, vl, 0.99, 0.95)
+    for g, o in ((adv, a_ref), (tgt, t_ref)):
+        ok, worst = close(np_(g), o, GAE_REL)
+        assert ok, worst
