@@ -45,6 +45,10 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-xplay", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
+    # profiling of a smaller case of the same kernel (not a bench line)
+    p.add_argument("--n-envs", type=int, default=None)
+    p.add_argument("--T", type=int, default=None)
+    p.add_argument("--no-e2e", action="store_true")
     return p.parse_args()
 
 
@@ -135,7 +139,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + ",".join(self.FIELDS),
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "20"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.thread = threading.Thread(target=self._read, daemon=True)
             self.thread.start()
@@ -219,7 +223,7 @@ def run_ours(args):
     peak_src = "measured" if peaks else "fallback"
 
     wl = W.WORKLOADS[WORKLOAD]
-    N, T = wl.n_envs, wl.T
+    N, T = args.n_envs or wl.n_envs, args.T or wl.T
     pop_np = W.population(wl)
     pop = [[(torch.from_numpy(Wt).to("cuda", torch.bfloat16), torch.from_numpy(b).to("cuda", torch.bfloat16))
             for Wt, b in p] for p in pop_np]
@@ -249,6 +253,7 @@ def run_ours(args):
         dist.barrier()
     torch.cuda.synchronize()
     with ClockSampler(dev_index) as clocks:
+        time.sleep(0.3)   # let the sampler start before the timed launches
         for k in range(args.steps):
             scrub.fill_(k & 0xFF)
             starts[k].record(stream)
@@ -275,7 +280,7 @@ def run_ours(args):
     d2h = sum(v.numel() * v.element_size() for v in host.values())
     e2e_s, e2e_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e2e_ms = []
-    for k in range(args.steps + 1):
+    for k in range(0 if args.no_e2e else args.steps + 1):
         torch.cuda.synchronize()
         e2e_s.record(stream)
         aht.aht_set_policy(ctx, wl.ego_id, ego_host, 1, aht.AHT_BF16)
@@ -287,7 +292,7 @@ def run_ours(args):
         if k > 0:
             e2e_ms.append(e2e_s.elapsed_time(e2e_e))
     aht.aht_sync(ctx)
-    e2e_ms_max = torch.tensor([sum(e2e_ms) / len(e2e_ms)], device="cuda")
+    e2e_ms_max = torch.tensor([sum(e2e_ms) / max(1, len(e2e_ms))], device="cuda")
     if world > 1:
         dist.all_reduce(e2e_ms_max, op=dist.ReduceOp.MAX)
 
@@ -324,7 +329,8 @@ def run_ours(args):
                          "hbm": {"achieved_gbs": achieved_gbs, "peak_gbs": hbm_peak,
                                  "frac": achieved_gbs / hbm_peak,
                                  "bytes_per_launch": env_steps * bytes_per_env_step}},
-            "e2e": {"value": world * env_steps / (float(e2e_ms_max) * 1e-3), "unit": UNIT,
+            "e2e": None if not e2e_ms else
+                   {"value": world * env_steps / (float(e2e_ms_max) * 1e-3), "unit": UNIT,
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": 3 * args.steps,
             "clocks": clocks.summary(),
