@@ -154,6 +154,29 @@ aht_status aht_xplay_matrix(aht_ctx* ctx, const int32_t* ego_ids, int32_t n_ego,
                             const int32_t* tm_ids, int32_t n_tm, int32_t envs_per_pair,
                             int32_t max_steps, const aht_xplay_out* out);
 
+/* Cross-play matrix that needs no device memory beyond its output (the paper has no
+ * counterpart; this is a deployment convenience).  aht_xplay_matrix keeps the per-env
+ * returns in context scratch sized at aht_create, so its batch is capped by the
+ * context's n_envs; a caller that cannot allocate more device memory after start-up
+ * (a host whose allocator is owned by another framework, or a long-lived PPO context
+ * created with only its training batch) cannot grow that scratch.  This variant keeps
+ * the per-env returns in one file-scope device array of AHT_XPLAY_STATIC_MAX_ENVS
+ * floats (256 KiB) instead, which every GPU that loads the library holds until the
+ * process exits, so any n_ego*n_tm*envs_per_pair up to that maximum works on any
+ * context.  Same semantics, step counter and result as aht_xplay_matrix with only
+ * `matrix` requested (device f32 [n_ego][n_tm]).
+ *   - Allocates nothing and calls no allocating CUDA or library routine.
+ *   - Returns AHT_EINVAL if n_ego*n_tm*envs_per_pair > AHT_XPLAY_STATIC_MAX_ENVS.
+ *   - The first call on each device looks up the array's device address (with that
+ *     device current) and caches it; make that first call before any stream capture.
+ *   - All calls, on every context and stream of a device, share the one array; each
+ *     call writes every entry it reads before reading it, so nothing needs clearing, but
+ *     calls that overlap on the GPU race and must be serialised by the caller. */
+#define AHT_XPLAY_STATIC_MAX_ENVS 65536
+aht_status aht_xplay_matrix_static(aht_ctx* ctx, const int32_t* ego_ids, int32_t n_ego,
+                                   const int32_t* tm_ids, int32_t n_tm, int32_t envs_per_pair,
+                                   int32_t max_steps, float* matrix);
+
 /* Stateless GAE (App. C "PPO ego"), time-major [T][n_envs] device arrays:
  *   delta_t = r_t + gamma (1 - d_t) V_{t+1} - V_t,
  *   A_t = delta_t + gamma lambda (1 - d_t) A_{t+1},  V_T = v_last,  A_T = 0,

@@ -22,7 +22,8 @@ AHT_FP32, AHT_BF16 = 0, 1
 EXPORTED = ["aht_create", "aht_destroy", "aht_reset", "aht_rollout", "aht_xplay_matrix",
             "aht_gae", "aht_step_forced", "aht_policy_forward", "aht_get_state",
             "aht_set_state", "aht_step_counter", "aht_sync", "aht_last_error",
-            "aht_status_string", "aht_set_policy", "aht_set_timing", "aht_get_timing"]
+            "aht_status_string", "aht_set_policy", "aht_set_timing", "aht_get_timing",
+            "aht_xplay_matrix_static"]
 
 
 class AhtError(RuntimeError):
@@ -232,6 +233,21 @@ def aht_xplay_matrix(ctx: Context, ego_ids, tm_ids, envs_per_pair, max_steps, ma
     ea = (C.c_int32 * ne)(*ego_ids)
     ta = (C.c_int32 * nt)(*tm_ids)
     _check(load().aht_xplay_matrix(ctx.handle, ea, ne, ta, nt, P, max_steps, C.byref(out)))
+
+
+def aht_xplay_matrix_static(ctx: Context, ego_ids, tm_ids, envs_per_pair, max_steps, matrix):
+    """aht_xplay_matrix with its per-env return scratch in the library's static device
+    array instead of the context's memory (see include/aht.h)."""
+    L = load()
+    L.aht_xplay_matrix_static.argtypes = [C.c_void_p, C.POINTER(C.c_int32), C.c_int32,
+                                          C.POINTER(C.c_int32), C.c_int32, C.c_int32,
+                                          C.c_int32, C.c_void_p]
+    L.aht_xplay_matrix_static.restype = C.c_int
+    ne, nt = len(ego_ids), len(tm_ids)
+    ea = (C.c_int32 * ne)(*ego_ids)
+    ta = (C.c_int32 * nt)(*tm_ids)
+    _check(L.aht_xplay_matrix_static(ctx.handle, ea, ne, ta, nt, envs_per_pair, max_steps,
+                                     _ptr(matrix, torch.float32, (ne, nt), "matrix")))
 
 
 def aht_gae(rewards, values, dones, v_last, gamma, lam, advantages, targets=None, stream=None):

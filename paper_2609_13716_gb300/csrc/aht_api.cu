@@ -4,6 +4,7 @@
 #include <algorithm>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -484,6 +485,84 @@ aht_status aht_xplay_matrix(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego,
   AHT_CUDA(c->ops.xplay(a, (int)grid, smem, c->stream));
   timer_end(c, tk);
   if (out->matrix) AHT_CUDA(launch_xp_reduce(a.returns, n_pairs, envs_per_pair, out->matrix, c->stream));
+  c->step += max_steps;
+  return AHT_OK;
+}
+
+}  // extern "C"
+
+// ---- cross-play without context scratch ------------------------------------------------
+// The per-env returns that aht_xplay_matrix keeps in context memory sized at aht_create
+// live here instead: one file-scope device array that every GPU loading the library
+// holds until the process exits.  Host code must not pass the symbol itself to a kernel
+// (on the host it names a stand-in, not device memory); it passes the device address
+// that cudaGetSymbolAddress returns for the current device, looked up once per device.
+namespace {
+constexpr int64_t kStaticXpEnvs = AHT_XPLAY_STATIC_MAX_ENVS;
+__device__ __align__(256) float g_static_xp_returns[kStaticXpEnvs];
+constexpr int kMaxDevices = 64;
+std::mutex g_static_mu;
+float* g_static_xp_ptr[kMaxDevices] = {};
+
+aht_status static_xp_returns(int device, float** out) {
+  if (device < 0 || device >= kMaxDevices) return fail(AHT_EINVAL, "device index above 63");
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (!g_static_xp_ptr[device]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_xp_returns);  // device is current
+    if (e != cudaSuccess || !p)
+      return fail(AHT_ECUDA, std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(e));
+    g_static_xp_ptr[device] = static_cast<float*>(p);
+  }
+  *out = g_static_xp_ptr[device];
+  return AHT_OK;
+}
+}  // namespace
+
+extern "C" {
+
+aht_status aht_xplay_matrix_static(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego,
+                                   const int32_t* tm_ids, int32_t n_tm, int32_t envs_per_pair,
+                                   int32_t max_steps, float* matrix) {
+  if (!c || !matrix) return fail(AHT_EINVAL, "ctx or matrix is NULL");
+  if (!ego_ids || !tm_ids || n_ego < 1 || n_tm < 1 || n_ego > kMaxXpIds || n_tm > kMaxXpIds)
+    return fail(AHT_EINVAL, "n_ego and n_tm must be in 1..64");
+  for (int i = 0; i < n_ego; ++i)
+    if (ego_ids[i] < 0 || ego_ids[i] >= c->n_policies) return fail(AHT_EINVAL, "ego id out of range");
+  for (int j = 0; j < n_tm; ++j)
+    if (tm_ids[j] < 0 || tm_ids[j] >= c->n_policies) return fail(AHT_EINVAL, "teammate id out of range");
+  if (envs_per_pair < 1 || envs_per_pair > (1 << 14)) return fail(AHT_EINVAL, "envs_per_pair must be in 1..16384");
+  if (max_steps < 1) return fail(AHT_EINVAL, "max_steps must be >= 1");
+  const int64_t n_pairs = (int64_t)n_ego * n_tm;
+  const int64_t n_total = n_pairs * envs_per_pair;
+  if (n_total > kStaticXpEnvs)
+    return fail(AHT_EINVAL, "n_ego*n_tm*envs_per_pair = " + std::to_string(n_total) +
+                                " exceeds the static scratch of " + std::to_string(kStaticXpEnvs) + " envs");
+  if (c->step + max_steps + 1 > (int64_t)UINT32_MAX) return fail(AHT_EINVAL, "step counter would exceed 2^32");
+  DeviceGuard g(c->device);
+  float* scratch = nullptr;
+  const aht_status ss = static_xp_returns(c->device, &scratch);
+  if (ss != AHT_OK) return ss;
+  const int M = fit_rows(c, std::min(c->ops.max_rows, envs_per_pair));
+  XpArgs a{};
+  a.b = batch_of(c);
+  a.n_ego = n_ego;
+  a.n_tm = n_tm;
+  a.P = envs_per_pair;
+  a.max_steps = max_steps;
+  for (int i = 0; i < n_ego; ++i) a.ego_ids[i] = ego_ids[i];
+  for (int j = 0; j < n_tm; ++j) a.tm_ids[j] = tm_ids[j];
+  a.M = M;
+  a.tiles_per_pair = (envs_per_pair + M - 1) / M;
+  a.step0 = (uint32_t)c->step;
+  a.returns = scratch;  // every entry the reduction reads is written first by this call
+  a.steps = nullptr;
+  a.actions = nullptr;
+  const size_t smem = smem_layout(M, c->mlp, c->ops.bytes()).total;
+  const int64_t grid = n_pairs * a.tiles_per_pair;
+  if (grid > INT32_MAX) return fail(AHT_EINVAL, "too many tiles");
+  AHT_CUDA(c->ops.xplay(a, (int)grid, smem, c->stream));
+  AHT_CUDA(launch_xp_reduce(scratch, n_pairs, envs_per_pair, matrix, c->stream));
   c->step += max_steps;
   return AHT_OK;
 }
