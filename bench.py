@@ -306,7 +306,7 @@ def run_ours(args):
     kern_ms = kernel_ms / max(1, kernel_launches)
     achieved_tflops = flops_launch / (kern_ms * 1e-3) / 1e12
     achieved_gbs = env_steps * bytes_per_env_step / (kern_ms * 1e-3) / 1e9
-    traffic = recorded_traffic("ppo_kernel")
+    traffic = recorded_traffic("ppo_tc_kernel")
 
     line = None
     if rank == 0:
@@ -315,7 +315,7 @@ def run_ours(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_max,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "f32", "data": "synthetic (random-init N(0,0.1) bf16 weights, seeded envs)",
+            "dtype": "bf16", "data": "synthetic (random-init N(0,0.1) bf16 weights, seeded envs)",
             "config": {"workload": WORKLOAD, "n_envs": N, "T": T, "pool": len(wl.pool),
                        "episode_len": wl.env.episode_len, "weights": "bf16",
                        "l2": "scrubbed: 256 MB write between timed steps (outside the events); "
@@ -323,7 +323,7 @@ def run_ours(args):
                        "parallelism": f"{world} independent replicas" if world > 1 else "1 GPU"},
             "roofline": {"bound": "tensor", "achieved": achieved_tflops, "peak": bf16_peak,
                          "unit": "TFLOP/s", "frac": achieved_tflops / bf16_peak,
-                         "traffic": traffic, "kernel": "ppo_kernel<EnvLbf>",
+                         "traffic": traffic, "kernel": "ppo_tc_kernel<EnvLbf>",
                          "kernel_ms": kern_ms, "flops_per_launch": flops_launch,
                          "peak_source": f"{peak_src} bf16 burst",
                          "hbm": {"achieved_gbs": achieved_gbs, "peak_gbs": hbm_peak,

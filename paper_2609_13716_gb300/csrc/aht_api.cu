@@ -10,6 +10,7 @@
 
 #include "kernels.h"
 #include "rollout_impl.cuh"
+#include "tc_common.cuh"
 
 using namespace aht;
 
@@ -96,6 +97,12 @@ struct aht_ctx {
   float* xp_returns = nullptr;
   float* last_value = nullptr;
   uint32_t* status = nullptr;
+  // tensor-core path (bf16 LBF populations that fit shared and tensor memory)
+  bool tc = false;
+  TcDims tcd{};
+  uint8_t* tcw = nullptr;
+  size_t tc_smem = 0;
+  uint8_t* tc_staging = nullptr;
   // pinned host staging for aht_set_policy, and the event pool of the kernel timer
   float* staging = nullptr;
   cudaEvent_t upload_done = nullptr;
@@ -222,6 +229,80 @@ aht_status pack_policy(const MlpDims& m, const void* const* W, const void* const
   return AHT_OK;
 }
 
+// Tensor-core block layout of one policy (see TcDims): bf16 canonical W1 [H0][KP],
+// W2 [H1][H0], W3 [N3][H1], then fp32 b1, b2, b3.
+TcDims make_tc_dims(const MlpDims& m) {
+  TcDims t{};
+  t.KP = m.KP;
+  t.H0 = m.H0;
+  t.H1 = m.H1;
+  t.N3 = 16;
+  uint32_t o = 0;
+  t.oW1 = o; o += (uint32_t)(m.H0 * m.KP * 2);
+  t.oW2 = o; o += (uint32_t)(m.H1 * m.H0 * 2);
+  t.oW3 = o; o += (uint32_t)(t.N3 * m.H1 * 2);
+  t.ob1 = o; o += (uint32_t)(m.H0 * 4);
+  t.ob2 = o; o += (uint32_t)(m.H1 * 4);
+  t.ob3 = o; o += (uint32_t)(t.N3 * 4);
+  t.pol_bytes = (uint32_t)align_up(o, 16);
+  return t;
+}
+
+// Shared memory of the tensor-core kernel: both policies' blocks, the u8 observation
+// tile [128][KP], 128 env states, 128 env ids.
+size_t tc_smem_bytes(const TcDims& t, int state_bytes) {
+  return 2 * (size_t)t.pol_bytes + 128 * (size_t)t.KP + align_up(128 * state_bytes, 16) + 512;
+}
+
+// The tensor-core path applies to bf16 populations of LBF whose padded observation
+// (KP/2 columns) and hidden layers (<= 128 columns each, multiples of 64) fit the
+// 256 tensor-memory columns each agent uses, and whose two policy blocks fit shared memory.
+bool tc_eligible(const aht_ctx* c, int dtype) {
+  const MlpDims& m = c->mlp;
+  if (dtype != AHT_BF16 || c->env.kind != AHT_LBF) return false;
+  if (m.KP > 256 || m.H0 > 128 || m.H1 > 128 || m.H0 % 64 || m.H1 % 64 || m.NA + 1 > 16) return false;
+  return tc_smem_bytes(make_tc_dims(m), c->ops.bytes()) <= c->smem_optin;
+}
+
+bool read_host(const void* p, size_t bytes, std::vector<uint8_t>& tmp, const void** out) {
+  cudaPointerAttributes at{};
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) cudaGetLastError();
+  if (at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged) {
+    tmp.resize(bytes);
+    if (cudaMemcpy(tmp.data(), p, bytes, cudaMemcpyDeviceToHost) != cudaSuccess) return false;
+    *out = tmp.data();
+  } else {
+    *out = p;
+  }
+  return true;
+}
+
+// Packs one bf16 policy into its tensor-core block (dst: t.pol_bytes bytes).
+aht_status pack_policy_tc(const MlpDims& m, const TcDims& t, const void* const* W,
+                          const void* const* b, int vh, uint8_t* dst) {
+  std::fill(dst, dst + t.pol_bytes, (uint8_t)0);
+  const int ins[3] = {m.K, m.H0, m.H1};
+  const int kpad[3] = {t.KP, m.H0, m.H1};
+  const int outs[3] = {m.H0, m.H1, m.NA + vh};
+  const uint32_t oW[3] = {t.oW1, t.oW2, t.oW3}, ob[3] = {t.ob1, t.ob2, t.ob3};
+  std::vector<uint8_t> tmp;
+  for (int l = 0; l < 3; ++l) {
+    const void* src = nullptr;
+    if (!W[l] || !b[l]) return fail(AHT_EINVAL, "NULL weight pointer");
+    if (!read_host(W[l], (size_t)outs[l] * ins[l] * 2, tmp, &src)) return fail(AHT_ECUDA, "copying weights failed");
+    const uint16_t* w = static_cast<const uint16_t*>(src);
+    for (int n = 0; n < outs[l]; ++n)
+      for (int k = 0; k < ins[l]; ++k)
+        std::memcpy(dst + oW[l] + tc::canon_offset(n, k, kpad[l]), &w[(int64_t)n * ins[l] + k], 2);
+    if (!read_host(b[l], (size_t)outs[l] * 2, tmp, &src)) return fail(AHT_ECUDA, "copying biases failed");
+    for (int n = 0; n < outs[l]; ++n) {
+      const float f = to_f32(src, n, AHT_BF16);
+      std::memcpy(dst + ob[l] + 4 * n, &f, 4);
+    }
+  }
+  return AHT_OK;
+}
+
 // Kernel timer: events around the main kernel of a call (see aht_set_timing).
 void timer_fold(aht_ctx* c) {
   for (int i = 0; i < c->n_pending; ++i) {
@@ -284,6 +365,8 @@ void aht_destroy(aht_ctx* c) {
   cudaFree(c->last_value);
   cudaFree(c->status);
   if (c->staging) cudaFreeHost(c->staging);
+  if (c->tc_staging) cudaFreeHost(c->tc_staging);
+  cudaFree(c->tcw);
   if (c->upload_done) cudaEventDestroy(c->upload_done);
   for (auto& e : c->ev)
     if (e) cudaEventDestroy(e);
@@ -365,6 +448,29 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
     return bail(AHT_ECUDA, "cudaEventCreate failed");
   for (auto& e : c->ev)
     if (cudaEventCreate(&e) != cudaSuccess) return bail(AHT_ECUDA, "cudaEventCreate failed");
+  if (tc_eligible(c, pop->weight_dtype)) {
+    c->tcd = make_tc_dims(m);
+    c->tc_smem = tc_smem_bytes(c->tcd, c->ops.bytes());
+    std::vector<uint8_t> blocks((size_t)c->tcd.pol_bytes * pop->n_policies);
+    for (int p = 0; p < pop->n_policies; ++p) {
+      const int vh = pop->has_value_head ? pop->has_value_head[p] : 0;
+      aht_status ps = pack_policy_tc(m, c->tcd, pop->W + 3 * p, pop->b + 3 * p, vh,
+                                     blocks.data() + (size_t)p * c->tcd.pol_bytes);
+      if (ps != AHT_OK) {
+        std::string msg = g_err;
+        return bail(ps, msg);
+      }
+    }
+    if (cudaMalloc((void**)&c->tcw, blocks.size()) != cudaSuccess) {
+      cudaGetLastError();
+      return bail(AHT_ENOMEM, "cudaMalloc of the tensor-core population failed");
+    }
+    if (cudaMemcpy(c->tcw, blocks.data(), blocks.size(), cudaMemcpyHostToDevice) != cudaSuccess)
+      return bail(AHT_ECUDA, "uploading the tensor-core population failed");
+    if (cudaMallocHost((void**)&c->tc_staging, c->tcd.pol_bytes) != cudaSuccess)
+      return bail(AHT_ENOMEM, "pinned staging allocation failed");
+    c->tc = true;
+  }
   *out = c;
   aht_status r = aht_reset(c, seed);
   if (r != AHT_OK) {
@@ -406,7 +512,7 @@ aht_status aht_rollout(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t 
   if (out->gamma < 0.f || out->gamma > 1.f || out->lambda < 0.f || out->lambda > 1.f)
     return fail(AHT_EINVAL, "gamma and lambda must be in [0, 1]");
   DeviceGuard g(c->device);
-  const int M = fit_rows(c, 128);
+  const int M = c->tc ? 128 : fit_rows(c, 128);
 
   GroupArgs ga{};
   ga.key = batch_of(c).key;
@@ -434,10 +540,28 @@ aht_status aht_rollout(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t 
   a.traj = TrajPtrs{out->obs, out->actions, out->tm_actions, out->logp, out->values,
                     out->rewards, out->dones,
                     out->last_value ? out->last_value : (out->advantages ? c->last_value : nullptr)};
-  const size_t smem = smem_layout(M, c->mlp, c->ops.bytes()).total;
-  const int tk = timer_begin(c);
-  AHT_CUDA(c->ops.ppo(a, ga.max_tiles, smem, c->stream));
-  timer_end(c, tk);
+  if (c->tc) {
+    PpoTcArgs ta{};
+    ta.b = a.b;
+    ta.tc = c->tcd;
+    ta.tcw = c->tcw;
+    ta.state = c->state;
+    ta.n_envs = c->n_envs;
+    ta.perm = c->perm;
+    ta.tiles = c->tiles;
+    ta.ego = ego_id;
+    ta.step0 = a.step0;
+    ta.T = T;
+    ta.traj = a.traj;
+    const int tk = timer_begin(c);
+    AHT_CUDA(lbf_ppo_tc(ta, ga.max_tiles, c->tc_smem, c->stream));
+    timer_end(c, tk);
+  } else {
+    const size_t smem = smem_layout(M, c->mlp, c->ops.bytes()).total;
+    const int tk = timer_begin(c);
+    AHT_CUDA(c->ops.ppo(a, ga.max_tiles, smem, c->stream));
+    timer_end(c, tk);
+  }
   if (out->advantages)
     AHT_CUDA(launch_gae(out->rewards, out->values, out->dones, a.traj.last_value, c->n_envs, T,
                         out->gamma, out->lambda, out->advantages, out->targets, c->stream));
@@ -648,6 +772,13 @@ aht_status aht_set_policy(aht_ctx* c, int32_t policy, const void* const* W, cons
   if (ps != AHT_OK) return ps;
   AHT_CUDA(cudaMemcpyAsync(c->weights + (int64_t)policy * c->mlp.stride, c->staging,
                            (size_t)c->mlp.stride * 4, cudaMemcpyHostToDevice, c->stream));
+  if (c->tc) {
+    if (weight_dtype != AHT_BF16) return fail(AHT_EINVAL, "this context's population is bf16");
+    ps = pack_policy_tc(c->mlp, c->tcd, W, b, has_value_head, c->tc_staging);
+    if (ps != AHT_OK) return ps;
+    AHT_CUDA(cudaMemcpyAsync(c->tcw + (int64_t)policy * c->tcd.pol_bytes, c->tc_staging,
+                             c->tcd.pol_bytes, cudaMemcpyHostToDevice, c->stream));
+  }
   AHT_CUDA(cudaEventRecord(c->upload_done, c->stream));
   return AHT_OK;
 }

@@ -18,6 +18,7 @@ enum : uint32_t {
   kStatusIllegalAction = 1u,
   kStatusActorMismatch = 2u,
   kStatusBadPolicy = 4u,
+  kStatusTimeout = 8u,   // a bounded device wait gave up
 };
 
 // Philox streams (counter word 2).

@@ -37,6 +37,28 @@ struct PpoArgs {
   TrajPtrs traj;
 };
 
+// Per-policy block of the tensor-core path: bf16 weights in the canonical K-major
+// layout (see tc_common.cuh) and fp32 biases; byte offsets within the block.
+struct TcDims {
+  int32_t KP, H0, H1, N3;  // padded obs dim, hidden sizes, padded outputs (16)
+  uint32_t oW1, oW2, oW3, ob1, ob2, ob3;
+  uint32_t pol_bytes;
+};
+
+struct PpoTcArgs {
+  Batch b;
+  TcDims tc;
+  const uint8_t* tcw;    // [n_policies][pol_bytes]
+  uint32_t* state;
+  int64_t n_envs;
+  const int32_t* perm;
+  const int4* tiles;     // tiles of up to 128 envs
+  int32_t ego;
+  uint32_t step0;
+  int32_t T;
+  TrajPtrs traj;
+};
+
 struct GroupArgs {
   Key key;
   int64_t n_envs;
@@ -103,6 +125,10 @@ struct PolicyArgs {
 AHT_DECLARE_ENV_LAUNCHERS(lbf)
 AHT_DECLARE_ENV_LAUNCHERS(overcooked)
 AHT_DECLARE_ENV_LAUNCHERS(hanabi)
+
+// Tensor-core PPO rollout (rollout_lbf.cu): LBF grids whose padded observation fits
+// 256 bf16 columns of tensor memory.
+cudaError_t lbf_ppo_tc(const PpoTcArgs&, int grid, size_t smem, cudaStream_t);
 
 // misc.cu
 cudaError_t launch_group(const GroupArgs&, cudaStream_t);

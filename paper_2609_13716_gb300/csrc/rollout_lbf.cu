@@ -1,7 +1,12 @@
-// rollout_lbf.cu -- kernel instantiations for the lbf rules.
+// rollout_lbf.cu -- kernel instantiations for the lbf rules (CUDA-core and tensor-core).
 #include "env_lbf.cuh"
 #include "rollout_impl.cuh"
+#include "rollout_tc.cuh"
 
 namespace aht {
 AHT_DEFINE_ENV_LAUNCHERS(lbf, EnvLbf)
+
+cudaError_t lbf_ppo_tc(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
+  return LaunchTc<EnvLbf>::ppo(a, grid, smem, s);
+}
 }  // namespace aht
