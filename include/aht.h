@@ -224,6 +224,12 @@ aht_status aht_step_forced(aht_ctx* ctx, const uint8_t* actions, const aht_step_
 aht_status aht_policy_forward(aht_ctx* ctx, int32_t policy, const uint8_t* obs, int64_t n,
                               float* out);
 
+/* The tanh of the tensor-core epilogue, elementwise: y[i] = tanh(x[i]) for device f32
+ * arrays of n elements (computed as sign(x)(1 - e)/(1 + e), e = exp(-2|x|), with one
+ * hardware exp2 and a Newton-Raphson reciprocal; absolute error ~1e-7).  Stateless;
+ * enqueued on cuda_stream. */
+aht_status aht_debug_tanh(const float* x, float* y, int64_t n, void* cuda_stream);
+
 /* Checkpoint of the PPO env state, the seed and the step counter into a host buffer.
  * Call with buf == NULL to get the size in *bytes.  Resuming from it is bit-exact:
  * every draw is a function of (seed, env, step, stream). */

@@ -23,7 +23,7 @@ EXPORTED = ["aht_create", "aht_destroy", "aht_reset", "aht_rollout", "aht_xplay_
             "aht_gae", "aht_step_forced", "aht_policy_forward", "aht_get_state",
             "aht_set_state", "aht_step_counter", "aht_sync", "aht_last_error",
             "aht_status_string", "aht_set_policy", "aht_set_timing", "aht_get_timing",
-            "aht_xplay_matrix_static"]
+            "aht_xplay_matrix_static", "aht_debug_tanh"]
 
 
 class AhtError(RuntimeError):
@@ -248,6 +248,16 @@ def aht_xplay_matrix_static(ctx: Context, ego_ids, tm_ids, envs_per_pair, max_st
     ta = (C.c_int32 * nt)(*tm_ids)
     _check(L.aht_xplay_matrix_static(ctx.handle, ea, ne, ta, nt, envs_per_pair, max_steps,
                                      _ptr(matrix, torch.float32, (ne, nt), "matrix")))
+
+
+def aht_debug_tanh(x, y, stream=None):
+    """The tensor-core epilogue's tanh applied elementwise (test hook)."""
+    L = load()
+    L.aht_debug_tanh.argtypes = [C.c_void_p, C.c_void_p, C.c_int64, C.c_void_p]
+    L.aht_debug_tanh.restype = C.c_int
+    n = x.numel()
+    _check(L.aht_debug_tanh(_ptr(x, torch.float32, None, "x"), _ptr(y, torch.float32, (n,), "y"),
+                            n, _stream(stream)))
 
 
 def aht_gae(rewards, values, dones, v_last, gamma, lam, advantages, targets=None, stream=None):

@@ -229,29 +229,28 @@ aht_status pack_policy(const MlpDims& m, const void* const* W, const void* const
   return AHT_OK;
 }
 
-// Tensor-core block layout of one policy (see TcDims): bf16 canonical W1 [H0][KP],
-// W2 [H1][H0], W3 [N3][H1], then fp32 b1, b2, b3.
+// Tensor-core block layout of one policy (see TcDims).
 TcDims make_tc_dims(const MlpDims& m) {
   TcDims t{};
-  t.KP = m.KP;
+  t.KP = (int)align_up(m.K + 1, 16);
   t.H0 = m.H0;
   t.H1 = m.H1;
-  t.N3 = 16;
   uint32_t o = 0;
-  t.oW1 = o; o += (uint32_t)(m.H0 * m.KP * 2);
+  t.oW1 = o; o += (uint32_t)(m.H0 * t.KP * 2);
   t.oW2 = o; o += (uint32_t)(m.H1 * m.H0 * 2);
-  t.oW3 = o; o += (uint32_t)(t.N3 * m.H1 * 2);
-  t.ob1 = o; o += (uint32_t)(m.H0 * 4);
+  t.oW3 = o; o += (uint32_t)(m.H1 * 8 * 4);
   t.ob2 = o; o += (uint32_t)(m.H1 * 4);
-  t.ob3 = o; o += (uint32_t)(t.N3 * 4);
+  t.ob3 = o; o += 8 * 4;
   t.pol_bytes = (uint32_t)align_up(o, 16);
   return t;
 }
 
 // Shared memory of the tensor-core kernel: both policies' blocks, the u8 observation
-// tile [128][KP], 128 env states, 128 env ids.
+// tile [128][KP], 128 env states, 128 env ids, 128 teammate actions and the output
+// layer's partial sums [2 agents][128][8] fp32.
 size_t tc_smem_bytes(const TcDims& t, int state_bytes) {
-  return 2 * (size_t)t.pol_bytes + 128 * (size_t)t.KP + align_up(128 * state_bytes, 16) + 512;
+  return 2 * (size_t)t.pol_bytes + 128 * (size_t)t.KP + align_up(128 * state_bytes, 16) + 512 + 128 +
+         2 * 128 * 8 * 4;
 }
 
 // The tensor-core path applies to bf16 populations of LBF whose padded observation
@@ -260,8 +259,9 @@ size_t tc_smem_bytes(const TcDims& t, int state_bytes) {
 bool tc_eligible(const aht_ctx* c, int dtype) {
   const MlpDims& m = c->mlp;
   if (dtype != AHT_BF16 || c->env.kind != AHT_LBF) return false;
-  if (m.KP > 256 || m.H0 > 128 || m.H1 > 128 || m.H0 % 64 || m.H1 % 64 || m.NA + 1 > 16) return false;
-  return tc_smem_bytes(make_tc_dims(m), c->ops.bytes()) <= c->smem_optin;
+  const TcDims t = make_tc_dims(m);
+  if (t.KP > 256 || m.H0 > 128 || m.H1 > 128 || m.H0 % 64 || m.H1 % 64 || m.NA + 1 > 8) return false;
+  return tc_smem_bytes(t, c->ops.bytes()) <= c->smem_optin;
 }
 
 bool read_host(const void* p, size_t bytes, std::vector<uint8_t>& tmp, const void** out) {
@@ -282,9 +282,7 @@ aht_status pack_policy_tc(const MlpDims& m, const TcDims& t, const void* const* 
                           const void* const* b, int vh, uint8_t* dst) {
   std::fill(dst, dst + t.pol_bytes, (uint8_t)0);
   const int ins[3] = {m.K, m.H0, m.H1};
-  const int kpad[3] = {t.KP, m.H0, m.H1};
   const int outs[3] = {m.H0, m.H1, m.NA + vh};
-  const uint32_t oW[3] = {t.oW1, t.oW2, t.oW3}, ob[3] = {t.ob1, t.ob2, t.ob3};
   std::vector<uint8_t> tmp;
   for (int l = 0; l < 3; ++l) {
     const void* src = nullptr;
@@ -292,12 +290,23 @@ aht_status pack_policy_tc(const MlpDims& m, const TcDims& t, const void* const* 
     if (!read_host(W[l], (size_t)outs[l] * ins[l] * 2, tmp, &src)) return fail(AHT_ECUDA, "copying weights failed");
     const uint16_t* w = static_cast<const uint16_t*>(src);
     for (int n = 0; n < outs[l]; ++n)
-      for (int k = 0; k < ins[l]; ++k)
-        std::memcpy(dst + oW[l] + tc::canon_offset(n, k, kpad[l]), &w[(int64_t)n * ins[l] + k], 2);
+      for (int k = 0; k < ins[l]; ++k) {
+        const int64_t i = (int64_t)n * ins[l] + k;
+        if (l == 0) std::memcpy(dst + t.oW1 + tc::canon_offset(n, k, t.KP), &w[i], 2);
+        if (l == 1) std::memcpy(dst + t.oW2 + tc::canon_offset(n, k, m.H0), &w[i], 2);
+        if (l == 2) {
+          const float f = to_f32(src, i, AHT_BF16);
+          std::memcpy(dst + t.oW3 + 4 * (k * 8 + n), &f, 4);
+        }
+      }
     if (!read_host(b[l], (size_t)outs[l] * 2, tmp, &src)) return fail(AHT_ECUDA, "copying biases failed");
+    const uint16_t* bb = static_cast<const uint16_t*>(src);
     for (int n = 0; n < outs[l]; ++n) {
       const float f = to_f32(src, n, AHT_BF16);
-      std::memcpy(dst + ob[l] + 4 * n, &f, 4);
+      if (l == 0)  // b1 = weight of the constant-1 input at K index obs_dim
+        std::memcpy(dst + t.oW1 + tc::canon_offset(n, m.K, t.KP), &bb[n], 2);
+      if (l == 1) std::memcpy(dst + t.ob2 + 4 * n, &f, 4);
+      if (l == 2) std::memcpy(dst + t.ob3 + 4 * n, &f, 4);
     }
   }
   return AHT_OK;
@@ -699,6 +708,12 @@ aht_status aht_gae(const float* r, const float* v, const uint8_t* d, const float
   if (gamma < 0.f || gamma > 1.f || lambda < 0.f || lambda > 1.f)
     return fail(AHT_EINVAL, "gamma and lambda must be in [0, 1]");
   AHT_CUDA(launch_gae(r, v, d, v_last, n_envs, T, gamma, lambda, adv, tgt, (cudaStream_t)cuda_stream));
+  return AHT_OK;
+}
+
+aht_status aht_debug_tanh(const float* x, float* y, int64_t n, void* cuda_stream) {
+  if (!x || !y || n < 1) return fail(AHT_EINVAL, "NULL array or n < 1");
+  AHT_CUDA(launch_tanh_probe(x, y, n, (cudaStream_t)cuda_stream));
   return AHT_OK;
 }
 

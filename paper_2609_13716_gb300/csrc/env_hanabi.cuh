@@ -11,6 +11,7 @@ namespace aht {
 
 struct EnvHanabi {
   static constexpr bool kTurnBased = true;
+  static constexpr int kNumActions = 20;
   static constexpr int kTurnCap = 100;
   struct State {
     uint8_t deck[52];

@@ -12,6 +12,7 @@ namespace aht {
 
 struct EnvLbf {
   static constexpr bool kTurnBased = false;
+  static constexpr int kNumActions = 6;
   struct State {
     uint8_t ax[2], ay[2];
     uint8_t al[2], F, eaten;  // eaten: bit k set when food k is gone (absent foods too)
@@ -128,6 +129,21 @@ struct EnvLbf {
     const int o = 1 - seat;
     w[s.ay[o] * d.width + s.ax[o]] = (uint32_t)s.al[o] << 8;
     w[s.ay[seat] * d.width + s.ax[seat]] = (uint32_t)s.al[seat];
+  }
+
+  // Words [w0, w1) of the same row (w1 <= cells): one cell per word.
+  __device__ static void obs_words(const DevEnv& d, const State& s, int seat, uint32_t* w, int w0,
+                                   int w1) {
+    for (int c = w0; c < w1; ++c) w[c] = 0x01000000u;
+    auto put = [&](int x, int y, uint32_t v) {
+      const int c = y * d.width + x;
+      if (c >= w0 && c < w1) w[c] = v;
+    };
+    for (int k = 0; k < d.n_food; ++k)
+      if (!((s.eaten >> k) & 1u)) put(s.fx[k], s.fy[k], (uint32_t)s.fl[k] << 16);
+    const int o = 1 - seat;
+    put(s.ax[o], s.ay[o], (uint32_t)s.al[o] << 8);
+    put(s.ax[seat], s.ay[seat], (uint32_t)s.al[seat]);
   }
 
   __device__ static uint32_t legal(const State&) { return 0x3Fu; }

@@ -17,6 +17,7 @@ __constant__ uint8_t kKitchenCell[20] = {1, 2, 1, 3, 1,   //
 
 struct EnvOvercooked {
   static constexpr bool kTurnBased = false;
+  static constexpr int kNumActions = 6;
   enum : uint8_t { kNone = 0, kOnion = 1, kDish = 2, kSoup = 3 };
   struct State {
     uint8_t ax[2], ay[2];

@@ -37,11 +37,16 @@ struct PpoArgs {
   TrajPtrs traj;
 };
 
-// Per-policy block of the tensor-core path: bf16 weights in the canonical K-major
-// layout (see tc_common.cuh) and fp32 biases; byte offsets within the block.
+// Per-policy block of the tensor-core path (byte offsets within the block):
+//   W1 [H0][KP] bf16, canonical K-major (see tc_common.cuh); column obs_dim holds b1
+//      (the observation tile carries a constant 1 there),
+//   W2 [H1][H0] bf16, canonical K-major,
+//   W3 fp32 [H1][8], transposed: row k holds W3[0..7][k] (outputs past n_actions, and the
+//      value row when absent, are zero),
+//   b2 fp32 [H1], b3 fp32 [8].
 struct TcDims {
-  int32_t KP, H0, H1, N3;  // padded obs dim, hidden sizes, padded outputs (16)
-  uint32_t oW1, oW2, oW3, ob1, ob2, ob3;
+  int32_t KP, H0, H1;      // padded obs dim (> obs_dim), hidden sizes
+  uint32_t oW1, oW2, oW3, ob2, ob3;
   uint32_t pol_bytes;
 };
 
@@ -134,6 +139,7 @@ cudaError_t lbf_ppo_tc(const PpoTcArgs&, int grid, size_t smem, cudaStream_t);
 cudaError_t launch_group(const GroupArgs&, cudaStream_t);
 cudaError_t launch_policy(const PolicyArgs&, int grid, size_t smem, cudaStream_t);
 cudaError_t policy_set_smem_limit(size_t bytes);
+cudaError_t launch_tanh_probe(const float* x, float* y, int64_t n, cudaStream_t);
 size_t group_smem_bytes(int pool_size);
 cudaError_t launch_gae(const float* r, const float* v, const uint8_t* d, const float* v_last,
                        int64_t n, int32_t T, float gamma, float lambda, float* adv, float* tgt,

@@ -3,6 +3,7 @@
 #include "kernels.h"
 #include "mlp_simt.cuh"
 #include "rollout_impl.cuh"
+#include "tc_common.cuh"
 
 namespace aht {
 
@@ -160,6 +161,17 @@ cudaError_t policy_set_smem_limit(size_t bytes) {
 
 cudaError_t launch_policy(const PolicyArgs& a, int grid, size_t smem, cudaStream_t s) {
   policy_kernel<<<grid, kThreads, smem, s>>>(a);
+  return cudaGetLastError();
+}
+
+// ---- the tensor-core epilogue's tanh, standalone (test hook) ---------------------------
+__global__ void tanh_probe_kernel(const float* __restrict__ x, float* __restrict__ y, int64_t n) {
+  const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (i < n) y[i] = tc::tanh_ex2(x[i]);
+}
+
+cudaError_t launch_tanh_probe(const float* x, float* y, int64_t n, cudaStream_t s) {
+  tanh_probe_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(x, y, n);
   return cudaGetLastError();
 }
 

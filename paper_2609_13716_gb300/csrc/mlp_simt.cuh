@@ -106,4 +106,36 @@ __device__ __forceinline__ int sample_row(const float* z, int K, uint32_t legal,
   return a;
 }
 
+// The same sample for a compile-time action count, all in registers.
+template <int K>
+__device__ __forceinline__ int sample_k(const float (&z)[16], uint32_t legal, float u, float& logp) {
+  float m = -INFINITY;
+#pragma unroll
+  for (int k = 0; k < K; ++k)
+    if ((legal >> k) & 1u) m = fmaxf(m, z[k]);
+  float S[K];
+  float run = 0.0f;
+#pragma unroll
+  for (int k = 0; k < K; ++k) {
+    if ((legal >> k) & 1u) run = __fadd_rn(run, expf(z[k] - m));
+    S[k] = run;
+  }
+  const float target = u * run;
+  int a = -1;
+#pragma unroll
+  for (int k = K - 1; k >= 0; --k)
+    if (target < S[k]) a = k;
+  if (a < 0) {
+#pragma unroll
+    for (int k = 0; k < K; ++k)
+      if ((legal >> k) & 1u) a = k;
+  }
+  float za = z[0];
+#pragma unroll
+  for (int k = 1; k < K; ++k)
+    if (a == k) za = z[k];
+  logp = za - m - logf(run);
+  return a;
+}
+
 }  // namespace aht

@@ -1,22 +1,30 @@
 // rollout_tc.cuh -- fused PPO rollout with the policy MLPs on tcgen05 tensor cores.
 //
-// One CTA (256 threads) owns a tile of up to 128 envs that share one teammate policy,
-// for all T steps.  Per step and agent (ego = seat 0, teammate = seat 1):
-//   obs (u8, shared memory) -> A operand in tensor memory (bf16, exact for small ints)
-//   L1: D = X W1^T                      (M = 128 envs, N = hidden0, K = obs_dim padded)
-//   epilogue: h = tanh(D + b1) split as h = hi + lo (two bf16) back into tensor memory
-//   L2: D = hi W2^T + lo W2^T           (the split keeps ~2^-17 relative precision)
-//   epilogue as above -> L3: z = hi W3^T + lo W3^T (logits, + value row for the ego)
-//   sampling, env step and the trajectory write happen in the thread that owns the env.
-// Weights (bf16, canonical K-major layout) are copied once per CTA into shared memory
-// with bulk (TMA) copies; biases stay fp32.  Thread 0 issues all MMAs; the ego and
-// teammate chains are interleaved so one agent's tensor-core work overlaps the other
-// agent's CUDA-core epilogue.  Every mbarrier wait is bounded: on expiry the CTA
-// records kStatusTimeout, drains its own MMAs (bounded), frees tensor memory and exits.
+// One CTA owns a tile of up to 128 envs that share one teammate policy, for all T steps.
+// Per step and agent (ego = seat 0, teammate = seat 1):
+//   obs (u8, shared memory, a constant 1 after the last feature) -> A operand in tensor
+//       memory as bf16 (exact: small integers)
+//   L1 (tensor cores): D = [o 1] [W1 b1]^T      (M = 128 envs, N = hidden0, K = KP)
+//   epilogue 1: h1 = tanh(D) split h1 = hi + lo (two bf16) into tensor memory, and b2
+//       written into the accumulator columns
+//   L2 (tensor cores): D = b2 + hi W2^T + lo W2^T  (the split keeps ~2^-17 relative
+//       precision of h1 with bf16 operands and fp32 accumulate)
+//   epilogue 2 (CUDA cores): h2 = tanh(D) in fp32 and z = W3 h2 + b3 directly (a handful
+//       of outputs: an N = 16 tensor-core instruction would cost as much as an N = 128 one)
+//   sampling (ego in warps 0-3, teammate in warps 4-7), env step, trajectory write.
+//
+// Warp roles: warps 0-7 ("compute", 256 threads) build observations, run the epilogues
+// (thread r and r + 128 own env row r, tensor-memory lane r; the halves split the
+// columns), sample and step the envs; warp 8 issues every MMA.  They meet only through
+// mbarriers: operand-ready (256 arrivals from the compute threads) and accumulator-ready
+// (a tcgen05.commit).  Each of these barriers completes once per step, so its phase
+// parity is the step's parity.  Compute warps synchronise among themselves with a named
+// barrier that also ORs an error flag.  Weights are bulk-copied (TMA) into shared memory
+// once per CTA.  Every wait is bounded: on expiry the CTA records kStatusTimeout, stops,
+// drains its own MMAs (bounded), frees tensor memory and exits.
 //
 // Tensor memory (512 columns): agent a uses columns [256a, 256a + 128) for its A operand
-// (X, then hi|lo of h1, then hi|lo of h2) and [256a + 128, 256a + 256) for its fp32
-// accumulator.
+// (X, then hi|lo of h1) and [256a + 128, 256a + 256) for its fp32 accumulator.
 #pragma once
 #include "kernels.h"
 #include "rollout_impl.cuh"
@@ -24,34 +32,58 @@
 
 namespace aht {
 
+constexpr int kTcCompute = 256;          // compute threads
+constexpr int kTcThreads = 288;          // + one MMA warp
+constexpr int kTcComputeBar = 1;         // named barrier id of the compute warps
+
 template <class Env>
-__global__ void __launch_bounds__(256, 1) ppo_tc_kernel(const PpoTcArgs a) {
+__global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a) {
   using State = typename Env::State;
+  constexpr int NA = Env::kNumActions;
   extern __shared__ __align__(16) uint8_t smem[];  // no-swizzle operands need 16 B
-  __shared__ __align__(8) uint64_t mbar[8];  // [3*agent + layer], [6] weights, [7] drain
+  __shared__ __align__(8) uint64_t acc_bar[4];     // [2*agent + layer], tcgen05.commit
+  __shared__ __align__(8) uint64_t opnd_bar[4];    // [2*agent + layer], 256 arrivals
+  __shared__ __align__(8) uint64_t wload_bar, drain_bar;
   __shared__ uint32_t tmem_slot;
+  __shared__ volatile int abort_flag;
 
   const int4 tile = a.tiles[blockIdx.x];
   const int count = tile.y;
   if (count == 0) return;
   const TcDims& d = a.tc;
-  const int tid = threadIdx.x, warp = tid >> 5, half = warp >> 2, row = tid & 127;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, half = (warp >> 2) & 1, row = tid & 127;
   const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
   const int64_t N = a.n_envs;
   const int od = a.b.env.obs_dim;
-  const int NA = a.b.mlp.NA;
+  const int cells = od / 4;          // observation words per row
+  const int chunks = d.KP / 16;      // 16-byte chunks per observation row
+  const int split = (chunks + 1) / 2;
+  const int my_c0 = half ? split : 0, my_c1 = half ? chunks : split;
+  const int my_w0 = min(4 * my_c0, cells), my_w1 = min(4 * my_c1, cells);
+  const bool with_boot = a.traj.last_value != nullptr;
 
-  uint8_t* sW[2] = {smem, smem + d.pol_bytes};
-  uint8_t* sObs = smem + 2 * d.pol_bytes;                                   // [128][KP] u8
+  uint8_t* const sW0 = smem;                                                // policy blocks
+  uint8_t* const sObs = smem + 2 * d.pol_bytes;                             // [128][KP] u8
   State* st = reinterpret_cast<State*>(sObs + 128 * d.KP);                  // [128]
   int32_t* envid = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(st) + align_up(128 * sizeof(State), 16));
+  uint8_t* act1s = reinterpret_cast<uint8_t*>(envid + 128);                 // [128]
+  float* zpart = reinterpret_cast<float*>(act1s + 128);                     // [2][128][8]
 
   if (tid == 0) {
-    for (int i = 0; i < 8; ++i) tc::mbar_init(&mbar[i], 1);
+    for (int i = 0; i < 4; ++i) {
+      tc::mbar_init(&acc_bar[i], 1);
+      tc::mbar_init(&opnd_bar[i], kTcCompute);
+    }
+    tc::mbar_init(&wload_bar, 1);
+    tc::mbar_init(&drain_bar, 1);
     tc::mbar_init_fence();
+    abort_flag = 0;
   }
   if (warp == 0) tc::tmem_alloc(&tmem_slot, 512);
-  for (int i = tid; i < 32 * d.KP; i += blockDim.x) reinterpret_cast<uint32_t*>(sObs)[i] = 0u;
+  for (int i = tid; i < 32 * d.KP; i += blockDim.x) {  // zero padding, constant 1 at obs_dim
+    const int r = i / (d.KP / 4), w = i - r * (d.KP / 4);
+    reinterpret_cast<uint32_t*>(sObs)[i] = w == cells ? 1u : 0u;
+  }
   if (tid < count) {
     const int env = a.perm[tile.x + tid];
     envid[tid] = env;
@@ -61,156 +93,202 @@ __global__ void __launch_bounds__(256, 1) ppo_tc_kernel(const PpoTcArgs a) {
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = tmem_slot;
-  const int pol[2] = {a.ego, tile.z};
-  if (tid == 0) {
-    tc::mbar_expect_tx(&mbar[6], 2u * d.pol_bytes);
-    for (int p = 0; p < 2; ++p) {
-      const uint8_t* src = a.tcw + (int64_t)pol[p] * d.pol_bytes;
-      for (uint32_t off = 0; off < d.pol_bytes; off += 32768u)
-        tc::bulk_g2s(sW[p] + off, src + off, min(32768u, d.pol_bytes - off), &mbar[6]);
+
+  if (warp == 8) {
+    // ================================ MMA warp =====================================
+    if (lane == 0) {
+      const int pol[2] = {a.ego, tile.z};
+      tc::mbar_expect_tx(&wload_bar, 2u * d.pol_bytes);
+      for (int p = 0; p < 2; ++p) {
+        const uint8_t* src = a.tcw + (int64_t)pol[p] * d.pol_bytes;
+        for (uint32_t off = 0; off < d.pol_bytes; off += 32768u)
+          tc::bulk_g2s(sW0 + p * d.pol_bytes + off, src + off, min(32768u, d.pol_bytes - off), &wload_bar);
+      }
+      bool ok = tc::mbar_wait(&wload_bar, 0);
+      const uint32_t idesc1 = tc::idesc_bf16(128, d.H0), idesc2 = tc::idesc_bf16(128, d.H1);
+      const uint32_t sbo1 = (uint32_t)(d.KP / 8) * 128u, sbo2 = (uint32_t)(d.H0 / 8) * 128u;
+      // agents in the order the compute warps release them: teammate, then ego
+      auto issue = [&](int ag, int layer, uint32_t parity) {
+        ok = false;
+        for (int tries = 0; tries < 1000 && !ok && !abort_flag; ++tries)
+          ok = tc::mbar_wait(&opnd_bar[2 * ag + layer], parity, 2000000ull);
+        if (!ok) return;
+        tc::fence_after_sync();
+        const uint32_t wbase = tc::smem_u32(sW0) + (uint32_t)ag * d.pol_bytes;
+        const uint32_t P = tmem + (uint32_t)(ag * 256), Q = P + 128;
+        if (layer == 0) {
+          const uint64_t w0 = tc::smem_desc(wbase + d.oW1, 128u, sbo1);
+          for (int ks = 0; ks < d.KP / 16; ++ks) tc::mma_ts(Q, P + 8 * ks, w0 + 16u * ks, idesc1, ks > 0);
+        } else {
+          const uint64_t w0 = tc::smem_desc(wbase + d.oW2, 128u, sbo2);
+          for (int ks = 0; ks < d.H0 / 16; ++ks) tc::mma_ts(Q, P + 8 * ks, w0 + 16u * ks, idesc2, 1u);
+          for (int ks = 0; ks < d.H0 / 16; ++ks) tc::mma_ts(Q, P + d.H0 / 2 + 8 * ks, w0 + 16u * ks, idesc2, 1u);
+        }
+        tc::commit(&acc_bar[2 * ag + layer]);
+      };
+      for (int t = 0; ok && t < a.T; ++t) {
+        const uint32_t par = (uint32_t)t & 1u;
+        issue(1, 0, par);
+        if (ok) issue(0, 0, par);
+        if (ok) issue(1, 1, par);
+        if (ok) issue(0, 1, par);
+      }
+      if (ok && with_boot) {
+        issue(0, 0, (uint32_t)a.T & 1u);
+        if (ok) issue(0, 1, (uint32_t)a.T & 1u);
+      }
+      if (!ok) abort_flag = 1;
     }
-  }
-  bool bad = !tc::mbar_wait(&mbar[6], 0);
-  uint32_t phase[6] = {0, 0, 0, 0, 0, 0};
-  const uint32_t idesc_h0 = tc::idesc_bf16(128, d.H0), idesc_h1 = tc::idesc_bf16(128, d.H1);
-  const uint32_t idesc_o = tc::idesc_bf16(128, d.N3);
+  } else {
+    // ============================== compute warps ===================================
+    bool bad = false;
+    auto wait_acc = [&](int ag, int layer, uint32_t parity) {
+      if (!bad && !tc::mbar_wait(&acc_bar[2 * ag + layer], parity)) bad = true;
+      bad = __any_sync(0xFFFFFFFFu, bad);  // warp-uniform: tensor-memory loads are collective
+      tc::fence_after_sync();
+    };
+    auto operand_ready = [&](int ag, int layer) {  // this thread's tensor-memory traffic is done
+      tc::fence_before_sync();
+      tc::mbar_arrive(&opnd_bar[2 * ag + layer]);
+    };
+    auto sync_or = [&]() { return tc::bar_or(kTcComputeBar, kTcCompute, bad || abort_flag); };
+    auto pol_block = [&](int ag) { return sW0 + (size_t)ag * d.pol_bytes; };
 
-  auto colP = [&](int ag) { return tmem + (uint32_t)(ag * 256); };
-  auto colQ = [&](int ag) { return tmem + (uint32_t)(ag * 256 + 128); };
-  auto bias = [&](int ag, uint32_t off) { return reinterpret_cast<const float*>(sW[ag] + off); };
-
-  // ---- MMA issue (thread 0) ----------------------------------------------------------
-  auto issue_layer = [&](int ag, int layer) {
-    tc::fence_after_sync();
-    const uint32_t wbase = tc::smem_u32(sW[ag]);
-    if (layer == 0) {
-      const uint32_t sbo = (uint32_t)(d.KP / 8) * 128u;
-      for (int ks = 0; ks < d.KP / 16; ++ks)
-        tc::mma_ts(colQ(ag), colP(ag) + ks * 8, tc::smem_desc(wbase + d.oW1 + ks * 256u, 128u, sbo),
-                   idesc_h0, ks > 0);
-    } else {
-      const int K = layer == 1 ? d.H0 : d.H1;
-      const uint32_t woff = layer == 1 ? d.oW2 : d.oW3;
-      const uint32_t idesc = layer == 1 ? idesc_h1 : idesc_o;
-      const uint32_t sbo = (uint32_t)(K / 8) * 128u;
-      for (int part = 0; part < 2; ++part)  // hi, then lo half of the split activations
-        for (int ks = 0; ks < K / 16; ++ks)
-          tc::mma_ts(colQ(ag), colP(ag) + part * (K / 2) + ks * 8,
-                     tc::smem_desc(wbase + woff + ks * 256u, 128u, sbo), idesc, (part | ks) != 0);
-    }
-    tc::commit(&mbar[3 * ag + layer]);
-  };
-
-  // ---- observation tile -> tensor memory (both halves, 8 columns per chunk) -----------
-  auto write_x = [&](int ag) {
-    const int chunks = d.KP / 16, first = half ? (chunks + 1) / 2 : 0, last = half ? chunks : (chunks + 1) / 2;
-    const uint8_t* rowp = sObs + row * d.KP;
-    for (int c = first; c < last; ++c) {
-      const uint4 q = *reinterpret_cast<const uint4*>(rowp + 16 * c);
-      const uint32_t w4[4] = {q.x, q.y, q.z, q.w};
-      uint32_t v[8];
+    // observation (built into this thread's half row) -> bf16 A operand of L1
+    auto obs_x = [&](int ag) {
+      if (row < count)
+        Env::obs_words(a.b.env, st[row], ag, reinterpret_cast<uint32_t*>(sObs + row * d.KP), my_w0, my_w1);
+      const uint8_t* rowp = sObs + row * d.KP;
+      const uint32_t P = tmem + (uint32_t)(ag * 256) + lane_base;
+      for (int c = my_c0; c < my_c1; ++c) {
+        const uint4 q = *reinterpret_cast<const uint4*>(rowp + 16 * c);
+        uint32_t v[8] = {tc::bytes_to_bf16x2(q.x, 0), tc::bytes_to_bf16x2(q.x, 2),
+                         tc::bytes_to_bf16x2(q.y, 0), tc::bytes_to_bf16x2(q.y, 2),
+                         tc::bytes_to_bf16x2(q.z, 0), tc::bytes_to_bf16x2(q.z, 2),
+                         tc::bytes_to_bf16x2(q.w, 0), tc::bytes_to_bf16x2(q.w, 2)};
+        tc::st_x8(P + 8 * c, v);
+      }
+      tc::wait_st();
+      operand_ready(ag, 0);
+    };
+    // epilogue 1: h1 = tanh(D) -> hi | lo bf16 A operand of L2; b2 into the accumulator
+    auto epilogue1 = [&](int ag) {
+      const int H = d.H0;
+      const uint32_t P = tmem + (uint32_t)(ag * 256) + lane_base, Q = P + 128;
+      const float* b2 = reinterpret_cast<const float*>(pol_block(ag) + d.ob2);
+      for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 32) {
+        uint32_t v[32];
+        tc::ld_x32(Q + c0, v);
+        tc::wait_ld();
+        uint32_t hi[16], lo[16];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const uint32_t x = w4[j];
-        v[2 * j] = tc::pack_bf16((float)(x & 0xFFu), (float)((x >> 8) & 0xFFu));
-        v[2 * j + 1] = tc::pack_bf16((float)((x >> 16) & 0xFFu), (float)(x >> 24));
-      }
-      tc::st_x8(colP(ag) + lane_base + 8 * c, v);
-    }
-    tc::wait_st();
-  };
-
-  // ---- hidden-layer epilogue: tanh(D + b), split into bf16 hi | lo -> A operand -------
-  auto epilogue = [&](int ag, int layer) {
-    const int H = layer == 0 ? d.H0 : d.H1;
-    const float* b = bias(ag, layer == 0 ? d.ob1 : d.ob2);
-    for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 32) {
-      uint32_t v[32];
-      tc::ld_x32(colQ(ag) + lane_base + c0, v);
-      tc::wait_ld();
-      uint32_t hi[16], lo[16];
+        for (int j = 0; j < 16; ++j)
+          tc::split_bf16x2(tc::tanh_ex2(__uint_as_float(v[2 * j])),
+                           tc::tanh_ex2(__uint_as_float(v[2 * j + 1])), hi[j], lo[j]);
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const float h0 = tanhf(__uint_as_float(v[2 * j]) + b[c0 + 2 * j]);
-        const float h1 = tanhf(__uint_as_float(v[2 * j + 1]) + b[c0 + 2 * j + 1]);
-        const __nv_bfloat16 a0 = __float2bfloat16_rn(h0), a1 = __float2bfloat16_rn(h1);
-        hi[j] = (uint32_t)__bfloat16_as_ushort(a0) | ((uint32_t)__bfloat16_as_ushort(a1) << 16);
-        lo[j] = tc::pack_bf16(h0 - __bfloat162float(a0), h1 - __bfloat162float(a1));
+        for (int j = 0; j < 32; j += 4) {
+          const float4 bb = *reinterpret_cast<const float4*>(b2 + c0 + j);
+          v[j] = __float_as_uint(bb.x); v[j + 1] = __float_as_uint(bb.y);
+          v[j + 2] = __float_as_uint(bb.z); v[j + 3] = __float_as_uint(bb.w);
+        }
+        tc::st_x16(P + c0 / 2, hi);
+        tc::st_x16(P + H / 2 + c0 / 2, lo);
+        tc::st_x32(Q + c0, v);
       }
-      tc::st_x16(colP(ag) + lane_base + c0 / 2, hi);
-      tc::st_x16(colP(ag) + lane_base + H / 2 + c0 / 2, lo);
-    }
-    tc::wait_st();
-  };
-
-  // ---- logits (warps 0-3 only): z = D + b3 ---------------------------------------------
-  auto logits = [&](int ag, float (&z)[16]) {
-    uint32_t v[16];
-    tc::ld_x16(colQ(ag) + lane_base, v);
-    tc::wait_ld();
-    const float* b = bias(ag, d.ob3);
+      tc::wait_st();
+      operand_ready(ag, 1);
+    };
+    // epilogue 2: h2 = tanh(D) and this half's partial z = sum_k W3[:, k] h2[k]
+    auto epilogue2 = [&](int ag, float (&z)[8]) {
+      const int H = d.H1;
+      const uint32_t Q = tmem + (uint32_t)(ag * 256 + 128) + lane_base;
+      const float* W3 = reinterpret_cast<const float*>(pol_block(ag) + d.oW3);
 #pragma unroll
-    for (int j = 0; j < 16; ++j) z[j] = __uint_as_float(v[j]) + b[j];
-  };
-
-  auto wait_layer = [&](int ag, int layer) {
-    const int i = 3 * ag + layer;
-    if (!tc::mbar_wait(&mbar[i], phase[i] & 1u)) bad = true;
-    phase[i] += 1;
-    tc::fence_after_sync();
-  };
-  // Barrier after which thread 0 may issue: tensor-memory traffic of all threads is done.
-  auto handoff = [&]() -> bool {
-    tc::fence_before_sync();
-    return __syncthreads_or(bad) != 0;
-  };
-
-  if (__syncthreads_or(bad)) goto drain;
-
-  for (int t = 0; t <= a.T; ++t) {
-    const bool boot = t == a.T;  // after the last step: the ego's V_T only
-    if (boot && !a.traj.last_value) break;
-    const uint32_t gt = a.step0 + (uint32_t)t;
-    // observations of both seats, L1 of each as soon as its tile is in tensor memory
-    for (int ag = 0; ag < (boot ? 1 : 2); ++ag) {
-      if (half == 0 && row < count) Env::obs(a.b.env, st[row], ag, sObs + row * d.KP);
-      __syncthreads();
-      if (ag == 0 && !boot && a.traj.obs)
-        copy_obs_rows(sObs, d.KP, count, envid, a.traj.obs + (int64_t)t * N * od, od);
-      write_x(ag);
-      if (handoff()) goto drain;
-      if (tid == 0) issue_layer(ag, 0);
-    }
-    for (int layer = 0; layer < 2; ++layer) {
-      for (int ag = 0; ag < (boot ? 1 : 2); ++ag) {
-        wait_layer(ag, layer);
-        epilogue(ag, layer);
-        if (handoff()) goto drain;
-        if (tid == 0) issue_layer(ag, layer + 1);
+      for (int o = 0; o < 8; ++o) z[o] = 0.0f;
+      for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 32) {
+        uint32_t v[32];
+        tc::ld_x32(Q + c0, v);
+        tc::wait_ld();
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const float h = tc::tanh_ex2(__uint_as_float(v[j]));
+          const float4 wa = *reinterpret_cast<const float4*>(W3 + (c0 + j) * 8);
+          const float4 wb = *reinterpret_cast<const float4*>(W3 + (c0 + j) * 8 + 4);
+          z[0] = fmaf(h, wa.x, z[0]); z[1] = fmaf(h, wa.y, z[1]);
+          z[2] = fmaf(h, wa.z, z[2]); z[3] = fmaf(h, wa.w, z[3]);
+          z[4] = fmaf(h, wb.x, z[4]); z[5] = fmaf(h, wb.y, z[5]);
+          z[6] = fmaf(h, wb.z, z[6]); z[7] = fmaf(h, wb.w, z[7]);
+        }
       }
-    }
-    float z[16];
-    int act0 = 0, act1 = 0;
-    float lp0 = 0.f, val0 = 0.f;
-    wait_layer(0, 2);
-    if (half == 0) {
-      logits(0, z);
-      val0 = z[NA];
-      if (boot) {
-        if (row < count) a.traj.last_value[envid[row]] = val0;
-      } else if (row < count) {
-        const float u = u01(draw0(a.b.key, (uint32_t)envid[row], gt, kStreamAct0));
-        act0 = sample_row(z, NA, 0xFFFFFFFFu >> (32 - NA), u, lp0);
+    };
+    // full logits of agent ag in the half that samples it: (half 0 + half 1) + b3
+    auto combine = [&](int ag, const float (&mine)[8], float (&z)[16]) {
+      const float* other = zpart + (ag * 128 + row) * 8;
+      const float* b3 = reinterpret_cast<const float*>(pol_block(ag) + d.ob3);
+#pragma unroll
+      for (int o = 0; o < 8; ++o) {
+        const float p0 = half == 0 ? mine[o] : other[o], p1 = half == 0 ? other[o] : mine[o];
+        z[o] = (p0 + p1) + b3[o];
       }
-    }
-    if (boot) break;
-    wait_layer(1, 2);
-    if (half == 0) {
-      logits(1, z);
+#pragma unroll
+      for (int o = 8; o < 16; ++o) z[o] = 0.0f;
+    };
+    auto publish = [&](int ag, const float (&mine)[8]) {  // for the other half to combine
+      float* dst = zpart + (ag * 128 + row) * 8;
+      *reinterpret_cast<float4*>(dst) = make_float4(mine[0], mine[1], mine[2], mine[3]);
+      *reinterpret_cast<float4*>(dst + 4) = make_float4(mine[4], mine[5], mine[6], mine[7]);
+    };
+    // ego observation rows -> trajectory, one warp per row
+    auto copy_obs = [&](int t) {
+      const int words = od / 4;
+      for (int r = warp; r < count; r += 8) {
+        const uint32_t* src = reinterpret_cast<const uint32_t*>(sObs + r * d.KP);
+        uint32_t* dst = reinterpret_cast<uint32_t*>(a.traj.obs + ((int64_t)t * N + envid[r]) * od);
+        for (int w = lane; w < words; w += 32) dst[w] = src[w];
+      }
+    };
+
+    int t = 0;
+    for (; t < a.T; ++t) {
+      const uint32_t par = (uint32_t)t & 1u, gt = a.step0 + (uint32_t)t;
+      obs_x(1);                       // teammate first: the ego's rows stay for the copy
+      obs_x(0);
+      wait_acc(1, 0, par);
+      if (!bad) epilogue1(1);
+      wait_acc(0, 0, par);
+      if (!bad) epilogue1(0);
+      if (a.traj.obs) {               // overlaps L2 on the tensor cores
+        if (sync_or()) break;
+        copy_obs(t);
+      }
+      float zt[8], ze[8];
+      wait_acc(1, 1, par);
+      if (!bad) epilogue2(1, zt);
+      if (half == 0) publish(1, zt);
+      wait_acc(0, 1, par);
+      if (!bad) epilogue2(0, ze);
+      if (half == 1) publish(0, ze);
+      if (sync_or()) break;
+      int act0 = 0;
+      float lp0 = 0.f, val0 = 0.f;
       if (row < count) {
-        float lp1;
-        const float u = u01(draw0(a.b.key, (uint32_t)envid[row], gt, kStreamAct1));
-        act1 = sample_row(z, NA, 0xFFFFFFFFu >> (32 - NA), u, lp1);
+        float z[16];
+        const int ag = half == 0 ? 0 : 1;
+        combine(ag, ag == 0 ? ze : zt, z);
+        const float u = u01(draw0(a.b.key, (uint32_t)envid[row], gt, kStreamAct0 + ag));
+        float lp;
+        const int act = sample_k<NA>(z, 0xFFFFFFFFu >> (32 - NA), u, lp);
+        if (ag == 1) {
+          act1s[row] = (uint8_t)act;
+        } else {
+          act0 = act;
+          lp0 = lp;
+          val0 = z[NA];
+        }
+      }
+      if (sync_or()) break;
+      if (half == 0 && row < count) {
+        const int act1 = act1s[row];
         const int env = envid[row];
         float r0, r1, team;
         const int done = Env::step(a.b.env, st[row], act0, act1, r0, r1, team);
@@ -223,19 +301,37 @@ __global__ void __launch_bounds__(256, 1) ppo_tc_kernel(const PpoTcArgs a) {
         if (a.traj.dones) a.traj.dones[o] = (uint8_t)(done > 0);
         if (done > 0) Env::reset(a.b.env, a.b.key, (uint32_t)env, gt + 1, st[row]);
       }
+      if (sync_or()) break;
     }
-    if (handoff()) goto drain;
+    if (t == a.T && with_boot && !bad && !abort_flag) {  // V_T of the state after the last step
+      const uint32_t par = (uint32_t)t & 1u;
+      obs_x(0);
+      wait_acc(0, 0, par);
+      if (!bad) epilogue1(0);
+      float ze[8];
+      wait_acc(0, 1, par);
+      if (!bad) epilogue2(0, ze);
+      if (half == 1) publish(0, ze);
+      if (!sync_or() && half == 0 && row < count) {
+        float z[16];
+        combine(0, ze, z);
+        a.traj.last_value[envid[row]] = z[NA];
+      }
+    }
+    if (bad || abort_flag) {
+      abort_flag = 1;
+    } else if (tid < count) {
+      store_state(a.state, N, envid[tid], st[tid]);
+    }
   }
-  if (tid < count) store_state(a.state, N, envid[tid], st[tid]);
 
-drain:
-  if (__syncthreads_or(bad)) {
-    if (tid == 0) atomicOr(a.b.status, kStatusTimeout);
-  }
-  // Wait (bounded) until every MMA this CTA issued has completed, then free tensor memory.
-  if (tid == 0) {
-    tc::commit(&mbar[7]);
-    tc::mbar_wait(&mbar[7], 0);
+  // ---- drain: every MMA this CTA issued completes (bounded), then free tensor memory ---
+  tc::fence_before_sync();
+  __syncthreads();
+  if (tid == 0 && abort_flag) atomicOr(a.b.status, kStatusTimeout);
+  if (warp == 8 && lane == 0) {
+    tc::commit(&drain_bar);
+    tc::mbar_wait(&drain_bar, 0);
   }
   tc::fence_before_sync();
   __syncthreads();
@@ -250,7 +346,7 @@ struct LaunchTc {
   static cudaError_t ppo(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
     cudaError_t e = cudaFuncSetAttribute(ppo_tc_kernel<Env>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    ppo_tc_kernel<Env><<<grid, 256, smem, s>>>(a);
+    ppo_tc_kernel<Env><<<grid, kTcThreads, smem, s>>>(a);
     return cudaGetLastError();
   }
 };

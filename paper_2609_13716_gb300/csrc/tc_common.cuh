@@ -85,6 +85,15 @@ __device__ __forceinline__ void st_x16(uint32_t taddr, const uint32_t (&v)[16]) 
       "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
       "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]));
 }
+__device__ __forceinline__ void st_x32(uint32_t taddr, const uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
+      "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]),
+      "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]),
+      "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31]));
+}
 __device__ __forceinline__ void ld_x16(uint32_t taddr, uint32_t (&v)[16]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
@@ -141,6 +150,21 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* mbar, uint32_t parity,
   return false;
 }
 
+__device__ __forceinline__ void mbar_arrive(uint64_t* mbar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(mbar)) : "memory");
+}
+
+// Named barrier over `count` threads with an OR reduction of `pred` (all get the OR).
+__device__ __forceinline__ bool bar_or(int id, int count, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n.reg .pred p, q;\nsetp.ne.u32 p, %1, 0;\nbar.red.or.pred q, %2, %3, p;\nselp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "r"(id), "r"(count)
+      : "memory");
+  return r != 0;
+}
+
 // 1-D bulk copy global -> shared (TMA), completion counted on mbar in bytes.
 __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* mbar) {
   asm volatile(
@@ -155,6 +179,54 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   uint32_t r;
   asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
   return r;
+}
+
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// tanh from the identity tanh(x) = sign(x) (1 - e) / (1 + e), e = exp(-2|x|)
+// = 2^(-2|x| / ln 2): one ex2.approx (relative error ~2^-22), then the reciprocal of
+// d = 1 + e in [1, 2] by Newton-Raphson (r <- r + r (1 - d r), error squared per step)
+// from a quadratic seed fitted to 1/d on [1, 2] (relative error 1.0e-2), two steps.
+// Absolute error ~1e-7 over the whole line, one transcendental-unit op per call.
+__device__ __forceinline__ float tanh_ex2(float x) {
+  const float e = ex2_approx(fabsf(x) * -2.8853900817779268f);
+  const float d = 1.0f + e;
+  float r = fmaf(fmaf(0.32323139905929565f, d, -1.4545434713363647f), d, 2.121211528778076f);
+  r = fmaf(r, fmaf(-d, r, 1.0f), r);
+  r = fmaf(r, fmaf(-d, r, 1.0f), r);
+  return copysignf(fmaf(-e, r, r), x);
+}
+
+// Bytes b0, b1 of a 32-bit word (unsigned 0..255) as a packed bf16x2 (b0 low), without
+// integer-to-float conversion instructions: 0x4B000000 | b is the float 2^23 + b, so
+// subtracting 2^23 gives b exactly; a value below 2^8 is exact in bf16, whose bits are
+// the float's upper 16 bits.
+__device__ __forceinline__ uint32_t bytes_to_bf16x2(uint32_t w, int first) {
+  const float f0 = __uint_as_float(__byte_perm(w, 0x4B000000u, 0x7440 + first)) - 8388608.0f;
+  const float f1 = __uint_as_float(__byte_perm(w, 0x4B000000u, 0x7441 + first)) - 8388608.0f;
+  return __byte_perm(__float_as_uint(f0), __float_as_uint(f1), 0x7632);
+}
+
+// Split h = hi + lo into two bf16 (hi = round(h), lo = round(h - hi)) for a pair of
+// values; the difference h - hi is exact in fp32.
+__device__ __forceinline__ void split_bf16x2(float h0, float h1, uint32_t& hi, uint32_t& lo) {
+  hi = pack_bf16(h0, h1);
+  const float r0 = h0 - __uint_as_float(hi << 16);
+  const float r1 = h1 - __uint_as_float(hi & 0xFFFF0000u);
+  lo = pack_bf16(r0, r1);
+}
+
+// D[tmem] (+)= A[smem desc] * B[smem desc]^T, M = 128, cta_group::1.
+__device__ __forceinline__ void mma_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                       uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate));
 }
 
 }  // namespace tc

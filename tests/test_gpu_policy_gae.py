@@ -55,6 +55,28 @@ def test_policy_outputs_match_fp64(name, policies):
             assert (got[:, K] == 0).all()
 
 
+def test_tensor_core_epilogue_tanh_error_bound():
+    # The epilogue's tanh (one hardware exp2 + Newton reciprocal) against fp64 tanh: the
+    # split-bf16 activations carry 2^-17 relative precision, so 3e-7 absolute suffices.
+    require_gpu()
+    x = torch.cat([torch.linspace(-12, 12, 2_000_001, dtype=torch.float64),
+                   torch.tensor([0.0, 1e-30, -1e-30, 1e-7, -1e-7, 1e-3, 20.0, -20.0, 88.0, -88.0,
+                                 float("inf"), float("-inf")], dtype=torch.float64)])
+    xf = x.to(torch.float32)
+    y = torch.empty_like(xf, device="cuda")
+    aht.aht_debug_tanh(xf.cuda(), y)
+    torch.cuda.synchronize()
+    got = y.cpu().double()
+    want = torch.tanh(xf.double())
+    err = (got - want).abs()
+    assert err.max().item() <= 3e-7, (err.max().item(), xf[err.argmax()].item())
+    assert torch.equal(y[xf == 0].cpu(), torch.zeros_like(y[xf == 0].cpu()))
+    neg = torch.empty_like(y)
+    aht.aht_debug_tanh((-xf).cuda(), neg)
+    assert torch.equal(neg, -y)                 # odd function, bit for bit
+    assert got.abs().max().item() <= 1.0
+
+
 @pytest.mark.parametrize("T,N,p_done", [(128, 5000, 0.02), (1, 1, 0.0), (7, 33, 0.5)])
 def test_gae_kernel(T, N, p_done):
     require_gpu()
