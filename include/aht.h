@@ -124,14 +124,17 @@ typedef struct aht_traj {
 } aht_traj;
 
 /* PPO rollout collection (App. C "PPO ego"; Sec. 3 ego vs teammates from T_train).
- * Each env draws its teammate once per call: pool[floor(x * pool_size / 2^32)] with x
- * the first draw of counter (env, step0, stream 3).  Then for t in 0..T-1 (step
+ * Teammates are assigned per block of AHT_TEAMMATE_BLOCK (128) consecutive envs, once per
+ * call: block k plays pool[floor(x * pool_size / 2^32)] with x the first draw of counter
+ * (128 k, step0, stream 3), so each env meets a uniformly drawn pool member and every
+ * block runs one teammate policy (one tensor-core tile).  Then for t in 0..T-1 (step
  * step0+t): both seats observe, the ego and the teammate MLPs run, actions are
  * sampled by inverse CDF with u from stream 0/1, the env steps, and an env whose
  * episode ended is reset at step step0+t+1 (stream 2).  Finally V_T is computed and
  * GAE (advantages, targets) is formed when `advantages` is non-NULL.  The step counter
  * advances by T.  Simultaneous-move envs only (LBF, Overcooked): AHT_EINVAL for Hanabi.
  * pool: host [pool_size] policy ids, 1 <= pool_size <= 256.  T >= 1. */
+#define AHT_TEAMMATE_BLOCK 128
 aht_status aht_rollout(aht_ctx* ctx, int32_t ego_id, const int32_t* pool, int32_t pool_size,
                        int32_t T, const aht_traj* out);
 
@@ -225,8 +228,8 @@ aht_status aht_policy_forward(aht_ctx* ctx, int32_t policy, const uint8_t* obs, 
                               float* out);
 
 /* The tanh of the tensor-core epilogue, elementwise: y[i] = tanh(x[i]) for device f32
- * arrays of n elements (computed as sign(x)(1 - e)/(1 + e), e = exp(-2|x|), with one
- * hardware exp2 and a Newton-Raphson reciprocal; absolute error ~1e-7).  Stateless;
+ * arrays of n elements (computed as sign(x)(1 - e)/(1 + e), e = exp(-2|x|), with the
+ * hardware exp2 and reciprocal approximations; absolute error below 1e-6).  Stateless;
  * enqueued on cuda_stream. */
 aht_status aht_debug_tanh(const float* x, float* y, int64_t n, void* cuda_stream);
 

@@ -874,7 +874,10 @@ extern "C" int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32
   std::vector<int> status(N, 0);
   parallel_for(N, io->n_threads, [&](int64_t e) {
     const uint32_t env = (uint32_t)(io->env_ids ? io->env_ids[e] : e);
-    const uint32_t x = orc_draw(io->seed, env, (uint32_t)io->step0, ORC_STREAM_TEAMMATE, 0);
+    // Teammate: one uniform pool draw per block of ORC_TEAMMATE_BLOCK consecutive envs
+    // and call, taken from the block's first env (counter (first env, step0, stream 3)).
+    const uint32_t first = env - env % ORC_TEAMMATE_BLOCK;
+    const uint32_t x = orc_draw(io->seed, first, (uint32_t)io->step0, ORC_STREAM_TEAMMATE, 0);
     const int tm_id = io->pool[orc_uniform_int(x, (uint32_t)io->pool_size)];
     if (io->teammate) io->teammate[e] = tm_id;
     const orc_mlp* tm = &pols[tm_id];

@@ -151,6 +151,8 @@ void orc_gae(const float* r, const float* v, const uint8_t* d, const float* v_la
              double* adv, double* targets);
 
 /* ---- PPO rollout collection (simultaneous-move envs) ---------------------------- */
+/* Envs 128k .. 128k+127 share the teammate drawn for env 128k. */
+enum { ORC_TEAMMATE_BLOCK = 128 };
 typedef struct orc_rollout_io {
   /* inputs */
   uint64_t seed;

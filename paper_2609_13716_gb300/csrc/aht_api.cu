@@ -246,11 +246,11 @@ TcDims make_tc_dims(const MlpDims& m) {
 }
 
 // Shared memory of the tensor-core kernel: both policies' blocks, the u8 observation
-// tile [128][KP], 128 env states, 128 env ids, 128 teammate actions and the output
-// layer's partial sums [2 agents][128][8] fp32.
-size_t tc_smem_bytes(const TcDims& t, int state_bytes) {
-  return 2 * (size_t)t.pol_bytes + 128 * (size_t)t.KP + align_up(128 * state_bytes, 16) + 512 + 128 +
-         2 * 128 * 8 * 4;
+// tile [128][obs_dim], 128 env states, 128 teammate actions and the output layer's
+// partial sums [2 agents][2 halves][128][8] fp32.
+size_t tc_smem_bytes(const TcDims& t, int obs_dim, int state_bytes) {
+  return 2 * (size_t)t.pol_bytes + align_up(128 * obs_dim, 16) + align_up(128 * state_bytes, 16) + 128 +
+         4 * 128 * 8 * 4;
 }
 
 // The tensor-core path applies to bf16 populations of LBF whose padded observation
@@ -261,7 +261,7 @@ bool tc_eligible(const aht_ctx* c, int dtype) {
   if (dtype != AHT_BF16 || c->env.kind != AHT_LBF) return false;
   const TcDims t = make_tc_dims(m);
   if (t.KP > 256 || m.H0 > 128 || m.H1 > 128 || m.H0 % 64 || m.H1 % 64 || m.NA + 1 > 8) return false;
-  return tc_smem_bytes(t, c->ops.bytes()) <= c->smem_optin;
+  return m.K % 4 == 0 && tc_smem_bytes(t, m.K, c->ops.bytes()) <= c->smem_optin;
 }
 
 bool read_host(const void* p, size_t bytes, std::vector<uint8_t>& tmp, const void** out) {
@@ -430,7 +430,7 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
   }
 
   const int words = c->ops.words();
-  c->max_tiles = (n_envs + 3) / 4 + kMaxPool;
+  c->max_tiles = group_tiles(n_envs, 4);  // the smallest tile any launch uses
   struct Alloc { void** p; size_t bytes; };
   Alloc allocs[] = {
       {(void**)&c->state, (size_t)words * n_envs * 4},
@@ -459,7 +459,7 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
     if (cudaEventCreate(&e) != cudaSuccess) return bail(AHT_ECUDA, "cudaEventCreate failed");
   if (tc_eligible(c, pop->weight_dtype)) {
     c->tcd = make_tc_dims(m);
-    c->tc_smem = tc_smem_bytes(c->tcd, c->ops.bytes());
+    c->tc_smem = tc_smem_bytes(c->tcd, m.K, c->ops.bytes());
     std::vector<uint8_t> blocks((size_t)c->tcd.pol_bytes * pop->n_policies);
     for (int p = 0; p < pop->n_policies; ++p) {
       const int vh = pop->has_value_head ? pop->has_value_head[p] : 0;
@@ -530,7 +530,7 @@ aht_status aht_rollout(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t 
   ga.pool_size = pool_size;
   for (int k = 0; k < pool_size; ++k) ga.pool[k] = pool[k];
   ga.M = M;
-  ga.max_tiles = (int)((c->n_envs + M - 1) / M + pool_size);
+  ga.max_tiles = group_tiles(c->n_envs, M);
   ga.perm = c->perm;
   ga.tiles = c->tiles;
   ga.teammate = out->teammate;

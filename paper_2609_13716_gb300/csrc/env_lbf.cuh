@@ -33,28 +33,32 @@ struct EnvLbf {
       F += s.fl[k];
     }
     s.F = (uint8_t)F;
-    // n_food + 2 steps of a Fisher-Yates shuffle of the cell indices, with the touched
-    // entries of the permutation kept in a small map (untouched entry p holds p).
+    // n_food + 2 steps of a Fisher-Yates shuffle of the cell indices (identity at the
+    // start).  Step i swaps positions i and j >= i; position i is final afterwards and
+    // never read again, so only the values written to the j's need remembering: wpos[m],
+    // wval[m] for step m (a later write to the same position wins).  Fixed-size loops keep
+    // everything in registers.
     const int cells = d.width * d.height;
-    int key_[10], val_[10], nmap = 0;
-    auto get = [&](int p) {
-      for (int m = 0; m < nmap; ++m)
-        if (key_[m] == p) return val_[m];
-      return p;
-    };
-    auto set = [&](int p, int v) {
-      for (int m = 0; m < nmap; ++m)
-        if (key_[m] == p) { val_[m] = v; return; }
-      key_[nmap] = p; val_[nmap] = v; ++nmap;
-    };
-    int placed[5];
     const int n_obj = d.n_food + 2;
-    for (int i = 0; i < n_obj; ++i) {
-      const int j = i + (int)uniform_int(r.next(), (uint32_t)(cells - i));
-      const int vi = get(i), vj = get(j);
-      set(i, vj);
-      set(j, vi);
-      placed[i] = vj;
+    int wpos[5], wval[5], placed[5];
+#pragma unroll
+    for (int i = 0; i < 5; ++i) {
+      if (i < n_obj) {
+        const int j = i + (int)uniform_int(r.next(), (uint32_t)(cells - i));
+        int vi = i, vj = j;
+#pragma unroll
+        for (int m = 0; m < i; ++m) {
+          if (wpos[m] == i) vi = wval[m];
+          if (wpos[m] == j) vj = wval[m];
+        }
+        placed[i] = vj;  // position i now holds the old value at j
+        wpos[i] = j;     // and position j the old value at i
+        wval[i] = vi;
+      } else {
+        placed[i] = 0;
+        wpos[i] = -1;
+        wval[i] = 0;
+      }
     }
     s.eaten = 0;
     for (int k = 0; k < 3; ++k) {
@@ -75,41 +79,50 @@ struct EnvLbf {
     s.ret = 0.0f;
   }
 
+  // Loops run over all three food slots: absent foods are marked eaten at reset, so the
+  // fixed trip counts keep the state in registers when the caller holds a copy.
   __device__ static int step(const DevEnv& d, State& s, int a0, int a1, float& r0, float& r1,
                              float& team) {
     r0 = 0.0f;
     r1 = 0.0f;
     uint32_t newly = 0;
-    for (int k = 0; k < d.n_food; ++k) {
-      if ((s.eaten >> k) & 1u) continue;
-      const bool l0 = a0 == 5 && abs((int)s.ax[0] - s.fx[k]) + abs((int)s.ay[0] - s.fy[k]) == 1;
-      const bool l1 = a1 == 5 && abs((int)s.ax[1] - s.fx[k]) + abs((int)s.ay[1] - s.fy[k]) == 1;
-      const int lsum = (l0 ? s.al[0] : 0) + (l1 ? s.al[1] : 0);
-      if (lsum > 0 && lsum >= s.fl[k]) {
-        newly |= 1u << k;
-        const float den = (float)(lsum * (int)s.F);
-        if (l0) r0 = __fadd_rn(r0, __fdiv_rn((float)(s.fl[k] * s.al[0]), den));
-        if (l1) r1 = __fadd_rn(r1, __fdiv_rn((float)(s.fl[k] * s.al[1]), den));
+    const int ax0 = s.ax[0], ay0 = s.ay[0], ax1 = s.ax[1], ay1 = s.ay[1];
+    if (a0 == 5 || a1 == 5) {
+#pragma unroll
+      for (int k = 0; k < 3; ++k) {
+        if ((s.eaten >> k) & 1u) continue;
+        const int fx = s.fx[k], fy = s.fy[k], fl = s.fl[k];
+        const bool l0 = a0 == 5 && abs(ax0 - fx) + abs(ay0 - fy) == 1;
+        const bool l1 = a1 == 5 && abs(ax1 - fx) + abs(ay1 - fy) == 1;
+        const int lsum = (l0 ? s.al[0] : 0) + (l1 ? s.al[1] : 0);
+        if (lsum > 0 && lsum >= fl) {
+          newly |= 1u << k;
+          const float den = (float)(lsum * (int)s.F);
+          if (l0) r0 = __fadd_rn(r0, __fdiv_rn((float)(fl * s.al[0]), den));
+          if (l1) r1 = __fadd_rn(r1, __fdiv_rn((float)(fl * s.al[1]), den));
+        }
       }
     }
     int tx[2], ty[2];
-    const int act[2] = {a0, a1};
+#pragma unroll
     for (int i = 0; i < 2; ++i) {
-      const int a = act[i];
+      const int a = i == 0 ? a0 : a1;
+      const int cx = i == 0 ? ax0 : ax1, cy = i == 0 ? ay0 : ay1;
       const int dx = (a == 4) - (a == 3), dy = (a == 2) - (a == 1);
-      int x = s.ax[i] + dx, y = s.ay[i] + dy;
+      const int x = cx + dx, y = cy + dy;
       bool ok = (dx | dy) != 0 && x >= 0 && x < d.width && y >= 0 && y < d.height;
-      for (int k = 0; k < d.n_food && ok; ++k)
+#pragma unroll
+      for (int k = 0; k < 3; ++k)
         if (!((s.eaten >> k) & 1u) && s.fx[k] == x && s.fy[k] == y) ok = false;
-      if (ok && ((s.ax[0] == x && s.ay[0] == y) || (s.ax[1] == x && s.ay[1] == y))) ok = false;
-      tx[i] = ok ? x : s.ax[i];
-      ty[i] = ok ? y : s.ay[i];
+      if ((ax0 == x && ay0 == y) || (ax1 == x && ay1 == y)) ok = false;
+      tx[i] = ok ? x : cx;
+      ty[i] = ok ? y : cy;
     }
     if (!(tx[0] == tx[1] && ty[0] == ty[1])) {
-      for (int i = 0; i < 2; ++i) {
-        s.ax[i] = (uint8_t)tx[i];
-        s.ay[i] = (uint8_t)ty[i];
-      }
+      s.ax[0] = (uint8_t)tx[0];
+      s.ay[0] = (uint8_t)ty[0];
+      s.ax[1] = (uint8_t)tx[1];
+      s.ay[1] = (uint8_t)ty[1];
     }
     s.eaten |= (uint8_t)newly;
     s.ep_t += 1;
@@ -139,7 +152,8 @@ struct EnvLbf {
       const int c = y * d.width + x;
       if (c >= w0 && c < w1) w[c] = v;
     };
-    for (int k = 0; k < d.n_food; ++k)
+#pragma unroll
+    for (int k = 0; k < 3; ++k)  // absent foods are marked eaten
       if (!((s.eaten >> k) & 1u)) put(s.fx[k], s.fy[k], (uint32_t)s.fl[k] << 16);
     const int o = 1 - seat;
     put(s.ax[o], s.ay[o], (uint32_t)s.al[o] << 8);

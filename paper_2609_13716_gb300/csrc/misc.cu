@@ -7,71 +7,34 @@
 
 namespace aht {
 
-// ---- teammate assignment + stable grouping (one CTA) -----------------------------------
-// Env e draws pool index b = floor(x * pool_size / 2^32), x = first draw of (e, step0,
-// stream 3).  Envs are then ordered by b (stable in e) so that every tile of M rows
-// shares one teammate policy.  cnt holds per-(bin, thread) counts, bin-major.
-__global__ void __launch_bounds__(kGroupThreads) group_kernel(const GroupArgs a) {
-  extern __shared__ uint32_t cnt[];  // [pool_size][kGroupThreads]
-  __shared__ uint32_t seg[kGroupThreads];
-  __shared__ uint32_t start[kMaxPool + 1];
-  const int tid = threadIdx.x;
-  const int P = a.pool_size;
-  const int64_t chunk = (a.n_envs + kGroupThreads - 1) / kGroupThreads;
-  const int64_t lo = tid * chunk, hi = min(a.n_envs, lo + chunk);
-  for (int b = 0; b < P; ++b) cnt[b * kGroupThreads + tid] = 0;
-  for (int64_t e = lo; e < hi; ++e) {
-    const uint32_t b = uniform_int(draw0(a.key, (uint32_t)e, a.step0, kStreamTeammate), (uint32_t)P);
-    cnt[b * kGroupThreads + tid] += 1;
-  }
-  __syncthreads();
-  // Exclusive scan of the flattened counts: thread j owns entries [j*P, (j+1)*P).
-  uint32_t run = 0;
-  for (int q = 0; q < P; ++q) run += cnt[tid * P + q];
-  seg[tid] = run;
-  __syncthreads();
-  if (tid == 0) {
-    uint32_t acc = 0;
-    for (int j = 0; j < kGroupThreads; ++j) {
-      const uint32_t v = seg[j];
-      seg[j] = acc;
-      acc += v;
+// ---- teammate assignment: one pool draw per block of kTeammateBlock envs ---------------
+// Block k (envs 128k .. 128k+127) plays pool[floor(x * pool_size / 2^32)], x = first draw
+// of (128k, step0, stream 3).  Tiles of up to M rows never cross a block, so each tile
+// runs one teammate policy; the env order is the identity (perm[e] = e).
+__global__ void group_kernel(const GroupArgs a) {
+  const int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (e >= a.n_envs) return;
+  const int64_t blk = e / kTeammateBlock, first = blk * kTeammateBlock;
+  const uint32_t b = uniform_int(draw0(a.key, (uint32_t)first, a.step0, kStreamTeammate), (uint32_t)a.pool_size);
+  const int tm = a.pool[b];
+  a.perm[e] = (int32_t)e;
+  if (a.teammate) a.teammate[e] = tm;
+  if (e == first) {
+    const int n_blk = (int)min((int64_t)kTeammateBlock, a.n_envs - first);
+    const int tpb = (kTeammateBlock + a.M - 1) / a.M;
+    for (int j = 0; j < tpb; ++j) {
+      const int r0 = j * a.M, cnt = max(0, min(a.M, n_blk - r0));
+      a.tiles[blk * tpb + j] = make_int4((int)first + r0, cnt, tm, 0);
     }
-  }
-  __syncthreads();
-  run = seg[tid];
-  for (int q = 0; q < P; ++q) {
-    const uint32_t v = cnt[tid * P + q];
-    cnt[tid * P + q] = run;
-    run += v;
-  }
-  __syncthreads();
-  for (int b = tid; b <= P; b += blockDim.x) start[b] = b < P ? cnt[b * kGroupThreads] : (uint32_t)a.n_envs;
-  __syncthreads();
-  for (int64_t e = lo; e < hi; ++e) {
-    const uint32_t b = uniform_int(draw0(a.key, (uint32_t)e, a.step0, kStreamTeammate), (uint32_t)P);
-    const uint32_t pos = cnt[b * kGroupThreads + tid]++;
-    a.perm[pos] = (int32_t)e;
-    if (a.teammate) a.teammate[e] = a.pool[b];
-  }
-  if (tid == 0) {
-    int t = 0;
-    for (int b = 0; b < P; ++b) {
-      const int n_b = (int)(start[b + 1] - start[b]);
-      for (int j = 0; j * a.M < n_b; ++j)
-        a.tiles[t++] = make_int4((int)start[b] + j * a.M, min(a.M, n_b - j * a.M), a.pool[b], 0);
-    }
-    for (; t < a.max_tiles; ++t) a.tiles[t] = make_int4(0, 0, 0, 0);
   }
 }
 
-size_t group_smem_bytes(int pool_size) { return (size_t)pool_size * kGroupThreads * 4; }
+int group_tiles(int64_t n_envs, int M) {
+  return (int)(((n_envs + kTeammateBlock - 1) / kTeammateBlock) * ((kTeammateBlock + M - 1) / M));
+}
 
 cudaError_t launch_group(const GroupArgs& a, cudaStream_t s) {
-  const size_t smem = group_smem_bytes(a.pool_size);
-  cudaError_t e = cudaFuncSetAttribute(group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  group_kernel<<<1, kGroupThreads, smem, s>>>(a);
+  group_kernel<<<(unsigned)((a.n_envs + 255) / 256), 256, 0, s>>>(a);
   return cudaGetLastError();
 }
 

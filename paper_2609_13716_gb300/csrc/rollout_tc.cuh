@@ -62,12 +62,15 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   const int my_w0 = min(4 * my_c0, cells), my_w1 = min(4 * my_c1, cells);
   const bool with_boot = a.traj.last_value != nullptr;
 
+  // The tile is the contiguous env range [tile.x, tile.x + count); observation rows are
+  // packed at obs_dim bytes (an odd number of words: no bank conflicts per thread row),
+  // so the tile's rows form one contiguous block for a single bulk store.
   uint8_t* const sW0 = smem;                                                // policy blocks
-  uint8_t* const sObs = smem + 2 * d.pol_bytes;                             // [128][KP] u8
-  State* st = reinterpret_cast<State*>(sObs + 128 * d.KP);                  // [128]
-  int32_t* envid = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(st) + align_up(128 * sizeof(State), 16));
-  uint8_t* act1s = reinterpret_cast<uint8_t*>(envid + 128);                 // [128]
-  float* zpart = reinterpret_cast<float*>(act1s + 128);                     // [2][128][8]
+  uint8_t* const sObs = smem + 2 * d.pol_bytes;                             // [128][obs_dim] u8
+  State* st = reinterpret_cast<State*>(sObs + align_up(128 * od, 16));      // [128]
+  uint8_t* act1s = reinterpret_cast<uint8_t*>(st) + align_up(128 * sizeof(State), 16);  // [128]
+  float* zpart = reinterpret_cast<float*>(act1s + 128);                     // [2][2][128][8]
+  const int64_t env0 = tile.x;
 
   if (tid == 0) {
     for (int i = 0; i < 4; ++i) {
@@ -80,15 +83,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     abort_flag = 0;
   }
   if (warp == 0) tc::tmem_alloc(&tmem_slot, 512);
-  for (int i = tid; i < 32 * d.KP; i += blockDim.x) {  // zero padding, constant 1 at obs_dim
-    const int r = i / (d.KP / 4), w = i - r * (d.KP / 4);
-    reinterpret_cast<uint32_t*>(sObs)[i] = w == cells ? 1u : 0u;
-  }
-  if (tid < count) {
-    const int env = a.perm[tile.x + tid];
-    envid[tid] = env;
-    load_state(a.state, N, env, st[tid]);
-  }
+  for (int i = tid; i < 32 * od; i += blockDim.x) reinterpret_cast<uint32_t*>(sObs)[i] = 0u;
+  if (tid < count) load_state(a.state, N, env0 + tid, st[tid]);
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
@@ -154,18 +150,25 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     auto sync_or = [&]() { return tc::bar_or(kTcComputeBar, kTcCompute, bad || abort_flag); };
     auto pol_block = [&](int ag) { return sW0 + (size_t)ag * d.pol_bytes; };
 
-    // observation (built into this thread's half row) -> bf16 A operand of L1
-    auto obs_x = [&](int ag) {
-      if (row < count)
-        Env::obs_words(a.b.env, st[row], ag, reinterpret_cast<uint32_t*>(sObs + row * d.KP), my_w0, my_w1);
-      const uint8_t* rowp = sObs + row * d.KP;
+    // observation (built into this thread's half row) -> bf16 A operand of L1; feature
+    // obs_dim is the constant 1 that carries b1, the rest of the padding is 0
+    auto obs_x = [&](int ag, const State& s) {
+      uint32_t* roww = reinterpret_cast<uint32_t*>(sObs + row * od);
+      if (row < count) Env::obs_words(a.b.env, s, ag, roww, my_w0, my_w1);
       const uint32_t P = tmem + (uint32_t)(ag * 256) + lane_base;
       for (int c = my_c0; c < my_c1; ++c) {
-        const uint4 q = *reinterpret_cast<const uint4*>(rowp + 16 * c);
-        uint32_t v[8] = {tc::bytes_to_bf16x2(q.x, 0), tc::bytes_to_bf16x2(q.x, 2),
-                         tc::bytes_to_bf16x2(q.y, 0), tc::bytes_to_bf16x2(q.y, 2),
-                         tc::bytes_to_bf16x2(q.z, 0), tc::bytes_to_bf16x2(q.z, 2),
-                         tc::bytes_to_bf16x2(q.w, 0), tc::bytes_to_bf16x2(q.w, 2)};
+        uint32_t w4[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int w = 4 * c + j;
+          w4[j] = w < cells ? roww[w] : (w == cells ? 1u : 0u);
+        }
+        uint32_t v[8];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          v[2 * j] = tc::bytes_to_bf16x2(w4[j], 0);
+          v[2 * j + 1] = tc::bytes_to_bf16x2(w4[j], 2);
+        }
         tc::st_x8(P + 8 * c, v);
       }
       tc::wait_st();
@@ -198,13 +201,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       tc::wait_st();
       operand_ready(ag, 1);
     };
-    // epilogue 2: h2 = tanh(D) and this half's partial z = sum_k W3[:, k] h2[k]
-    auto epilogue2 = [&](int ag, float (&z)[8]) {
+    // epilogue 2: h2 = tanh(D) and this half's partial z = sum_k W3[:, k] h2[k], stored
+    // for the half that samples the agent
+    auto epilogue2 = [&](int ag) {
       const int H = d.H1;
       const uint32_t Q = tmem + (uint32_t)(ag * 256 + 128) + lane_base;
       const float* W3 = reinterpret_cast<const float*>(pol_block(ag) + d.oW3);
-#pragma unroll
-      for (int o = 0; o < 8; ++o) z[o] = 0.0f;
+      uint64_t z2[4] = {0, 0, 0, 0};  // output pairs (0,1) (2,3) (4,5) (6,7), fp32 each
       for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 32) {
         uint32_t v[32];
         tc::ld_x32(Q + c0, v);
@@ -212,72 +215,90 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
           const float h = tc::tanh_ex2(__uint_as_float(v[j]));
-          const float4 wa = *reinterpret_cast<const float4*>(W3 + (c0 + j) * 8);
-          const float4 wb = *reinterpret_cast<const float4*>(W3 + (c0 + j) * 8 + 4);
-          z[0] = fmaf(h, wa.x, z[0]); z[1] = fmaf(h, wa.y, z[1]);
-          z[2] = fmaf(h, wa.z, z[2]); z[3] = fmaf(h, wa.w, z[3]);
-          z[4] = fmaf(h, wb.x, z[4]); z[5] = fmaf(h, wb.y, z[5]);
-          z[6] = fmaf(h, wb.z, z[6]); z[7] = fmaf(h, wb.w, z[7]);
+          const uint64_t hh = tc::f2_pack(h, h);
+          const ulonglong2 wa = *reinterpret_cast<const ulonglong2*>(W3 + (c0 + j) * 8);
+          const ulonglong2 wb = *reinterpret_cast<const ulonglong2*>(W3 + (c0 + j) * 8 + 4);
+          z2[0] = tc::f2_fma(hh, wa.x, z2[0]);
+          z2[1] = tc::f2_fma(hh, wa.y, z2[1]);
+          z2[2] = tc::f2_fma(hh, wb.x, z2[2]);
+          z2[3] = tc::f2_fma(hh, wb.y, z2[3]);
         }
       }
+      ulonglong2* dst = reinterpret_cast<ulonglong2*>(zpart + ((ag * 2 + half) * 128 + row) * 8);
+      dst[0] = make_ulonglong2(z2[0], z2[1]);
+      dst[1] = make_ulonglong2(z2[2], z2[3]);
     };
-    // full logits of agent ag in the half that samples it: (half 0 + half 1) + b3
-    auto combine = [&](int ag, const float (&mine)[8], float (&z)[16]) {
-      const float* other = zpart + (ag * 128 + row) * 8;
+    // full logits of agent ag: (half-0 partial + half-1 partial) + b3
+    auto logits = [&](int ag, float (&z)[16]) {
+      const float* p0 = zpart + ((ag * 2 + 0) * 128 + row) * 8;
+      const float* p1 = zpart + ((ag * 2 + 1) * 128 + row) * 8;
       const float* b3 = reinterpret_cast<const float*>(pol_block(ag) + d.ob3);
 #pragma unroll
-      for (int o = 0; o < 8; ++o) {
-        const float p0 = half == 0 ? mine[o] : other[o], p1 = half == 0 ? other[o] : mine[o];
-        z[o] = (p0 + p1) + b3[o];
-      }
+      for (int o = 0; o < 8; ++o) z[o] = (p0[o] + p1[o]) + b3[o];
 #pragma unroll
       for (int o = 8; o < 16; ++o) z[o] = 0.0f;
     };
-    auto publish = [&](int ag, const float (&mine)[8]) {  // for the other half to combine
-      float* dst = zpart + (ag * 128 + row) * 8;
-      *reinterpret_cast<float4*>(dst) = make_float4(mine[0], mine[1], mine[2], mine[3]);
-      *reinterpret_cast<float4*>(dst + 4) = make_float4(mine[4], mine[5], mine[6], mine[7]);
-    };
-    // ego observation rows -> trajectory, one warp per row
+    // the tile's ego observation rows -> trajectory [t][env0 .. env0+count): one contiguous
+    // block, written by one bulk (TMA) store when 16-byte aligned, else by all threads
+    const bool bulk_obs = a.traj.obs && (count * od) % 16 == 0;
     auto copy_obs = [&](int t) {
-      const int words = od / 4;
-      for (int r = warp; r < count; r += 8) {
-        const uint32_t* src = reinterpret_cast<const uint32_t*>(sObs + r * d.KP);
-        uint32_t* dst = reinterpret_cast<uint32_t*>(a.traj.obs + ((int64_t)t * N + envid[r]) * od);
-        for (int w = lane; w < words; w += 32) dst[w] = src[w];
+      uint8_t* dst = a.traj.obs + ((int64_t)t * N + env0) * od;
+      const uint32_t bytes = (uint32_t)(count * od);
+      if (bulk_obs && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
+        if (tid == 0) {
+          tc::bulk_s2g(dst, sObs, bytes);
+          tc::bulk_commit();
+        }
+      } else {
+        const uint32_t* src = reinterpret_cast<const uint32_t*>(sObs);
+        uint32_t* d32 = reinterpret_cast<uint32_t*>(dst);
+        for (uint32_t w = tid; w < bytes / 4; w += kTcCompute) d32[w] = src[w];
       }
     };
 
-    int t = 0;
-    for (; t < a.T; ++t) {
+    // Steps 0..T-1, then (if requested) the ego's V_T of the state after the last step.
+    // The agent loops are not unrolled so that every phase's code exists once.
+    for (int t = 0; t <= a.T; ++t) {
+      const bool boot = t == a.T;
+      if (boot && !with_boot) break;
+      const int first = boot ? 0 : 1;  // teammate first: the ego's rows stay for the copy
       const uint32_t par = (uint32_t)t & 1u, gt = a.step0 + (uint32_t)t;
-      obs_x(1);                       // teammate first: the ego's rows stay for the copy
-      obs_x(0);
-      wait_acc(1, 0, par);
-      if (!bad) epilogue1(1);
-      wait_acc(0, 0, par);
-      if (!bad) epilogue1(0);
-      if (a.traj.obs) {               // overlaps L2 on the tensor cores
+      // this half's action draw (ego: warps 0-3, teammate: warps 4-7), ahead of its use
+      const float u_act = boot ? 0.0f : u01(draw0(a.b.key, (uint32_t)(env0 + row), gt, kStreamAct0 + half));
+      State s = st[row];  // register copy for this step (rows past count are never used)
+#pragma unroll 1
+      for (int i = first; i >= 0; --i) obs_x(i, s);
+#pragma unroll 1
+      for (int i = first; i >= 0; --i) {
+        wait_acc(i, 0, par);
+        if (!bad) epilogue1(i);
+      }
+      if (!boot && a.traj.obs) {       // overlaps L2 on the tensor cores
+        tc::fence_proxy_async();       // the rows were written by ordinary stores
         if (sync_or()) break;
         copy_obs(t);
       }
-      float zt[8], ze[8];
-      wait_acc(1, 1, par);
-      if (!bad) epilogue2(1, zt);
-      if (half == 0) publish(1, zt);
-      wait_acc(0, 1, par);
-      if (!bad) epilogue2(0, ze);
-      if (half == 1) publish(0, ze);
+#pragma unroll 1
+      for (int i = first; i >= 0; --i) {
+        wait_acc(i, 1, par);
+        if (!bad) epilogue2(i);
+      }
       if (sync_or()) break;
+      float z[16];
+      if (boot) {
+        if (half == 0 && row < count) {
+          logits(0, z);
+          a.traj.last_value[env0 + row] = z[NA];
+        }
+        break;
+      }
       int act0 = 0;
       float lp0 = 0.f, val0 = 0.f;
       if (row < count) {
-        float z[16];
         const int ag = half == 0 ? 0 : 1;
-        combine(ag, ag == 0 ? ze : zt, z);
-        const float u = u01(draw0(a.b.key, (uint32_t)envid[row], gt, kStreamAct0 + ag));
+        logits(ag, z);
         float lp;
-        const int act = sample_k<NA>(z, 0xFFFFFFFFu >> (32 - NA), u, lp);
+        const int act = sample_k<NA>(z, 0xFFFFFFFFu >> (32 - NA), u_act, lp);
         if (ag == 1) {
           act1s[row] = (uint8_t)act;
         } else {
@@ -289,9 +310,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       if (sync_or()) break;
       if (half == 0 && row < count) {
         const int act1 = act1s[row];
-        const int env = envid[row];
+        const int64_t env = env0 + row;
         float r0, r1, team;
-        const int done = Env::step(a.b.env, st[row], act0, act1, r0, r1, team);
+        const int done = Env::step(a.b.env, s, act0, act1, r0, r1, team);
         const int64_t o = (int64_t)t * N + env;
         if (a.traj.actions) a.traj.actions[o] = (uint8_t)act0;
         if (a.traj.tm_actions) a.traj.tm_actions[o] = (uint8_t)act1;
@@ -299,29 +320,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         if (a.traj.values) a.traj.values[o] = val0;
         if (a.traj.rewards) a.traj.rewards[o] = team;
         if (a.traj.dones) a.traj.dones[o] = (uint8_t)(done > 0);
-        if (done > 0) Env::reset(a.b.env, a.b.key, (uint32_t)env, gt + 1, st[row]);
+        if (done > 0) Env::reset(a.b.env, a.b.key, (uint32_t)env, gt + 1, s);
+        st[row] = s;
       }
+      if (tid == 0 && bulk_obs) tc::bulk_wait_read();  // the rows may be rebuilt
       if (sync_or()) break;
     }
-    if (t == a.T && with_boot && !bad && !abort_flag) {  // V_T of the state after the last step
-      const uint32_t par = (uint32_t)t & 1u;
-      obs_x(0);
-      wait_acc(0, 0, par);
-      if (!bad) epilogue1(0);
-      float ze[8];
-      wait_acc(0, 1, par);
-      if (!bad) epilogue2(0, ze);
-      if (half == 1) publish(0, ze);
-      if (!sync_or() && half == 0 && row < count) {
-        float z[16];
-        combine(0, ze, z);
-        a.traj.last_value[envid[row]] = z[NA];
-      }
-    }
+    if (tid == 0 && bulk_obs) tc::bulk_wait_all();
     if (bad || abort_flag) {
       abort_flag = 1;
     } else if (tid < count) {
-      store_state(a.state, N, envid[tid], st[tid]);
+      store_state(a.state, N, env0 + tid, st[tid]);
     }
   }
 

@@ -174,6 +174,21 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       : "memory");
 }
 
+// 1-D bulk copy shared -> global (TMA), tracked by bulk groups of the issuing thread.
+// Both addresses 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void bulk_s2g(void* dst, const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst),
+               "r"(smem_u32(src)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// Until the sources of all committed bulk stores have been read (shared memory reusable).
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+// Until all committed bulk stores are complete.
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
 // Two fp32 -> packed bf16x2 (lo in the low half).
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   uint32_t r;
@@ -187,17 +202,18 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 
+__device__ __forceinline__ float rcp_approx(float x) {
+  float y;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // tanh from the identity tanh(x) = sign(x) (1 - e) / (1 + e), e = exp(-2|x|)
-// = 2^(-2|x| / ln 2): one ex2.approx (relative error ~2^-22), then the reciprocal of
-// d = 1 + e in [1, 2] by Newton-Raphson (r <- r + r (1 - d r), error squared per step)
-// from a quadratic seed fitted to 1/d on [1, 2] (relative error 1.0e-2), two steps.
-// Absolute error ~1e-7 over the whole line, one transcendental-unit op per call.
+// = 2^(-2|x| / ln 2), with the hardware approximations of 2^x and 1/x (relative errors
+// ~2^-22 each): six instructions, absolute error below 1e-6 over the whole line.
 __device__ __forceinline__ float tanh_ex2(float x) {
   const float e = ex2_approx(fabsf(x) * -2.8853900817779268f);
-  const float d = 1.0f + e;
-  float r = fmaf(fmaf(0.32323139905929565f, d, -1.4545434713363647f), d, 2.121211528778076f);
-  r = fmaf(r, fmaf(-d, r, 1.0f), r);
-  r = fmaf(r, fmaf(-d, r, 1.0f), r);
+  const float r = rcp_approx(1.0f + e);
   return copysignf(fmaf(-e, r, r), x);
 }
 
@@ -211,12 +227,33 @@ __device__ __forceinline__ uint32_t bytes_to_bf16x2(uint32_t w, int first) {
   return __byte_perm(__float_as_uint(f0), __float_as_uint(f1), 0x7632);
 }
 
+// ---- packed fp32 pairs (sm_100+ f32x2 arithmetic; each lane is IEEE fp32) -------------
+__device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_sub(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
 // Split h = hi + lo into two bf16 (hi = round(h), lo = round(h - hi)) for a pair of
 // values; the difference h - hi is exact in fp32.
 __device__ __forceinline__ void split_bf16x2(float h0, float h1, uint32_t& hi, uint32_t& lo) {
   hi = pack_bf16(h0, h1);
-  const float r0 = h0 - __uint_as_float(hi << 16);
-  const float r1 = h1 - __uint_as_float(hi & 0xFFFF0000u);
+  float r0, r1;
+  f2_unpack(f2_sub(f2_pack(h0, h1), f2_pack(__uint_as_float(hi << 16), __uint_as_float(hi & 0xFFFF0000u))),
+            r0, r1);
   lo = pack_bf16(r0, r1);
 }
 

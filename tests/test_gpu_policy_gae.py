@@ -56,8 +56,9 @@ def test_policy_outputs_match_fp64(name, policies):
 
 
 def test_tensor_core_epilogue_tanh_error_bound():
-    # The epilogue's tanh (one hardware exp2 + Newton reciprocal) against fp64 tanh: the
-    # split-bf16 activations carry 2^-17 relative precision, so 3e-7 absolute suffices.
+    # The epilogue's tanh (hardware exp2 and reciprocal) against fp64 tanh.  A hidden unit
+    # error e moves a logit by about |W3 row| e ~ 0.1 * sqrt(128) e ~ 1.1 e, so 1e-6 keeps
+    # logits far inside the 1e-4 tolerance and the 1e-5 CDF margin.
     require_gpu()
     x = torch.cat([torch.linspace(-12, 12, 2_000_001, dtype=torch.float64),
                    torch.tensor([0.0, 1e-30, -1e-30, 1e-7, -1e-7, 1e-3, 20.0, -20.0, 88.0, -88.0,
@@ -69,7 +70,7 @@ def test_tensor_core_epilogue_tanh_error_bound():
     got = y.cpu().double()
     want = torch.tanh(xf.double())
     err = (got - want).abs()
-    assert err.max().item() <= 3e-7, (err.max().item(), xf[err.argmax()].item())
+    assert err.max().item() <= 1e-6, (err.max().item(), xf[err.argmax()].item())
     assert torch.equal(y[xf == 0].cpu(), torch.zeros_like(y[xf == 0].cpu()))
     neg = torch.empty_like(y)
     aht.aht_debug_tanh((-xf).cuda(), neg)

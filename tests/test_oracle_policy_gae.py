@@ -145,16 +145,25 @@ def test_rollout_matches_stepwise_replay(orc):
     assert np.array_equal(out["actions"], out["own_actions"])
 
 
-def test_rollout_teammate_draw_is_uniform(orc):
+def test_rollout_teammate_draw_is_uniform_per_block(orc):
+    # One uniform pool draw per block of 128 consecutive envs (the last block may be
+    # partial): constant within blocks, uniform over the pool across blocks.
     wl = W.WORKLOADS["lbf7x7_64x50_fp32"]
     d = orc.env_desc(*wl.env.astuple())
     pols = orc.Policies(W.population(wl) * 4)   # 8 policies
-    N = 4000
-    st = orc.reset_all(d, 1, N)
-    out = orc.rollout(d, pols, 1, st, 0, 1, 0, [1, 3, 5, 7])
-    c = np.bincount(out["teammate"], minlength=8)
+    tms = []
+    for seed in range(12):
+        N = 128 * 40 + 77
+        st = orc.reset_all(d, seed, N)
+        out = orc.rollout(d, pols, seed, st, 0, 1, 0, [1, 3, 5, 7])
+        tm = out["teammate"]
+        blocks = [tm[i:i + 128] for i in range(0, N, 128)]
+        assert all((b == b[0]).all() for b in blocks)
+        tms += [int(b[0]) for b in blocks]
+    c = np.bincount(tms, minlength=8)
     assert c[[0, 2, 4, 6]].sum() == 0
-    assert np.abs(c[[1, 3, 5, 7]] - 1000).max() < 5 * np.sqrt(1000)
+    n = len(tms) / 4
+    assert np.abs(c[[1, 3, 5, 7]] - n).max() < 5 * np.sqrt(n)
 
 
 def test_xplay_matrix_is_pair_mean(orc):
