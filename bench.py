@@ -26,7 +26,6 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 WORKLOAD = "lbf7x7_ppo_16384x128"
-XPLAY_WORKLOAD = "lbf7x7_xplay_8x16x256"
 METRIC = "env-steps/sec (LBF 7x7 PPO rollout collection + GAE, ego vs 32-policy population)"
 UNIT = "env-steps/s"
 L2_BYTES = 129 * 2 ** 20
@@ -336,7 +335,7 @@ def run_ours(args):
             "clocks": clocks.summary(),
         }
     if not args.no_xplay:
-        xp = run_xplay(args, aht, W, torch)
+        xp = run_xplay(args, aht, W, torch, bf16_peak)
         if line is not None:
             line["xplay"] = xp
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -350,35 +349,52 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-def run_xplay(args, aht, W, torch):
-    """Cross-play cells/s on the 8x16 LBF matrix, 256 envs per pair, 128-step episodes."""
-    wl = W.WORKLOADS[XPLAY_WORKLOAD]
-    pop = [[(torch.from_numpy(Wt).cuda(), torch.from_numpy(b).cuda()) for Wt, b in p]
-           for p in W.population(wl)]
-    n = wl.xplay_envs
-    ctx = aht.aht_create(wl.env, pop, n, wl.env_seed, weight_dtype=aht.AHT_FP32)
-    ne, nt = len(wl.ego_ids), len(wl.tm_ids)
-    matrix = torch.empty(ne, nt, device="cuda")
-    steps = torch.empty(ne, nt, wl.envs_per_pair, dtype=torch.int32, device="cuda")
-    call = lambda: aht.aht_xplay_matrix(ctx, list(wl.ego_ids), list(wl.tm_ids),
-                                        wl.envs_per_pair, wl.max_steps, matrix, None, steps)
-    for _ in range(3):
-        call()
-    torch.cuda.synchronize()
-    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    K = max(3, args.steps)
-    s.record()
-    for _ in range(K):
-        call()
-    e.record()
-    torch.cuda.synchronize()
-    ms = s.elapsed_time(e) / K
-    active = int(steps.sum())
-    aht.aht_sync(ctx)
-    ctx.close()
-    return {"workload": XPLAY_WORKLOAD, "cells_per_s": ne * nt / (ms * 1e-3),
-            "ms_per_matrix": ms, "active_env_steps_per_s": active / (ms * 1e-3),
-            "dtype": "f32"}
+XPLAY_WORKLOADS = ("lbf7x7_xplay_8x16x256", "overcooked5x4_xplay_8x8x64", "hanabi_xplay_16x16x32")
+
+
+def run_xplay(args, aht, W, torch, bf16_peak):
+    """Cross-play matrices: cells/s and active env-steps/s of each cross-play workload, and
+    the fraction of the tensor roofline (MLP FLOPs of the env-steps that actually ran, one
+    forward per acting agent, at the bf16 peak)."""
+    res = {}
+    for name in XPLAY_WORKLOADS:
+        wl = W.WORKLOADS[name]
+        dt = torch.bfloat16 if wl.weight_dtype == W.BF16 else torch.float32
+        pop = [[(torch.from_numpy(Wt).to("cuda", dt), torch.from_numpy(b).to("cuda", dt)) for Wt, b in p]
+               for p in W.population(wl)]
+        n = wl.xplay_envs
+        ctx = aht.aht_create(wl.env, pop, n, wl.env_seed,
+                             weight_dtype=aht.AHT_BF16 if wl.weight_dtype == W.BF16 else aht.AHT_FP32)
+        ne, nt = len(wl.ego_ids), len(wl.tm_ids)
+        matrix = torch.empty(ne, nt, device="cuda")
+        steps = torch.empty(ne, nt, wl.envs_per_pair, dtype=torch.int32, device="cuda")
+        call = lambda: aht.aht_xplay_matrix(ctx, list(wl.ego_ids), list(wl.tm_ids),
+                                            wl.envs_per_pair, wl.max_steps, matrix, None, steps)
+        for _ in range(3):
+            call()
+        torch.cuda.synchronize()
+        s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        K = max(3, args.steps)
+        s.record()
+        for _ in range(K):
+            call()
+        e.record()
+        torch.cuda.synchronize()
+        ms = s.elapsed_time(e) / K
+        active = int(steps.sum())
+        aht.aht_sync(ctx)
+        ctx.close()
+        dims = [wl.env.obs_dim, *wl.hidden, wl.env.n_actions]
+        acting = 1 if wl.env.kind == W.HANABI else 2        # Hanabi: one actor per turn
+        flops = active * acting * mlp_flops(dims)
+        tflops = flops / (ms * 1e-3) / 1e12
+        res[name] = {"cells_per_s": ne * nt / (ms * 1e-3), "ms_per_matrix": ms,
+                     "active_env_steps": active, "active_env_steps_per_s": active / (ms * 1e-3),
+                     "weights": "bf16" if wl.weight_dtype == W.BF16 else "f32",
+                     "roofline": {"bound": "tensor", "achieved": tflops, "peak": bf16_peak,
+                                  "unit": "TFLOP/s", "frac": tflops / bf16_peak,
+                                  "flops_per_matrix": flops}}
+    return res
 
 
 def main():
