@@ -48,6 +48,9 @@ def parse():
     p.add_argument("--n-envs", type=int, default=None)
     p.add_argument("--T", type=int, default=None)
     p.add_argument("--no-e2e", action="store_true")
+    # cross-play only (profiling of the cross-play kernels; not a bench line)
+    p.add_argument("--xplay-only", default=None,
+                   help="comma-separated cross-play workloads to time without the rollout")
     return p.parse_args()
 
 
@@ -221,6 +224,11 @@ def run_ours(args):
     hbm_peak = peaks.get("hbm_gbs", 6800.0)
     peak_src = "measured" if peaks else "fallback"
 
+    if args.xplay_only:
+        xp = run_xplay(args, aht, W, torch, bf16_peak, args.xplay_only.split(","))
+        if rank == 0:
+            print(json.dumps({"xplay": xp}), flush=True)
+        return
     wl = W.WORKLOADS[WORKLOAD]
     N, T = args.n_envs or wl.n_envs, args.T or wl.T
     pop_np = W.population(wl)
@@ -352,12 +360,12 @@ def run_ours(args):
 XPLAY_WORKLOADS = ("lbf7x7_xplay_8x16x256", "overcooked5x4_xplay_8x8x64", "hanabi_xplay_16x16x32")
 
 
-def run_xplay(args, aht, W, torch, bf16_peak):
+def run_xplay(args, aht, W, torch, bf16_peak, names=XPLAY_WORKLOADS):
     """Cross-play matrices: cells/s and active env-steps/s of each cross-play workload, and
     the fraction of the tensor roofline (MLP FLOPs of the env-steps that actually ran, one
     forward per acting agent, at the bf16 peak)."""
     res = {}
-    for name in XPLAY_WORKLOADS:
+    for name in names:
         wl = W.WORKLOADS[name]
         dt = torch.bfloat16 if wl.weight_dtype == W.BF16 else torch.float32
         pop = [[(torch.from_numpy(Wt).to("cuda", dt), torch.from_numpy(b).to("cuda", dt)) for Wt, b in p]

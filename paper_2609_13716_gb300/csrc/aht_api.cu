@@ -103,6 +103,15 @@ struct aht_ctx {
   uint8_t* tcw = nullptr;
   size_t tc_smem = 0;
   uint8_t* tc_staging = nullptr;
+  // streamed tensor-core cross-play (bf16 Overcooked / Hanabi populations of width 256/512)
+  bool wide = false;
+  WideDims wd{};
+  uint8_t* wtcw = nullptr;
+  size_t wide_smem = 0;
+  uint32_t* xp_st[2] = {};
+  uint8_t* xp_act[2] = {};
+  uint8_t* xp_alive[2] = {};
+  int32_t* xp_nsteps = nullptr;
   // pinned host staging for aht_set_policy, and the event pool of the kernel timer
   float* staging = nullptr;
   cudaEvent_t upload_done = nullptr;
@@ -264,6 +273,31 @@ bool tc_eligible(const aht_ctx* c, int dtype) {
   return m.K % 4 == 0 && tc_smem_bytes(t, m.K, c->ops.bytes()) <= c->smem_optin;
 }
 
+// Streamed tensor-core block of a wide policy (see WideDims).
+WideDims make_wide_dims(const MlpDims& m) {
+  WideDims w{};
+  w.KP = (int)align_up(m.K + 1, 16);
+  w.H = m.H0;
+  w.NAP = (int)align_up(m.NA, 4);
+  w.n_l1 = (w.H / 256) * (w.KP / 16);
+  w.n_l2 = (w.H / 256) * (w.H / 16);
+  uint32_t o = (uint32_t)(w.n_l1 + w.n_l2) * kWideChunk;
+  w.oW3 = o; o += (uint32_t)(w.H * w.NAP * 4);
+  w.ob2 = o; o += (uint32_t)(w.H * 4);
+  w.ob3 = o; o += (uint32_t)(w.NAP * 4);
+  w.pol_bytes = (uint32_t)align_up(o, 1024);
+  return w;
+}
+
+// Binary-observation games with bf16 weights and equal hidden widths of 256 or 512 run
+// their cross-play steps on the streamed tensor-core kernel.
+bool wide_eligible(const aht_ctx* c, int dtype) {
+  const MlpDims& m = c->mlp;
+  if (dtype != AHT_BF16 || (c->env.kind != AHT_OVERCOOKED && c->env.kind != AHT_HANABI)) return false;
+  if (m.H0 != m.H1 || (m.H0 != 256 && m.H0 != 512)) return false;
+  return xp_tc_smem_bytes(make_wide_dims(m)) <= c->smem_optin;
+}
+
 bool read_host(const void* p, size_t bytes, std::vector<uint8_t>& tmp, const void** out) {
   cudaPointerAttributes at{};
   if (cudaPointerGetAttributes(&at, p) != cudaSuccess) cudaGetLastError();
@@ -312,6 +346,48 @@ aht_status pack_policy_tc(const MlpDims& m, const TcDims& t, const void* const* 
   return AHT_OK;
 }
 
+// Packs one bf16 policy into its streamed block (dst: w.pol_bytes bytes).  A value row,
+// if present, is not used by cross-play and is left out.
+aht_status pack_policy_wide(const MlpDims& m, const WideDims& w, const void* const* W,
+                            const void* const* b, int vh, uint8_t* dst) {
+  std::fill(dst, dst + w.pol_bytes, (uint8_t)0);
+  const int ins[3] = {m.K, m.H0, m.H1};
+  const int outs[3] = {m.H0, m.H1, m.NA + vh};
+  std::vector<uint8_t> tmp;
+  auto w1_at = [&](int n, int k) {
+    return dst + (size_t)((n / 256) * (w.KP / 16) + k / 16) * kWideChunk + tc::canon_offset(n % 256, k % 16, 16);
+  };
+  auto w2_at = [&](int n, int k) {
+    return dst + (size_t)(w.n_l1 + (n / 256) * (w.H / 16) + k / 16) * kWideChunk +
+           tc::canon_offset(n % 256, k % 16, 16);
+  };
+  for (int l = 0; l < 3; ++l) {
+    const void* src = nullptr;
+    if (!W[l] || !b[l]) return fail(AHT_EINVAL, "NULL weight pointer");
+    if (!read_host(W[l], (size_t)outs[l] * ins[l] * 2, tmp, &src)) return fail(AHT_ECUDA, "copying weights failed");
+    const uint16_t* wv = static_cast<const uint16_t*>(src);
+    for (int n = 0; n < outs[l]; ++n)
+      for (int k = 0; k < ins[l]; ++k) {
+        const int64_t i = (int64_t)n * ins[l] + k;
+        if (l == 0) std::memcpy(w1_at(n, k), &wv[i], 2);
+        if (l == 1) std::memcpy(w2_at(n, k), &wv[i], 2);
+        if (l == 2 && n < m.NA) {
+          const float f = to_f32(src, i, AHT_BF16);
+          std::memcpy(dst + w.oW3 + 4 * ((size_t)k * w.NAP + n), &f, 4);
+        }
+      }
+    if (!read_host(b[l], (size_t)outs[l] * 2, tmp, &src)) return fail(AHT_ECUDA, "copying biases failed");
+    const uint16_t* bb = static_cast<const uint16_t*>(src);
+    for (int n = 0; n < outs[l]; ++n) {
+      const float f = to_f32(src, n, AHT_BF16);
+      if (l == 0) std::memcpy(w1_at(n, m.K), &bb[n], 2);  // b1: weight of the constant-1 input
+      if (l == 1) std::memcpy(dst + w.ob2 + 4 * n, &f, 4);
+      if (l == 2 && n < m.NA) std::memcpy(dst + w.ob3 + 4 * n, &f, 4);
+    }
+  }
+  return AHT_OK;
+}
+
 // Kernel timer: events around the main kernel of a call (see aht_set_timing).
 void timer_fold(aht_ctx* c) {
   for (int i = 0; i < c->n_pending; ++i) {
@@ -335,6 +411,51 @@ int timer_begin(aht_ctx* c) {
 
 void timer_end(aht_ctx* c, int i) {
   if (i >= 0) cudaEventRecord(c->ev[2 * i + 1], c->stream);
+}
+
+// Cross-play on the streamed tensor-core kernel: max_steps + 1 launches, one per step
+// (the last applies the final transition), then the exact pair means.
+aht_status xplay_wide(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego, const int32_t* tm_ids,
+                      int32_t n_tm, int32_t P, int32_t max_steps, const aht_xplay_out* out) {
+  XpTcArgs a{};
+  a.b = batch_of(c);
+  a.w = c->wd;
+  a.tcw = c->wtcw;
+  a.n_ego = n_ego;
+  a.n_tm = n_tm;
+  a.P = P;
+  a.max_steps = max_steps;
+  for (int i = 0; i < n_ego; ++i) a.ego_ids[i] = ego_ids[i];
+  for (int j = 0; j < n_tm; ++j) a.tm_ids[j] = tm_ids[j];
+  a.step0 = (uint32_t)c->step;
+  a.n_total = (int64_t)n_ego * n_tm * P;
+  a.nsteps = c->xp_nsteps;
+  a.returns = out->returns ? out->returns : c->xp_returns;
+  a.steps = out->steps;
+  a.actions = out->actions;
+  const int64_t T0 = ((int64_t)n_tm * P + 127) / 128, T1 = ((int64_t)n_ego * P + 127) / 128;
+  const int64_t tiles0 = n_ego * T0, tiles1 = n_tm * T1;
+  if (tiles0 + tiles1 > INT32_MAX) return fail(AHT_EINVAL, "too many tiles");
+  const bool turn = c->env.kind == AHT_HANABI;
+  auto launch = c->env.kind == AHT_HANABI ? hanabi_xplay_tc : overcooked_xplay_tc;
+  const int tk = timer_begin(c);
+  for (int s = 0; s <= max_steps; ++s) {
+    a.s = s;
+    a.st_in = c->xp_st[s & 1];
+    a.st_out = c->xp_st[(s + 1) & 1];
+    a.alive_in = c->xp_alive[s & 1];
+    a.alive_out = c->xp_alive[(s + 1) & 1];
+    a.act_in = c->xp_act[(s + 1) & 1];
+    a.act_out = c->xp_act[s & 1];
+    int64_t grid;
+    if (turn) grid = (s & 1) ? tiles1 : tiles0;
+    else grid = s < max_steps ? tiles0 + tiles1 : tiles0;
+    AHT_CUDA(launch(a, (int)grid, c->wide_smem, c->stream));
+  }
+  timer_end(c, tk);
+  const int64_t n_pairs = (int64_t)n_ego * n_tm;
+  if (out->matrix) AHT_CUDA(launch_xp_reduce(a.returns, n_pairs, P, out->matrix, c->stream));
+  return AHT_OK;
 }
 
 // Tile rows for an M-row launch that fits in shared memory (M multiple of 4).
@@ -376,6 +497,13 @@ void aht_destroy(aht_ctx* c) {
   if (c->staging) cudaFreeHost(c->staging);
   if (c->tc_staging) cudaFreeHost(c->tc_staging);
   cudaFree(c->tcw);
+  cudaFree(c->wtcw);
+  for (int i = 0; i < 2; ++i) {
+    cudaFree(c->xp_st[i]);
+    cudaFree(c->xp_act[i]);
+    cudaFree(c->xp_alive[i]);
+  }
+  cudaFree(c->xp_nsteps);
   if (c->upload_done) cudaEventDestroy(c->upload_done);
   for (auto& e : c->ev)
     if (e) cudaEventDestroy(e);
@@ -479,6 +607,41 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
     if (cudaMallocHost((void**)&c->tc_staging, c->tcd.pol_bytes) != cudaSuccess)
       return bail(AHT_ENOMEM, "pinned staging allocation failed");
     c->tc = true;
+  }
+  if (wide_eligible(c, pop->weight_dtype)) {
+    c->wd = make_wide_dims(m);
+    c->wide_smem = xp_tc_smem_bytes(c->wd);
+    std::vector<uint8_t> blocks((size_t)c->wd.pol_bytes * pop->n_policies);
+    for (int p = 0; p < pop->n_policies; ++p) {
+      const int vh = pop->has_value_head ? pop->has_value_head[p] : 0;
+      aht_status ps = pack_policy_wide(m, c->wd, pop->W + 3 * p, pop->b + 3 * p, vh,
+                                       blocks.data() + (size_t)p * c->wd.pol_bytes);
+      if (ps != AHT_OK) {
+        std::string msg = g_err;
+        return bail(ps, msg);
+      }
+    }
+    Alloc wa[] = {
+        {(void**)&c->wtcw, blocks.size()},
+        {(void**)&c->xp_st[0], (size_t)words * n_envs * 4},
+        {(void**)&c->xp_st[1], (size_t)words * n_envs * 4},
+        {(void**)&c->xp_act[0], (size_t)n_envs * 2},
+        {(void**)&c->xp_act[1], (size_t)n_envs * 2},
+        {(void**)&c->xp_alive[0], (size_t)n_envs},
+        {(void**)&c->xp_alive[1], (size_t)n_envs},
+        {(void**)&c->xp_nsteps, (size_t)n_envs * 4},
+    };
+    for (auto& x : wa)
+      if (cudaMalloc(x.p, x.bytes) != cudaSuccess) {
+        cudaGetLastError();
+        return bail(AHT_ENOMEM, "cudaMalloc of " + std::to_string(x.bytes) + " bytes failed");
+      }
+    if (cudaMemcpy(c->wtcw, blocks.data(), blocks.size(), cudaMemcpyHostToDevice) != cudaSuccess)
+      return bail(AHT_ECUDA, "uploading the streamed tensor-core population failed");
+    const cudaError_t se = env.kind == AHT_HANABI ? hanabi_xplay_tc_smem_limit(c->wide_smem)
+                                                  : overcooked_xplay_tc_smem_limit(c->wide_smem);
+    if (se != cudaSuccess) return bail(AHT_ECUDA, "setting the shared-memory limit failed");
+    c->wide = true;
   }
   *out = c;
   aht_status r = aht_reset(c, seed);
@@ -595,6 +758,13 @@ aht_status aht_xplay_matrix(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego,
   if (n_total > c->n_envs) return fail(AHT_EINVAL, "n_ego*n_tm*envs_per_pair exceeds the context's n_envs");
   if (c->step + max_steps + 1 > (int64_t)UINT32_MAX) return fail(AHT_EINVAL, "step counter would exceed 2^32");
   DeviceGuard g(c->device);
+  if (out->actions) AHT_CUDA(cudaMemsetAsync(out->actions, 255, (size_t)max_steps * n_total * 2, c->stream));
+  if (c->wide) {
+    const aht_status ws = xplay_wide(c, ego_ids, n_ego, tm_ids, n_tm, envs_per_pair, max_steps, out);
+    if (ws != AHT_OK) return ws;
+    c->step += max_steps;
+    return AHT_OK;
+  }
   const int M = fit_rows(c, std::min(c->ops.max_rows, envs_per_pair));
   XpArgs a{};
   a.b = batch_of(c);
@@ -610,7 +780,6 @@ aht_status aht_xplay_matrix(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego,
   a.returns = out->returns ? out->returns : c->xp_returns;
   a.steps = out->steps;
   a.actions = out->actions;
-  if (out->actions) AHT_CUDA(cudaMemsetAsync(out->actions, 255, (size_t)max_steps * n_total * 2, c->stream));
   const size_t smem = smem_layout(M, c->mlp, c->ops.bytes()).total;
   const int64_t grid = n_pairs * a.tiles_per_pair;
   if (grid > INT32_MAX) return fail(AHT_EINVAL, "too many tiles");

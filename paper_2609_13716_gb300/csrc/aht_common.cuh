@@ -82,6 +82,52 @@ __device__ __forceinline__ float u01(uint32_t x) {
   return __uint2float_rn(x >> 8) * (1.0f / 16777216.0f);
 }
 
+// Observation writers.  The env rules fill a row through clear(), set(k, v) (feature k
+// := v), set_bits(k, bits, n) (features k .. k+n-1 := bits 0 .. n-1, n <= 32) and
+// set_run(k, n) (features k .. k+n-1 := 1); every feature is written at most once after
+// clear(), so a writer that only records ones is exact.
+struct ObsBytes {  // one u8 per feature (obs_dim bytes, 4-byte aligned)
+  uint8_t* p;
+  int words;
+  __device__ void clear() {
+    uint32_t* w = reinterpret_cast<uint32_t*>(p);
+    for (int i = 0; i < words; ++i) w[i] = 0u;
+  }
+  __device__ void set(int k, uint32_t v) { p[k] = (uint8_t)v; }
+  __device__ void set_bits(int k, uint32_t bits, int n) {
+    for (int b = 0; b < n; ++b) p[k + b] = (uint8_t)((bits >> b) & 1u);
+  }
+  __device__ void set_run(int k, int n) {
+    for (int b = 0; b < n; ++b) p[k + b] = 1;
+  }
+};
+
+struct ObsBits {  // one bit per feature of binary observations: bit k % 32 of word k / 32
+  uint32_t* w;
+  int words;
+  __device__ void clear() {
+    for (int i = 0; i < words; ++i) w[i] = 0u;
+  }
+  __device__ void set(int k, uint32_t v) {
+    if (v) w[k >> 5] |= 1u << (k & 31);
+  }
+  __device__ void set_bits(int k, uint32_t bits, int n) {
+    if (n < 32) bits &= (1u << n) - 1u;
+    if (!bits) return;
+    const int s = k & 31;
+    w[k >> 5] |= bits << s;
+    if (s && s + n > 32) w[(k >> 5) + 1] |= bits >> (32 - s);
+  }
+  __device__ void set_run(int k, int n) {
+    while (n > 0) {
+      const int m = n < 32 ? n : 32;
+      set_bits(k, m == 32 ? 0xFFFFFFFFu : (1u << m) - 1u, m);
+      k += m;
+      n -= m;
+    }
+  }
+};
+
 __host__ __device__ constexpr inline int64_t align_up(int64_t x, int64_t a) {
   return (x + a - 1) / a * a;
 }

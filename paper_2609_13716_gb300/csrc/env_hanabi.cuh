@@ -197,48 +197,45 @@ struct EnvHanabi {
   }
 
   // 660 binary features for `seat` (see the section offsets below).
-  __device__ static void obs(const DevEnv&, const State& s, int seat, uint8_t* row) {
-    uint32_t* w = reinterpret_cast<uint32_t*>(row);
-    for (int i = 0; i < 165; ++i) w[i] = 0u;
+  template <class Row>
+  __device__ static void obs_into(const DevEnv&, const State& s, int seat, Row& row) {
+    row.clear();
     const int me = seat, pa = seat ^ 1;
-    for (int k = 0; k < s.n_hand[pa]; ++k) row[k * 25 + s.hand[pa][k]] = 1;       // [0,125)
-    for (int q = 0; q < 2; ++q) {                                                // [125,375)
+    for (int k = 0; k < s.n_hand[pa]; ++k) row.set(k * 25 + s.hand[pa][k], 1);  // [0,125)
+    for (int q = 0; q < 2; ++q) {                                              // [125,375)
       const int who = q == 0 ? me : pa;
-      uint8_t* o = row + 125 + q * 125;
-      for (int k = 0; k < s.n_hand[who]; ++k) {
-        const uint32_t m = s.know[who][k];
-        for (int b = 0; b < 25; ++b) o[k * 25 + b] = (uint8_t)((m >> b) & 1u);
-      }
+      for (int k = 0; k < s.n_hand[who]; ++k) row.set_bits(125 + q * 125 + k * 25, s.know[who][k], 25);
     }
-    for (int c = 0; c < 5; ++c)                                                  // [375,400)
-      if (s.fw[c]) row[375 + c * 5 + s.fw[c] - 1] = 1;
-    for (int i = 0; i < s.info; ++i) row[400 + i] = 1;                           // [400,408)
-    for (int i = 0; i < s.lives; ++i) row[408 + i] = 1;                          // [408,411)
-    for (int i = 0; i < 50 - s.ptr; ++i) row[411 + i] = 1;                       // [411,451)
+    for (int c = 0; c < 5; ++c)                                                // [375,400)
+      if (s.fw[c]) row.set(375 + c * 5 + s.fw[c] - 1, 1);
+    row.set_run(400, s.info);                                                  // [400,408)
+    row.set_run(408, s.lives);                                                 // [408,411)
+    row.set_run(411, 50 - s.ptr);                                              // [411,451)
     const uint8_t base[5] = {0, 3, 5, 7, 9};
-    for (int t = 0; t < 25; ++t)                                                 // [451,501)
-      for (int i = 0; i < s.disc[t]; ++i) row[451 + (t / 5) * 10 + base[t % 5] + i] = 1;
-    if (s.la_flags & 1u) {                                                       // [501,554)
-      uint8_t* o = row + 501;
-      o[((s.la_flags >> 1) & 1u) == (uint32_t)me ? 0 : 1] = 1;
-      o[2 + s.la_type] = 1;
-      if (s.la_colour != 255) o[6 + s.la_colour] = 1;
-      if (s.la_rank) o[11 + s.la_rank - 1] = 1;
-      if (s.la_slot != 255) o[16 + s.la_slot] = 1;
-      if (s.la_card != 255) o[21 + s.la_card] = 1;
-      for (int k = 0; k < 5; ++k)
-        if ((s.la_hinted >> k) & 1u) o[46 + k] = 1;
-      if (s.la_flags & 4u) o[51] = 1;
-      if (s.la_flags & 8u) o[52] = 1;
+    for (int t = 0; t < 25; ++t)                                               // [451,501)
+      row.set_run(451 + (t / 5) * 10 + base[t % 5], s.disc[t]);
+    if (s.la_flags & 1u) {                                                     // [501,554)
+      const int o = 501;
+      row.set(o + (((s.la_flags >> 1) & 1u) == (uint32_t)me ? 0 : 1), 1);
+      row.set(o + 2 + s.la_type, 1);
+      if (s.la_colour != 255) row.set(o + 6 + s.la_colour, 1);
+      if (s.la_rank) row.set(o + 11 + s.la_rank - 1, 1);
+      if (s.la_slot != 255) row.set(o + 16 + s.la_slot, 1);
+      if (s.la_card != 255) row.set(o + 21 + s.la_card, 1);
+      row.set_bits(o + 46, s.la_hinted, 5);
+      if (s.la_flags & 4u) row.set(o + 51, 1);
+      if (s.la_flags & 8u) row.set(o + 52, 1);
     }
-    for (int q = 0; q < 2; ++q) {                                                // [554,654)
+    for (int q = 0; q < 2; ++q) {                                              // [554,654)
       const int who = q == 0 ? me : pa;
-      uint8_t* o = row + 554 + q * 50;
-      for (int k = 0; k < 5; ++k)
-        for (int b = 0; b < 10; ++b) o[k * 10 + b] = (uint8_t)((s.hints[who][k] >> b) & 1u);
+      for (int k = 0; k < 5; ++k) row.set_bits(554 + q * 50 + k * 10, s.hints[who][k], 10);
     }
-    for (int k = 0; k < s.n_hand[me]; ++k) row[654 + k] = 1;                     // [654,659)
-    if (s.fr >= 0) row[659] = 1;                                                 // [659]
+    row.set_run(654, s.n_hand[me]);                                            // [654,659)
+    if (s.fr >= 0) row.set(659, 1);                                            // [659]
+  }
+  __device__ static void obs(const DevEnv& d, const State& s, int seat, uint8_t* row) {
+    ObsBytes w{row, 165};
+    obs_into(d, s, seat, w);
   }
 
   __device__ static float ret(const State& s) { return s.ret; }

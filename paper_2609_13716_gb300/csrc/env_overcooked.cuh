@@ -125,39 +125,43 @@ struct EnvOvercooked {
   }
 
   // 26 binary channels per cell, index (y*5 + x)*26 + c.
-  __device__ static void obs(const DevEnv& d, const State& s, int seat, uint8_t* row) {
-    uint32_t* w = reinterpret_cast<uint32_t*>(row);
-    for (int i = 0; i < 130; ++i) w[i] = 0u;
+  template <class Row>
+  __device__ static void obs_into(const DevEnv& d, const State& s, int seat, Row& row) {
+    row.clear();
     const bool urgent = d.episode_len - (int)s.ep_t <= 40;
     for (int c = 0; c < 20; ++c) {
-      uint8_t* o = row + c * 26;
+      const int o = c * 26;
       const int t = kKitchenCell[c];
       if (t == 1) {
-        o[10] = 1;
-        if (s.item[c] != kNone) o[14 + s.item[c]] = 1;
+        row.set(o + 10, 1);
+        if (s.item[c] != kNone) row.set(o + 14 + s.item[c], 1);
       } else if (t == 2) {
-        o[12] = 1;
+        row.set(o + 12, 1);
       } else if (t == 3) {
-        o[11] = 1;
-        if (s.pot_n >= 1) o[17 + s.pot_n] = 1;
-        if (s.pot_n == 3) o[s.pot_timer > 0 ? 21 : 22] = 1;
+        row.set(o + 11, 1);
+        if (s.pot_n >= 1) row.set(o + 17 + s.pot_n, 1);
+        if (s.pot_n == 3) row.set(o + (s.pot_timer > 0 ? 21 : 22), 1);
       } else if (t == 4) {
-        o[13] = 1;
+        row.set(o + 13, 1);
       } else if (t == 5) {
-        o[14] = 1;
+        row.set(o + 14, 1);
       }
-      if (urgent) o[25] = 1;
+      if (urgent) row.set(o + 25, 1);
     }
     for (int who = 0; who < 2; ++who) {
       const int i = who == 0 ? seat : 1 - seat;
-      uint8_t* o = row + (s.ay[i] * 5 + s.ax[i]) * 26;
-      o[who] = 1;
-      o[2 + 4 * who + s.face[i]] = 1;
+      const int o = (s.ay[i] * 5 + s.ax[i]) * 26;
+      row.set(o + who, 1);
+      row.set(o + 2 + 4 * who + s.face[i], 1);
       if (s.held[i] != kNone) {
-        o[23 + who] = 1;
-        o[14 + s.held[i]] = 1;
+        row.set(o + 23 + who, 1);
+        row.set(o + 14 + s.held[i], 1);
       }
     }
+  }
+  __device__ static void obs(const DevEnv& d, const State& s, int seat, uint8_t* row) {
+    ObsBytes w{row, 130};
+    obs_into(d, s, seat, w);
   }
 
   __device__ static uint32_t legal(const State&) { return 0x3Fu; }

@@ -64,6 +64,45 @@ struct PpoTcArgs {
   TrajPtrs traj;
 };
 
+// Per-policy block of the streamed tensor-core path (binary observations, hidden width H
+// = 256 or 512 for both layers).  W1 and W2 are cut into 8 KB chunks, each a [256][16]
+// bf16 slice (256 output rows, 16 inputs) in the canonical K-major layout, so that one
+// chunk is the B operand of one N = 256, K = 16 MMA:
+//   chunk nh * (KP / 16) + ks            W1 rows [256 nh, 256 nh + 256), inputs [16 ks, 16 ks + 16)
+//   n_l1 + nh * (H / 16) + ks            W2 likewise (inputs are layer-1 units)
+// Input column obs_dim of W1 holds b1 (the observation carries a constant 1 there).
+// Then W3 fp32 [H][NAP] (row k = the NAP outputs' weights of hidden unit k), b2 fp32 [H],
+// b3 fp32 [NAP].
+struct WideDims {
+  int32_t KP, H, NAP;      // padded input (a multiple of 16), hidden width, padded outputs
+  int32_t n_l1, n_l2;      // chunks of W1 and W2
+  uint32_t oW3, ob2, ob3;  // byte offsets
+  uint32_t pol_bytes;
+};
+constexpr uint32_t kWideChunk = 8192;
+
+// One launch = one step s of a cross-play batch (see xplay_tc.cuh).
+struct XpTcArgs {
+  Batch b;
+  WideDims w;
+  const uint8_t* tcw;      // [n_policies][pol_bytes]
+  int32_t n_ego, n_tm, P, max_steps, s;
+  int32_t ego_ids[kMaxXpIds];
+  int32_t tm_ids[kMaxXpIds];
+  uint32_t step0;
+  int64_t n_total;         // n_ego * n_tm * P
+  const uint32_t* st_in;   // SoA state [words][n_total]: after step s - 1
+  uint32_t* st_out;        // after step s (written by the owning tiles)
+  const uint8_t* act_in;   // [n_total][2] actions of step s - 1
+  uint8_t* act_out;        // [n_total][2] actions of step s
+  const uint8_t* alive_in; // [n_total]
+  uint8_t* alive_out;
+  int32_t* nsteps;         // [n_total] steps taken
+  float* returns;          // [n_total]
+  int32_t* steps;          // optional [n_total]
+  uint8_t* actions;        // optional [max_steps][n_total][2]
+};
+
 struct GroupArgs {
   Key key;
   int64_t n_envs;
@@ -134,6 +173,14 @@ AHT_DECLARE_ENV_LAUNCHERS(hanabi)
 // Tensor-core PPO rollout (rollout_lbf.cu): LBF grids whose padded observation fits
 // 256 bf16 columns of tensor memory.
 cudaError_t lbf_ppo_tc(const PpoTcArgs&, int grid, size_t smem, cudaStream_t);
+
+// Streamed tensor-core cross-play step (rollout_overcooked.cu, rollout_hanabi.cu).
+// grid = the launch's tiles (xp_tc_tiles), smem = xp_tc_smem_bytes.
+cudaError_t overcooked_xplay_tc(const XpTcArgs&, int grid, size_t smem, cudaStream_t);
+cudaError_t hanabi_xplay_tc(const XpTcArgs&, int grid, size_t smem, cudaStream_t);
+cudaError_t overcooked_xplay_tc_smem_limit(size_t smem);  // once per device, before launches
+cudaError_t hanabi_xplay_tc_smem_limit(size_t smem);
+size_t xp_tc_smem_bytes(const WideDims& w);
 
 // misc.cu
 cudaError_t launch_group(const GroupArgs&, cudaStream_t);

@@ -107,8 +107,9 @@ __device__ __forceinline__ int sample_row(const float* z, int K, uint32_t legal,
 }
 
 // The same sample for a compile-time action count, all in registers.
-template <int K>
-__device__ __forceinline__ int sample_k(const float (&z)[16], uint32_t legal, float u, float& logp) {
+template <int K, int N>
+__device__ __forceinline__ int sample_k(const float (&z)[N], uint32_t legal, float u, float& logp) {
+  static_assert(K <= N, "logit array shorter than the action count");
   float m = -INFINITY;
 #pragma unroll
   for (int k = 0; k < K; ++k)

@@ -1,7 +1,15 @@
 // rollout_overcooked.cu -- kernel instantiations for the overcooked rules.
 #include "env_overcooked.cuh"
 #include "rollout_impl.cuh"
+#include "xplay_tc.cuh"
 
 namespace aht {
 AHT_DEFINE_ENV_LAUNCHERS(overcooked, EnvOvercooked)
+
+cudaError_t overcooked_xplay_tc(const XpTcArgs& a, int grid, size_t smem, cudaStream_t s) {
+  return launch_xp_tc<EnvOvercooked>(a, grid, smem, s);
+}
+cudaError_t overcooked_xplay_tc_smem_limit(size_t smem) { return xp_tc_smem_limit<EnvOvercooked>(smem); }
+
+size_t xp_tc_smem_bytes(const WideDims& w) { return xp_tc_layout(w).total; }
 }  // namespace aht

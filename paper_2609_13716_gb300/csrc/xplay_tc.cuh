@@ -1,0 +1,496 @@
+// xplay_tc.cuh -- one step of a cross-play batch whose policies are wide bf16 MLPs
+// (hidden width 256 or 512: the Overcooked-style kitchen and Hanabi), with every layer
+// contraction on tcgen05 tensor cores and the weights streamed from L2.
+//
+// The batch holds n_ego x n_tm pairs of P envs each, env e = (i n_tm + j) P + k (ego i,
+// teammate j).  One launch is one step s of every env (J_AHT of Sec. 3 estimated per
+// pair, XP matrix of App. B).  A tile is up to 128 envs whose acting agent in seat
+// `seat` runs the same policy: seat 0 groups the envs of ego i (pairs (i, 0..n_tm-1),
+// contiguous), seat 1 those of teammate j (pairs (0..n_ego-1, j)).  The envs of a tile
+// change with the seat, so the env state goes through L2 between launches (the SoA
+// state, alive flag and actions are double-buffered by step parity):
+//   1. transition: the tile's envs take step s - 1 with the actions chosen by the
+//      previous launch (step 0: reset).  Each env has one owning tile that writes the
+//      new state, alive flag, step count and return (turn-based games: the tile of the
+//      seat acting at s; simultaneous games: the seat-0 tile; a seat-1 tile of a
+//      simultaneous game computes the same transition for its own use);
+//   2. the acting seat's binary observation -> bf16 A operand in shared memory (exact);
+//   3. L1 = [o 1] W1^T on tensor cores (N = 256 per instruction, b1 folded into W1);
+//   4. epilogue 1: h1 = tanh(L1), split h1 = hi + lo (two bf16) -> A operands of L2;
+//   5. L2 = hi W2^T + lo W2^T on tensor cores (fp32 accumulate in tensor memory);
+//   6. epilogue 2: h2 = tanh(L2 + b2) and z = W3 h2 + b3 on CUDA cores (fp32);
+//   7. masked inverse-CDF sample of the acting seat's action (Philox stream = seat).
+// Launch max_steps only applies the last transition.
+//
+// Warp roles (320 threads): warps 0-7 compute (thread r and r + 128 own env row r,
+// tensor-memory lane r; the halves split the columns), warp 8 issues the MMAs, warp 9
+// streams the 8 KB weight chunks of the tile's policy, in the order the MMAs consume
+// them, through a ring of shared-memory stages of several chunks each (one TMA bulk copy
+// and one full / empty mbarrier pair per stage).  Every wait is bounded; on expiry the CTA records kStatusTimeout, stops,
+// drains its MMAs and copies, frees tensor memory and exits.
+//
+// Tensor memory (512 columns), R0 = [0, 256), R1 = [256, 512):
+//   H = 256: L1 -> R0; epilogue 1 rewrites each 32-column block of R0 in place as
+//            16 columns hi | 16 columns lo; L2 -> R1.
+//   H = 512: L1 units [0, 256) -> R0, [256, 512) -> R1; epilogue 1 writes hi to shared
+//            memory (a [128][512] canonical A operand over the dead observation tile)
+//            and packs lo of all 512 units into R0; L2 runs as two N = 256 halves, each
+//            into R1 (the second after epilogue 2 has read the first).
+#pragma once
+#include "kernels.h"
+#include "mlp_simt.cuh"
+#include "rollout_impl.cuh"
+#include "tc_common.cuh"
+
+namespace aht {
+
+constexpr int kXpCompute = 256;
+constexpr int kXpThreads = 320;
+constexpr int kXpComputeBar = 1;
+constexpr int kXpMaxStages = 3;
+constexpr int kXpMaxChunksPerStage = 4;
+constexpr uint32_t kXpSmemBudget = 231424;  // opt-in maximum minus a margin for static data
+
+struct XpTcSmem {
+  uint32_t a_bytes;    // env states / observation tile / hi operand, W3 b2 b3, partials
+  uint32_t w3_off;     // W3, b2, b3 (bulk-copied once L1 is done), within the A region
+  uint32_t w3_bytes;
+  uint32_t stage_off;  // weight stages
+  uint32_t bits_off;   // per-row observation bits
+  uint32_t total;
+  int nst;             // stages
+  int spc;             // 8 KB chunks per stage (one bulk copy, one full / empty barrier pair)
+  int bit_words;       // 32-bit words per observation bit row
+};
+
+__host__ __device__ inline XpTcSmem xp_tc_layout(const WideDims& w) {
+  XpTcSmem L;
+  // L1: observation tile.  L2 and after: hi (H = 512) or the output partials, then W3.
+  const uint32_t obs = 128u * (uint32_t)w.KP * 2u;
+  const uint32_t hi = w.H == 512 ? 128u * 512u * 2u : 0u;
+  const uint32_t zp = 2u * 128u * (uint32_t)w.NAP * 4u;
+  L.w3_off = (uint32_t)align_up(hi > zp ? hi : zp, 1024);
+  L.w3_bytes = w.pol_bytes - w.oW3;
+  const uint32_t a = L.w3_off + L.w3_bytes > obs ? L.w3_off + L.w3_bytes : obs;
+  L.a_bytes = (uint32_t)align_up(a, 1024);
+  L.bit_words = (w.KP + 31) / 32;
+  const uint32_t bits = (uint32_t)align_up(128 * L.bit_words * 4, 1024);
+  // Stages are as large as two of them fit: each barrier completion of a bulk copy or an
+  // MMA commit reaches its waiter some 500 cycles later (measured on GB300), so the bytes
+  // moved per completion, not the number of copies in flight, set the stream's rate.
+  const int slots = (int)((kXpSmemBudget - L.a_bytes - bits) / kWideChunk);
+  L.spc = slots / 2 > kXpMaxChunksPerStage ? kXpMaxChunksPerStage : slots / 2;
+  L.nst = slots / L.spc > kXpMaxStages ? kXpMaxStages : slots / L.spc;
+  L.stage_off = L.a_bytes;
+  L.bits_off = L.stage_off + (uint32_t)(L.nst * L.spc) * kWideChunk;
+  L.total = L.bits_off + bits;
+  return L;
+}
+
+// Two binary features (bits 0, 1 of x) as a bf16 pair: 0 or 1.0 (0x3F80) each.
+__device__ __forceinline__ uint32_t bits_to_bf16x2(uint32_t x) {
+  return ((x & 1u) * 0x3F80u) | ((x & 2u) * 0x1FC00000u);
+}
+
+template <class Env>
+__global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) {
+  using State = typename Env::State;
+  constexpr int NA = Env::kNumActions;
+  constexpr int NAP = (NA + 3) / 4 * 4;
+  constexpr bool kTurn = Env::kTurnBased;
+  extern __shared__ __align__(16) uint8_t smem[];  // the no-swizzle operands need 16 B
+  __shared__ __align__(8) uint64_t full_bar[kXpMaxStages], empty_bar[kXpMaxStages];
+  __shared__ __align__(8) uint64_t obs_bar, acc_bar[3], epi1_bar, epi2_bar, w3_bar, drain_bar;
+  __shared__ uint32_t tmem_slot;
+  __shared__ volatile int abort_flag;
+  bool w3_issued = false;  // (MMA lane) the W3 copy is in flight or done
+  int next_chunk = 0;      // (producer lane) stages issued
+
+  const WideDims& w = a.w;
+  const XpTcSmem L = xp_tc_layout(w);
+  const int NST = L.nst;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, row = tid & 127;
+  const int half = (warp >> 2) & 1;
+
+  // ---- the tile: seat, acting policy, rows ------------------------------------------
+  const int G0 = a.n_tm * a.P, G1 = a.n_ego * a.P;
+  const int T0 = (G0 + 127) / 128, T1 = (G1 + 127) / 128;
+  int seat, t = blockIdx.x;
+  if (kTurn) {
+    seat = a.s & 1;
+  } else {
+    seat = t < a.n_ego * T0 ? 0 : 1;
+    if (seat) t -= a.n_ego * T0;
+  }
+  const int Tn = seat ? T1 : T0, G = seat ? G1 : G0;
+  const int group = t / Tn, q0 = (t - group * Tn) * 128;
+  const int count = min(128, G - q0);
+  const int pol = seat ? a.tm_ids[group] : a.ego_ids[group];
+  const bool owner = kTurn || seat == 0;
+  auto env_of = [&](int r) -> int64_t {
+    const int q = q0 + r;
+    if (seat == 0) return (int64_t)group * G0 + q;
+    const int i = q / a.P, k = q - i * a.P;
+    return ((int64_t)i * a.n_tm + group) * a.P + k;
+  };
+
+  uint8_t* const sA = smem;
+  uint8_t* const sStage = smem + L.stage_off;
+  uint32_t* const sBits = reinterpret_cast<uint32_t*>(smem + L.bits_off);
+  const uint8_t* const pblk = a.tcw + (int64_t)pol * w.pol_bytes;
+  const uint32_t gt = a.step0 + (uint32_t)a.s;
+
+  // ---- 1. transition of step s - 1, and this step's observation bits -----------------
+  bool alive = false;
+  float u_act = 0.0f;
+  uint32_t legal = 0xFFFFFFFFu >> (32 - NA);
+  int64_t e = -1;
+  if (tid < 128) {
+    uint32_t* bits = sBits + row * L.bit_words;
+    if (row < count) {
+      e = env_of(row);
+      // the state lives in shared memory (the A region is free until the observation is
+      // expanded): per-thread local copies would spill past the small L1 left beside
+      // this kernel's shared memory
+      State& s = reinterpret_cast<State*>(sA)[row];
+      int nst = 0;
+      if (a.s == 0) {
+        Env::reset(a.b.env, a.b.key, (uint32_t)e, a.step0, s);
+        alive = true;
+      } else {
+        load_state(a.st_in, a.n_total, e, s);
+        alive = a.alive_in[e] != 0;
+        if (owner) nst = a.nsteps[e];
+        if (alive) {
+          const int actor = kTurn ? ((a.s - 1) & 1) : -1;
+          const int a0 = (actor < 0 || actor == 0) ? a.act_in[2 * e] : 0;
+          const int a1 = (actor < 0 || actor == 1) ? a.act_in[2 * e + 1] : 0;
+          if (owner && a.actions) {
+            uint8_t* rec = a.actions + ((int64_t)(a.s - 1) * a.n_total + e) * 2;
+            rec[0] = (actor < 0 || actor == 0) ? (uint8_t)a0 : 255;
+            rec[1] = (actor < 0 || actor == 1) ? (uint8_t)a1 : 255;
+          }
+          float r0, r1, team;
+          const int done = Env::step(a.b.env, s, a0, a1, r0, r1, team);
+          if (done < 0) {
+            if (owner) atomicOr(a.b.status, kStatusIllegalAction);
+            alive = false;
+          } else {
+            nst += 1;
+            if (done) alive = false;
+          }
+        }
+      }
+      if (owner) {
+        store_state(a.st_out, a.n_total, e, s);
+        a.alive_out[e] = (uint8_t)alive;
+        a.nsteps[e] = nst;
+        a.returns[e] = Env::ret(s);
+        if (a.steps) a.steps[e] = nst;
+      }
+      if (alive && a.s < a.max_steps) {
+        ObsBits wr{bits, L.bit_words};
+        Env::obs_into(a.b.env, s, seat, wr);
+        wr.set(a.b.env.obs_dim, 1);  // the constant input that carries b1
+        if (kTurn) {
+          legal = Env::legal(s);
+          if (Env::actor(s) != seat) atomicOr(a.b.status, kStatusActorMismatch);
+        }
+        u_act = u01(draw0(a.b.key, (uint32_t)e, gt, kStreamAct0 + seat));
+      } else {
+        for (int i = 0; i < L.bit_words; ++i) bits[i] = 0u;
+      }
+    } else {
+      for (int i = 0; i < L.bit_words; ++i) bits[i] = 0u;
+    }
+  }
+  if (!__syncthreads_or(alive) || a.s == a.max_steps) return;  // nothing left to act
+
+  if (tid == 0) {
+    for (int i = 0; i < NST; ++i) {
+      tc::mbar_init(&full_bar[i], 1);
+      tc::mbar_init(&empty_bar[i], 1);
+    }
+    tc::mbar_init(&obs_bar, kXpCompute);
+    for (int i = 0; i < 3; ++i) tc::mbar_init(&acc_bar[i], 1);
+    tc::mbar_init(&epi1_bar, kXpCompute);
+    tc::mbar_init(&epi2_bar, kXpCompute);
+    tc::mbar_init(&w3_bar, 1);
+    tc::mbar_init(&drain_bar, 1);
+    tc::mbar_init_fence();
+    abort_flag = 0;
+  }
+  if (warp == 0) tc::tmem_alloc(&tmem_slot, 512);
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = tmem_slot;
+  const int n_chunks = w.n_l1 + w.n_l2;
+
+  const int SPC = L.spc, n_stages = (n_chunks + SPC - 1) / SPC;
+  const uint32_t stage_bytes = (uint32_t)SPC * kWideChunk;
+
+  if (warp == 9) {
+    // ============================ weight producer ===================================
+    if (lane == 0) {
+      int k = 0;
+      bool ok = true;
+      const uint64_t keep = tc::l2_evict_last();  // every step re-reads the population
+      for (; k < n_stages; ++k) {
+        const int slot = k % NST;
+        const uint32_t use = (uint32_t)(k / NST);
+        if (use > 0) {
+          ok = false;
+          for (int tries = 0; tries < 1000 && !ok && !abort_flag; ++tries)
+            ok = tc::mbar_wait(&empty_bar[slot], (use - 1) & 1u, 2000000ull);
+          if (!ok) break;
+        }
+        const uint32_t bytes = (uint32_t)min(SPC, n_chunks - k * SPC) * kWideChunk;
+        tc::mbar_expect_tx(&full_bar[slot], bytes);
+        tc::bulk_g2s_hint(sStage + slot * stage_bytes, pblk + (int64_t)k * stage_bytes, bytes, &full_bar[slot], keep);
+      }
+      if (!ok) abort_flag = 1;
+      next_chunk = k;  // stages issued
+    }
+  } else if (warp == 8) {
+    // ================================ MMA issue =====================================
+    if (lane == 0) {
+      const uint32_t idesc = tc::idesc_bf16(128, 256);
+      auto wait_for = [&](uint64_t* bar, uint32_t parity) {
+        bool ok = false;
+        for (int tries = 0; tries < 1000 && !ok && !abort_flag; ++tries)
+          ok = tc::mbar_wait(bar, parity, 2000000ull);
+        if (ok) tc::fence_after_sync();
+        return ok;
+      };
+      int c = 0;
+      auto chunk = [&](uint64_t& desc) {  // waits for weight chunk c, returns its descriptor
+        const int k = c / SPC, slot = k % NST, sub = c - k * SPC;
+        if (sub == 0 && !wait_for(&full_bar[slot], (uint32_t)(k / NST) & 1u)) return false;
+        desc = tc::smem_desc(tc::smem_u32(sStage + slot * stage_bytes + sub * kWideChunk), 128u, 256u);
+        return true;
+      };
+      auto release = [&]() {  // the stage is free once the MMAs reading its last chunk finish
+        if (c % SPC == SPC - 1 || c == n_chunks - 1) tc::commit(&empty_bar[(c / SPC) % NST]);
+        ++c;
+      };
+      bool ok = wait_for(&obs_bar, 0);
+      const uint32_t aobs = tc::smem_u32(sA), sbo_obs = (uint32_t)(w.KP / 8) * 128u;
+      for (int nh = 0; ok && nh < w.H / 256; ++nh)
+        for (int ks = 0; ok && ks < w.KP / 16; ++ks) {
+          uint64_t bd;
+          if (!(ok = chunk(bd))) break;
+          tc::mma_ss(tmem + 256u * nh, tc::smem_desc(aobs + 256u * ks, 128u, sbo_obs), bd, idesc, ks > 0);
+          release();
+        }
+      if (ok) tc::commit(&acc_bar[0]);
+      // once L1 has read the observation tile, W3 b2 b3 go to the A region's tail
+      if (ok) ok = wait_for(&acc_bar[0], 0);
+      if (ok) {
+        tc::mbar_expect_tx(&w3_bar, L.w3_bytes);
+        tc::bulk_g2s(sA + L.w3_off, pblk + w.oW3, L.w3_bytes, &w3_bar);
+        w3_issued = true;
+      }
+      if (ok) ok = wait_for(&epi1_bar, 0);
+      if (ok && w.H == 256) {
+        for (int ks = 0; ok && ks < 16; ++ks) {
+          uint64_t bd;
+          if (!(ok = chunk(bd))) break;
+          const uint32_t hi = tmem + 32u * (ks >> 1) + 8u * (ks & 1);
+          tc::mma_ts(tmem + 256u, hi, bd, idesc, ks > 0);
+          tc::mma_ts(tmem + 256u, hi + 16u, bd, idesc, 1u);
+          release();
+        }
+        if (ok) tc::commit(&acc_bar[1]);
+      } else if (ok) {
+        const uint32_t ahi = tc::smem_u32(sA);
+        for (int nh = 0; ok && nh < 2; ++nh) {
+          if (nh == 1 && !(ok = wait_for(&epi2_bar, 0))) break;
+          for (int ks = 0; ok && ks < 32; ++ks) {
+            uint64_t bd;
+            if (!(ok = chunk(bd))) break;
+            tc::mma_ss(tmem + 256u, tc::smem_desc(ahi + 256u * ks, 128u, 64u * 128u), bd, idesc, ks > 0);
+            tc::mma_ts(tmem + 256u, tmem + 8u * ks, bd, idesc, 1u);
+            release();
+          }
+          if (ok) tc::commit(&acc_bar[1 + nh]);
+        }
+      }
+      if (!ok) abort_flag = 1;
+    }
+  } else {
+    // ============================== compute warps ===================================
+    bool bad = false;
+    const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+    const uint32_t R0 = tmem + lane_base, R1 = tmem + 256u + lane_base;
+    auto wait_acc = [&](uint64_t* bar) {
+      if (!bad && !tc::mbar_wait(bar, 0)) bad = true;
+      bad = __any_sync(0xFFFFFFFFu, bad);
+      tc::fence_after_sync();
+    };
+    auto sync_or = [&]() { return tc::bar_or(kXpComputeBar, kXpCompute, bad || abort_flag); };
+
+    // 2. observation bits -> bf16 A operand (canonical K-major [128][KP]); each half of
+    //    the threads expands half of the row's 8-feature chunks
+    {
+      const uint32_t* bits = sBits + row * L.bit_words;
+      const int nkb = w.KP / 8, split = (nkb + 1) / 2;
+      const int kb0 = half ? split : 0, kb1 = half ? nkb : split;
+      for (int kb = kb0; kb < kb1; ++kb) {
+        const uint32_t byte = (bits[kb >> 2] >> (8 * (kb & 3))) & 0xFFu;
+        uint4 v;
+        v.x = bits_to_bf16x2(byte);
+        v.y = bits_to_bf16x2(byte >> 2);
+        v.z = bits_to_bf16x2(byte >> 4);
+        v.w = bits_to_bf16x2(byte >> 6);
+        *reinterpret_cast<uint4*>(sA + tc::canon_offset(row, 8 * kb, w.KP)) = v;
+      }
+      tc::fence_proxy_async();
+      tc::mbar_arrive(&obs_bar);
+    }
+
+    // 4. epilogue 1
+    wait_acc(&acc_bar[0]);
+    if (!bad && w.H == 256) {
+      for (int c0 = 128 * half; c0 < 128 * half + 128; c0 += 32) {
+        uint32_t v[32], hi[16], lo[16];
+        tc::ld_x32(R0 + c0, v);
+        tc::wait_ld();
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+          tc::split_bf16x2(tc::tanh_ex2(__uint_as_float(v[2 * j])), tc::tanh_ex2(__uint_as_float(v[2 * j + 1])),
+                           hi[j], lo[j]);
+        tc::st_x16(R0 + c0, hi);
+        tc::st_x16(R0 + c0 + 16, lo);
+      }
+      tc::wait_st();
+    } else if (w.H == 512) {
+      // half 0: units [0, 256) from R0; half 1: units [256, 512) from R1.  hi -> shared
+      // memory; lo -> packed in place at the start of the region read
+      const uint32_t src = half ? R1 : R0;
+      for (int cb = 0; cb < 8 && !bad; ++cb) {
+        uint32_t v[32], hi[16], lo[16];
+        tc::ld_x32(src + 32u * cb, v);
+        tc::wait_ld();
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+          tc::split_bf16x2(tc::tanh_ex2(__uint_as_float(v[2 * j])), tc::tanh_ex2(__uint_as_float(v[2 * j + 1])),
+                           hi[j], lo[j]);
+        const int u0 = 256 * half + 32 * cb;
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          *reinterpret_cast<uint4*>(sA + tc::canon_offset(row, u0 + 8 * q, 512)) =
+              make_uint4(hi[4 * q], hi[4 * q + 1], hi[4 * q + 2], hi[4 * q + 3]);
+        tc::st_x16(src + 16u * cb, lo);
+      }
+      tc::wait_st();
+      tc::fence_before_sync();
+      bad = sync_or();  // half 0 has read R0 [128, 256) before half 1 writes there
+      tc::fence_after_sync();
+      if (!bad && half) {
+        for (int cb = 0; cb < 4; ++cb) {
+          uint32_t v[32];
+          tc::ld_x32(R1 + 32u * cb, v);
+          tc::wait_ld();
+          tc::st_x32(R0 + 128u + 32u * cb, v);
+        }
+        tc::wait_st();
+      }
+    }
+    tc::fence_proxy_async();  // hi written by ordinary stores, read by the tensor cores
+    tc::fence_before_sync();
+    tc::mbar_arrive(&epi1_bar);
+
+    // 6. epilogue 2: this half's columns of each N = 256 block of L2
+    const float* W3 = reinterpret_cast<const float*>(sA + L.w3_off);
+    const float* b2 = reinterpret_cast<const float*>(sA + L.w3_off + (w.ob2 - w.oW3));
+    const float* b3 = reinterpret_cast<const float*>(sA + L.w3_off + (w.ob3 - w.oW3));
+    if (!bad && !tc::mbar_wait(&w3_bar, 0)) bad = true;
+    bad = __any_sync(0xFFFFFFFFu, bad);
+    uint64_t z2[NAP / 2];
+#pragma unroll
+    for (int o = 0; o < NAP / 2; ++o) z2[o] = 0ull;
+    const int n_blocks = w.H / 256;
+    for (int nh = 0; nh < n_blocks; ++nh) {
+      wait_acc(&acc_bar[1 + nh]);
+      if (bad) break;
+      for (int c0 = 128 * half; c0 < 128 * half + 128; c0 += 32) {
+        uint32_t v[32];
+        tc::ld_x32(R1 + c0, v);
+        tc::wait_ld();
+        const int u0 = 256 * nh + c0;
+#pragma unroll 8
+        for (int j = 0; j < 32; ++j) {
+          const float h = tc::tanh_ex2(__uint_as_float(v[j]) + b2[u0 + j]);
+          const uint64_t hh = tc::f2_pack(h, h);
+          const ulonglong2* wr = reinterpret_cast<const ulonglong2*>(W3 + (int64_t)(u0 + j) * NAP);
+#pragma unroll
+          for (int o = 0; o < NAP / 4; ++o) {
+            const ulonglong2 wv = wr[o];
+            z2[2 * o] = tc::f2_fma(hh, wv.x, z2[2 * o]);
+            z2[2 * o + 1] = tc::f2_fma(hh, wv.y, z2[2 * o + 1]);
+          }
+        }
+      }
+      if (nh == 0 && n_blocks == 2) {
+        tc::fence_before_sync();
+        tc::mbar_arrive(&epi2_bar);  // R1 may take the second half
+      }
+    }
+    // partial sums of the two halves -> shared memory (the A region is dead now)
+    float* zpart = reinterpret_cast<float*>(sA);
+    if (!bad) {
+      uint64_t* dst = reinterpret_cast<uint64_t*>(zpart + (half * 128 + row) * NAP);
+#pragma unroll
+      for (int o = 0; o < NAP / 2; ++o) dst[o] = z2[o];
+    }
+    bad = sync_or();
+
+    // 7. sample the acting seat's action (half 0 threads, live rows)
+    if (!bad && tid < 128 && alive) {
+      float z[NAP];
+#pragma unroll
+      for (int o = 0; o < NAP; ++o)
+        z[o] = (zpart[row * NAP + o] + zpart[(128 + row) * NAP + o]) + b3[o];
+      float lp;
+      const int act = sample_k<NA>(z, legal, u_act, lp);
+      a.act_out[2 * e + seat] = (uint8_t)act;
+    }
+    if (bad) abort_flag = 1;
+  }
+
+  // ---- drain: every MMA and copy of this CTA completes (bounded), free tensor memory ---
+  tc::fence_before_sync();
+  __syncthreads();
+  if (tid == 0 && abort_flag) atomicOr(a.b.status, kStatusTimeout);
+  if (warp == 8 && lane == 0) {
+    tc::commit(&drain_bar);
+    tc::mbar_wait(&drain_bar, 0);
+    if (w3_issued) tc::mbar_wait(&w3_bar, 0);
+  }
+  if (warp == 9 && lane == 0 && abort_flag) {
+    // the MMA lane consumed (waited for) every stage unless the CTA aborted; then the
+    // copies that may be in flight land before the CTA leaves (bounded waits)
+    for (int d = next_chunk - 1; d >= 0 && d >= next_chunk - NST; --d)
+      tc::mbar_wait(&full_bar[d % NST], (uint32_t)(d / NST) & 1u);
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(tmem, 512);
+  }
+}
+
+template <class Env>
+cudaError_t launch_xp_tc(const XpTcArgs& a, int grid, size_t smem, cudaStream_t s) {
+  xp_tc_kernel<Env><<<grid, kXpThreads, smem, s>>>(a);
+  return cudaGetLastError();
+}
+
+template <class Env>
+cudaError_t xp_tc_smem_limit(size_t smem) {
+  return cudaFuncSetAttribute(xp_tc_kernel<Env>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+}
+
+}  // namespace aht
