@@ -227,10 +227,11 @@ aht_status aht_step_forced(aht_ctx* ctx, const uint8_t* actions, const aht_step_
 aht_status aht_policy_forward(aht_ctx* ctx, int32_t policy, const uint8_t* obs, int64_t n,
                               float* out);
 
-/* The tanh of the tensor-core epilogue, elementwise: y[i] = tanh(x[i]) for device f32
- * arrays of n elements (computed as sign(x)(1 - e)/(1 + e), e = exp(-2|x|), with the
- * hardware exp2 and reciprocal approximations; absolute error below 1e-6).  Stateless;
- * enqueued on cuda_stream. */
+/* The tanh of the tensor-core epilogues, elementwise: y[i] = tanh(x[i]) for device f32
+ * arrays of n elements, computed for the pairs (x[2j], x[2j + 1]) as 1 - 2 / (1 + e),
+ * e = exp(2x), with the hardware exp2 and reciprocal approximations and packed fp32x2
+ * arithmetic; absolute error below 1e-6, tanh(0) = 0 exactly.  Stateless; enqueued on
+ * cuda_stream. */
 aht_status aht_debug_tanh(const float* x, float* y, int64_t n, void* cuda_stream);
 
 /* Checkpoint of the PPO env state, the seed and the step counter into a host buffer.

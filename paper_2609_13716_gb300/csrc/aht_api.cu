@@ -328,9 +328,9 @@ aht_status pack_policy_tc(const MlpDims& m, const TcDims& t, const void* const* 
         const int64_t i = (int64_t)n * ins[l] + k;
         if (l == 0) std::memcpy(dst + t.oW1 + tc::canon_offset(n, k, t.KP), &w[i], 2);
         if (l == 1) std::memcpy(dst + t.oW2 + tc::canon_offset(n, k, m.H0), &w[i], 2);
-        if (l == 2) {
+        if (l == 2) {  // hidden units in pairs: [k / 2][output][k % 2]
           const float f = to_f32(src, i, AHT_BF16);
-          std::memcpy(dst + t.oW3 + 4 * (k * 8 + n), &f, 4);
+          std::memcpy(dst + t.oW3 + 4 * (((k / 2) * 8 + n) * 2 + (k % 2)), &f, 4);
         }
       }
     if (!read_host(b[l], (size_t)outs[l] * 2, tmp, &src)) return fail(AHT_ECUDA, "copying biases failed");
@@ -371,9 +371,9 @@ aht_status pack_policy_wide(const MlpDims& m, const WideDims& w, const void* con
         const int64_t i = (int64_t)n * ins[l] + k;
         if (l == 0) std::memcpy(w1_at(n, k), &wv[i], 2);
         if (l == 1) std::memcpy(w2_at(n, k), &wv[i], 2);
-        if (l == 2 && n < m.NA) {
+        if (l == 2 && n < m.NA) {  // hidden units in pairs: [k / 2][output][k % 2]
           const float f = to_f32(src, i, AHT_BF16);
-          std::memcpy(dst + w.oW3 + 4 * ((size_t)k * w.NAP + n), &f, 4);
+          std::memcpy(dst + w.oW3 + 4 * (((size_t)(k / 2) * w.NAP + n) * 2 + (k % 2)), &f, 4);
         }
       }
     if (!read_host(b[l], (size_t)outs[l] * 2, tmp, &src)) return fail(AHT_ECUDA, "copying biases failed");

@@ -41,8 +41,9 @@ struct PpoArgs {
 //   W1 [H0][KP] bf16, canonical K-major (see tc_common.cuh); column obs_dim holds b1
 //      (the observation tile carries a constant 1 there),
 //   W2 [H1][H0] bf16, canonical K-major,
-//   W3 fp32 [H1][8], transposed: row k holds W3[0..7][k] (outputs past n_actions, and the
-//      value row when absent, are zero),
+//   W3 fp32 [H1 / 2][8][2]: entry (p, o, i) = W3[o][2p + i], hidden units in pairs
+//      for packed fp32x2 FMAs (outputs past n_actions, and the value row when absent,
+//      are zero),
 //   b2 fp32 [H1], b3 fp32 [8].
 struct TcDims {
   int32_t KP, H0, H1;      // padded obs dim (> obs_dim), hidden sizes
@@ -71,8 +72,8 @@ struct PpoTcArgs {
 //   chunk nh * (KP / 16) + ks            W1 rows [256 nh, 256 nh + 256), inputs [16 ks, 16 ks + 16)
 //   n_l1 + nh * (H / 16) + ks            W2 likewise (inputs are layer-1 units)
 // Input column obs_dim of W1 holds b1 (the observation carries a constant 1 there).
-// Then W3 fp32 [H][NAP] (row k = the NAP outputs' weights of hidden unit k), b2 fp32 [H],
-// b3 fp32 [NAP].
+// Then W3 fp32 [H / 2][NAP][2] (entry (p, o, i) = W3[o][2p + i]: hidden units in pairs
+// for packed fp32x2 FMAs), b2 fp32 [H], b3 fp32 [NAP].
 struct WideDims {
   int32_t KP, H, NAP;      // padded input (a multiple of 16), hidden width, padded outputs
   int32_t n_l1, n_l2;      // chunks of W1 and W2

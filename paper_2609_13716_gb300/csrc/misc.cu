@@ -129,12 +129,18 @@ cudaError_t launch_policy(const PolicyArgs& a, int grid, size_t smem, cudaStream
 
 // ---- the tensor-core epilogue's tanh, standalone (test hook) ---------------------------
 __global__ void tanh_probe_kernel(const float* __restrict__ x, float* __restrict__ y, int64_t n) {
-  const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (i < n) y[i] = tc::tanh_ex2(x[i]);
+  const int64_t i = 2 * (blockIdx.x * (int64_t)blockDim.x + threadIdx.x);  // elements i, i + 1
+  if (i >= n) return;
+  const float x1 = i + 1 < n ? x[i + 1] : 0.0f;
+  float y0, y1;
+  tc::f2_unpack(tc::tanh2(tc::f2_pack(x[i], x1)), y0, y1);
+  y[i] = y0;
+  if (i + 1 < n) y[i + 1] = y1;
 }
 
 cudaError_t launch_tanh_probe(const float* x, float* y, int64_t n, cudaStream_t s) {
-  tanh_probe_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(x, y, n);
+  const int64_t pairs = (n + 1) / 2;
+  tanh_probe_kernel<<<(unsigned)((pairs + 255) / 256), 256, 0, s>>>(x, y, n);
   return cudaGetLastError();
 }
 

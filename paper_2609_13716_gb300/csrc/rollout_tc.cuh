@@ -186,8 +186,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         uint32_t hi[16], lo[16];
 #pragma unroll
         for (int j = 0; j < 16; ++j)
-          tc::split_bf16x2(tc::tanh_ex2(__uint_as_float(v[2 * j])),
-                           tc::tanh_ex2(__uint_as_float(v[2 * j + 1])), hi[j], lo[j]);
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]))),
+                             hi[j], lo[j]);
 #pragma unroll
         for (int j = 0; j < 32; j += 4) {
           const float4 bb = *reinterpret_cast<const float4*>(b2 + c0 + j);
@@ -202,31 +202,39 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       operand_ready(ag, 1);
     };
     // epilogue 2: h2 = tanh(D) and this half's partial z = sum_k W3[:, k] h2[k], stored
-    // for the half that samples the agent
+    // for the half that samples the agent.  Hidden units go in pairs (2p, 2p + 1): the
+    // packed FMA of output o accumulates W3[o][2p] h2[2p] and W3[o][2p + 1] h2[2p + 1].
     auto epilogue2 = [&](int ag) {
       const int H = d.H1;
       const uint32_t Q = tmem + (uint32_t)(ag * 256 + 128) + lane_base;
       const float* W3 = reinterpret_cast<const float*>(pol_block(ag) + d.oW3);
-      uint64_t z2[4] = {0, 0, 0, 0};  // output pairs (0,1) (2,3) (4,5) (6,7), fp32 each
+      uint64_t acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
       for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 32) {
         uint32_t v[32];
         tc::ld_x32(Q + c0, v);
         tc::wait_ld();
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const float h = tc::tanh_ex2(__uint_as_float(v[j]));
-          const uint64_t hh = tc::f2_pack(h, h);
-          const ulonglong2 wa = *reinterpret_cast<const ulonglong2*>(W3 + (c0 + j) * 8);
-          const ulonglong2 wb = *reinterpret_cast<const ulonglong2*>(W3 + (c0 + j) * 8 + 4);
-          z2[0] = tc::f2_fma(hh, wa.x, z2[0]);
-          z2[1] = tc::f2_fma(hh, wa.y, z2[1]);
-          z2[2] = tc::f2_fma(hh, wb.x, z2[2]);
-          z2[3] = tc::f2_fma(hh, wb.y, z2[3]);
+        for (int j = 0; j < 32; j += 2) {
+          const uint64_t h = tc::tanh2(tc::f2_pack(__uint_as_float(v[j]), __uint_as_float(v[j + 1])));
+          const ulonglong2* wp = reinterpret_cast<const ulonglong2*>(W3 + (c0 + j) * 8);
+#pragma unroll
+          for (int o = 0; o < 8; o += 2) {
+            const ulonglong2 ww = wp[o / 2];
+            acc[o] = tc::f2_fma(h, ww.x, acc[o]);
+            acc[o + 1] = tc::f2_fma(h, ww.y, acc[o + 1]);
+          }
         }
       }
-      ulonglong2* dst = reinterpret_cast<ulonglong2*>(zpart + ((ag * 2 + half) * 128 + row) * 8);
-      dst[0] = make_ulonglong2(z2[0], z2[1]);
-      dst[1] = make_ulonglong2(z2[2], z2[3]);
+      float z8[8];
+#pragma unroll
+      for (int o = 0; o < 8; ++o) {
+        float e, f;
+        tc::f2_unpack(acc[o], e, f);
+        z8[o] = e + f;
+      }
+      float4* dst = reinterpret_cast<float4*>(zpart + ((ag * 2 + half) * 128 + row) * 8);
+      dst[0] = make_float4(z8[0], z8[1], z8[2], z8[3]);
+      dst[1] = make_float4(z8[4], z8[5], z8[6], z8[7]);
     };
     // full logits of agent ag: (half-0 partial + half-1 partial) + b3
     auto logits = [&](int ag, float (&z)[16]) {

@@ -226,15 +226,6 @@ __device__ __forceinline__ float rcp_approx(float x) {
   return y;
 }
 
-// tanh from the identity tanh(x) = sign(x) (1 - e) / (1 + e), e = exp(-2|x|)
-// = 2^(-2|x| / ln 2), with the hardware approximations of 2^x and 1/x (relative errors
-// ~2^-22 each): six instructions, absolute error below 1e-6 over the whole line.
-__device__ __forceinline__ float tanh_ex2(float x) {
-  const float e = ex2_approx(fabsf(x) * -2.8853900817779268f);
-  const float r = rcp_approx(1.0f + e);
-  return copysignf(fmaf(-e, r, r), x);
-}
-
 // Bytes b0, b1 of a 32-bit word (unsigned 0..255) as a packed bf16x2 (b0 low), without
 // integer-to-float conversion instructions: 0x4B000000 | b is the float 2^23 + b, so
 // subtracting 2^23 gives b exactly; a value below 2^8 is exact in bf16, whose bits are
@@ -265,13 +256,40 @@ __device__ __forceinline__ uint64_t f2_sub(uint64_t a, uint64_t b) {
   return d;
 }
 
-// Split h = hi + lo into two bf16 (hi = round(h), lo = round(h - hi)) for a pair of
-// values; the difference h - hi is exact in fp32.
-__device__ __forceinline__ void split_bf16x2(float h0, float h1, uint32_t& hi, uint32_t& lo) {
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+// tanh of a pair from tanh(x) = 1 - 2 / (1 + e), e = exp(2x) = 2^(2x / ln 2): the
+// hardware exp2 and reciprocal approximations on each value, the rest as packed fp32x2
+// arithmetic.  Saturates by itself (e = inf gives 1, e = 0 gives -1), 0 maps to 0
+// exactly (1 / 2 is exact); absolute error below 1e-6 over the whole line.
+__device__ __forceinline__ uint64_t tanh2(uint64_t x) {
+  const uint64_t k = 0x4038AA3B4038AA3Bull;    // 2 / ln 2 = 2.8853900... in each half
+  const uint64_t one = 0x3F8000003F800000ull;  // 1.0f, 1.0f
+  const uint64_t m2 = 0xC0000000C0000000ull;   // -2.0f, -2.0f
+  float a, b;
+  f2_unpack(f2_mul(x, k), a, b);
+  float ea = ex2_approx(a), eb = ex2_approx(b);
+  f2_unpack(f2_add(f2_pack(ea, eb), one), a, b);
+  return f2_fma(f2_pack(rcp_approx(a), rcp_approx(b)), m2, one);
+}
+
+// Split a packed pair h = hi + lo into two bf16 (hi = round(h), lo = round(h - hi));
+// the difference h - hi is exact in fp32.
+__device__ __forceinline__ void split_bf16x2_p(uint64_t h, uint32_t& hi, uint32_t& lo) {
+  float h0, h1;
+  f2_unpack(h, h0, h1);
   hi = pack_bf16(h0, h1);
   float r0, r1;
-  f2_unpack(f2_sub(f2_pack(h0, h1), f2_pack(__uint_as_float(hi << 16), __uint_as_float(hi & 0xFFFF0000u))),
-            r0, r1);
+  f2_unpack(f2_sub(h, f2_pack(__uint_as_float(hi << 16), __uint_as_float(hi & 0xFFFF0000u))), r0, r1);
   lo = pack_bf16(r0, r1);
 }
 

@@ -358,8 +358,8 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
         tc::wait_ld();
 #pragma unroll
         for (int j = 0; j < 16; ++j)
-          tc::split_bf16x2(tc::tanh_ex2(__uint_as_float(v[2 * j])), tc::tanh_ex2(__uint_as_float(v[2 * j + 1])),
-                           hi[j], lo[j]);
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]))),
+                             hi[j], lo[j]);
         tc::st_x16(R0 + c0, hi);
         tc::st_x16(R0 + c0 + 16, lo);
       }
@@ -374,8 +374,8 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
         tc::wait_ld();
 #pragma unroll
         for (int j = 0; j < 16; ++j)
-          tc::split_bf16x2(tc::tanh_ex2(__uint_as_float(v[2 * j])), tc::tanh_ex2(__uint_as_float(v[2 * j + 1])),
-                           hi[j], lo[j]);
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]))),
+                             hi[j], lo[j]);
         const int u0 = 256 * half + 32 * cb;
 #pragma unroll
         for (int q = 0; q < 4; ++q)
@@ -407,9 +407,11 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
     const float* b3 = reinterpret_cast<const float*>(sA + L.w3_off + (w.ob3 - w.oW3));
     if (!bad && !tc::mbar_wait(&w3_bar, 0)) bad = true;
     bad = __any_sync(0xFFFFFFFFu, bad);
-    uint64_t z2[NAP / 2];
+    // hidden units in pairs (2p, 2p + 1): the packed FMA of output o accumulates
+    // W3[o][2p] h2[2p] and W3[o][2p + 1] h2[2p + 1] in its two halves
+    uint64_t acc[NAP];
 #pragma unroll
-    for (int o = 0; o < NAP / 2; ++o) z2[o] = 0ull;
+    for (int o = 0; o < NAP; ++o) acc[o] = 0ull;
     const int n_blocks = w.H / 256;
     for (int nh = 0; nh < n_blocks; ++nh) {
       wait_acc(&acc_bar[1 + nh]);
@@ -419,16 +421,16 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
         tc::ld_x32(R1 + c0, v);
         tc::wait_ld();
         const int u0 = 256 * nh + c0;
-#pragma unroll 8
-        for (int j = 0; j < 32; ++j) {
-          const float h = tc::tanh_ex2(__uint_as_float(v[j]) + b2[u0 + j]);
-          const uint64_t hh = tc::f2_pack(h, h);
+#pragma unroll 4
+        for (int j = 0; j < 32; j += 2) {
+          const uint64_t bb = *reinterpret_cast<const uint64_t*>(b2 + u0 + j);
+          const uint64_t h = tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(v[j]), __uint_as_float(v[j + 1])), bb));
           const ulonglong2* wr = reinterpret_cast<const ulonglong2*>(W3 + (int64_t)(u0 + j) * NAP);
 #pragma unroll
-          for (int o = 0; o < NAP / 4; ++o) {
-            const ulonglong2 wv = wr[o];
-            z2[2 * o] = tc::f2_fma(hh, wv.x, z2[2 * o]);
-            z2[2 * o + 1] = tc::f2_fma(hh, wv.y, z2[2 * o + 1]);
+          for (int o = 0; o < NAP; o += 2) {
+            const ulonglong2 wv = wr[o / 2];
+            acc[o] = tc::f2_fma(h, wv.x, acc[o]);
+            acc[o + 1] = tc::f2_fma(h, wv.y, acc[o + 1]);
           }
         }
       }
@@ -440,9 +442,13 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
     // partial sums of the two halves -> shared memory (the A region is dead now)
     float* zpart = reinterpret_cast<float*>(sA);
     if (!bad) {
-      uint64_t* dst = reinterpret_cast<uint64_t*>(zpart + (half * 128 + row) * NAP);
+      float* dst = zpart + (half * 128 + row) * NAP;
 #pragma unroll
-      for (int o = 0; o < NAP / 2; ++o) dst[o] = z2[o];
+      for (int o = 0; o < NAP; ++o) {
+        float e2, f2;
+        tc::f2_unpack(acc[o], e2, f2);
+        dst[o] = e2 + f2;
+      }
     }
     bad = sync_or();
 
