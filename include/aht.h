@@ -166,8 +166,11 @@ aht_status aht_xplay_matrix(aht_ctx* ctx, const int32_t* ego_ids, int32_t n_ego,
  * the per-env returns in one file-scope device array of AHT_XPLAY_STATIC_MAX_ENVS
  * floats (256 KiB) instead, which every GPU that loads the library holds until the
  * process exits, so any n_ego*n_tm*envs_per_pair up to that maximum works on any
- * context.  Same semantics, step counter and result as aht_xplay_matrix with only
- * `matrix` requested (device f32 [n_ego][n_tm]).
+ * context.  Same semantics and step counter as aht_xplay_matrix with only `matrix`
+ * requested (device f32 [n_ego][n_tm]), and the same result for LBF contexts; for bf16
+ * Overcooked and Hanabi contexts aht_xplay_matrix runs a streamed tensor-core kernel
+ * whose buffers are sized by the context, this variant the CUDA-core kernel, so an
+ * action can differ where the sampling CDF lies within ~1e-6 of the draw.
  *   - Allocates nothing and calls no allocating CUDA or library routine.
  *   - Returns AHT_EINVAL if n_ego*n_tm*envs_per_pair > AHT_XPLAY_STATIC_MAX_ENVS.
  *   - The first call on each device looks up the array's device address (with that

@@ -98,6 +98,7 @@ struct aht_ctx {
   float* last_value = nullptr;
   uint32_t* status = nullptr;
   // tensor-core path (bf16 LBF populations that fit shared and tensor memory)
+  int32_t weight_dtype = AHT_BF16;
   bool tc = false;
   TcDims tcd{};
   uint8_t* tcw = nullptr;
@@ -107,6 +108,7 @@ struct aht_ctx {
   bool wide = false;
   WideDims wd{};
   uint8_t* wtcw = nullptr;
+  uint8_t* wide_staging = nullptr;  // pinned, one streamed block (aht_set_policy)
   size_t wide_smem = 0;
   uint32_t* xp_st[2] = {};
   uint8_t* xp_act[2] = {};
@@ -238,15 +240,21 @@ aht_status pack_policy(const MlpDims& m, const void* const* W, const void* const
   return AHT_OK;
 }
 
-// Tensor-core block layout of one policy (see TcDims).
-TcDims make_tc_dims(const MlpDims& m) {
+// Tensor-core block layout of one policy (see TcDims); fp32 populations get the bf16
+// remainder copies of W1 and W2.
+TcDims make_tc_dims(const MlpDims& m, bool split) {
   TcDims t{};
   t.KP = (int)align_up(m.K + 1, 16);
   t.H0 = m.H0;
   t.H1 = m.H1;
+  t.split = split ? 1 : 0;
   uint32_t o = 0;
   t.oW1 = o; o += (uint32_t)(m.H0 * t.KP * 2);
   t.oW2 = o; o += (uint32_t)(m.H1 * m.H0 * 2);
+  if (split) {
+    t.oW1lo = o; o += (uint32_t)(m.H0 * t.KP * 2);
+    t.oW2lo = o; o += (uint32_t)(m.H1 * m.H0 * 2);
+  }
   t.oW3 = o; o += (uint32_t)(m.H1 * 8 * 4);
   t.ob2 = o; o += (uint32_t)(m.H1 * 4);
   t.ob3 = o; o += 8 * 4;
@@ -262,13 +270,14 @@ size_t tc_smem_bytes(const TcDims& t, int obs_dim, int state_bytes) {
          4 * 128 * 8 * 4;
 }
 
-// The tensor-core path applies to bf16 populations of LBF whose padded observation
-// (KP/2 columns) and hidden layers (<= 128 columns each, multiples of 64) fit the
-// 256 tensor-memory columns each agent uses, and whose two policy blocks fit shared memory.
+// The tensor-core path applies to LBF populations whose padded observation (KP/2
+// columns) and hidden layers (<= 128 columns each, multiples of 64) fit the 256
+// tensor-memory columns each agent uses, and whose two policy blocks fit shared memory
+// (fp32 populations hold each weight as a bf16 pair, twice the bytes).
 bool tc_eligible(const aht_ctx* c, int dtype) {
   const MlpDims& m = c->mlp;
-  if (dtype != AHT_BF16 || c->env.kind != AHT_LBF) return false;
-  const TcDims t = make_tc_dims(m);
+  if (c->env.kind != AHT_LBF) return false;
+  const TcDims t = make_tc_dims(m, dtype == AHT_FP32);
   if (t.KP > 256 || m.H0 > 128 || m.H1 > 128 || m.H0 % 64 || m.H1 % 64 || m.NA + 1 > 8) return false;
   return m.K % 4 == 0 && tc_smem_bytes(t, m.K, c->ops.bytes()) <= c->smem_optin;
 }
@@ -311,34 +320,55 @@ bool read_host(const void* p, size_t bytes, std::vector<uint8_t>& tmp, const voi
   return true;
 }
 
-// Packs one bf16 policy into its tensor-core block (dst: t.pol_bytes bytes).
+// Nearest-even bf16 of an fp32 value (bits), and the fp32 value of bf16 bits.
+uint16_t bf16_rne(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  return (uint16_t)((u + 0x7FFFu + ((u >> 16) & 1u)) >> 16);
+}
+float bf16_val(uint16_t h) {
+  const uint32_t u = (uint32_t)h << 16;
+  float f;
+  std::memcpy(&f, &u, 4);
+  return f;
+}
+
+// Packs one policy into its tensor-core block (dst: t.pol_bytes bytes).  bf16 weights go
+// in as they are; fp32 weights w as hi = bf16(w) and lo = bf16(w - hi) (w - hi is exact
+// in fp32).
 aht_status pack_policy_tc(const MlpDims& m, const TcDims& t, const void* const* W,
-                          const void* const* b, int vh, uint8_t* dst) {
+                          const void* const* b, int vh, int dtype, uint8_t* dst) {
+  if ((dtype == AHT_FP32) != (t.split != 0)) return fail(AHT_EINVAL, "weight dtype differs from the context's population");
   std::fill(dst, dst + t.pol_bytes, (uint8_t)0);
+  const int esz = dtype == AHT_FP32 ? 4 : 2;
   const int ins[3] = {m.K, m.H0, m.H1};
   const int outs[3] = {m.H0, m.H1, m.NA + vh};
   std::vector<uint8_t> tmp;
+  auto put = [&](uint32_t o_hi, uint32_t o_lo, uint32_t off, float f) {  // a bf16 matrix entry
+    const uint16_t hi = bf16_rne(f);
+    std::memcpy(dst + o_hi + off, &hi, 2);
+    if (t.split) {
+      const uint16_t lo = bf16_rne(f - bf16_val(hi));
+      std::memcpy(dst + o_lo + off, &lo, 2);
+    }
+  };
   for (int l = 0; l < 3; ++l) {
     const void* src = nullptr;
     if (!W[l] || !b[l]) return fail(AHT_EINVAL, "NULL weight pointer");
-    if (!read_host(W[l], (size_t)outs[l] * ins[l] * 2, tmp, &src)) return fail(AHT_ECUDA, "copying weights failed");
-    const uint16_t* w = static_cast<const uint16_t*>(src);
+    if (!read_host(W[l], (size_t)outs[l] * ins[l] * esz, tmp, &src)) return fail(AHT_ECUDA, "copying weights failed");
     for (int n = 0; n < outs[l]; ++n)
       for (int k = 0; k < ins[l]; ++k) {
         const int64_t i = (int64_t)n * ins[l] + k;
-        if (l == 0) std::memcpy(dst + t.oW1 + tc::canon_offset(n, k, t.KP), &w[i], 2);
-        if (l == 1) std::memcpy(dst + t.oW2 + tc::canon_offset(n, k, m.H0), &w[i], 2);
-        if (l == 2) {  // hidden units in pairs: [k / 2][output][k % 2]
-          const float f = to_f32(src, i, AHT_BF16);
+        const float f = to_f32(src, i, dtype);
+        if (l == 0) put(t.oW1, t.oW1lo, tc::canon_offset(n, k, t.KP), f);
+        if (l == 1) put(t.oW2, t.oW2lo, tc::canon_offset(n, k, m.H0), f);
+        if (l == 2)  // hidden units in pairs: [k / 2][output][k % 2]
           std::memcpy(dst + t.oW3 + 4 * (((k / 2) * 8 + n) * 2 + (k % 2)), &f, 4);
-        }
       }
-    if (!read_host(b[l], (size_t)outs[l] * 2, tmp, &src)) return fail(AHT_ECUDA, "copying biases failed");
-    const uint16_t* bb = static_cast<const uint16_t*>(src);
+    if (!read_host(b[l], (size_t)outs[l] * esz, tmp, &src)) return fail(AHT_ECUDA, "copying biases failed");
     for (int n = 0; n < outs[l]; ++n) {
-      const float f = to_f32(src, n, AHT_BF16);
-      if (l == 0)  // b1 = weight of the constant-1 input at K index obs_dim
-        std::memcpy(dst + t.oW1 + tc::canon_offset(n, m.K, t.KP), &bb[n], 2);
+      const float f = to_f32(src, n, dtype);
+      if (l == 0) put(t.oW1, t.oW1lo, tc::canon_offset(n, m.K, t.KP), f);  // b1: weight of the constant-1 input
       if (l == 1) std::memcpy(dst + t.ob2 + 4 * n, &f, 4);
       if (l == 2) std::memcpy(dst + t.ob3 + 4 * n, &f, 4);
     }
@@ -458,6 +488,37 @@ aht_status xplay_wide(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego, const i
   return AHT_OK;
 }
 
+// Cross-play of an LBF context on the tensor-core rollout kernel (tiles of up to 128 envs
+// of one pair), then the exact pair means.
+aht_status xplay_lbf_tc(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego, const int32_t* tm_ids,
+                        int32_t n_tm, int32_t P, int32_t max_steps, float* returns, int32_t* steps,
+                        uint8_t* actions, float* matrix) {
+  PpoTcArgs ta{};
+  ta.b = batch_of(c);
+  ta.tc = c->tcd;
+  ta.tcw = c->tcw;
+  ta.n_envs = c->n_envs;
+  ta.step0 = (uint32_t)c->step;
+  ta.xp.n_tm = n_tm;
+  ta.xp.P = P;
+  ta.xp.tpp = (P + 127) / 128;
+  ta.xp.max_steps = max_steps;
+  ta.xp.n_total = (int64_t)n_ego * n_tm * P;
+  for (int i = 0; i < n_ego; ++i) ta.xp.ego_ids[i] = ego_ids[i];
+  for (int j = 0; j < n_tm; ++j) ta.xp.tm_ids[j] = tm_ids[j];
+  ta.xp.returns = returns;
+  ta.xp.steps = steps;
+  ta.xp.actions = actions;
+  const int64_t n_pairs = (int64_t)n_ego * n_tm;
+  const int64_t grid = n_pairs * ta.xp.tpp;
+  if (grid > INT32_MAX) return fail(AHT_EINVAL, "too many tiles");
+  const int tk = timer_begin(c);
+  AHT_CUDA(lbf_xplay_tc(ta, (int)grid, c->tc_smem, c->stream));
+  timer_end(c, tk);
+  if (matrix) AHT_CUDA(launch_xp_reduce(returns, n_pairs, P, matrix, c->stream));
+  return AHT_OK;
+}
+
 // Tile rows for an M-row launch that fits in shared memory (M multiple of 4).
 int fit_rows(const aht_ctx* c, int want) {
   int M = (int)align_up(want, 4);
@@ -496,6 +557,7 @@ void aht_destroy(aht_ctx* c) {
   cudaFree(c->status);
   if (c->staging) cudaFreeHost(c->staging);
   if (c->tc_staging) cudaFreeHost(c->tc_staging);
+  if (c->wide_staging) cudaFreeHost(c->wide_staging);
   cudaFree(c->tcw);
   cudaFree(c->wtcw);
   for (int i = 0; i < 2; ++i) {
@@ -585,13 +647,14 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
     return bail(AHT_ECUDA, "cudaEventCreate failed");
   for (auto& e : c->ev)
     if (cudaEventCreate(&e) != cudaSuccess) return bail(AHT_ECUDA, "cudaEventCreate failed");
+  c->weight_dtype = pop->weight_dtype;
   if (tc_eligible(c, pop->weight_dtype)) {
-    c->tcd = make_tc_dims(m);
+    c->tcd = make_tc_dims(m, pop->weight_dtype == AHT_FP32);
     c->tc_smem = tc_smem_bytes(c->tcd, m.K, c->ops.bytes());
     std::vector<uint8_t> blocks((size_t)c->tcd.pol_bytes * pop->n_policies);
     for (int p = 0; p < pop->n_policies; ++p) {
       const int vh = pop->has_value_head ? pop->has_value_head[p] : 0;
-      aht_status ps = pack_policy_tc(m, c->tcd, pop->W + 3 * p, pop->b + 3 * p, vh,
+      aht_status ps = pack_policy_tc(m, c->tcd, pop->W + 3 * p, pop->b + 3 * p, vh, pop->weight_dtype,
                                      blocks.data() + (size_t)p * c->tcd.pol_bytes);
       if (ps != AHT_OK) {
         std::string msg = g_err;
@@ -641,6 +704,8 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
     const cudaError_t se = env.kind == AHT_HANABI ? hanabi_xplay_tc_smem_limit(c->wide_smem)
                                                   : overcooked_xplay_tc_smem_limit(c->wide_smem);
     if (se != cudaSuccess) return bail(AHT_ECUDA, "setting the shared-memory limit failed");
+    if (cudaMallocHost((void**)&c->wide_staging, c->wd.pol_bytes) != cudaSuccess)
+      return bail(AHT_ENOMEM, "pinned staging allocation failed");
     c->wide = true;
   }
   *out = c;
@@ -765,6 +830,14 @@ aht_status aht_xplay_matrix(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego,
     c->step += max_steps;
     return AHT_OK;
   }
+  if (c->tc) {  // LBF: the tensor-core rollout kernel in cross-play mode
+    const aht_status ts = xplay_lbf_tc(c, ego_ids, n_ego, tm_ids, n_tm, envs_per_pair, max_steps,
+                                       out->returns ? out->returns : c->xp_returns, out->steps, out->actions,
+                                       out->matrix);
+    if (ts != AHT_OK) return ts;
+    c->step += max_steps;
+    return AHT_OK;
+  }
   const int M = fit_rows(c, std::min(c->ops.max_rows, envs_per_pair));
   XpArgs a{};
   a.b = batch_of(c);
@@ -845,6 +918,13 @@ aht_status aht_xplay_matrix_static(aht_ctx* c, const int32_t* ego_ids, int32_t n
   float* scratch = nullptr;
   const aht_status ss = static_xp_returns(c->device, &scratch);
   if (ss != AHT_OK) return ss;
+  if (c->tc) {  // the same kernel as aht_xplay_matrix, which needs no context scratch here
+    const aht_status ts = xplay_lbf_tc(c, ego_ids, n_ego, tm_ids, n_tm, envs_per_pair, max_steps, scratch,
+                                       nullptr, nullptr, matrix);
+    if (ts != AHT_OK) return ts;
+    c->step += max_steps;
+    return AHT_OK;
+  }
   const int M = fit_rows(c, std::min(c->ops.max_rows, envs_per_pair));
   XpArgs a{};
   a.b = batch_of(c);
@@ -957,11 +1037,17 @@ aht_status aht_set_policy(aht_ctx* c, int32_t policy, const void* const* W, cons
   AHT_CUDA(cudaMemcpyAsync(c->weights + (int64_t)policy * c->mlp.stride, c->staging,
                            (size_t)c->mlp.stride * 4, cudaMemcpyHostToDevice, c->stream));
   if (c->tc) {
-    if (weight_dtype != AHT_BF16) return fail(AHT_EINVAL, "this context's population is bf16");
-    ps = pack_policy_tc(c->mlp, c->tcd, W, b, has_value_head, c->tc_staging);
+    ps = pack_policy_tc(c->mlp, c->tcd, W, b, has_value_head, weight_dtype, c->tc_staging);
     if (ps != AHT_OK) return ps;
     AHT_CUDA(cudaMemcpyAsync(c->tcw + (int64_t)policy * c->tcd.pol_bytes, c->tc_staging,
                              c->tcd.pol_bytes, cudaMemcpyHostToDevice, c->stream));
+  }
+  if (c->wide) {
+    if (weight_dtype != AHT_BF16) return fail(AHT_EINVAL, "this context's population is bf16");
+    ps = pack_policy_wide(c->mlp, c->wd, W, b, has_value_head, c->wide_staging);
+    if (ps != AHT_OK) return ps;
+    AHT_CUDA(cudaMemcpyAsync(c->wtcw + (int64_t)policy * c->wd.pol_bytes, c->wide_staging,
+                             c->wd.pol_bytes, cudaMemcpyHostToDevice, c->stream));
   }
   AHT_CUDA(cudaEventRecord(c->upload_done, c->stream));
   return AHT_OK;

@@ -44,11 +44,28 @@ struct PpoArgs {
 //   W3 fp32 [H1 / 2][8][2]: entry (p, o, i) = W3[o][2p + i], hidden units in pairs
 //      for packed fp32x2 FMAs (outputs past n_actions, and the value row when absent,
 //      are zero),
-//   b2 fp32 [H1], b3 fp32 [8].
+//   b2 fp32 [H1], b3 fp32 [8],
+// and for fp32 populations ("split" blocks) W1lo and W2lo, the bf16 remainders
+// W - bf16(W) in the same layouts as W1 and W2: W = W1 + W1lo to about 2^-17 relative
+// (the weight of the constant-1 input likewise carries b1 as two parts).
 struct TcDims {
   int32_t KP, H0, H1;      // padded obs dim (> obs_dim), hidden sizes
-  uint32_t oW1, oW2, oW3, ob2, ob3;
+  int32_t split;           // 1: fp32 weights as bf16 pairs (W1lo, W2lo present)
+  uint32_t oW1, oW2, oW3, ob2, ob3, oW1lo, oW2lo;
   uint32_t pol_bytes;
+};
+
+// Cross-play tiles of the tensor-core rollout kernel: tile t is chunk t % tpp of pair
+// t / tpp, envs [pair P + 128 chunk, min(pair P + 128 chunk + 128, (pair + 1) P)), ego
+// ego_ids[pair / n_tm], teammate tm_ids[pair % n_tm].
+struct TcXp {
+  int32_t n_tm, P, tpp, max_steps;
+  int64_t n_total;
+  int32_t ego_ids[kMaxXpIds];
+  int32_t tm_ids[kMaxXpIds];
+  float* returns;          // [n_total]
+  int32_t* steps;          // optional [n_total]
+  uint8_t* actions;        // optional [max_steps][n_total][2], pre-filled with 255
 };
 
 struct PpoTcArgs {
@@ -63,6 +80,7 @@ struct PpoTcArgs {
   uint32_t step0;
   int32_t T;
   TrajPtrs traj;
+  TcXp xp;               // cross-play launches only
 };
 
 // Per-policy block of the streamed tensor-core path (binary observations, hidden width H
@@ -171,9 +189,11 @@ AHT_DECLARE_ENV_LAUNCHERS(lbf)
 AHT_DECLARE_ENV_LAUNCHERS(overcooked)
 AHT_DECLARE_ENV_LAUNCHERS(hanabi)
 
-// Tensor-core PPO rollout (rollout_lbf.cu): LBF grids whose padded observation fits
-// 256 bf16 columns of tensor memory.
+// Tensor-core rollout (rollout_lbf.cu): LBF grids whose padded observation fits 256 bf16
+// columns of tensor memory; PPO collection (grid = tile table entries) and cross-play
+// (grid = pairs x tpp).  a.tc.split selects the fp32 (split-weight) variant.
 cudaError_t lbf_ppo_tc(const PpoTcArgs&, int grid, size_t smem, cudaStream_t);
+cudaError_t lbf_xplay_tc(const PpoTcArgs&, int grid, size_t smem, cudaStream_t);
 
 // Streamed tensor-core cross-play step (rollout_overcooked.cu, rollout_hanabi.cu).
 // grid = the launch's tiles (xp_tc_tiles), smem = xp_tc_smem_bytes.

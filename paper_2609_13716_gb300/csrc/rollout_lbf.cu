@@ -9,4 +9,8 @@ AHT_DEFINE_ENV_LAUNCHERS(lbf, EnvLbf)
 cudaError_t lbf_ppo_tc(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
   return LaunchTc<EnvLbf>::ppo(a, grid, smem, s);
 }
+
+cudaError_t lbf_xplay_tc(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
+  return LaunchTc<EnvLbf>::xplay(a, grid, smem, s);
+}
 }  // namespace aht

@@ -36,7 +36,12 @@ constexpr int kTcCompute = 256;          // compute threads
 constexpr int kTcThreads = 288;          // + one MMA warp
 constexpr int kTcComputeBar = 1;         // named barrier id of the compute warps
 
-template <class Env>
+// kXp: cross-play (each tile is a chunk of one pair's envs, reset at the call's first
+// step, frozen once done; the per-env return and episode length are the outputs) instead
+// of PPO collection.  kSplit: fp32 weights held as bf16 pairs W = W_hi + W_lo, L1 =
+// X W1_hi + X W1_lo and L2 = b2 + hi W2_hi + lo W2_hi + hi W2_lo (lo W2_lo is below
+// 2^-16 of the sum and left out).
+template <class Env, bool kXp, bool kSplit>
 __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a) {
   using State = typename Env::State;
   constexpr int NA = Env::kNumActions;
@@ -46,10 +51,24 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   __shared__ __align__(8) uint64_t wload_bar, drain_bar;
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
+  __shared__ volatile int stop_flag;               // cross-play: every env of the tile is done
 
-  const int4 tile = a.tiles[blockIdx.x];
-  const int count = tile.y;
-  if (count == 0) return;
+  int64_t env0;
+  int count, ego_pol, tm_pol;
+  if constexpr (kXp) {
+    const int pair = blockIdx.x / a.xp.tpp, chunk = blockIdx.x - pair * a.xp.tpp;
+    env0 = (int64_t)pair * a.xp.P + 128 * chunk;
+    count = min(128, a.xp.P - 128 * chunk);
+    ego_pol = a.xp.ego_ids[pair / a.xp.n_tm];
+    tm_pol = a.xp.tm_ids[pair % a.xp.n_tm];
+  } else {
+    const int4 tile = a.tiles[blockIdx.x];
+    env0 = tile.x;
+    count = tile.y;
+    ego_pol = a.ego;
+    tm_pol = tile.z;
+  }
+  if (count <= 0) return;
   const TcDims& d = a.tc;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, half = (warp >> 2) & 1, row = tid & 127;
   const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
@@ -60,7 +79,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   const int split = (chunks + 1) / 2;
   const int my_c0 = half ? split : 0, my_c1 = half ? chunks : split;
   const int my_w0 = min(4 * my_c0, cells), my_w1 = min(4 * my_c1, cells);
-  const bool with_boot = a.traj.last_value != nullptr;
+  const bool with_boot = !kXp && a.traj.last_value != nullptr;
 
   // The tile is the contiguous env range [tile.x, tile.x + count); observation rows are
   // packed at obs_dim bytes (an odd number of words: no bank conflicts per thread row),
@@ -70,7 +89,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   State* st = reinterpret_cast<State*>(sObs + align_up(128 * od, 16));      // [128]
   uint8_t* act1s = reinterpret_cast<uint8_t*>(st) + align_up(128 * sizeof(State), 16);  // [128]
   float* zpart = reinterpret_cast<float*>(act1s + 128);                     // [2][2][128][8]
-  const int64_t env0 = tile.x;
 
   if (tid == 0) {
     for (int i = 0; i < 4; ++i) {
@@ -81,10 +99,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     tc::mbar_init(&drain_bar, 1);
     tc::mbar_init_fence();
     abort_flag = 0;
+    stop_flag = 0;
   }
   if (warp == 0) tc::tmem_alloc(&tmem_slot, 512);
   for (int i = tid; i < 32 * od; i += blockDim.x) reinterpret_cast<uint32_t*>(sObs)[i] = 0u;
-  if (tid < count) load_state(a.state, N, env0 + tid, st[tid]);
+  if (tid < count) {
+    if constexpr (kXp) Env::reset(a.b.env, a.b.key, (uint32_t)(env0 + tid), a.step0, st[tid]);
+    else load_state(a.state, N, env0 + tid, st[tid]);
+  }
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
@@ -93,7 +115,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   if (warp == 8) {
     // ================================ MMA warp =====================================
     if (lane == 0) {
-      const int pol[2] = {a.ego, tile.z};
+      const int pol[2] = {ego_pol, tm_pol};
       tc::mbar_expect_tx(&wload_bar, 2u * d.pol_bytes);
       for (int p = 0; p < 2; ++p) {
         const uint8_t* src = a.tcw + (int64_t)pol[p] * d.pol_bytes;
@@ -104,30 +126,44 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       const uint32_t idesc1 = tc::idesc_bf16(128, d.H0), idesc2 = tc::idesc_bf16(128, d.H1);
       const uint32_t sbo1 = (uint32_t)(d.KP / 8) * 128u, sbo2 = (uint32_t)(d.H0 / 8) * 128u;
       // agents in the order the compute warps release them: teammate, then ego
+      bool stopped = false;
       auto issue = [&](int ag, int layer, uint32_t parity) {
         ok = false;
         for (int tries = 0; tries < 1000 && !ok && !abort_flag; ++tries)
           ok = tc::mbar_wait(&opnd_bar[2 * ag + layer], parity, 2000000ull);
         if (!ok) return;
+        if (kXp && stop_flag) {  // released without operands: the tile is finished
+          stopped = true;
+          return;
+        }
         tc::fence_after_sync();
         const uint32_t wbase = tc::smem_u32(sW0) + (uint32_t)ag * d.pol_bytes;
         const uint32_t P = tmem + (uint32_t)(ag * 256), Q = P + 128;
         if (layer == 0) {
           const uint64_t w0 = tc::smem_desc(wbase + d.oW1, 128u, sbo1);
           for (int ks = 0; ks < d.KP / 16; ++ks) tc::mma_ts(Q, P + 8 * ks, w0 + 16u * ks, idesc1, ks > 0);
+          if constexpr (kSplit) {
+            const uint64_t w1 = tc::smem_desc(wbase + d.oW1lo, 128u, sbo1);
+            for (int ks = 0; ks < d.KP / 16; ++ks) tc::mma_ts(Q, P + 8 * ks, w1 + 16u * ks, idesc1, 1u);
+          }
         } else {
           const uint64_t w0 = tc::smem_desc(wbase + d.oW2, 128u, sbo2);
           for (int ks = 0; ks < d.H0 / 16; ++ks) tc::mma_ts(Q, P + 8 * ks, w0 + 16u * ks, idesc2, 1u);
           for (int ks = 0; ks < d.H0 / 16; ++ks) tc::mma_ts(Q, P + d.H0 / 2 + 8 * ks, w0 + 16u * ks, idesc2, 1u);
+          if constexpr (kSplit) {
+            const uint64_t w1 = tc::smem_desc(wbase + d.oW2lo, 128u, sbo2);
+            for (int ks = 0; ks < d.H0 / 16; ++ks) tc::mma_ts(Q, P + 8 * ks, w1 + 16u * ks, idesc2, 1u);
+          }
         }
         tc::commit(&acc_bar[2 * ag + layer]);
       };
-      for (int t = 0; ok && t < a.T; ++t) {
+      const int n_steps = kXp ? a.xp.max_steps : a.T;
+      for (int t = 0; ok && !stopped && t < n_steps; ++t) {
         const uint32_t par = (uint32_t)t & 1u;
         issue(1, 0, par);
-        if (ok) issue(0, 0, par);
-        if (ok) issue(1, 1, par);
-        if (ok) issue(0, 1, par);
+        if (ok && !stopped) issue(0, 0, par);
+        if (ok && !stopped) issue(1, 1, par);
+        if (ok && !stopped) issue(0, 1, par);
       }
       if (ok && with_boot) {
         issue(0, 0, (uint32_t)a.T & 1u);
@@ -248,7 +284,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     };
     // the tile's ego observation rows -> trajectory [t][env0 .. env0+count): one contiguous
     // block, written by one bulk (TMA) store when 16-byte aligned, else by all threads
-    const bool bulk_obs = a.traj.obs && (count * od) % 16 == 0;
+    const bool bulk_obs = !kXp && a.traj.obs && (count * od) % 16 == 0;
     auto copy_obs = [&](int t) {
       uint8_t* dst = a.traj.obs + ((int64_t)t * N + env0) * od;
       const uint32_t bytes = (uint32_t)(count * od);
@@ -266,9 +302,20 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
 
     // Steps 0..T-1, then (if requested) the ego's V_T of the state after the last step.
     // The agent loops are not unrolled so that every phase's code exists once.
-    for (int t = 0; t <= a.T; ++t) {
-      const bool boot = t == a.T;
+    const int n_steps = kXp ? a.xp.max_steps : a.T;
+    bool alive = true;  // cross-play: the row's episode is running (half-0 threads)
+    int nsteps = 0;
+    for (int t = 0; t <= n_steps; ++t) {
+      const bool boot = t == n_steps;
       if (boot && !with_boot) break;
+      if constexpr (kXp) {
+        // every env of the tile is done: release the MMA warp without operands and stop
+        if (!tc::bar_or(kTcComputeBar, kTcCompute, half == 0 && row < count && alive)) {
+          if (tid == 0) stop_flag = 1;
+          tc::mbar_arrive(&opnd_bar[2]);  // the teammate's L1 barrier it waits on
+          break;
+        }
+      }
       const int first = boot ? 0 : 1;  // teammate first: the ego's rows stay for the copy
       const uint32_t par = (uint32_t)t & 1u, gt = a.step0 + (uint32_t)t;
       // this half's action draw (ego: warps 0-3, teammate: warps 4-7), ahead of its use
@@ -281,7 +328,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         wait_acc(i, 0, par);
         if (!bad) epilogue1(i);
       }
-      if (!boot && a.traj.obs) {       // overlaps L2 on the tensor cores
+      if (!kXp && !boot && a.traj.obs) {  // overlaps L2 on the tensor cores
         tc::fence_proxy_async();       // the rows were written by ordinary stores
         if (sync_or()) break;
         copy_obs(t);
@@ -316,7 +363,25 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         }
       }
       if (sync_or()) break;
-      if (half == 0 && row < count) {
+      if (kXp && half == 0 && row < count && alive) {
+        const int act1 = act1s[row];
+        const int64_t env = env0 + row;
+        if (a.xp.actions) {
+          uint8_t* rec = a.xp.actions + ((int64_t)t * a.xp.n_total + env) * 2;
+          rec[0] = (uint8_t)act0;
+          rec[1] = (uint8_t)act1;
+        }
+        float r0, r1, team;
+        const int done = Env::step(a.b.env, s, act0, act1, r0, r1, team);
+        if (done < 0) {
+          atomicOr(a.b.status, kStatusIllegalAction);
+          alive = false;
+        } else {
+          nsteps += 1;
+          if (done) alive = false;
+        }
+        st[row] = s;
+      } else if (!kXp && half == 0 && row < count) {
         const int act1 = act1s[row];
         const int64_t env = env0 + row;
         float r0, r1, team;
@@ -338,7 +403,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     if (bad || abort_flag) {
       abort_flag = 1;
     } else if (tid < count) {
-      store_state(a.state, N, env0 + tid, st[tid]);
+      if constexpr (kXp) {
+        a.xp.returns[env0 + tid] = Env::ret(st[tid]);
+        if (a.xp.steps) a.xp.steps[env0 + tid] = nsteps;
+      } else {
+        store_state(a.state, N, env0 + tid, st[tid]);
+      }
     }
   }
 
@@ -360,11 +430,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
 
 template <class Env>
 struct LaunchTc {
-  static cudaError_t ppo(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
-    cudaError_t e = cudaFuncSetAttribute(ppo_tc_kernel<Env>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  template <bool kXp, bool kSplit>
+  static cudaError_t run(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
+    cudaError_t e = cudaFuncSetAttribute(ppo_tc_kernel<Env, kXp, kSplit>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    ppo_tc_kernel<Env><<<grid, kTcThreads, smem, s>>>(a);
+    ppo_tc_kernel<Env, kXp, kSplit><<<grid, kTcThreads, smem, s>>>(a);
     return cudaGetLastError();
+  }
+  static cudaError_t ppo(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
+    return a.tc.split ? run<false, true>(a, grid, smem, s) : run<false, false>(a, grid, smem, s);
+  }
+  static cudaError_t xplay(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
+    return a.tc.split ? run<true, true>(a, grid, smem, s) : run<true, false>(a, grid, smem, s);
   }
 };
 
