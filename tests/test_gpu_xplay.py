@@ -99,3 +99,29 @@ def test_full_size_xplay_sampled(name):
     ids = np.unique(np.concatenate([[0, n - 1], np.random.default_rng(1).integers(0, n, 30)]))
     check(wl, pop_np, list(wl.ego_ids), list(wl.tm_ids), wl.envs_per_pair, wl.max_steps, out,
           wl.env_seed, env_ids=ids)
+
+
+@pytest.mark.parametrize("name,P,S", [("overcooked5x4_xplay_8x8x64", 40, 60),
+                                      ("lbf7x7_xplay_8x16x256", 70, 40)])
+def test_set_policy_reaches_every_kernel_copy(name, P, S):
+    # Context A uploads policy 3's weights into slot 0 with aht_set_policy; context B is
+    # created with that population.  Same seed and step: the matrices must be identical,
+    # so the kernel's own packed copy (streamed tensor-core blocks for Overcooked, split
+    # fp32 tensor-core blocks for LBF) was refreshed.
+    require_gpu()
+    wl = W.WORKLOADS[name]
+    pop_np = W.population(wl)
+    swapped = [pop_np[3]] + pop_np[1:]
+    ego, tm = [0, 1], [wl.tm_ids[0], wl.tm_ids[1]]
+    a, _ = make_ctx(wl, len(ego) * len(tm) * P, pop_np=pop_np)
+    b, _ = make_ctx(wl, len(ego) * len(tm) * P, pop_np=swapped)
+    dt = torch.float32 if wl.weight_dtype == W.FP32 else torch.bfloat16
+    host = [(torch.from_numpy(Wt).to(dt), torch.from_numpy(bb).to(dt)) for Wt, bb in pop_np[3]]
+    aht.aht_set_policy(a, 0, host, 0, aht.AHT_FP32 if wl.weight_dtype == W.FP32 else aht.AHT_BF16)
+    ma = torch.empty(len(ego), len(tm), device="cuda")
+    mb = torch.empty_like(ma)
+    aht.aht_xplay_matrix(a, ego, tm, P, S, ma)
+    aht.aht_xplay_matrix(b, ego, tm, P, S, mb)
+    aht.aht_sync(a)
+    aht.aht_sync(b)
+    assert torch.equal(ma, mb)
