@@ -48,7 +48,7 @@ constexpr int kXpCompute = 256;
 constexpr int kXpThreads = 320;
 constexpr int kXpComputeBar = 1;
 constexpr int kXpMaxStages = 3;
-constexpr int kXpMaxChunksPerStage = 4;
+constexpr int kXpMaxChunksPerStage = 5;
 constexpr uint32_t kXpSmemBudget = 231424;  // opt-in maximum minus a margin for static data
 
 struct XpTcSmem {
@@ -75,9 +75,9 @@ __host__ __device__ inline XpTcSmem xp_tc_layout(const WideDims& w) {
   L.a_bytes = (uint32_t)align_up(a, 1024);
   L.bit_words = (w.KP + 31) / 32;
   const uint32_t bits = (uint32_t)align_up(128 * L.bit_words * 4, 1024);
-  // Stages are as large as two of them fit: each barrier completion of a bulk copy or an
-  // MMA commit reaches its waiter some 500 cycles later (measured on GB300), so the bytes
-  // moved per completion, not the number of copies in flight, set the stream's rate.
+  // Two stages as large as fit: on GB300 a bulk copy takes about the same 500-2000 cycles
+  // to land for 8 KB as for 32 KB, and copies in flight barely overlap (measured, also
+  // with several issuing warps), so the bytes per copy set the stream's rate.
   const int slots = (int)((kXpSmemBudget - L.a_bytes - bits) / kWideChunk);
   L.spc = slots / 2 > kXpMaxChunksPerStage ? kXpMaxChunksPerStage : slots / 2;
   L.nst = slots / L.spc > kXpMaxStages ? kXpMaxStages : slots / L.spc;
@@ -233,12 +233,11 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
   if (warp == 9) {
     // ============================ weight producer ===================================
     if (lane == 0) {
-      int k = 0;
+      int k = 0, slot = 0;
+      uint32_t use = 0;  // times the slot was filled before
       bool ok = true;
       const uint64_t keep = tc::l2_evict_last();  // every step re-reads the population
       for (; k < n_stages; ++k) {
-        const int slot = k % NST;
-        const uint32_t use = (uint32_t)(k / NST);
         if (use > 0) {
           ok = false;
           for (int tries = 0; tries < 1000 && !ok && !abort_flag; ++tries)
@@ -248,6 +247,10 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
         const uint32_t bytes = (uint32_t)min(SPC, n_chunks - k * SPC) * kWideChunk;
         tc::mbar_expect_tx(&full_bar[slot], bytes);
         tc::bulk_g2s_hint(sStage + slot * stage_bytes, pblk + (int64_t)k * stage_bytes, bytes, &full_bar[slot], keep);
+        if (++slot == NST) {
+          slot = 0;
+          ++use;
+        }
       }
       if (!ok) abort_flag = 1;
       next_chunk = k;  // stages issued
@@ -263,15 +266,26 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
         if (ok) tc::fence_after_sync();
         return ok;
       };
-      int c = 0;
+      // ring cursor of the next chunk: its stage's slot, its position in the stage, the
+      // slot's full-barrier parity; advanced by increments (a runtime division per chunk
+      // costs this single thread hundreds of cycles)
+      int c = 0, sub = 0, slot = 0;
+      uint32_t fpar = 0;
+      const uint32_t stage0 = tc::smem_u32(sStage);
       auto chunk = [&](uint64_t& desc) {  // waits for weight chunk c, returns its descriptor
-        const int k = c / SPC, slot = k % NST, sub = c - k * SPC;
-        if (sub == 0 && !wait_for(&full_bar[slot], (uint32_t)(k / NST) & 1u)) return false;
-        desc = tc::smem_desc(tc::smem_u32(sStage + slot * stage_bytes + sub * kWideChunk), 128u, 256u);
+        if (sub == 0 && !wait_for(&full_bar[slot], fpar)) return false;
+        desc = tc::smem_desc(stage0 + (uint32_t)slot * stage_bytes + (uint32_t)sub * kWideChunk, 128u, 256u);
         return true;
       };
       auto release = [&]() {  // the stage is free once the MMAs reading its last chunk finish
-        if (c % SPC == SPC - 1 || c == n_chunks - 1) tc::commit(&empty_bar[(c / SPC) % NST]);
+        if (++sub == SPC || c == n_chunks - 1) {
+          tc::commit(&empty_bar[slot]);
+          sub = 0;
+          if (++slot == NST) {
+            slot = 0;
+            fpar ^= 1u;
+          }
+        }
         ++c;
       };
       bool ok = wait_for(&obs_bar, 0);
