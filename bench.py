@@ -54,6 +54,17 @@ def parse():
     return p.parse_args()
 
 
+def max_over_ranks(value, device):
+    """The largest value over all ranks (timings only: the data path has no collective)."""
+    import torch
+    import torch.distributed as dist
+    if not dist.is_available() or not dist.is_initialized() or dist.get_world_size() == 1:
+        return float(value)
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t)
+
+
 def dist_env():
     return (int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)),
             int(os.environ.get("WORLD_SIZE", 1)))
@@ -182,12 +193,16 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+# the sources the fused rollout kernel is compiled from
+ROLLOUT_SOURCES = ("rollout_tc.cuh", "tc_common.cuh", "env_lbf.cuh", "aht_common.cuh", "mlp_simt.cuh",
+                   "rollout_impl.cuh", "kernels.h", "rollout_lbf.cu")
+
+
 def csrc_hash():
     h = hashlib.sha256()
     d = os.path.join(ROOT, "paper_2609_13716_gb300", "csrc")
-    for f in sorted(os.listdir(d)):
-        if f.endswith((".cu", ".cuh", ".h")):
-            h.update(open(os.path.join(d, f), "rb").read())
+    for f in ROLLOUT_SOURCES:
+        h.update(open(os.path.join(d, f), "rb").read())
     return h.hexdigest()[:16]
 
 
@@ -273,10 +288,7 @@ def run_ours(args):
     kernel_ms, kernel_launches = aht.aht_get_timing(ctx)
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, stops)]
     ms = sum(step_ms) / len(step_ms)
-    ms_t = torch.tensor([ms], device="cuda")
-    if world > 1:
-        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)   # timing only, not the data path
-    ms_max = float(ms_t)
+    ms_max = max_over_ranks(ms, "cuda")
     aht.aht_sync(ctx)
 
     # ---- end to end: ego weights from pinned host memory in, whole trajectory out ------
@@ -299,9 +311,7 @@ def run_ours(args):
         if k > 0:
             e2e_ms.append(e2e_s.elapsed_time(e2e_e))
     aht.aht_sync(ctx)
-    e2e_ms_max = torch.tensor([sum(e2e_ms) / max(1, len(e2e_ms))], device="cuda")
-    if world > 1:
-        dist.all_reduce(e2e_ms_max, op=dist.ReduceOp.MAX)
+    e2e_ms_max = max_over_ranks(sum(e2e_ms) / max(1, len(e2e_ms)), "cuda")
 
     # ---- roofline of the dominant kernel (the fused rollout) ----------------------------
     env_steps = N * T

@@ -24,7 +24,12 @@
  *     aht_sync, which synchronise that stream.
  *   - Host-side argument errors are returned immediately (AHT_EINVAL) and nothing is
  *     enqueued.  Errors detected on the device (an out-of-range id, an illegal forced
- *     Hanabi action) are latched in a device status word and returned by aht_sync.
+ *     Hanabi action, a wait of a tensor-core kernel that ran past its time limit) are
+ *     latched in a device status word and returned by aht_sync.
+ *   - Every wait of a kernel on another warp's progress (mbarriers, named barriers fed
+ *     by them) is bounded by %globaltimer, 2 s by default: on expiry the kernel latches
+ *     the timeout bit, stops its work, drains its own tensor-core operations and copies,
+ *     frees its tensor memory and returns, so the context stays usable.
  *   - Only aht_create allocates device memory.  Every other call allocates nothing.
  *   - Seat 0 is the ego, seat 1 the teammate.  XP matrices are [ego][teammate]
  *     (the transpose of the paper's figures, whose rows are teammates).
@@ -50,7 +55,7 @@ typedef enum aht_status {
   AHT_EINVAL = 1,   /* invalid argument (host check) */
   AHT_ENOMEM = 2,   /* device allocation failed in aht_create */
   AHT_ECUDA = 3,    /* a CUDA runtime call failed */
-  AHT_ETIMEOUT = 4, /* reserved: a bounded device wait gave up */
+  AHT_ETIMEOUT = 4, /* a bounded device wait gave up (reported by aht_sync) */
   AHT_EDEVICE = 5   /* the device status word recorded an error */
 } aht_status;
 
@@ -246,9 +251,16 @@ aht_status aht_set_state(aht_ctx* ctx, const void* buf, size_t bytes);
 /* Global step counter (the next step index). */
 int64_t aht_step_counter(const aht_ctx* ctx);
 
-/* Synchronises the context's stream and returns AHT_EDEVICE if the device status word
- * recorded an error since the last aht_sync (the word is then cleared). */
+/* Synchronises the context's stream and returns AHT_ETIMEOUT if the device status word
+ * recorded only expired waits since the last aht_sync, AHT_EDEVICE if it recorded any
+ * other device error (the word is then cleared), else AHT_OK. */
 aht_status aht_sync(aht_ctx* ctx);
+
+/* Failure-detection hook (no paper counterpart): enqueues on the context's stream one
+ * thread that waits, with the kernels' bounded wait and a limit of limit_ns nanoseconds
+ * (1 .. 10^9), on an mbarrier nothing arrives on; the wait expires and latches the
+ * timeout bit, so the next aht_sync returns AHT_ETIMEOUT.  No fault, no hang. */
+aht_status aht_debug_expire_wait(aht_ctx* ctx, int64_t limit_ns);
 
 const char* aht_last_error(void);
 const char* aht_status_string(aht_status s);

@@ -23,7 +23,7 @@ EXPORTED = ["aht_create", "aht_destroy", "aht_reset", "aht_rollout", "aht_xplay_
             "aht_gae", "aht_step_forced", "aht_policy_forward", "aht_get_state",
             "aht_set_state", "aht_step_counter", "aht_sync", "aht_last_error",
             "aht_status_string", "aht_set_policy", "aht_set_timing", "aht_get_timing",
-            "aht_xplay_matrix_static", "aht_debug_tanh"]
+            "aht_xplay_matrix_static", "aht_debug_tanh", "aht_debug_expire_wait"]
 
 
 class AhtError(RuntimeError):
@@ -328,3 +328,12 @@ def aht_step_counter(ctx: Context) -> int:
 
 def aht_sync(ctx: Context):
     _check(load().aht_sync(ctx.handle))
+
+
+def aht_debug_expire_wait(ctx: Context, limit_ns: int):
+    """Failure-detection hook: a kernel's bounded wait on a barrier nothing arrives on
+    expires after limit_ns; the next aht_sync raises AhtError with AHT_ETIMEOUT."""
+    L = load()
+    L.aht_debug_expire_wait.argtypes = [C.c_void_p, C.c_int64]
+    L.aht_debug_expire_wait.restype = C.c_int
+    _check(L.aht_debug_expire_wait(ctx.handle, int(limit_ns)))

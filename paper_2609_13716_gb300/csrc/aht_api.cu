@@ -1081,9 +1081,20 @@ aht_status aht_sync(aht_ctx* c) {
   AHT_CUDA(cudaMemcpy(&s, c->status, 4, cudaMemcpyDeviceToHost));
   if (s != 0) {
     AHT_CUDA(cudaMemset(c->status, 0, 4));
-    return fail(AHT_EDEVICE, "device status word 0x" + [&] { char b[16]; std::snprintf(b, sizeof b, "%x", s); return std::string(b); }() +
-                                 " (1 illegal action, 2 actor mismatch, 4 bad policy)");
+    char hex[16];
+    std::snprintf(hex, sizeof hex, "%x", s);
+    const std::string msg = std::string("device status word 0x") + hex +
+                            " (1 illegal action, 2 actor mismatch, 4 bad policy, 8 a bounded wait expired)";
+    return fail(s == kStatusTimeout ? AHT_ETIMEOUT : AHT_EDEVICE, msg);
   }
+  return AHT_OK;
+}
+
+aht_status aht_debug_expire_wait(aht_ctx* c, int64_t limit_ns) {
+  if (!c) return fail(AHT_EINVAL, "ctx is NULL");
+  if (limit_ns < 1 || limit_ns > 1000000000) return fail(AHT_EINVAL, "limit_ns must be in 1..1e9");
+  DeviceGuard g(c->device);
+  AHT_CUDA(launch_expire_wait(c->status, (uint64_t)limit_ns, c->stream));
   return AHT_OK;
 }
 

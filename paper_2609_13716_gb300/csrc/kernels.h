@@ -208,6 +208,7 @@ cudaError_t launch_group(const GroupArgs&, cudaStream_t);
 cudaError_t launch_policy(const PolicyArgs&, int grid, size_t smem, cudaStream_t);
 cudaError_t policy_set_smem_limit(size_t bytes);
 cudaError_t launch_tanh_probe(const float* x, float* y, int64_t n, cudaStream_t);
+cudaError_t launch_expire_wait(uint32_t* status, uint64_t limit_ns, cudaStream_t);
 int group_tiles(int64_t n_envs, int M);  // tile-table entries of a launch
 cudaError_t launch_gae(const float* r, const float* v, const uint8_t* d, const float* v_last,
                        int64_t n, int32_t T, float gamma, float lambda, float* adv, float* tgt,

@@ -138,6 +138,20 @@ __global__ void tanh_probe_kernel(const float* __restrict__ x, float* __restrict
   if (i + 1 < n) y[i + 1] = y1;
 }
 
+// One thread waits on an mbarrier that nothing arrives on, with the kernels' bounded wait:
+// the wait expires after limit_ns and the timeout bit is latched.
+__global__ void expire_wait_kernel(uint32_t* status, uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  tc::mbar_init(&bar, 1);
+  tc::mbar_init_fence();
+  if (!tc::mbar_wait(&bar, 0, limit_ns)) atomicOr(status, kStatusTimeout);
+}
+
+cudaError_t launch_expire_wait(uint32_t* status, uint64_t limit_ns, cudaStream_t s) {
+  expire_wait_kernel<<<1, 1, 0, s>>>(status, limit_ns);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_tanh_probe(const float* x, float* y, int64_t n, cudaStream_t s) {
   const int64_t pairs = (n + 1) / 2;
   tanh_probe_kernel<<<(unsigned)((pairs + 255) / 256), 256, 0, s>>>(x, y, n);

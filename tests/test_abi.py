@@ -53,4 +53,6 @@ def test_host_validation_needs_no_gpu(lib):
     assert L.aht_create(C.byref(bad), None, 4, 0, None, C.byref(h)) == aht.AHT_EINVAL
     assert b"width" in L.aht_last_error()
     assert L.aht_gae(None, None, None, None, 1, 1, 0.9, 0.9, None, None, None) == aht.AHT_EINVAL
+    L.aht_debug_expire_wait.argtypes = [C.c_void_p, C.c_int64]
+    assert L.aht_debug_expire_wait(None, 1000) == aht.AHT_EINVAL
 
