@@ -140,6 +140,49 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
   const uint8_t* const pblk = a.tcw + (int64_t)pol * w.pol_bytes;
   const uint32_t gt = a.step0 + (uint32_t)a.s;
 
+  // ---- 0. overlap with the previous step's launch (programmatic dependent launch) ------
+  // The next step's CTAs may start now; everything up to griddepcontrol.wait touches
+  // nothing the previous step writes (barriers, tensor memory).
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  if (tid == 0) {
+    for (int i = 0; i < NST; ++i) {
+      tc::mbar_init(&full_bar[i], 1);
+      tc::mbar_init(&empty_bar[i], 1);
+    }
+    tc::mbar_init(&obs_bar, kXpCompute);
+    for (int i = 0; i < 3; ++i) tc::mbar_init(&acc_bar[i], 1);
+    tc::mbar_init(&epi1_bar, kXpCompute);
+    tc::mbar_init(&epi2_bar, kXpCompute);
+    tc::mbar_init(&w3_bar, 1);
+    tc::mbar_init(&drain_bar, 1);
+    tc::mbar_init_fence();
+    abort_flag = 0;
+  }
+  if (warp == 0) tc::tmem_alloc(&tmem_slot, 512);
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const int n_chunks = w.n_l1 + w.n_l2;
+  const int SPC = L.spc, n_stages = (n_chunks + SPC - 1) / SPC;
+  const uint32_t stage_bytes = (uint32_t)SPC * kWideChunk;
+  // producer state (warp 9, lane 0): next stage, its ring slot, uses of that slot so far
+  int pk = 0, pslot = 0;
+  uint32_t puse = 0;
+  if (warp == 9 && lane == 0) {  // the first stages: the population is read-only
+    const uint64_t keep = tc::l2_evict_last();
+    for (; pk < n_stages && pk < NST; ++pk, ++pslot) {
+      const uint32_t bytes = (uint32_t)min(SPC, n_chunks - pk * SPC) * kWideChunk;
+      tc::mbar_expect_tx(&full_bar[pslot], bytes);
+      tc::bulk_g2s_hint(sStage + pslot * stage_bytes, pblk + (int64_t)pk * stage_bytes, bytes, &full_bar[pslot], keep);
+    }
+    if (pslot == NST) {
+      pslot = 0;
+      puse = 1;
+    }
+  }
+  // the previous step's state, alive flags and actions are complete and visible
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+
   // ---- 1. transition of step s - 1, and this step's observation bits -----------------
   bool alive = false;
   float u_act = 0.0f;
@@ -204,37 +247,21 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
       for (int i = 0; i < L.bit_words; ++i) bits[i] = 0u;
     }
   }
-  if (!__syncthreads_or(alive) || a.s == a.max_steps) return;  // nothing left to act
-
-  if (tid == 0) {
-    for (int i = 0; i < NST; ++i) {
-      tc::mbar_init(&full_bar[i], 1);
-      tc::mbar_init(&empty_bar[i], 1);
-    }
-    tc::mbar_init(&obs_bar, kXpCompute);
-    for (int i = 0; i < 3; ++i) tc::mbar_init(&acc_bar[i], 1);
-    tc::mbar_init(&epi1_bar, kXpCompute);
-    tc::mbar_init(&epi2_bar, kXpCompute);
-    tc::mbar_init(&w3_bar, 1);
-    tc::mbar_init(&drain_bar, 1);
-    tc::mbar_init_fence();
-    abort_flag = 0;
-  }
-  if (warp == 0) tc::tmem_alloc(&tmem_slot, 512);
   tc::fence_before_sync();
-  __syncthreads();
+  const bool proceed = __syncthreads_or(alive) && a.s < a.max_steps;
   tc::fence_after_sync();
   const uint32_t tmem = tmem_slot;
-  const int n_chunks = w.n_l1 + w.n_l2;
-
-  const int SPC = L.spc, n_stages = (n_chunks + SPC - 1) / SPC;
-  const uint32_t stage_bytes = (uint32_t)SPC * kWideChunk;
-
+  if (!proceed) {  // nothing left to act this step: the prefetched stages land, then exit
+    if (warp == 9 && lane == 0)
+      for (int d = 0; d < pk; ++d) tc::mbar_wait(&full_bar[d], 0u);
+    if (warp == 0) tc::tmem_dealloc(tmem, 512);
+    return;
+  }
   if (warp == 9) {
     // ============================ weight producer ===================================
     if (lane == 0) {
-      int k = 0, slot = 0;
-      uint32_t use = 0;  // times the slot was filled before
+      int k = pk, slot = pslot;  // continues after the prefetched stages
+      uint32_t use = puse;       // times the slot was filled before
       bool ok = true;
       const uint64_t keep = tc::l2_evict_last();  // every step re-reads the population
       for (; k < n_stages; ++k) {
@@ -502,10 +529,23 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
   }
 }
 
+// Steps after the first are launched with programmatic stream serialization: their CTAs
+// may start while the previous step finishes, and the kernel waits (griddepcontrol.wait)
+// before it reads or writes anything the previous step touches.  Step 0 follows
+// ordinary stream order (its predecessor may be a memset).
 template <class Env>
 cudaError_t launch_xp_tc(const XpTcArgs& a, int grid, size_t smem, cudaStream_t s) {
-  xp_tc_kernel<Env><<<grid, kXpThreads, smem, s>>>(a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kXpThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = a.s > 0 ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, xp_tc_kernel<Env>, a);
 }
 
 template <class Env>
