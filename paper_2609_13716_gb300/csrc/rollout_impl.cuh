@@ -33,19 +33,25 @@ __host__ __device__ inline SmemLayout smem_layout(int M, const MlpDims& m, int s
   return L;
 }
 
+// All of an env's state words are requested at once (one memory latency, not one per
+// word): the loads complete into registers before any is stored.
 template <class S>
 __device__ __forceinline__ void load_state(const uint32_t* __restrict__ g, int64_t n, int64_t e,
                                            S& s) {
+  constexpr int kW = (int)(sizeof(S) / 4);
+  uint32_t v[kW];
+#pragma unroll
+  for (int w = 0; w < kW; ++w) v[w] = __ldg(g + (int64_t)w * n + e);
   uint32_t* p = reinterpret_cast<uint32_t*>(&s);
-#pragma unroll 4
-  for (int w = 0; w < (int)(sizeof(S) / 4); ++w) p[w] = g[(int64_t)w * n + e];
+#pragma unroll
+  for (int w = 0; w < kW; ++w) p[w] = v[w];
 }
 
 template <class S>
 __device__ __forceinline__ void store_state(uint32_t* __restrict__ g, int64_t n, int64_t e,
                                             const S& s) {
   const uint32_t* p = reinterpret_cast<const uint32_t*>(&s);
-#pragma unroll 4
+#pragma unroll
   for (int w = 0; w < (int)(sizeof(S) / 4); ++w) g[(int64_t)w * n + e] = p[w];
 }
 

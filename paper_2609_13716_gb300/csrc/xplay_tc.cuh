@@ -56,7 +56,8 @@ struct XpTcSmem {
   uint32_t w3_off;     // W3, b2, b3 (bulk-copied once L1 is done), within the A region
   uint32_t w3_bytes;
   uint32_t stage_off;  // weight stages
-  uint32_t bits_off;   // per-row observation bits
+  uint32_t bits_off;   // per-row observation bits: the tail of the stage area, dead once the
+                       // observation is expanded (stages overlapping it are filled after that)
   uint32_t total;
   int nst;             // stages
   int spc;             // 8 KB chunks per stage (one bulk copy, one full / empty barrier pair)
@@ -78,12 +79,22 @@ __host__ __device__ inline XpTcSmem xp_tc_layout(const WideDims& w) {
   // Two stages as large as fit: on GB300 a bulk copy takes about the same 500-2000 cycles
   // to land for 8 KB as for 32 KB, and copies in flight barely overlap (measured, also
   // with several issuing warps), so the bytes per copy set the stream's rate.
-  const int slots = (int)((kXpSmemBudget - L.a_bytes - bits) / kWideChunk);
-  L.spc = slots / 2 > kXpMaxChunksPerStage ? kXpMaxChunksPerStage : slots / 2;
-  L.nst = slots / L.spc > kXpMaxStages ? kXpMaxStages : slots / L.spc;
+  // The observation bits share the last stage's space when that buys larger stages (they
+  // are dead once the observation is expanded), else they sit after the stages.
+  auto config = [&](int slots, int& spc, int& nst) {
+    spc = slots / 2 > kXpMaxChunksPerStage ? kXpMaxChunksPerStage : slots / 2;
+    nst = slots / spc > kXpMaxStages ? kXpMaxStages : slots / spc;
+  };
+  int spc_s, nst_s, spc_a, nst_a;
+  config((int)((kXpSmemBudget - L.a_bytes - bits) / kWideChunk), spc_s, nst_s);
+  config((int)((kXpSmemBudget - L.a_bytes) / kWideChunk), spc_a, nst_a);
+  const bool alias = spc_a * nst_a > spc_s * nst_s;
+  L.spc = alias ? spc_a : spc_s;
+  L.nst = alias ? nst_a : nst_s;
   L.stage_off = L.a_bytes;
-  L.bits_off = L.stage_off + (uint32_t)(L.nst * L.spc) * kWideChunk;
-  L.total = L.bits_off + bits;
+  const uint32_t stages_end = L.stage_off + (uint32_t)(L.nst * L.spc) * kWideChunk;
+  L.bits_off = alias ? stages_end - bits : stages_end;
+  L.total = alias ? stages_end : stages_end + bits;
   return L;
 }
 
@@ -168,9 +179,11 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
   // producer state (warp 9, lane 0): next stage, its ring slot, uses of that slot so far
   int pk = 0, pslot = 0;
   uint32_t puse = 0;
+  // stages whose slot ends at or below the observation bits may be filled at once
+  const int free_slots = (int)((L.bits_off - L.stage_off) / stage_bytes);
   if (warp == 9 && lane == 0) {  // the first stages: the population is read-only
     const uint64_t keep = tc::l2_evict_last();
-    for (; pk < n_stages && pk < NST; ++pk, ++pslot) {
+    for (; pk < n_stages && pk < NST && pk < free_slots; ++pk, ++pslot) {
       const uint32_t bytes = (uint32_t)min(SPC, n_chunks - pk * SPC) * kWideChunk;
       tc::mbar_expect_tx(&full_bar[pslot], bytes);
       tc::bulk_g2s_hint(sStage + pslot * stage_bytes, pblk + (int64_t)pk * stage_bytes, bytes, &full_bar[pslot], keep);
@@ -262,9 +275,16 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
     if (lane == 0) {
       int k = pk, slot = pslot;  // continues after the prefetched stages
       uint32_t use = puse;       // times the slot was filled before
-      bool ok = true;
+      bool ok = true, obs_seen = false;
       const uint64_t keep = tc::l2_evict_last();  // every step re-reads the population
       for (; k < n_stages; ++k) {
+        if (use == 0 && slot >= free_slots && !obs_seen) {  // the bits are read by then
+          ok = false;
+          for (int tries = 0; tries < 1000 && !ok && !abort_flag; ++tries)
+            ok = tc::mbar_wait(&obs_bar, 0u, 2000000ull);
+          if (!ok) break;
+          obs_seen = true;
+        }
         if (use > 0) {
           ok = false;
           for (int tries = 0; tries < 1000 && !ok && !abort_flag; ++tries)
