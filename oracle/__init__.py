@@ -153,6 +153,7 @@ def lib() -> C.CDLL:
             L.orc_xplay.argtypes = [C.POINTER(EnvDesc), C.POINTER(Mlp), C.c_int32, C.POINTER(XplayIO)]
             L.orc_xplay.restype = C.c_int32
             L.orc_policy_outputs.argtypes = [C.POINTER(Mlp), _P, C.c_int64, _P]
+            L.orc_xp_stats.argtypes = [_P, C.c_int32, C.c_int32, _P, _P, _P, _P, _P, _P, _P, _P]
             _lib = L
     return _lib
 
@@ -325,4 +326,22 @@ def xplay(d, pols: Policies, seed, step0, ego_ids, tm_ids, P, max_steps, forced=
                  **{k: _ptr(v) for k, v in out.items()})
     rc = lib().orc_xplay(C.byref(d), pols.arr, pols.n, C.byref(io))
     out["rc"] = rc
+    return out
+
+
+def xp_stats(xp, upper=None):
+    """Cross-play matrix consumers (App. B upper bounds, Sec. 3 J_AHT, App. A regret and
+    BRDiv objective) of an fp32 [n_ego][n_tm] matrix; ``upper`` is the prior bound per
+    teammate (default -inf).  Returns fp64 arrays (``brdiv`` None unless square)."""
+    xp = np.ascontiguousarray(xp, np.float32)
+    ne, nt = xp.shape
+    up = np.full(nt, -np.inf) if upper is None else np.array(upper, np.float64)
+    out = dict(norm=np.zeros((ne, nt)), regret=np.zeros((ne, nt)), j_aht=np.zeros(ne),
+               j_norm=np.zeros(ne), max_regret=np.zeros(ne), worst=np.zeros(ne, np.int32))
+    bd = np.zeros(1)
+    lib().orc_xp_stats(_ptr(xp), ne, nt, _ptr(up), _ptr(out["norm"]), _ptr(out["regret"]),
+                       _ptr(out["j_aht"]), _ptr(out["j_norm"]), _ptr(out["max_regret"]),
+                       _ptr(out["worst"]), _ptr(bd) if ne == nt else None)
+    out["upper"] = up
+    out["brdiv"] = float(bd[0]) if ne == nt else None
     return out

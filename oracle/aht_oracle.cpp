@@ -9,6 +9,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <limits>
 #include <thread>
 #include <vector>
 
@@ -845,6 +846,50 @@ extern "C" void orc_gae(const float* r, const float* v, const uint8_t* d, const 
       next_a = a;
       next_v = (double)v[i];
     }
+  }
+}
+
+// ======================================================================================
+// Cross-play matrix consumers (App. B "Upper bound estimation"; Sec. 3 J_AHT; App. A
+// ROTATE regret and BRDiv objective), fp64.
+// ======================================================================================
+extern "C" void orc_xp_stats(const float* xp, int32_t n_ego, int32_t n_tm, double* upper,
+                             double* norm, double* regret, double* j_aht, double* j_norm,
+                             double* max_regret, int32_t* worst, double* brdiv) {
+  // the bound of teammate m rises to any XP score of its column above the recorded value
+  for (int m = 0; m < n_tm; ++m)
+    for (int e = 0; e < n_ego; ++e)
+      if ((double)xp[(int64_t)e * n_tm + m] > upper[m]) upper[m] = (double)xp[(int64_t)e * n_tm + m];
+  std::vector<double> off_row(n_ego, 0.0);
+  for (int e = 0; e < n_ego; ++e) {
+    double sum = 0.0, sum_norm = 0.0, best = 0.0;
+    int arg = 0;
+    for (int m = 0; m < n_tm; ++m) {
+      const double x = (double)xp[(int64_t)e * n_tm + m];
+      const double u = upper[m];
+      const double nr = u > 0.0 ? x / u : std::numeric_limits<double>::quiet_NaN();
+      const double rg = u - x;
+      if (norm) norm[(int64_t)e * n_tm + m] = nr;
+      if (regret) regret[(int64_t)e * n_tm + m] = rg;
+      sum += x;
+      sum_norm += nr;
+      if (m == 0 || rg > best) {
+        best = rg;
+        arg = m;
+      }
+      if (m != e) off_row[e] += x;
+    }
+    if (j_aht) j_aht[e] = sum / n_tm;
+    if (j_norm) j_norm[e] = sum_norm / n_tm;
+    if (max_regret) max_regret[e] = best;
+    if (worst) worst[e] = arg;
+  }
+  if (brdiv && n_ego == n_tm) {
+    const int n = n_ego;
+    double diag = 0.0, off = 0.0;
+    for (int i = 0; i < n; ++i) diag += (double)xp[(int64_t)i * n + i];
+    for (int i = 0; i < n; ++i) off += off_row[i];
+    *brdiv = diag / n - (n > 1 ? off / ((double)n * (n - 1)) : 0.0);
   }
 }
 

@@ -17,7 +17,9 @@
  *     masked categorical sampling (App. B, masked categorical) in fp64;
  *   - PPO's generalised advantage estimate (App. C, "PPO ego") in fp64;
  *   - the ego-by-teammate cross-play return matrix (App. B, "Cross-play matrix
- *     construction"; Sec. 3 J_AHT as its row mean).
+ *     construction"; Sec. 3 J_AHT as its row mean) and what is computed from it:
+ *     best-response upper bounds, normalised returns, cooperative regret and the
+ *     BRDiv cross-play objective (App. B "Upper bound estimation"; App. A).
  * Randomness is Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11) keyed by the seed,
  * with counter (env, step, stream, block).
  *
@@ -220,6 +222,29 @@ typedef struct orc_xplay_io {
 } orc_xplay_io;
 int32_t orc_xplay(const orc_env_desc* d, const orc_mlp* pols, int32_t n_pols,
                   orc_xplay_io* io);
+
+/* ---- Cross-play matrix consumers (fp64) ------------------------------------------ */
+/* xp [n_ego][n_tm]: rows are the policies in the ego seat (best responses, or the ego),
+ * columns the evaluation teammates.
+ *   upper[m] (in/out), App. B "Upper bound estimation": the recorded bound of teammate m
+ *     is replaced by each XP score of column m that exceeds it, rows in order (strict >,
+ *     so a NaN bound stays NaN; pass -inf for "no bound yet").
+ *   norm[e][m] = xp[e][m] / upper[m], the return relative to the best response's
+ *     (Sec. 3; App. B "normalized return"); NaN where upper[m] <= 0.
+ *   regret[e][m] = upper[m] - xp[e][m], the cooperative regret of App. A (ROTATE):
+ *     best-response return minus the return of the row's policy.
+ *   j_aht[e] = (1/n_tm) sum_m xp[e][m], Sec. 3 J_AHT with T_eval uniform; j_norm[e] the
+ *     same mean of norm[e][.] (unrounded fp64 terms).
+ *   max_regret[e] = max_m regret[e][m] (strict >, lowest m wins ties), worst[e] that m.
+ *   brdiv (n_ego == n_tm only; NULL otherwise) = (1/n) sum_i xp[i][i]
+ *     - (1/(n(n-1))) sum_i sum_{j != i} xp[i][j]: matched teammate/best-response returns
+ *     up, mismatched cross-play down (App. A, BRDiv), unit weights; the second term is 0
+ *     for n = 1.
+ * Every sum runs left to right in fp64; the off-diagonal sum adds each row's own partial
+ * sum, rows in order.  Output pointers other than upper may be NULL. */
+void orc_xp_stats(const float* xp, int32_t n_ego, int32_t n_tm, double* upper, double* norm,
+                  double* regret, double* j_aht, double* j_norm, double* max_regret,
+                  int32_t* worst, double* brdiv);
 
 /* Policy outputs z for n observations (u8 [n][obs_dim]) -> [n][n_out]. */
 void orc_policy_outputs(const orc_mlp* p, const uint8_t* obs, int64_t n, double* out);
