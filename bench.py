@@ -400,6 +400,23 @@ def run_xplay(args, aht, W, torch, bf16_peak, names=XPLAY_WORKLOADS):
         torch.cuda.synchronize()
         ms = s.elapsed_time(e) / K
         active = int(steps.sum())
+        # the matrix's consumers (bounds, normalised returns, regret, J_AHT, BRDiv)
+        upper = torch.full((nt,), float("-inf"), device="cuda")
+        so = dict(norm=torch.empty(ne, nt, device="cuda"), regret=torch.empty(ne, nt, device="cuda"),
+                  j_aht=torch.empty(ne, device="cuda"), j_norm=torch.empty(ne, device="cuda"),
+                  max_regret=torch.empty(ne, device="cuda"),
+                  worst_tm=torch.empty(ne, dtype=torch.int32, device="cuda"),
+                  brdiv=torch.empty(1, device="cuda") if ne == nt else None)
+        stream = torch.cuda.current_stream()
+        for _ in range(3):
+            aht.aht_xp_stats(matrix, upper, **so, stream=stream)
+        torch.cuda.synchronize()
+        s.record()
+        for _ in range(K):
+            aht.aht_xp_stats(matrix, upper, **so, stream=stream)
+        e.record()
+        torch.cuda.synchronize()
+        stats_us = s.elapsed_time(e) / K * 1e3
         aht.aht_sync(ctx)
         ctx.close()
         dims = [wl.env.obs_dim, *wl.hidden, wl.env.n_actions]
@@ -411,7 +428,8 @@ def run_xplay(args, aht, W, torch, bf16_peak, names=XPLAY_WORKLOADS):
                      "weights": "bf16" if wl.weight_dtype == W.BF16 else "f32",
                      "roofline": {"bound": "tensor", "achieved": tflops, "peak": bf16_peak,
                                   "unit": "TFLOP/s", "frac": tflops / bf16_peak,
-                                  "flops_per_matrix": flops}}
+                                  "flops_per_matrix": flops},
+                     "xp_stats_us": stats_us}
     return res
 
 

@@ -188,6 +188,42 @@ aht_status aht_xplay_matrix_static(aht_ctx* ctx, const int32_t* ego_ids, int32_t
                                    const int32_t* tm_ids, int32_t n_tm, int32_t envs_per_pair,
                                    int32_t max_steps, float* matrix);
 
+/* Outputs of aht_xp_stats (caller-owned device memory; NULL members not written). */
+typedef struct aht_xp_stats_out {
+  float* norm;        /* [n_ego][n_tm] xp / upper, NaN where upper <= 0 */
+  float* regret;      /* [n_ego][n_tm] upper - xp */
+  float* j_aht;       /* [n_ego] mean of the row (J_AHT, teammates uniform) */
+  float* j_norm;      /* [n_ego] mean of the row of norm (NaN if any bound <= 0) */
+  float* max_regret;  /* [n_ego] largest regret of the row */
+  int32_t* worst_tm;  /* [n_ego] its column (the lowest on ties) */
+  float* brdiv;       /* [1] BRDiv cross-play objective; n_ego == n_tm only */
+} aht_xp_stats_out;
+
+/* What the evaluation and teammate-generation stages compute from a cross-play matrix
+ * (device f32 [n_ego][n_tm], e.g. aht_xplay_matrix's; rows are the policies in the ego
+ * seat -- best responses or the ego -- and columns the evaluation teammates):
+ *   - upper (device f32 [n_tm], in/out): App. B "Upper bound estimation" -- each
+ *     teammate's recorded best-response bound is replaced by any score of its column
+ *     that exceeds it (strict >: pass -inf for "no bound yet"; a NaN bound stays NaN);
+ *   - norm = xp / upper: the return relative to the best response's (Sec. 3, App. B
+ *     "normalized return"), NaN where the bound is <= 0;
+ *   - regret = upper - xp: App. A ROTATE's cooperative regret (best-response return minus
+ *     the return achieved), max_regret / worst_tm its row maximum and that teammate;
+ *   - j_aht: Sec. 3 J_AHT with the teammates weighted uniformly; j_norm the same of norm;
+ *   - brdiv = mean of the diagonal - mean of the off-diagonal entries (App. A BRDiv:
+ *     matched teammate/best-response returns high, mismatched cross-play low; unit
+ *     weights, the off-diagonal term 0 for n = 1).
+ * Arithmetic is fp64, each output rounded to f32 once; the elementwise outputs, bounds
+ * and max_regret/worst_tm are exact, the means are sums in a fixed order (a warp per row,
+ * lanes over every 32nd column, then a shuffle tree), deterministic from call to call and
+ * within one f32 rounding of any other summation order.  One small kernel on
+ * cuda_stream (a cudaStream_t, NULL = default stream); allocates nothing.
+ * Returns AHT_EINVAL for NULL xp/upper/out, n_ego or n_tm outside 1..AHT_XP_STATS_MAX,
+ * or brdiv requested for a non-square matrix. */
+#define AHT_XP_STATS_MAX 2048
+aht_status aht_xp_stats(const float* xp, int32_t n_ego, int32_t n_tm, float* upper,
+                        const aht_xp_stats_out* out, void* cuda_stream);
+
 /* Stateless GAE (App. C "PPO ego"), time-major [T][n_envs] device arrays:
  *   delta_t = r_t + gamma (1 - d_t) V_{t+1} - V_t,
  *   A_t = delta_t + gamma lambda (1 - d_t) A_{t+1},  V_T = v_last,  A_T = 0,

@@ -23,7 +23,8 @@ EXPORTED = ["aht_create", "aht_destroy", "aht_reset", "aht_rollout", "aht_xplay_
             "aht_gae", "aht_step_forced", "aht_policy_forward", "aht_get_state",
             "aht_set_state", "aht_step_counter", "aht_sync", "aht_last_error",
             "aht_status_string", "aht_set_policy", "aht_set_timing", "aht_get_timing",
-            "aht_xplay_matrix_static", "aht_debug_tanh", "aht_debug_expire_wait"]
+            "aht_xplay_matrix_static", "aht_debug_tanh", "aht_debug_expire_wait",
+            "aht_xp_stats"]
 
 
 class AhtError(RuntimeError):
@@ -59,6 +60,12 @@ class XplayOut(C.Structure):
                 ("actions", C.c_void_p)]
 
 
+class XpStatsOut(C.Structure):
+    _fields_ = [("norm", C.c_void_p), ("regret", C.c_void_p), ("j_aht", C.c_void_p),
+                ("j_norm", C.c_void_p), ("max_regret", C.c_void_p), ("worst_tm", C.c_void_p),
+                ("brdiv", C.c_void_p)]
+
+
 class StepOut(C.Structure):
     _fields_ = [("rewards", C.c_void_p), ("team", C.c_void_p), ("dones", C.c_void_p),
                 ("obs", C.c_void_p)]
@@ -90,6 +97,7 @@ def load() -> C.CDLL:
             L.aht_rollout.argtypes = [vp, i32, C.POINTER(i32), i32, i32, C.POINTER(Traj)]
             L.aht_xplay_matrix.argtypes = [vp, C.POINTER(i32), i32, C.POINTER(i32), i32, i32, i32, C.POINTER(XplayOut)]
             L.aht_gae.argtypes = [vp, vp, vp, vp, i64, i32, C.c_float, C.c_float, vp, vp, vp]
+            L.aht_xp_stats.argtypes = [vp, i32, i32, vp, C.POINTER(XpStatsOut), vp]
             L.aht_step_forced.argtypes = [vp, vp, C.POINTER(StepOut)]
             L.aht_policy_forward.argtypes = [vp, i32, vp, i64, vp]
             L.aht_get_state.argtypes = [vp, vp, C.POINTER(C.c_size_t)]
@@ -104,7 +112,7 @@ def load() -> C.CDLL:
             L.aht_last_error.restype = C.c_char_p
             L.aht_status_string.argtypes = [C.c_int]
             L.aht_status_string.restype = C.c_char_p
-            for f in ("aht_create", "aht_reset", "aht_rollout", "aht_xplay_matrix", "aht_gae",
+            for f in ("aht_create", "aht_reset", "aht_rollout", "aht_xplay_matrix", "aht_gae", "aht_xp_stats",
                       "aht_step_forced", "aht_policy_forward", "aht_get_state", "aht_set_state",
                       "aht_sync", "aht_set_policy", "aht_set_timing", "aht_get_timing"):
                 getattr(L, f).restype = C.c_int
@@ -267,6 +275,20 @@ def aht_gae(rewards, values, dones, v_last, gamma, lam, advantages, targets=None
                           _ptr(dones, torch.uint8, (T, N), "dones"), _ptr(v_last, f32, (N,), "v_last"),
                           N, T, gamma, lam, _ptr(advantages, f32, (T, N), "advantages"),
                           _ptr(targets, f32, (T, N), "targets"), _stream(stream)))
+
+
+def aht_xp_stats(xp, upper, norm=None, regret=None, j_aht=None, j_norm=None, max_regret=None,
+                 worst_tm=None, brdiv=None, stream=None):
+    """Cross-play matrix consumers on the device: ``upper`` (f32 [n_tm]) is refined in
+    place; the other outputs are optional preallocated CUDA tensors."""
+    ne, nt = xp.shape
+    f32 = torch.float32
+    out = XpStatsOut(_ptr(norm, f32, (ne, nt), "norm"), _ptr(regret, f32, (ne, nt), "regret"),
+                     _ptr(j_aht, f32, (ne,), "j_aht"), _ptr(j_norm, f32, (ne,), "j_norm"),
+                     _ptr(max_regret, f32, (ne,), "max_regret"),
+                     _ptr(worst_tm, torch.int32, (ne,), "worst_tm"), _ptr(brdiv, f32, (1,), "brdiv"))
+    _check(load().aht_xp_stats(_ptr(xp, f32, (ne, nt), "xp"), ne, nt, _ptr(upper, f32, (nt,), "upper"),
+                               C.byref(out), _stream(stream)))
 
 
 def aht_step_forced(ctx: Context, actions, rewards=None, team=None, dones=None, obs=None):

@@ -960,6 +960,19 @@ aht_status aht_gae(const float* r, const float* v, const uint8_t* d, const float
   return AHT_OK;
 }
 
+aht_status aht_xp_stats(const float* xp, int32_t n_ego, int32_t n_tm, float* upper,
+                        const aht_xp_stats_out* out, void* cuda_stream) {
+  if (!xp || !upper || !out) return fail(AHT_EINVAL, "NULL matrix, bounds or output struct");
+  if (n_ego < 1 || n_tm < 1 || n_ego > AHT_XP_STATS_MAX || n_tm > AHT_XP_STATS_MAX)
+    return fail(AHT_EINVAL, "n_ego and n_tm must be in 1..AHT_XP_STATS_MAX");
+  if (out->brdiv && n_ego != n_tm) return fail(AHT_EINVAL, "brdiv needs a square matrix");
+  static_assert(AHT_XP_STATS_MAX == kXpStatsMax, "cross-play statistics limit");
+  XpStatsArgs a{xp, n_ego, n_tm, upper, out->norm, out->regret, out->j_aht, out->j_norm,
+                out->max_regret, out->brdiv, out->worst_tm};
+  AHT_CUDA(launch_xp_stats(a, (cudaStream_t)cuda_stream));
+  return AHT_OK;
+}
+
 aht_status aht_debug_tanh(const float* x, float* y, int64_t n, void* cuda_stream) {
   if (!x || !y || n < 1) return fail(AHT_EINVAL, "NULL array or n < 1");
   AHT_CUDA(launch_tanh_probe(x, y, n, (cudaStream_t)cuda_stream));

@@ -216,4 +216,15 @@ cudaError_t launch_gae(const float* r, const float* v, const uint8_t* d, const f
 cudaError_t launch_xp_reduce(const float* returns, int64_t n_pairs, int32_t P, float* matrix,
                              cudaStream_t);
 
+// Cross-play matrix consumers (misc.cu): one CTA; n_ego, n_tm <= kXpStatsMax.
+constexpr int kXpStatsMax = 2048;
+struct XpStatsArgs {
+  const float* xp;  // [n_ego][n_tm]
+  int32_t n_ego, n_tm;
+  float* upper;     // [n_tm] in/out
+  float *norm, *regret, *j_aht, *j_norm, *max_regret, *brdiv;  // each may be null
+  int32_t* worst;
+};
+cudaError_t launch_xp_stats(const XpStatsArgs&, cudaStream_t);
+
 }  // namespace aht

@@ -1,5 +1,7 @@
-// misc.cu -- env-independent kernels: teammate grouping, GAE, cross-play reduction and the
-// standalone policy forward.
+// misc.cu -- env-independent kernels: teammate grouping, GAE, cross-play reduction, the
+// cross-play matrix consumers and the standalone policy forward.
+#include <climits>
+
 #include "kernels.h"
 #include "mlp_simt.cuh"
 #include "rollout_impl.cuh"
@@ -89,6 +91,107 @@ __global__ void xp_reduce_kernel(const float* __restrict__ returns, int32_t P,
 cudaError_t launch_xp_reduce(const float* returns, int64_t n_pairs, int32_t P, float* matrix,
                              cudaStream_t s) {
   xp_reduce_kernel<<<(unsigned)n_pairs, 256, 0, s>>>(returns, P, matrix);
+  return cudaGetLastError();
+}
+
+// ---- cross-play matrix consumers -------------------------------------------------------
+// xp [n_ego][n_tm]: rows are the policies in the ego seat (best responses, or the ego),
+// columns the evaluation teammates.  App. B "Upper bound estimation": each teammate's
+// recorded bound is raised to any cross-play score that exceeds it.  Returns are reported
+// relative to that bound (Sec. 3, the best response's return); J_AHT is the row mean
+// (Sec. 3, teammates uniform); the cooperative regret is bound minus return (App. A,
+// ROTATE); BRDiv's cross-play objective is the matched (diagonal) mean minus the
+// mismatched mean (App. A).  One CTA of 1024 threads: a thread per column for the bounds
+// (rows in order), then a warp per row -- lanes take every 32nd column, in fp64, and the
+// row's sums and its largest regret are combined by shuffles -- then warp 0 for the BRDiv
+// sums.  FP64 is slow on this part, so the divisions run across lanes, not in a chain.
+constexpr int kXpStatsThreads = 1024;
+
+__device__ __forceinline__ double warp_sum_f64(double v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = __dadd_rn(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
+  return v;
+}
+
+__global__ void __launch_bounds__(kXpStatsThreads) xp_stats_kernel(const XpStatsArgs a) {
+  __shared__ float up[kXpStatsMax];
+  __shared__ double off_row[kXpStatsMax];
+  const int ne = a.n_ego, nt = a.n_tm;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, n_warps = blockDim.x >> 5;
+  for (int m = threadIdx.x; m < nt; m += blockDim.x) {
+    float u = a.upper[m];
+    for (int e = 0; e < ne; ++e) {
+      const float x = a.xp[(int64_t)e * nt + m];
+      if (x > u) u = x;  // strict: a NaN bound is never exceeded
+    }
+    up[m] = u;
+    a.upper[m] = u;
+  }
+  __syncthreads();
+  const double nan = __longlong_as_double(0x7FF8000000000000ll);
+  for (int e = warp; e < ne; e += n_warps) {
+    double sum = 0.0, sum_norm = 0.0, off = 0.0, best = -INFINITY;
+    int arg = INT_MAX;  // this lane's largest non-NaN regret, its first column
+    for (int m = lane; m < nt; m += 32) {
+      const int64_t i = (int64_t)e * nt + m;
+      const double x = (double)a.xp[i], u = (double)up[m];
+      const double nr = u > 0.0 ? __ddiv_rn(x, u) : nan;
+      const double rg = __dsub_rn(u, x);
+      if (a.norm) a.norm[i] = __double2float_rn(nr);
+      if (a.regret) a.regret[i] = __double2float_rn(rg);
+      sum = __dadd_rn(sum, x);
+      sum_norm = __dadd_rn(sum_norm, nr);
+      if (rg > best) {
+        best = rg;
+        arg = m;
+      }
+      if (m != e) off = __dadd_rn(off, x);
+    }
+    sum = warp_sum_f64(sum);
+    sum_norm = warp_sum_f64(sum_norm);
+    off = warp_sum_f64(off);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const double ob = __shfl_xor_sync(0xFFFFFFFFu, best, o);
+      const int oa = __shfl_xor_sync(0xFFFFFFFFu, arg, o);
+      if (ob > best || (ob == best && oa < arg)) {
+        best = ob;
+        arg = oa;
+      }
+    }
+    if (lane == 0) {
+      // the scan's reading: start at column 0 and move on to strictly larger regrets, so
+      // a NaN at column 0 stays (the bound of teammate 0 is NaN) and later NaNs never win
+      const double rg0 = __dsub_rn((double)up[0], (double)a.xp[(int64_t)e * nt]);
+      if (rg0 != rg0 || arg == INT_MAX) {
+        best = rg0;
+        arg = 0;
+      }
+      if (a.j_aht) a.j_aht[e] = __double2float_rn(__ddiv_rn(sum, (double)nt));
+      if (a.j_norm) a.j_norm[e] = __double2float_rn(__ddiv_rn(sum_norm, (double)nt));
+      if (a.max_regret) a.max_regret[e] = __double2float_rn(best);
+      if (a.worst) a.worst[e] = arg;
+      off_row[e] = off;
+    }
+  }
+  __syncthreads();
+  if (warp == 0 && a.brdiv && ne == nt) {
+    double diag = 0.0, off = 0.0;
+    for (int i = lane; i < ne; i += 32) {
+      diag = __dadd_rn(diag, (double)a.xp[(int64_t)i * nt + i]);
+      off = __dadd_rn(off, off_row[i]);
+    }
+    diag = warp_sum_f64(diag);
+    off = warp_sum_f64(off);
+    if (lane == 0) {
+      const double mis = ne > 1 ? __ddiv_rn(off, (double)ne * (double)(ne - 1)) : 0.0;
+      *a.brdiv = __double2float_rn(__dsub_rn(__ddiv_rn(diag, (double)ne), mis));
+    }
+  }
+}
+
+cudaError_t launch_xp_stats(const XpStatsArgs& a, cudaStream_t s) {
+  xp_stats_kernel<<<1, kXpStatsThreads, 0, s>>>(a);
   return cudaGetLastError();
 }
 

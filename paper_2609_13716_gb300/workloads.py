@@ -155,3 +155,19 @@ def random_actions(seed: int, shape, n_actions: int) -> np.ndarray:
     """Uniform forced actions for env-rule parity tests."""
     rng = np.random.Generator(np.random.Philox(seed))
     return rng.integers(0, n_actions, size=shape, dtype=np.uint8)
+
+
+def xp_matrix(seed: int, n_ego: int, n_tm: int, scale: float = 1.0,
+              quantum: float = 0.0) -> np.ndarray:
+    """Synthetic cross-play return matrix [n_ego][n_tm] (f32) shaped like the paper's (App.
+    B figures): entries uniform in [0, 0.6) * scale, the matched pairs of the leading
+    diagonal 0.4 * scale higher.  ``quantum`` > 0 rounds every entry to a multiple of it
+    (integer game scores averaged over a fixed number of episodes), which makes ties."""
+    rng = np.random.Generator(np.random.Philox(seed))
+    m = rng.uniform(0.0, 0.6, (n_ego, n_tm))
+    k = min(n_ego, n_tm)
+    m[np.arange(k), np.arange(k)] += 0.4
+    m *= scale
+    if quantum > 0:
+        m = np.round(m / quantum) * quantum
+    return m.astype(np.float32)

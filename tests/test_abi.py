@@ -56,3 +56,11 @@ def test_host_validation_needs_no_gpu(lib):
     L.aht_debug_expire_wait.argtypes = [C.c_void_p, C.c_int64]
     assert L.aht_debug_expire_wait(None, 1000) == aht.AHT_EINVAL
 
+    out = aht.XpStatsOut()
+    fake = C.c_void_p(16)  # never dereferenced: every case below fails a host check
+    assert L.aht_xp_stats(None, 2, 2, fake, C.byref(out), None) == aht.AHT_EINVAL
+    assert L.aht_xp_stats(fake, 0, 2, fake, C.byref(out), None) == aht.AHT_EINVAL
+    assert L.aht_xp_stats(fake, 2, 2049, fake, C.byref(out), None) == aht.AHT_EINVAL
+    out.brdiv = 16
+    assert L.aht_xp_stats(fake, 2, 3, fake, C.byref(out), None) == aht.AHT_EINVAL
+    assert b"square" in L.aht_last_error()
