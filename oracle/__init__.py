@@ -21,7 +21,7 @@ import numpy as np
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _BUILD = os.path.join(_HERE, "_build")
 _SO = os.path.join(_BUILD, "liboracle.so")
-_SRC = [os.path.join(_HERE, "aht_oracle.cpp")]
+_SRC = [os.path.join(_HERE, "aht_oracle.cpp"), os.path.join(_HERE, "ppo_oracle.cpp")]
 _HDR = os.path.join(_HERE, "aht_oracle.h")
 _lock = threading.Lock()
 _lib = None
@@ -90,6 +90,23 @@ class Mlp(C.Structure):
 _P = C.c_void_p
 
 
+class PpoNet(C.Structure):
+    _fields_ = [("obs_dim", C.c_int32), ("h0", C.c_int32), ("h1", C.c_int32), ("n_act", C.c_int32)]
+
+
+class PpoHp(C.Structure):
+    _fields_ = [("epochs", C.c_int32), ("minibatches", C.c_int32), ("lr", C.c_double),
+                ("clip_eps", C.c_double), ("vf_coef", C.c_double), ("ent_coef", C.c_double),
+                ("max_grad_norm", C.c_double), ("adam_b1", C.c_double), ("adam_b2", C.c_double),
+                ("adam_eps", C.c_double), ("seed", C.c_uint64), ("epoch0", C.c_int64),
+                ("round_bf16", C.c_int32)]
+
+
+class PpoBatch(C.Structure):
+    _fields_ = [("obs", C.c_void_p), ("actions", C.c_void_p), ("logp", C.c_void_p),
+                ("values", C.c_void_p), ("advantages", C.c_void_p), ("targets", C.c_void_p)]
+
+
 class RolloutIO(C.Structure):
     _fields_ = [("seed", C.c_uint64), ("n_envs", C.c_int64), ("step0", C.c_int64),
                 ("T", C.c_int32), ("ego_id", C.c_int32), ("pool", _P), ("pool_size", C.c_int32),
@@ -153,6 +170,17 @@ def lib() -> C.CDLL:
             L.orc_xplay.argtypes = [C.POINTER(EnvDesc), C.POINTER(Mlp), C.c_int32, C.POINTER(XplayIO)]
             L.orc_xplay.restype = C.c_int32
             L.orc_policy_outputs.argtypes = [C.POINTER(Mlp), _P, C.c_int64, _P]
+            L.orc_ppo_n_params.argtypes = [C.POINTER(PpoNet)]
+            L.orc_ppo_n_params.restype = C.c_int64
+            L.orc_bf16_round.argtypes = [C.c_double]
+            L.orc_bf16_round.restype = C.c_double
+            L.orc_perm_index.argtypes = [C.c_uint64, C.c_int64, C.c_int64, C.c_int64]
+            L.orc_perm_index.restype = C.c_int64
+            L.orc_ppo_grad.argtypes = [C.POINTER(PpoNet), _P, C.POINTER(PpoBatch), _P, C.c_int64,
+                                       C.POINTER(PpoHp), _P, _P, C.c_int32]
+            L.orc_adam_step.argtypes = [C.c_int64, _P, _P, _P, _P, _P, C.POINTER(PpoHp)]
+            L.orc_ppo_update.argtypes = [C.POINTER(PpoNet), _P, _P, _P, _P, C.POINTER(PpoBatch),
+                                         C.c_int64, C.POINTER(PpoHp), _P, C.c_int32]
             L.orc_xp_stats.argtypes = [_P, C.c_int32, C.c_int32, _P, _P, _P, _P, _P, _P, _P, _P]
             _lib = L
     return _lib
@@ -345,3 +373,96 @@ def xp_stats(xp, upper=None):
     out["upper"] = up
     out["brdiv"] = float(bd[0]) if ne == nt else None
     return out
+
+
+# ---------------------------------------------------------------------------------
+# PPO ego update (ppo_oracle.cpp)
+# ---------------------------------------------------------------------------------
+PPO_DEFAULTS = dict(epochs=4, minibatches=4, lr=2.5e-4, clip_eps=0.2, vf_coef=0.5, ent_coef=0.01,
+                    max_grad_norm=0.5, adam_b1=0.9, adam_b2=0.999, adam_eps=1e-5, seed=0,
+                    epoch0=0, round_bf16=1)
+
+
+def ppo_hp(**kw):
+    d = dict(PPO_DEFAULTS)
+    d.update(kw)
+    return PpoHp(**d)
+
+
+def ppo_net(obs_dim, h0, h1, n_act):
+    return PpoNet(obs_dim, h0, h1, n_act)
+
+
+def ppo_n_params(net):
+    return int(lib().orc_ppo_n_params(C.byref(net)))
+
+
+def flat_params(layers):
+    """[(W1, b1), (W2, b2), (W3, b3)] -> one fp64 vector in the oracle's order."""
+    return np.concatenate([np.asarray(a, np.float64).ravel() for wb in layers for a in wb])
+
+
+def unflat_params(net, p):
+    D, H0, H1, O = net.obs_dim, net.h0, net.h1, net.n_act + 1
+    sizes = [(H0, D), (H0,), (H1, H0), (H1,), (O, H1), (O,)]
+    out, i = [], 0
+    for sh in sizes:
+        n = int(np.prod(sh))
+        out.append(np.asarray(p[i:i + n]).reshape(sh))
+        i += n
+    return [(out[0], out[1]), (out[2], out[3]), (out[4], out[5])]
+
+
+class PpoBatchNp:
+    """Flattened (time-major) trajectory arrays, kept alive for the C structure."""
+
+    def __init__(self, obs, actions, logp, values, advantages, targets):
+        D = obs.shape[-1]
+        self.obs = np.ascontiguousarray(obs, np.uint8).reshape(-1, D)
+        self.actions = np.ascontiguousarray(actions, np.uint8).ravel()
+        self.logp = np.ascontiguousarray(logp, np.float32).ravel()
+        self.values = np.ascontiguousarray(values, np.float32).ravel()
+        self.advantages = np.ascontiguousarray(advantages, np.float32).ravel()
+        self.targets = np.ascontiguousarray(targets, np.float32).ravel()
+        self.S = self.actions.size
+        self.c = PpoBatch(*(_ptr(a) for a in (self.obs, self.actions, self.logp, self.values,
+                                               self.advantages, self.targets)))
+
+
+def perm_index(seed, epoch, S, x):
+    return int(lib().orc_perm_index(seed, epoch, S, x))
+
+
+def perm(seed, epoch, S):
+    return np.array([perm_index(seed, epoch, S, x) for x in range(S)], np.int64)
+
+
+def bf16_round(w):
+    return float(lib().orc_bf16_round(float(w)))
+
+
+def ppo_grad(net, params, batch: PpoBatchNp, idx, hp, n_threads=1):
+    params = np.ascontiguousarray(params, np.float64)
+    idx = np.ascontiguousarray(idx, np.int64)
+    grad = np.zeros(ppo_n_params(net))
+    stats = np.zeros(6)
+    lib().orc_ppo_grad(C.byref(net), _ptr(params), C.byref(batch.c), _ptr(idx), len(idx),
+                       C.byref(hp), _ptr(grad), _ptr(stats), n_threads)
+    return grad, stats
+
+
+def adam_step(params, m, v, t, grad, hp):
+    """In place on params, m, v, grad (fp64 arrays); returns the new step count."""
+    tt = C.c_int64(t)
+    lib().orc_adam_step(len(params), _ptr(params), _ptr(m), _ptr(v), C.byref(tt), _ptr(grad),
+                        C.byref(hp))
+    return tt.value
+
+
+def ppo_update(net, params, m, v, t, batch: PpoBatchNp, hp, n_threads=1):
+    """In place on params, m, v (fp64); returns (t, stats [E*M][6])."""
+    tt = C.c_int64(t)
+    stats = np.zeros((hp.epochs * hp.minibatches, 6))
+    lib().orc_ppo_update(C.byref(net), _ptr(params), _ptr(m), _ptr(v), C.byref(tt),
+                         C.byref(batch.c), batch.S, C.byref(hp), _ptr(stats), n_threads)
+    return tt.value, stats

@@ -19,7 +19,9 @@
  *   - the ego-by-teammate cross-play return matrix (App. B, "Cross-play matrix
  *     construction"; Sec. 3 J_AHT as its row mean) and what is computed from it:
  *     best-response upper bounds, normalised returns, cooperative regret and the
- *     BRDiv cross-play objective (App. B "Upper bound estimation"; App. A).
+ *     BRDiv cross-play objective (App. B "Upper bound estimation"; App. A);
+ *   - the PPO ego update (App. C "PPO ego"): clipped-surrogate loss, its gradient, and
+ *     Adam over permuted minibatches of a collected trajectory.
  * Randomness is Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11) keyed by the seed,
  * with counter (env, step, stream, block).
  *
@@ -245,6 +247,56 @@ int32_t orc_xplay(const orc_env_desc* d, const orc_mlp* pols, int32_t n_pols,
 void orc_xp_stats(const float* xp, int32_t n_ego, int32_t n_tm, double* upper, double* norm,
                   double* regret, double* j_aht, double* j_norm, double* max_regret,
                   int32_t* worst, double* brdiv);
+
+/* ---- PPO ego update (fp64; ppo_oracle.cpp) -------------------------------------- */
+/* App. C "PPO ego": PPO (Schulman et al. 2017) with the clipped surrogate, a clipped
+ * value loss and an entropy bonus, per-minibatch advantage normalisation, global-norm
+ * gradient clipping and Adam (Kingma & Ba 2015).  Readings in DESIGN.md "PPO update".
+ * Parameters are one flat array: W1 [h0][obs_dim], b1 [h0], W2 [h1][h0], b2 [h1],
+ * W3 [n_act + 1][h1], b3 [n_act + 1] (the last output row is the value estimate). */
+enum { ORC_STREAM_PERMUTE = 4 };
+typedef struct orc_ppo_net {
+  int32_t obs_dim, h0, h1, n_act;
+} orc_ppo_net;
+typedef struct orc_ppo_hp {
+  int32_t epochs, minibatches;
+  double lr, clip_eps, vf_coef, ent_coef, max_grad_norm, adam_b1, adam_b2, adam_eps;
+  uint64_t seed;      /* minibatch permutation key */
+  int64_t epoch0;     /* permutation counter of the first epoch */
+  int32_t round_bf16; /* 1: the forward and backward use bf16(W1), bf16(W2) */
+} orc_ppo_hp;
+/* Samples s in [0, S): the [T][N] trajectory arrays flattened time-major (s = t*N + n). */
+typedef struct orc_ppo_batch {
+  const uint8_t* obs;       /* [S][obs_dim] */
+  const uint8_t* actions;   /* [S] */
+  const float* logp;        /* [S] log-probability under the rollout policy */
+  const float* values;      /* [S] value estimate of the rollout */
+  const float* advantages;  /* [S] GAE */
+  const float* targets;     /* [S] value targets (advantages + values) */
+} orc_ppo_batch;
+int64_t orc_ppo_n_params(const orc_ppo_net* n);
+/* bf16 nearest-even of fp32(w). */
+double orc_bf16_round(double w);
+/* pi_epoch(x) for x in [0, S): a 4-round Feistel network on the smallest w >= 2 bits
+ * with 2^w >= S (high half L = w - w/2 bits, low half R = w/2 bits; round r XORs the low
+ * half's Philox word into L for even r, the high half's into R for odd r, Philox key
+ * (seed lo, seed hi), counter (other half, epoch, ORC_STREAM_PERMUTE, r), word 0), walked
+ * until the value falls below S.  Minibatch b of epoch e is pi_e(b*B .. (b+1)*B - 1). */
+int64_t orc_perm_index(uint64_t seed, int64_t epoch, int64_t S, int64_t x);
+/* Gradient of the minibatch loss at params over the B samples idx[] (the loss is the
+ * mean over them); stats (may be NULL) = {loss, policy loss, value loss, entropy,
+ * mean(logp_old - logp), fraction with |ratio - 1| > clip_eps}. */
+void orc_ppo_grad(const orc_ppo_net* n, const double* params, const orc_ppo_batch* tb,
+                  const int64_t* idx, int64_t B, const orc_ppo_hp* hp, double* grad,
+                  double* stats, int32_t n_threads);
+/* One optimiser step: clip grad (in place) to global norm max_grad_norm (if > 0), t += 1,
+ * Adam with bias correction, params -= lr m_hat / (sqrt(v_hat) + adam_eps). */
+void orc_adam_step(int64_t n_params, double* params, double* m, double* v, int64_t* t,
+                   double* grad, const orc_ppo_hp* hp);
+/* epochs x minibatches steps over S samples (B = S / minibatches); stats [E*M][6]. */
+void orc_ppo_update(const orc_ppo_net* n, double* params, double* m, double* v, int64_t* t,
+                    const orc_ppo_batch* tb, int64_t S, const orc_ppo_hp* hp, double* stats,
+                    int32_t n_threads);
 
 /* Policy outputs z for n observations (u8 [n][obs_dim]) -> [n][n_out]. */
 void orc_policy_outputs(const orc_mlp* p, const uint8_t* obs, int64_t n, double* out);
