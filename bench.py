@@ -43,6 +43,7 @@ def parse():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-xplay", action="store_true")
+    p.add_argument("--no-ppo", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     # profiling of a smaller case of the same kernel (not a bench line)
     p.add_argument("--n-envs", type=int, default=None)
@@ -352,6 +353,10 @@ def run_ours(args):
             "gpu_launches": 3 * args.steps,
             "clocks": clocks.summary(),
         }
+    if not args.no_ppo:
+        pu = run_ppo_update(args, aht, wl, pop_np, traj, torch, bf16_peak, stream)
+        if line is not None:
+            line["ppo_update"] = pu
     if not args.no_xplay:
         xp = run_xplay(args, aht, W, torch, bf16_peak)
         if line is not None:
@@ -365,6 +370,60 @@ def run_ours(args):
     ctx.close()
     if world > 1:
         dist.destroy_process_group()
+
+
+PPO_FLOPS_PER_SAMPLE = 204032   # forward 84,736 + backward 119,296 (dW1, dW2, dh1, dW3, dh2)
+
+
+def run_ppo_update(args, aht, wl, pop_np, traj, torch, bf16_peak, stream):
+    """The PPO ego update (4 epochs x 4 minibatches, Adam) over the trajectory the last
+    timed rollout wrote: ms per update, sample-epochs/s and the fraction of the tensor
+    roofline of its algorithmic FLOPs; beside it the fp64 oracle's gradient rate on a
+    bounded sample of the same trajectory."""
+    import numpy as np
+    T, N = traj["actions"].shape
+    layers = [(torch.from_numpy(np.asarray(Wt, np.float32)), torch.from_numpy(np.asarray(b, np.float32)))
+              for Wt, b in pop_np[wl.ego_id]]
+    L = aht.aht_learner_create(wl.env.obs_dim, wl.env.n_actions, layers, stream=stream)
+    start = [torch.empty(L.n_params, device="cuda") for _ in range(3)]
+    aht.aht_learner_get(L, *start)
+    for _ in range(2):
+        aht.aht_ppo_update(L, traj)
+    torch.cuda.synchronize()
+    K = max(3, min(args.steps, 10))
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    ev[0].record(stream)
+    for _ in range(K):
+        aht.aht_ppo_update(L, traj)
+    ev[1].record(stream)
+    torch.cuda.synchronize()
+    aht.aht_learner_sync(L)
+    ms = ev[0].elapsed_time(ev[1]) / K
+    E, M = L.cfg["epochs"], L.cfg["minibatches"]
+    samples = T * N * E
+    tflops = samples * PPO_FLOPS_PER_SAMPLE / (ms * 1e-3) / 1e12
+    res = {"workload": f"ppo_update_lbf7x7_{N}x{T}_{E}ep_{M}mb", "ms_per_update": ms,
+           "sample_epochs_per_s": samples / (ms * 1e-3),
+           "gpu_launches_per_update": 2 + 3 * E * M,
+           "roofline": {"bound": "tensor", "achieved": tflops, "peak": bf16_peak, "unit": "TFLOP/s",
+                        "frac": tflops / bf16_peak, "flops_per_update": samples * PPO_FLOPS_PER_SAMPLE}}
+    L.close()
+    if not args.no_cpu_baseline:
+        import oracle as O
+        b = {k: traj[k][:, :1024].contiguous().cpu().numpy() for k in
+             ("obs", "actions", "logp", "values", "advantages", "targets")}
+        batch = O.PpoBatchNp(**b)
+        net = O.ppo_net(wl.env.obs_dim, wl.hidden[0], wl.hidden[1], wl.env.n_actions)
+        p0 = O.flat_params([(np.asarray(Wt, np.float64), np.asarray(bb, np.float64)) for Wt, bb in pop_np[wl.ego_id]])
+        threads = os.cpu_count() or 1
+        n = min(batch.S, 32768)
+        idx = np.arange(n, dtype=np.int64)
+        t0 = time.perf_counter()
+        O.ppo_grad(net, p0, batch, idx, O.ppo_hp(), n_threads=threads)
+        dt = time.perf_counter() - t0
+        res["cpu_baseline"] = {"value": n / dt, "unit": "sample-epochs/s", "cores": threads, "kind": "oracle",
+                               "sample": f"gradient of one {n}-sample minibatch of the same trajectory, fp64"}
+    return res
 
 
 XPLAY_WORKLOADS = ("lbf7x7_xplay_8x16x256", "overcooked5x4_xplay_8x8x64", "hanabi_xplay_16x16x32")

@@ -224,6 +224,83 @@ typedef struct aht_xp_stats_out {
 aht_status aht_xp_stats(const float* xp, int32_t n_ego, int32_t n_tm, float* upper,
                         const aht_xp_stats_out* out, void* cuda_stream);
 
+/* ---- PPO ego update (App. C "PPO ego") ----------------------------------------------
+ * The paper trains the ego with PPO (Schulman et al. 2017) against its teammates and
+ * states no loss details; the update implemented is that paper's clipped surrogate:
+ *   per sample  rho = exp(logp(a) - logp_old),  A_n = (A - mean_mb A) / (std_mb A + 1e-8),
+ *   L = -min(rho A_n, clip(rho, 1 - clip_eps, 1 + clip_eps) A_n)
+ *       + vf_coef * 0.5 max((V - R)^2, (V_old + clip(V - V_old, -clip_eps, clip_eps) - R)^2)
+ *       - ent_coef * H(pi),
+ * averaged over each minibatch (mean and population std of A over the minibatch, R the
+ * targets); the gradient is clipped to global norm max_grad_norm (if > 0) and applied by
+ * Adam (Kingma & Ba 2015; m_hat / (sqrt(v_hat) + adam_eps), bias-corrected).  Each of
+ * `epochs` epochs draws a pseudorandom permutation pi of the S = T * n_envs samples
+ * (flattened time-major, s = t * n_envs + env) and splits it into `minibatches` runs of
+ * B = S / minibatches: a 4-round Feistel network on w bits (2^w >= S, w >= 2; high half
+ * w - w/2 bits, low half w/2 bits; round r XORs word 0 of Philox(key = seed, counter =
+ * (other half, epoch counter, 4, r)) into the high half for even r, the low half for odd
+ * r), walked until the value is below S.  The epoch counter of epoch e of the k-th update
+ * of a learner is k * epochs + e.
+ * The network is the actor-critic ego of aht_pop_desc: obs_dim -> 128 -> 128 ->
+ * n_actions + 1 (the last output is the value).  The learner keeps fp32 master weights
+ * and Adam moments; the forward and backward of the update use bf16 copies of W1 and W2
+ * (the precision the bf16 rollout runs) and fp32 for W3 and the biases; activations and
+ * gradients are carried as two bf16 (hi + lo) through fp32-accumulating tensor cores. */
+typedef struct aht_ppo_config {
+  int32_t epochs;         /* >= 1 (4) */
+  int32_t minibatches;    /* >= 1 (4) */
+  float lr;               /* Adam step size (2.5e-4) */
+  float clip_eps;         /* ratio and value clip (0.2) */
+  float vf_coef;          /* value-loss weight (0.5) */
+  float ent_coef;         /* entropy-bonus weight (0.01) */
+  float max_grad_norm;    /* global-norm clip, <= 0 disables (0.5) */
+  float adam_b1, adam_b2, adam_eps;  /* (0.9, 0.999, 1e-5) */
+  uint64_t seed;          /* key of the minibatch permutations */
+} aht_ppo_config;
+
+typedef struct aht_learner aht_learner; /* opaque, library-owned */
+
+/* Creates a PPO learner for the actor-critic ego (W[l], b[l] fp32 of the aht_pop_desc
+ * shapes with hidden0 = hidden1 = 128 and the value row, host or device memory; copied).
+ * obs_dim 1..207 and a multiple of 4, n_actions 1..7.  Allocates all device memory the
+ * learner uses (master weights, Adam moments, the packed bf16 copy, per-SM gradient
+ * partials of about 27 MB); the other learner calls allocate nothing.  Work runs on
+ * cuda_stream (a cudaStream_t, NULL = default stream). */
+aht_status aht_learner_create(int32_t obs_dim, int32_t n_actions, const float* const* W,
+                              const float* const* b, const aht_ppo_config* cfg,
+                              void* cuda_stream, aht_learner** out);
+void aht_learner_destroy(aht_learner* L);
+/* Number of parameters: 128 obs_dim + 128 + 128*128 + 128 + (n_actions + 1)(128 + 1). */
+int64_t aht_learner_n_params(const aht_learner* L);
+
+/* One PPO update over a trajectory of aht_rollout (device arrays obs, actions, logp,
+ * values, advantages and targets of traj, [T][n_envs]; the other members are not read):
+ * epochs x minibatches optimiser steps.  stats (device f32 [epochs*minibatches][6], or
+ * NULL) receives per step the minibatch means of {loss, policy loss, value loss, entropy,
+ * logp_old - logp, |rho - 1| > clip_eps}.  Requires T * n_envs < 2^31 and a multiple of
+ * 64 * minibatches.  Asynchronous; aht_learner_sync reports device errors. */
+aht_status aht_ppo_update(aht_learner* L, const aht_traj* traj, int64_t n_envs, int32_t T,
+                          float* stats);
+/* The gradient (device f32 [n_params], before clipping) and stats (device f32 [6], or
+ * NULL) of minibatch `minibatch` of epoch `epoch` of the learner's next update, at its
+ * current weights; changes nothing.  Same requirements as aht_ppo_update. */
+aht_status aht_ppo_grad(aht_learner* L, const aht_traj* traj, int64_t n_envs, int32_t T,
+                        int32_t epoch, int32_t minibatch, float* grad, float* stats);
+/* Copies out / replaces the learner state (device f32 [n_params] arrays, each may be
+ * NULL on get; params required on set, NULL moments on set mean zero): flat parameter
+ * order W1, b1, W2, b2, W3, b3 (row-major), the Adam moments, step count t and the
+ * number of completed updates (the permutation epoch counter is updates * epochs + e). */
+aht_status aht_learner_get(aht_learner* L, float* params, float* adam_m, float* adam_v,
+                           int64_t* t, int64_t* updates);
+aht_status aht_learner_set(aht_learner* L, const float* params, const float* adam_m,
+                           const float* adam_v, int64_t t, int64_t updates);
+/* Writes the learner's current weights into policy `policy` of ctx (aht_set_policy with
+ * fp32 weights; the ctx's own packing rounds them to its weight type). */
+aht_status aht_learner_push(aht_learner* L, aht_ctx* ctx, int32_t policy);
+/* Synchronises the learner's stream; AHT_ETIMEOUT if a bounded wait of its kernels
+ * expired (the status word is then cleared). */
+aht_status aht_learner_sync(aht_learner* L);
+
 /* Stateless GAE (App. C "PPO ego"), time-major [T][n_envs] device arrays:
  *   delta_t = r_t + gamma (1 - d_t) V_{t+1} - V_t,
  *   A_t = delta_t + gamma lambda (1 - d_t) A_{t+1},  V_T = v_last,  A_T = 0,

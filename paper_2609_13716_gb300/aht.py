@@ -24,7 +24,9 @@ EXPORTED = ["aht_create", "aht_destroy", "aht_reset", "aht_rollout", "aht_xplay_
             "aht_set_state", "aht_step_counter", "aht_sync", "aht_last_error",
             "aht_status_string", "aht_set_policy", "aht_set_timing", "aht_get_timing",
             "aht_xplay_matrix_static", "aht_debug_tanh", "aht_debug_expire_wait",
-            "aht_xp_stats"]
+            "aht_xp_stats", "aht_learner_create", "aht_learner_destroy", "aht_learner_n_params",
+            "aht_ppo_update", "aht_ppo_grad", "aht_learner_get", "aht_learner_set",
+            "aht_learner_push", "aht_learner_sync"]
 
 
 class AhtError(RuntimeError):
@@ -66,6 +68,17 @@ class XpStatsOut(C.Structure):
                 ("brdiv", C.c_void_p)]
 
 
+class PpoConfig(C.Structure):
+    _fields_ = [("epochs", C.c_int32), ("minibatches", C.c_int32), ("lr", C.c_float),
+                ("clip_eps", C.c_float), ("vf_coef", C.c_float), ("ent_coef", C.c_float),
+                ("max_grad_norm", C.c_float), ("adam_b1", C.c_float), ("adam_b2", C.c_float),
+                ("adam_eps", C.c_float), ("seed", C.c_uint64)]
+
+
+PPO_DEFAULTS = dict(epochs=4, minibatches=4, lr=2.5e-4, clip_eps=0.2, vf_coef=0.5, ent_coef=0.01,
+                    max_grad_norm=0.5, adam_b1=0.9, adam_b2=0.999, adam_eps=1e-5, seed=0)
+
+
 class StepOut(C.Structure):
     _fields_ = [("rewards", C.c_void_p), ("team", C.c_void_p), ("dones", C.c_void_p),
                 ("obs", C.c_void_p)]
@@ -99,6 +112,18 @@ def load() -> C.CDLL:
             L.aht_gae.argtypes = [vp, vp, vp, vp, i64, i32, C.c_float, C.c_float, vp, vp, vp]
             L.aht_xp_stats.argtypes = [vp, i32, i32, vp, C.POINTER(XpStatsOut), vp]
             L.aht_step_forced.argtypes = [vp, vp, C.POINTER(StepOut)]
+            L.aht_learner_create.argtypes = [i32, i32, C.POINTER(vp), C.POINTER(vp), C.POINTER(PpoConfig),
+                                             vp, C.POINTER(vp)]
+            L.aht_learner_destroy.argtypes = [vp]
+            L.aht_learner_destroy.restype = None
+            L.aht_learner_n_params.argtypes = [vp]
+            L.aht_learner_n_params.restype = i64
+            L.aht_ppo_update.argtypes = [vp, C.POINTER(Traj), i64, i32, vp]
+            L.aht_ppo_grad.argtypes = [vp, C.POINTER(Traj), i64, i32, i32, i32, vp, vp]
+            L.aht_learner_get.argtypes = [vp, vp, vp, vp, C.POINTER(i64), C.POINTER(i64)]
+            L.aht_learner_set.argtypes = [vp, vp, vp, vp, i64, i64]
+            L.aht_learner_push.argtypes = [vp, vp, i32]
+            L.aht_learner_sync.argtypes = [vp]
             L.aht_policy_forward.argtypes = [vp, i32, vp, i64, vp]
             L.aht_get_state.argtypes = [vp, vp, C.POINTER(C.c_size_t)]
             L.aht_set_state.argtypes = [vp, vp, C.c_size_t]
@@ -112,6 +137,9 @@ def load() -> C.CDLL:
             L.aht_last_error.restype = C.c_char_p
             L.aht_status_string.argtypes = [C.c_int]
             L.aht_status_string.restype = C.c_char_p
+            for f in ("aht_learner_create", "aht_ppo_update", "aht_ppo_grad", "aht_learner_get",
+                      "aht_learner_set", "aht_learner_push", "aht_learner_sync"):
+                getattr(L, f).restype = C.c_int
             for f in ("aht_create", "aht_reset", "aht_rollout", "aht_xplay_matrix", "aht_gae", "aht_xp_stats",
                       "aht_step_forced", "aht_policy_forward", "aht_get_state", "aht_set_state",
                       "aht_sync", "aht_set_policy", "aht_set_timing", "aht_get_timing"):
@@ -359,3 +387,89 @@ def aht_debug_expire_wait(ctx: Context, limit_ns: int):
     L.aht_debug_expire_wait.argtypes = [C.c_void_p, C.c_int64]
     L.aht_debug_expire_wait.restype = C.c_int
     _check(L.aht_debug_expire_wait(ctx.handle, int(limit_ns)))
+
+
+# ---------------------------------------------------------------------------------
+# PPO learner
+# ---------------------------------------------------------------------------------
+class Learner:
+    """Owns an aht_learner handle (aht_learner_destroy on close / garbage collection)."""
+
+    def __init__(self, handle, obs_dim, n_actions, n_params, cfg):
+        self.handle = handle
+        self.obs_dim, self.n_actions, self.n_params, self.cfg = obs_dim, n_actions, n_params, cfg
+
+    def close(self):
+        if self.handle:
+            load().aht_learner_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def aht_learner_create(obs_dim, n_actions, layers, stream=None, **cfg) -> Learner:
+    """layers: [(W1, b1), (W2, b2), (W3, b3)] torch tensors (converted to fp32)."""
+    L = load()
+    c = dict(PPO_DEFAULTS)
+    c.update(cfg)
+    conf = PpoConfig(**c)
+    keep = [(W.float().contiguous(), b.float().contiguous()) for W, b in layers]
+    Ws = (C.c_void_p * 3)(*[W.data_ptr() for W, _ in keep])
+    bs = (C.c_void_p * 3)(*[b.data_ptr() for _, b in keep])
+    h = C.c_void_p()
+    _check(L.aht_learner_create(obs_dim, n_actions, Ws, bs, C.byref(conf), _stream(stream), C.byref(h)))
+    del keep
+    return Learner(h, obs_dim, n_actions, int(L.aht_learner_n_params(h)), c)
+
+
+def _ppo_traj(learner, traj, T, N):
+    f32, u8 = torch.float32, torch.uint8
+    g = traj.get
+    return Traj(_ptr(g("obs"), u8, (T, N, learner.obs_dim), "obs"), _ptr(g("actions"), u8, (T, N), "actions"),
+                None, _ptr(g("logp"), f32, (T, N), "logp"), _ptr(g("values"), f32, (T, N), "values"),
+                None, None, _ptr(g("advantages"), f32, (T, N), "advantages"),
+                _ptr(g("targets"), f32, (T, N), "targets"), None, None, 0.0, 0.0)
+
+
+def aht_ppo_update(learner: Learner, traj: dict, stats=None):
+    T, N = traj["actions"].shape
+    t = _ppo_traj(learner, traj, T, N)
+    E, M = learner.cfg["epochs"], learner.cfg["minibatches"]
+    _check(load().aht_ppo_update(learner.handle, C.byref(t), N, T,
+                                 _ptr(stats, torch.float32, (E * M, 6), "stats")))
+
+
+def aht_ppo_grad(learner: Learner, traj: dict, epoch, minibatch, grad, stats=None):
+    T, N = traj["actions"].shape
+    t = _ppo_traj(learner, traj, T, N)
+    _check(load().aht_ppo_grad(learner.handle, C.byref(t), N, T, epoch, minibatch,
+                               _ptr(grad, torch.float32, (learner.n_params,), "grad"),
+                               _ptr(stats, torch.float32, (6,), "stats")))
+
+
+def aht_learner_get(learner: Learner, params=None, adam_m=None, adam_v=None):
+    n = learner.n_params
+    t, u = C.c_int64(0), C.c_int64(0)
+    _check(load().aht_learner_get(learner.handle, _ptr(params, torch.float32, (n,), "params"),
+                                  _ptr(adam_m, torch.float32, (n,), "adam_m"),
+                                  _ptr(adam_v, torch.float32, (n,), "adam_v"), C.byref(t), C.byref(u)))
+    return t.value, u.value
+
+
+def aht_learner_set(learner: Learner, params, adam_m=None, adam_v=None, t=0, updates=0):
+    n = learner.n_params
+    _check(load().aht_learner_set(learner.handle, _ptr(params, torch.float32, (n,), "params"),
+                                  _ptr(adam_m, torch.float32, (n,), "adam_m"),
+                                  _ptr(adam_v, torch.float32, (n,), "adam_v"), t, updates))
+
+
+def aht_learner_push(learner: Learner, ctx: Context, policy):
+    _check(load().aht_learner_push(learner.handle, ctx.handle, policy))
+
+
+def aht_learner_sync(learner: Learner):
+    _check(load().aht_learner_sync(learner.handle))

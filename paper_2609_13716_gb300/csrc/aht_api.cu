@@ -2,6 +2,7 @@
 // context memory, weight packing and kernel launches.  No compute happens on the host
 // except packing the population once in aht_create.
 #include <algorithm>
+#include <cmath>
 #include <cstdio>
 #include <cstring>
 #include <mutex>
@@ -1108,6 +1109,300 @@ aht_status aht_debug_expire_wait(aht_ctx* c, int64_t limit_ns) {
   if (limit_ns < 1 || limit_ns > 1000000000) return fail(AHT_EINVAL, "limit_ns must be in 1..1e9");
   DeviceGuard g(c->device);
   AHT_CUDA(launch_expire_wait(c->status, (uint64_t)limit_ns, c->stream));
+  return AHT_OK;
+}
+
+}  // extern "C"
+
+// ======================================================================================
+// PPO learner (App. C "PPO ego"): fp32 master weights, Adam moments, the packed bf16 copy
+// the gradient kernel loads, per-CTA gradient partials.
+// ======================================================================================
+struct aht_learner {
+  int device = 0;
+  cudaStream_t stream = nullptr;
+  aht_ppo_config cfg{};
+  PpoLayout L{};
+  int n_act = 0;
+  int max_grid = 0;          // SMs
+  int64_t part_stride = 0;   // floats per CTA partial
+  int n_blocks = 0;          // reduction blocks
+  int64_t t = 0, updates = 0;
+  float *params = nullptr, *m = nullptr, *v = nullptr, *partials = nullptr;
+  float* mbstat = nullptr;   // [epochs * minibatches][2]
+  double *grad = nullptr, *blocksq = nullptr, *advpart = nullptr;
+  uint8_t* packed = nullptr;
+  uint32_t* status = nullptr;
+};
+
+namespace {
+
+PpoLayout ppo_layout(int D, int n_act) {
+  PpoLayout L{};
+  const int64_t H = kPpoHidden, O = n_act + 1;
+  L.D = D;
+  L.O = (int32_t)O;
+  L.ob1 = H * D;
+  L.oW2 = L.ob1 + H;
+  L.ob2 = L.oW2 + H * H;
+  L.oW3 = L.ob2 + H;
+  L.ob3 = L.oW3 + O * H;
+  L.n_params = L.ob3 + O;
+  return L;
+}
+
+void learner_free(aht_learner* L) {
+  for (void* p : {(void*)L->params, (void*)L->m, (void*)L->v, (void*)L->partials, (void*)L->mbstat,
+                  (void*)L->grad, (void*)L->blocksq, (void*)L->advpart, (void*)L->packed, (void*)L->status})
+    if (p) cudaFree(p);
+}
+
+aht_status check_traj(const aht_learner* L, const aht_traj* tr, int64_t n_envs, int32_t T) {
+  if (!tr || !tr->obs || !tr->actions || !tr->logp || !tr->values || !tr->advantages || !tr->targets)
+    return fail(AHT_EINVAL, "traj needs obs, actions, logp, values, advantages and targets");
+  if (n_envs < 1 || T < 1) return fail(AHT_EINVAL, "n_envs and T must be >= 1");
+  const int64_t S = n_envs * (int64_t)T;
+  if (S >= (int64_t(1) << 31)) return fail(AHT_EINVAL, "T * n_envs must be below 2^31");
+  if (S % ((int64_t)kPpoTile * L->cfg.minibatches) != 0)
+    return fail(AHT_EINVAL, "T * n_envs must be a multiple of 64 * minibatches");
+  return AHT_OK;
+}
+
+int perm_bits(int64_t S) {
+  int w = 2;
+  while ((int64_t(1) << w) < S) ++w;
+  return w;
+}
+
+// One minibatch: grad kernel, reduction, and (step) clip + Adam + repack.
+aht_status learner_minibatch(aht_learner* L, const aht_traj* tr, int64_t n_envs, int32_t T,
+                             uint32_t epoch, int e, int b, float* stats, bool step) {
+  const int64_t S = n_envs * (int64_t)T;
+  const uint32_t B = (uint32_t)(S / L->cfg.minibatches);
+  const int n_tiles = (int)(B / kPpoTile);
+  const int G = std::min(L->max_grid, n_tiles);
+  PpoGradArgs a{};
+  a.packed = L->packed;
+  a.obs = tr->obs;
+  a.act = tr->actions;
+  a.logp = tr->logp;
+  a.val = tr->values;
+  a.adv = tr->advantages;
+  a.tgt = tr->targets;
+  a.D = L->L.D;
+  a.n_act = L->n_act;
+  a.S = (uint32_t)S;
+  a.w = perm_bits(S);
+  a.key = Key{(uint32_t)(L->cfg.seed & 0xffffffffu), (uint32_t)(L->cfg.seed >> 32)};
+  a.epoch = epoch;
+  a.B = B;
+  a.mb = (uint32_t)b;
+  a.mbstat = L->mbstat + 2 * ((int64_t)e * L->cfg.minibatches + b);
+  a.clip_eps = L->cfg.clip_eps;
+  a.vf_coef = L->cfg.vf_coef;
+  a.ent_coef = L->cfg.ent_coef;
+  a.partials = L->partials;
+  a.part_stride = L->part_stride;
+  a.n_params = L->L.n_params;
+  a.oW1 = 0;
+  a.ob1 = L->L.ob1;
+  a.oW2 = L->L.oW2;
+  a.ob2 = L->L.ob2;
+  a.oW3 = L->L.oW3;
+  a.ob3 = L->L.ob3;
+  a.status = L->status;
+  AHT_CUDA(launch_ppo_grad(a, G, L->stream));
+  PpoAdamArgs ad{};
+  ad.L = L->L;
+  ad.grad = L->grad;
+  ad.blocksq = L->blocksq;
+  ad.n_blocks = L->n_blocks;
+  ad.params = L->params;
+  ad.m = L->m;
+  ad.v = L->v;
+  ad.packed = L->packed;
+  ad.lr = L->cfg.lr;
+  ad.b1 = L->cfg.adam_b1;
+  ad.b2 = L->cfg.adam_b2;
+  ad.eps = L->cfg.adam_eps;
+  ad.max_grad_norm = L->cfg.max_grad_norm;
+  if (step) {
+    L->t += 1;
+    ad.c1 = (float)(1.0 - std::pow((double)L->cfg.adam_b1, (double)L->t));
+    ad.c2 = (float)(1.0 - std::pow((double)L->cfg.adam_b2, (double)L->t));
+  }
+  AHT_CUDA(launch_ppo_reduce_adam(L->partials, G, L->part_stride, ad, stats, 1.0f / (float)B, step,
+                                  L->stream));
+  return AHT_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+aht_status aht_learner_create(int32_t obs_dim, int32_t n_actions, const float* const* W,
+                              const float* const* b, const aht_ppo_config* cfg,
+                              void* cuda_stream, aht_learner** out) {
+  if (!out) return fail(AHT_EINVAL, "out is NULL");
+  *out = nullptr;
+  if (!W || !b || !cfg) return fail(AHT_EINVAL, "NULL weights or config");
+  if (obs_dim < 1 || obs_dim >= kPpoKP || obs_dim % 4 != 0)
+    return fail(AHT_EINVAL, "obs_dim must be a multiple of 4 in 4..204");
+  if (n_actions < 1 || n_actions + 1 > kPpoMaxOut) return fail(AHT_EINVAL, "n_actions must be in 1..7");
+  if (cfg->epochs < 1 || cfg->minibatches < 1) return fail(AHT_EINVAL, "epochs and minibatches must be >= 1");
+  if (!(cfg->lr > 0.f) || !(cfg->clip_eps >= 0.f) || !(cfg->adam_eps > 0.f) || !(cfg->adam_b1 >= 0.f) ||
+      !(cfg->adam_b1 < 1.f) || !(cfg->adam_b2 >= 0.f) || !(cfg->adam_b2 < 1.f))
+    return fail(AHT_EINVAL, "lr, adam_eps > 0; clip_eps >= 0; adam betas in [0, 1)");
+  for (int l = 0; l < 3; ++l)
+    if (!W[l] || !b[l]) return fail(AHT_EINVAL, "NULL weight pointer");
+  auto* L = new aht_learner();
+  L->cfg = *cfg;
+  L->n_act = n_actions;
+  L->L = ppo_layout(obs_dim, n_actions);
+  L->stream = (cudaStream_t)cuda_stream;
+  auto bail = [&](aht_status st) {
+    learner_free(L);
+    delete L;
+    return st;
+  };
+  if (cudaGetDevice(&L->device) != cudaSuccess) return bail(fail(AHT_ECUDA, "no CUDA device"));
+  cudaDeviceProp prop{};
+  if (cudaGetDeviceProperties(&prop, L->device) != cudaSuccess) return bail(fail(AHT_ECUDA, "device query failed"));
+  L->max_grid = prop.multiProcessorCount;
+  const int64_t np = L->L.n_params;
+  L->part_stride = np + 8;
+  L->n_blocks = (int)((np + 255) / 256);
+  const int n_mb = cfg->epochs * cfg->minibatches;
+  bool okm = cudaMalloc(&L->params, np * 4) == cudaSuccess && cudaMalloc(&L->m, np * 4) == cudaSuccess &&
+             cudaMalloc(&L->v, np * 4) == cudaSuccess &&
+             cudaMalloc(&L->partials, (size_t)L->max_grid * L->part_stride * 4) == cudaSuccess &&
+             cudaMalloc(&L->mbstat, (size_t)n_mb * 2 * 4) == cudaSuccess &&
+             cudaMalloc(&L->grad, np * 8) == cudaSuccess &&
+             cudaMalloc(&L->blocksq, (size_t)L->n_blocks * 8) == cudaSuccess &&
+             cudaMalloc(&L->advpart, (size_t)n_mb * kPpoStatBlocks * 2 * 8) == cudaSuccess &&
+             cudaMalloc(&L->packed, kPpoPackedBytes) == cudaSuccess && cudaMalloc(&L->status, 4) == cudaSuccess;
+  if (!okm) return bail(fail(AHT_ENOMEM, "device allocation failed"));
+  const int64_t sizes[6] = {128LL * obs_dim, 128, 128LL * 128, 128, (int64_t)(n_actions + 1) * 128, n_actions + 1};
+  const int64_t offs[6] = {0, L->L.ob1, L->L.oW2, L->L.ob2, L->L.oW3, L->L.ob3};
+  for (int k = 0; k < 6; ++k) {
+    const float* src = (k & 1) ? b[k / 2] : W[k / 2];
+    if (cudaMemcpyAsync(L->params + offs[k], src, sizes[k] * 4, cudaMemcpyDefault, L->stream) != cudaSuccess)
+      return bail(fail(AHT_ECUDA, "copying the weights failed"));
+  }
+  if (cudaMemsetAsync(L->m, 0, np * 4, L->stream) != cudaSuccess ||
+      cudaMemsetAsync(L->v, 0, np * 4, L->stream) != cudaSuccess ||
+      cudaMemsetAsync(L->packed, 0, kPpoPackedBytes, L->stream) != cudaSuccess ||
+      cudaMemsetAsync(L->status, 0, 4, L->stream) != cudaSuccess ||
+      launch_ppo_pack(L->L, L->params, L->packed, L->stream) != cudaSuccess ||
+      ppo_grad_set_smem() != cudaSuccess || cudaStreamSynchronize(L->stream) != cudaSuccess)
+    return bail(fail(AHT_ECUDA, "learner initialisation failed"));
+  *out = L;
+  return AHT_OK;
+}
+
+void aht_learner_destroy(aht_learner* L) {
+  if (!L) return;
+  DeviceGuard g(L->device);
+  cudaStreamSynchronize(L->stream);
+  learner_free(L);
+  delete L;
+}
+
+int64_t aht_learner_n_params(const aht_learner* L) { return L ? L->L.n_params : -1; }
+
+aht_status aht_ppo_update(aht_learner* L, const aht_traj* tr, int64_t n_envs, int32_t T, float* stats) {
+  if (!L) return fail(AHT_EINVAL, "learner is NULL");
+  aht_status st = check_traj(L, tr, n_envs, T);
+  if (st != AHT_OK) return st;
+  DeviceGuard g(L->device);
+  const int64_t S = n_envs * (int64_t)T;
+  const int E = L->cfg.epochs, M = L->cfg.minibatches;
+  const uint32_t B = (uint32_t)(S / M);
+  const uint32_t epoch0 = (uint32_t)(L->updates * E);
+  const Key key{(uint32_t)(L->cfg.seed & 0xffffffffu), (uint32_t)(L->cfg.seed >> 32)};
+  AHT_CUDA(launch_ppo_advstat(tr->advantages, (uint32_t)S, perm_bits(S), key, epoch0, E, M, B,
+                              L->advpart, L->mbstat, L->stream));
+  for (int e = 0; e < E; ++e)
+    for (int b = 0; b < M; ++b) {
+      st = learner_minibatch(L, tr, n_envs, T, epoch0 + (uint32_t)e, e, b,
+                             stats ? stats + 6 * ((int64_t)e * M + b) : nullptr, true);
+      if (st != AHT_OK) return st;
+    }
+  L->updates += 1;
+  return AHT_OK;
+}
+
+aht_status aht_ppo_grad(aht_learner* L, const aht_traj* tr, int64_t n_envs, int32_t T, int32_t epoch,
+                        int32_t minibatch, float* grad, float* stats) {
+  if (!L || !grad) return fail(AHT_EINVAL, "NULL learner or grad");
+  aht_status st = check_traj(L, tr, n_envs, T);
+  if (st != AHT_OK) return st;
+  if (epoch < 0 || epoch >= L->cfg.epochs || minibatch < 0 || minibatch >= L->cfg.minibatches)
+    return fail(AHT_EINVAL, "epoch / minibatch out of range");
+  DeviceGuard g(L->device);
+  const int64_t S = n_envs * (int64_t)T;
+  const int E = L->cfg.epochs, M = L->cfg.minibatches;
+  const uint32_t B = (uint32_t)(S / M);
+  const uint32_t epoch0 = (uint32_t)(L->updates * E);
+  const Key key{(uint32_t)(L->cfg.seed & 0xffffffffu), (uint32_t)(L->cfg.seed >> 32)};
+  AHT_CUDA(launch_ppo_advstat(tr->advantages, (uint32_t)S, perm_bits(S), key, epoch0, E, M, B,
+                              L->advpart, L->mbstat, L->stream));
+  st = learner_minibatch(L, tr, n_envs, T, epoch0 + (uint32_t)epoch, epoch, minibatch, stats, false);
+  if (st != AHT_OK) return st;
+  AHT_CUDA(launch_f64_to_f32(L->grad, grad, L->L.n_params, L->stream));
+  return AHT_OK;
+}
+
+aht_status aht_learner_get(aht_learner* L, float* params, float* adam_m, float* adam_v, int64_t* t,
+                           int64_t* updates) {
+  if (!L) return fail(AHT_EINVAL, "learner is NULL");
+  DeviceGuard g(L->device);
+  const size_t bytes = (size_t)L->L.n_params * 4;
+  if (params) AHT_CUDA(cudaMemcpyAsync(params, L->params, bytes, cudaMemcpyDefault, L->stream));
+  if (adam_m) AHT_CUDA(cudaMemcpyAsync(adam_m, L->m, bytes, cudaMemcpyDefault, L->stream));
+  if (adam_v) AHT_CUDA(cudaMemcpyAsync(adam_v, L->v, bytes, cudaMemcpyDefault, L->stream));
+  if (t) *t = L->t;
+  if (updates) *updates = L->updates;
+  return AHT_OK;
+}
+
+aht_status aht_learner_set(aht_learner* L, const float* params, const float* adam_m, const float* adam_v,
+                           int64_t t, int64_t updates) {
+  if (!L || !params) return fail(AHT_EINVAL, "NULL learner or params");
+  if (t < 0 || updates < 0) return fail(AHT_EINVAL, "t and updates must be >= 0");
+  DeviceGuard g(L->device);
+  const size_t bytes = (size_t)L->L.n_params * 4;
+  AHT_CUDA(cudaMemcpyAsync(L->params, params, bytes, cudaMemcpyDefault, L->stream));
+  if (adam_m) AHT_CUDA(cudaMemcpyAsync(L->m, adam_m, bytes, cudaMemcpyDefault, L->stream));
+  else AHT_CUDA(cudaMemsetAsync(L->m, 0, bytes, L->stream));
+  if (adam_v) AHT_CUDA(cudaMemcpyAsync(L->v, adam_v, bytes, cudaMemcpyDefault, L->stream));
+  else AHT_CUDA(cudaMemsetAsync(L->v, 0, bytes, L->stream));
+  AHT_CUDA(launch_ppo_pack(L->L, L->params, L->packed, L->stream));
+  L->t = t;
+  L->updates = updates;
+  return AHT_OK;
+}
+
+aht_status aht_learner_push(aht_learner* L, aht_ctx* c, int32_t policy) {
+  if (!L || !c) return fail(AHT_EINVAL, "NULL learner or ctx");
+  DeviceGuard g(L->device);
+  AHT_CUDA(cudaStreamSynchronize(L->stream));
+  const float* p = L->params;
+  const void* W[3] = {p, p + L->L.oW2, p + L->L.oW3};
+  const void* bb[3] = {p + L->L.ob1, p + L->L.ob2, p + L->L.ob3};
+  return aht_set_policy(c, policy, W, bb, AHT_FP32, 1);
+}
+
+aht_status aht_learner_sync(aht_learner* L) {
+  if (!L) return fail(AHT_EINVAL, "learner is NULL");
+  DeviceGuard g(L->device);
+  AHT_CUDA(cudaStreamSynchronize(L->stream));
+  uint32_t s = 0;
+  AHT_CUDA(cudaMemcpy(&s, L->status, 4, cudaMemcpyDeviceToHost));
+  if (s != 0) {
+    AHT_CUDA(cudaMemset(L->status, 0, 4));
+    return fail(s == kStatusTimeout ? AHT_ETIMEOUT : AHT_EDEVICE, "learner status word nonzero");
+  }
   return AHT_OK;
 }
 

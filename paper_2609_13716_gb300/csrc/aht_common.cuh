@@ -22,7 +22,8 @@ enum : uint32_t {
 };
 
 // Philox streams (counter word 2).
-enum : uint32_t { kStreamAct0 = 0, kStreamAct1 = 1, kStreamReset = 2, kStreamTeammate = 3 };
+enum : uint32_t { kStreamAct0 = 0, kStreamAct1 = 1, kStreamReset = 2, kStreamTeammate = 3,
+                  kStreamPermute = 4 /* PPO minibatch permutation */ };
 
 struct DevEnv {
   int32_t kind, width, height, n_food, max_level, episode_len, cook_time, soup_reward;

@@ -216,6 +216,57 @@ cudaError_t launch_gae(const float* r, const float* v, const uint8_t* d, const f
 cudaError_t launch_xp_reduce(const float* returns, int64_t n_pairs, int32_t P, float* matrix,
                              cudaStream_t);
 
+// PPO ego update (ppo_update.cu).  Actor-critic ego obs_dim -> 128 -> 128 -> n_act + 1.
+constexpr int kPpoTile = 64;        // samples per tile of the gradient kernel
+constexpr int kPpoKP = 208;         // padded input width (obs_dim <= 207, the bias column)
+constexpr int kPpoHidden = 128;
+constexpr int kPpoMaxOut = 8;       // n_act + 1 <= 8
+constexpr int kPpoStatBlocks = 64;  // blocks per minibatch of the advantage statistics
+// packed block (bytes): W1 bf16 canonical [128][208], W2 bf16 canonical [128][128],
+// W3 fp32 [64 pairs][8 outputs][2], b1 [128], b2 [128], b3 [8] fp32
+constexpr uint32_t kPkW1 = 0, kPkW2 = 53248, kPkW3 = 86016, kPkB1 = 90112, kPkB2 = 90624,
+                   kPkB3 = 91136, kPpoPackedBytes = 91168;
+struct PpoLayout {  // flat parameter vector: W1 [128][D], b1, W2 [128][128], b2, W3 [O][128], b3
+  int32_t D, O;
+  int64_t n_params, ob1, oW2, ob2, oW3, ob3;
+};
+struct PpoGradArgs {
+  const uint8_t* packed;
+  const uint8_t* obs;       // [S][D]
+  const uint8_t* act;       // [S]
+  const float *logp, *val, *adv, *tgt;
+  int32_t D, n_act;
+  uint32_t S;               // samples
+  int32_t w;                // permutation bits
+  Key key;                  // permutation key
+  uint32_t epoch;           // permutation counter
+  uint32_t B, mb;           // samples per minibatch, minibatch index
+  const float* mbstat;      // [2]: mean, 1 / (std + 1e-8) of the minibatch's advantages
+  float clip_eps, vf_coef, ent_coef;
+  float* partials;          // [grid][part_stride]: gradient partials, then 6 loss sums
+  int64_t part_stride, n_params, oW1, ob1, oW2, ob2, oW3, ob3;
+  uint32_t* status;
+};
+struct PpoAdamArgs {
+  PpoLayout L;
+  double* grad;     // [n_params] written by the reduction
+  double* blocksq;  // [n_blocks] squared-norm partials
+  int32_t n_blocks;
+  float *params, *m, *v;
+  uint8_t* packed;
+  float lr, b1, b2, eps, c1, c2, max_grad_norm;
+};
+size_t ppo_grad_smem_bytes();
+cudaError_t ppo_grad_set_smem();
+cudaError_t launch_ppo_grad(const PpoGradArgs&, int grid, cudaStream_t);
+cudaError_t launch_ppo_advstat(const float* adv, uint32_t S, int w, Key key, uint32_t epoch0, int E,
+                               int M, uint32_t B, double* part, float* mbstat, cudaStream_t);
+cudaError_t launch_ppo_pack(const PpoLayout&, const float* params, uint8_t* packed, cudaStream_t);
+// Sums the partials (grad, blocksq, stats[6] = means), then (step) clips and takes the Adam step.
+cudaError_t launch_f64_to_f32(const double* x, float* y, int64_t n, cudaStream_t);
+cudaError_t launch_ppo_reduce_adam(const float* partials, int G, int64_t stride, const PpoAdamArgs&,
+                                   float* stats, float inv_b, bool step, cudaStream_t);
+
 // Cross-play matrix consumers (misc.cu): one CTA; n_ego, n_tm <= kXpStatsMax.
 constexpr int kXpStatsMax = 2048;
 struct XpStatsArgs {

@@ -64,3 +64,14 @@ def test_host_validation_needs_no_gpu(lib):
     out.brdiv = 16
     assert L.aht_xp_stats(fake, 2, 3, fake, C.byref(out), None) == aht.AHT_EINVAL
     assert b"square" in L.aht_last_error()
+    # PPO learner: host checks before any CUDA call
+    cfg = aht.PpoConfig(**aht.PPO_DEFAULTS)
+    ptrs = (C.c_void_p * 3)(16, 16, 16)
+    out_l = C.c_void_p()
+    assert L.aht_learner_create(195, 6, ptrs, ptrs, C.byref(cfg), None, C.byref(out_l)) == aht.AHT_EINVAL
+    assert b"obs_dim" in L.aht_last_error()
+    assert L.aht_learner_create(196, 8, ptrs, ptrs, C.byref(cfg), None, C.byref(out_l)) == aht.AHT_EINVAL
+    bad_cfg = aht.PpoConfig(**dict(aht.PPO_DEFAULTS, minibatches=0))
+    assert L.aht_learner_create(196, 6, ptrs, ptrs, C.byref(bad_cfg), None, C.byref(out_l)) == aht.AHT_EINVAL
+    assert L.aht_ppo_update(None, None, 64, 1, None) == aht.AHT_EINVAL
+    assert L.aht_learner_n_params(None) == -1
