@@ -44,6 +44,8 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-xplay", action="store_true")
     p.add_argument("--no-ppo", action="store_true")
+    # PPO update only, on the trajectory of one rollout (profiling; not a bench line)
+    p.add_argument("--ppo-only", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     # profiling of a smaller case of the same kernel (not a bench line)
     p.add_argument("--n-envs", type=int, default=None)
@@ -258,6 +260,13 @@ def run_ours(args):
 
     def step():
         aht.aht_rollout(ctx, wl.ego_id, wl.pool, T, traj, wl.gamma, wl.lam)
+
+    if args.ppo_only:
+        step()
+        pu = run_ppo_update(args, aht, wl, pop_np, traj, torch, bf16_peak, stream)
+        if rank == 0:
+            print(json.dumps({"ppo_update": pu}), flush=True)
+        return
 
     for _ in range(max(3, args.warmup)):
         step()

@@ -222,10 +222,11 @@ constexpr int kPpoKP = 208;         // padded input width (obs_dim <= 207, the b
 constexpr int kPpoHidden = 128;
 constexpr int kPpoMaxOut = 8;       // n_act + 1 <= 8
 constexpr int kPpoStatBlocks = 64;  // blocks per minibatch of the advantage statistics
-// packed block (bytes): W1 bf16 canonical [128][208], W2 bf16 canonical [128][128],
-// W3 fp32 [64 pairs][8 outputs][2], b1 [128], b2 [128], b3 [8] fp32
-constexpr uint32_t kPkW1 = 0, kPkW2 = 53248, kPkW3 = 86016, kPkB1 = 90112, kPkB2 = 90624,
-                   kPkB3 = 91136, kPpoPackedBytes = 91168;
+// packed block (bytes): W1 bf16 canonical [128][208], W2 bf16 canonical [128][128], W3 as
+// two bf16 canonical [16][128] (hi, lo; rows past n_act + 1 zero), b1 [128], b2 [128],
+// b3 [8] fp32
+constexpr uint32_t kPkW1 = 0, kPkW2 = 53248, kPkW3hi = 86016, kPkW3lo = 90112, kPkB1 = 94208,
+                   kPkB2 = 94720, kPkB3 = 95232, kPpoPackedBytes = 95264;
 struct PpoLayout {  // flat parameter vector: W1 [128][D], b1, W2 [128][128], b2, W3 [O][128], b3
   int32_t D, O;
   int64_t n_params, ob1, oW2, ob2, oW3, ob3;

@@ -4,11 +4,10 @@
 // collected trajectory drawn by a keyed permutation.
 //
 // ppo_grad_kernel: one CTA per SM, each a contiguous run of 64-sample tiles of the
-// minibatch.  Per tile the forward (L1, L2 as tcgen05 MMAs, the output layer on CUDA
-// cores), the per-sample loss gradient, and the backward run in one pass; the weight
-// gradients accumulate in tensor memory over the CTA's tiles (dW1 208 columns, dW2 144,
-// dW3^T 16, the working accumulator 128: 496 of 512) and leave once, as the CTA's partial
-// sum.  Operands live in shared memory as rows of samples (8 x 16-byte core matrices, 8
+// minibatch.  Per tile the forward (L1, L2 and the output layer as tcgen05 MMAs), the
+// per-sample loss gradient, and the backward run in one pass; the weight gradients
+// accumulate in tensor memory over the CTA's tiles (dW1 208 columns, dW2 144, dW3^T 16,
+// the working accumulator 128: 496 of 512) and leave once, as the CTA's partial sum.  Operands live in shared memory as rows of samples (8 x 16-byte core matrices, 8
 // samples x 8 features): the same buffer is the K-major A operand of a forward product
 // (samples as M) and the MN-major operand of a weight-gradient product (samples as K).
 // Forward products run with M = 128 over a 64-sample tile: the upper 64 rows read the
@@ -28,8 +27,12 @@ constexpr int kKP = kPpoKP;          // padded input width: obs + the bias colum
 constexpr int kH = kPpoHidden;       // hidden width
 constexpr int kH1P = 144;            // h1 row width as the B operand of dW2 (+ ones + pad)
 constexpr int kNO = 8;               // output rows (actions + value), padded
-constexpr int kThreadsPpo = 192;     // warps 0, 1, 4, 5 compute; warp 2 issues MMAs
-constexpr int kCompute = 128;
+// Warps w with w % 4 in {0, 1} reach tensor-memory lanes 0..63 (the tile's samples): the 8
+// compute warps 0, 1, 4, 5, 8, 9, 12, 13 (four threads per sample, 32 features each).
+// Warp 2 issues the MMAs; warps 3, 6, 7 and 10 load the next tile; warp 11 idles.
+constexpr int kThreadsPpo = 448;
+constexpr int kCompute = 256;
+constexpr int kLoaders = 128;
 constexpr int kComputeBar = 1;
 
 // shared memory (bytes from the 1024-aligned base)
@@ -43,11 +46,13 @@ constexpr uint32_t kOffH2lo = kOffH2hi + kRows * kH * 2;
 constexpr uint32_t kOffDZhi = kOffH2lo + kRows * kH * 2;       // [64][16]
 constexpr uint32_t kOffDZlo = kOffDZhi + kRows * 16 * 2;
 constexpr uint32_t kOffPK = kOffDZlo + kRows * 16 * 2;         // packed weights
-constexpr uint32_t kOffZX = kOffPK + kPpoPackedBytes;          // [2][64][8] f32
-constexpr uint32_t kSmemUsed = kOffZX + 2 * kRows * kNO * 4;
+constexpr uint32_t kOffSC = kOffPK + kPpoPackedBytes;          // [2][5][64] per-sample scalars
+constexpr uint32_t kSmemUsed = kOffSC + 2 * 5 * kRows * 4;
+constexpr uint32_t kOffRed = kOffDA2hi;                        // [64][16] f32 end-of-kernel sums
 static_assert(kOffH1hi == 26624 && kOffPK == 133120, "layout");
 // every M = 128 A operand of a 64-sample buffer reads 64 more rows from what follows
-static_assert(kOffX + 2 * kRows * kKP * 2 <= kSmemUsed && kOffDA2lo + 2 * kRows * kH * 2 <= kSmemUsed,
+static_assert(kOffX + 2 * kRows * kKP * 2 <= kSmemUsed && kOffDA2lo + 2 * kRows * kH * 2 <= kSmemUsed &&
+                  kOffH2lo + 2 * kRows * kH * 2 <= kSmemUsed && kOffDZlo + 2 * kRows * 16 * 2 <= kSmemUsed,
               "A operands stay inside shared memory");
 
 // tensor memory columns
@@ -91,13 +96,16 @@ __device__ __forceinline__ void split2(float x0, float x1, uint32_t& hi, uint32_
 }  // namespace
 
 __global__ void __launch_bounds__(kThreadsPpo, 1) ppo_grad_kernel(const PpoGradArgs a) {
-  extern __shared__ __align__(16) uint8_t smem_raw[];
-  uint8_t* const sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t opnd_bar[4];  // X ready, h1 ready, backward operands, da1
-  __shared__ __align__(8) uint64_t acc_bar[4];   // L1, L2, backward products, dW1 done
+  extern __shared__ __align__(16) uint8_t sm[];  // no-swizzle operands need 16 B
+  // operands ready (threads -> MMA warp): X, h1, h2, dz, da2, da1
+  __shared__ __align__(8) uint64_t opnd_bar[6];
+  // products done (commit -> threads): L1, L2, logits, dL/dh2, dL/dh1, dW1 (the tile's last)
+  __shared__ __align__(8) uint64_t acc_bar[6];
   __shared__ __align__(8) uint64_t wload_bar, drain_bar;
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
+  enum { kX = 0, kH1 = 1, kH2 = 2, kDZ = 3, kDA2 = 4, kDA1 = 5 };
+  enum { kL1 = 0, kL2 = 1, kZ = 2, kDH2 = 3, kDH1 = 4, kDW1 = 5 };
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int n_tiles = (int)(a.B / kRows);
@@ -108,8 +116,9 @@ __global__ void __launch_bounds__(kThreadsPpo, 1) ppo_grad_kernel(const PpoGradA
   const uint8_t* pk = sm + kOffPK;
 
   if (tid == 0) {
-    for (int i = 0; i < 4; ++i) {
-      tc::mbar_init(&opnd_bar[i], kCompute);
+    for (int i = 0; i < 6; ++i) {
+      // X: the loader warps; dz: the 64 threads that compute the sample's loss
+      tc::mbar_init(&opnd_bar[i], i == kX ? kLoaders : (i == kDZ ? kRows : kCompute));
       tc::mbar_init(&acc_bar[i], 1);
     }
     tc::mbar_init(&wload_bar, 1);
@@ -118,7 +127,8 @@ __global__ void __launch_bounds__(kThreadsPpo, 1) ppo_grad_kernel(const PpoGradA
     abort_flag = 0;
   }
   if (warp == 0) tc::tmem_alloc(&tmem_slot, 512);
-  // constant columns: h1's "ones" feature 128 (carries db2 through dW2), zero pad; dz 8..15
+  // constant columns: h1's "ones" feature 128 (carries db2 through dW2) and zero pad; the
+  // dz rows' columns 8..15
   for (int r = tid; r < kRows; r += blockDim.x) {
     *reinterpret_cast<uint4*>(sm + kOffH1hi + canon(r, 128, kH1P)) = make_uint4(0x3F80u, 0u, 0u, 0u);
     *reinterpret_cast<uint4*>(sm + kOffH1hi + canon(r, 136, kH1P)) = make_uint4(0u, 0u, 0u, 0u);
@@ -141,81 +151,173 @@ __global__ void __launch_bounds__(kThreadsPpo, 1) ppo_grad_kernel(const PpoGradA
         tc::bulk_g2s(sm + kOffPK + off, a.packed + off, min(32768u, kPpoPackedBytes - off), &wload_bar);
       bool ok = tc::mbar_wait(&wload_bar, 0);
       const uint32_t idL = tc::idesc_bf16(128, kH);                               // L1, L2
-      const uint32_t idH = tc::idesc_bf16(128, kH) | (1u << 16);                  // dh1: B MN-major
+      const uint32_t idZ = tc::idesc_bf16(128, 16);                               // logits
+      const uint32_t idH = tc::idesc_bf16(128, kH) | (1u << 16);                  // B MN-major
       const uint32_t id3 = tc::idesc_bf16(128, 16) | (1u << 15) | (1u << 16);     // dW3^T
       const uint32_t id2 = tc::idesc_bf16(128, kH1P) | (1u << 15) | (1u << 16);   // dW2
       const uint32_t id1 = tc::idesc_bf16(128, kKP) | (1u << 15) | (1u << 16);    // dW1
-      const uint32_t pW1 = base + kOffPK + kPkW1, pW2 = base + kOffPK + kPkW2;
+      // descriptors at K-step 0; a K-step adds (its byte stride >> 4) to the address field
+      auto kmaj = [&](uint32_t off, int K) { return tc::smem_desc(base + off, 128u, (uint32_t)(K / 8) * 128u); };
+      auto mnmaj = [&](uint32_t off, int MN) { return tc::smem_desc(base + off, (uint32_t)(MN / 8) * 128u, 128u); };
+      const uint64_t dX = kmaj(kOffX, kKP), dW1 = kmaj(kOffPK + kPkW1, kKP);
+      const uint64_t dH1[2] = {kmaj(kOffH1hi, kH1P), kmaj(kOffH1lo, kH1P)};
+      const uint64_t dW2 = kmaj(kOffPK + kPkW2, kH), dW2t = mnmaj(kOffPK + kPkW2, kH);
+      const uint64_t dH2[2] = {kmaj(kOffH2hi, kH), kmaj(kOffH2lo, kH)};
+      const uint64_t dW3[2] = {kmaj(kOffPK + kPkW3hi, kH), kmaj(kOffPK + kPkW3lo, kH)};
+      const uint64_t dW3t[2] = {mnmaj(kOffPK + kPkW3hi, kH), mnmaj(kOffPK + kPkW3lo, kH)};
+      const uint64_t dDZ[2] = {kmaj(kOffDZhi, 16), kmaj(kOffDZlo, 16)};
+      const uint64_t dDA2[2] = {kmaj(kOffDA2hi, kH), kmaj(kOffDA2lo, kH)};
+      const uint64_t tDA2[2] = {mnmaj(kOffDA2hi, kH), mnmaj(kOffDA2lo, kH)};
+      const uint64_t tH2[2] = {mnmaj(kOffH2hi, kH), mnmaj(kOffH2lo, kH)};  // h2, later dL/da1
+      const uint64_t tH1[2] = {mnmaj(kOffH1hi, kH1P), mnmaj(kOffH1lo, kH1P)};
+      const uint64_t tDZ[2] = {mnmaj(kOffDZhi, 16), mnmaj(kOffDZlo, 16)};
+      const uint64_t tX = mnmaj(kOffX, kKP);
+      constexpr uint64_t kS16 = 16;                               // 256 B: 16 features
+      constexpr uint64_t kSampK = 2ull * (kH / 8) * 128 >> 4;     // 16 samples of a 128-wide buffer
+      constexpr uint64_t kSampK1 = 2ull * (kH1P / 8) * 128 >> 4;  // ... of h1 (144 wide)
+      constexpr uint64_t kSampKZ = 2ull * (16 / 8) * 128 >> 4;    // ... of dz (16 wide)
+      constexpr uint64_t kSampKX = 2ull * (kKP / 8) * 128 >> 4;   // ... of x (208 wide)
       auto wait_opnd = [&](int i, uint32_t par) {
         if (ok) ok = tc::mbar_wait(&opnd_bar[i], par) && !abort_flag;
         if (ok) tc::fence_after_sync();
         return ok;
       };
+      // the three products of a split pair: hi*hi, hi*lo, lo*hi (lo*lo is below 2^-16)
       for (int it = 0; ok && it < n_it; ++it) {
         const uint32_t par = (uint32_t)it & 1u;
-        const bool first = it == 0;
+        const uint32_t fresh = it == 0 ? 0u : 1u;  // the first tile starts the gradient sums
         // L1: acc = X W1^T (13 K-steps of 16 features)
-        if (!wait_opnd(0, par)) break;
+        if (!wait_opnd(kX, par)) break;
+#pragma unroll
         for (int ks = 0; ks < kKP / 16; ++ks)
-          tc::mma_ss(tmem + kTmAcc, tc::smem_desc(base + kOffX + 256u * ks, 128u, (kKP / 8) * 128u),
-                     tc::smem_desc(pW1 + 256u * ks, 128u, (kKP / 8) * 128u), idL, ks > 0);
-        tc::commit(&acc_bar[0]);
+          tc::mma_ss(tmem + kTmAcc, dX + kS16 * ks, dW1 + kS16 * ks, idL, ks > 0);
+        tc::commit(&acc_bar[kL1]);
         // L2: acc = (h1_hi + h1_lo) W2^T
-        if (!wait_opnd(1, par)) break;
-        for (int part = 0; part < 2; ++part) {
-          const uint32_t h1 = base + (part ? kOffH1lo : kOffH1hi);
+        if (!wait_opnd(kH1, par)) break;
+#pragma unroll
+        for (int part = 0; part < 2; ++part)
+#pragma unroll
           for (int ks = 0; ks < kH / 16; ++ks)
-            tc::mma_ss(tmem + kTmAcc, tc::smem_desc(h1 + 256u * ks, 128u, (kH1P / 8) * 128u),
-                       tc::smem_desc(pW2 + 256u * ks, 128u, (kH / 8) * 128u), idL, (part | ks) != 0);
-        }
-        tc::commit(&acc_bar[1]);
-        // backward: dW3^T += h2^T dz, dW2 += da2^T [h1 | 1], acc = da2 W2 (= dL/dh1)
-        if (!wait_opnd(2, par)) break;
-        {
-          const uint32_t Ah[3] = {kOffH2hi, kOffH2hi, kOffH2lo}, Bz[3] = {kOffDZhi, kOffDZlo, kOffDZhi};
-          for (int p = 0; p < 3; ++p)
-            for (int ks = 0; ks < kRows / 16; ++ks)
-              tc::mma_ss(tmem + kTmDW3, tc::smem_desc(base + Ah[p] + 4096u * ks, 2048u, 128u),
-                         tc::smem_desc(base + Bz[p] + 512u * ks, 256u, 128u), id3,
-                         !(first && p == 0 && ks == 0));
-          const uint32_t Ad[3] = {kOffDA2hi, kOffDA2hi, kOffDA2lo}, Bh[3] = {kOffH1hi, kOffH1lo, kOffH1hi};
-          for (int p = 0; p < 3; ++p)
-            for (int ks = 0; ks < kRows / 16; ++ks)
-              tc::mma_ss(tmem + kTmDW2, tc::smem_desc(base + Ad[p] + 4096u * ks, 2048u, 128u),
-                         tc::smem_desc(base + Bh[p] + 4608u * ks, (kH1P / 8) * 128u, 128u), id2,
-                         !(first && p == 0 && ks == 0));
-          for (int part = 0; part < 2; ++part) {
-            const uint32_t da = base + (part ? kOffDA2lo : kOffDA2hi);
-            for (int ks = 0; ks < kH / 16; ++ks)
-              tc::mma_ss(tmem + kTmAcc, tc::smem_desc(da + 256u * ks, 128u, (kH / 8) * 128u),
-                         tc::smem_desc(pW2 + 4096u * ks, 2048u, 128u), idH, (part | ks) != 0);
-          }
-        }
-        tc::commit(&acc_bar[2]);
-        // dW1 += da1^T [x | 1]
-        if (!wait_opnd(3, par)) break;
-        for (int p = 0; p < 2; ++p)
+            tc::mma_ss(tmem + kTmAcc, dH1[part] + kS16 * ks, dW2 + kS16 * ks, idL, (part | ks) != 0);
+        tc::commit(&acc_bar[kL2]);
+        // output layer: acc[0..16) = h2 W3^T
+        if (!wait_opnd(kH2, par)) break;
+#pragma unroll
+        for (int p = 0; p < 3; ++p)
+#pragma unroll
+          for (int ks = 0; ks < kH / 16; ++ks)
+            tc::mma_ss(tmem + kTmAcc, dH2[p == 2 ? 1 : 0] + kS16 * ks, dW3[p == 1 ? 1 : 0] + kS16 * ks, idZ,
+                       (p | ks) != 0);
+        tc::commit(&acc_bar[kZ]);
+        // dL/dh2 = dz W3 into acc, then dW3^T += h2^T dz
+        if (!wait_opnd(kDZ, par)) break;
+#pragma unroll
+        for (int p = 0; p < 3; ++p)
+          tc::mma_ss(tmem + kTmAcc, dDZ[p == 2 ? 1 : 0], dW3t[p == 1 ? 1 : 0], idH, p != 0);
+        tc::commit(&acc_bar[kDH2]);
+#pragma unroll
+        for (int p = 0; p < 3; ++p)
+#pragma unroll
           for (int ks = 0; ks < kRows / 16; ++ks)
-            tc::mma_ss(tmem + kTmDW1, tc::smem_desc(base + (p ? kOffH2lo : kOffH2hi) + 4096u * ks, 2048u, 128u),
-                       tc::smem_desc(base + kOffX + 6656u * ks, (kKP / 8) * 128u, 128u), id1,
-                       !(first && p == 0 && ks == 0));
-        tc::commit(&acc_bar[3]);
+            tc::mma_ss(tmem + kTmDW3, tH2[p == 2 ? 1 : 0] + kSampK * ks, tDZ[p == 1 ? 1 : 0] + kSampKZ * ks,
+                       id3, (p | ks) != 0 ? 1u : fresh);
+        // dL/dh1 = da2 W2 into acc (its commit also covers dW3: h2's rows may be reused),
+        // then dW2 += da2^T [h1 | 1] under epilogue 3
+        if (!wait_opnd(kDA2, par)) break;
+#pragma unroll
+        for (int part = 0; part < 2; ++part)
+#pragma unroll
+          for (int ks = 0; ks < kH / 16; ++ks)
+            tc::mma_ss(tmem + kTmAcc, dDA2[part] + kS16 * ks, dW2t + kSampK * ks, idH, (part | ks) != 0);
+        tc::commit(&acc_bar[kDH1]);
+#pragma unroll
+        for (int p = 0; p < 3; ++p)
+#pragma unroll
+          for (int ks = 0; ks < kRows / 16; ++ks)
+            tc::mma_ss(tmem + kTmDW2, tDA2[p == 2 ? 1 : 0] + kSampK * ks, tH1[p == 1 ? 1 : 0] + kSampK1 * ks,
+                       id2, (p | ks) != 0 ? 1u : fresh);
+        // dW1 += da1^T [x | 1]
+        if (!wait_opnd(kDA1, par)) break;
+#pragma unroll
+        for (int p = 0; p < 2; ++p)
+#pragma unroll
+          for (int ks = 0; ks < kRows / 16; ++ks)
+            tc::mma_ss(tmem + kTmDW1, tH2[p] + kSampK * ks, tX + kSampKX * ks, id1, (p | ks) != 0 ? 1u : fresh);
+        tc::commit(&acc_bar[kDW1]);
       }
       if (!ok) abort_flag = 1;
     }
-  } else if (warp != 3) {
+  } else if (warp == 3 || warp == 6 || warp == 7 || warp == 10) {
+    // =============================== loader warps ===================================
+    // Loader k (warps 3, 6, 7, 10) owns rows 16k .. 16k + 15 of every tile, two lanes per
+    // row (words 26h .. 26h + 25 of the observation row for lane half h): it draws the
+    // sample from the permutation and loads its observation words and scalars one tile
+    // ahead, into registers; once the previous tile's last MMA has completed it writes
+    // them out as the X operand (feature D is the constant 1 that carries db1 through
+    // dW1) and the scalar rows, and releases the tile.  The next tile's loads are issued
+    // once epilogue 1 is over: the loads slow whatever epilogue they overlap (~1-1.5 K
+    // cycles, measured), and epilogue 2 suffers least.
+    if (n_it > 0) {
+      const int D = a.D, nw = D / 4;
+      const int li = warp == 3 ? 0 : (warp == 6 ? 1 : (warp == 7 ? 2 : 3));
+      const int row = li * 16 + (lane >> 1), hw = lane & 1;
+      constexpr int kHalfWords = kKP / 8;   // 26 words per lane
+      const float mu = a.mbstat[0], inv_sd = a.mbstat[1];
+      uint32_t ow[kHalfWords];
+      float sc[5];
+      auto load_tile = [&](int it) {
+        const uint32_t j = a.mb * a.B + (uint32_t)(t0 + it) * kRows + (uint32_t)row;
+        const uint32_t smp = perm_index(a.key, a.epoch, a.w, a.S, j);
+        const uint32_t* orow = reinterpret_cast<const uint32_t*>(a.obs + (size_t)smp * D);
+#pragma unroll
+        for (int q0 = 0; q0 < kHalfWords; ++q0) {
+          const int q = hw * kHalfWords + q0;
+          ow[q0] = q < nw ? __ldg(orow + q) : (q == nw ? 1u : 0u);
+        }
+        if (hw == 0) {
+          sc[0] = __int_as_float((int)a.act[smp]);
+          sc[1] = a.logp[smp];
+          sc[2] = a.val[smp];
+          sc[3] = (a.adv[smp] - mu) * inv_sd;
+          sc[4] = a.tgt[smp];
+        }
+      };
+      bool ok = true;
+      load_tile(0);
+      for (int it = 0; it < n_it; ++it) {
+        if (it > 0 && ok) ok = tc::mbar_wait(&acc_bar[kDW1], (uint32_t)(it - 1) & 1u);
+        ok = __all_sync(0xFFFFFFFFu, ok) && !abort_flag;
+        if (!ok) break;
+        float* scw = reinterpret_cast<float*>(sm + kOffSC) + (it & 1) * 5 * kRows;
+#pragma unroll
+        for (int c = 0; c < kHalfWords / 2; ++c)
+          *reinterpret_cast<uint4*>(sm + kOffX + canon(row, 8 * (hw * kHalfWords / 2 + c), kKP)) =
+              make_uint4(tc::bytes_to_bf16x2(ow[2 * c], 0), tc::bytes_to_bf16x2(ow[2 * c], 2),
+                         tc::bytes_to_bf16x2(ow[2 * c + 1], 0), tc::bytes_to_bf16x2(ow[2 * c + 1], 2));
+        if (hw == 0) {
+#pragma unroll
+          for (int k = 0; k < 5; ++k) scw[k * kRows + row] = sc[k];
+        }
+        tc::fence_proxy_async();
+        tc::mbar_arrive(&opnd_bar[kX]);
+        if (it + 1 < n_it) {
+          if (ok) ok = tc::mbar_wait(&acc_bar[kL2], (uint32_t)it & 1u);  // epilogue 1 is over
+          load_tile(it + 1);
+        }
+      }
+      if (!ok) abort_flag = 1;
+    }
+  } else if ((warp & 2) == 0) {
     // ============================== compute warps ===================================
-    const int half = warp >= 4 ? 1 : 0;
+    const int quarter = warp >> 2;                                 // features 32q .. 32q + 31
     const int row = (warp & 1) * 32 + lane;                       // sample row of the tile
+    const int c0 = quarter * 32;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;  // tensor-memory lanes
-    const int D = a.D, A = a.n_act;
-    const float mu = a.mbstat[0], inv_sd = a.mbstat[1];
+    const int A = a.n_act;
     const float eps = a.clip_eps, inv_b = 1.0f / (float)a.B;
     const float* b1 = reinterpret_cast<const float*>(pk + kPkB1);
     const float* b2 = reinterpret_cast<const float*>(pk + kPkB2);
     const float* b3 = reinterpret_cast<const float*>(pk + kPkB3);
-    const float* W3 = reinterpret_cast<const float*>(pk + kPkW3);   // [64 pairs][8][2]
-    float* ZX = reinterpret_cast<float*>(sm + kOffZX);
     bool bad = n_it > 0 && !tc::mbar_wait(&wload_bar, 0);
     float st_loss = 0.f, st_pg = 0.f, st_v = 0.f, st_ent = 0.f, st_kl = 0.f, st_clip = 0.f;
     float dzsum[kNO] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
@@ -230,133 +332,119 @@ __global__ void __launch_bounds__(kThreadsPpo, 1) ppo_grad_kernel(const PpoGradA
       tc::mbar_arrive(&opnd_bar[i]);
     };
     auto sync_or = [&]() { return tc::bar_or(kComputeBar, kCompute, bad || abort_flag); };
+    // tanh(acc + bias) of this thread's 32 columns -> hi | lo bf16 rows at dst (row width W)
+    auto act_rows = [&](const float* bias, uint32_t dst_hi, uint32_t dst_lo, int W) {
+      uint32_t v[32];
+      tc::ld_x32(tmem + kTmAcc + lane_base + c0, v);
+      tc::wait_ld();
+      uint32_t hi[16], lo[16];
+#pragma unroll
+      for (int q = 0; q < 16; ++q) {
+        const uint64_t x = tc::f2_add(tc::f2_pack(__uint_as_float(v[2 * q]), __uint_as_float(v[2 * q + 1])),
+                                      tc::f2_pack(bias[c0 + 2 * q], bias[c0 + 2 * q + 1]));
+        tc::split_bf16x2_p(tc::tanh2(x), hi[q], lo[q]);
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        *reinterpret_cast<uint4*>(sm + dst_hi + canon(row, c0 + 8 * q, W)) =
+            make_uint4(hi[4 * q], hi[4 * q + 1], hi[4 * q + 2], hi[4 * q + 3]);
+        *reinterpret_cast<uint4*>(sm + dst_lo + canon(row, c0 + 8 * q, W)) =
+            make_uint4(lo[4 * q], lo[4 * q + 1], lo[4 * q + 2], lo[4 * q + 3]);
+      }
+    };
+    // g (1 - h^2), h = hi + lo from the rows at src (row width W), -> hi | lo rows at dst
+    auto grad_rows = [&](uint32_t src_hi, uint32_t src_lo, int W, uint32_t dst_hi, uint32_t dst_lo) {
+      uint32_t v[32];
+      tc::ld_x32(tmem + kTmAcc + lane_base + c0, v);
+      tc::wait_ld();
+#pragma unroll
+      for (int q8 = 0; q8 < 4; ++q8) {
+        const int c = c0 + 8 * q8;
+        const uint4 hh = *reinterpret_cast<const uint4*>(sm + src_hi + canon(row, c, W));
+        const uint4 hl = *reinterpret_cast<const uint4*>(sm + src_lo + canon(row, c, W));
+        const uint32_t hv[4] = {hh.x, hh.y, hh.z, hh.w}, lv4[4] = {hl.x, hl.y, hl.z, hl.w};
+        uint32_t dh[4], dl[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          float h0a, h0b, h1a, h1b;
+          unpack_bf16x2(hv[q], h0a, h1a);
+          unpack_bf16x2(lv4[q], h0b, h1b);
+          const uint64_t h = tc::f2_add(tc::f2_pack(h0a, h1a), tc::f2_pack(h0b, h1b));
+          const uint64_t one_m = tc::f2_fma(h, tc::f2_sub(0ull, h), tc::f2_pack(1.0f, 1.0f));  // 1 - h^2
+          const uint64_t g = tc::f2_pack(__uint_as_float(v[8 * q8 + 2 * q]), __uint_as_float(v[8 * q8 + 2 * q + 1]));
+          tc::split_bf16x2_p(tc::f2_mul(g, one_m), dh[q], dl[q]);
+        }
+        *reinterpret_cast<uint4*>(sm + dst_hi + canon(row, c, kH)) = make_uint4(dh[0], dh[1], dh[2], dh[3]);
+        *reinterpret_cast<uint4*>(sm + dst_lo + canon(row, c, kH)) = make_uint4(dl[0], dl[1], dl[2], dl[3]);
+      }
+    };
 
     for (int it = 0; it < n_it; ++it) {
       const uint32_t par = (uint32_t)it & 1u;
-      if (it > 0) wait_acc(3, par ^ 1u);        // the previous tile's dW1 read X and da1
+      // the loader wrote this tile's X and scalars, after the previous tile's last MMA:
+      // every operand buffer is free again
+      if (!bad && !tc::mbar_wait(&opnd_bar[kX], par)) bad = true;
       if (sync_or()) { bad = true; break; }
-      // ---- gather: sample s of this row, its observation half and scalars ----------
-      const uint32_t j = a.mb * a.B + (uint32_t)(t0 + it) * kRows + (uint32_t)row;
-      const uint32_t s = perm_index(a.key, a.epoch, a.w, a.S, j);
-      {
-        const uint32_t* orow = reinterpret_cast<const uint32_t*>(a.obs + (size_t)s * D);
-        for (int c = half * 13; c < half * 13 + 13; ++c) {
-          uint32_t w2[2];
-#pragma unroll
-          for (int q = 0; q < 2; ++q) {
-            const int f = 8 * c + 4 * q;
-            w2[q] = f < D ? __ldg(orow + f / 4) : (f == D ? 1u : 0u);
-          }
-          const uint4 v = make_uint4(tc::bytes_to_bf16x2(w2[0], 0), tc::bytes_to_bf16x2(w2[0], 2),
-                                     tc::bytes_to_bf16x2(w2[1], 0), tc::bytes_to_bf16x2(w2[1], 2));
-          *reinterpret_cast<uint4*>(sm + kOffX + canon(row, 8 * c, kKP)) = v;
-        }
-      }
-      const int act = a.act[s];
-      const float lp_old = a.logp[s], v_old = a.val[s], ret = a.tgt[s];
-      const float adv_n = (a.adv[s] - mu) * inv_sd;
-      release(0);
       // ---- epilogue 1: h1 = tanh(acc + b1) -> hi | lo rows -------------------------
-      wait_acc(0, par);
+      wait_acc(kL1, par);
       if (sync_or()) { bad = true; break; }   // every compute thread leaves at the same point
-      for (int c0 = half * 64; c0 < half * 64 + 64; c0 += 32) {
-        uint32_t v[32];
-        tc::ld_x32(tmem + kTmAcc + lane_base + c0, v);
+      act_rows(b1, kOffH1hi, kOffH1lo, kH1P);
+      release(kH1);
+      // ---- epilogue 2: h2 = tanh(acc + b2) -> hi | lo rows -------------------------
+      wait_acc(kL2, par);
+      if (sync_or()) { bad = true; break; }
+      act_rows(b2, kOffH2hi, kOffH2lo, kH);
+      release(kH2);
+      // ---- the sample's loss and dL/dz (quarter 0, one thread per sample) -----------
+      wait_acc(kZ, par);
+      if (sync_or()) { bad = true; break; }
+      if (quarter == 0) {
+        const float* sc = reinterpret_cast<const float*>(sm + kOffSC) + (it & 1) * 5 * kRows;
+        const int act = __float_as_int(sc[row]);
+        const float lp_old = sc[kRows + row], v_old = sc[2 * kRows + row];
+        const float adv_n = sc[3 * kRows + row], ret = sc[4 * kRows + row];
+        uint32_t zr[16];
+        tc::ld_x16(tmem + kTmAcc + lane_base, zr);
         tc::wait_ld();
-        uint32_t hi[16], lo[16];
+        float z[kNO];
 #pragma unroll
-        for (int q = 0; q < 16; ++q) {
-          const uint64_t x = tc::f2_add(tc::f2_pack(__uint_as_float(v[2 * q]), __uint_as_float(v[2 * q + 1])),
-                                        tc::f2_pack(b1[c0 + 2 * q], b1[c0 + 2 * q + 1]));
-          tc::split_bf16x2_p(tc::tanh2(x), hi[q], lo[q]);
+        for (int o = 0; o < kNO; ++o) z[o] = __uint_as_float(zr[o]) + b3[o];
+        // log-softmax, entropy, ratio, clipped surrogate, clipped value loss
+        float mx = -FLT_MAX;
+#pragma unroll
+        for (int o = 0; o < kNO; ++o)
+          if (o < A) mx = fmaxf(mx, z[o]);
+        float se = 0.f;
+#pragma unroll
+        for (int o = 0; o < kNO; ++o)
+          if (o < A) se += __expf(z[o] - mx);
+        const float lse = mx + __logf(se);
+        float logp[kNO], prob[kNO], ent = 0.f, lp_a = 0.f;
+#pragma unroll
+        for (int o = 0; o < kNO; ++o) {
+          logp[o] = z[o] - lse;
+          prob[o] = o < A ? __expf(logp[o]) : 0.f;
+          if (o < A) ent -= prob[o] * logp[o];
+          if (o == act) lp_a = logp[o];
         }
+        const float rho = __expf(lp_a - lp_old);
+        const float rho_c = fminf(fmaxf(rho, 1.0f - eps), 1.0f + eps);
+        const float un = rho * adv_n, cl = rho_c * adv_n;
+        const float g_rho = un <= cl ? -adv_n : 0.0f;
+        float V = 0.f;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          *reinterpret_cast<uint4*>(sm + kOffH1hi + canon(row, c0 + 8 * q, kH1P)) =
-              make_uint4(hi[4 * q], hi[4 * q + 1], hi[4 * q + 2], hi[4 * q + 3]);
-          *reinterpret_cast<uint4*>(sm + kOffH1lo + canon(row, c0 + 8 * q, kH1P)) =
-              make_uint4(lo[4 * q], lo[4 * q + 1], lo[4 * q + 2], lo[4 * q + 3]);
+        for (int o = 0; o < kNO; ++o)
+          if (o == A) V = z[o];
+        const float vc = v_old + fminf(fmaxf(V - v_old, -eps), eps);
+        const float u = V - ret, w = vc - ret;
+        const float dV = u * u >= w * w ? u : 0.0f;
+        float dz[kNO];
+#pragma unroll
+        for (int o = 0; o < kNO; ++o) {
+          const float pol = g_rho * rho * ((o == act ? 1.0f : 0.0f) - prob[o]) +
+                            a.ent_coef * prob[o] * (logp[o] + ent);
+          dz[o] = o < A ? pol * inv_b : (o == A ? a.vf_coef * dV * inv_b : 0.0f);
         }
-      }
-      release(1);
-      // ---- epilogue 2: h2, logits, the sample's loss gradient, dL/da2 ---------------
-      wait_acc(1, par);
-      if (sync_or()) { bad = true; break; }   // every compute thread leaves at the same point
-      uint64_t zacc[kNO] = {0, 0, 0, 0, 0, 0, 0, 0};
-      for (int c0 = half * 64; c0 < half * 64 + 64; c0 += 32) {
-        uint32_t v[32];
-        tc::ld_x32(tmem + kTmAcc + lane_base + c0, v);
-        tc::wait_ld();
-        uint32_t hi[16], lo[16];
-#pragma unroll
-        for (int q = 0; q < 16; ++q) {
-          const uint64_t x = tc::f2_add(tc::f2_pack(__uint_as_float(v[2 * q]), __uint_as_float(v[2 * q + 1])),
-                                        tc::f2_pack(b2[c0 + 2 * q], b2[c0 + 2 * q + 1]));
-          const uint64_t h = tc::tanh2(x);
-          tc::split_bf16x2_p(h, hi[q], lo[q]);
-          const ulonglong2* wp = reinterpret_cast<const ulonglong2*>(W3 + (c0 + 2 * q) * kNO);
-#pragma unroll
-          for (int o = 0; o < kNO; o += 2) {
-            const ulonglong2 ww = wp[o / 2];
-            zacc[o] = tc::f2_fma(h, ww.x, zacc[o]);
-            zacc[o + 1] = tc::f2_fma(h, ww.y, zacc[o + 1]);
-          }
-        }
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          *reinterpret_cast<uint4*>(sm + kOffH2hi + canon(row, c0 + 8 * q, kH)) =
-              make_uint4(hi[4 * q], hi[4 * q + 1], hi[4 * q + 2], hi[4 * q + 3]);
-          *reinterpret_cast<uint4*>(sm + kOffH2lo + canon(row, c0 + 8 * q, kH)) =
-              make_uint4(lo[4 * q], lo[4 * q + 1], lo[4 * q + 2], lo[4 * q + 3]);
-        }
-      }
-#pragma unroll
-      for (int o = 0; o < kNO; ++o) {
-        float e0, e1;
-        tc::f2_unpack(zacc[o], e0, e1);
-        ZX[(half * kRows + row) * kNO + o] = e0 + e1;
-      }
-      tc::bar_or(kComputeBar, kCompute, false);
-      float z[kNO];
-#pragma unroll
-      for (int o = 0; o < kNO; ++o) z[o] = (ZX[row * kNO + o] + ZX[(kRows + row) * kNO + o]) + b3[o];
-      // log-softmax, entropy, ratio, clipped surrogate, clipped value loss
-      float mx = -FLT_MAX;
-#pragma unroll
-      for (int o = 0; o < kNO; ++o)
-        if (o < A) mx = fmaxf(mx, z[o]);
-      float se = 0.f;
-#pragma unroll
-      for (int o = 0; o < kNO; ++o)
-        if (o < A) se += expf(z[o] - mx);
-      const float lse = mx + logf(se);
-      float logp[kNO], prob[kNO], ent = 0.f, lp_a = 0.f;
-#pragma unroll
-      for (int o = 0; o < kNO; ++o) {
-        logp[o] = z[o] - lse;
-        prob[o] = o < A ? expf(logp[o]) : 0.f;
-        if (o < A) ent -= prob[o] * logp[o];
-        if (o == act) lp_a = logp[o];
-      }
-      const float rho = expf(lp_a - lp_old);
-      const float rho_c = fminf(fmaxf(rho, 1.0f - eps), 1.0f + eps);
-      const float un = rho * adv_n, cl = rho_c * adv_n;
-      const float g_rho = un <= cl ? -adv_n : 0.0f;
-      float V = 0.f;
-#pragma unroll
-      for (int o = 0; o < kNO; ++o)
-        if (o == A) V = z[o];
-      const float vc = v_old + fminf(fmaxf(V - v_old, -eps), eps);
-      const float u = V - ret, w = vc - ret;
-      const float dV = u * u >= w * w ? u : 0.0f;
-      float dz[kNO];
-#pragma unroll
-      for (int o = 0; o < kNO; ++o) {
-        const float pol = g_rho * rho * ((o == act ? 1.0f : 0.0f) - prob[o]) +
-                          a.ent_coef * prob[o] * (logp[o] + ent);
-        dz[o] = o < A ? pol * inv_b : (o == A ? a.vf_coef * dV * inv_b : 0.0f);
-      }
-      if (half == 0) {
         const float pg = -fminf(un, cl), lv = 0.5f * fmaxf(u * u, w * w);
         st_loss += pg + a.vf_coef * lv - a.ent_coef * ent;
         st_pg += pg;
@@ -364,79 +452,35 @@ __global__ void __launch_bounds__(kThreadsPpo, 1) ppo_grad_kernel(const PpoGradA
         st_ent += ent;
         st_kl += lp_old - lp_a;
         st_clip += fabsf(rho - 1.0f) > eps ? 1.0f : 0.0f;
-#pragma unroll
-        for (int o = 0; o < kNO; ++o) dzsum[o] += dz[o];
         uint32_t zh[4], zl[4];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) split2(dz[2 * q], dz[2 * q + 1], zh[q], zl[q]);
+        for (int q = 0; q < 4; ++q) {
+          dzsum[2 * q] += dz[2 * q];
+          dzsum[2 * q + 1] += dz[2 * q + 1];
+          split2(dz[2 * q], dz[2 * q + 1], zh[q], zl[q]);
+        }
         *reinterpret_cast<uint4*>(sm + kOffDZhi + canon(row, 0, 16)) = make_uint4(zh[0], zh[1], zh[2], zh[3]);
         *reinterpret_cast<uint4*>(sm + kOffDZlo + canon(row, 0, 16)) = make_uint4(zl[0], zl[1], zl[2], zl[3]);
+        release(kDZ);
       }
-      // dL/dh2 = W3^T dz and dL/da2 = dL/dh2 (1 - h2^2) for this half's features
-      for (int c0 = half * 64; c0 < half * 64 + 64; c0 += 8) {
-        const uint4 hh = *reinterpret_cast<const uint4*>(sm + kOffH2hi + canon(row, c0, kH));
-        const uint4 hl = *reinterpret_cast<const uint4*>(sm + kOffH2lo + canon(row, c0, kH));
-        const uint32_t hv[4] = {hh.x, hh.y, hh.z, hh.w}, lv4[4] = {hl.x, hl.y, hl.z, hl.w};
-        uint32_t dh[4], dl[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int c = c0 + 2 * q;
-          const ulonglong2* wp = reinterpret_cast<const ulonglong2*>(W3 + c * kNO);
-          uint64_t g = 0;
-#pragma unroll
-          for (int o = 0; o < kNO; o += 2) {
-            const ulonglong2 ww = wp[o / 2];
-            g = tc::f2_fma(tc::f2_pack(dz[o], dz[o]), ww.x, g);
-            g = tc::f2_fma(tc::f2_pack(dz[o + 1], dz[o + 1]), ww.y, g);
-          }
-          float h0a, h0b, h1a, h1b;
-          unpack_bf16x2(hv[q], h0a, h1a);
-          unpack_bf16x2(lv4[q], h0b, h1b);
-          const uint64_t h = tc::f2_add(tc::f2_pack(h0a, h1a), tc::f2_pack(h0b, h1b));
-          const uint64_t one_m = tc::f2_fma(h, tc::f2_sub(0ull, h), tc::f2_pack(1.0f, 1.0f));  // 1 - h^2
-          tc::split_bf16x2_p(tc::f2_mul(g, one_m), dh[q], dl[q]);
-        }
-        *reinterpret_cast<uint4*>(sm + kOffDA2hi + canon(row, c0, kH)) = make_uint4(dh[0], dh[1], dh[2], dh[3]);
-        *reinterpret_cast<uint4*>(sm + kOffDA2lo + canon(row, c0, kH)) = make_uint4(dl[0], dl[1], dl[2], dl[3]);
-      }
-      release(2);
-      // ---- epilogue 3: dL/da1 = (da2 W2) (1 - h1^2) into the h2 buffers --------------
-      wait_acc(2, par);
-      if (sync_or()) { bad = true; break; }   // every compute thread leaves at the same point
-      for (int c0 = half * 64; c0 < half * 64 + 64; c0 += 32) {
-        uint32_t v[32];
-        tc::ld_x32(tmem + kTmAcc + lane_base + c0, v);
-        tc::wait_ld();
-#pragma unroll
-        for (int q8 = 0; q8 < 4; ++q8) {
-          const int c = c0 + 8 * q8;
-          const uint4 hh = *reinterpret_cast<const uint4*>(sm + kOffH1hi + canon(row, c, kH1P));
-          const uint4 hl = *reinterpret_cast<const uint4*>(sm + kOffH1lo + canon(row, c, kH1P));
-          const uint32_t hv[4] = {hh.x, hh.y, hh.z, hh.w}, lv4[4] = {hl.x, hl.y, hl.z, hl.w};
-          uint32_t dh[4], dl[4];
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            float h0a, h0b, h1a, h1b;
-            unpack_bf16x2(hv[q], h0a, h1a);
-            unpack_bf16x2(lv4[q], h0b, h1b);
-            const uint64_t h = tc::f2_add(tc::f2_pack(h0a, h1a), tc::f2_pack(h0b, h1b));
-            const uint64_t one_m = tc::f2_fma(h, tc::f2_sub(0ull, h), tc::f2_pack(1.0f, 1.0f));
-            const uint64_t g = tc::f2_pack(__uint_as_float(v[8 * q8 + 2 * q]), __uint_as_float(v[8 * q8 + 2 * q + 1]));
-            tc::split_bf16x2_p(tc::f2_mul(g, one_m), dh[q], dl[q]);
-          }
-          *reinterpret_cast<uint4*>(sm + kOffH2hi + canon(row, c, kH)) = make_uint4(dh[0], dh[1], dh[2], dh[3]);
-          *reinterpret_cast<uint4*>(sm + kOffH2lo + canon(row, c, kH)) = make_uint4(dl[0], dl[1], dl[2], dl[3]);
-        }
-      }
-      release(3);
+      // ---- dL/da2 = (dz W3) (1 - h2^2) --------------------------------------------
+      wait_acc(kDH2, par);
+      if (sync_or()) { bad = true; break; }
+      grad_rows(kOffH2hi, kOffH2lo, kH, kOffDA2hi, kOffDA2lo);
+      release(kDA2);
+      // ---- epilogue 3: dL/da1 = (da2 W2) (1 - h1^2) into the h2 rows ----------------
+      wait_acc(kDH1, par);
+      if (sync_or()) { bad = true; break; }
+      grad_rows(kOffH1hi, kOffH1lo, kH1P, kOffH2hi, kOffH2lo);
+      release(kDA1);
     }
-    if (n_it > 0 && !bad) wait_acc(3, (uint32_t)(n_it - 1) & 1u);  // the last dW1
+    if (n_it > 0 && !bad) wait_acc(kDW1, (uint32_t)(n_it - 1) & 1u);  // the last dW1 (all MMAs)
     if (bad) abort_flag = 1;
-    // per-CTA sums of the half-0 rows: dz (db3) and the loss diagnostics, in row order
+    // per-CTA sums over the quarter-0 threads: dz (db3) and the loss diagnostics, row order
     __syncwarp();
     tc::bar_or(kComputeBar, kCompute, false);
-    float* red = reinterpret_cast<float*>(sm + kOffZX);  // [64][16]
-    if (half == 0) {
+    float* red = reinterpret_cast<float*>(sm + kOffRed);  // [64][16]
+    if (quarter == 0) {
 #pragma unroll
       for (int o = 0; o < kNO; ++o) red[row * 16 + o] = dzsum[o];
       red[row * 16 + 8] = st_loss;
@@ -461,6 +505,7 @@ __global__ void __launch_bounds__(kThreadsPpo, 1) ppo_grad_kernel(const PpoGradA
       uint32_t v[16];
       tc::ld_x16(tmem + kTmDW1 + lb + c0, v);
       tc::wait_ld();
+#pragma unroll
       for (int k = 0; k < 16; ++k) {
         const int c = c0 + k;
         if (n_it == 0) v[k] = 0u;
@@ -472,6 +517,7 @@ __global__ void __launch_bounds__(kThreadsPpo, 1) ppo_grad_kernel(const PpoGradA
       uint32_t v[16];
       tc::ld_x16(tmem + kTmDW2 + lb + c0, v);
       tc::wait_ld();
+#pragma unroll
       for (int k = 0; k < 16; ++k) {
         const int c = c0 + k;
         if (n_it == 0) v[k] = 0u;
@@ -483,11 +529,13 @@ __global__ void __launch_bounds__(kThreadsPpo, 1) ppo_grad_kernel(const PpoGradA
       uint32_t v[16];
       tc::ld_x16(tmem + kTmDW3 + lb, v);
       tc::wait_ld();
-      for (int jj = 0; jj < A1; ++jj) part[a.oW3 + (int64_t)jj * kH + o] = n_it == 0 ? 0.f : __uint_as_float(v[jj]);
+#pragma unroll
+      for (int jj = 0; jj < kNO; ++jj)
+        if (jj < A1) part[a.oW3 + (int64_t)jj * kH + o] = n_it == 0 ? 0.f : __uint_as_float(v[jj]);
     }
   }
   if (!abort_flag && tid < 16) {
-    const float* red = reinterpret_cast<const float*>(sm + kOffZX);
+    const float* red = reinterpret_cast<const float*>(sm + kOffRed);
     float acc = 0.f;
     for (int r = 0; r < kRows; ++r) acc += n_it == 0 ? 0.f : red[r * 16 + tid];
     if (tid < a.n_act + 1) part[a.ob3 + tid] = acc;
@@ -510,7 +558,7 @@ __global__ void __launch_bounds__(kThreadsPpo, 1) ppo_grad_kernel(const PpoGradA
   }
 }
 
-size_t ppo_grad_smem_bytes() { return kSmemUsed + 1024; }
+size_t ppo_grad_smem_bytes() { return kSmemUsed; }
 
 cudaError_t ppo_grad_set_smem() {
   return cudaFuncSetAttribute(ppo_grad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -610,7 +658,10 @@ __device__ __forceinline__ void pack_one(const PpoLayout& L, uint8_t* pk, int64_
   } else if (i < L.ob3) {
     const int64_t r = i - L.oW3;
     const int jj = (int)(r / kH), k = (int)(r - (int64_t)jj * kH);
-    reinterpret_cast<float*>(pk + kPkW3)[((k >> 1) * kNO + jj) * 2 + (k & 1)] = p;
+    const __nv_bfloat16 hi = __float2bfloat16_rn(p);
+    const uint32_t off = tc::canon_offset(jj, k, kH);
+    *reinterpret_cast<__nv_bfloat16*>(pk + kPkW3hi + off) = hi;
+    *reinterpret_cast<__nv_bfloat16*>(pk + kPkW3lo + off) = __float2bfloat16_rn(p - __bfloat162float(hi));
   } else {
     reinterpret_cast<float*>(pk + kPkB3)[i - L.ob3] = p;
   }

@@ -150,6 +150,29 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* mbar, uint32_t parity,
   return false;
 }
 
+// Non-blocking probe of the phase (no suspension).
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* mbar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n.reg .pred p;\nmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\nselp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(done)
+      : "r"(smem_u32(mbar)), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+// Bounded wait that polls without suspending: for short waits whose waker must be seen
+// at once (several warps released together); gives up after limit_ns of wall time.
+__device__ __forceinline__ bool mbar_wait_spin(uint64_t* mbar, uint32_t parity,
+                                               uint64_t limit_ns = 2000000000ull) {
+  if (mbar_test_wait(mbar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 0; i < (1u << 30); ++i) {
+    if (mbar_test_wait(mbar, parity)) return true;
+    if ((i & 63u) == 63u && globaltimer_ns() - t0 > limit_ns) return false;
+  }
+  return false;
+}
+
 __device__ __forceinline__ void mbar_arrive(uint64_t* mbar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(mbar)) : "memory");
 }
