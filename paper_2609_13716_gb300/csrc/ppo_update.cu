@@ -624,7 +624,16 @@ __global__ void ppo_reduce_kernel(const float* __restrict__ partials, int G, int
   const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   double g = 0.0;
   if (i < n_params) {
-    for (int c = 0; c < G; ++c) g += (double)partials[c * stride + i];
+    // four interleaved fp32 chains (CTA c into chain c % 4), joined in fp64: a fixed order
+    // that keeps the dependent-add chain a quarter as long (fp64 adds are slow here)
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    int c = 0;
+    for (; c + 4 <= G; c += 4) {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) acc[k] += partials[(int64_t)(c + k) * stride + i];
+    }
+    for (int k = 0; c < G; ++c, ++k) acc[k] += partials[(int64_t)c * stride + i];
+    g = ((double)acc[0] + (double)acc[1]) + ((double)acc[2] + (double)acc[3]);
     grad[i] = g;
   }
   __shared__ double sq[256];
