@@ -29,6 +29,15 @@ _lib = None
 LBF, OVERCOOKED, HANABI = 0, 1, 2
 STREAM_ACT0, STREAM_ACT1, STREAM_RESET, STREAM_TEAMMATE = 0, 1, 2, 3
 STATE_BYTES = 768
+# LBF heuristic teammates: teammate id -1 - k (App. F LBF suite; rules in aht_oracle.h)
+LBF_HEURISTICS = ("greedy_closest_self", "greedy_closest_teammate", "greedy_closest_avg",
+                  "greedy_lowest_level", "greedy_highest_level", "seq_lexicographic",
+                  "seq_reverse_lexicographic", "seq_column_major", "seq_reverse_column_major",
+                  "seq_nearest_agent", "seq_farthest_agent")
+
+
+def heuristic_id(name):
+    return -1 - LBF_HEURISTICS.index(name)
 
 
 def build(force: bool = False) -> str:
@@ -56,7 +65,8 @@ class LbfState(C.Structure):
     _fields_ = [("ax", C.c_int32 * 2), ("ay", C.c_int32 * 2), ("al", C.c_int32 * 2),
                 ("fx", C.c_int32 * 3), ("fy", C.c_int32 * 3), ("fl", C.c_int32 * 3),
                 ("eaten", C.c_int32 * 3), ("F", C.c_int32), ("ep_t", C.c_int32),
-                ("done", C.c_int32), ("ret", C.c_float)]
+                ("done", C.c_int32), ("ret", C.c_float), ("ix", C.c_int32 * 2),
+                ("iy", C.c_int32 * 2)]
 
 
 class OcState(C.Structure):
@@ -143,6 +153,8 @@ def lib() -> C.CDLL:
             L.orc_lbf_step.argtypes = [C.POINTER(EnvDesc), C.POINTER(LbfState), C.c_int32, C.c_int32, _P, _P]
             L.orc_lbf_step.restype = C.c_int32
             L.orc_lbf_obs.argtypes = [C.POINTER(EnvDesc), C.POINTER(LbfState), C.c_int32, _P]
+            L.orc_lbf_heuristic.argtypes = [C.POINTER(EnvDesc), C.POINTER(LbfState), C.c_int32, C.c_int32]
+            L.orc_lbf_heuristic.restype = C.c_int32
             L.orc_oc_cell.argtypes = [C.c_int32, C.c_int32]
             L.orc_oc_cell.restype = C.c_int32
             L.orc_oc_reset.argtypes = [C.POINTER(EnvDesc), C.POINTER(OcState)]
@@ -466,3 +478,7 @@ def ppo_update(net, params, m, v, t, batch: PpoBatchNp, hp, n_threads=1):
     lib().orc_ppo_update(C.byref(net), _ptr(params), _ptr(m), _ptr(v), C.byref(tt),
                          C.byref(batch.c), batch.S, C.byref(hp), _ptr(stats), n_threads)
     return tt.value, stats
+
+
+def lbf_heuristic(d, state, seat, k):
+    return int(lib().orc_lbf_heuristic(C.byref(d), C.byref(state), seat, k))

@@ -152,6 +152,8 @@ extern "C" void orc_lbf_reset(const orc_env_desc* d, uint64_t seed, uint32_t env
   for (int i = 0; i < 2; ++i) {
     s->ax[i] = perm[d->n_food + i] % d->width;
     s->ay[i] = perm[d->n_food + i] / d->width;
+    s->ix[i] = s->ax[i];
+    s->iy[i] = s->ay[i];
   }
   s->ep_t = 0;
   s->done = 0;
@@ -224,6 +226,56 @@ extern "C" int32_t orc_lbf_step(const orc_env_desc* d, orc_lbf_state* s, int32_t
   *team = r[0] + r[1];
   s->ret = s->ret + *team;
   return s->done;
+}
+
+extern "C" int32_t orc_lbf_heuristic(const orc_env_desc* d, const orc_lbf_state* s, int32_t seat,
+                                     int32_t k) {
+  const int me = seat, other = 1 - seat;
+  auto dist = [&](int x, int y, int f) { return std::abs(x - s->fx[f]) + std::abs(y - s->fy[f]); };
+  // the food to go for
+  int target = -1;
+  long best = 0;
+  for (int f = 0; f < d->n_food; ++f) {
+    if (s->eaten[f]) continue;
+    long key = 0;
+    switch (k) {
+      case 0: key = dist(s->ax[me], s->ay[me], f); break;
+      case 1: key = dist(s->ax[other], s->ay[other], f); break;
+      case 2: key = dist(s->ax[me], s->ay[me], f) + dist(s->ax[other], s->ay[other], f); break;
+      case 3: key = s->fl[f]; break;
+      case 4: key = -s->fl[f]; break;
+      case 5: key = s->fy[f] * d->width + s->fx[f]; break;
+      case 6: key = -(s->fy[f] * d->width + s->fx[f]); break;
+      case 7: key = s->fx[f] * d->height + s->fy[f]; break;
+      case 8: key = -(s->fx[f] * d->height + s->fy[f]); break;
+      case 9: key = dist(s->ix[me], s->iy[me], f); break;
+      case 10: key = -dist(s->ix[me], s->iy[me], f); break;
+      default: return 0;
+    }
+    if (target < 0 || key < best) {  // strict: the lower food index wins ties
+      target = f;
+      best = key;
+    }
+  }
+  if (target < 0) return 0;
+  const int x = s->ax[me], y = s->ay[me];
+  const int dx = s->fx[target] - x, dy = s->fy[target] - y;
+  if (std::abs(dx) + std::abs(dy) == 1) return kLbfLoad;
+  auto free_cell = [&](int cx, int cy) {
+    if (cx < 0 || cx >= d->width || cy < 0 || cy >= d->height) return false;
+    for (int f = 0; f < d->n_food; ++f)
+      if (!s->eaten[f] && s->fx[f] == cx && s->fy[f] == cy) return false;
+    return !(s->ax[other] == cx && s->ay[other] == cy);
+  };
+  const int x_act = dx > 0 ? 4 : 3, y_act = dy > 0 ? 2 : 1;  // E / W, S / N
+  const int sx = dx > 0 ? 1 : -1, sy = dy > 0 ? 1 : -1;
+  const bool x_first = std::abs(dx) >= std::abs(dy);
+  for (int c = 0; c < 2; ++c) {
+    const bool along_x = (c == 0) == x_first;
+    if (along_x && dx != 0 && free_cell(x + sx, y)) return x_act;
+    if (!along_x && dy != 0 && free_cell(x, y + sy)) return y_act;
+  }
+  return 0;
 }
 
 extern "C" void orc_lbf_obs(const orc_env_desc* d, const orc_lbf_state* s, int32_t seat,
@@ -909,8 +961,9 @@ extern "C" int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32
   if (orc_check_desc(d) != 0) return -1;
   if (turn_based(d)) return -3;  // PPO collection is for simultaneous-move games
   if (io->ego_id < 0 || io->ego_id >= n_pols || io->pool_size < 1) return -4;
+  const int min_id = d->kind == ORC_LBF ? -ORC_LBF_N_HEURISTICS : 0;  // heuristic teammates
   for (int k = 0; k < io->pool_size; ++k)
-    if (io->pool[k] < 0 || io->pool[k] >= n_pols) return -4;
+    if (io->pool[k] < min_id || io->pool[k] >= n_pols) return -4;
   const int od = orc_obs_dim(d), K = orc_n_actions(d);
   const int64_t N = io->n_envs;
   const int T = io->T;
@@ -925,10 +978,10 @@ extern "C" int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32
     const uint32_t x = orc_draw(io->seed, first, (uint32_t)io->step0, ORC_STREAM_TEAMMATE, 0);
     const int tm_id = io->pool[orc_uniform_int(x, (uint32_t)io->pool_size)];
     if (io->teammate) io->teammate[e] = tm_id;
-    const orc_mlp* tm = &pols[tm_id];
+    const orc_mlp* tm = tm_id >= 0 ? &pols[tm_id] : nullptr;  // null: a heuristic teammate
     orc_state* st = &io->states[e];
     std::vector<uint8_t> o0(od), o1(od), legal(K, 1);
-    std::vector<double> z0(ego->n_out), z1(tm->n_out);
+    std::vector<double> z0(ego->n_out), z1(tm ? tm->n_out : 1);
     for (int t = 0; t < T; ++t) {
       const uint32_t gt = (uint32_t)(io->step0 + t);
       const int64_t i = (int64_t)t * N + e;
@@ -937,13 +990,19 @@ extern "C" int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32
       if (io->obs) std::memcpy(io->obs + i * od, o0.data(), od);
       if (io->obs_tm) std::memcpy(io->obs_tm + i * od, o1.data(), od);
       orc_mlp_forward(ego, obs_to_double(o0.data(), od).data(), z0.data());
-      orc_mlp_forward(tm, obs_to_double(o1.data(), od).data(), z1.data());
       int own[2];
       double lp[2], mg[2];
       orc_sample(z0.data(), legal.data(), K, orc_u01(orc_draw(io->seed, env, gt, ORC_STREAM_ACT0, 0)),
                  &own[0], &lp[0], &mg[0]);
-      orc_sample(z1.data(), legal.data(), K, orc_u01(orc_draw(io->seed, env, gt, ORC_STREAM_ACT1, 0)),
-                 &own[1], &lp[1], &mg[1]);
+      if (tm) {
+        orc_mlp_forward(tm, obs_to_double(o1.data(), od).data(), z1.data());
+        orc_sample(z1.data(), legal.data(), K, orc_u01(orc_draw(io->seed, env, gt, ORC_STREAM_ACT1, 0)),
+                   &own[1], &lp[1], &mg[1]);
+      } else {
+        own[1] = orc_lbf_heuristic(d, (const orc_lbf_state*)st, 1, -1 - tm_id);
+        lp[1] = 0.0;
+        mg[1] = 2.0;  // no draw: never flagged
+      }
       int act[2] = {own[0], own[1]};
       if (io->forced) {
         act[0] = io->forced[i * 2];
@@ -978,8 +1037,9 @@ extern "C" int32_t orc_xplay(const orc_env_desc* d, const orc_mlp* pols, int32_t
   if (orc_check_desc(d) != 0) return -1;
   for (int i = 0; i < io->n_ego; ++i)
     if (io->ego_ids[i] < 0 || io->ego_ids[i] >= n_pols) return -4;
+  const int min_id = d->kind == ORC_LBF ? -ORC_LBF_N_HEURISTICS : 0;  // heuristic teammates
   for (int j = 0; j < io->n_tm; ++j)
-    if (io->tm_ids[j] < 0 || io->tm_ids[j] >= n_pols) return -4;
+    if (io->tm_ids[j] < min_id || io->tm_ids[j] >= n_pols) return -4;
   const int od = orc_obs_dim(d), K = orc_n_actions(d);
   const int P = io->envs_per_pair;
   const int64_t n_all = (int64_t)io->n_ego * io->n_tm * P;
@@ -992,11 +1052,12 @@ extern "C" int32_t orc_xplay(const orc_env_desc* d, const orc_mlp* pols, int32_t
     const int64_t g = io->env_ids ? io->env_ids[e] : e;  // global env index
     const uint32_t env = (uint32_t)g;
     const int64_t pair = g / P;
-    const orc_mlp* pol[2] = {&pols[io->ego_ids[pair / io->n_tm]], &pols[io->tm_ids[pair % io->n_tm]]};
+    const int tm_id = io->tm_ids[pair % io->n_tm];
+    const orc_mlp* pol[2] = {&pols[io->ego_ids[pair / io->n_tm]], tm_id >= 0 ? &pols[tm_id] : nullptr};
     orc_state st;
     env_reset(d, io->seed, env, (uint32_t)io->step0, &st);
     std::vector<uint8_t> o(od), legal(K);
-    std::vector<double> z(std::max(pol[0]->n_out, pol[1]->n_out));
+    std::vector<double> z(std::max(pol[0]->n_out, pol[1] ? pol[1]->n_out : 1));
     int steps = 0;
     bool done = false;
     for (int s = 0; s < io->max_steps; ++s) {
@@ -1010,6 +1071,14 @@ extern "C" int32_t orc_xplay(const orc_env_desc* d, const orc_mlp* pols, int32_t
       int act[2] = {0, 0};
       for (int seat = 0; seat < 2; ++seat) {
         if (actor >= 0 && seat != actor) continue;
+        if (!pol[seat]) {  // heuristic teammate: its rule, no draw
+          act[seat] = io->forced ? io->forced[i * 2 + seat]
+                                 : orc_lbf_heuristic(d, (const orc_lbf_state*)&st, seat, -1 - tm_id);
+          if (io->actions) io->actions[i * 2 + seat] = (uint8_t)act[seat];
+          if (io->own_actions)
+            io->own_actions[i * 2 + seat] = (uint8_t)orc_lbf_heuristic(d, (const orc_lbf_state*)&st, seat, -1 - tm_id);
+          continue;
+        }
         env_obs(d, &st, seat, o.data());
         env_legal(d, &st, legal.data());
         orc_mlp_forward(pol[seat], obs_to_double(o.data(), od).data(), z.data());

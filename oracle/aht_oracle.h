@@ -75,6 +75,7 @@ typedef struct orc_lbf_state {
   int32_t ep_t;                        /* steps taken in this episode */
   int32_t done;                        /* the last step ended the episode */
   float ret;                           /* team return of this episode */
+  int32_t ix[2], iy[2];                /* agent positions at the episode's start */
 } orc_lbf_state;
 void orc_lbf_reset(const orc_env_desc* d, uint64_t seed, uint32_t env, uint32_t step,
                    orc_lbf_state* s);
@@ -82,6 +83,22 @@ void orc_lbf_reset(const orc_env_desc* d, uint64_t seed, uint32_t env, uint32_t 
 int32_t orc_lbf_step(const orc_env_desc* d, orc_lbf_state* s, int32_t a0, int32_t a1,
                      float r[2], float* team);
 void orc_lbf_obs(const orc_env_desc* d, const orc_lbf_state* s, int32_t seat, uint8_t* out);
+
+/* Rule-based LBF teammates (App. F, LBF heuristic suite: Greedy picks the next uneaten
+ * food online by a criterion, Sequential plans a food order before the episode).  The
+ * paper names the criteria and orderings only; the rules are the readings in the design doc:
+ *   k = 0..4  Greedy: argmin over uneaten foods of dist(self) | dist(teammate) |
+ *             dist(self) + dist(teammate) | level | -level (ties: lower food index);
+ *   k = 5..10 Sequential: the first uneaten food in the order of row-major cell index
+ *             (y W + x) ascending | descending, column-major index (x H + y) ascending |
+ *             descending, distance from the agent's position at the episode's start
+ *             ascending | descending (ties: lower food index);
+ * then the action toward it: load (5) when 4-adjacent; else a step along the axis with
+ * the larger remaining distance (ties: x), or along the other axis if that cell is off
+ * the grid, an uneaten food or the other agent; else noop.  dist is Manhattan.  A
+ * teammate id t < 0 in a pool or teammate list means heuristic k = -1 - t (LBF only). */
+enum { ORC_LBF_N_HEURISTICS = 11 };
+int32_t orc_lbf_heuristic(const orc_env_desc* d, const orc_lbf_state* s, int32_t seat, int32_t k);
 
 /* ---- Overcooked-style kitchen (fixed 5x4 layout) -------------------------------- */
 enum { ORC_OC_NONE = 0, ORC_OC_ONION = 1, ORC_OC_DISH = 2, ORC_OC_SOUP = 3 };
