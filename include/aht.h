@@ -98,6 +98,25 @@ typedef struct aht_pop_desc {
   const void* const* b;          /* host array of 3*n_policies pointers */
 } aht_pop_desc;
 
+/* Rule-based LBF teammates (App. F, LBF heuristic suite).  A teammate id -1 - k in a
+ * pool (aht_rollout) or teammate list (aht_xplay_matrix, aht_xplay_matrix_static) of an
+ * LBF context whose policies run on the tensor-core path (hidden widths 64 or 128,
+ * obs_dim <= 255, at most 7 actions + value; fp32 or bf16) selects heuristic k instead of
+ * a network (other contexts return AHT_EINVAL for negative ids):
+ *   k 0..4  Greedy: the uneaten food with the least distance to itself | distance to the
+ *           ego | sum of the two | level | the greatest level (ties: lower food index);
+ *   k 5..10 Sequential: the first uneaten food in the order of row-major cell index
+ *           (y*width + x) ascending | descending, column-major index (x*height + y)
+ *           ascending | descending, distance from its own position at the episode's start
+ *           ascending | descending (ties: lower food index);
+ * then: load when 4-adjacent to it; else one step along the axis with the larger
+ * remaining distance (ties: x), or along the other axis when that cell is off the grid,
+ * an uneaten food or the ego; else noop (distances Manhattan).  The rule draws nothing;
+ * the teammate's recorded action is the rule's.  The paper names the criteria and
+ * orderings only: the rules above are this library's reading. */
+#define AHT_LBF_N_HEURISTICS 11
+#define AHT_LBF_HEURISTIC(k) (-1 - (k))
+
 /* Creates a context for up to n_envs concurrent envs (PPO state and cross-play batch
  * capacity), packs the population and resets every env with `seed` (step counter 0).
  * cuda_stream is a cudaStream_t (NULL = default stream).  Allocates all device memory

@@ -741,8 +741,11 @@ aht_status aht_rollout(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t 
   if (c->env.kind == AHT_HANABI) return fail(AHT_EINVAL, "PPO collection needs a simultaneous-move env (LBF, Overcooked)");
   if (ego_id < 0 || ego_id >= c->n_policies) return fail(AHT_EINVAL, "ego_id out of range");
   if (!pool || pool_size < 1 || pool_size > kMaxPool) return fail(AHT_EINVAL, "pool_size must be in 1..256");
-  for (int k = 0; k < pool_size; ++k)
-    if (pool[k] < 0 || pool[k] >= c->n_policies) return fail(AHT_EINVAL, "pool id out of range");
+  for (int k = 0; k < pool_size; ++k) {
+    if (pool[k] >= c->n_policies || pool[k] < -AHT_LBF_N_HEURISTICS) return fail(AHT_EINVAL, "pool id out of range");
+    if (pool[k] < 0 && !(c->env.kind == AHT_LBF && c->tc))
+      return fail(AHT_EINVAL, "heuristic teammates (negative ids) need an LBF context on the tensor-core path");
+  }
   if (T < 1) return fail(AHT_EINVAL, "T must be >= 1");
   if (c->step + T + 1 > (int64_t)UINT32_MAX) return fail(AHT_EINVAL, "step counter would exceed 2^32");
   if (out->advantages && (!out->rewards || !out->values || !out->dones))
@@ -815,8 +818,12 @@ aht_status aht_xplay_matrix(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego,
     return fail(AHT_EINVAL, "n_ego and n_tm must be in 1..64");
   for (int i = 0; i < n_ego; ++i)
     if (ego_ids[i] < 0 || ego_ids[i] >= c->n_policies) return fail(AHT_EINVAL, "ego id out of range");
-  for (int j = 0; j < n_tm; ++j)
-    if (tm_ids[j] < 0 || tm_ids[j] >= c->n_policies) return fail(AHT_EINVAL, "teammate id out of range");
+  for (int j = 0; j < n_tm; ++j) {
+    if (tm_ids[j] >= c->n_policies || tm_ids[j] < -AHT_LBF_N_HEURISTICS)
+      return fail(AHT_EINVAL, "teammate id out of range");
+    if (tm_ids[j] < 0 && !(c->env.kind == AHT_LBF && c->tc))
+      return fail(AHT_EINVAL, "heuristic teammates (negative ids) need an LBF context on the tensor-core path");
+  }
   if (envs_per_pair < 1 || envs_per_pair > (1 << 14)) return fail(AHT_EINVAL, "envs_per_pair must be in 1..16384");
   if (max_steps < 1) return fail(AHT_EINVAL, "max_steps must be >= 1");
   const int64_t n_pairs = (int64_t)n_ego * n_tm;
@@ -905,8 +912,12 @@ aht_status aht_xplay_matrix_static(aht_ctx* c, const int32_t* ego_ids, int32_t n
     return fail(AHT_EINVAL, "n_ego and n_tm must be in 1..64");
   for (int i = 0; i < n_ego; ++i)
     if (ego_ids[i] < 0 || ego_ids[i] >= c->n_policies) return fail(AHT_EINVAL, "ego id out of range");
-  for (int j = 0; j < n_tm; ++j)
-    if (tm_ids[j] < 0 || tm_ids[j] >= c->n_policies) return fail(AHT_EINVAL, "teammate id out of range");
+  for (int j = 0; j < n_tm; ++j) {
+    if (tm_ids[j] >= c->n_policies || tm_ids[j] < -AHT_LBF_N_HEURISTICS)
+      return fail(AHT_EINVAL, "teammate id out of range");
+    if (tm_ids[j] < 0 && !(c->env.kind == AHT_LBF && c->tc))
+      return fail(AHT_EINVAL, "heuristic teammates (negative ids) need an LBF context on the tensor-core path");
+  }
   if (envs_per_pair < 1 || envs_per_pair > (1 << 14)) return fail(AHT_EINVAL, "envs_per_pair must be in 1..16384");
   if (max_steps < 1) return fail(AHT_EINVAL, "max_steps must be >= 1");
   const int64_t n_pairs = (int64_t)n_ego * n_tm;

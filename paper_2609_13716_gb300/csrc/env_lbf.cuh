@@ -16,7 +16,7 @@ struct EnvLbf {
   struct State {
     uint8_t ax[2], ay[2];
     uint8_t al[2], F, eaten;  // eaten: bit k set when food k is gone (absent foods too)
-    uint8_t fx[4], fy[4], fl[4];
+    uint8_t fx[4], fy[4], fl[4];  // slot 3 of fx / fy: agent 1's position at the episode start
     uint32_t ep_t;
     float ret;
   };
@@ -70,11 +70,13 @@ struct EnvLbf {
         s.eaten |= (uint8_t)(1u << k);
       }
     }
-    s.fx[3] = s.fy[3] = s.fl[3] = 0;
+    s.fl[3] = 0;
     for (int i = 0; i < 2; ++i) {
       s.ax[i] = (uint8_t)(placed[d.n_food + i] % d.width);
       s.ay[i] = (uint8_t)(placed[d.n_food + i] / d.width);
     }
+    s.fx[3] = s.ax[1];  // the start position a Sequential teammate plans from
+    s.fy[3] = s.ay[1];
     s.ep_t = 0;
     s.ret = 0.0f;
   }
@@ -158,6 +160,57 @@ struct EnvLbf {
     const int o = 1 - seat;
     put(s.ax[o], s.ay[o], (uint32_t)s.al[o] << 8);
     put(s.ax[seat], s.ay[seat], (uint32_t)s.al[seat]);
+  }
+
+  // Rule-based teammate k in seat 1 (the LBF heuristic suite: Greedy criteria 0..4,
+  // Sequential orderings 5..10): the food to go for, then load when 4-adjacent, else a
+  // step along the axis with the larger remaining distance (ties: x), else along the
+  // other axis, when the cell is on the grid and free of uneaten food and of agent 0.
+  __device__ static int heuristic(const DevEnv& d, const State& s, int k) {
+    const int x = s.ax[1], y = s.ay[1], ox = s.ax[0], oy = s.ay[0];
+    int target = -1, best = 0;
+#pragma unroll
+    for (int f = 0; f < 3; ++f) {
+      if ((s.eaten >> f) & 1u) continue;  // absent foods are marked eaten
+      const int fx = s.fx[f], fy = s.fy[f];
+      const int d_me = abs(x - fx) + abs(y - fy), d_tm = abs(ox - fx) + abs(oy - fy);
+      const int d_start = abs((int)s.fx[3] - fx) + abs((int)s.fy[3] - fy);
+      const int rm = fy * d.width + fx, cm = fx * d.height + fy;
+      int key;
+      switch (k) {
+        case 0: key = d_me; break;
+        case 1: key = d_tm; break;
+        case 2: key = d_me + d_tm; break;
+        case 3: key = s.fl[f]; break;
+        case 4: key = -(int)s.fl[f]; break;
+        case 5: key = rm; break;
+        case 6: key = -rm; break;
+        case 7: key = cm; break;
+        case 8: key = -cm; break;
+        case 9: key = d_start; break;
+        default: key = -d_start; break;
+      }
+      if (target < 0 || key < best) {
+        target = f;
+        best = key;
+      }
+    }
+    if (target < 0) return 0;
+    const int dx = (int)s.fx[target] - x, dy = (int)s.fy[target] - y;
+    if (abs(dx) + abs(dy) == 1) return 5;
+    auto free_cell = [&](int cx, int cy) {
+      if (cx < 0 || cx >= d.width || cy < 0 || cy >= d.height) return false;
+#pragma unroll
+      for (int f = 0; f < 3; ++f)
+        if (!((s.eaten >> f) & 1u) && s.fx[f] == cx && s.fy[f] == cy) return false;
+      return !(ox == cx && oy == cy);
+    };
+    const int sx = dx > 0 ? 1 : -1, sy = dy > 0 ? 1 : -1;
+    const bool xmove = dx != 0 && free_cell(x + sx, y);
+    const bool ymove = dy != 0 && free_cell(x, y + sy);
+    const int x_act = dx > 0 ? 4 : 3, y_act = dy > 0 ? 2 : 1;
+    if (abs(dx) >= abs(dy)) return xmove ? x_act : (ymove ? y_act : 0);
+    return ymove ? y_act : (xmove ? x_act : 0);
   }
 
   __device__ static uint32_t legal(const State&) { return 0x3Fu; }

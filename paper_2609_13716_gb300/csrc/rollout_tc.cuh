@@ -69,6 +69,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     tm_pol = tile.z;
   }
   if (count <= 0) return;
+  // a negative teammate id is LBF heuristic -1 - id: no teammate network, its rule acts
+  const bool tm_rule = tm_pol < 0;
+  const int tm_k = -1 - tm_pol;
   const TcDims& d = a.tc;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, half = (warp >> 2) & 1, row = tid & 127;
   const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
@@ -116,8 +119,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     // ================================ MMA warp =====================================
     if (lane == 0) {
       const int pol[2] = {ego_pol, tm_pol};
-      tc::mbar_expect_tx(&wload_bar, 2u * d.pol_bytes);
-      for (int p = 0; p < 2; ++p) {
+      const int n_pol = tm_rule ? 1 : 2;
+      tc::mbar_expect_tx(&wload_bar, (uint32_t)n_pol * d.pol_bytes);
+      for (int p = 0; p < n_pol; ++p) {
         const uint8_t* src = a.tcw + (int64_t)pol[p] * d.pol_bytes;
         for (uint32_t off = 0; off < d.pol_bytes; off += 32768u)
           tc::bulk_g2s(sW0 + p * d.pol_bytes + off, src + off, min(32768u, d.pol_bytes - off), &wload_bar);
@@ -160,9 +164,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       const int n_steps = kXp ? a.xp.max_steps : a.T;
       for (int t = 0; ok && !stopped && t < n_steps; ++t) {
         const uint32_t par = (uint32_t)t & 1u;
-        issue(1, 0, par);
+        if (!tm_rule) issue(1, 0, par);
         if (ok && !stopped) issue(0, 0, par);
-        if (ok && !stopped) issue(1, 1, par);
+        if (ok && !stopped && !tm_rule) issue(1, 1, par);
         if (ok && !stopped) issue(0, 1, par);
       }
       if (ok && with_boot) {
@@ -312,11 +316,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         // every env of the tile is done: release the MMA warp without operands and stop
         if (!tc::bar_or(kTcComputeBar, kTcCompute, half == 0 && row < count && alive)) {
           if (tid == 0) stop_flag = 1;
-          tc::mbar_arrive(&opnd_bar[2]);  // the teammate's L1 barrier it waits on
+          tc::mbar_arrive(&opnd_bar[tm_rule ? 0 : 2]);  // the first L1 barrier it waits on
           break;
         }
       }
-      const int first = boot ? 0 : 1;  // teammate first: the ego's rows stay for the copy
+      const int first = boot || tm_rule ? 0 : 1;  // teammate first: the ego's rows stay for the copy
       const uint32_t par = (uint32_t)t & 1u, gt = a.step0 + (uint32_t)t;
       // this half's action draw (ego: warps 0-3, teammate: warps 4-7), ahead of its use
       const float u_act = boot ? 0.0f : u01(draw0(a.b.key, (uint32_t)(env0 + row), gt, kStreamAct0 + half));
@@ -349,7 +353,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       }
       int act0 = 0;
       float lp0 = 0.f, val0 = 0.f;
-      if (row < count) {
+      if (row < count && half == 1 && tm_rule) {
+        act1s[row] = (uint8_t)Env::heuristic(a.b.env, s, tm_k);
+      } else if (row < count) {
         const int ag = half == 0 ? 0 : 1;
         logits(ag, z);
         float lp;
