@@ -435,7 +435,8 @@ def run_ppo_update(args, aht, wl, pop_np, traj, torch, bf16_peak, stream):
     return res
 
 
-XPLAY_WORKLOADS = ("lbf7x7_xplay_8x16x256", "overcooked5x4_xplay_8x8x64", "hanabi_xplay_16x16x32")
+XPLAY_WORKLOADS = ("lbf7x7_xplay_8x16x256", "lbf7x7_xplay_heuristics_8x11x256",
+                   "overcooked5x4_xplay_8x8x64", "hanabi_xplay_16x16x32")
 
 
 def run_xplay(args, aht, W, torch, bf16_peak, names=XPLAY_WORKLOADS):
@@ -489,6 +490,8 @@ def run_xplay(args, aht, W, torch, bf16_peak, names=XPLAY_WORKLOADS):
         ctx.close()
         dims = [wl.env.obs_dim, *wl.hidden, wl.env.n_actions]
         acting = 1 if wl.env.kind == W.HANABI else 2        # Hanabi: one actor per turn
+        if min(wl.tm_ids) < 0:                              # rule-based teammates: no network
+            acting = 1
         flops = active * acting * mlp_flops(dims)
         tflops = flops / (ms * 1e-3) / 1e12
         res[name] = {"cells_per_s": ne * nt / (ms * 1e-3), "ms_per_matrix": ms,

@@ -95,6 +95,12 @@ WORKLOADS = {
         weight_dtype=FP32, n_policies=24, value_head=(0,) * 24, mode="xplay", env_seed=1,
         ego_ids=tuple(range(8)), tm_ids=tuple(range(8, 24)), envs_per_pair=256,
         max_steps=128),
+    # The same 8 egos (same seeds) against the 11 rule-based LBF teammates (ids -1..-11).
+    "lbf7x7_xplay_heuristics_8x11x256": Workload(
+        name="lbf7x7_xplay_heuristics_8x11x256", index=1, env=_lbf(128), hidden=(64, 64),
+        weight_dtype=FP32, n_policies=8, value_head=(0,) * 8, mode="xplay", env_seed=1,
+        ego_ids=tuple(range(8)), tm_ids=tuple(-1 - k for k in range(11)), envs_per_pair=256,
+        max_steps=128),
     # LBF 7x7 PPO collection: 16384 envs x 128 steps, ego actor-critic 196-128-128-(6+1),
     # teammates drawn uniformly from a 32-policy population, bf16 weights.
     "lbf7x7_ppo_16384x128": Workload(
