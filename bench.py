@@ -436,7 +436,7 @@ def run_ppo_update(args, aht, wl, pop_np, traj, torch, bf16_peak, stream):
 
 
 XPLAY_WORKLOADS = ("lbf7x7_xplay_8x16x256", "lbf7x7_xplay_heuristics_8x11x256",
-                   "overcooked5x4_xplay_8x8x64", "hanabi_xplay_16x16x32")
+                   "lbf12x12_xplay_8x16x128", "overcooked5x4_xplay_8x8x64", "hanabi_xplay_16x16x32")
 
 
 def run_xplay(args, aht, W, torch, bf16_peak, names=XPLAY_WORKLOADS):
@@ -476,16 +476,22 @@ def run_xplay(args, aht, W, torch, bf16_peak, names=XPLAY_WORKLOADS):
                   max_regret=torch.empty(ne, device="cuda"),
                   worst_tm=torch.empty(ne, dtype=torch.int32, device="cuda"),
                   brdiv=torch.empty(1, device="cuda") if ne == nt else None)
-        stream = torch.cuda.current_stream()
         for _ in range(3):
-            aht.aht_xp_stats(matrix, upper, **so, stream=stream)
+            aht.aht_xp_stats(matrix, upper, **so)
+        torch.cuda.synchronize()
+        # one small kernel per call: replay a CUDA graph of 50 calls, so that the host's
+        # per-call binding overhead does not leave the device idle between them
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            for _ in range(50):
+                aht.aht_xp_stats(matrix, upper, **so)
+        graph.replay()
         torch.cuda.synchronize()
         s.record()
-        for _ in range(K):
-            aht.aht_xp_stats(matrix, upper, **so, stream=stream)
+        graph.replay()
         e.record()
         torch.cuda.synchronize()
-        stats_us = s.elapsed_time(e) / K * 1e3
+        stats_us = s.elapsed_time(e) / 50 * 1e3
         aht.aht_sync(ctx)
         ctx.close()
         dims = [wl.env.obs_dim, *wl.hidden, wl.env.n_actions]

@@ -101,6 +101,20 @@ WORKLOADS = {
         weight_dtype=FP32, n_policies=8, value_head=(0,) * 8, mode="xplay", env_seed=1,
         ego_ids=tuple(range(8)), tm_ids=tuple(-1 - k for k in range(11)), envs_per_pair=256,
         max_steps=128),
+    # LBF 12x12 (the paper's second LBF grid, Sec. 4 Table "JaxAHT Environments"): 8 egos
+    # x 16 teammates, 128 envs per pair, 128-step episodes, fp32 576-64-64-6 MLPs.
+    "lbf12x12_xplay_8x16x128": Workload(
+        name="lbf12x12_xplay_8x16x128", index=6, env=EnvSpec(kind=LBF, width=12, height=12, n_food=3,
+                                                           max_agent_level=3, episode_len=128),
+        hidden=(64, 64), weight_dtype=FP32, n_policies=24, value_head=(0,) * 24, mode="xplay",
+        env_seed=6, ego_ids=tuple(range(8)), tm_ids=tuple(range(8, 24)), envs_per_pair=128,
+        max_steps=128),
+    # LBF 12x12 PPO collection: 4096 envs x 128 steps, ego 576-128-128-(6+1) vs 8 teammates, bf16.
+    "lbf12x12_ppo_4096x128": Workload(
+        name="lbf12x12_ppo_4096x128", index=7, env=EnvSpec(kind=LBF, width=12, height=12, n_food=3,
+                                                         max_agent_level=3, episode_len=50),
+        hidden=(128, 128), weight_dtype=BF16, n_policies=9, value_head=(1,) + (0,) * 8, mode="ppo",
+        env_seed=7, n_envs=4096, T=128, ego_id=0, pool=tuple(range(1, 9))),
     # LBF 7x7 PPO collection: 16384 envs x 128 steps, ego actor-critic 196-128-128-(6+1),
     # teammates drawn uniformly from a 32-policy population, bf16 weights.
     "lbf7x7_ppo_16384x128": Workload(
