@@ -166,7 +166,7 @@ struct EnvLbf {
   // Sequential orderings 5..10): the food to go for, then load when 4-adjacent, else a
   // step along the axis with the larger remaining distance (ties: x), else along the
   // other axis, when the cell is on the grid and free of uneaten food and of agent 0.
-  __device__ static int heuristic(const DevEnv& d, const State& s, int k) {
+  __device__ __noinline__ static int heuristic(const DevEnv& d, const State& s, int k) {
     const int x = s.ax[1], y = s.ay[1], ox = s.ax[0], oy = s.ay[0];
     int target = -1, best = 0;
 #pragma unroll

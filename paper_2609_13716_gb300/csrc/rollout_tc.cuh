@@ -71,7 +71,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   if (count <= 0) return;
   // a negative teammate id is LBF heuristic -1 - id: no teammate network, its rule acts
   const bool tm_rule = tm_pol < 0;
-  const int tm_k = -1 - tm_pol;
   const TcDims& d = a.tc;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, half = (warp >> 2) & 1, row = tid & 127;
   const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
@@ -354,7 +353,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       int act0 = 0;
       float lp0 = 0.f, val0 = 0.f;
       if (row < count && half == 1 && tm_rule) {
-        act1s[row] = (uint8_t)Env::heuristic(a.b.env, s, tm_k);
+        act1s[row] = (uint8_t)Env::heuristic(a.b.env, st[row], -1 - tm_pol);  // st[row] == s here
       } else if (row < count) {
         const int ag = half == 0 ? 0 : 1;
         logits(ag, z);
