@@ -26,7 +26,7 @@ _HDR = os.path.join(_HERE, "aht_oracle.h")
 _lock = threading.Lock()
 _lib = None
 
-LBF, OVERCOOKED, HANABI = 0, 1, 2
+LBF, OVERCOOKED, HANABI, MINI_HANABI = 0, 1, 2, 3
 STREAM_ACT0, STREAM_ACT1, STREAM_RESET, STREAM_TEAMMATE = 0, 1, 2, 3
 STATE_BYTES = 768
 # LBF heuristic teammates: teammate id -1 - k (App. F LBF suite; rules in aht_oracle.h)
@@ -74,6 +74,19 @@ class OcState(C.Structure):
                 ("held", C.c_int32 * 2), ("pot_n", C.c_int32), ("pot_timer", C.c_int32),
                 ("counter_item", C.c_int32 * 20), ("ep_t", C.c_int32), ("done", C.c_int32),
                 ("ret", C.c_float)]
+
+
+class MiniHanabiState(C.Structure):
+    _fields_ = [("deck", C.c_int32 * 18), ("ptr", C.c_int32),
+                ("hand", (C.c_int32 * 2) * 2), ("n_hand", C.c_int32 * 2),
+                ("know", (C.c_uint32 * 2) * 2), ("hint_col", (C.c_uint32 * 2) * 2),
+                ("hint_rank", (C.c_uint32 * 2) * 2), ("fw", C.c_int32 * 3),
+                ("info", C.c_int32), ("lives", C.c_int32), ("score", C.c_int32),
+                ("disc", C.c_int32 * 9), ("fr", C.c_int32), ("turn", C.c_int32),
+                ("la_valid", C.c_int32), ("la_actor", C.c_int32), ("la_type", C.c_int32),
+                ("la_colour", C.c_int32), ("la_rank", C.c_int32), ("la_slot", C.c_int32),
+                ("la_card", C.c_int32), ("la_hinted", C.c_int32), ("la_success", C.c_int32),
+                ("la_bomb", C.c_int32), ("done", C.c_int32), ("ret", C.c_float)]
 
 
 class HanabiState(C.Structure):
@@ -166,6 +179,11 @@ def lib() -> C.CDLL:
             L.orc_hanabi_step.argtypes = [C.POINTER(HanabiState), C.c_int32, _P]
             L.orc_hanabi_step.restype = C.c_int32
             L.orc_hanabi_obs.argtypes = [C.POINTER(HanabiState), C.c_int32, _P]
+            L.orc_mhanabi_reset.argtypes = [C.c_uint64, C.c_uint32, C.c_uint32, C.POINTER(MiniHanabiState)]
+            L.orc_mhanabi_legal.argtypes = [C.POINTER(MiniHanabiState), _P]
+            L.orc_mhanabi_step.argtypes = [C.POINTER(MiniHanabiState), C.c_int32, _P]
+            L.orc_mhanabi_step.restype = C.c_int32
+            L.orc_mhanabi_obs.argtypes = [C.POINTER(MiniHanabiState), C.c_int32, _P]
             L.orc_mlp_forward.argtypes = [C.POINTER(Mlp), _P, _P]
             L.orc_sample.argtypes = [_P, _P, C.c_int32, C.c_double, _P, _P, _P]
             L.orc_logp.argtypes = [_P, _P, C.c_int32, C.c_int32]

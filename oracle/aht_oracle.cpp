@@ -74,6 +74,7 @@ extern "C" int32_t orc_obs_dim(const orc_env_desc* d) {
     case ORC_LBF: return d->width * d->height * 4;
     case ORC_OVERCOOKED: return 5 * 4 * 26;
     case ORC_HANABI: return 660;
+    case ORC_MINI_HANABI: return 153;
   }
   return -1;
 }
@@ -83,6 +84,7 @@ extern "C" int32_t orc_n_actions(const orc_env_desc* d) {
     case ORC_LBF: return 6;
     case ORC_OVERCOOKED: return 6;
     case ORC_HANABI: return 20;
+    case ORC_MINI_HANABI: return 10;
   }
   return -1;
 }
@@ -100,7 +102,7 @@ extern "C" int32_t orc_check_desc(const orc_env_desc* d) {
     if (d->episode_len < 1 || d->cook_time < 0 || d->cook_time > 255) return -4;
     return 0;
   }
-  if (d->kind == ORC_HANABI) {
+  if (d->kind == ORC_HANABI || d->kind == ORC_MINI_HANABI) {
     if (d->episode_len != 0) return -4;
     return 0;
   }
@@ -703,32 +705,267 @@ extern "C" void orc_hanabi_obs(const orc_hanabi_state* s, int32_t seat, uint8_t*
 }
 
 // ======================================================================================
+// Mini Hanabi, 2 players: 3 colours x ranks (1,1,1,2,2,3), 2-card hands, 3 info and 1
+// life tokens.  Card type = colour*3 + (rank-1).  Actions: 0-1 play slot, 2-3 discard
+// slot, 4-6 hint colour, 7-9 hint rank (to the partner).
+// ======================================================================================
+namespace {
+const int kMhRankOfCopy[6] = {1, 1, 1, 2, 2, 3};
+const int kMhDiscardBase[3] = {0, 3, 5};  // thermometer offset per rank (copies 3, 2, 1)
+const uint32_t kMhAllCards = (1u << 9) - 1;
+uint32_t mh_colour_mask(int c) { return 0x7u << (3 * c); }
+uint32_t mh_rank_mask(int r) {  // r in 1..3
+  uint32_t m = 0;
+  for (int c = 0; c < 3; ++c) m |= 1u << (3 * c + r - 1);
+  return m;
+}
+
+void mh_remove_slot(orc_mhanabi_state* s, int seat, int slot) {
+  for (int k = slot; k < s->n_hand[seat] - 1; ++k) {
+    s->hand[seat][k] = s->hand[seat][k + 1];
+    s->know[seat][k] = s->know[seat][k + 1];
+    s->hint_col[seat][k] = s->hint_col[seat][k + 1];
+    s->hint_rank[seat][k] = s->hint_rank[seat][k + 1];
+  }
+  const int last = s->n_hand[seat] - 1;
+  s->hand[seat][last] = -1;
+  s->know[seat][last] = 0;
+  s->hint_col[seat][last] = 0;
+  s->hint_rank[seat][last] = 0;
+  s->n_hand[seat] -= 1;
+}
+
+void mh_draw(orc_mhanabi_state* s, int seat) {
+  if (s->ptr >= 18) return;
+  const int k = s->n_hand[seat];
+  s->hand[seat][k] = s->deck[s->ptr];
+  s->know[seat][k] = kMhAllCards;
+  s->hint_col[seat][k] = 0;
+  s->hint_rank[seat][k] = 0;
+  s->n_hand[seat] += 1;
+  s->ptr += 1;
+  if (s->ptr == 18) s->fr = 2;
+}
+}  // namespace
+
+extern "C" void orc_mhanabi_reset(uint64_t seed, uint32_t env, uint32_t step,
+                                  orc_mhanabi_state* s) {
+  std::memset(s, 0, sizeof(*s));
+  for (int c = 0; c < 3; ++c)
+    for (int i = 0; i < 6; ++i) s->deck[c * 6 + i] = c * 3 + (kMhRankOfCopy[i] - 1);
+  DrawSeq draws(seed, env, step, ORC_STREAM_RESET);
+  for (int i = 17; i >= 1; --i) {
+    const int j = (int)orc_uniform_int(draws.next(), (uint32_t)(i + 1));
+    std::swap(s->deck[i], s->deck[j]);
+  }
+  for (int seat = 0; seat < 2; ++seat) {
+    for (int k = 0; k < 2; ++k) {
+      s->hand[seat][k] = s->deck[seat * 2 + k];
+      s->know[seat][k] = kMhAllCards;
+    }
+    s->n_hand[seat] = 2;
+  }
+  s->ptr = 4;
+  s->info = 3;
+  s->lives = 1;
+  s->fr = -1;
+}
+
+extern "C" void orc_mhanabi_legal(const orc_mhanabi_state* s, uint8_t legal[10]) {
+  const int me = s->turn % 2, partner = 1 - me;
+  for (int k = 0; k < 2; ++k) {
+    legal[k] = (k < s->n_hand[me]) ? 1 : 0;
+    legal[2 + k] = (k < s->n_hand[me] && s->info < 3) ? 1 : 0;
+  }
+  for (int v = 0; v < 3; ++v) {
+    bool col = false, rank = false;
+    for (int k = 0; k < s->n_hand[partner]; ++k) {
+      const int card = s->hand[partner][k];
+      if (card / 3 == v) col = true;
+      if (card % 3 == v) rank = true;
+    }
+    legal[4 + v] = (s->info > 0 && col) ? 1 : 0;
+    legal[7 + v] = (s->info > 0 && rank) ? 1 : 0;
+  }
+}
+
+extern "C" int32_t orc_mhanabi_step(orc_mhanabi_state* s, int32_t a, float* team) {
+  uint8_t legal[10];
+  orc_mhanabi_legal(s, legal);
+  if (a < 0 || a >= 10 || !legal[a]) return -1;
+  const int me = s->turn % 2, partner = 1 - me;
+  const int fr_start = s->fr;
+  const int score_before = s->score;
+  float reward = 0.0f;
+  s->la_valid = 1;
+  s->la_actor = me;
+  s->la_colour = -1;
+  s->la_rank = 0;
+  s->la_slot = -1;
+  s->la_card = -1;
+  s->la_hinted = 0;
+  s->la_success = 0;
+  s->la_bomb = 0;
+  if (a < 4) {
+    const int slot = a % 2;
+    const int card = s->hand[me][slot];
+    const int c = card / 3, rank = card % 3 + 1;
+    s->la_type = (a < 2) ? 0 : 1;
+    s->la_colour = c;
+    s->la_rank = rank;
+    s->la_slot = slot;
+    s->la_card = card;
+    mh_remove_slot(s, me, slot);
+    if (a < 2) {
+      if (s->fw[c] == rank - 1) {
+        s->fw[c] = rank;
+        s->score += 1;
+        reward = 1.0f;
+        if (rank == 3 && s->info < 3) s->info += 1;
+        s->la_success = 1;
+      } else {
+        s->lives -= 1;
+        s->disc[card] += 1;
+        s->la_bomb = 1;
+      }
+    } else {
+      s->disc[card] += 1;
+      s->info += 1;
+    }
+    mh_draw(s, me);
+  } else {
+    const bool by_colour = (a < 7);
+    const int v = (a - 4) % 3;
+    const uint32_t m = by_colour ? mh_colour_mask(v) : mh_rank_mask(v + 1);
+    s->info -= 1;
+    s->la_type = by_colour ? 2 : 3;
+    if (by_colour) s->la_colour = v; else s->la_rank = v + 1;
+    for (int k = 0; k < s->n_hand[partner]; ++k) {
+      const int card = s->hand[partner][k];
+      const bool match = by_colour ? (card / 3 == v) : (card % 3 == v);
+      if (match) {
+        s->know[partner][k] &= m;
+        if (by_colour) s->hint_col[partner][k] |= 1u << v;
+        else s->hint_rank[partner][k] |= 1u << v;
+        s->la_hinted |= 1 << k;
+      } else {
+        s->know[partner][k] &= ~m;
+      }
+    }
+  }
+  s->turn += 1;
+  int done = 0;
+  if (s->lives == 0) {
+    done = 1;
+    reward = -(float)score_before;
+  } else if (s->score == 9) {
+    done = 1;
+  } else if (fr_start >= 1) {
+    s->fr = fr_start - 1;
+    if (s->fr == 0) done = 1;
+  }
+  s->done = done;
+  *team = reward;
+  s->ret = s->ret + reward;
+  return done;
+}
+
+// 153 bits: partner hand 18, own knowledge 18, partner knowledge 18, fireworks 9, info 3,
+// lives 1, deck 14, discards 18, last action 27, explicit hints 12 + 12, slots 2, final 1.
+extern "C" void orc_mhanabi_obs(const orc_mhanabi_state* s, int32_t seat, uint8_t* out) {
+  std::memset(out, 0, 153);
+  const int me = seat, partner = 1 - seat;
+  int o = 0;
+  for (int k = 0; k < 2; ++k)
+    if (k < s->n_hand[partner]) out[o + k * 9 + s->hand[partner][k]] = 1;
+  o += 18;
+  for (int k = 0; k < 2; ++k)
+    for (int b = 0; b < 9; ++b)
+      if (k < s->n_hand[me] && ((s->know[me][k] >> b) & 1u)) out[o + k * 9 + b] = 1;
+  o += 18;
+  for (int k = 0; k < 2; ++k)
+    for (int b = 0; b < 9; ++b)
+      if (k < s->n_hand[partner] && ((s->know[partner][k] >> b) & 1u)) out[o + k * 9 + b] = 1;
+  o += 18;
+  for (int c = 0; c < 3; ++c)
+    if (s->fw[c] >= 1) out[o + c * 3 + s->fw[c] - 1] = 1;
+  o += 9;
+  for (int i = 0; i < s->info; ++i) out[o + i] = 1;
+  o += 3;
+  for (int i = 0; i < s->lives; ++i) out[o + i] = 1;
+  o += 1;
+  for (int i = 0; i < 18 - s->ptr; ++i) out[o + i] = 1;
+  o += 14;
+  for (int c = 0; c < 3; ++c)
+    for (int r = 1; r <= 3; ++r)
+      for (int i = 0; i < s->disc[c * 3 + r - 1]; ++i) out[o + c * 6 + kMhDiscardBase[r - 1] + i] = 1;
+  o += 18;
+  if (s->la_valid) {  // last action, 27 bits
+    out[o + (s->la_actor == me ? 0 : 1)] = 1;
+    out[o + 2 + s->la_type] = 1;
+    if (s->la_colour >= 0) out[o + 6 + s->la_colour] = 1;
+    if (s->la_rank >= 1) out[o + 9 + s->la_rank - 1] = 1;
+    if (s->la_slot >= 0) out[o + 12 + s->la_slot] = 1;
+    if (s->la_card >= 0) out[o + 14 + s->la_card] = 1;
+    for (int k = 0; k < 2; ++k)
+      if ((s->la_hinted >> k) & 1) out[o + 23 + k] = 1;
+    if (s->la_success) out[o + 25] = 1;
+    if (s->la_bomb) out[o + 26] = 1;
+  }
+  o += 27;
+  for (int pass = 0; pass < 2; ++pass) {  // explicit hints: own, then partner
+    const int who = pass == 0 ? me : partner;
+    for (int k = 0; k < 2; ++k)
+      for (int b = 0; b < 3; ++b) {
+        if ((s->hint_col[who][k] >> b) & 1u) out[o + k * 6 + b] = 1;
+        if ((s->hint_rank[who][k] >> b) & 1u) out[o + k * 6 + 3 + b] = 1;
+      }
+    o += 12;
+  }
+  for (int k = 0; k < 2; ++k)
+    if (k < s->n_hand[me]) out[o + k] = 1;
+  o += 2;
+  if (s->fr >= 0) out[o] = 1;
+  o += 1;
+}
+
+// ======================================================================================
 // Generic env dispatch over orc_state blobs.
 // ======================================================================================
 namespace {
 static_assert(sizeof(orc_lbf_state) <= ORC_STATE_BYTES, "state blob too small");
 static_assert(sizeof(orc_oc_state) <= ORC_STATE_BYTES, "state blob too small");
 static_assert(sizeof(orc_hanabi_state) <= ORC_STATE_BYTES, "state blob too small");
+static_assert(sizeof(orc_mhanabi_state) <= ORC_STATE_BYTES, "state blob too small");
 
-bool turn_based(const orc_env_desc* d) { return d->kind == ORC_HANABI; }
+bool turn_based(const orc_env_desc* d) { return d->kind == ORC_HANABI || d->kind == ORC_MINI_HANABI; }
 
 void env_reset(const orc_env_desc* d, uint64_t seed, uint32_t env, uint32_t step, orc_state* st) {
   std::memset(st, 0, sizeof(*st));
   if (d->kind == ORC_LBF) orc_lbf_reset(d, seed, env, step, (orc_lbf_state*)st);
   if (d->kind == ORC_OVERCOOKED) orc_oc_reset(d, (orc_oc_state*)st);
   if (d->kind == ORC_HANABI) orc_hanabi_reset(seed, env, step, (orc_hanabi_state*)st);
+  if (d->kind == ORC_MINI_HANABI) orc_mhanabi_reset(seed, env, step, (orc_mhanabi_state*)st);
 }
 
 void env_obs(const orc_env_desc* d, const orc_state* st, int seat, uint8_t* out) {
   if (d->kind == ORC_LBF) orc_lbf_obs(d, (const orc_lbf_state*)st, seat, out);
   if (d->kind == ORC_OVERCOOKED) orc_oc_obs(d, (const orc_oc_state*)st, seat, out);
   if (d->kind == ORC_HANABI) orc_hanabi_obs((const orc_hanabi_state*)st, seat, out);
+  if (d->kind == ORC_MINI_HANABI) orc_mhanabi_obs((const orc_mhanabi_state*)st, seat, out);
 }
 
 // Returns done, or -1 for an illegal action.
 int env_step(const orc_env_desc* d, orc_state* st, int a0, int a1, float r[2], float* team) {
   if (d->kind == ORC_LBF) return orc_lbf_step(d, (orc_lbf_state*)st, a0, a1, r, team);
   if (d->kind == ORC_OVERCOOKED) return orc_oc_step(d, (orc_oc_state*)st, a0, a1, r, team);
+  if (d->kind == ORC_MINI_HANABI) {
+    orc_mhanabi_state* m = (orc_mhanabi_state*)st;
+    const int done = orc_mhanabi_step(m, (m->turn % 2 == 0) ? a0 : a1, team);
+    r[0] = r[1] = *team;
+    if (done == 0 && m->turn >= 100) return -2;
+    return done;
+  }
   orc_hanabi_state* h = (orc_hanabi_state*)st;
   int a = (h->turn % 2 == 0) ? a0 : a1;
   int done = orc_hanabi_step(h, a, team);
@@ -739,12 +976,17 @@ int env_step(const orc_env_desc* d, orc_state* st, int a0, int a1, float r[2], f
 
 int acting_seat(const orc_env_desc* d, const orc_state* st) {
   if (!turn_based(d)) return -1;
+  if (d->kind == ORC_MINI_HANABI) return ((const orc_mhanabi_state*)st)->turn % 2;
   return ((const orc_hanabi_state*)st)->turn % 2;
 }
 
 void env_legal(const orc_env_desc* d, const orc_state* st, uint8_t* legal) {
   if (d->kind == ORC_HANABI) {
     orc_hanabi_legal((const orc_hanabi_state*)st, legal);
+    return;
+  }
+  if (d->kind == ORC_MINI_HANABI) {
+    orc_mhanabi_legal((const orc_mhanabi_state*)st, legal);
     return;
   }
   for (int k = 0; k < orc_n_actions(d); ++k) legal[k] = 1;
@@ -1102,6 +1344,7 @@ extern "C" int32_t orc_xplay(const orc_env_desc* d, const orc_mlp* pols, int32_t
     if (d->kind == ORC_LBF) ret = ((orc_lbf_state*)&st)->ret;
     if (d->kind == ORC_OVERCOOKED) ret = ((orc_oc_state*)&st)->ret;
     if (d->kind == ORC_HANABI) ret = ((orc_hanabi_state*)&st)->ret;
+    if (d->kind == ORC_MINI_HANABI) ret = ((orc_mhanabi_state*)&st)->ret;
     returns[e] = ret;
     if (io->returns) io->returns[e] = ret;
     if (io->steps) io->steps[e] = steps;

@@ -50,7 +50,7 @@ uint32_t orc_uniform_int(uint32_t x, uint32_t n);
 double orc_u01(uint32_t x);
 
 /* ---- environment description ------------------------------------------------------ */
-enum { ORC_LBF = 0, ORC_OVERCOOKED = 1, ORC_HANABI = 2 };
+enum { ORC_LBF = 0, ORC_OVERCOOKED = 1, ORC_HANABI = 2, ORC_MINI_HANABI = 3 };
 typedef struct orc_env_desc {
   int32_t kind;            /* ORC_LBF / ORC_OVERCOOKED / ORC_HANABI */
   int32_t width, height;   /* LBF grid (3..12); Overcooked 5x4; Hanabi ignored */
@@ -143,6 +143,35 @@ void orc_hanabi_legal(const orc_hanabi_state* s, uint8_t legal[20]); /* for the 
  * if a is illegal. */
 int32_t orc_hanabi_step(orc_hanabi_state* s, int32_t a, float* team);
 void orc_hanabi_obs(const orc_hanabi_state* s, int32_t seat, uint8_t* out);
+
+/* ---- Mini Hanabi, 2 players (Sec. 4 Table "JaxAHT Environments": 3 colours x 3 ranks).
+ * The paper gives only the colour and rank counts; the rest is the reading in the design doc:
+ * 18-card deck (ranks 1,1,1,2,2,3 per colour), 2-card hands, 3 info and 1 life tokens,
+ * 10 actions (play slot 0-1, discard slot 0-1, hint colour 0-2, hint rank 1-3), card type
+ * = colour*3 + rank-1, and the full game's rules and observation sections at this size
+ * (153 bits).  A game lasts at most 40 turns; the library stops any game at 100. */
+typedef struct orc_mhanabi_state {
+  int32_t deck[18];
+  int32_t ptr;
+  int32_t hand[2][2];         /* card type, -1 if empty */
+  int32_t n_hand[2];
+  uint32_t know[2][2];        /* 9-bit possible-card masks */
+  uint32_t hint_col[2][2];    /* 3 bits */
+  uint32_t hint_rank[2][2];   /* 3 bits */
+  int32_t fw[3];
+  int32_t info, lives, score;
+  int32_t disc[9];
+  int32_t fr;
+  int32_t turn;
+  int32_t la_valid, la_actor, la_type, la_colour, la_rank, la_slot, la_card, la_hinted,
+          la_success, la_bomb;
+  int32_t done;
+  float ret;
+} orc_mhanabi_state;
+void orc_mhanabi_reset(uint64_t seed, uint32_t env, uint32_t step, orc_mhanabi_state* s);
+void orc_mhanabi_legal(const orc_mhanabi_state* s, uint8_t legal[10]);
+int32_t orc_mhanabi_step(orc_mhanabi_state* s, int32_t a, float* team);
+void orc_mhanabi_obs(const orc_mhanabi_state* s, int32_t seat, uint8_t* out);
 
 /* ---- generic env state ------------------------------------------------------------ */
 enum { ORC_STATE_BYTES = 768 };   /* >= sizeof of every state struct above */
