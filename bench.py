@@ -239,6 +239,7 @@ def run_ours(args):
     if os.path.exists(pk):
         peaks = json.load(open(pk))
     bf16_peak = peaks.get("bf16_tflops", 1900.0)
+    bf16_sustained = peaks.get("bf16_tflops_sustained", 1700.0)
     hbm_peak = peaks.get("hbm_gbs", 6800.0)
     peak_src = "measured" if peaks else "fallback"
 
@@ -353,6 +354,7 @@ def run_ours(args):
                          "traffic": traffic, "kernel": "ppo_tc_kernel<EnvLbf>",
                          "kernel_ms": kern_ms, "flops_per_launch": flops_launch,
                          "peak_source": f"{peak_src} bf16 burst",
+                         "frac_of_sustained": achieved_tflops / bf16_sustained,
                          "hbm": {"achieved_gbs": achieved_gbs, "peak_gbs": hbm_peak,
                                  "frac": achieved_gbs / hbm_peak,
                                  "bytes_per_launch": env_steps * bytes_per_env_step}},
@@ -362,12 +364,14 @@ def run_ours(args):
             "gpu_launches": 3 * args.steps,
             "clocks": clocks.summary(),
         }
+    if line is not None and not args.n_envs and not args.T:
+        line["c0"] = run_c0(aht, W, torch, stream)
     if not args.no_ppo:
         pu = run_ppo_update(args, aht, wl, pop_np, traj, torch, bf16_peak, stream)
         if line is not None:
             line["ppo_update"] = pu
     if not args.no_xplay:
-        xp = run_xplay(args, aht, W, torch, bf16_peak)
+        xp = run_xplay(args, aht, W, torch, bf16_peak, bf16_sustained=bf16_sustained)
         if line is not None:
             line["xplay"] = xp
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -379,6 +383,32 @@ def run_ours(args):
     ctx.close()
     if world > 1:
         dist.destroy_process_group()
+
+
+def run_c0(aht, W, torch, stream):
+    """The smallest configuration (64 LBF 7x7 envs x 50 steps, fp32 64-wide MLPs): too
+    small to fill the GPU, so only its latency and env-steps/s are reported."""
+    import numpy as np
+    wl = W.WORKLOADS["lbf7x7_64x50_fp32"]
+    pop = [[(torch.from_numpy(Wt).cuda(), torch.from_numpy(b).cuda()) for Wt, b in p]
+           for p in W.population(wl)]
+    ctx = aht.aht_create(wl.env, pop, wl.n_envs, wl.env_seed, weight_dtype=aht.AHT_FP32, stream=stream)
+    traj = aht.traj_buffers(ctx, wl.T)
+    for _ in range(3):
+        aht.aht_rollout(ctx, wl.ego_id, wl.pool, wl.T, traj)
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    K = 10
+    ev[0].record(stream)
+    for _ in range(K):
+        aht.aht_rollout(ctx, wl.ego_id, wl.pool, wl.T, traj)
+    ev[1].record(stream)
+    torch.cuda.synchronize()
+    aht.aht_sync(ctx)
+    ms = ev[0].elapsed_time(ev[1]) / K
+    ctx.close()
+    return {"workload": wl.name, "ms_per_call": ms, "env_steps_per_s": wl.n_envs * wl.T / (ms * 1e-3),
+            "bound": "latency (64 envs fill one tile; no roofline target)"}
 
 
 PPO_FLOPS_PER_SAMPLE = 204032   # forward 84,736 + backward 119,296 (dW1, dW2, dh1, dW3, dh2)
@@ -436,10 +466,11 @@ def run_ppo_update(args, aht, wl, pop_np, traj, torch, bf16_peak, stream):
 
 
 XPLAY_WORKLOADS = ("lbf7x7_xplay_8x16x256", "lbf7x7_xplay_heuristics_8x11x256",
-                   "lbf12x12_xplay_8x16x128", "overcooked5x4_xplay_8x8x64", "hanabi_xplay_16x16x32")
+                   "lbf12x12_xplay_8x16x128", "overcooked5x4_xplay_8x8x64", "hanabi_xplay_16x16x32",
+                   "minihanabi_xplay_16x16x32")
 
 
-def run_xplay(args, aht, W, torch, bf16_peak, names=XPLAY_WORKLOADS):
+def run_xplay(args, aht, W, torch, bf16_peak, names=XPLAY_WORKLOADS, bf16_sustained=1717.4):
     """Cross-play matrices: cells/s and active env-steps/s of each cross-play workload, and
     the fraction of the tensor roofline (MLP FLOPs of the env-steps that actually ran, one
     forward per acting agent, at the bf16 peak)."""
@@ -495,7 +526,7 @@ def run_xplay(args, aht, W, torch, bf16_peak, names=XPLAY_WORKLOADS):
         aht.aht_sync(ctx)
         ctx.close()
         dims = [wl.env.obs_dim, *wl.hidden, wl.env.n_actions]
-        acting = 1 if wl.env.kind == W.HANABI else 2        # Hanabi: one actor per turn
+        acting = 1 if wl.env.kind in (W.HANABI, W.MINI_HANABI) else 2   # one actor per turn
         if min(wl.tm_ids) < 0:                              # rule-based teammates: no network
             acting = 1
         flops = active * acting * mlp_flops(dims)
@@ -505,6 +536,7 @@ def run_xplay(args, aht, W, torch, bf16_peak, names=XPLAY_WORKLOADS):
                      "weights": "bf16" if wl.weight_dtype == W.BF16 else "f32",
                      "roofline": {"bound": "tensor", "achieved": tflops, "peak": bf16_peak,
                                   "unit": "TFLOP/s", "frac": tflops / bf16_peak,
+                                  "frac_of_sustained": tflops / bf16_sustained,
                                   "flops_per_matrix": flops},
                      "xp_stats_us": stats_us}
     return res

@@ -59,7 +59,7 @@ typedef enum aht_status {
   AHT_EDEVICE = 5   /* the device status word recorded an error */
 } aht_status;
 
-enum { AHT_LBF = 0, AHT_OVERCOOKED = 1, AHT_HANABI = 2 };
+enum { AHT_LBF = 0, AHT_OVERCOOKED = 1, AHT_HANABI = 2, AHT_MINI_HANABI = 3 };
 enum { AHT_FP32 = 0, AHT_BF16 = 1 };
 
 /* Environment (Sec. 4, Table "JaxAHT Environments"; the Dec-POMDP of Sec. 3).
@@ -69,7 +69,11 @@ enum { AHT_FP32 = 0, AHT_BF16 = 1 };
  *        cook_time 0..255; soup_reward.  Obs = 520 u8, actions 6.
  *   Hanabi: 2 players, full deck; episode_len must be 0 (run to termination; a game
  *        lasts at most 97 turns, the library stops any game at 100).  Obs = 660 u8,
- *        actions 20 with illegal-action masking. */
+ *        actions 20 with illegal-action masking.
+ *   Mini Hanabi (Sec. 4 Table: 3 colours x 3 ranks): 2 players, ranks 1,1,1,2,2,3 per
+ *        colour (18 cards), 2-card hands, 3 info and 1 life tokens; episode_len must be
+ *        0.  Obs = 156 u8 (153 features + 3 zero), actions 10 (play slot 0-1, discard
+ *        slot 0-1, hint colour 0-2, hint rank 1-3) with illegal-action masking. */
 typedef struct aht_env_desc {
   int32_t kind;
   int32_t width, height;

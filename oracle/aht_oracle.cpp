@@ -74,7 +74,7 @@ extern "C" int32_t orc_obs_dim(const orc_env_desc* d) {
     case ORC_LBF: return d->width * d->height * 4;
     case ORC_OVERCOOKED: return 5 * 4 * 26;
     case ORC_HANABI: return 660;
-    case ORC_MINI_HANABI: return 153;
+    case ORC_MINI_HANABI: return 156;
   }
   return -1;
 }
@@ -871,9 +871,10 @@ extern "C" int32_t orc_mhanabi_step(orc_mhanabi_state* s, int32_t a, float* team
 }
 
 // 153 bits: partner hand 18, own knowledge 18, partner knowledge 18, fireworks 9, info 3,
-// lives 1, deck 14, discards 18, last action 27, explicit hints 12 + 12, slots 2, final 1.
+// lives 1, deck 14, discards 18, last action 27, explicit hints 12 + 12, slots 2, final 1;
+// then 3 zero features (156: observation rows stay 4-byte multiples).
 extern "C" void orc_mhanabi_obs(const orc_mhanabi_state* s, int32_t seat, uint8_t* out) {
-  std::memset(out, 0, 153);
+  std::memset(out, 0, 156);
   const int me = seat, partner = 1 - seat;
   int o = 0;
   for (int k = 0; k < 2; ++k)

@@ -149,7 +149,7 @@ void orc_hanabi_obs(const orc_hanabi_state* s, int32_t seat, uint8_t* out);
  * 18-card deck (ranks 1,1,1,2,2,3 per colour), 2-card hands, 3 info and 1 life tokens,
  * 10 actions (play slot 0-1, discard slot 0-1, hint colour 0-2, hint rank 1-3), card type
  * = colour*3 + rank-1, and the full game's rules and observation sections at this size
- * (153 bits).  A game lasts at most 40 turns; the library stops any game at 100. */
+ * (153 bits, then 3 zero features: 156).  The library stops any game at 100 turns. */
 typedef struct orc_mhanabi_state {
   int32_t deck[18];
   int32_t ptr;

@@ -16,7 +16,7 @@ import torch
 from . import build as _build
 
 AHT_OK, AHT_EINVAL, AHT_ENOMEM, AHT_ECUDA, AHT_ETIMEOUT, AHT_EDEVICE = range(6)
-AHT_LBF, AHT_OVERCOOKED, AHT_HANABI = range(3)
+AHT_LBF, AHT_OVERCOOKED, AHT_HANABI, AHT_MINI_HANABI = range(4)
 AHT_FP32, AHT_BF16 = 0, 1
 
 EXPORTED = ["aht_create", "aht_destroy", "aht_reset", "aht_rollout", "aht_xplay_matrix",

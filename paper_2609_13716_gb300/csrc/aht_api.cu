@@ -60,6 +60,9 @@ EnvOps ops_for(int kind) {
     case AHT_OVERCOOKED:
       return {overcooked_ppo, overcooked_xplay, overcooked_forced, overcooked_reset,
               overcooked_state_words, overcooked_state_bytes, overcooked_set_smem_limit, 64};
+    case AHT_MINI_HANABI:
+      return {minihanabi_ppo, minihanabi_xplay, minihanabi_forced, minihanabi_reset,
+              minihanabi_state_words, minihanabi_state_bytes, minihanabi_set_smem_limit, 64};
     default:
       return {hanabi_ppo, hanabi_xplay, hanabi_forced, hanabi_reset, hanabi_state_words,
               hanabi_state_bytes, hanabi_set_smem_limit, 32};
@@ -168,6 +171,10 @@ aht_status check_env(const aht_env_desc* d, DevEnv* out) {
     if (d->episode_len != 0) return fail(AHT_EINVAL, "Hanabi episode_len must be 0 (to termination)");
     e.obs_dim = 660;
     e.n_actions = 20;
+  } else if (d->kind == AHT_MINI_HANABI) {
+    if (d->episode_len != 0) return fail(AHT_EINVAL, "Mini Hanabi episode_len must be 0 (to termination)");
+    e.obs_dim = 156;
+    e.n_actions = 10;
   } else {
     return fail(AHT_EINVAL, "unknown env kind");
   }
@@ -303,7 +310,7 @@ WideDims make_wide_dims(const MlpDims& m) {
 // their cross-play steps on the streamed tensor-core kernel.
 bool wide_eligible(const aht_ctx* c, int dtype) {
   const MlpDims& m = c->mlp;
-  if (dtype != AHT_BF16 || (c->env.kind != AHT_OVERCOOKED && c->env.kind != AHT_HANABI)) return false;
+  if (dtype != AHT_BF16 || c->env.kind == AHT_LBF) return false;
   if (m.H0 != m.H1 || (m.H0 != 256 && m.H0 != 512)) return false;
   return xp_tc_smem_bytes(make_wide_dims(m)) <= c->smem_optin;
 }
@@ -467,8 +474,10 @@ aht_status xplay_wide(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego, const i
   const int64_t T0 = ((int64_t)n_tm * P + 127) / 128, T1 = ((int64_t)n_ego * P + 127) / 128;
   const int64_t tiles0 = n_ego * T0, tiles1 = n_tm * T1;
   if (tiles0 + tiles1 > INT32_MAX) return fail(AHT_EINVAL, "too many tiles");
-  const bool turn = c->env.kind == AHT_HANABI;
-  auto launch = c->env.kind == AHT_HANABI ? hanabi_xplay_tc : overcooked_xplay_tc;
+  const bool turn = c->env.kind == AHT_HANABI || c->env.kind == AHT_MINI_HANABI;
+  auto launch = c->env.kind == AHT_HANABI        ? hanabi_xplay_tc
+                : c->env.kind == AHT_MINI_HANABI ? minihanabi_xplay_tc
+                                                 : overcooked_xplay_tc;
   const int tk = timer_begin(c);
   for (int s = 0; s <= max_steps; ++s) {
     a.s = s;
@@ -702,7 +711,8 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
       }
     if (cudaMemcpy(c->wtcw, blocks.data(), blocks.size(), cudaMemcpyHostToDevice) != cudaSuccess)
       return bail(AHT_ECUDA, "uploading the streamed tensor-core population failed");
-    const cudaError_t se = env.kind == AHT_HANABI ? hanabi_xplay_tc_smem_limit(c->wide_smem)
+    const cudaError_t se = env.kind == AHT_MINI_HANABI ? minihanabi_xplay_tc_smem_limit(c->wide_smem)
+                           : env.kind == AHT_HANABI    ? hanabi_xplay_tc_smem_limit(c->wide_smem)
                                                   : overcooked_xplay_tc_smem_limit(c->wide_smem);
     if (se != cudaSuccess) return bail(AHT_ECUDA, "setting the shared-memory limit failed");
     if (cudaMallocHost((void**)&c->wide_staging, c->wd.pol_bytes) != cudaSuccess)
@@ -738,7 +748,8 @@ aht_status aht_reset(aht_ctx* c, uint64_t seed) {
 aht_status aht_rollout(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t pool_size,
                        int32_t T, const aht_traj* out) {
   if (!c || !out) return fail(AHT_EINVAL, "ctx or out is NULL");
-  if (c->env.kind == AHT_HANABI) return fail(AHT_EINVAL, "PPO collection needs a simultaneous-move env (LBF, Overcooked)");
+  if (c->env.kind == AHT_HANABI || c->env.kind == AHT_MINI_HANABI)
+    return fail(AHT_EINVAL, "PPO collection needs a simultaneous-move env (LBF, Overcooked)");
   if (ego_id < 0 || ego_id >= c->n_policies) return fail(AHT_EINVAL, "ego_id out of range");
   if (!pool || pool_size < 1 || pool_size > kMaxPool) return fail(AHT_EINVAL, "pool_size must be in 1..256");
   for (int k = 0; k < pool_size; ++k) {

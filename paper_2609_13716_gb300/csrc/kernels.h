@@ -188,6 +188,7 @@ struct PolicyArgs {
 AHT_DECLARE_ENV_LAUNCHERS(lbf)
 AHT_DECLARE_ENV_LAUNCHERS(overcooked)
 AHT_DECLARE_ENV_LAUNCHERS(hanabi)
+AHT_DECLARE_ENV_LAUNCHERS(minihanabi)
 
 // Tensor-core rollout (rollout_lbf.cu): LBF grids whose padded observation fits 256 bf16
 // columns of tensor memory; PPO collection (grid = tile table entries) and cross-play
@@ -201,6 +202,8 @@ cudaError_t overcooked_xplay_tc(const XpTcArgs&, int grid, size_t smem, cudaStre
 cudaError_t hanabi_xplay_tc(const XpTcArgs&, int grid, size_t smem, cudaStream_t);
 cudaError_t overcooked_xplay_tc_smem_limit(size_t smem);  // once per device, before launches
 cudaError_t hanabi_xplay_tc_smem_limit(size_t smem);
+cudaError_t minihanabi_xplay_tc(const XpTcArgs&, int grid, size_t smem, cudaStream_t);
+cudaError_t minihanabi_xplay_tc_smem_limit(size_t smem);
 size_t xp_tc_smem_bytes(const WideDims& w);
 
 // misc.cu

@@ -14,7 +14,7 @@ from dataclasses import dataclass, field
 
 import numpy as np
 
-LBF, OVERCOOKED, HANABI = 0, 1, 2
+LBF, OVERCOOKED, HANABI, MINI_HANABI = 0, 1, 2, 3
 FP32, BF16 = 0, 1
 
 
@@ -35,11 +35,13 @@ class EnvSpec:
             return self.width * self.height * 4
         if self.kind == OVERCOOKED:
             return 5 * 4 * 26
+        if self.kind == MINI_HANABI:
+            return 156
         return 660
 
     @property
     def n_actions(self) -> int:
-        return 20 if self.kind == HANABI else 6
+        return {HANABI: 20, MINI_HANABI: 10}.get(self.kind, 6)
 
     def astuple(self):
         return (self.kind, self.width, self.height, self.n_food, self.max_agent_level,
@@ -136,6 +138,13 @@ WORKLOADS = {
         name="hanabi_xplay_16x16x32", index=4, env=EnvSpec(kind=HANABI, episode_len=0),
         hidden=(512, 512), weight_dtype=BF16, n_policies=32, value_head=(0,) * 32,
         mode="xplay", env_seed=4, ego_ids=tuple(range(16)), tm_ids=tuple(range(16, 32)),
+        envs_per_pair=32, max_steps=100),
+    # 2-player Mini Hanabi (3 colours x 3 ranks): 16 x 16 pairs, 32 envs per pair, to
+    # termination, 156-256-256-10 bf16 MLPs with illegal-action masking.
+    "minihanabi_xplay_16x16x32": Workload(
+        name="minihanabi_xplay_16x16x32", index=8, env=EnvSpec(kind=MINI_HANABI, episode_len=0),
+        hidden=(256, 256), weight_dtype=BF16, n_policies=32, value_head=(0,) * 32,
+        mode="xplay", env_seed=8, ego_ids=tuple(range(16)), tm_ids=tuple(range(16, 32)),
         envs_per_pair=32, max_steps=100),
 }
 

@@ -28,7 +28,7 @@ def step(orc, s, a):
 
 
 def obs(orc, s, seat):
-    out = np.zeros(153, np.uint8)
+    out = np.zeros(156, np.uint8)
     orc.lib().orc_mhanabi_obs(C.byref(s), seat, out.ctypes.data_as(C.c_void_p))
     return out
 
@@ -156,3 +156,4 @@ def test_observation_sections_by_hand(orc):
     assert not o[54:63].any()
     assert o[63:66].all() and o[66] == 1 and o[67:81].all() and not o[81:99].any()
     assert not o[99:150].any() and o[150:152].all() and o[152] == 0
+    assert not o[153:].any()   # the 3 padding features
