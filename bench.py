@@ -465,7 +465,7 @@ def run_ppo_update(args, aht, wl, pop_np, traj, torch, bf16_peak, stream):
     return res
 
 
-XPLAY_WORKLOADS = ("lbf7x7_xplay_8x16x256", "lbf7x7_xplay_heuristics_8x11x256",
+XPLAY_WORKLOADS = ("lbf7x7_xplay_8x16x256", "lbf7x7_xplay_heuristics_8x12x256",
                    "lbf12x12_xplay_8x16x128", "overcooked5x4_xplay_8x8x64", "hanabi_xplay_16x16x32",
                    "minihanabi_xplay_16x16x32")
 

@@ -113,12 +113,17 @@ typedef struct aht_pop_desc {
  *           (y*width + x) ascending | descending, column-major index (x*height + y)
  *           ascending | descending, distance from its own position at the episode's start
  *           ascending | descending (ties: lower food index);
- * then: load when 4-adjacent to it; else one step along the axis with the larger
- * remaining distance (ties: x), or along the other axis when that cell is off the grid,
- * an uneaten food or the ego; else noop (distances Manhattan).  The rule draws nothing;
- * the teammate's recorded action is the rule's.  The paper names the criteria and
- * orderings only: the rules above are this library's reading. */
-#define AHT_LBF_N_HEURISTICS 11
+ *           then: load when 4-adjacent to it;
+ *   k 11    Entitled: the pair of squares of the lowest-index uneaten food is its first
+ *           two neighbours in the order W, E, N, S that lie on the grid and hold no
+ *           uneaten food (fewer than two: noop); noop until the ego stands on one of them,
+ *           then it goes for the other and loads when standing on it;
+ * a move is one step along the axis with the larger remaining distance (ties: x), or
+ * along the other axis when that cell is off the grid, an uneaten food or the ego; else
+ * noop (distances Manhattan).  The rule draws nothing; the teammate's recorded action is
+ * the rule's.  The paper names the criteria and orderings only: the rules above are this
+ * library's reading. */
+#define AHT_LBF_N_HEURISTICS 12
 #define AHT_LBF_HEURISTIC(k) (-1 - (k))
 
 /* Creates a context for up to n_envs concurrent envs (PPO state and cross-play batch

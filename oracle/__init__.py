@@ -33,7 +33,7 @@ STATE_BYTES = 768
 LBF_HEURISTICS = ("greedy_closest_self", "greedy_closest_teammate", "greedy_closest_avg",
                   "greedy_lowest_level", "greedy_highest_level", "seq_lexicographic",
                   "seq_reverse_lexicographic", "seq_column_major", "seq_reverse_column_major",
-                  "seq_nearest_agent", "seq_farthest_agent")
+                  "seq_nearest_agent", "seq_farthest_agent", "entitled")
 
 
 def heuristic_id(name):

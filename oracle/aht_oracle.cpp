@@ -234,6 +234,47 @@ extern "C" int32_t orc_lbf_heuristic(const orc_env_desc* d, const orc_lbf_state*
                                      int32_t k) {
   const int me = seat, other = 1 - seat;
   auto dist = [&](int x, int y, int f) { return std::abs(x - s->fx[f]) + std::abs(y - s->fy[f]); };
+  auto free_cell = [&](int cx, int cy) {
+    if (cx < 0 || cx >= d->width || cy < 0 || cy >= d->height) return false;
+    for (int f = 0; f < d->n_food; ++f)
+      if (!s->eaten[f] && s->fx[f] == cx && s->fy[f] == cy) return false;
+    return !(s->ax[other] == cx && s->ay[other] == cy);
+  };
+  // one step from (x, y) toward (tx, ty): the axis with the larger distance first (ties:
+  // x), the other axis if that cell is not free; noop if neither is
+  auto step_toward = [&](int x, int y, int tx, int ty) {
+    const int dx = tx - x, dy = ty - y;
+    const int x_act = dx > 0 ? 4 : 3, y_act = dy > 0 ? 2 : 1;
+    const int sx = dx > 0 ? 1 : -1, sy = dy > 0 ? 1 : -1;
+    const bool x_first = std::abs(dx) >= std::abs(dy);
+    for (int c = 0; c < 2; ++c) {
+      const bool along_x = (c == 0) == x_first;
+      if (along_x && dx != 0 && free_cell(x + sx, y)) return x_act;
+      if (!along_x && dy != 0 && free_cell(x, y + sy)) return y_act;
+    }
+    return 0;
+  };
+  if (k == 11) {  // Entitled
+    int f = 0;
+    while (f < d->n_food && s->eaten[f]) ++f;
+    if (f >= d->n_food) return 0;
+    const int nx[4] = {s->fx[f] - 1, s->fx[f] + 1, s->fx[f], s->fx[f]};
+    const int ny[4] = {s->fy[f], s->fy[f], s->fy[f] - 1, s->fy[f] + 1};
+    int pair[2], n = 0;
+    for (int q = 0; q < 4 && n < 2; ++q) {
+      bool ok = nx[q] >= 0 && nx[q] < d->width && ny[q] >= 0 && ny[q] < d->height;
+      for (int g = 0; ok && g < d->n_food; ++g)
+        if (!s->eaten[g] && s->fx[g] == nx[q] && s->fy[g] == ny[q]) ok = false;
+      if (ok) pair[n++] = q;
+    }
+    if (n < 2) return 0;
+    int mine = -1;
+    for (int q = 0; q < 2; ++q)
+      if (s->ax[other] == nx[pair[q]] && s->ay[other] == ny[pair[q]]) mine = pair[1 - q];
+    if (mine < 0) return 0;  // wait for the other agent to take one square
+    if (s->ax[me] == nx[mine] && s->ay[me] == ny[mine]) return kLbfLoad;
+    return step_toward(s->ax[me], s->ay[me], nx[mine], ny[mine]);
+  }
   // the food to go for
   int target = -1;
   long best = 0;
@@ -261,23 +302,8 @@ extern "C" int32_t orc_lbf_heuristic(const orc_env_desc* d, const orc_lbf_state*
   }
   if (target < 0) return 0;
   const int x = s->ax[me], y = s->ay[me];
-  const int dx = s->fx[target] - x, dy = s->fy[target] - y;
-  if (std::abs(dx) + std::abs(dy) == 1) return kLbfLoad;
-  auto free_cell = [&](int cx, int cy) {
-    if (cx < 0 || cx >= d->width || cy < 0 || cy >= d->height) return false;
-    for (int f = 0; f < d->n_food; ++f)
-      if (!s->eaten[f] && s->fx[f] == cx && s->fy[f] == cy) return false;
-    return !(s->ax[other] == cx && s->ay[other] == cy);
-  };
-  const int x_act = dx > 0 ? 4 : 3, y_act = dy > 0 ? 2 : 1;  // E / W, S / N
-  const int sx = dx > 0 ? 1 : -1, sy = dy > 0 ? 1 : -1;
-  const bool x_first = std::abs(dx) >= std::abs(dy);
-  for (int c = 0; c < 2; ++c) {
-    const bool along_x = (c == 0) == x_first;
-    if (along_x && dx != 0 && free_cell(x + sx, y)) return x_act;
-    if (!along_x && dy != 0 && free_cell(x, y + sy)) return y_act;
-  }
-  return 0;
+  if (dist(x, y, target) == 1) return kLbfLoad;
+  return step_toward(x, y, s->fx[target], s->fy[target]);
 }
 
 extern "C" void orc_lbf_obs(const orc_env_desc* d, const orc_lbf_state* s, int32_t seat,

@@ -95,9 +95,14 @@ void orc_lbf_obs(const orc_env_desc* d, const orc_lbf_state* s, int32_t seat, ui
  *             ascending | descending (ties: lower food index);
  * then the action toward it: load (5) when 4-adjacent; else a step along the axis with
  * the larger remaining distance (ties: x), or along the other axis if that cell is off
- * the grid, an uneaten food or the other agent; else noop.  dist is Manhattan.  A
- * teammate id t < 0 in a pool or teammate list means heuristic k = -1 - t (LBF only). */
-enum { ORC_LBF_N_HEURISTICS = 11 };
+ * the grid, an uneaten food or the other agent; else noop.  dist is Manhattan.
+ *   k = 11    Entitled: for the lowest-index uneaten food, the pair of squares is its
+ *             first two 4-neighbours in the order W, E, N, S that are on the grid and
+ *             hold no uneaten food (fewer than two: noop); while the other
+ *             agent stands on neither, noop; once it stands on one, go to the other (the
+ *             step rule above, toward that cell) and load when standing on it.
+ * A teammate id t < 0 in a pool or teammate list means heuristic k = -1 - t (LBF only). */
+enum { ORC_LBF_N_HEURISTICS = 12 };
 int32_t orc_lbf_heuristic(const orc_env_desc* d, const orc_lbf_state* s, int32_t seat, int32_t k);
 
 /* ---- Overcooked-style kitchen (fixed 5x4 layout) -------------------------------- */

@@ -163,11 +163,58 @@ struct EnvLbf {
   }
 
   // Rule-based teammate k in seat 1 (the LBF heuristic suite: Greedy criteria 0..4,
-  // Sequential orderings 5..10): the food to go for, then load when 4-adjacent, else a
-  // step along the axis with the larger remaining distance (ties: x), else along the
-  // other axis, when the cell is on the grid and free of uneaten food and of agent 0.
+  // Sequential orderings 5..10, Entitled 11): the cell to go for, then load when there,
+  // else a step along the axis with the larger remaining distance (ties: x), else along
+  // the other axis, when the cell is on the grid and free of uneaten food and of agent 0.
+  // Greedy and Sequential go for a food and load when 4-adjacent to it; Entitled takes
+  // the lowest-index uneaten food's pair of squares (its first two neighbours W, E, N, S
+  // on the grid and free of uneaten food) and waits until agent 0 stands on one of them,
+  // then goes for the other and loads there.
   __device__ __noinline__ static int heuristic(const DevEnv& d, const State& s, int k) {
     const int x = s.ax[1], y = s.ay[1], ox = s.ax[0], oy = s.ay[0];
+    auto food_at = [&](int cx, int cy) {
+#pragma unroll
+      for (int f = 0; f < 3; ++f)
+        if (!((s.eaten >> f) & 1u) && s.fx[f] == cx && s.fy[f] == cy) return true;
+      return false;
+    };
+    auto free_cell = [&](int cx, int cy) {
+      if (cx < 0 || cx >= d.width || cy < 0 || cy >= d.height) return false;
+      return !food_at(cx, cy) && !(ox == cx && oy == cy);
+    };
+    auto step_to = [&](int tx, int ty) {
+      const int dx = tx - x, dy = ty - y;
+      const int sx = dx > 0 ? 1 : -1, sy = dy > 0 ? 1 : -1;
+      const bool xmove = dx != 0 && free_cell(x + sx, y);
+      const bool ymove = dy != 0 && free_cell(x, y + sy);
+      const int x_act = dx > 0 ? 4 : 3, y_act = dy > 0 ? 2 : 1;
+      if (abs(dx) >= abs(dy)) return xmove ? x_act : (ymove ? y_act : 0);
+      return ymove ? y_act : (xmove ? x_act : 0);
+    };
+    if (k == 11) {
+      int f = 0;
+      while (f < 3 && ((s.eaten >> f) & 1u)) ++f;
+      if (f == 3) return 0;
+      const int cx = s.fx[f], cy = s.fy[f];
+      int px[2], py[2], n = 0;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int nx = cx + (q == 0 ? -1 : q == 1 ? 1 : 0);
+        const int ny = cy + (q == 2 ? -1 : q == 3 ? 1 : 0);
+        if (n < 2 && nx >= 0 && nx < d.width && ny >= 0 && ny < d.height && !food_at(nx, ny)) {
+          px[n] = nx;
+          py[n] = ny;
+          ++n;
+        }
+      }
+      if (n < 2) return 0;
+      int q;
+      if (ox == px[0] && oy == py[0]) q = 1;
+      else if (ox == px[1] && oy == py[1]) q = 0;
+      else return 0;
+      if (x == px[q] && y == py[q]) return 5;
+      return step_to(px[q], py[q]);
+    }
     int target = -1, best = 0;
 #pragma unroll
     for (int f = 0; f < 3; ++f) {
@@ -196,21 +243,8 @@ struct EnvLbf {
       }
     }
     if (target < 0) return 0;
-    const int dx = (int)s.fx[target] - x, dy = (int)s.fy[target] - y;
-    if (abs(dx) + abs(dy) == 1) return 5;
-    auto free_cell = [&](int cx, int cy) {
-      if (cx < 0 || cx >= d.width || cy < 0 || cy >= d.height) return false;
-#pragma unroll
-      for (int f = 0; f < 3; ++f)
-        if (!((s.eaten >> f) & 1u) && s.fx[f] == cx && s.fy[f] == cy) return false;
-      return !(ox == cx && oy == cy);
-    };
-    const int sx = dx > 0 ? 1 : -1, sy = dy > 0 ? 1 : -1;
-    const bool xmove = dx != 0 && free_cell(x + sx, y);
-    const bool ymove = dy != 0 && free_cell(x, y + sy);
-    const int x_act = dx > 0 ? 4 : 3, y_act = dy > 0 ? 2 : 1;
-    if (abs(dx) >= abs(dy)) return xmove ? x_act : (ymove ? y_act : 0);
-    return ymove ? y_act : (xmove ? x_act : 0);
+    if (abs((int)s.fx[target] - x) + abs((int)s.fy[target] - y) == 1) return 5;
+    return step_to(s.fx[target], s.fy[target]);
   }
 
   __device__ static uint32_t legal(const State&) { return 0x3Fu; }

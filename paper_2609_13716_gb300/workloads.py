@@ -97,11 +97,11 @@ WORKLOADS = {
         weight_dtype=FP32, n_policies=24, value_head=(0,) * 24, mode="xplay", env_seed=1,
         ego_ids=tuple(range(8)), tm_ids=tuple(range(8, 24)), envs_per_pair=256,
         max_steps=128),
-    # The same 8 egos (same seeds) against the 11 rule-based LBF teammates (ids -1..-11).
-    "lbf7x7_xplay_heuristics_8x11x256": Workload(
-        name="lbf7x7_xplay_heuristics_8x11x256", index=1, env=_lbf(128), hidden=(64, 64),
+    # The same 8 egos (same seeds) against the 12 rule-based LBF teammates (ids -1..-12).
+    "lbf7x7_xplay_heuristics_8x12x256": Workload(
+        name="lbf7x7_xplay_heuristics_8x12x256", index=1, env=_lbf(128), hidden=(64, 64),
         weight_dtype=FP32, n_policies=8, value_head=(0,) * 8, mode="xplay", env_seed=1,
-        ego_ids=tuple(range(8)), tm_ids=tuple(-1 - k for k in range(11)), envs_per_pair=256,
+        ego_ids=tuple(range(8)), tm_ids=tuple(-1 - k for k in range(12)), envs_per_pair=256,
         max_steps=128),
     # LBF 12x12 (the paper's second LBF grid, Sec. 4 Table "JaxAHT Environments"): 8 egos
     # x 16 teammates, 128 envs per pair, 128-step episodes, fp32 576-64-64-6 MLPs.

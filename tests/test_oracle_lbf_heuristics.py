@@ -3,7 +3,9 @@
 The paper's LBF heuristic suite (App. F): Greedy picks the next uneaten food online by
 closest_self / closest_teammate / closest_avg / lowest_level / highest_level; Sequential
 plans a food order before the episode by lexicographic / reverse_lexicographic /
-column_major / reverse_column_major / nearest_agent / farthest_agent.  The movement and
+column_major / reverse_column_major / nearest_agent / farthest_agent; Entitled picks a pair
+of squares beside a food and waits for the teammate to stand on one before taking the
+other and loading.  The movement and
 tie rules are the readings stated in aht_oracle.h.  Every expected action below is worked
 out by hand from those statements on a 5 x 5 grid (x right, y down; 1 N, 2 S, 3 W, 4 E,
 5 load, 0 noop).
@@ -119,6 +121,8 @@ def test_moves_close_in_on_the_target_random_states():
         foods = [(x, y, int(rng.integers(1, 5))) for x, y in pos[:3]]
         s = state(pos[3], pos[4], foods, init1=pos[4])
         for name, k in H.items():
+            if name == "entitled":
+                continue
             a = O.lbf_heuristic(d, s, 1, k)
             assert 0 <= a <= 5
             # the target by brute force over the three foods
@@ -157,4 +161,71 @@ def test_rollout_and_xplay_accept_heuristic_teammates():
     # the teammate seat's actions are its rule's, and no draw is flagged for it
     assert (out["margin"][..., 1] == 2.0).all()
     xp = O.xplay(d, pols, 4, 0, [0], [O.heuristic_id(n) for n in O.LBF_HEURISTICS], 8, 50)
-    assert xp["rc"] == 0 and xp["matrix"].shape == (1, 11)
+    assert xp["rc"] == 0 and xp["matrix"].shape == (1, 12)
+
+
+# Entitled, food 0 at (2, 2) level 2 on a 5 x 5 grid: its pair is W (1, 2) and E (3, 2)
+E_FOODS = [(2, 2, 2), (4, 4, 1)]
+
+
+def test_entitled_waits_until_the_teammate_takes_a_square():
+    # agent 0 on neither square: wait, wherever the heuristic (agent 1) stands
+    for a1 in [(0, 0), (3, 2), (1, 2), (4, 0)]:
+        s = state(a0=(0, 4), a1=a1, foods=E_FOODS)
+        assert O.lbf_heuristic(desc(n_food=2), s, 1, H["entitled"]) == NOOP, a1
+    # agent 0 on W (1, 2): go to E (3, 2) -- from (4, 0): dx = -1, dy = 2 -> south
+    s = state(a0=(1, 2), a1=(4, 0), foods=E_FOODS)
+    assert O.lbf_heuristic(desc(n_food=2), s, 1, H["entitled"]) == S_
+    # ... and load once standing on it
+    s = state(a0=(1, 2), a1=(3, 2), foods=E_FOODS)
+    assert O.lbf_heuristic(desc(n_food=2), s, 1, H["entitled"]) == LOAD
+    # agent 0 on E: the target is W (1, 2); from (1, 0): dx = 0, dy = 2 -> south
+    s = state(a0=(3, 2), a1=(1, 0), foods=E_FOODS)
+    assert O.lbf_heuristic(desc(n_food=2), s, 1, H["entitled"]) == S_
+
+
+def test_entitled_pairs_at_edges_and_next_to_foods():
+    # food 0 at (0, 0): W and N off the grid -> pair E (1, 0), S (0, 1)
+    foods = [(0, 0, 1), (4, 4, 1)]
+    s = state(a0=(0, 1), a1=(3, 0), foods=foods)
+    assert O.lbf_heuristic(desc(n_food=2), s, 1, H["entitled"]) == W_   # to (1, 0)
+    s = state(a0=(1, 0), a1=(0, 3), foods=foods)
+    assert O.lbf_heuristic(desc(n_food=2), s, 1, H["entitled"]) == N_   # to (0, 1)
+    # food 1 on (1, 2), W of food 0 at (2, 2): the pair becomes E (3, 2), N (2, 1)
+    foods = [(2, 2, 1), (1, 2, 1)]
+    s = state(a0=(2, 1), a1=(3, 4), foods=foods)
+    assert O.lbf_heuristic(desc(n_food=2), s, 1, H["entitled"]) == N_   # to (3, 2)
+    s = state(a0=(1, 3), a1=(3, 4), foods=foods)                        # (1, 3): no square
+    assert O.lbf_heuristic(desc(n_food=2), s, 1, H["entitled"]) == NOOP
+    # food 0 eaten: the pair belongs to food 1 at (4, 4): W (3, 4), N (4, 3)
+    s = state(a0=(4, 3), a1=(0, 4), foods=[(2, 2, 1), (4, 4, 1)], eaten=(1, 0, 0))
+    assert O.lbf_heuristic(desc(n_food=2), s, 1, H["entitled"]) == E_
+    # all eaten: noop
+    s = state(a0=(4, 3), a1=(0, 4), foods=[(2, 2, 1), (4, 4, 1)], eaten=(1, 1, 1))
+    assert O.lbf_heuristic(desc(n_food=2), s, 1, H["entitled"]) == NOOP
+    # a food in a 1-wide corridor with a single free neighbour has no pair: noop
+    d = O.env_desc(O.LBF, 3, 1, 1, 3, 50)
+    s = state(a0=(1, 0), a1=(2, 0), foods=[(0, 0, 1)])
+    assert O.lbf_heuristic(d, s, 1, H["entitled"]) == NOOP
+
+
+def test_entitled_pair_load_together():
+    """Two Entitled agents off the pair both wait; with the other agent on W, an Entitled
+    agent walks to E by the step rule and loads there."""
+    d = desc(n_food=2)
+    s = state(a0=(0, 4), a1=(4, 4), foods=[(2, 2, 2), (0, 0, 1)])
+    assert [O.lbf_heuristic(d, s, seat, H["entitled"]) for seat in (0, 1)] == [NOOP, NOOP]
+    s = state(a0=(1, 2), a1=(4, 4), foods=[(2, 2, 2), (0, 0, 1)], levels=(1, 1))
+    seen = []
+    for t in range(10):
+        a = O.lbf_heuristic(d, s, 1, H["entitled"])
+        seen.append(a)
+        if a == LOAD:
+            break
+        dx = (a == E_) - (a == W_)
+        dy = (a == S_) - (a == N_)
+        s.ax[1] += dx
+        s.ay[1] += dy
+    assert seen[-1] == LOAD and (s.ax[1], s.ay[1]) == (3, 2)
+    # (4,4) -N-> (4,3) -W-> (3,3) (tie: x first) -N-> (3,2), then load
+    assert seen == [N_, W_, N_, LOAD]
