@@ -366,6 +366,7 @@ def run_ours(args):
         }
     if line is not None and not args.n_envs and not args.T:
         line["c0"] = run_c0(aht, W, torch, stream)
+        line["ippo"] = run_ippo(aht, W, torch, stream, bf16_peak)
     if not args.no_ppo:
         pu = run_ppo_update(args, aht, wl, pop_np, traj, torch, bf16_peak, stream)
         if line is not None:
@@ -409,6 +410,50 @@ def run_c0(aht, W, torch, stream):
     ctx.close()
     return {"workload": wl.name, "ms_per_call": ms, "env_steps_per_s": wl.n_envs * wl.T / (ms * 1e-3),
             "bound": "latency (64 envs fill one tile; no roofline target)"}
+
+
+def run_ippo(aht, W, torch, stream, bf16_peak):
+    """IPPO collection (both seats learn): 16384 LBF 7x7 envs x 128 steps, two bf16
+    196-128-128-(6+1) policies, both seats' trajectories and GAE.  ms per call from CUDA
+    events (L2 scrubbed between calls, outside the events) and the tensor roofline of the
+    fused rollout kernel's algorithmic FLOPs (both forwards per env-step, both V_T)."""
+    wl = W.WORKLOADS["lbf7x7_ippo_16384x128"]
+    pop = [[(torch.from_numpy(Wt).to("cuda", torch.bfloat16), torch.from_numpy(b).to("cuda", torch.bfloat16))
+            for Wt, b in p] for p in W.population(wl)]
+    ctx = aht.aht_create(wl.env, pop, wl.n_envs, wl.env_seed, has_value_head=list(wl.value_head),
+                         weight_dtype=aht.AHT_BF16, stream=stream)
+    t0, t1 = aht.traj_buffers(ctx, wl.T), aht.traj_buffers(ctx, wl.T)
+    scrub = torch.empty(256 * 2 ** 20, dtype=torch.uint8, device="cuda")
+
+    def call():
+        aht.aht_rollout_ippo(ctx, 0, 1, wl.T, t0, t1, wl.gamma, wl.lam)
+
+    for _ in range(3):
+        call()
+    torch.cuda.synchronize()
+    K = 5
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    aht.aht_get_timing(ctx)
+    aht.aht_set_timing(ctx, True)
+    for k in range(K):
+        scrub.fill_(k & 0xFF)
+        ev[k][0].record(stream)
+        call()
+        ev[k][1].record(stream)
+    torch.cuda.synchronize()
+    aht.aht_set_timing(ctx, False)
+    kernel_ms, launches = aht.aht_get_timing(ctx)
+    aht.aht_sync(ctx)
+    ctx.close()
+    ms = sum(a.elapsed_time(b) for a, b in ev) / K
+    kern_ms = kernel_ms / max(1, launches)
+    dims = [wl.env.obs_dim, *wl.hidden, wl.env.n_actions + 1]
+    flops = (wl.n_envs * wl.T + wl.n_envs) * 2 * mlp_flops(dims)
+    achieved = flops / (kern_ms * 1e-3) / 1e12
+    return {"workload": wl.name, "ms_per_call": ms, "env_steps_per_s": wl.n_envs * wl.T / (ms * 1e-3),
+            "learner_samples_per_s": 2 * wl.n_envs * wl.T / (ms * 1e-3), "kernel_ms": kern_ms,
+            "roofline": {"bound": "tensor", "achieved": achieved, "peak": bf16_peak, "unit": "TFLOP/s",
+                         "frac": achieved / bf16_peak, "flops_per_launch": flops}}
 
 
 PPO_FLOPS_PER_SAMPLE = 204032   # forward 84,736 + backward 119,296 (dW1, dW2, dh1, dW3, dh2)

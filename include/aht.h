@@ -171,6 +171,19 @@ typedef struct aht_traj {
 aht_status aht_rollout(aht_ctx* ctx, int32_t ego_id, const int32_t* pool, int32_t pool_size,
                        int32_t T, const aht_traj* out);
 
+/* IPPO collection (Sec. 3, the MARL baseline IPPO: both seats learn, each with its own
+ * PPO of App. C).  Every env pairs policy0 in seat 0 with policy1 in seat 1; the call is
+ * aht_rollout(ctx, policy0, {policy1}, 1, T, out0) -- the same draws, states and seat-0
+ * trajectory -- and it also writes seat 1's learner trajectory to out1, in the layout
+ * of aht_traj: obs = seat 1's observation (4-byte aligned), actions = seat 1's action,
+ * tm_actions = seat 0's, logp / values / last_value of policy1 (values 0 without its
+ * value row), the shared team reward, dones, and GAE into out1's advantages / targets
+ * when those are non-NULL.  out1->teammate is not written.  policy1 is a network
+ * (0 <= policy1 < n_policies); a trajectory of out1 is an aht_ppo_update input for a
+ * learner of policy1. */
+aht_status aht_rollout_ippo(aht_ctx* ctx, int32_t policy0, int32_t policy1, int32_t T,
+                            const aht_traj* out0, const aht_traj* out1);
+
 /* Outputs of aht_xplay_matrix (caller-owned device memory; NULL members not written). */
 typedef struct aht_xplay_out {
   float* matrix;        /* [n_ego][n_tm] mean team return over the pair's envs */
@@ -323,7 +336,7 @@ aht_status aht_learner_get(aht_learner* L, float* params, float* adam_m, float* 
 aht_status aht_learner_set(aht_learner* L, const float* params, const float* adam_m,
                            const float* adam_v, int64_t t, int64_t updates);
 /* Writes the learner's current weights into policy `policy` of ctx (aht_set_policy with
- * fp32 weights; the ctx's own packing rounds them to its weight type). */
+ * the fp32 weights for an fp32 population, their nearest-even bf16 for a bf16 one). */
 aht_status aht_learner_push(aht_learner* L, aht_ctx* ctx, int32_t policy);
 /* Synchronises the learner's stream; AHT_ETIMEOUT if a bounded wait of its kernels
  * expired (the status word is then cleared). */

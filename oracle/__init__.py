@@ -136,7 +136,8 @@ class RolloutIO(C.Structure):
                 ("forced", _P), ("env_ids", _P), ("states", _P), ("n_threads", C.c_int32),
                 ("teammate", _P), ("obs", _P), ("obs_tm", _P), ("actions", _P),
                 ("own_actions", _P), ("margin", _P), ("logits", _P), ("logp", _P),
-                ("values", _P), ("rewards", _P), ("dones", _P), ("last_value", _P)]
+                ("values", _P), ("rewards", _P), ("dones", _P), ("last_value", _P),
+                ("logp_tm", _P), ("values_tm", _P), ("last_value_tm", _P)]
 
 
 class XplayIO(C.Structure):
@@ -347,7 +348,9 @@ def rollout(d, pols: Policies, seed, states, step0, T, ego_id, pool, forced=None
         own_actions=np.zeros((T, N, 2), np.uint8), margin=np.zeros((T, N, 2), np.float64),
         logits=np.zeros((T, N, n_out), np.float64), logp=np.zeros((T, N), np.float64),
         values=np.zeros((T, N), np.float64), rewards=np.zeros((T, N), np.float32),
-        dones=np.zeros((T, N), np.uint8), last_value=np.zeros(N, np.float64))
+        dones=np.zeros((T, N), np.uint8), last_value=np.zeros(N, np.float64),
+        logp_tm=np.zeros((T, N), np.float64), values_tm=np.zeros((T, N), np.float64),
+        last_value_tm=np.zeros(N, np.float64))
     if forced is not None:
         forced = np.ascontiguousarray(forced, np.uint8)
         assert forced.shape == (T, N, 2)

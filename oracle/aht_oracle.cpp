@@ -1283,6 +1283,8 @@ extern "C" int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32
       if (io->logits) std::memcpy(io->logits + i * ego->n_out, z0.data(), sizeof(double) * ego->n_out);
       if (io->logp) io->logp[i] = orc_logp(z0.data(), legal.data(), K, act[0]);
       if (io->values) io->values[i] = has_value ? z0[K] : 0.0;
+      if (io->logp_tm) io->logp_tm[i] = tm ? orc_logp(z1.data(), legal.data(), K, act[1]) : 0.0;
+      if (io->values_tm) io->values_tm[i] = tm && tm->n_out > K ? z1[K] : 0.0;
       float r[2], team;
       int done = env_step(d, st, act[0], act[1], r, &team);
       if (done < 0) { status[e] = -2; done = 0; team = 0.0f; }
@@ -1294,6 +1296,15 @@ extern "C" int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32
       env_obs(d, st, 0, o0.data());
       orc_mlp_forward(ego, obs_to_double(o0.data(), od).data(), z0.data());
       io->last_value[e] = has_value ? z0[K] : 0.0;
+    }
+    if (io->last_value_tm) {
+      double v = 0.0;
+      if (tm && tm->n_out > K) {
+        env_obs(d, st, 1, o1.data());
+        orc_mlp_forward(tm, obs_to_double(o1.data(), od).data(), z1.data());
+        v = z1[K];
+      }
+      io->last_value_tm[e] = v;
     }
   });
   for (int64_t e = 0; e < N; ++e)

@@ -234,6 +234,10 @@ typedef struct orc_rollout_io {
   float* rewards;              /* [T][N] team reward */
   uint8_t* dones;              /* [T][N] */
   double* last_value;          /* [N] value of the state after the last step */
+  /* the teammate seat's learner outputs (IPPO, both seats learn; 0 for a rule teammate) */
+  double* logp_tm;             /* [T][N] teammate logp of its applied action */
+  double* values_tm;           /* [T][N] teammate value (0 without a value row) */
+  double* last_value_tm;       /* [N] teammate value of the state after the last step */
 } orc_rollout_io;
 int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32_t n_pols,
                     orc_rollout_io* io);

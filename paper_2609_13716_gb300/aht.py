@@ -26,7 +26,7 @@ EXPORTED = ["aht_create", "aht_destroy", "aht_reset", "aht_rollout", "aht_xplay_
             "aht_xplay_matrix_static", "aht_debug_tanh", "aht_debug_expire_wait",
             "aht_xp_stats", "aht_learner_create", "aht_learner_destroy", "aht_learner_n_params",
             "aht_ppo_update", "aht_ppo_grad", "aht_learner_get", "aht_learner_set",
-            "aht_learner_push", "aht_learner_sync"]
+            "aht_learner_push", "aht_learner_sync", "aht_rollout_ippo"]
 
 
 class AhtError(RuntimeError):
@@ -108,6 +108,7 @@ def load() -> C.CDLL:
             L.aht_destroy.restype = None
             L.aht_reset.argtypes = [vp, u64]
             L.aht_rollout.argtypes = [vp, i32, C.POINTER(i32), i32, i32, C.POINTER(Traj)]
+            L.aht_rollout_ippo.argtypes = [vp, i32, i32, i32, C.POINTER(Traj), C.POINTER(Traj)]
             L.aht_xplay_matrix.argtypes = [vp, C.POINTER(i32), i32, C.POINTER(i32), i32, i32, i32, C.POINTER(XplayOut)]
             L.aht_gae.argtypes = [vp, vp, vp, vp, i64, i32, C.c_float, C.c_float, vp, vp, vp]
             L.aht_xp_stats.argtypes = [vp, i32, i32, vp, C.POINTER(XpStatsOut), vp]
@@ -140,7 +141,8 @@ def load() -> C.CDLL:
             for f in ("aht_learner_create", "aht_ppo_update", "aht_ppo_grad", "aht_learner_get",
                       "aht_learner_set", "aht_learner_push", "aht_learner_sync"):
                 getattr(L, f).restype = C.c_int
-            for f in ("aht_create", "aht_reset", "aht_rollout", "aht_xplay_matrix", "aht_gae", "aht_xp_stats",
+            for f in ("aht_create", "aht_reset", "aht_rollout", "aht_rollout_ippo", "aht_xplay_matrix",
+                      "aht_gae", "aht_xp_stats",
                       "aht_step_forced", "aht_policy_forward", "aht_get_state", "aht_set_state",
                       "aht_sync", "aht_set_policy", "aht_set_timing", "aht_get_timing"):
                 getattr(L, f).restype = C.c_int
@@ -241,11 +243,11 @@ def traj_buffers(ctx: Context, T: int, device="cuda", obs=True):
                 last_value=z((N,), torch.float32), teammate=z((N,), torch.int32))
 
 
-def aht_rollout(ctx: Context, ego_id, pool, T, traj: dict, gamma=0.99, lam=0.95):
+def _traj(ctx: Context, T, traj: dict, gamma, lam):
     N = ctx.n_envs
     f32, u8 = torch.float32, torch.uint8
     g = traj.get
-    t = Traj(_ptr(g("obs"), u8, (T, N, ctx.obs_dim), "obs"),
+    return Traj(_ptr(g("obs"), u8, (T, N, ctx.obs_dim), "obs"),
              _ptr(g("actions"), u8, (T, N), "actions"),
              _ptr(g("tm_actions"), u8, (T, N), "tm_actions"),
              _ptr(g("logp"), f32, (T, N), "logp"), _ptr(g("values"), f32, (T, N), "values"),
@@ -254,9 +256,21 @@ def aht_rollout(ctx: Context, ego_id, pool, T, traj: dict, gamma=0.99, lam=0.95)
              _ptr(g("targets"), f32, (T, N), "targets"),
              _ptr(g("last_value"), f32, (N,), "last_value"),
              _ptr(g("teammate"), torch.int32, (N,), "teammate"), gamma, lam)
+
+
+def aht_rollout(ctx: Context, ego_id, pool, T, traj: dict, gamma=0.99, lam=0.95):
+    t = _traj(ctx, T, traj, gamma, lam)
     pool = list(pool)
     parr = (C.c_int32 * len(pool))(*pool)
     _check(load().aht_rollout(ctx.handle, ego_id, parr, len(pool), T, C.byref(t)))
+
+
+def aht_rollout_ippo(ctx: Context, policy0, policy1, T, traj0: dict, traj1: dict,
+                     gamma=0.99, lam=0.95):
+    """IPPO collection: traj0 gets seat 0's (policy0) trajectory, traj1 seat 1's."""
+    t0 = _traj(ctx, T, traj0, gamma, lam)
+    t1 = _traj(ctx, T, traj1, gamma, lam)
+    _check(load().aht_rollout_ippo(ctx.handle, policy0, policy1, T, C.byref(t0), C.byref(t1)))
 
 
 def aht_xplay_matrix(ctx: Context, ego_ids, tm_ids, envs_per_pair, max_steps, matrix,

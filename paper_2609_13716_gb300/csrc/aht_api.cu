@@ -638,7 +638,7 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
       {(void**)&c->perm, (size_t)n_envs * 4},
       {(void**)&c->tiles, (size_t)c->max_tiles * sizeof(int4)},
       {(void**)&c->xp_returns, (size_t)n_envs * 4},
-      {(void**)&c->last_value, (size_t)n_envs * 4},
+      {(void**)&c->last_value, (size_t)n_envs * 8},  // V_T scratch of seat 0 and seat 1
       {(void**)&c->status, 4},
   };
   for (auto& a : allocs)
@@ -745,8 +745,18 @@ aht_status aht_reset(aht_ctx* c, uint64_t seed) {
   return AHT_OK;
 }
 
-aht_status aht_rollout(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t pool_size,
-                       int32_t T, const aht_traj* out) {
+static aht_status check_traj_out(const aht_traj* out) {
+  if (out->advantages && (!out->rewards || !out->values || !out->dones))
+    return fail(AHT_EINVAL, "advantages need rewards, values and dones");
+  if (out->gamma < 0.f || out->gamma > 1.f || out->lambda < 0.f || out->lambda > 1.f)
+    return fail(AHT_EINVAL, "gamma and lambda must be in [0, 1]");
+  return AHT_OK;
+}
+
+// PPO collection with pool-drawn teammates; out1 (may be NULL) receives seat 1's learner
+// trajectory (IPPO).
+static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t pool_size,
+                                 int32_t T, const aht_traj* out, const aht_traj* out1) {
   if (!c || !out) return fail(AHT_EINVAL, "ctx or out is NULL");
   if (c->env.kind == AHT_HANABI || c->env.kind == AHT_MINI_HANABI)
     return fail(AHT_EINVAL, "PPO collection needs a simultaneous-move env (LBF, Overcooked)");
@@ -759,10 +769,12 @@ aht_status aht_rollout(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t 
   }
   if (T < 1) return fail(AHT_EINVAL, "T must be >= 1");
   if (c->step + T + 1 > (int64_t)UINT32_MAX) return fail(AHT_EINVAL, "step counter would exceed 2^32");
-  if (out->advantages && (!out->rewards || !out->values || !out->dones))
-    return fail(AHT_EINVAL, "advantages need rewards, values and dones");
-  if (out->gamma < 0.f || out->gamma > 1.f || out->lambda < 0.f || out->lambda > 1.f)
-    return fail(AHT_EINVAL, "gamma and lambda must be in [0, 1]");
+  if (aht_status e = check_traj_out(out)) return e;
+  if (out1) {
+    if (aht_status e = check_traj_out(out1)) return e;
+    if (reinterpret_cast<uintptr_t>(out1->obs) & 3u)
+      return fail(AHT_EINVAL, "out1->obs must be 4-byte aligned");
+  }
   DeviceGuard g(c->device);
   const int M = c->tc ? 128 : fit_rows(c, 128);
 
@@ -792,6 +804,11 @@ aht_status aht_rollout(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t 
   a.traj = TrajPtrs{out->obs, out->actions, out->tm_actions, out->logp, out->values,
                     out->rewards, out->dones,
                     out->last_value ? out->last_value : (out->advantages ? c->last_value : nullptr)};
+  if (out1)
+    a.traj1 = TrajPtrs{out1->obs, out1->actions, out1->tm_actions, out1->logp, out1->values,
+                       out1->rewards, out1->dones,
+                       out1->last_value ? out1->last_value
+                                        : (out1->advantages ? c->last_value + c->n_envs : nullptr)};
   if (c->tc) {
     PpoTcArgs ta{};
     ta.b = a.b;
@@ -805,6 +822,7 @@ aht_status aht_rollout(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t 
     ta.step0 = a.step0;
     ta.T = T;
     ta.traj = a.traj;
+    ta.traj1 = a.traj1;
     const int tk = timer_begin(c);
     AHT_CUDA(lbf_ppo_tc(ta, ga.max_tiles, c->tc_smem, c->stream));
     timer_end(c, tk);
@@ -817,8 +835,23 @@ aht_status aht_rollout(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t 
   if (out->advantages)
     AHT_CUDA(launch_gae(out->rewards, out->values, out->dones, a.traj.last_value, c->n_envs, T,
                         out->gamma, out->lambda, out->advantages, out->targets, c->stream));
+  if (out1 && out1->advantages)
+    AHT_CUDA(launch_gae(out1->rewards, out1->values, out1->dones, a.traj1.last_value, c->n_envs, T,
+                        out1->gamma, out1->lambda, out1->advantages, out1->targets, c->stream));
   c->step += T;
   return AHT_OK;
+}
+
+aht_status aht_rollout(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t pool_size,
+                       int32_t T, const aht_traj* out) {
+  return rollout_common(c, ego_id, pool, pool_size, T, out, nullptr);
+}
+
+aht_status aht_rollout_ippo(aht_ctx* c, int32_t policy0, int32_t policy1, int32_t T,
+                            const aht_traj* out0, const aht_traj* out1) {
+  if (!c || !out1) return fail(AHT_EINVAL, "ctx or out1 is NULL");
+  if (policy1 < 0 || policy1 >= c->n_policies) return fail(AHT_EINVAL, "policy1 out of range");
+  return rollout_common(c, policy0, &policy1, 1, T, out0, out1);
 }
 
 aht_status aht_xplay_matrix(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego,
@@ -1410,9 +1443,21 @@ aht_status aht_learner_push(aht_learner* L, aht_ctx* c, int32_t policy) {
   DeviceGuard g(L->device);
   AHT_CUDA(cudaStreamSynchronize(L->stream));
   const float* p = L->params;
-  const void* W[3] = {p, p + L->L.oW2, p + L->L.oW3};
-  const void* bb[3] = {p + L->L.ob1, p + L->L.ob2, p + L->L.ob3};
-  return aht_set_policy(c, policy, W, bb, AHT_FP32, 1);
+  if (c->weight_dtype == AHT_FP32) {
+    const void* W[3] = {p, p + L->L.oW2, p + L->L.oW3};
+    const void* bb[3] = {p + L->L.ob1, p + L->L.ob2, p + L->L.ob3};
+    return aht_set_policy(c, policy, W, bb, AHT_FP32, 1);
+  }
+  // a bf16 population: the nearest-even bf16 of every parameter
+  const int64_t n = L->L.n_params;
+  std::vector<float> host((size_t)n);
+  AHT_CUDA(cudaMemcpy(host.data(), p, (size_t)n * 4, cudaMemcpyDeviceToHost));
+  std::vector<uint16_t> h16((size_t)n);
+  for (int64_t i = 0; i < n; ++i) h16[(size_t)i] = bf16_rne(host[(size_t)i]);
+  const uint16_t* q = h16.data();
+  const void* W[3] = {q, q + L->L.oW2, q + L->L.oW3};
+  const void* bb[3] = {q + L->L.ob1, q + L->L.ob2, q + L->L.ob3};
+  return aht_set_policy(c, policy, W, bb, AHT_BF16, 1);
 }
 
 aht_status aht_learner_sync(aht_learner* L) {

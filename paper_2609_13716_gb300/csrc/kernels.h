@@ -35,6 +35,9 @@ struct PpoArgs {
   uint32_t step0;
   int32_t T;
   TrajPtrs traj;
+  TrajPtrs traj1;        // seat 1's learner trajectory (IPPO); all NULL otherwise: obs,
+                         // actions = its own, tm_actions = seat 0's, logp, values,
+                         // rewards, dones, last_value of the seat-1 policy
 };
 
 // Per-policy block of the tensor-core path (byte offsets within the block):
@@ -80,6 +83,7 @@ struct PpoTcArgs {
   uint32_t step0;
   int32_t T;
   TrajPtrs traj;
+  TrajPtrs traj1;        // as in PpoArgs
   TcXp xp;               // cross-play launches only
 };
 

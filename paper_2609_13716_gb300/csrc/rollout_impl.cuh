@@ -110,6 +110,8 @@ __global__ void __launch_bounds__(kThreads) ppo_kernel(const PpoArgs a) {
       __syncthreads();
       if (seat == 0 && a.traj.obs)
         copy_obs_rows(X, m.KP, count, envid, a.traj.obs + (int64_t)t * N * od, od);
+      if (seat == 1 && a.traj1.obs)
+        copy_obs_rows(X, m.KP, count, envid, a.traj1.obs + (int64_t)t * N * od, od);
       mlp_tile(w_pol[seat], m, X, H1, H2, Z, M);
       for (int i = tid; i < count; i += blockDim.x) {
         const float u = u01(draw0(a.b.key, (uint32_t)envid[i], gt, kStreamAct0 + seat));
@@ -119,6 +121,10 @@ __global__ void __launch_bounds__(kThreads) ppo_kernel(const PpoArgs a) {
         if (seat == 0) {
           lp[i] = logp;
           val[i] = Z[i * m.NOP + m.NA];
+        } else {
+          const int64_t o = (int64_t)t * N + envid[i];
+          if (a.traj1.logp) a.traj1.logp[o] = logp;
+          if (a.traj1.values) a.traj1.values[o] = Z[i * m.NOP + m.NA];
         }
       }
       __syncthreads();
@@ -134,6 +140,10 @@ __global__ void __launch_bounds__(kThreads) ppo_kernel(const PpoArgs a) {
       if (a.traj.values) a.traj.values[o] = val[i];
       if (a.traj.rewards) a.traj.rewards[o] = team;
       if (a.traj.dones) a.traj.dones[o] = (uint8_t)(done > 0);
+      if (a.traj1.actions) a.traj1.actions[o] = act[2 * i + 1];
+      if (a.traj1.tm_actions) a.traj1.tm_actions[o] = act[2 * i];
+      if (a.traj1.rewards) a.traj1.rewards[o] = team;
+      if (a.traj1.dones) a.traj1.dones[o] = (uint8_t)(done > 0);
       if (done > 0) Env::reset(a.b.env, a.b.key, (uint32_t)env, gt + 1, st[i]);
     }
     __syncthreads();
@@ -144,6 +154,13 @@ __global__ void __launch_bounds__(kThreads) ppo_kernel(const PpoArgs a) {
     __syncthreads();
     mlp_tile(w_pol[0], m, X, H1, H2, Z, M);
     for (int i = tid; i < count; i += blockDim.x) a.traj.last_value[envid[i]] = Z[i * m.NOP + m.NA];
+    __syncthreads();
+  }
+  if (a.traj1.last_value) {  // seat 1's V_T (IPPO)
+    for (int i = tid; i < count; i += blockDim.x) Env::obs(a.b.env, st[i], 1, X + i * m.KP);
+    __syncthreads();
+    mlp_tile(w_pol[1], m, X, H1, H2, Z, M);
+    for (int i = tid; i < count; i += blockDim.x) a.traj1.last_value[envid[i]] = Z[i * m.NOP + m.NA];
   }
   for (int i = tid; i < count; i += blockDim.x) store_state(a.state, N, envid[i], st[i]);
 }

@@ -40,9 +40,11 @@ constexpr int kTcComputeBar = 1;         // named barrier id of the compute warp
 // step, frozen once done; the per-env return and episode length are the outputs) instead
 // of PPO collection.  kSplit: fp32 weights held as bf16 pairs W = W_hi + W_lo, L1 =
 // X W1_hi + X W1_lo and L2 = b2 + hi W2_hi + lo W2_hi + hi W2_lo (lo W2_lo is below
-// 2^-16 of the sum and left out).
-template <class Env, bool kXp, bool kSplit>
+// 2^-16 of the sum and left out).  kIppo (PPO collection only): seat 1 learns too, and
+// its trajectory goes to a.traj1.
+template <class Env, bool kXp, bool kSplit, bool kIppo>
 __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a) {
+  static_assert(!(kXp && kIppo), "seat-1 trajectories belong to PPO collection");
   using State = typename Env::State;
   constexpr int NA = Env::kNumActions;
   extern __shared__ __align__(16) uint8_t smem[];  // no-swizzle operands need 16 B
@@ -81,7 +83,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   const int split = (chunks + 1) / 2;
   const int my_c0 = half ? split : 0, my_c1 = half ? chunks : split;
   const int my_w0 = min(4 * my_c0, cells), my_w1 = min(4 * my_c1, cells);
-  const bool with_boot = !kXp && a.traj.last_value != nullptr;
+  // V_T after the last step: the ego's, and seat 1's when it learns too (IPPO)
+  const bool boot1 = kIppo && !tm_rule && a.traj1.last_value != nullptr;
+  const bool with_boot = !kXp && (a.traj.last_value != nullptr || boot1);
 
   // The tile is the contiguous env range [tile.x, tile.x + count); observation rows are
   // packed at obs_dim bytes (an odd number of words: no bank conflicts per thread row),
@@ -169,8 +173,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         if (ok && !stopped) issue(0, 1, par);
       }
       if (ok && with_boot) {
-        issue(0, 0, (uint32_t)a.T & 1u);
-        if (ok) issue(0, 1, (uint32_t)a.T & 1u);
+        const uint32_t par = (uint32_t)a.T & 1u;
+        if (boot1) issue(1, 0, par);
+        if (ok) issue(0, 0, par);
+        if (ok && boot1) issue(1, 1, par);
+        if (ok) issue(0, 1, par);
       }
       if (!ok) abort_flag = 1;
     }
@@ -190,10 +197,15 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     auto pol_block = [&](int ag) { return sW0 + (size_t)ag * d.pol_bytes; };
 
     // observation (built into this thread's half row) -> bf16 A operand of L1; feature
-    // obs_dim is the constant 1 that carries b1, the rest of the padding is 0
-    auto obs_x = [&](int ag, const State& s) {
+    // obs_dim is the constant 1 that carries b1, the rest of the padding is 0.  obs1:
+    // seat 1's trajectory row (IPPO), which gets this thread's words of the row.
+    auto obs_x = [&](int ag, const State& s, uint32_t* obs1) {
       uint32_t* roww = reinterpret_cast<uint32_t*>(sObs + row * od);
-      if (row < count) Env::obs_words(a.b.env, s, ag, roww, my_w0, my_w1);
+      if (row < count) {
+        Env::obs_words(a.b.env, s, ag, roww, my_w0, my_w1);
+        if (ag == 1 && obs1)
+          for (int w = my_w0; w < my_w1; ++w) obs1[w] = roww[w];
+      }
       const uint32_t P = tmem + (uint32_t)(ag * 256) + lane_base;
       for (int c = my_c0; c < my_c1; ++c) {
         uint32_t w4[4];
@@ -319,13 +331,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
           break;
         }
       }
-      const int first = boot || tm_rule ? 0 : 1;  // teammate first: the ego's rows stay for the copy
+      // teammate first: the ego's rows stay for the copy
+      const int first = (boot && !boot1) || tm_rule ? 0 : 1;
       const uint32_t par = (uint32_t)t & 1u, gt = a.step0 + (uint32_t)t;
       // this half's action draw (ego: warps 0-3, teammate: warps 4-7), ahead of its use
       const float u_act = boot ? 0.0f : u01(draw0(a.b.key, (uint32_t)(env0 + row), gt, kStreamAct0 + half));
       State s = st[row];  // register copy for this step (rows past count are never used)
+      uint32_t* obs1 = kIppo && !boot && a.traj1.obs
+                           ? reinterpret_cast<uint32_t*>(a.traj1.obs + ((int64_t)t * N + env0 + row) * od)
+                           : nullptr;
 #pragma unroll 1
-      for (int i = first; i >= 0; --i) obs_x(i, s);
+      for (int i = first; i >= 0; --i) obs_x(i, s, obs1);
 #pragma unroll 1
       for (int i = first; i >= 0; --i) {
         wait_acc(i, 0, par);
@@ -344,9 +360,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       if (sync_or()) break;
       float z[16];
       if (boot) {
-        if (half == 0 && row < count) {
+        if (half == 0 && row < count && a.traj.last_value) {
           logits(0, z);
           a.traj.last_value[env0 + row] = z[NA];
+        } else if (kIppo && half == 1 && row < count && boot1) {
+          logits(1, z);
+          a.traj1.last_value[env0 + row] = z[NA];
         }
         break;
       }
@@ -361,6 +380,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         const int act = sample_k<NA>(z, 0xFFFFFFFFu >> (32 - NA), u_act, lp);
         if (ag == 1) {
           act1s[row] = (uint8_t)act;
+          if constexpr (kIppo) {
+            const int64_t o = (int64_t)t * N + env0 + row;
+            if (a.traj1.logp) a.traj1.logp[o] = lp;
+            if (a.traj1.values) a.traj1.values[o] = z[NA];
+          }
         } else {
           act0 = act;
           lp0 = lp;
@@ -398,6 +422,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         if (a.traj.values) a.traj.values[o] = val0;
         if (a.traj.rewards) a.traj.rewards[o] = team;
         if (a.traj.dones) a.traj.dones[o] = (uint8_t)(done > 0);
+        if constexpr (kIppo) {
+          if (a.traj1.actions) a.traj1.actions[o] = (uint8_t)act1;
+          if (a.traj1.tm_actions) a.traj1.tm_actions[o] = (uint8_t)act0;
+          if (a.traj1.rewards) a.traj1.rewards[o] = team;
+          if (a.traj1.dones) a.traj1.dones[o] = (uint8_t)(done > 0);
+        }
         if (done > 0) Env::reset(a.b.env, a.b.key, (uint32_t)env, gt + 1, s);
         st[row] = s;
       }
@@ -435,19 +465,24 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
 
 template <class Env>
 struct LaunchTc {
-  template <bool kXp, bool kSplit>
+  template <bool kXp, bool kSplit, bool kIppo>
   static cudaError_t run(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
-    cudaError_t e = cudaFuncSetAttribute(ppo_tc_kernel<Env, kXp, kSplit>,
+    cudaError_t e = cudaFuncSetAttribute(ppo_tc_kernel<Env, kXp, kSplit, kIppo>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    ppo_tc_kernel<Env, kXp, kSplit><<<grid, kTcThreads, smem, s>>>(a);
+    ppo_tc_kernel<Env, kXp, kSplit, kIppo><<<grid, kTcThreads, smem, s>>>(a);
     return cudaGetLastError();
   }
   static cudaError_t ppo(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
-    return a.tc.split ? run<false, true>(a, grid, smem, s) : run<false, false>(a, grid, smem, s);
+    const TrajPtrs& u = a.traj1;
+    const bool ippo = u.obs || u.actions || u.tm_actions || u.logp || u.values || u.rewards ||
+                      u.dones || u.last_value;
+    if (ippo)
+      return a.tc.split ? run<false, true, true>(a, grid, smem, s) : run<false, false, true>(a, grid, smem, s);
+    return a.tc.split ? run<false, true, false>(a, grid, smem, s) : run<false, false, false>(a, grid, smem, s);
   }
   static cudaError_t xplay(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
-    return a.tc.split ? run<true, true>(a, grid, smem, s) : run<true, false>(a, grid, smem, s);
+    return a.tc.split ? run<true, true, false>(a, grid, smem, s) : run<true, false, false>(a, grid, smem, s);
   }
 };
 

@@ -123,6 +123,12 @@ WORKLOADS = {
         name="lbf7x7_ppo_16384x128", index=2, env=_lbf(50), hidden=(128, 128),
         weight_dtype=BF16, n_policies=33, value_head=(1,) + (0,) * 32, mode="ppo",
         env_seed=2, n_envs=16384, T=128, ego_id=0, pool=tuple(range(1, 33))),
+    # IPPO collection (both seats learn): two bf16 196-128-128-(6+1) policies with value
+    # rows, 16384 envs x 128 steps, seat 0 = policy 0, seat 1 = policy 1 in every env.
+    "lbf7x7_ippo_16384x128": Workload(
+        name="lbf7x7_ippo_16384x128", index=9, env=_lbf(50), hidden=(128, 128),
+        weight_dtype=BF16, n_policies=2, value_head=(1, 1), mode="ppo",
+        env_seed=9, n_envs=16384, T=128, ego_id=0, pool=(1,)),
     # 5x4 kitchen: 8 x 8 pairs, 64 envs per pair (4096 envs), 400-step episodes,
     # 520-256-256-6 bf16 MLPs.
     "overcooked5x4_xplay_8x8x64": Workload(
