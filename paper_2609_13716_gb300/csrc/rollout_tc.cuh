@@ -35,6 +35,7 @@ namespace aht {
 constexpr int kTcCompute = 256;          // compute threads
 constexpr int kTcThreads = 288;          // + one MMA warp
 constexpr int kTcComputeBar = 1;         // named barrier id of the compute warps
+constexpr int kTcPairBar = 2;            // ids 2..5: warps q and q + 4 (rows 32q .. 32q + 31)
 
 // kXp: cross-play (each tile is a chunk of one pair's envs, reset at the call's first
 // step, frozen once done; the per-env return and episode length are the outputs) instead
@@ -197,15 +198,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     auto pol_block = [&](int ag) { return sW0 + (size_t)ag * d.pol_bytes; };
 
     // observation (built into this thread's half row) -> bf16 A operand of L1; feature
-    // obs_dim is the constant 1 that carries b1, the rest of the padding is 0.  obs1:
-    // seat 1's trajectory row (IPPO), which gets this thread's words of the row.
-    auto obs_x = [&](int ag, const State& s, uint32_t* obs1) {
+    // obs_dim is the constant 1 that carries b1, the rest of the padding is 0
+    auto obs_x = [&](int ag, const State& s) {
       uint32_t* roww = reinterpret_cast<uint32_t*>(sObs + row * od);
-      if (row < count) {
-        Env::obs_words(a.b.env, s, ag, roww, my_w0, my_w1);
-        if (ag == 1 && obs1)
-          for (int w = my_w0; w < my_w1; ++w) obs1[w] = roww[w];
-      }
+      if (row < count) Env::obs_words(a.b.env, s, ag, roww, my_w0, my_w1);
       const uint32_t P = tmem + (uint32_t)(ag * 256) + lane_base;
       for (int c = my_c0; c < my_c1; ++c) {
         uint32_t w4[4];
@@ -337,11 +333,24 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       // this half's action draw (ego: warps 0-3, teammate: warps 4-7), ahead of its use
       const float u_act = boot ? 0.0f : u01(draw0(a.b.key, (uint32_t)(env0 + row), gt, kStreamAct0 + half));
       State s = st[row];  // register copy for this step (rows past count are never used)
-      uint32_t* obs1 = kIppo && !boot && a.traj1.obs
-                           ? reinterpret_cast<uint32_t*>(a.traj1.obs + ((int64_t)t * N + env0 + row) * od)
-                           : nullptr;
 #pragma unroll 1
-      for (int i = first; i >= 0; --i) obs_x(i, s, obs1);
+      for (int i = first; i >= 0; --i) {
+        obs_x(i, s);
+        if (kIppo && i == 1 && !boot && a.traj1.obs) {
+          // seat 1's rows -> its trajectory before the ego's overwrite them: warps q and
+          // q + 4 built rows 32q .. 32q + 31, a contiguous block in shared and in global
+          // memory, which they store with consecutive words
+          const int q = warp & 3, pt = half * 32 + lane;
+          tc::bar_sync(kTcPairBar + q, 64);
+          const int rows = min(32, count - 32 * q);
+          if (rows > 0) {
+            const uint32_t* src = reinterpret_cast<const uint32_t*>(sObs + 32 * q * od);
+            uint32_t* dst = reinterpret_cast<uint32_t*>(a.traj1.obs + ((int64_t)t * N + env0 + 32 * q) * od);
+            for (int w = pt; w < rows * cells; w += 64) dst[w] = src[w];
+          }
+          tc::bar_sync(kTcPairBar + q, 64);
+        }
+      }
 #pragma unroll 1
       for (int i = first; i >= 0; --i) {
         wait_acc(i, 0, par);
