@@ -137,7 +137,8 @@ class RolloutIO(C.Structure):
                 ("teammate", _P), ("obs", _P), ("obs_tm", _P), ("actions", _P),
                 ("own_actions", _P), ("margin", _P), ("logits", _P), ("logp", _P),
                 ("values", _P), ("rewards", _P), ("dones", _P), ("last_value", _P),
-                ("logp_tm", _P), ("values_tm", _P), ("last_value_tm", _P)]
+                ("logp_tm", _P), ("values_tm", _P), ("last_value_tm", _P),
+                ("resample", C.c_int32), ("ep_step", _P), ("teammates_t", _P)]
 
 
 class XplayIO(C.Structure):
@@ -331,9 +332,11 @@ def step_forced(d, seed, step, states, actions):
 
 
 def rollout(d, pols: Policies, seed, states, step0, T, ego_id, pool, forced=None, n_threads=1,
-            env_ids=None):
+            env_ids=None, ep_step=None, resample=False):
     """PPO collection.  Returns a dict of numpy arrays; states are updated in place.
-    env_ids: global env index of each state row (default 0..N-1)."""
+    env_ids: global env index of each state row (default 0..N-1).  ep_step: uint32 [N]
+    step at which each env's episode began, updated in place at auto-resets; resample:
+    per-episode teammates (needs ep_step)."""
     N = states.shape[0]
     if env_ids is not None:
         env_ids = np.ascontiguousarray(env_ids, np.int64)
@@ -350,13 +353,15 @@ def rollout(d, pols: Policies, seed, states, step0, T, ego_id, pool, forced=None
         values=np.zeros((T, N), np.float64), rewards=np.zeros((T, N), np.float32),
         dones=np.zeros((T, N), np.uint8), last_value=np.zeros(N, np.float64),
         logp_tm=np.zeros((T, N), np.float64), values_tm=np.zeros((T, N), np.float64),
-        last_value_tm=np.zeros(N, np.float64))
+        last_value_tm=np.zeros(N, np.float64), teammates_t=np.zeros((T, N), np.int32))
+    if ep_step is not None:
+        assert ep_step.dtype == np.uint32 and ep_step.shape == (N,) and ep_step.flags.c_contiguous
     if forced is not None:
         forced = np.ascontiguousarray(forced, np.uint8)
         assert forced.shape == (T, N, 2)
     io = RolloutIO(seed=seed, n_envs=N, step0=step0, T=T, ego_id=ego_id, pool=_ptr(pool),
                    pool_size=len(pool), forced=_ptr(forced), env_ids=_ptr(env_ids),
-                   states=_ptr(states),
+                   states=_ptr(states), resample=int(resample), ep_step=_ptr(ep_step),
                    n_threads=n_threads, **{k: _ptr(v) for k, v in out.items()})
     rc = lib().orc_rollout(C.byref(d), pols.arr, pols.n, C.byref(io))
     out["rc"] = rc

@@ -1230,6 +1230,7 @@ extern "C" int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32
   if (orc_check_desc(d) != 0) return -1;
   if (turn_based(d)) return -3;  // PPO collection is for simultaneous-move games
   if (io->ego_id < 0 || io->ego_id >= n_pols || io->pool_size < 1) return -4;
+  if (io->resample && !io->ep_step) return -4;
   const int min_id = d->kind == ORC_LBF ? -ORC_LBF_N_HEURISTICS : 0;  // heuristic teammates
   for (int k = 0; k < io->pool_size; ++k)
     if (io->pool[k] < min_id || io->pool[k] >= n_pols) return -4;
@@ -1243,17 +1244,27 @@ extern "C" int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32
     const uint32_t env = (uint32_t)(io->env_ids ? io->env_ids[e] : e);
     // Teammate: one uniform pool draw per block of ORC_TEAMMATE_BLOCK consecutive envs
     // and call, taken from the block's first env (counter (first env, step0, stream 3)).
+    // Per-episode mode: the teammate of the episode that began at step s.
+    auto episode_teammate = [&](uint32_t s) {
+      const uint32_t x = orc_draw(io->seed, env, s, ORC_STREAM_EPISODE_TEAMMATE, 0);
+      return io->pool[orc_uniform_int(x, (uint32_t)io->pool_size)];
+    };
     const uint32_t first = env - env % ORC_TEAMMATE_BLOCK;
     const uint32_t x = orc_draw(io->seed, first, (uint32_t)io->step0, ORC_STREAM_TEAMMATE, 0);
-    const int tm_id = io->pool[orc_uniform_int(x, (uint32_t)io->pool_size)];
+    int tm_id = io->resample ? episode_teammate(io->ep_step[e])
+                             : io->pool[orc_uniform_int(x, (uint32_t)io->pool_size)];
     if (io->teammate) io->teammate[e] = tm_id;
     const orc_mlp* tm = tm_id >= 0 ? &pols[tm_id] : nullptr;  // null: a heuristic teammate
     orc_state* st = &io->states[e];
     std::vector<uint8_t> o0(od), o1(od), legal(K, 1);
-    std::vector<double> z0(ego->n_out), z1(tm ? tm->n_out : 1);
+    int max_out = 1;
+    for (int k = 0; k < io->pool_size; ++k)
+      if (io->pool[k] >= 0) max_out = std::max(max_out, pols[io->pool[k]].n_out);
+    std::vector<double> z0(ego->n_out), z1(max_out);
     for (int t = 0; t < T; ++t) {
       const uint32_t gt = (uint32_t)(io->step0 + t);
       const int64_t i = (int64_t)t * N + e;
+      if (io->teammates_t) io->teammates_t[i] = tm_id;
       env_obs(d, st, 0, o0.data());
       env_obs(d, st, 1, o1.data());
       if (io->obs) std::memcpy(io->obs + i * od, o0.data(), od);
@@ -1290,7 +1301,14 @@ extern "C" int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32
       if (done < 0) { status[e] = -2; done = 0; team = 0.0f; }
       if (io->rewards) io->rewards[i] = team;
       if (io->dones) io->dones[i] = (uint8_t)done;
-      if (done) env_reset(d, io->seed, env, gt + 1, st);
+      if (done) {
+        env_reset(d, io->seed, env, gt + 1, st);
+        if (io->ep_step) io->ep_step[e] = gt + 1;
+        if (io->resample) {  // the next episode's teammate
+          tm_id = episode_teammate(gt + 1);
+          tm = tm_id >= 0 ? &pols[tm_id] : nullptr;
+        }
+      }
     }
     if (io->last_value) {
       env_obs(d, st, 0, o0.data());

@@ -37,7 +37,8 @@ extern "C" {
 #endif
 
 /* ---- randomness --------------------------------------------------------------- */
-enum { ORC_STREAM_ACT0 = 0, ORC_STREAM_ACT1 = 1, ORC_STREAM_RESET = 2, ORC_STREAM_TEAMMATE = 3 };
+enum { ORC_STREAM_ACT0 = 0, ORC_STREAM_ACT1 = 1, ORC_STREAM_RESET = 2, ORC_STREAM_TEAMMATE = 3,
+       ORC_STREAM_EPISODE_TEAMMATE = 5 };
 
 /* One Philox4x32-10 block: key (k0, k1), counter ctr[4] -> out[4]. */
 void orc_philox4x32_10(uint32_t k0, uint32_t k1, const uint32_t ctr[4], uint32_t out[4]);
@@ -206,7 +207,13 @@ void orc_gae(const float* r, const float* v, const uint8_t* d, const float* v_la
              double* adv, double* targets);
 
 /* ---- PPO rollout collection (simultaneous-move envs) ---------------------------- */
-/* Envs 128k .. 128k+127 share the teammate drawn for env 128k. */
+/* Teammates (Sec. 3: the ego meets teammates drawn from the training set).  Block mode:
+ * envs 128k .. 128k+127 share for the whole call the teammate drawn for env 128k at the
+ * call's first step.  Per-episode mode (resample = 1): each episode draws its own
+ * teammate when it begins -- env e whose current episode began at step s plays
+ * pool[uniform_int(x, pool_size)], x = word 0 of counter (e, s, stream 5); the step an
+ * episode began is carried per env in ep_step (0 after a reset of the whole batch), and
+ * every auto-reset at step s' sets it to s'. */
 enum { ORC_TEAMMATE_BLOCK = 128 };
 typedef struct orc_rollout_io {
   /* inputs */
@@ -238,6 +245,10 @@ typedef struct orc_rollout_io {
   double* logp_tm;             /* [T][N] teammate logp of its applied action */
   double* values_tm;           /* [T][N] teammate value (0 without a value row) */
   double* last_value_tm;       /* [N] teammate value of the state after the last step */
+  /* per-episode teammates */
+  int32_t resample;            /* 0: block mode, 1: per-episode mode (ep_step required) */
+  uint32_t* ep_step;           /* [N] in/out, or NULL in block mode */
+  int32_t* teammates_t;        /* [T][N] teammate policy id at each step, or NULL */
 } orc_rollout_io;
 int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32_t n_pols,
                     orc_rollout_io* io);
