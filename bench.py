@@ -367,6 +367,7 @@ def run_ours(args):
     if line is not None and not args.n_envs and not args.T:
         line["c0"] = run_c0(aht, W, torch, stream)
         line["ippo"] = run_ippo(aht, W, torch, stream, bf16_peak)
+        line["resample"] = run_resample(aht, wl, pop, torch, stream, bf16_peak)
     if not args.no_ppo:
         pu = run_ppo_update(args, aht, wl, pop_np, traj, torch, bf16_peak, stream)
         if line is not None:
@@ -454,6 +455,49 @@ def run_ippo(aht, W, torch, stream, bf16_peak):
             "learner_samples_per_s": 2 * wl.n_envs * wl.T / (ms * 1e-3), "kernel_ms": kern_ms,
             "roofline": {"bound": "tensor", "achieved": achieved, "peak": bf16_peak, "unit": "TFLOP/s",
                          "frac": achieved / bf16_peak, "flops_per_launch": flops}}
+
+
+def run_resample(aht, wl, pop, torch, stream, bf16_peak):
+    """The bench workload with a fresh teammate per episode (aht_rollout_resample): each
+    step regroups the 16384 envs by teammate (one grouping launch, one fused-rollout
+    launch), 2T launches per call.  ms per call from CUDA events (L2 scrubbed between
+    calls, outside the events)."""
+    ctx = aht.aht_create(wl.env, pop, wl.n_envs, wl.env_seed, has_value_head=list(wl.value_head),
+                         weight_dtype=aht.AHT_BF16, stream=stream)
+    traj = aht.traj_buffers(ctx, wl.T)
+    scrub = torch.empty(256 * 2 ** 20, dtype=torch.uint8, device="cuda")
+
+    def call():
+        aht.aht_rollout_resample(ctx, wl.ego_id, wl.pool, wl.T, traj, None, wl.gamma, wl.lam)
+
+    for _ in range(3):
+        call()
+    torch.cuda.synchronize()
+    K = 5
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    aht.aht_get_timing(ctx)
+    aht.aht_set_timing(ctx, True)
+    for k in range(K):
+        scrub.fill_(k & 0xFF)
+        ev[k][0].record(stream)
+        call()
+        ev[k][1].record(stream)
+    torch.cuda.synchronize()
+    aht.aht_set_timing(ctx, False)
+    kernel_ms, launches = aht.aht_get_timing(ctx)
+    aht.aht_sync(ctx)
+    ctx.close()
+    ms = sum(a.elapsed_time(b) for a, b in ev) / K
+    rollout_ms = kernel_ms / K           # the T fused-rollout launches of one call
+    ego = [wl.env.obs_dim, *wl.hidden, wl.env.n_actions + 1]
+    tm = [wl.env.obs_dim, *wl.hidden, wl.env.n_actions]
+    flops = wl.n_envs * wl.T * (mlp_flops(ego) + mlp_flops(tm)) + wl.n_envs * mlp_flops(ego)
+    achieved = flops / (rollout_ms * 1e-3) / 1e12
+    return {"workload": wl.name + "_per_episode_teammates", "ms_per_call": ms,
+            "env_steps_per_s": wl.n_envs * wl.T / (ms * 1e-3), "rollout_kernels_ms": rollout_ms,
+            "launches_per_call": 2 * wl.T + 1,
+            "roofline": {"bound": "tensor", "achieved": achieved, "peak": bf16_peak, "unit": "TFLOP/s",
+                         "frac": achieved / bf16_peak, "flops_per_call": flops}}
 
 
 PPO_FLOPS_PER_SAMPLE = 204032   # forward 84,736 + backward 119,296 (dW1, dW2, dh1, dW3, dh2)

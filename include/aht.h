@@ -171,6 +171,21 @@ typedef struct aht_traj {
 aht_status aht_rollout(aht_ctx* ctx, int32_t ego_id, const int32_t* pool, int32_t pool_size,
                        int32_t T, const aht_traj* out);
 
+/* PPO collection with per-episode teammates (Sec. 3: every episode pairs the ego with a
+ * teammate drawn from the training set).  The episode of env e that began at step s
+ * plays pool[floor(x * pool_size / 2^32)], x the first draw of counter (e, s, stream 5);
+ * the context carries per env the step its current episode began (aht_reset: 0; every
+ * auto-reset at step s' -- in any collection call or aht_step_forced -- sets s'; part of
+ * the checkpoint).  Each step regroups the envs by teammate (a grouping kernel, then one
+ * launch of the fused rollout over the groups' tiles), so this call runs 2T launches
+ * instead of 1; otherwise the step, the draws and the trajectory layout are those of
+ * aht_rollout.  out->teammate receives the teammate of the call's first step; teammates
+ * (device int32 [T][N], or NULL) the teammate of every step.  out->obs must be 4-byte
+ * aligned.  Same pool rules as aht_rollout (rule teammates on LBF tensor-core contexts). */
+aht_status aht_rollout_resample(aht_ctx* ctx, int32_t ego_id, const int32_t* pool,
+                                int32_t pool_size, int32_t T, const aht_traj* out,
+                                int32_t* teammates);
+
 /* IPPO collection (Sec. 3, the MARL baseline IPPO: both seats learn, each with its own
  * PPO of App. C).  Every env pairs policy0 in seat 0 with policy1 in seat 1; the call is
  * aht_rollout(ctx, policy0, {policy1}, 1, T, out0) -- the same draws, states and seat-0

@@ -26,7 +26,7 @@ EXPORTED = ["aht_create", "aht_destroy", "aht_reset", "aht_rollout", "aht_xplay_
             "aht_xplay_matrix_static", "aht_debug_tanh", "aht_debug_expire_wait",
             "aht_xp_stats", "aht_learner_create", "aht_learner_destroy", "aht_learner_n_params",
             "aht_ppo_update", "aht_ppo_grad", "aht_learner_get", "aht_learner_set",
-            "aht_learner_push", "aht_learner_sync", "aht_rollout_ippo"]
+            "aht_learner_push", "aht_learner_sync", "aht_rollout_ippo", "aht_rollout_resample"]
 
 
 class AhtError(RuntimeError):
@@ -109,6 +109,7 @@ def load() -> C.CDLL:
             L.aht_reset.argtypes = [vp, u64]
             L.aht_rollout.argtypes = [vp, i32, C.POINTER(i32), i32, i32, C.POINTER(Traj)]
             L.aht_rollout_ippo.argtypes = [vp, i32, i32, i32, C.POINTER(Traj), C.POINTER(Traj)]
+            L.aht_rollout_resample.argtypes = [vp, i32, C.POINTER(i32), i32, i32, C.POINTER(Traj), vp]
             L.aht_xplay_matrix.argtypes = [vp, C.POINTER(i32), i32, C.POINTER(i32), i32, i32, i32, C.POINTER(XplayOut)]
             L.aht_gae.argtypes = [vp, vp, vp, vp, i64, i32, C.c_float, C.c_float, vp, vp, vp]
             L.aht_xp_stats.argtypes = [vp, i32, i32, vp, C.POINTER(XpStatsOut), vp]
@@ -141,7 +142,8 @@ def load() -> C.CDLL:
             for f in ("aht_learner_create", "aht_ppo_update", "aht_ppo_grad", "aht_learner_get",
                       "aht_learner_set", "aht_learner_push", "aht_learner_sync"):
                 getattr(L, f).restype = C.c_int
-            for f in ("aht_create", "aht_reset", "aht_rollout", "aht_rollout_ippo", "aht_xplay_matrix",
+            for f in ("aht_create", "aht_reset", "aht_rollout", "aht_rollout_ippo", "aht_rollout_resample",
+                      "aht_xplay_matrix",
                       "aht_gae", "aht_xp_stats",
                       "aht_step_forced", "aht_policy_forward", "aht_get_state", "aht_set_state",
                       "aht_sync", "aht_set_policy", "aht_set_timing", "aht_get_timing"):
@@ -263,6 +265,16 @@ def aht_rollout(ctx: Context, ego_id, pool, T, traj: dict, gamma=0.99, lam=0.95)
     pool = list(pool)
     parr = (C.c_int32 * len(pool))(*pool)
     _check(load().aht_rollout(ctx.handle, ego_id, parr, len(pool), T, C.byref(t)))
+
+
+def aht_rollout_resample(ctx: Context, ego_id, pool, T, traj: dict, teammates=None,
+                         gamma=0.99, lam=0.95):
+    """PPO collection with a fresh teammate per episode; teammates: int32 [T][N] or None."""
+    t = _traj(ctx, T, traj, gamma, lam)
+    pool = list(pool)
+    parr = (C.c_int32 * len(pool))(*pool)
+    tm = _ptr(teammates, torch.int32, (T, ctx.n_envs), "teammates")
+    _check(load().aht_rollout_resample(ctx.handle, ego_id, parr, len(pool), T, C.byref(t), tm))
 
 
 def aht_rollout_ippo(ctx: Context, policy0, policy1, T, traj0: dict, traj1: dict,

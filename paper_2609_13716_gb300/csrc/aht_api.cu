@@ -100,6 +100,7 @@ struct aht_ctx {
   int4* tiles = nullptr;
   float* xp_returns = nullptr;
   float* last_value = nullptr;
+  uint32_t* ep_step = nullptr;  // [n_envs] step each env's current episode began
   uint32_t* status = nullptr;
   // tensor-core path (bf16 LBF populations that fit shared and tensor memory)
   int32_t weight_dtype = AHT_BF16;
@@ -559,6 +560,7 @@ void aht_destroy(aht_ctx* c) {
   DeviceGuard g(c->device);
   cudaStreamSynchronize(c->stream);
   cudaFree(c->state);
+  cudaFree(c->ep_step);
   cudaFree(c->weights);
   cudaFree(c->perm);
   cudaFree(c->tiles);
@@ -630,10 +632,13 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
   }
 
   const int words = c->ops.words();
-  c->max_tiles = group_tiles(n_envs, 4);  // the smallest tile any launch uses
+  // the smallest tile any launch uses, plus one partial tile per pool member of the
+  // per-episode grouping
+  c->max_tiles = group_tiles(n_envs, 4) + kMaxPool;
   struct Alloc { void** p; size_t bytes; };
   Alloc allocs[] = {
       {(void**)&c->state, (size_t)words * n_envs * 4},
+      {(void**)&c->ep_step, (size_t)n_envs * 4},
       {(void**)&c->weights, packed.size() * 4},
       {(void**)&c->perm, (size_t)n_envs * 4},
       {(void**)&c->tiles, (size_t)c->max_tiles * sizeof(int4)},
@@ -740,7 +745,7 @@ aht_status aht_reset(aht_ctx* c, uint64_t seed) {
   DeviceGuard g(c->device);
   c->seed = seed;
   c->step = 0;
-  ResetArgs a{batch_of(c), c->state, c->n_envs, 0u};
+  ResetArgs a{batch_of(c), c->state, c->n_envs, 0u, c->ep_step};
   AHT_CUDA(c->ops.reset(a, c->stream));
   return AHT_OK;
 }
@@ -801,6 +806,7 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
   a.ego = ego_id;
   a.step0 = (uint32_t)c->step;
   a.T = T;
+  a.ep_step = c->ep_step;
   a.traj = TrajPtrs{out->obs, out->actions, out->tm_actions, out->logp, out->values,
                     out->rewards, out->dones,
                     out->last_value ? out->last_value : (out->advantages ? c->last_value : nullptr)};
@@ -823,6 +829,7 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
     ta.T = T;
     ta.traj = a.traj;
     ta.traj1 = a.traj1;
+    ta.ep_step = c->ep_step;
     const int tk = timer_begin(c);
     AHT_CUDA(lbf_ppo_tc(ta, ga.max_tiles, c->tc_smem, c->stream));
     timer_end(c, tk);
@@ -845,6 +852,96 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
 aht_status aht_rollout(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t pool_size,
                        int32_t T, const aht_traj* out) {
   return rollout_common(c, ego_id, pool, pool_size, T, out, nullptr);
+}
+
+aht_status aht_rollout_resample(aht_ctx* c, int32_t ego_id, const int32_t* pool, int32_t pool_size,
+                                int32_t T, const aht_traj* out, int32_t* teammates) {
+  if (!c || !out) return fail(AHT_EINVAL, "ctx or out is NULL");
+  if (c->env.kind == AHT_HANABI || c->env.kind == AHT_MINI_HANABI)
+    return fail(AHT_EINVAL, "PPO collection needs a simultaneous-move env (LBF, Overcooked)");
+  if (ego_id < 0 || ego_id >= c->n_policies) return fail(AHT_EINVAL, "ego_id out of range");
+  if (!pool || pool_size < 1 || pool_size > kMaxPool) return fail(AHT_EINVAL, "pool_size must be in 1..256");
+  for (int k = 0; k < pool_size; ++k) {
+    if (pool[k] >= c->n_policies || pool[k] < -AHT_LBF_N_HEURISTICS) return fail(AHT_EINVAL, "pool id out of range");
+    if (pool[k] < 0 && !(c->env.kind == AHT_LBF && c->tc))
+      return fail(AHT_EINVAL, "heuristic teammates (negative ids) need an LBF context on the tensor-core path");
+  }
+  if (T < 1) return fail(AHT_EINVAL, "T must be >= 1");
+  if (c->step + T + 1 > (int64_t)UINT32_MAX) return fail(AHT_EINVAL, "step counter would exceed 2^32");
+  if (aht_status e = check_traj_out(out)) return e;
+  if (reinterpret_cast<uintptr_t>(out->obs) & 3u) return fail(AHT_EINVAL, "out->obs must be 4-byte aligned");
+  DeviceGuard g(c->device);
+  const int M = c->tc ? 128 : fit_rows(c, 128);
+  const int64_t N = c->n_envs;
+  const int od = c->env.obs_dim;
+  const int grid = resample_tiles(N, M, pool_size);
+  float* last_value = out->last_value ? out->last_value : (out->advantages ? c->last_value : nullptr);
+
+  ResampleGroupArgs ga{};
+  ga.key = batch_of(c).key;
+  ga.n_envs = N;
+  ga.ep_step = c->ep_step;
+  ga.pool_size = pool_size;
+  for (int k = 0; k < pool_size; ++k) ga.pool[k] = pool[k];
+  ga.M = M;
+  ga.max_tiles = grid;
+  ga.perm = c->perm;
+  ga.tiles = c->tiles;
+  // One launch per step: group the envs by their episode's teammate, then one step of
+  // every group (the envs that finish their episode draw their next teammate from the
+  // ep_step the step writes).
+  for (int t = 0; t < T; ++t) {
+    const int64_t o = (int64_t)t * N;
+    ga.teammate = teammates ? teammates + o : nullptr;
+    ga.teammate2 = t == 0 ? out->teammate : nullptr;
+    AHT_CUDA(launch_resample_group(ga, c->stream));
+    TrajPtrs tp{out->obs ? out->obs + o * od : nullptr, out->actions ? out->actions + o : nullptr,
+                out->tm_actions ? out->tm_actions + o : nullptr, out->logp ? out->logp + o : nullptr,
+                out->values ? out->values + o : nullptr, out->rewards ? out->rewards + o : nullptr,
+                out->dones ? out->dones + o : nullptr, t == T - 1 ? last_value : nullptr};
+    const uint32_t step = (uint32_t)(c->step + t);
+    if (c->tc) {
+      PpoTcArgs ta{};
+      ta.b = batch_of(c);
+      ta.tc = c->tcd;
+      ta.tcw = c->tcw;
+      ta.state = c->state;
+      ta.n_envs = N;
+      ta.perm = c->perm;
+      ta.tiles = c->tiles;
+      ta.ego = ego_id;
+      ta.step0 = step;
+      ta.T = 1;
+      ta.ep_step = c->ep_step;
+      ta.gather = 1;
+      ta.traj = tp;
+      const int tk = timer_begin(c);
+      AHT_CUDA(lbf_ppo_tc(ta, grid, c->tc_smem, c->stream));
+      timer_end(c, tk);
+    } else {
+      PpoArgs a{};
+      a.b = batch_of(c);
+      a.state = c->state;
+      a.n_envs = N;
+      a.perm = c->perm;
+      a.tiles = c->tiles;
+      a.M = M;
+      a.ego = ego_id;
+      a.step0 = step;
+      a.T = 1;
+      a.ep_step = c->ep_step;
+      a.traj = tp;
+      const size_t smem = smem_layout(M, c->mlp, c->ops.bytes()).total;
+      const int tk = timer_begin(c);
+      AHT_CUDA(c->ops.ppo(a, grid, smem, c->stream));
+      timer_end(c, tk);
+    }
+  }
+  if (out->advantages)
+    AHT_CUDA(launch_gae(out->rewards, out->values, out->dones, last_value, N, T, out->gamma,
+                        out->lambda, out->advantages, out->targets, c->stream));
+  c->step += T;
+  return AHT_OK;
 }
 
 aht_status aht_rollout_ippo(aht_ctx* c, int32_t policy0, int32_t policy1, int32_t T,
@@ -1040,7 +1137,7 @@ aht_status aht_step_forced(aht_ctx* c, const uint8_t* actions, const aht_step_ou
   if (c->step + 2 > (int64_t)UINT32_MAX) return fail(AHT_EINVAL, "step counter would exceed 2^32");
   DeviceGuard g(c->device);
   ForcedArgs a{batch_of(c), c->state, c->n_envs, (uint32_t)c->step, actions, out->rewards,
-               out->team, out->dones, out->obs};
+               out->team, out->dones, out->obs, c->ep_step};
   AHT_CUDA(c->ops.forced(a, c->stream));
   c->step += 1;
   return AHT_OK;
@@ -1063,8 +1160,8 @@ aht_status aht_policy_forward(aht_ctx* c, int32_t policy, const uint8_t* obs, in
 
 aht_status aht_get_state(aht_ctx* c, void* buf, size_t* bytes) {
   if (!c || !bytes) return fail(AHT_EINVAL, "NULL argument");
-  const size_t body = (size_t)c->ops.words() * c->n_envs * 4;
-  const size_t need = sizeof(StateHeader) + body;
+  const size_t body = (size_t)c->ops.words() * c->n_envs * 4, eps = (size_t)c->n_envs * 4;
+  const size_t need = sizeof(StateHeader) + body + eps;
   if (!buf) {
     *bytes = need;
     return AHT_OK;
@@ -1074,6 +1171,8 @@ aht_status aht_get_state(aht_ctx* c, void* buf, size_t* bytes) {
   StateHeader h{kStateMagic, (uint32_t)c->env.kind, (uint32_t)c->ops.words(), 0, c->n_envs, c->seed, c->step};
   std::memcpy(buf, &h, sizeof(h));
   AHT_CUDA(cudaMemcpyAsync(static_cast<uint8_t*>(buf) + sizeof(h), c->state, body, cudaMemcpyDeviceToHost, c->stream));
+  AHT_CUDA(cudaMemcpyAsync(static_cast<uint8_t*>(buf) + sizeof(h) + body, c->ep_step, eps,
+                           cudaMemcpyDeviceToHost, c->stream));
   AHT_CUDA(cudaStreamSynchronize(c->stream));
   *bytes = need;
   return AHT_OK;
@@ -1083,12 +1182,14 @@ aht_status aht_set_state(aht_ctx* c, const void* buf, size_t bytes) {
   if (!c || !buf || bytes < sizeof(StateHeader)) return fail(AHT_EINVAL, "NULL or short buffer");
   StateHeader h;
   std::memcpy(&h, buf, sizeof(h));
-  const size_t body = (size_t)c->ops.words() * c->n_envs * 4;
+  const size_t body = (size_t)c->ops.words() * c->n_envs * 4, eps = (size_t)c->n_envs * 4;
   if (h.magic != kStateMagic || h.kind != (uint32_t)c->env.kind || h.n_words != (uint32_t)c->ops.words() ||
-      h.n_envs != c->n_envs || bytes != sizeof(h) + body)
+      h.n_envs != c->n_envs || bytes != sizeof(h) + body + eps)
     return fail(AHT_EINVAL, "state buffer does not match this context");
   DeviceGuard g(c->device);
   AHT_CUDA(cudaMemcpyAsync(c->state, static_cast<const uint8_t*>(buf) + sizeof(h), body, cudaMemcpyHostToDevice, c->stream));
+  AHT_CUDA(cudaMemcpyAsync(c->ep_step, static_cast<const uint8_t*>(buf) + sizeof(h) + body, eps,
+                           cudaMemcpyHostToDevice, c->stream));
   AHT_CUDA(cudaStreamSynchronize(c->stream));
   c->seed = h.seed;
   c->step = h.step;

@@ -23,7 +23,8 @@ enum : uint32_t {
 
 // Philox streams (counter word 2).
 enum : uint32_t { kStreamAct0 = 0, kStreamAct1 = 1, kStreamReset = 2, kStreamTeammate = 3,
-                  kStreamPermute = 4 /* PPO minibatch permutation */ };
+                  kStreamPermute = 4 /* PPO minibatch permutation */,
+                  kStreamEpisodeTeammate = 5 /* per-episode teammate draw */ };
 
 struct DevEnv {
   int32_t kind, width, height, n_food, max_level, episode_len, cook_time, soup_reward;

@@ -34,6 +34,7 @@ struct PpoArgs {
   int32_t ego;
   uint32_t step0;
   int32_t T;
+  uint32_t* ep_step;     // [n_envs] step each env's episode began, set at every auto-reset
   TrajPtrs traj;
   TrajPtrs traj1;        // seat 1's learner trajectory (IPPO); all NULL otherwise: obs,
                          // actions = its own, tm_actions = seat 0's, logp, values,
@@ -82,6 +83,8 @@ struct PpoTcArgs {
   int32_t ego;
   uint32_t step0;
   int32_t T;
+  uint32_t* ep_step;     // as in PpoArgs
+  int32_t gather;        // rows are perm[tile.x + r] (per-episode teammates, T = 1)
   TrajPtrs traj;
   TrajPtrs traj1;        // as in PpoArgs
   TcXp xp;               // cross-play launches only
@@ -139,6 +142,23 @@ struct GroupArgs {
   int32_t* teammate;     // optional [n_envs]
 };
 
+// Per-episode teammates: env e plays pool[uniform_int(x, pool_size)] with x the first
+// draw of counter (e, ep_step[e], stream 5); perm lists the envs grouped by pool index,
+// tiles (perm offset, count, policy, -) cover each group in tiles of up to M envs.
+struct ResampleGroupArgs {
+  Key key;
+  int64_t n_envs;
+  const uint32_t* ep_step;
+  int32_t pool_size;
+  int32_t pool[kMaxPool];
+  int32_t M;
+  int32_t max_tiles;
+  int32_t* perm;
+  int4* tiles;
+  int32_t* teammate;     // optional [n_envs]: the policy each env plays at this step
+  int32_t* teammate2;    // optional second copy (the call's first step)
+};
+
 struct XpArgs {
   Batch b;
   int32_t n_ego, n_tm, P, max_steps;
@@ -161,6 +181,7 @@ struct ForcedArgs {
   float* team;
   uint8_t* dones;
   uint8_t* obs;            // [N][2][obs_dim]
+  uint32_t* ep_step;       // optional [N]
 };
 
 struct ResetArgs {
@@ -168,6 +189,7 @@ struct ResetArgs {
   uint32_t* state;
   int64_t n_envs;
   uint32_t step;
+  uint32_t* ep_step;       // optional [N]: set to step
 };
 
 struct PolicyArgs {
@@ -217,6 +239,8 @@ cudaError_t policy_set_smem_limit(size_t bytes);
 cudaError_t launch_tanh_probe(const float* x, float* y, int64_t n, cudaStream_t);
 cudaError_t launch_expire_wait(uint32_t* status, uint64_t limit_ns, cudaStream_t);
 int group_tiles(int64_t n_envs, int M);  // tile-table entries of a launch
+cudaError_t launch_resample_group(const ResampleGroupArgs&, cudaStream_t);
+int resample_tiles(int64_t n_envs, int M, int pool_size);  // tile-table entries, per-episode mode
 cudaError_t launch_gae(const float* r, const float* v, const uint8_t* d, const float* v_last,
                        int64_t n, int32_t T, float gamma, float lambda, float* adv, float* tgt,
                        cudaStream_t);

@@ -40,6 +40,60 @@ cudaError_t launch_group(const GroupArgs& a, cudaStream_t s) {
   return cudaGetLastError();
 }
 
+// ---- per-episode teammates: group the envs by their episode's pool index ----------------
+// One CTA: count the envs per pool index (shared-memory atomics), lay the groups out
+// back to back in perm and cut each into tiles of up to M envs, then scatter the env ids.
+// The order of the envs inside a group is not fixed (atomic slots); every row's result
+// depends on its env id only.
+__global__ void __launch_bounds__(1024) resample_group_kernel(const ResampleGroupArgs a) {
+  __shared__ int cnt[kMaxPool], base[kMaxPool], tile0[kMaxPool];
+  __shared__ int n_tiles;
+  const int tid = threadIdx.x;
+  const uint32_t P = (uint32_t)a.pool_size;
+  auto index_of = [&](int64_t e) {
+    return (int)uniform_int(draw0(a.key, (uint32_t)e, a.ep_step[e], kStreamEpisodeTeammate), P);
+  };
+  for (int k = tid; k < a.pool_size; k += blockDim.x) cnt[k] = 0;
+  __syncthreads();
+  for (int64_t e = tid; e < a.n_envs; e += blockDim.x) atomicAdd(&cnt[index_of(e)], 1);
+  __syncthreads();
+  if (tid == 0) {
+    int off = 0, t = 0;
+    for (int k = 0; k < a.pool_size; ++k) {
+      base[k] = off;
+      tile0[k] = t;
+      off += cnt[k];
+      t += (cnt[k] + a.M - 1) / a.M;
+    }
+    n_tiles = t;
+  }
+  __syncthreads();
+  for (int k = tid; k < a.pool_size; k += blockDim.x) {
+    const int n = cnt[k];
+    for (int j = 0; j * a.M < n; ++j)
+      a.tiles[tile0[k] + j] = make_int4(base[k] + j * a.M, min(a.M, n - j * a.M), a.pool[k], 0);
+  }
+  for (int j = n_tiles + tid; j < a.max_tiles; j += blockDim.x) a.tiles[j] = make_int4(0, 0, 0, 0);
+  __syncthreads();
+  for (int k = tid; k < a.pool_size; k += blockDim.x) cnt[k] = base[k];  // slot cursors
+  __syncthreads();
+  for (int64_t e = tid; e < a.n_envs; e += blockDim.x) {
+    const int k = index_of(e);
+    a.perm[atomicAdd(&cnt[k], 1)] = (int32_t)e;
+    if (a.teammate) a.teammate[e] = a.pool[k];
+    if (a.teammate2) a.teammate2[e] = a.pool[k];
+  }
+}
+
+int resample_tiles(int64_t n_envs, int M, int pool_size) {
+  return (int)((n_envs + M - 1) / M) + pool_size;
+}
+
+cudaError_t launch_resample_group(const ResampleGroupArgs& a, cudaStream_t s) {
+  resample_group_kernel<<<1, 1024, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
 // ---- GAE: one thread per env, reverse scan over T (time-major, coalesced across envs) --
 __global__ void gae_kernel(const float* __restrict__ r, const float* __restrict__ v,
                            const uint8_t* __restrict__ d, const float* __restrict__ v_last,

@@ -144,7 +144,10 @@ __global__ void __launch_bounds__(kThreads) ppo_kernel(const PpoArgs a) {
       if (a.traj1.tm_actions) a.traj1.tm_actions[o] = act[2 * i];
       if (a.traj1.rewards) a.traj1.rewards[o] = team;
       if (a.traj1.dones) a.traj1.dones[o] = (uint8_t)(done > 0);
-      if (done > 0) Env::reset(a.b.env, a.b.key, (uint32_t)env, gt + 1, st[i]);
+      if (done > 0) {
+        Env::reset(a.b.env, a.b.key, (uint32_t)env, gt + 1, st[i]);
+        if (a.ep_step) a.ep_step[env] = gt + 1;
+      }
     }
     __syncthreads();
   }
@@ -268,7 +271,10 @@ __global__ void forced_kernel(const ForcedArgs a) {
     done = 0;
     r0 = r1 = team = 0.0f;
   }
-  if (done) Env::reset(a.b.env, a.b.key, (uint32_t)e, a.step + 1, s);
+  if (done) {
+    Env::reset(a.b.env, a.b.key, (uint32_t)e, a.step + 1, s);
+    if (a.ep_step) a.ep_step[e] = a.step + 1;
+  }
   if (a.rewards) { a.rewards[2 * e] = r0; a.rewards[2 * e + 1] = r1; }
   if (a.team) a.team[e] = team;
   if (a.dones) a.dones[e] = (uint8_t)done;
@@ -288,6 +294,7 @@ __global__ void reset_kernel(const ResetArgs a) {
   State s;
   Env::reset(a.b.env, a.b.key, (uint32_t)e, a.step, s);
   store_state(a.state, a.n_envs, e, s);
+  if (a.ep_step) a.ep_step[e] = a.step;
 }
 
 template <class Env>

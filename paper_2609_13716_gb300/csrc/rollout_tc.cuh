@@ -42,10 +42,13 @@ constexpr int kTcPairBar = 2;            // ids 2..5: warps q and q + 4 (rows 32
 // of PPO collection.  kSplit: fp32 weights held as bf16 pairs W = W_hi + W_lo, L1 =
 // X W1_hi + X W1_lo and L2 = b2 + hi W2_hi + lo W2_hi + hi W2_lo (lo W2_lo is below
 // 2^-16 of the sum and left out).  kIppo (PPO collection only): seat 1 learns too, and
-// its trajectory goes to a.traj1.
-template <class Env, bool kXp, bool kSplit, bool kIppo>
+// its trajectory goes to a.traj1.  kGather (PPO collection, one step per launch): the
+// tile's rows are the envs perm[tile.x + r] (a group of envs whose episodes drew the
+// same teammate) instead of a contiguous range.
+template <class Env, bool kXp, bool kSplit, bool kIppo, bool kGather>
 __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a) {
   static_assert(!(kXp && kIppo), "seat-1 trajectories belong to PPO collection");
+  static_assert(!(kGather && (kXp || kIppo)), "gathered tiles are plain PPO collection");
   using State = typename Env::State;
   constexpr int NA = Env::kNumActions;
   extern __shared__ __align__(16) uint8_t smem[];  // no-swizzle operands need 16 B
@@ -76,6 +79,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   const bool tm_rule = tm_pol < 0;
   const TcDims& d = a.tc;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, half = (warp >> 2) & 1, row = tid & 127;
+  // env index of tile row r (r < count)
+  auto env_of = [&](int r) -> int64_t { return kGather ? (int64_t)a.perm[env0 + r] : env0 + r; };
+  const int64_t my_env = row < count ? env_of(row) : 0;
   const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
   const int64_t N = a.n_envs;
   const int od = a.b.env.obs_dim;
@@ -112,7 +118,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   for (int i = tid; i < 32 * od; i += blockDim.x) reinterpret_cast<uint32_t*>(sObs)[i] = 0u;
   if (tid < count) {
     if constexpr (kXp) Env::reset(a.b.env, a.b.key, (uint32_t)(env0 + tid), a.step0, st[tid]);
-    else load_state(a.state, N, env0 + tid, st[tid]);
+    else load_state(a.state, N, env_of(tid), st[tid]);
   }
   tc::fence_before_sync();
   __syncthreads();
@@ -295,8 +301,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     };
     // the tile's ego observation rows -> trajectory [t][env0 .. env0+count): one contiguous
     // block, written by one bulk (TMA) store when 16-byte aligned, else by all threads
-    const bool bulk_obs = !kXp && a.traj.obs && (count * od) % 16 == 0;
+    const bool bulk_obs = !kXp && !kGather && a.traj.obs && (count * od) % 16 == 0;
     auto copy_obs = [&](int t) {
+      if constexpr (kGather) {  // scattered rows: warps q and q + 4 store rows 32q .. 32q + 31
+        const int q = warp & 3, pt = half * 32 + lane;
+        for (int r = 32 * q; r < min(32 * q + 32, count); ++r) {
+          uint32_t* d32 = reinterpret_cast<uint32_t*>(a.traj.obs + ((int64_t)t * N + env_of(r)) * od);
+          const uint32_t* s32 = reinterpret_cast<const uint32_t*>(sObs + r * od);
+          for (int w = pt; w < cells; w += 64) d32[w] = s32[w];
+        }
+        return;
+      }
       uint8_t* dst = a.traj.obs + ((int64_t)t * N + env0) * od;
       const uint32_t bytes = (uint32_t)(count * od);
       if (bulk_obs && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
@@ -331,7 +346,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       const int first = (boot && !boot1) || tm_rule ? 0 : 1;
       const uint32_t par = (uint32_t)t & 1u, gt = a.step0 + (uint32_t)t;
       // this half's action draw (ego: warps 0-3, teammate: warps 4-7), ahead of its use
-      const float u_act = boot ? 0.0f : u01(draw0(a.b.key, (uint32_t)(env0 + row), gt, kStreamAct0 + half));
+      const float u_act = boot ? 0.0f : u01(draw0(a.b.key, (uint32_t)my_env, gt, kStreamAct0 + half));
       State s = st[row];  // register copy for this step (rows past count are never used)
 #pragma unroll 1
       for (int i = first; i >= 0; --i) {
@@ -371,10 +386,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       if (boot) {
         if (half == 0 && row < count && a.traj.last_value) {
           logits(0, z);
-          a.traj.last_value[env0 + row] = z[NA];
+          a.traj.last_value[my_env] = z[NA];
         } else if (kIppo && half == 1 && row < count && boot1) {
           logits(1, z);
-          a.traj1.last_value[env0 + row] = z[NA];
+          a.traj1.last_value[my_env] = z[NA];
         }
         break;
       }
@@ -390,7 +405,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         if (ag == 1) {
           act1s[row] = (uint8_t)act;
           if constexpr (kIppo) {
-            const int64_t o = (int64_t)t * N + env0 + row;
+            const int64_t o = (int64_t)t * N + my_env;
             if (a.traj1.logp) a.traj1.logp[o] = lp;
             if (a.traj1.values) a.traj1.values[o] = z[NA];
           }
@@ -421,7 +436,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         st[row] = s;
       } else if (!kXp && half == 0 && row < count) {
         const int act1 = act1s[row];
-        const int64_t env = env0 + row;
+        const int64_t env = my_env;
         float r0, r1, team;
         const int done = Env::step(a.b.env, s, act0, act1, r0, r1, team);
         const int64_t o = (int64_t)t * N + env;
@@ -437,7 +452,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
           if (a.traj1.rewards) a.traj1.rewards[o] = team;
           if (a.traj1.dones) a.traj1.dones[o] = (uint8_t)(done > 0);
         }
-        if (done > 0) Env::reset(a.b.env, a.b.key, (uint32_t)env, gt + 1, s);
+        if (done > 0) {
+          Env::reset(a.b.env, a.b.key, (uint32_t)env, gt + 1, s);
+          if (a.ep_step) a.ep_step[env] = gt + 1;
+        }
         st[row] = s;
       }
       if (tid == 0 && bulk_obs) tc::bulk_wait_read();  // the rows may be rebuilt
@@ -451,7 +469,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         a.xp.returns[env0 + tid] = Env::ret(st[tid]);
         if (a.xp.steps) a.xp.steps[env0 + tid] = nsteps;
       } else {
-        store_state(a.state, N, env0 + tid, st[tid]);
+        store_state(a.state, N, env_of(tid), st[tid]);
       }
     }
   }
@@ -474,18 +492,21 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
 
 template <class Env>
 struct LaunchTc {
-  template <bool kXp, bool kSplit, bool kIppo>
+  template <bool kXp, bool kSplit, bool kIppo, bool kGather = false>
   static cudaError_t run(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
-    cudaError_t e = cudaFuncSetAttribute(ppo_tc_kernel<Env, kXp, kSplit, kIppo>,
+    cudaError_t e = cudaFuncSetAttribute(ppo_tc_kernel<Env, kXp, kSplit, kIppo, kGather>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    ppo_tc_kernel<Env, kXp, kSplit, kIppo><<<grid, kTcThreads, smem, s>>>(a);
+    ppo_tc_kernel<Env, kXp, kSplit, kIppo, kGather><<<grid, kTcThreads, smem, s>>>(a);
     return cudaGetLastError();
   }
   static cudaError_t ppo(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
     const TrajPtrs& u = a.traj1;
     const bool ippo = u.obs || u.actions || u.tm_actions || u.logp || u.values || u.rewards ||
                       u.dones || u.last_value;
+    if (a.gather)
+      return a.tc.split ? run<false, true, false, true>(a, grid, smem, s)
+                        : run<false, false, false, true>(a, grid, smem, s);
     if (ippo)
       return a.tc.split ? run<false, true, true>(a, grid, smem, s) : run<false, false, true>(a, grid, smem, s);
     return a.tc.split ? run<false, true, false>(a, grid, smem, s) : run<false, false, false>(a, grid, smem, s);

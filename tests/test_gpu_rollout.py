@@ -19,12 +19,17 @@ from gpu_util import CDF_MARGIN, GAE_REL, close, make_ctx, np_, oracle_of, requi
 pytestmark = pytest.mark.gpu
 
 
-def check_rollout(wl, pop_np, traj, states, seed, step0, T, ego, pool, env_ids=None):
+def check_rollout(wl, pop_np, traj, states, seed, step0, T, ego, pool, env_ids=None, ep_step=None,
+                  resample=False, teammates=None):
+    """Replays the GPU's applied actions in the oracle and compares.  ep_step / resample:
+    per-episode teammates (teammates: the GPU's per-step teammate ids, compared exactly)."""
     d, pols = oracle_of(wl.env, pop_np)
     sel = slice(None) if env_ids is None else env_ids
     acts = np.stack([np_(traj["actions"])[:, sel], np_(traj["tm_actions"])[:, sel]], -1)
     ref = O.rollout(d, pols, seed, states, step0, T, ego, pool, forced=acts, n_threads=8,
-                    env_ids=env_ids)
+                    env_ids=env_ids, ep_step=ep_step, resample=resample)
+    if teammates is not None:
+        assert np.array_equal(np_(teammates)[:, sel], ref["teammates_t"]), "per-step teammates"
     assert ref["rc"] == 0
     assert np.array_equal(np_(traj["teammate"])[sel], ref["teammate"]), "teammate draw"
     if traj.get("obs") is not None:
