@@ -101,6 +101,8 @@ struct aht_ctx {
   float* xp_returns = nullptr;
   float* last_value = nullptr;
   uint32_t* ep_step = nullptr;  // [n_envs] step each env's current episode began
+  uint8_t* rs_kidx = nullptr;   // [2][align_up(n_envs, 16)] per-episode pool index by step parity
+  int32_t* rs_hist = nullptr;   // [3][kMaxPool] envs per pool index, by step mod 3
   uint32_t* status = nullptr;
   // tensor-core path (bf16 LBF populations that fit shared and tensor memory)
   int32_t weight_dtype = AHT_BF16;
@@ -561,6 +563,8 @@ void aht_destroy(aht_ctx* c) {
   cudaStreamSynchronize(c->stream);
   cudaFree(c->state);
   cudaFree(c->ep_step);
+  cudaFree(c->rs_kidx);
+  cudaFree(c->rs_hist);
   cudaFree(c->weights);
   cudaFree(c->perm);
   cudaFree(c->tiles);
@@ -639,6 +643,8 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
   Alloc allocs[] = {
       {(void**)&c->state, (size_t)words * n_envs * 4},
       {(void**)&c->ep_step, (size_t)n_envs * 4},
+      {(void**)&c->rs_kidx, 2 * (size_t)align_up(n_envs, 16)},
+      {(void**)&c->rs_hist, 3 * (size_t)kMaxPool * 4},
       {(void**)&c->weights, packed.size() * 4},
       {(void**)&c->perm, (size_t)n_envs * 4},
       {(void**)&c->tiles, (size_t)c->max_tiles * sizeof(int4)},
@@ -877,6 +883,53 @@ aht_status aht_rollout_resample(aht_ctx* c, int32_t ego_id, const int32_t* pool,
   const int grid = resample_tiles(N, M, pool_size);
   float* last_value = out->last_value ? out->last_value : (out->advantages ? c->last_value : nullptr);
 
+  if (c->tc) {
+    // Tensor-core path: each step's launch groups its own rows (TcGather).
+    const size_t smem = c->tc_smem + kTcGatherScratch;
+    if (smem > c->smem_optin) return fail(AHT_EINVAL, "no shared memory left for the per-episode grouping");
+    const size_t ks = (size_t)align_up(N, 16);
+    AHT_CUDA(cudaMemsetAsync(c->rs_hist, 0, 3 * (size_t)kMaxPool * 4, c->stream));
+    AHT_CUDA(launch_resample_init(batch_of(c).key, N, c->ep_step, pool_size, c->rs_kidx, c->rs_hist,
+                                  c->stream));
+    PpoTcArgs ta{};
+    ta.b = batch_of(c);
+    ta.tc = c->tcd;
+    ta.tcw = c->tcw;
+    ta.state = c->state;
+    ta.n_envs = N;
+    ta.ego = ego_id;
+    ta.T = 1;
+    ta.ep_step = c->ep_step;
+    ta.gather = 1;
+    ta.g.scratch_off = (uint32_t)c->tc_smem;
+    ta.g.pool_size = pool_size;
+    for (int k = 0; k < pool_size; ++k) ta.g.pool[k] = pool[k];
+    for (int t = 0; t < T; ++t) {
+      const int64_t o = (int64_t)t * N;
+      ta.step0 = (uint32_t)(c->step + t);
+      ta.traj = TrajPtrs{out->obs ? out->obs + o * od : nullptr, out->actions ? out->actions + o : nullptr,
+                         out->tm_actions ? out->tm_actions + o : nullptr, out->logp ? out->logp + o : nullptr,
+                         out->values ? out->values + o : nullptr, out->rewards ? out->rewards + o : nullptr,
+                         out->dones ? out->dones + o : nullptr, t == T - 1 ? last_value : nullptr};
+      ta.g.kidx_cur = c->rs_kidx + (t & 1) * ks;
+      ta.g.kidx_next = c->rs_kidx + ((t + 1) & 1) * ks;
+      ta.g.hist_cur = c->rs_hist + (t % 3) * kMaxPool;
+      ta.g.hist_next = c->rs_hist + ((t + 1) % 3) * kMaxPool;
+      ta.g.hist_zero = c->rs_hist + ((t + 2) % 3) * kMaxPool;
+      ta.g.teammate = teammates ? teammates + o : nullptr;
+      ta.g.teammate2 = t == 0 ? out->teammate : nullptr;
+      const int tk = timer_begin(c);
+      AHT_CUDA(lbf_ppo_tc(ta, resample_tiles(N, 128, pool_size), smem, c->stream));
+      timer_end(c, tk);
+    }
+    if (out->advantages)
+      AHT_CUDA(launch_gae(out->rewards, out->values, out->dones, last_value, N, T, out->gamma,
+                          out->lambda, out->advantages, out->targets, c->stream));
+    c->step += T;
+    return AHT_OK;
+  }
+
+  // CUDA-core path: a grouping launch, then one rollout launch over the groups' tiles.
   ResampleGroupArgs ga{};
   ga.key = batch_of(c).key;
   ga.n_envs = N;
@@ -900,25 +953,7 @@ aht_status aht_rollout_resample(aht_ctx* c, int32_t ego_id, const int32_t* pool,
                 out->values ? out->values + o : nullptr, out->rewards ? out->rewards + o : nullptr,
                 out->dones ? out->dones + o : nullptr, t == T - 1 ? last_value : nullptr};
     const uint32_t step = (uint32_t)(c->step + t);
-    if (c->tc) {
-      PpoTcArgs ta{};
-      ta.b = batch_of(c);
-      ta.tc = c->tcd;
-      ta.tcw = c->tcw;
-      ta.state = c->state;
-      ta.n_envs = N;
-      ta.perm = c->perm;
-      ta.tiles = c->tiles;
-      ta.ego = ego_id;
-      ta.step0 = step;
-      ta.T = 1;
-      ta.ep_step = c->ep_step;
-      ta.gather = 1;
-      ta.traj = tp;
-      const int tk = timer_begin(c);
-      AHT_CUDA(lbf_ppo_tc(ta, grid, c->tc_smem, c->stream));
-      timer_end(c, tk);
-    } else {
+    {
       PpoArgs a{};
       a.b = batch_of(c);
       a.state = c->state;

@@ -19,6 +19,7 @@ enum : uint32_t {
   kStatusActorMismatch = 2u,
   kStatusBadPolicy = 4u,
   kStatusTimeout = 8u,   // a bounded device wait gave up
+  kStatusGrouping = 16u, // a per-episode tile did not find all its envs (tile skipped)
 };
 
 // Philox streams (counter word 2).

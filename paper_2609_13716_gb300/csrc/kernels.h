@@ -72,6 +72,27 @@ struct TcXp {
   uint8_t* actions;        // optional [max_steps][n_total][2], pre-filled with 255
 };
 
+// Per-episode teammates on the tensor-core rollout, one launch per step.  Each env
+// carries the pool index of its episode's teammate (kidx, double-buffered by step) and
+// the launch carries the envs per index (hist, triple-buffered).  CTA j takes tile j of
+// the groups laid out in pool-index order (each group cut into tiles of up to 128 envs
+// in env order), finds its envs by a rank scan of kidx, steps them, writes each env's
+// index for the next step (a new draw after an auto-reset) and adds the next step's
+// counts; CTA 0 zeroes the buffer the step after next will count into.
+struct TcGather {
+  const uint8_t* kidx_cur;  // [N] pool index per env at this step (16-byte aligned)
+  uint8_t* kidx_next;       // [N] at the next step
+  const int32_t* hist_cur;  // [pool_size] envs per index at this step
+  int32_t* hist_next;       // [pool_size] accumulated for the next step (zero on entry)
+  int32_t* hist_zero;       // [pool_size] zeroed by CTA 0
+  int32_t* teammate;        // optional [N]: policy of each env at this step
+  int32_t* teammate2;       // optional second copy
+  uint32_t scratch_off;     // dynamic shared-memory offset of the scan scratch
+  int32_t pool_size;
+  int32_t pool[kMaxPool];
+};
+constexpr uint32_t kTcGatherScratch = 128 * 4 + 16 * 4;  // row envs, warp totals, selection
+
 struct PpoTcArgs {
   Batch b;
   TcDims tc;
@@ -84,10 +105,11 @@ struct PpoTcArgs {
   uint32_t step0;
   int32_t T;
   uint32_t* ep_step;     // as in PpoArgs
-  int32_t gather;        // rows are perm[tile.x + r] (per-episode teammates, T = 1)
+  int32_t gather;        // per-episode teammates, one step per launch (see TcGather)
   TrajPtrs traj;
   TrajPtrs traj1;        // as in PpoArgs
   TcXp xp;               // cross-play launches only
+  TcGather g;            // gather launches only
 };
 
 // Per-policy block of the streamed tensor-core path (binary observations, hidden width H
@@ -241,6 +263,9 @@ cudaError_t launch_expire_wait(uint32_t* status, uint64_t limit_ns, cudaStream_t
 int group_tiles(int64_t n_envs, int M);  // tile-table entries of a launch
 cudaError_t launch_resample_group(const ResampleGroupArgs&, cudaStream_t);
 int resample_tiles(int64_t n_envs, int M, int pool_size);  // tile-table entries, per-episode mode
+// kidx[e] = pool index of env e's episode teammate, hist[k] += envs with index k
+cudaError_t launch_resample_init(const Key& key, int64_t n_envs, const uint32_t* ep_step,
+                                 int32_t pool_size, uint8_t* kidx, int32_t* hist, cudaStream_t);
 cudaError_t launch_gae(const float* r, const float* v, const uint8_t* d, const float* v_last,
                        int64_t n, int32_t T, float gamma, float lambda, float* adv, float* tgt,
                        cudaStream_t);

@@ -85,6 +85,29 @@ __global__ void __launch_bounds__(1024) resample_group_kernel(const ResampleGrou
   }
 }
 
+__global__ void resample_init_kernel(const Key key, int64_t n, const uint32_t* __restrict__ ep_step,
+                                     uint32_t P, uint8_t* __restrict__ kidx, int32_t* __restrict__ hist) {
+  __shared__ int cnt[kMaxPool];
+  for (int k = threadIdx.x; k < (int)P; k += blockDim.x) cnt[k] = 0;
+  __syncthreads();
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
+    const uint32_t k = uniform_int(draw0(key, (uint32_t)e, ep_step[e], kStreamEpisodeTeammate), P);
+    kidx[e] = (uint8_t)k;
+    atomicAdd(&cnt[k], 1);
+  }
+  __syncthreads();
+  for (int k = threadIdx.x; k < (int)P; k += blockDim.x)
+    if (cnt[k]) atomicAdd(&hist[k], cnt[k]);
+}
+
+cudaError_t launch_resample_init(const Key& key, int64_t n_envs, const uint32_t* ep_step,
+                                 int32_t pool_size, uint8_t* kidx, int32_t* hist, cudaStream_t s) {
+  int64_t blocks = (n_envs + 255) / 256;
+  if (blocks > 148) blocks = 148;
+  resample_init_kernel<<<(unsigned)blocks, 256, 0, s>>>(key, n_envs, ep_step, (uint32_t)pool_size, kidx, hist);
+  return cudaGetLastError();
+}
+
 int resample_tiles(int64_t n_envs, int M, int pool_size) {
   return (int)((n_envs + M - 1) / M) + pool_size;
 }

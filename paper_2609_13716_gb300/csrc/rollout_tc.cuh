@@ -61,12 +61,108 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
 
   int64_t env0;
   int count, ego_pol, tm_pol;
+  int g_k = 0;                                      // gather: the tile's pool index
+  int32_t* const rowenv = kGather ? reinterpret_cast<int32_t*>(smem + a.g.scratch_off) : nullptr;
   if constexpr (kXp) {
     const int pair = blockIdx.x / a.xp.tpp, chunk = blockIdx.x - pair * a.xp.tpp;
     env0 = (int64_t)pair * a.xp.P + 128 * chunk;
     count = min(128, a.xp.P - 128 * chunk);
     ego_pol = a.xp.ego_ids[pair / a.xp.n_tm];
     tm_pol = a.xp.tm_ids[pair % a.xp.n_tm];
+  } else if constexpr (kGather) {
+    // Tile blockIdx.x of the groups in pool-index order: group k holds hist_cur[k] envs,
+    // cut into tiles of up to 128 in env order.  Rows are found by a rank scan of kidx:
+    // each thread counts its contiguous chunk's envs of group k, an exclusive scan gives
+    // the chunk's first rank, and the envs of ranks [r0, r0 + count) become rows.
+    int* wsum = reinterpret_cast<int*>(rowenv + 128);  // [0, 9) warp totals, [10, 13) selection
+    const int t0 = threadIdx.x, w0 = t0 >> 5, l0 = t0 & 31;
+    if (blockIdx.x == 0)
+      for (int k = t0; k < a.g.pool_size; k += blockDim.x) a.g.hist_zero[k] = 0;
+    if (t0 < 128) rowenv[t0] = -1;
+    if (t0 == 0) {
+      int cum = 0, ks = -1, r0 = 0, cnt = 0;
+      for (int k = 0; k < a.g.pool_size; ++k) {
+        const int h = a.g.hist_cur[k], nt = (h + 127) >> 7;
+        if (ks < 0 && (int)blockIdx.x < cum + nt) {
+          ks = k;
+          r0 = ((int)blockIdx.x - cum) * 128;
+          cnt = min(128, h - r0);
+        }
+        cum += nt;
+      }
+      wsum[10] = ks;
+      wsum[11] = r0;
+      wsum[12] = ks < 0 ? 0 : cnt;
+    }
+    __syncthreads();
+    g_k = wsum[10];
+    const int r0 = wsum[11];
+    count = wsum[12];
+    env0 = 0;
+    ego_pol = a.ego;
+    tm_pol = g_k < 0 ? 0 : a.g.pool[g_k];
+    if (count > 0) {  // block-uniform
+      const int64_t n = a.n_envs, nthr = blockDim.x;
+      const int64_t C = (((n + nthr - 1) / nthr) + 15) & ~(int64_t)15;  // bytes per thread
+      const int64_t b0 = t0 * C, b1 = min(n, b0 + C);
+      const uint8_t* kx = a.g.kidx_cur;
+      const uint32_t kk = 0x01010101u * (uint32_t)g_k;
+      // 16 indices of [e, e + 16) as match bytes (0xFF where kidx == g_k, 0 past b1);
+      // b0 is a multiple of 16 and kidx is 16-byte aligned
+      auto matches = [&](int64_t e) {
+        uint4 m;
+        if (e + 16 <= b1) {
+          const uint4 v = __ldg(reinterpret_cast<const uint4*>(kx + e));
+          m = make_uint4(__vcmpeq4(v.x, kk), __vcmpeq4(v.y, kk), __vcmpeq4(v.z, kk), __vcmpeq4(v.w, kk));
+        } else {
+          uint32_t w[4] = {0u, 0u, 0u, 0u};
+          for (int64_t f = e; f < b1; ++f)
+            if (kx[f] == (uint8_t)g_k) w[(f - e) >> 2] |= 0xFFu << (8 * ((f - e) & 3));
+          m = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+        return m;
+      };
+      int c = 0;
+#pragma unroll 4
+      for (int64_t e = b0; e < b1; e += 16) {
+        const uint4 m = matches(e);
+        c += (__popc(m.x) + __popc(m.y) + __popc(m.z) + __popc(m.w)) >> 3;
+      }
+      int incl = c;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (l0 >= o) incl += y;
+      }
+      if (l0 == 31) wsum[w0] = incl;
+      __syncthreads();
+      int rank = incl - c;
+      for (int w = 0; w < w0; ++w) rank += wsum[w];
+      if (c > 0 && rank < r0 + count && rank + c > r0) {
+#pragma unroll 4
+        for (int64_t e = b0; e < b1; e += 16) {
+          const uint4 m = matches(e);
+          const uint32_t mw[4] = {m.x, m.y, m.z, m.w};
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            uint32_t bits = mw[q] & 0x80808080u;  // one bit per matching byte
+            while (bits) {
+              const int byte = (__ffs(bits) - 1) >> 3;
+              bits &= bits - 1;
+              if (rank >= r0 && rank < r0 + count) rowenv[rank - r0] = (int32_t)(e + 4 * q + byte);
+              ++rank;
+            }
+          }
+        }
+      }
+    }
+    __syncthreads();
+    // every row must have found its env (the counts and the indices agree by
+    // construction); otherwise the tile is skipped and the status word says so
+    if (!__syncthreads_and(t0 >= count || (rowenv[t0] >= 0 && rowenv[t0] < a.n_envs))) {
+      if (t0 == 0) atomicOr(a.b.status, kStatusGrouping);
+      count = 0;
+    }
   } else {
     const int4 tile = a.tiles[blockIdx.x];
     env0 = tile.x;
@@ -80,7 +176,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   const TcDims& d = a.tc;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, half = (warp >> 2) & 1, row = tid & 127;
   // env index of tile row r (r < count)
-  auto env_of = [&](int r) -> int64_t { return kGather ? (int64_t)a.perm[env0 + r] : env0 + r; };
+  auto env_of = [&](int r) -> int64_t { return kGather ? (int64_t)rowenv[r] : env0 + r; };
   const int64_t my_env = row < count ? env_of(row) : 0;
   const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
   const int64_t N = a.n_envs;
@@ -303,11 +399,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     // block, written by one bulk (TMA) store when 16-byte aligned, else by all threads
     const bool bulk_obs = !kXp && !kGather && a.traj.obs && (count * od) % 16 == 0;
     auto copy_obs = [&](int t) {
-      if constexpr (kGather) {  // scattered rows: warps q and q + 4 store rows 32q .. 32q + 31
-        const int q = warp & 3, pt = half * 32 + lane;
-        for (int r = 32 * q; r < min(32 * q + 32, count); ++r) {
-          uint32_t* d32 = reinterpret_cast<uint32_t*>(a.traj.obs + ((int64_t)t * N + env_of(r)) * od);
-          const uint32_t* s32 = reinterpret_cast<const uint32_t*>(sObs + r * od);
+      if constexpr (kGather) {
+        // scattered rows: warps q and q + 4 store rows 32q .. 32q + 31, one row at a time
+        // with consecutive words; lane i of either warp holds the env of row 32q + i
+        const int q = warp & 3, pt = half * 32 + lane, n = min(32, count - 32 * q);
+        for (int i = 0; i < n; ++i) {
+          const int env = __shfl_sync(0xFFFFFFFFu, (int)my_env, i);
+          uint32_t* d32 = reinterpret_cast<uint32_t*>(a.traj.obs + ((int64_t)t * N + env) * od);
+          const uint32_t* s32 = reinterpret_cast<const uint32_t*>(sObs + (32 * q + i) * od);
           for (int w = pt; w < cells; w += 64) d32[w] = s32[w];
         }
         return;
@@ -394,6 +493,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         break;
       }
       int act0 = 0;
+      bool stayed = false;  // gather: the row's env keeps its teammate for the next step
       float lp0 = 0.f, val0 = 0.f;
       if (row < count && half == 1 && tm_rule) {
         act1s[row] = (uint8_t)Env::heuristic(a.b.env, st[row], -1 - tm_pol);  // st[row] == s here
@@ -437,6 +537,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       } else if (!kXp && half == 0 && row < count) {
         const int act1 = act1s[row];
         const int64_t env = my_env;
+        if constexpr (kGather) {
+          if (a.g.teammate) a.g.teammate[env] = tm_pol;
+          if (a.g.teammate2) a.g.teammate2[env] = tm_pol;
+        }
         float r0, r1, team;
         const int done = Env::step(a.b.env, s, act0, act1, r0, r1, team);
         const int64_t o = (int64_t)t * N + env;
@@ -456,7 +560,23 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
           Env::reset(a.b.env, a.b.key, (uint32_t)env, gt + 1, s);
           if (a.ep_step) a.ep_step[env] = gt + 1;
         }
+        if constexpr (kGather) {  // the next step's pool index: a new episode draws again
+          int kn = g_k;
+          if (done > 0) {
+            kn = (int)uniform_int(draw0(a.b.key, (uint32_t)env, gt + 1, kStreamEpisodeTeammate),
+                                  (uint32_t)a.g.pool_size);
+            atomicAdd(&a.g.hist_next[kn], 1);
+          }
+          a.g.kidx_next[env] = (uint8_t)kn;
+          stayed = done <= 0;
+        }
         st[row] = s;
+      }
+      if constexpr (kGather) {
+        if (half == 0) {  // warps 0-3: one count per warp of the rows that keep the teammate
+          const unsigned m = __ballot_sync(0xFFFFFFFFu, stayed);
+          if (lane == 0 && m) atomicAdd(&a.g.hist_next[g_k], __popc(m));
+        }
       }
       if (tid == 0 && bulk_obs) tc::bulk_wait_read();  // the rows may be rebuilt
       if (sync_or()) break;
