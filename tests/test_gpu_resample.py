@@ -129,3 +129,30 @@ def test_full_size_16384x128_sampled_envs():
                            wl.ego_id, list(wl.pool), env_ids=ids)
     # every pool member is met, and each env changes teammate at its episode ends only
     assert set(np.unique(tms)) == set(wl.pool)
+
+
+@pytest.mark.parametrize("N,pool_size", [(1, 3), (131, 256), (300, 1)])
+def test_edge_sizes_and_pools(N, pool_size):
+    """One env; a ragged batch with a 256-entry pool (more groups than envs, most of them
+    empty, indices up to 255); a one-member pool."""
+    require_gpu()
+    wl = short_lbf(W.WORKLOADS["lbf7x7_ppo_16384x128"], 6)
+    ctx, pop_np = make_ctx(wl, N)
+    d, _ = oracle_of(wl.env, pop_np)
+    st = O.reset_all(d, wl.env_seed, N)
+    pool = [1 + (k * 7) % 32 for k in range(pool_size)]
+    ep = np.zeros(N, np.uint32)
+    for call in range(2):
+        run_and_check(wl, ctx, pop_np, st, ep, call * 17, 17, 0, pool)
+
+
+def test_rule_teammates_only():
+    require_gpu()
+    wl = short_lbf(W.WORKLOADS["lbf7x7_ppo_16384x128"], 10)
+    N = 257
+    ctx, pop_np = make_ctx(wl, N)
+    d, _ = oracle_of(wl.env, pop_np)
+    st = O.reset_all(d, wl.env_seed, N)
+    pool = [O.heuristic_id(n) for n in O.LBF_HEURISTICS]
+    _, tms = run_and_check(wl, ctx, pop_np, st, np.zeros(N, np.uint32), 0, 40, 0, pool)
+    assert (tms < 0).all()
