@@ -628,6 +628,12 @@ def run_xplay(args, aht, W, torch, bf16_peak, names=XPLAY_WORKLOADS, bf16_sustai
                                   "frac_of_sustained": tflops / bf16_sustained,
                                   "flops_per_matrix": flops},
                      "xp_stats_us": stats_us}
+        if wl.env.kind == W.LBF and wl.env.obs_dim > 255:
+            # the CUDA-core path: its first layer adds only the observation's changed
+            # features to a per-policy constant, so these are dense-equivalent FLOPs
+            res[name]["roofline"]["flops_basis"] = (
+                "dense-equivalent MLP FLOPs; the CUDA-core kernel's first layer skips the "
+                "observation's unchanged features")
     return res
 
 

@@ -185,7 +185,7 @@ aht_status check_env(const aht_env_desc* d, DevEnv* out) {
   return AHT_OK;
 }
 
-MlpDims make_dims(int K, int H0, int H1, int NA) {
+MlpDims make_dims(int K, int H0, int H1, int NA, bool sparse) {
   MlpDims m{};
   m.K = K;
   m.KP = (int)align_up(K, 16);
@@ -200,6 +200,8 @@ MlpDims make_dims(int K, int H0, int H1, int NA) {
   m.ob2 = o; o += H1;
   m.oW3 = o; o += (int64_t)H1 * m.NOP;
   m.ob3 = o; o += m.NOP;
+  m.sparse = sparse ? 1 : 0;
+  m.oC = o; o += sparse ? H0 : 0;
   m.stride = align_up(o, 4);
   return m;
 }
@@ -247,6 +249,17 @@ aht_status pack_policy(const MlpDims& m, const void* const* W, const void* const
         dst[oW[l] + (int64_t)k * cols[l] + n] = to_f32(src, (int64_t)n * ins[l] + k, dtype);
     if (!host_view(b[l], (size_t)outs[l] * esz, &src)) return fail(AHT_ECUDA, "copying biases failed");
     for (int n = 0; n < outs[l]; ++n) dst[ob[l] + n] = to_f32(src, n, dtype);
+  }
+  if (m.sparse) {  // c = b1 + W1 x_default in fp64, rounded once
+    for (int n = 0; n < m.H0; ++n) {
+      double acc = dst[m.ob1 + n];
+      for (int w = 0; w < m.K / 4; ++w)
+        for (int kk = 0; kk < 4; ++kk) {
+          const uint32_t x = (kSparseDefaultWord >> (8 * kk)) & 0xFFu;
+          if (x) acc += (double)x * dst[m.oW1 + (int64_t)(4 * w + kk) * m.H0 + n];
+        }
+      dst[m.oC + n] = (float)acc;
+    }
   }
   return AHT_OK;
 }
@@ -613,7 +626,7 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
   c->seed = seed;
   c->step = 0;
   c->stream = (cudaStream_t)cuda_stream;
-  c->mlp = make_dims(env.obs_dim, pop->hidden0, pop->hidden1, env.n_actions);
+  c->mlp = make_dims(env.obs_dim, pop->hidden0, pop->hidden1, env.n_actions, env.kind == AHT_LBF);
   auto bail = [&](aht_status s, const std::string& m) {
     aht_destroy(c);
     return fail(s, m);

@@ -38,7 +38,14 @@ struct MlpDims {
   int32_t K, KP, H0, H1, NA, NOP;
   int64_t stride;  // floats per policy
   int64_t oW1, ob1, oW2, ob2, oW3, ob3;
+  // Observations that are a fixed pattern (LBF: every cell word 0x01000000, the open-cell
+  // feature set) plus a few changed bytes: the first layer is c + sum over the changed
+  // features, c = b1 + W1 x_default kept per policy at oC.
+  int32_t sparse;
+  int64_t oC;
 };
+constexpr uint32_t kSparseDefaultWord = 0x01000000u;
+constexpr int kSparseCap = 32;  // list entries per row: a count and up to 31 changed features
 
 struct Key {
   uint32_t k0, k1;

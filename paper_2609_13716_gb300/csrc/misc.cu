@@ -290,7 +290,8 @@ __global__ void __launch_bounds__(kThreads) policy_kernel(const PolicyArgs a) {
     X[idx] = (i < count && k < od) ? a.obs[(r0 + i) * od + k] : (uint8_t)0;
   }
   __syncthreads();
-  mlp_tile(a.b.weights + (int64_t)a.policy * m.stride, m, X, H1, H2, Z, M);
+  mlp_tile(a.b.weights + (int64_t)a.policy * m.stride, m, X, H1, H2, Z, M,
+           reinterpret_cast<uint32_t*>(smem + L.list), count);
   const int no = m.NA + 1;
   for (int idx = threadIdx.x; idx < count * no; idx += blockDim.x) {
     const int i = idx / no, c = idx - i * no;

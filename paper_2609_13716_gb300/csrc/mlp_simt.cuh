@@ -69,12 +69,95 @@ __device__ __forceinline__ void dense_tile(const void* __restrict__ in, int in_l
   }
 }
 
-// Whole policy forward for an M-row tile: X u8 [M][KP] -> Z f32 [M][NOP].
+// First layer for m.sparse observations: each row is the default pattern (every word
+// kSparseDefaultWord) except a few bytes, so W1 o + b1 = c + sum over the changed
+// features f of (o_f - default_f) W1[:, f], with c = b1 + W1 x_default packed per policy.
+// One warp per row lists the changed features in increasing order (list[r][0] = count,
+// entries (f << 8) | (delta & 0xFF)); then every output adds its row's entries in that
+// order, so the result is deterministic.  A row with more changed bytes than the list
+// holds (any observation that is not of the pattern) takes the dense sum b1 + W1 o.
+// Rows from `live` on are not computed.
+__device__ __forceinline__ void sparse_l1_tile(const uint8_t* X, const MlpDims& m, int live,
+                                               const float* __restrict__ Wt, const float* __restrict__ b1,
+                                               const float* __restrict__ c, uint32_t* list, float* H1) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  const int words = m.K >> 2;
+  for (int r = warp; r < live; r += nw) {
+    const uint32_t* row = reinterpret_cast<const uint32_t*>(X + r * m.KP);
+    uint32_t* L = list + r * kSparseCap;
+    int base = 0;
+    for (int w0 = 0; w0 < words; w0 += 32) {
+      const int wi = w0 + lane;
+      const uint32_t v = wi < words ? row[wi] : kSparseDefaultWord;
+      int d[4], n = 0;
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {
+        d[kk] = (int)((v >> (8 * kk)) & 0xFFu) - (int)((kSparseDefaultWord >> (8 * kk)) & 0xFFu);
+        n += d[kk] != 0;
+      }
+      int incl = n;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      int pos = base + incl - n;
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)
+        if (d[kk] != 0) {
+          if (pos < kSparseCap - 1) L[1 + pos] = ((uint32_t)(4 * wi + kk) << 8) | ((uint32_t)d[kk] & 0xFFu);
+          ++pos;
+        }
+      base += __shfl_sync(0xFFFFFFFFu, incl, 31);
+    }
+    if (lane == 0) L[0] = (uint32_t)base;
+  }
+  __syncthreads();
+  const int ncb = m.H0 >> 2;
+  for (int blk = threadIdx.x; blk < live * ncb; blk += blockDim.x) {
+    const int r = blk / ncb, c0 = (blk - r * ncb) << 2;
+    const uint32_t* L = list + r * kSparseCap;
+    const int n = (int)L[0];
+    if (n > kSparseCap - 1) {  // not of the pattern: the dense sum
+      float4 acc = __ldg(reinterpret_cast<const float4*>(b1 + c0));
+      for (int k = 0; k < m.K; ++k) {
+        const float x = (float)X[r * m.KP + k];
+        const float4 wv = __ldg(reinterpret_cast<const float4*>(Wt + (int64_t)k * m.H0 + c0));
+        acc.x = fmaf(x, wv.x, acc.x);
+        acc.y = fmaf(x, wv.y, acc.y);
+        acc.z = fmaf(x, wv.z, acc.z);
+        acc.w = fmaf(x, wv.w, acc.w);
+      }
+      *reinterpret_cast<float4*>(H1 + r * m.H0 + c0) =
+          make_float4(tanhf(acc.x), tanhf(acc.y), tanhf(acc.z), tanhf(acc.w));
+      continue;
+    }
+    float4 acc = __ldg(reinterpret_cast<const float4*>(c + c0));
+    for (int j = 1; j <= n; ++j) {
+      const uint32_t e = L[j];
+      const float dv = (float)(int8_t)(e & 0xFFu);
+      const float4 wv = __ldg(reinterpret_cast<const float4*>(Wt + (int64_t)(e >> 8) * m.H0 + c0));
+      acc.x = fmaf(dv, wv.x, acc.x);
+      acc.y = fmaf(dv, wv.y, acc.y);
+      acc.z = fmaf(dv, wv.z, acc.z);
+      acc.w = fmaf(dv, wv.w, acc.w);
+    }
+    *reinterpret_cast<float4*>(H1 + r * m.H0 + c0) =
+        make_float4(tanhf(acc.x), tanhf(acc.y), tanhf(acc.z), tanhf(acc.w));
+  }
+}
+
+// Whole policy forward for an M-row tile: X u8 [M][KP] -> Z f32 [M][NOP].  list: the
+// sparse first layer's scratch (M * kSparseCap words; unused unless m.sparse), which
+// computes rows < live only (the others' outputs are then undefined).
 // Synchronises the CTA between layers and at the end.
 __device__ __forceinline__ void mlp_tile(const float* __restrict__ w, const MlpDims& m,
                                          const uint8_t* X, float* H1, float* H2, float* Z,
-                                         int M) {
-  dense_tile<true, true>(X, m.KP, M, m.K, w + m.oW1, w + m.ob1, m.H0, H1, m.H0);
+                                         int M, uint32_t* list, int live) {
+  if (m.sparse)
+    sparse_l1_tile(X, m, live, w + m.oW1, w + m.ob1, w + m.oC, list, H1);
+  else
+    dense_tile<true, true>(X, m.KP, M, m.K, w + m.oW1, w + m.ob1, m.H0, H1, m.H0);
   __syncthreads();
   dense_tile<false, true>(H1, m.H0, M, m.H0, w + m.oW2, w + m.ob2, m.H1, H2, m.H1);
   __syncthreads();

@@ -12,7 +12,7 @@
 namespace aht {
 
 struct SmemLayout {
-  int64_t st, X, H1, H2, Z, envid, act, lp, val, alive, steps, total;
+  int64_t st, X, H1, H2, Z, envid, act, lp, val, alive, steps, list, total;
 };
 
 __host__ __device__ inline SmemLayout smem_layout(int M, const MlpDims& m, int state_bytes) {
@@ -29,6 +29,7 @@ __host__ __device__ inline SmemLayout smem_layout(int M, const MlpDims& m, int s
   L.val = o;   o = align_up(o + (int64_t)M * 4, 16);
   L.alive = o; o = align_up(o + (int64_t)M * 4, 16);
   L.steps = o; o = align_up(o + (int64_t)M * 4, 16);
+  L.list = o;  o = align_up(o + (m.sparse ? (int64_t)M * kSparseCap * 4 : 0), 16);
   L.total = o;
   return L;
 }
@@ -112,7 +113,7 @@ __global__ void __launch_bounds__(kThreads) ppo_kernel(const PpoArgs a) {
         copy_obs_rows(X, m.KP, count, envid, a.traj.obs + (int64_t)t * N * od, od);
       if (seat == 1 && a.traj1.obs)
         copy_obs_rows(X, m.KP, count, envid, a.traj1.obs + (int64_t)t * N * od, od);
-      mlp_tile(w_pol[seat], m, X, H1, H2, Z, M);
+      mlp_tile(w_pol[seat], m, X, H1, H2, Z, M, reinterpret_cast<uint32_t*>(smem + L.list), count);
       for (int i = tid; i < count; i += blockDim.x) {
         const float u = u01(draw0(a.b.key, (uint32_t)envid[i], gt, kStreamAct0 + seat));
         float logp;
@@ -155,14 +156,14 @@ __global__ void __launch_bounds__(kThreads) ppo_kernel(const PpoArgs a) {
   if (a.traj.last_value) {
     for (int i = tid; i < count; i += blockDim.x) Env::obs(a.b.env, st[i], 0, X + i * m.KP);
     __syncthreads();
-    mlp_tile(w_pol[0], m, X, H1, H2, Z, M);
+    mlp_tile(w_pol[0], m, X, H1, H2, Z, M, reinterpret_cast<uint32_t*>(smem + L.list), count);
     for (int i = tid; i < count; i += blockDim.x) a.traj.last_value[envid[i]] = Z[i * m.NOP + m.NA];
     __syncthreads();
   }
   if (a.traj1.last_value) {  // seat 1's V_T (IPPO)
     for (int i = tid; i < count; i += blockDim.x) Env::obs(a.b.env, st[i], 1, X + i * m.KP);
     __syncthreads();
-    mlp_tile(w_pol[1], m, X, H1, H2, Z, M);
+    mlp_tile(w_pol[1], m, X, H1, H2, Z, M, reinterpret_cast<uint32_t*>(smem + L.list), count);
     for (int i = tid; i < count; i += blockDim.x) a.traj1.last_value[envid[i]] = Z[i * m.NOP + m.NA];
   }
   for (int i = tid; i < count; i += blockDim.x) store_state(a.state, N, envid[i], st[i]);
@@ -212,7 +213,7 @@ __global__ void __launch_bounds__(kThreads) xplay_kernel(const XpArgs a) {
       for (int i = tid; i < count; i += blockDim.x)
         if (alive[i]) Env::obs(a.b.env, st[i], seat, X + i * m.KP);
       __syncthreads();
-      mlp_tile(w_pol[seat], m, X, H1, H2, Z, M);
+      mlp_tile(w_pol[seat], m, X, H1, H2, Z, M, reinterpret_cast<uint32_t*>(smem + L.list), count);
       for (int i = tid; i < count; i += blockDim.x) {
         if (!alive[i]) continue;
         uint32_t legal = 0xFFFFFFFFu >> (32 - m.NA);
