@@ -51,21 +51,25 @@ struct EnvOps {
   int (*bytes)();
   cudaError_t (*smem_limit)(size_t);
   int max_rows;  // largest tile that fits the hidden activations of typical sizes
+  int (*occupancy)(int which, size_t smem);  // resident CTAs per SM of the CUDA-core kernels
 };
 
 EnvOps ops_for(int kind) {
   switch (kind) {
     case AHT_LBF:
-      return {lbf_ppo, lbf_xplay, lbf_forced, lbf_reset, lbf_state_words, lbf_state_bytes, lbf_set_smem_limit, 128};
+      return {lbf_ppo, lbf_xplay, lbf_forced, lbf_reset, lbf_state_words, lbf_state_bytes, lbf_set_smem_limit,
+              128, lbf_occupancy};
     case AHT_OVERCOOKED:
       return {overcooked_ppo, overcooked_xplay, overcooked_forced, overcooked_reset,
-              overcooked_state_words, overcooked_state_bytes, overcooked_set_smem_limit, 64};
+              overcooked_state_words, overcooked_state_bytes, overcooked_set_smem_limit, 64,
+              overcooked_occupancy};
     case AHT_MINI_HANABI:
       return {minihanabi_ppo, minihanabi_xplay, minihanabi_forced, minihanabi_reset,
-              minihanabi_state_words, minihanabi_state_bytes, minihanabi_set_smem_limit, 64};
+              minihanabi_state_words, minihanabi_state_bytes, minihanabi_set_smem_limit, 64,
+              minihanabi_occupancy};
     default:
       return {hanabi_ppo, hanabi_xplay, hanabi_forced, hanabi_reset, hanabi_state_words,
-              hanabi_state_bytes, hanabi_set_smem_limit, 32};
+              hanabi_state_bytes, hanabi_set_smem_limit, 32, hanabi_occupancy};
   }
 }
 
@@ -92,6 +96,7 @@ struct aht_ctx {
   uint64_t seed = 0;
   int64_t step = 0;
   size_t smem_optin = 0;
+  int n_sms = 0;
   int64_t max_tiles = 0;
   // device memory, all allocated in aht_create
   uint32_t* state = nullptr;
@@ -552,6 +557,20 @@ int fit_rows(const aht_ctx* c, int want) {
   return M;
 }
 
+// The CUDA-core kernels are latency-bound per CTA: halve the tile (down to 32 rows)
+// while every tile of the launch still fits in one wave of resident CTAs, so that more
+// SMs, and more CTAs per SM, share the work.  tiles(M): the launch's tile count.
+template <class F>
+int spread_rows(const aht_ctx* c, int M, int which, F tiles) {
+  while (M >= 64) {
+    const int M2 = (int)align_up(M / 2, 4);
+    const int per_sm = c->ops.occupancy(which, smem_layout(M2, c->mlp, c->ops.bytes()).total);
+    if (per_sm < 1 || tiles(M2) > (int64_t)per_sm * c->n_sms) break;
+    M = M2;
+  }
+  return M;
+}
+
 }  // namespace
 
 extern "C" {
@@ -635,6 +654,9 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
   int optin = 0;
   cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, c->device);
   c->smem_optin = (size_t)optin;
+  int sms = 0;
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
+  c->n_sms = sms;
 
   const MlpDims& m = c->mlp;
   std::vector<float> packed((size_t)m.stride * pop->n_policies, 0.0f);
@@ -800,7 +822,9 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
       return fail(AHT_EINVAL, "out1->obs must be 4-byte aligned");
   }
   DeviceGuard g(c->device);
-  const int M = c->tc ? 128 : fit_rows(c, 128);
+  const int64_t Nall = c->n_envs;
+  const int M = c->tc ? 128
+                      : spread_rows(c, fit_rows(c, 128), 0, [&](int m) { return (int64_t)group_tiles(Nall, m); });
 
   GroupArgs ga{};
   ga.key = batch_of(c).key;
@@ -1035,7 +1059,8 @@ aht_status aht_xplay_matrix(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego,
     c->step += max_steps;
     return AHT_OK;
   }
-  const int M = fit_rows(c, std::min(c->ops.max_rows, envs_per_pair));
+  const int M = spread_rows(c, fit_rows(c, std::min(c->ops.max_rows, envs_per_pair)), 1,
+                            [&](int m) { return n_pairs * ((envs_per_pair + m - 1) / m); });
   XpArgs a{};
   a.b = batch_of(c);
   a.n_ego = n_ego;
@@ -1126,7 +1151,8 @@ aht_status aht_xplay_matrix_static(aht_ctx* c, const int32_t* ego_ids, int32_t n
     c->step += max_steps;
     return AHT_OK;
   }
-  const int M = fit_rows(c, std::min(c->ops.max_rows, envs_per_pair));
+  const int M = spread_rows(c, fit_rows(c, std::min(c->ops.max_rows, envs_per_pair)), 1,
+                            [&](int m) { return n_pairs * ((envs_per_pair + m - 1) / m); });
   XpArgs a{};
   a.b = batch_of(c);
   a.n_ego = n_ego;

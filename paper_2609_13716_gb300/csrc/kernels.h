@@ -231,7 +231,8 @@ struct PolicyArgs {
   cudaError_t name##_reset(const ResetArgs&, cudaStream_t);                       \
   int name##_state_words();                                                      \
   int name##_state_bytes();                                                      \
-  cudaError_t name##_set_smem_limit(size_t bytes);
+  cudaError_t name##_set_smem_limit(size_t bytes);                                \
+  int name##_occupancy(int which /* 0 PPO, 1 cross-play */, size_t smem);
 
 AHT_DECLARE_ENV_LAUNCHERS(lbf)
 AHT_DECLARE_ENV_LAUNCHERS(overcooked)

@@ -337,6 +337,13 @@ struct Launch {
   cudaError_t name##_reset(const ResetArgs& a, cudaStream_t s) { return Launch<EnvT>::reset(a, s); }    \
   int name##_state_words() { return (int)(sizeof(EnvT::State) / 4); }                          \
   int name##_state_bytes() { return (int)sizeof(EnvT::State); }                                \
-  cudaError_t name##_set_smem_limit(size_t b) { return Launch<EnvT>::smem_limit(b); }
+  cudaError_t name##_set_smem_limit(size_t b) { return Launch<EnvT>::smem_limit(b); }            \
+  int name##_occupancy(int which, size_t sm) {                                                 \
+    int n = 0;                                                                                 \
+    if (which == 0) cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, ppo_kernel<EnvT>, kThreads, sm); \
+    else cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, xplay_kernel<EnvT>, kThreads, sm);  \
+    cudaGetLastError();                                                                        \
+    return n;                                                                                  \
+  }
 
 }  // namespace aht
