@@ -303,24 +303,46 @@ def run_ours(args):
     aht.aht_sync(ctx)
 
     # ---- end to end: ego weights from pinned host memory in, whole trajectory out ------
+    # Two trajectory buffers, as a user would double-buffer: step k's trajectory is copied
+    # to pinned host memory on a copy stream while step k + 1 runs on the library's
+    # stream.  Every step's upload and download lies inside the timed region, which ends
+    # when the last download has landed.
     ego_host = [(W_.to(torch.bfloat16).cpu().pin_memory(), b.to(torch.bfloat16).cpu().pin_memory())
                 for W_, b in [(torch.from_numpy(a), torch.from_numpy(c)) for a, c in pop_np[wl.ego_id]]]
-    host = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in traj.items() if v is not None}
-    h2d = sum(W_.numel() * 2 + b.numel() * 2 for W_, b in ego_host)
-    d2h = sum(v.numel() * v.element_size() for v in host.values())
-    e2e_s, e2e_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e2e_ms = []
-    for k in range(0 if args.no_e2e else args.steps + 1):
+    h2d = sum(W_.numel() * 2 + b.numel() * 2 for W_, b in ego_host)
+    d2h = sum(v.numel() * v.element_size() for v in traj.values() if v is not None)
+    if not args.no_e2e:
+        trajs = [traj, aht.traj_buffers(ctx, T)]
+        hosts = [{k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in t.items() if v is not None}
+                 for t in trajs]
+        copy_stream = torch.cuda.Stream()
+        rolled = [torch.cuda.Event(), torch.cuda.Event()]
+        copied = [torch.cuda.Event(), torch.cuda.Event()]
+
+        def e2e_step(k):
+            b = k % 2
+            stream.wait_event(copied[b])            # buffer b's previous download is done
+            aht.aht_set_policy(ctx, wl.ego_id, ego_host, 1, aht.AHT_BF16)
+            aht.aht_rollout(ctx, wl.ego_id, wl.pool, T, trajs[b], wl.gamma, wl.lam)
+            rolled[b].record(stream)
+            copy_stream.wait_event(rolled[b])
+            with torch.cuda.stream(copy_stream):
+                for key, hv in hosts[b].items():
+                    hv.copy_(trajs[b][key], non_blocking=True)
+            copied[b].record(copy_stream)
+
+        for k in range(2):
+            e2e_step(k)
         torch.cuda.synchronize()
+        e2e_s, e2e_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e2e_s.record(stream)
-        aht.aht_set_policy(ctx, wl.ego_id, ego_host, 1, aht.AHT_BF16)
-        step()
-        for key, hv in host.items():
-            hv.copy_(traj[key], non_blocking=True)
+        for k in range(args.steps):
+            e2e_step(k)
+        stream.wait_stream(copy_stream)
         e2e_e.record(stream)
         torch.cuda.synchronize()
-        if k > 0:
-            e2e_ms.append(e2e_s.elapsed_time(e2e_e))
+        e2e_ms = [e2e_s.elapsed_time(e2e_e) / args.steps]
     aht.aht_sync(ctx)
     e2e_ms_max = max_over_ranks(sum(e2e_ms) / max(1, len(e2e_ms)), "cuda")
 
