@@ -865,7 +865,6 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
     ta.tcw = c->tcw;
     ta.state = c->state;
     ta.n_envs = c->n_envs;
-    ta.perm = c->perm;
     ta.tiles = c->tiles;
     ta.ego = ego_id;
     ta.step0 = a.step0;

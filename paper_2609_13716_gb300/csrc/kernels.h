@@ -99,8 +99,7 @@ struct PpoTcArgs {
   const uint8_t* tcw;    // [n_policies][pol_bytes]
   uint32_t* state;
   int64_t n_envs;
-  const int32_t* perm;
-  const int4* tiles;     // tiles of up to 128 envs
+  const int4* tiles;     // tiles of up to 128 contiguous envs (not read by gather launches)
   int32_t ego;
   uint32_t step0;
   int32_t T;

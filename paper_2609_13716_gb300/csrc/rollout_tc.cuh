@@ -1,6 +1,7 @@
 // rollout_tc.cuh -- fused PPO rollout with the policy MLPs on tcgen05 tensor cores.
 //
-// One CTA owns a tile of up to 128 envs that share one teammate policy, for all T steps.
+// One CTA owns a tile of up to 128 envs that share one teammate policy, for all T steps
+// (per-episode teammates: for one step, the tile's envs found by a rank scan, kGather).
 // Per step and agent (ego = seat 0, teammate = seat 1):
 //   obs (u8, shared memory, a constant 1 after the last feature) -> A operand in tensor
 //       memory as bf16 (exact: small integers)
