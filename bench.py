@@ -651,11 +651,12 @@ def run_xplay(args, aht, W, torch, bf16_peak, names=XPLAY_WORKLOADS, bf16_sustai
                                   "flops_per_matrix": flops},
                      "xp_stats_us": stats_us}
         if wl.env.kind == W.LBF and wl.env.obs_dim > 255:
-            # the CUDA-core path: its first layer adds only the observation's changed
-            # features to a per-policy constant, so these are dense-equivalent FLOPs
+            # wider than the tensor-memory operand: the first layer adds only the
+            # observation's changed features to a per-policy constant (CUDA cores), so
+            # these are dense-equivalent FLOPs
             res[name]["roofline"]["flops_basis"] = (
-                "dense-equivalent MLP FLOPs; the CUDA-core kernel's first layer skips the "
-                "observation's unchanged features")
+                "dense-equivalent MLP FLOPs; the first layer is formed on CUDA cores from the "
+                "observation's changed features, the second on the tensor cores")
     return res
 
 

@@ -277,11 +277,15 @@ TcDims make_tc_dims(const MlpDims& m, bool split) {
   t.H0 = m.H0;
   t.H1 = m.H1;
   t.split = split ? 1 : 0;
+  // an observation wider than an agent's 256 A-operand columns: the first layer runs on
+  // CUDA cores from the observation's changed features (LBF), W1 stays out of the block
+  t.sparse = (m.sparse && t.KP > 256) ? 1 : 0;
+  const uint32_t w1 = t.sparse ? 0u : (uint32_t)(m.H0 * t.KP * 2);
   uint32_t o = 0;
-  t.oW1 = o; o += (uint32_t)(m.H0 * t.KP * 2);
+  t.oW1 = o; o += w1;
   t.oW2 = o; o += (uint32_t)(m.H1 * m.H0 * 2);
   if (split) {
-    t.oW1lo = o; o += (uint32_t)(m.H0 * t.KP * 2);
+    t.oW1lo = o; o += w1;
     t.oW2lo = o; o += (uint32_t)(m.H1 * m.H0 * 2);
   }
   t.oW3 = o; o += (uint32_t)(m.H1 * 8 * 4);
@@ -307,7 +311,8 @@ bool tc_eligible(const aht_ctx* c, int dtype) {
   const MlpDims& m = c->mlp;
   if (c->env.kind != AHT_LBF) return false;
   const TcDims t = make_tc_dims(m, dtype == AHT_FP32);
-  if (t.KP > 256 || m.H0 > 128 || m.H1 > 128 || m.H0 % 64 || m.H1 % 64 || m.NA + 1 > 8) return false;
+  if ((t.KP > 256 && !t.sparse) || m.H0 > 128 || m.H1 > 128 || m.H0 % 64 || m.H1 % 64 || m.NA + 1 > 8)
+    return false;
   return m.K % 4 == 0 && tc_smem_bytes(t, m.K, c->ops.bytes()) <= c->smem_optin;
 }
 
@@ -389,7 +394,7 @@ aht_status pack_policy_tc(const MlpDims& m, const TcDims& t, const void* const* 
       for (int k = 0; k < ins[l]; ++k) {
         const int64_t i = (int64_t)n * ins[l] + k;
         const float f = to_f32(src, i, dtype);
-        if (l == 0) put(t.oW1, t.oW1lo, tc::canon_offset(n, k, t.KP), f);
+        if (l == 0 && !t.sparse) put(t.oW1, t.oW1lo, tc::canon_offset(n, k, t.KP), f);
         if (l == 1) put(t.oW2, t.oW2lo, tc::canon_offset(n, k, m.H0), f);
         if (l == 2)  // hidden units in pairs: [k / 2][output][k % 2]
           std::memcpy(dst + t.oW3 + 4 * (((k / 2) * 8 + n) * 2 + (k % 2)), &f, 4);
@@ -397,7 +402,8 @@ aht_status pack_policy_tc(const MlpDims& m, const TcDims& t, const void* const* 
     if (!read_host(b[l], (size_t)outs[l] * esz, tmp, &src)) return fail(AHT_ECUDA, "copying biases failed");
     for (int n = 0; n < outs[l]; ++n) {
       const float f = to_f32(src, n, dtype);
-      if (l == 0) put(t.oW1, t.oW1lo, tc::canon_offset(n, m.K, t.KP), f);  // b1: weight of the constant-1 input
+      if (l == 0 && !t.sparse)  // b1: weight of the constant-1 input
+        put(t.oW1, t.oW1lo, tc::canon_offset(n, m.K, t.KP), f);
       if (l == 1) std::memcpy(dst + t.ob2 + 4 * n, &f, 4);
       if (l == 2) std::memcpy(dst + t.ob3 + 4 * n, &f, 4);
     }
@@ -823,8 +829,11 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
   }
   DeviceGuard g(c->device);
   const int64_t Nall = c->n_envs;
-  const int M = c->tc ? 128
-                      : spread_rows(c, fit_rows(c, 128), 0, [&](int m) { return (int64_t)group_tiles(Nall, m); });
+  // the sparse-first-layer tensor-core kernel does plain collection; IPPO there runs on
+  // the CUDA-core kernel
+  const bool use_tc = c->tc && !(c->tcd.sparse && out1);
+  const int M = use_tc ? 128
+                       : spread_rows(c, fit_rows(c, 128), 0, [&](int m) { return (int64_t)group_tiles(Nall, m); });
 
   GroupArgs ga{};
   ga.key = batch_of(c).key;
@@ -858,7 +867,7 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
                        out1->rewards, out1->dones,
                        out1->last_value ? out1->last_value
                                         : (out1->advantages ? c->last_value + c->n_envs : nullptr)};
-  if (c->tc) {
+  if (use_tc) {
     PpoTcArgs ta{};
     ta.b = a.b;
     ta.tc = c->tcd;
@@ -905,21 +914,25 @@ aht_status aht_rollout_resample(aht_ctx* c, int32_t ego_id, const int32_t* pool,
   if (!pool || pool_size < 1 || pool_size > kMaxPool) return fail(AHT_EINVAL, "pool_size must be in 1..256");
   for (int k = 0; k < pool_size; ++k) {
     if (pool[k] >= c->n_policies || pool[k] < -AHT_LBF_N_HEURISTICS) return fail(AHT_EINVAL, "pool id out of range");
-    if (pool[k] < 0 && !(c->env.kind == AHT_LBF && c->tc))
-      return fail(AHT_EINVAL, "heuristic teammates (negative ids) need an LBF context on the tensor-core path");
+    if (pool[k] < 0 && !(c->env.kind == AHT_LBF && c->tc && !c->tcd.sparse))
+      return fail(AHT_EINVAL, "heuristic teammates (negative ids) need an LBF context on the tensor-core path "
+                              "with the observation in tensor memory");
   }
   if (T < 1) return fail(AHT_EINVAL, "T must be >= 1");
   if (c->step + T + 1 > (int64_t)UINT32_MAX) return fail(AHT_EINVAL, "step counter would exceed 2^32");
   if (aht_status e = check_traj_out(out)) return e;
   if (reinterpret_cast<uintptr_t>(out->obs) & 3u) return fail(AHT_EINVAL, "out->obs must be 4-byte aligned");
   DeviceGuard g(c->device);
-  const int M = c->tc ? 128 : fit_rows(c, 128);
+  // the gathered per-episode tiles run on the dense-first-layer tensor-core kernel; the
+  // sparse-first-layer contexts (LBF beyond 256 tensor-memory columns) on CUDA cores
+  const bool use_tc = c->tc && !c->tcd.sparse;
+  const int M = use_tc ? 128 : fit_rows(c, 128);
   const int64_t N = c->n_envs;
   const int od = c->env.obs_dim;
   const int grid = resample_tiles(N, M, pool_size);
   float* last_value = out->last_value ? out->last_value : (out->advantages ? c->last_value : nullptr);
 
-  if (c->tc) {
+  if (use_tc) {
     // Tensor-core path: each step's launch groups its own rows (TcGather).
     const size_t smem = c->tc_smem + kTcGatherScratch;
     if (smem > c->smem_optin) return fail(AHT_EINVAL, "no shared memory left for the per-episode grouping");

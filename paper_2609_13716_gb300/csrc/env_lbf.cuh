@@ -146,6 +146,28 @@ struct EnvLbf {
     w[s.ay[seat] * d.width + s.ax[seat]] = (uint32_t)s.al[seat];
   }
 
+  // The observation as changes to the all-empty pattern (every cell word 0x01000000):
+  // slot i (foods 0-2, the other agent, the agent itself) is the cell's two changed
+  // features, +value in its channel and -1 in channel 3, as entries (feature << 8) |
+  // (delta & 0xFF) in e[2i], e[2i + 1].  Returns the mask of the entries in use (eaten
+  // foods have none).  The rules keep occupied cells distinct, so this equals obs().
+  __device__ static uint32_t sparse_obs(const DevEnv& d, const State& s, int seat, uint32_t (&e)[10]) {
+    auto cell = [&](int i, int x, int y, int ch, int v) {
+      const uint32_t c = (uint32_t)(y * d.width + x);
+      e[2 * i] = ((4u * c + (uint32_t)ch) << 8) | (uint32_t)(v & 0xFF);
+      e[2 * i + 1] = ((4u * c + 3u) << 8) | 0xFFu;
+    };
+    uint32_t mask = 0x3C0u;
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {
+      cell(k, s.fx[k], s.fy[k], 2, s.fl[k]);
+      if (!((s.eaten >> k) & 1u)) mask |= 3u << (2 * k);
+    }
+    cell(3, s.ax[1 - seat], s.ay[1 - seat], 1, s.al[1 - seat]);
+    cell(4, s.ax[seat], s.ay[seat], 0, s.al[seat]);
+    return mask;
+  }
+
   // Words [w0, w1) of the same row (w1 <= cells): one cell per word.
   __device__ static void obs_words(const DevEnv& d, const State& s, int seat, uint32_t* w, int w0,
                                    int w1) {

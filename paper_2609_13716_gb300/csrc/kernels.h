@@ -55,6 +55,9 @@ struct PpoArgs {
 struct TcDims {
   int32_t KP, H0, H1;      // padded obs dim (> obs_dim), hidden sizes
   int32_t split;           // 1: fp32 weights as bf16 pairs (W1lo, W2lo present)
+  int32_t sparse;          // 1: no W1 in the block; the first layer runs on CUDA cores from
+                           // the env's changed features and the fp32 W1^T / c of the
+                           // CUDA-core population (LBF grids beyond 256 tensor-memory columns)
   uint32_t oW1, oW2, oW3, ob2, ob3, oW1lo, oW2lo;
   uint32_t pol_bytes;
 };

@@ -45,11 +45,16 @@ constexpr int kTcPairBar = 2;            // ids 2..5: warps q and q + 4 (rows 32
 // 2^-16 of the sum and left out).  kIppo (PPO collection only): seat 1 learns too, and
 // its trajectory goes to a.traj1.  kGather (PPO collection, one step per launch): the
 // tile's rows are the envs perm[tile.x + r] (a group of envs whose episodes drew the
-// same teammate) instead of a contiguous range.
-template <class Env, bool kXp, bool kSplit, bool kIppo, bool kGather>
+// same teammate) instead of a contiguous range.  kSparse (observations wider than the
+// 256 tensor-memory columns of an agent's A operand; Env::sparse_obs required): no first
+// layer on the tensor cores -- each thread forms its half of h1 = tanh(c + sum over the
+// observation's changed features of delta W1[:, f]) on CUDA cores from the fp32 W1^T and
+// c of the CUDA-core population, and writes it as the A operand of L2 directly.
+template <class Env, bool kXp, bool kSplit, bool kIppo, bool kGather, bool kSparse>
 __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a) {
   static_assert(!(kXp && kIppo), "seat-1 trajectories belong to PPO collection");
   static_assert(!(kGather && (kXp || kIppo)), "gathered tiles are plain PPO collection");
+  static_assert(!(kSparse && (kIppo || kGather)), "the sparse first layer serves plain collection and cross-play");
   using State = typename Env::State;
   constexpr int NA = Env::kNumActions;
   extern __shared__ __align__(16) uint8_t smem[];  // no-swizzle operands need 16 B
@@ -271,15 +276,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       const int n_steps = kXp ? a.xp.max_steps : a.T;
       for (int t = 0; ok && !stopped && t < n_steps; ++t) {
         const uint32_t par = (uint32_t)t & 1u;
-        if (!tm_rule) issue(1, 0, par);
-        if (ok && !stopped) issue(0, 0, par);
+        if (!kSparse) {
+          if (!tm_rule) issue(1, 0, par);
+          if (ok && !stopped) issue(0, 0, par);
+        }
         if (ok && !stopped && !tm_rule) issue(1, 1, par);
         if (ok && !stopped) issue(0, 1, par);
       }
       if (ok && with_boot) {
         const uint32_t par = (uint32_t)a.T & 1u;
-        if (boot1) issue(1, 0, par);
-        if (ok) issue(0, 0, par);
+        if (!kSparse) {
+          if (boot1) issue(1, 0, par);
+          if (ok) issue(0, 0, par);
+        }
         if (ok && boot1) issue(1, 1, par);
         if (ok) issue(0, 1, par);
       }
@@ -347,6 +356,56 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         tc::st_x16(P + c0 / 2, hi);
         tc::st_x16(P + H / 2 + c0 / 2, lo);
         tc::st_x32(Q + c0, v);
+      }
+      tc::wait_st();
+      operand_ready(ag, 1);
+    };
+    // kSparse: h1 = tanh(c + sum over the changed features f of delta W1[:, f]) for this
+    // thread's half of the units, written like epilogue 1 (hi | lo operand of L2, b2 into
+    // the accumulator); rows past count take c alone
+    auto sparse_h1 = [&](int ag, const State& s) {
+      const int H = d.H0;
+      const uint32_t P = tmem + (uint32_t)(ag * 256) + lane_base, Q = P + 128;
+      const float* pw = a.b.weights + (int64_t)(ag == 0 ? ego_pol : tm_pol) * a.b.mlp.stride;
+      const float* W1t = pw + a.b.mlp.oW1;
+      const float* cvec = pw + a.b.mlp.oC;
+      const float* b2 = reinterpret_cast<const float*>(pol_block(ag) + d.ob2);
+      uint32_t e[10];
+      const uint32_t mask = row < count ? Env::sparse_obs(a.b.env, s, ag, e) : 0u;
+      for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 32) {
+        float v[32];
+#pragma unroll
+        for (int j = 0; j < 32; j += 4) {
+          const float4 cc = __ldg(reinterpret_cast<const float4*>(cvec + c0 + j));
+          v[j] = cc.x; v[j + 1] = cc.y; v[j + 2] = cc.z; v[j + 3] = cc.w;
+        }
+#pragma unroll
+        for (int q = 0; q < 10; ++q) {
+          if (!((mask >> q) & 1u)) continue;
+          const float dv = (float)(int8_t)(e[q] & 0xFFu);
+          const float* wr = W1t + (int64_t)(e[q] >> 8) * H + c0;
+#pragma unroll
+          for (int j = 0; j < 32; j += 4) {
+            const float4 w4 = __ldg(reinterpret_cast<const float4*>(wr + j));
+            v[j] = fmaf(dv, w4.x, v[j]);
+            v[j + 1] = fmaf(dv, w4.y, v[j + 1]);
+            v[j + 2] = fmaf(dv, w4.z, v[j + 2]);
+            v[j + 3] = fmaf(dv, w4.w, v[j + 3]);
+          }
+        }
+        uint32_t hi[16], lo[16], bb[32];
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(v[2 * j], v[2 * j + 1])), hi[j], lo[j]);
+#pragma unroll
+        for (int j = 0; j < 32; j += 4) {
+          const float4 b4 = *reinterpret_cast<const float4*>(b2 + c0 + j);
+          bb[j] = __float_as_uint(b4.x); bb[j + 1] = __float_as_uint(b4.y);
+          bb[j + 2] = __float_as_uint(b4.z); bb[j + 3] = __float_as_uint(b4.w);
+        }
+        tc::st_x16(P + c0 / 2, hi);
+        tc::st_x16(P + H / 2 + c0 / 2, lo);
+        tc::st_x32(Q + c0, bb);
       }
       tc::wait_st();
       operand_ready(ag, 1);
@@ -438,7 +497,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         // every env of the tile is done: release the MMA warp without operands and stop
         if (!tc::bar_or(kTcComputeBar, kTcCompute, half == 0 && row < count && alive)) {
           if (tid == 0) stop_flag = 1;
-          tc::mbar_arrive(&opnd_bar[tm_rule ? 0 : 2]);  // the first L1 barrier it waits on
+          // the first barrier it waits on: L1 of the first agent (L2 without a first layer)
+          tc::mbar_arrive(&opnd_bar[(tm_rule ? 0 : 2) + (kSparse ? 1 : 0)]);
           break;
         }
       }
@@ -450,6 +510,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       State s = st[row];  // register copy for this step (rows past count are never used)
 #pragma unroll 1
       for (int i = first; i >= 0; --i) {
+        if constexpr (kSparse) {
+          // the ego's u8 row is the trajectory's observation; no first layer to feed
+          if (!kXp && i == 0 && !boot && a.traj.obs && row < count)
+            Env::obs_words(a.b.env, s, 0, reinterpret_cast<uint32_t*>(sObs + row * od), my_w0, my_w1);
+          if (!bad) sparse_h1(i, s);
+          continue;
+        }
         obs_x(i, s);
         if (kIppo && i == 1 && !boot && a.traj1.obs) {
           // seat 1's rows -> its trajectory before the ego's overwrite them: warps q and
@@ -467,7 +534,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         }
       }
 #pragma unroll 1
-      for (int i = first; i >= 0; --i) {
+      for (int i = first; i >= 0 && !kSparse; --i) {
         wait_acc(i, 0, par);
         if (!bad) epilogue1(i);
       }
@@ -613,18 +680,23 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
 
 template <class Env>
 struct LaunchTc {
-  template <bool kXp, bool kSplit, bool kIppo, bool kGather = false>
+  template <bool kXp, bool kSplit, bool kIppo, bool kGather = false, bool kSparse = false>
   static cudaError_t run(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
-    cudaError_t e = cudaFuncSetAttribute(ppo_tc_kernel<Env, kXp, kSplit, kIppo, kGather>,
+    cudaError_t e = cudaFuncSetAttribute(ppo_tc_kernel<Env, kXp, kSplit, kIppo, kGather, kSparse>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    ppo_tc_kernel<Env, kXp, kSplit, kIppo, kGather><<<grid, kTcThreads, smem, s>>>(a);
+    ppo_tc_kernel<Env, kXp, kSplit, kIppo, kGather, kSparse><<<grid, kTcThreads, smem, s>>>(a);
     return cudaGetLastError();
   }
   static cudaError_t ppo(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
     const TrajPtrs& u = a.traj1;
     const bool ippo = u.obs || u.actions || u.tm_actions || u.logp || u.values || u.rewards ||
                       u.dones || u.last_value;
+    if (a.tc.sparse) {  // plain collection only (the host keeps the others on CUDA cores)
+      if (ippo || a.gather) return cudaErrorNotSupported;
+      return a.tc.split ? run<false, true, false, false, true>(a, grid, smem, s)
+                        : run<false, false, false, false, true>(a, grid, smem, s);
+    }
     if (a.gather)
       return a.tc.split ? run<false, true, false, true>(a, grid, smem, s)
                         : run<false, false, false, true>(a, grid, smem, s);
@@ -633,6 +705,9 @@ struct LaunchTc {
     return a.tc.split ? run<false, true, false>(a, grid, smem, s) : run<false, false, false>(a, grid, smem, s);
   }
   static cudaError_t xplay(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
+    if (a.tc.sparse)
+      return a.tc.split ? run<true, true, false, false, true>(a, grid, smem, s)
+                        : run<true, false, false, false, true>(a, grid, smem, s);
     return a.tc.split ? run<true, true, false>(a, grid, smem, s) : run<true, false, false>(a, grid, smem, s);
   }
 };
