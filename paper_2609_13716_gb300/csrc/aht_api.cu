@@ -325,7 +325,9 @@ WideDims make_wide_dims(const MlpDims& m) {
   w.n_l1 = (w.H / 256) * (w.KP / 16);
   w.n_l2 = (w.H / 256) * (w.H / 16);
   uint32_t o = (uint32_t)(w.n_l1 + w.n_l2) * kWideChunk;
-  w.oW3 = o; o += (uint32_t)(w.H * w.NAP * 4);
+  // W3 as bf16 B fragments of mma.sync m16n8k16: [H / 16 unit chunks][n-tiles of 8
+  // outputs][32 threads][2 words]
+  w.oW3 = o; o += (uint32_t)(w.H / 16) * (uint32_t)((w.NAP + 7) / 8) * 256u;
   w.ob2 = o; o += (uint32_t)(w.H * 4);
   w.ob3 = o; o += (uint32_t)(w.NAP * 4);
   w.pol_bytes = (uint32_t)align_up(o, 1024);
@@ -436,9 +438,13 @@ aht_status pack_policy_wide(const MlpDims& m, const WideDims& w, const void* con
         const int64_t i = (int64_t)n * ins[l] + k;
         if (l == 0) std::memcpy(w1_at(n, k), &wv[i], 2);
         if (l == 1) std::memcpy(w2_at(n, k), &wv[i], 2);
-        if (l == 2 && n < m.NA) {  // hidden units in pairs: [k / 2][output][k % 2]
+        if (l == 2 && n < m.NA) {  // B fragment of chunk k / 16, n-tile n / 8 (see WideDims)
           const float f = to_f32(src, i, AHT_BF16);
-          std::memcpy(dst + w.oW3 + 4 * (((size_t)(k / 2) * w.NAP + n) * 2 + (k % 2)), &f, 4);
+          const int kk = k % 16, nt_tiles = (w.NAP + 7) / 8;
+          const int t = 4 * (n % 8) + (kk % 8) / 2;                 // thread of the fragment
+          const size_t off = ((size_t)((k / 16) * nt_tiles + n / 8) * 32 + t) * 8 + (kk / 8) * 4 + (kk % 2) * 2;
+          const uint16_t hb = bf16_rne(f);
+          std::memcpy(dst + w.oW3 + off, &hb, 2);
         }
       }
     if (!read_host(b[l], (size_t)outs[l] * 2, tmp, &src)) return fail(AHT_ECUDA, "copying biases failed");

@@ -121,8 +121,11 @@ struct PpoTcArgs {
 //   chunk nh * (KP / 16) + ks            W1 rows [256 nh, 256 nh + 256), inputs [16 ks, 16 ks + 16)
 //   n_l1 + nh * (H / 16) + ks            W2 likewise (inputs are layer-1 units)
 // Input column obs_dim of W1 holds b1 (the observation carries a constant 1 there).
-// Then W3 fp32 [H / 2][NAP][2] (entry (p, o, i) = W3[o][2p + i]: hidden units in pairs
-// for packed fp32x2 FMAs), b2 fp32 [H], b3 fp32 [NAP].
+// Then W3 as bf16 B fragments of mma.sync m16n8k16 (the output layer runs on the legacy
+// tensor-core path from registers): [H / 16 unit chunks j][ceil(NAP / 8) n-tiles][32
+// threads t][2 words], word i of thread t holding W3[8 nt + t / 4][16 j + 8 i + 2 (t % 4)]
+// in its low and W3[same][... + 1] in its high half (zero past the outputs); b2 fp32 [H],
+// b3 fp32 [NAP].
 struct WideDims {
   int32_t KP, H, NAP;      // padded input (a multiple of 16), hidden width, padded outputs
   int32_t n_l1, n_l2;      // chunks of W1 and W2

@@ -468,30 +468,54 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
     const float* b3 = reinterpret_cast<const float*>(sA + L.w3_off + (w.ob3 - w.oW3));
     if (!bad && !tc::mbar_wait(&w3_bar, 0)) bad = true;
     bad = __any_sync(0xFFFFFFFFu, bad);
-    // hidden units in pairs (2p, 2p + 1): the packed FMA of output o accumulates
-    // W3[o][2p] h2[2p] and W3[o][2p + 1] h2[2p + 1] in its two halves
-    uint64_t acc[NAP];
+    // The output layer on the tensor cores from registers (mma.sync m16n8k16): each warp
+    // takes its 32 rows as two groups of 16 and its half's 128 units of each N = 256
+    // block as chunks of 16.  Two 16x256b loads of the accumulator give the thread the
+    // values of the A fragment (rows g, g + 8; units 2c, 2c + 1 and 2c + 8, 2c + 9 of the
+    // chunk, g = lane / 4, c = lane % 4); h2 = tanh(acc + b2) is split h2 = hi + lo (two
+    // bf16) and z accumulates hi W3^T + lo W3^T in fp32, n-tiles of 8 outputs.
+    constexpr int NT = (NAP + 7) / 8;
+    const uint32_t* W3f = reinterpret_cast<const uint32_t*>(W3);
+    const int g = lane >> 2, c4 = lane & 3;
+    float zacc[2][NT][4];
 #pragma unroll
-    for (int o = 0; o < NAP; ++o) acc[o] = 0ull;
+    for (int rg = 0; rg < 2; ++rg)
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) zacc[rg][nt][i] = 0.0f;
     const int n_blocks = w.H / 256;
+    const uint32_t R1q = tmem + 256u + ((uint32_t)((warp & 3) * 32) << 16);  // this warp's rows
     for (int nh = 0; nh < n_blocks; ++nh) {
       wait_acc(&acc_bar[1 + nh]);
       if (bad) break;
-      for (int c0 = 128 * half; c0 < 128 * half + 128; c0 += 32) {
-        uint32_t v[32];
-        tc::ld_x32(R1 + c0, v);
-        tc::wait_ld();
-        const int u0 = 256 * nh + c0;
-#pragma unroll 4
-        for (int j = 0; j < 32; j += 2) {
-          const uint64_t bb = *reinterpret_cast<const uint64_t*>(b2 + u0 + j);
-          const uint64_t h = tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(v[j]), __uint_as_float(v[j + 1])), bb));
-          const ulonglong2* wr = reinterpret_cast<const ulonglong2*>(W3 + (int64_t)(u0 + j) * NAP);
+#pragma unroll 1
+      for (int kc = 0; kc < 8; ++kc) {
+        const int c0 = 128 * half + 16 * kc;             // column of the N = 256 block
+        const int u0 = 256 * nh + c0;                    // hidden unit
+        const int j = u0 / 16;                           // W3 chunk
+        const uint64_t bA = *reinterpret_cast<const uint64_t*>(b2 + u0 + 2 * c4);
+        const uint64_t bB = *reinterpret_cast<const uint64_t*>(b2 + u0 + 8 + 2 * c4);
 #pragma unroll
-          for (int o = 0; o < NAP; o += 2) {
-            const ulonglong2 wv = wr[o / 2];
-            acc[o] = tc::f2_fma(h, wv.x, acc[o]);
-            acc[o + 1] = tc::f2_fma(h, wv.y, acc[o + 1]);
+        for (int rg = 0; rg < 2; ++rg) {
+          uint32_t t0[4], t1[4];
+          tc::ld_16x256b(R1q + ((uint32_t)(16 * rg) << 16) + (uint32_t)c0, t0);
+          tc::ld_16x256b(R1q + ((uint32_t)(16 * rg) << 16) + (uint32_t)(c0 + 8), t1);
+          tc::wait_ld();
+          uint32_t ahi[4], alo[4];
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t0[0]), __uint_as_float(t0[1])), bA)),
+                             ahi[0], alo[0]);
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t0[2]), __uint_as_float(t0[3])), bA)),
+                             ahi[1], alo[1]);
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t1[0]), __uint_as_float(t1[1])), bB)),
+                             ahi[2], alo[2]);
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t1[2]), __uint_as_float(t1[3])), bB)),
+                             ahi[3], alo[3]);
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            const uint2 bw = *reinterpret_cast<const uint2*>(W3f + ((j * NT + nt) * 32 + lane) * 2);
+            tc::mma_m16n8k16_bf16(zacc[rg][nt], ahi, bw.x, bw.y);
+            tc::mma_m16n8k16_bf16(zacc[rg][nt], alo, bw.x, bw.y);
           }
         }
       }
@@ -503,12 +527,16 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
     // partial sums of the two halves -> shared memory (the A region is dead now)
     float* zpart = reinterpret_cast<float*>(sA);
     if (!bad) {
-      float* dst = zpart + (half * 128 + row) * NAP;
 #pragma unroll
-      for (int o = 0; o < NAP; ++o) {
-        float e2, f2;
-        tc::f2_unpack(acc[o], e2, f2);
-        dst[o] = e2 + f2;
+      for (int rg = 0; rg < 2; ++rg) {
+        const int r0 = 32 * (warp & 3) + 16 * rg + g;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int o = 8 * nt + 2 * c4 + (i & 1), r = r0 + 8 * (i >> 1);
+            if (o < NAP) zpart[(half * 128 + r) * NAP + o] = zacc[rg][nt][i];
+          }
       }
     }
     bad = sync_or();
