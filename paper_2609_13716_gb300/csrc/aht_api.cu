@@ -398,8 +398,11 @@ aht_status pack_policy_tc(const MlpDims& m, const TcDims& t, const void* const* 
         const float f = to_f32(src, i, dtype);
         if (l == 0 && !t.sparse) put(t.oW1, t.oW1lo, tc::canon_offset(n, k, t.KP), f);
         if (l == 1) put(t.oW2, t.oW2lo, tc::canon_offset(n, k, m.H0), f);
-        if (l == 2)  // hidden units in pairs: [k / 2][output][k % 2]
-          std::memcpy(dst + t.oW3 + 4 * (((k / 2) * 8 + n) * 2 + (k % 2)), &f, 4);
+        if (l == 2) {  // B fragment of chunk k / 16 (see TcDims), remainders for split blocks
+          const int kk = k % 16, thr = 4 * n + (kk % 8) / 2;
+          const uint32_t off = (uint32_t)(((k / 16) * 32 + thr) * 8 + (kk / 8) * 4 + (kk % 2) * 2);
+          put(t.oW3, t.oW3 + (uint32_t)m.H1 * 16u, off, f);
+        }
       }
     if (!read_host(b[l], (size_t)outs[l] * esz, tmp, &src)) return fail(AHT_ECUDA, "copying biases failed");
     for (int n = 0; n < outs[l]; ++n) {

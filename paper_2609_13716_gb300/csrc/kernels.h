@@ -45,9 +45,11 @@ struct PpoArgs {
 //   W1 [H0][KP] bf16, canonical K-major (see tc_common.cuh); column obs_dim holds b1
 //      (the observation tile carries a constant 1 there),
 //   W2 [H1][H0] bf16, canonical K-major,
-//   W3 fp32 [H1 / 2][8][2]: entry (p, o, i) = W3[o][2p + i], hidden units in pairs
-//      for packed fp32x2 FMAs (outputs past n_actions, and the value row when absent,
-//      are zero),
+//   W3 [H1 * 32 bytes]: bf16 B fragments of mma.sync m16n8k16, [H1 / 16 unit chunks j]
+//      [32 threads t][2 words], word i of thread t holding W3[t / 4][16 j + 8 i + 2 (t % 4)]
+//      in its low and W3[t / 4][... + 1] in its high half (outputs past n_actions, and the
+//      value row when absent, are zero); split blocks follow with the bf16 remainders
+//      W3 - bf16(W3) in the same layout at + H1 * 16 bytes,
 //   b2 fp32 [H1], b3 fp32 [8],
 // and for fp32 populations ("split" blocks) W1lo and W2lo, the bf16 remainders
 // W - bf16(W) in the same layouts as W1 and W2: W = W1 + W1lo to about 2^-17 relative

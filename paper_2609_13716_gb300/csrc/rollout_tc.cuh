@@ -410,40 +410,49 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       tc::wait_st();
       operand_ready(ag, 1);
     };
-    // epilogue 2: h2 = tanh(D) and this half's partial z = sum_k W3[:, k] h2[k], stored
-    // for the half that samples the agent.  Hidden units go in pairs (2p, 2p + 1): the
-    // packed FMA of output o accumulates W3[o][2p] h2[2p] and W3[o][2p + 1] h2[2p + 1].
+    // epilogue 2: h2 = tanh(D) and this half's partial z = sum_k W3[:, k] h2[k] on the
+    // tensor cores from registers (mma.sync m16n8k16, one n-tile of 8 outputs): the warp
+    // takes its 32 rows as two groups of 16 and its half's units as chunks of 16; two
+    // 16x256b loads of the accumulator give the thread its A fragment (rows g, g + 8 with
+    // g = lane / 4; units 2c, 2c + 1 and 2c + 8, 2c + 9 of the chunk, c = lane % 4);
+    // h2 = hi + lo (two bf16) and z += hi W3^T + lo W3^T (+ hi W3lo^T for split blocks),
+    // fp32 accumulate.  The partial sums go to shared memory for the sampling half.
     auto epilogue2 = [&](int ag) {
       const int H = d.H1;
-      const uint32_t Q = tmem + (uint32_t)(ag * 256 + 128) + lane_base;
-      const float* W3 = reinterpret_cast<const float*>(pol_block(ag) + d.oW3);
-      uint64_t acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-      for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 32) {
-        uint32_t v[32];
-        tc::ld_x32(Q + c0, v);
-        tc::wait_ld();
+      const uint32_t Qq = tmem + (uint32_t)(ag * 256 + 128) + ((uint32_t)((warp & 3) * 32) << 16);
+      const uint32_t* W3f = reinterpret_cast<const uint32_t*>(pol_block(ag) + d.oW3);
+      const uint32_t* W3l = W3f + H * 4;  // split blocks: the remainders
+      const int g = lane >> 2, c4 = lane & 3;
+      float zacc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+#pragma unroll 1
+      for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 16) {
+        const int j = c0 >> 4;
+        const uint2 bw = *reinterpret_cast<const uint2*>(W3f + (j * 32 + lane) * 2);
+        uint2 bl = make_uint2(0u, 0u);
+        if constexpr (kSplit) bl = *reinterpret_cast<const uint2*>(W3l + (j * 32 + lane) * 2);
 #pragma unroll
-        for (int j = 0; j < 32; j += 2) {
-          const uint64_t h = tc::tanh2(tc::f2_pack(__uint_as_float(v[j]), __uint_as_float(v[j + 1])));
-          const ulonglong2* wp = reinterpret_cast<const ulonglong2*>(W3 + (c0 + j) * 8);
-#pragma unroll
-          for (int o = 0; o < 8; o += 2) {
-            const ulonglong2 ww = wp[o / 2];
-            acc[o] = tc::f2_fma(h, ww.x, acc[o]);
-            acc[o + 1] = tc::f2_fma(h, ww.y, acc[o + 1]);
-          }
+        for (int rg = 0; rg < 2; ++rg) {
+          uint32_t t0[4], t1[4];
+          tc::ld_16x256b(Qq + ((uint32_t)(16 * rg) << 16) + (uint32_t)c0, t0);
+          tc::ld_16x256b(Qq + ((uint32_t)(16 * rg) << 16) + (uint32_t)(c0 + 8), t1);
+          tc::wait_ld();
+          uint32_t ahi[4], alo[4];
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(t0[0]), __uint_as_float(t0[1]))), ahi[0], alo[0]);
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(t0[2]), __uint_as_float(t0[3]))), ahi[1], alo[1]);
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(t1[0]), __uint_as_float(t1[1]))), ahi[2], alo[2]);
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(t1[2]), __uint_as_float(t1[3]))), ahi[3], alo[3]);
+          tc::mma_m16n8k16_bf16(zacc[rg], ahi, bw.x, bw.y);
+          tc::mma_m16n8k16_bf16(zacc[rg], alo, bw.x, bw.y);
+          if constexpr (kSplit) tc::mma_m16n8k16_bf16(zacc[rg], ahi, bl.x, bl.y);
         }
       }
-      float z8[8];
+      float* zp = zpart + (ag * 2 + half) * 128 * 8;
 #pragma unroll
-      for (int o = 0; o < 8; ++o) {
-        float e, f;
-        tc::f2_unpack(acc[o], e, f);
-        z8[o] = e + f;
+      for (int rg = 0; rg < 2; ++rg) {
+        const int r = 32 * (warp & 3) + 16 * rg + g;
+        *reinterpret_cast<float2*>(zp + r * 8 + 2 * c4) = make_float2(zacc[rg][0], zacc[rg][1]);
+        *reinterpret_cast<float2*>(zp + (r + 8) * 8 + 2 * c4) = make_float2(zacc[rg][2], zacc[rg][3]);
       }
-      float4* dst = reinterpret_cast<float4*>(zpart + ((ag * 2 + half) * 128 + row) * 8);
-      dst[0] = make_float4(z8[0], z8[1], z8[2], z8[3]);
-      dst[1] = make_float4(z8[4], z8[5], z8[6], z8[7]);
     };
     // full logits of agent ag: (half-0 partial + half-1 partial) + b3
     auto logits = [&](int ag, float (&z)[16]) {
