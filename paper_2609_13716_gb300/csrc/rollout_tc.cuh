@@ -6,12 +6,12 @@
 //   obs (u8, shared memory, a constant 1 after the last feature) -> A operand in tensor
 //       memory as bf16 (exact: small integers)
 //   L1 (tensor cores): D = [o 1] [W1 b1]^T      (M = 128 envs, N = hidden0, K = KP)
-//   epilogue 1: h1 = tanh(D) split h1 = hi + lo (two bf16) into tensor memory, and b2
-//       written into the accumulator columns
-//   L2 (tensor cores): D = b2 + hi W2^T + lo W2^T  (the split keeps ~2^-17 relative
-//       precision of h1 with bf16 operands and fp32 accumulate)
-//   epilogue 2 (CUDA cores): h2 = tanh(D) in fp32 and z = W3 h2 + b3 directly (a handful
-//       of outputs: an N = 16 tensor-core instruction would cost as much as an N = 128 one)
+//   epilogue 1: h1 = tanh(D) split h1 = hi + lo (two bf16) into tensor memory
+//   L2 (tensor cores): D = hi W2^T + lo W2^T  (the split keeps ~2^-17 relative precision
+//       of h1 with bf16 operands and fp32 accumulate)
+//   epilogue 2: h2 = tanh(D + b2), split again, and z = W3 h2 + b3 by mma.sync m16n8k16
+//       from registers (16x256b accumulator loads are its fragment layout; a handful of
+//       outputs would waste an N = 16 tcgen05 instruction's round trip)
 //   sampling (ego in warps 0-3, teammate in warps 4-7), env step, trajectory write.
 //
 // Warp roles: warps 0-7 ("compute", 256 threads) build observations, run the epilogues
@@ -264,7 +264,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
           }
         } else {
           const uint64_t w0 = tc::smem_desc(wbase + d.oW2, 128u, sbo2);
-          for (int ks = 0; ks < d.H0 / 16; ++ks) tc::mma_ts(Q, P + 8 * ks, w0 + 16u * ks, idesc2, 1u);
+          for (int ks = 0; ks < d.H0 / 16; ++ks) tc::mma_ts(Q, P + 8 * ks, w0 + 16u * ks, idesc2, ks > 0);
           for (int ks = 0; ks < d.H0 / 16; ++ks) tc::mma_ts(Q, P + d.H0 / 2 + 8 * ks, w0 + 16u * ks, idesc2, 1u);
           if constexpr (kSplit) {
             const uint64_t w1 = tc::smem_desc(wbase + d.oW2lo, 128u, sbo2);
@@ -333,11 +333,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       tc::wait_st();
       operand_ready(ag, 0);
     };
-    // epilogue 1: h1 = tanh(D) -> hi | lo bf16 A operand of L2; b2 into the accumulator
+    // epilogue 1: h1 = tanh(D) -> hi | lo bf16 A operand of L2 (b2 is added in epilogue 2)
     auto epilogue1 = [&](int ag) {
       const int H = d.H0;
       const uint32_t P = tmem + (uint32_t)(ag * 256) + lane_base, Q = P + 128;
-      const float* b2 = reinterpret_cast<const float*>(pol_block(ag) + d.ob2);
       for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 32) {
         uint32_t v[32];
         tc::ld_x32(Q + c0, v);
@@ -347,29 +346,21 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         for (int j = 0; j < 16; ++j)
           tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]))),
                              hi[j], lo[j]);
-#pragma unroll
-        for (int j = 0; j < 32; j += 4) {
-          const float4 bb = *reinterpret_cast<const float4*>(b2 + c0 + j);
-          v[j] = __float_as_uint(bb.x); v[j + 1] = __float_as_uint(bb.y);
-          v[j + 2] = __float_as_uint(bb.z); v[j + 3] = __float_as_uint(bb.w);
-        }
         tc::st_x16(P + c0 / 2, hi);
         tc::st_x16(P + H / 2 + c0 / 2, lo);
-        tc::st_x32(Q + c0, v);
       }
       tc::wait_st();
       operand_ready(ag, 1);
     };
     // kSparse: h1 = tanh(c + sum over the changed features f of delta W1[:, f]) for this
-    // thread's half of the units, written like epilogue 1 (hi | lo operand of L2, b2 into
-    // the accumulator); rows past count take c alone
+    // thread's half of the units, written like epilogue 1 (hi | lo operand of L2); rows
+    // past count take c alone
     auto sparse_h1 = [&](int ag, const State& s) {
       const int H = d.H0;
       const uint32_t P = tmem + (uint32_t)(ag * 256) + lane_base, Q = P + 128;
       const float* pw = a.b.weights + (int64_t)(ag == 0 ? ego_pol : tm_pol) * a.b.mlp.stride;
       const float* W1t = pw + a.b.mlp.oW1;
       const float* cvec = pw + a.b.mlp.oC;
-      const float* b2 = reinterpret_cast<const float*>(pol_block(ag) + d.ob2);
       uint32_t e[10];
       const uint32_t mask = row < count ? Env::sparse_obs(a.b.env, s, ag, e) : 0u;
       for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 32) {
@@ -393,19 +384,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
             v[j + 3] = fmaf(dv, w4.w, v[j + 3]);
           }
         }
-        uint32_t hi[16], lo[16], bb[32];
+        uint32_t hi[16], lo[16];
 #pragma unroll
         for (int j = 0; j < 16; ++j)
           tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(v[2 * j], v[2 * j + 1])), hi[j], lo[j]);
-#pragma unroll
-        for (int j = 0; j < 32; j += 4) {
-          const float4 b4 = *reinterpret_cast<const float4*>(b2 + c0 + j);
-          bb[j] = __float_as_uint(b4.x); bb[j + 1] = __float_as_uint(b4.y);
-          bb[j + 2] = __float_as_uint(b4.z); bb[j + 3] = __float_as_uint(b4.w);
-        }
         tc::st_x16(P + c0 / 2, hi);
         tc::st_x16(P + H / 2 + c0 / 2, lo);
-        tc::st_x32(Q + c0, bb);
       }
       tc::wait_st();
       operand_ready(ag, 1);
@@ -415,10 +399,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     // takes its 32 rows as two groups of 16 and its half's units as chunks of 16; two
     // 16x256b loads of the accumulator give the thread its A fragment (rows g, g + 8 with
     // g = lane / 4; units 2c, 2c + 1 and 2c + 8, 2c + 9 of the chunk, c = lane % 4);
-    // h2 = hi + lo (two bf16) and z += hi W3^T + lo W3^T (+ hi W3lo^T for split blocks),
-    // fp32 accumulate.  The partial sums go to shared memory for the sampling half.
+    // h2 = tanh(D + b2) = hi + lo (two bf16) and z += hi W3^T + lo W3^T (+ hi W3lo^T for
+    // split blocks), fp32 accumulate.  The partial sums go to shared memory for the
+    // sampling half.
     auto epilogue2 = [&](int ag) {
       const int H = d.H1;
+      const float* b2 = reinterpret_cast<const float*>(pol_block(ag) + d.ob2);
       const uint32_t Qq = tmem + (uint32_t)(ag * 256 + 128) + ((uint32_t)((warp & 3) * 32) << 16);
       const uint32_t* W3f = reinterpret_cast<const uint32_t*>(pol_block(ag) + d.oW3);
       const uint32_t* W3l = W3f + H * 4;  // split blocks: the remainders
@@ -428,6 +414,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 16) {
         const int j = c0 >> 4;
         const uint2 bw = *reinterpret_cast<const uint2*>(W3f + (j * 32 + lane) * 2);
+        const uint64_t bA = *reinterpret_cast<const uint64_t*>(b2 + c0 + 2 * c4);
+        const uint64_t bB = *reinterpret_cast<const uint64_t*>(b2 + c0 + 8 + 2 * c4);
         uint2 bl = make_uint2(0u, 0u);
         if constexpr (kSplit) bl = *reinterpret_cast<const uint2*>(W3l + (j * 32 + lane) * 2);
 #pragma unroll
@@ -437,10 +425,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
           tc::ld_16x256b(Qq + ((uint32_t)(16 * rg) << 16) + (uint32_t)(c0 + 8), t1);
           tc::wait_ld();
           uint32_t ahi[4], alo[4];
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(t0[0]), __uint_as_float(t0[1]))), ahi[0], alo[0]);
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(t0[2]), __uint_as_float(t0[3]))), ahi[1], alo[1]);
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(t1[0]), __uint_as_float(t1[1]))), ahi[2], alo[2]);
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(t1[2]), __uint_as_float(t1[3]))), ahi[3], alo[3]);
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t0[0]), __uint_as_float(t0[1])), bA)),
+                             ahi[0], alo[0]);
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t0[2]), __uint_as_float(t0[3])), bA)),
+                             ahi[1], alo[1]);
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t1[0]), __uint_as_float(t1[1])), bB)),
+                             ahi[2], alo[2]);
+          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t1[2]), __uint_as_float(t1[3])), bB)),
+                             ahi[3], alo[3]);
           tc::mma_m16n8k16_bf16(zacc[rg], ahi, bw.x, bw.y);
           tc::mma_m16n8k16_bf16(zacc[rg], alo, bw.x, bw.y);
           if constexpr (kSplit) tc::mma_m16n8k16_bf16(zacc[rg], ahi, bl.x, bl.y);
