@@ -841,8 +841,14 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
   // the sparse-first-layer tensor-core kernel does plain collection; IPPO there runs on
   // the CUDA-core kernel
   const bool use_tc = c->tc && !(c->tcd.sparse && out1);
-  const int M = use_tc ? 128
-                       : spread_rows(c, fit_rows(c, 128), 0, [&](int m) { return (int64_t)group_tiles(Nall, m); });
+  int M = 128;
+  if (use_tc) {
+    // a tensor-core tile's step takes about as long for 32 rows as for 128: while the
+    // batch would leave SMs idle, cut the teammate blocks into smaller tiles
+    while (M > 32 && group_tiles(Nall, M / 2) <= c->n_sms) M /= 2;
+  } else {
+    M = spread_rows(c, fit_rows(c, 128), 0, [&](int m) { return (int64_t)group_tiles(Nall, m); });
+  }
 
   GroupArgs ga{};
   ga.key = batch_of(c).key;
