@@ -86,3 +86,24 @@ def test_lbf12_ippo_and_per_episode_calls():
     aht.aht_sync(ctx)
     check_rollout(wl, pop_np, traj, st, wl.env_seed, T, T, 0, [2, 3, 4], ep_step=ep,
                   resample=True, teammates=tms)
+
+
+def test_lbf9x9_xplay_and_ppo_take_the_sparse_path():
+    """A grid between the two paper sizes: 9x9 x 4 channels = 324 features (past 256
+    tensor-memory columns), random 1-2 foods and level 2 agents, cross-play and a PPO call."""
+    require_gpu()
+    base = W.WORKLOADS["lbf12x12_xplay_8x16x128"]
+    env = dataclasses.replace(base.env, width=9, height=9, n_food=2, max_agent_level=2, episode_len=40)
+    wl = dataclasses.replace(base, env=env, n_policies=6, value_head=(1,) + (0,) * 5)
+    ego, tm, P = [0, 1], [2, 5], 50
+    ctx, pop_np = make_ctx(wl, len(ego) * len(tm) * P)
+    out = run_xplay(ctx, ego, tm, P, 40)
+    check(wl, pop_np, ego, tm, P, 40, out, wl.env_seed)
+    N, T = 200, 25
+    ctx2, _ = make_ctx(wl, N, pop_np=pop_np)
+    d, _ = oracle_of(wl.env, pop_np)
+    st = O.reset_all(d, wl.env_seed, N)
+    traj = aht.traj_buffers(ctx2, T)
+    aht.aht_rollout(ctx2, 0, [3, 4], T, traj)
+    aht.aht_sync(ctx2)
+    check_rollout(wl, pop_np, traj, st, wl.env_seed, 0, T, 0, [3, 4])
