@@ -89,8 +89,11 @@ def test_step_counter_advances_between_calls():
 
 
 @pytest.mark.parametrize("name", ["lbf7x7_xplay_8x16x256", "overcooked5x4_xplay_8x8x64",
-                                  "hanabi_xplay_16x16x32"])
+                                  "hanabi_xplay_16x16x32", "lbf7x7_xplay_heuristics_8x12x256",
+                                  "lbf12x12_xplay_8x16x128", "minihanabi_xplay_16x16x32"])
 def test_full_size_xplay_sampled(name):
+    """Every cross-play workload the bench times, in its launch configuration; the oracle
+    replays a sample of the envs."""
     require_gpu()
     wl = W.WORKLOADS[name]
     n = wl.xplay_envs
