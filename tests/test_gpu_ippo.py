@@ -21,27 +21,29 @@ from test_gpu_rollout import check_rollout
 pytestmark = pytest.mark.gpu
 
 
-def check_seat1(wl, pop_np, traj0, traj1, states, seed, step0, T, p0, p1):
+def check_seat1(wl, pop_np, traj0, traj1, states, seed, step0, T, p0, p1, env_ids=None):
     d, pols = oracle_of(wl.env, pop_np)
-    acts = np.stack([np_(traj0["actions"]), np_(traj0["tm_actions"])], -1)
-    ref = O.rollout(d, pols, seed, states, step0, T, p0, [p1], forced=acts, n_threads=8)
+    sel = slice(None) if env_ids is None else env_ids
+    g = lambda k: np_(traj1[k])[:, sel] if traj1[k].dim() > 1 else np_(traj1[k])[sel]
+    acts = np.stack([np_(traj0["actions"])[:, sel], np_(traj0["tm_actions"])[:, sel]], -1)
+    ref = O.rollout(d, pols, seed, states, step0, T, p0, [p1], forced=acts, n_threads=8,
+                    env_ids=env_ids)
     assert ref["rc"] == 0
-    assert np.array_equal(np_(traj1["obs"]), ref["obs_tm"]), "seat-1 observations"
-    assert np.array_equal(np_(traj1["actions"]), np_(traj0["tm_actions"]))
-    assert np.array_equal(np_(traj1["tm_actions"]), np_(traj0["actions"]))
-    assert np.array_equal(np_(traj1["rewards"]), ref["rewards"])
-    assert np.array_equal(np_(traj1["dones"]), ref["dones"])
-    ok, worst = close(np_(traj1["logp"]), ref["logp_tm"])
+    assert np.array_equal(g("obs"), ref["obs_tm"]), "seat-1 observations"
+    assert np.array_equal(g("actions"), acts[..., 1])
+    assert np.array_equal(g("tm_actions"), acts[..., 0])
+    assert np.array_equal(g("rewards"), ref["rewards"])
+    assert np.array_equal(g("dones"), ref["dones"])
+    ok, worst = close(g("logp"), ref["logp_tm"])
     assert ok, f"seat-1 logp {worst:.3g}"
-    ok, worst = close(np_(traj1["values"]), ref["values_tm"])
+    ok, worst = close(g("values"), ref["values_tm"])
     assert ok, f"seat-1 values {worst:.3g}"
-    ok, worst = close(np_(traj1["last_value"]), ref["last_value_tm"])
+    ok, worst = close(g("last_value"), ref["last_value_tm"])
     assert ok, f"seat-1 V_T {worst:.3g}"
-    a_ref, t_ref = O.gae(np_(traj1["rewards"]), np_(traj1["values"]), np_(traj1["dones"]),
-                         np_(traj1["last_value"]), 0.99, 0.95)
-    ok, worst = close(np_(traj1["advantages"]), a_ref, GAE_REL)
+    a_ref, t_ref = O.gae(g("rewards"), g("values"), g("dones"), g("last_value"), 0.99, 0.95)
+    ok, worst = close(g("advantages"), a_ref, GAE_REL)
     assert ok, f"seat-1 advantages {worst:.3g}"
-    ok, worst = close(np_(traj1["targets"]), t_ref, GAE_REL)
+    ok, worst = close(g("targets"), t_ref, GAE_REL)
     assert ok, f"seat-1 targets {worst:.3g}"
 
 
@@ -140,3 +142,19 @@ def test_ippo_rejects_rule_and_out_of_range_seat1():
     for bad in (-1, 2):
         with pytest.raises(aht.AhtError):
             aht.aht_rollout_ippo(ctx, 0, bad, 4, t0, t1)
+
+
+def test_ippo_full_size_16384x128_sampled():
+    """The bench's IPPO configuration; the oracle replays a sample of the envs."""
+    require_gpu()
+    wl = W.WORKLOADS["lbf7x7_ippo_16384x128"]
+    ctx, pop_np = make_ctx(wl, wl.n_envs)
+    t0, t1 = aht.traj_buffers(ctx, wl.T), aht.traj_buffers(ctx, wl.T)
+    aht.aht_rollout_ippo(ctx, 0, 1, wl.T, t0, t1)
+    aht.aht_sync(ctx)
+    ids = np.unique(np.concatenate([[0, wl.n_envs - 1], np.random.default_rng(2).integers(0, wl.n_envs, 30)]))
+    d, _ = oracle_of(wl.env, pop_np)
+    st = O.reset_envs(d, wl.env_seed, ids)
+    st1 = st.copy()
+    check_rollout(wl, pop_np, t0, st, wl.env_seed, 0, wl.T, 0, [1], env_ids=ids)
+    check_seat1(wl, pop_np, t0, t1, st1, wl.env_seed, 0, wl.T, 0, 1, env_ids=ids)

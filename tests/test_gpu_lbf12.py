@@ -107,3 +107,17 @@ def test_lbf9x9_xplay_and_ppo_take_the_sparse_path():
     aht.aht_rollout(ctx2, 0, [3, 4], T, traj)
     aht.aht_sync(ctx2)
     check_rollout(wl, pop_np, traj, st, wl.env_seed, 0, T, 0, [3, 4])
+
+
+def test_lbf12_ppo_full_size_4096x128_sampled():
+    """The bench's 12x12 PPO configuration (32-env tiles); the oracle replays a sample."""
+    require_gpu()
+    wl = W.WORKLOADS["lbf12x12_ppo_4096x128"]
+    ctx, pop_np = make_ctx(wl, wl.n_envs)
+    traj = aht.traj_buffers(ctx, wl.T)
+    aht.aht_rollout(ctx, wl.ego_id, wl.pool, wl.T, traj)
+    aht.aht_sync(ctx)
+    ids = np.unique(np.concatenate([[0, wl.n_envs - 1], np.random.default_rng(3).integers(0, wl.n_envs, 30)]))
+    d, _ = oracle_of(wl.env, pop_np)
+    st = O.reset_envs(d, wl.env_seed, ids)
+    check_rollout(wl, pop_np, traj, st, wl.env_seed, 0, wl.T, wl.ego_id, list(wl.pool), env_ids=ids)
