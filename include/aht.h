@@ -126,8 +126,9 @@ typedef struct aht_pop_desc {
 #define AHT_LBF_N_HEURISTICS 12
 #define AHT_LBF_HEURISTIC(k) (-1 - (k))
 
-/* Creates a context for up to n_envs concurrent envs (PPO state and cross-play batch
- * capacity), packs the population and resets every env with `seed` (step counter 0).
+/* Creates a context for up to n_envs concurrent envs (1 <= n_envs <= 2^30; PPO state and
+ * cross-play batch capacity), packs the population and resets every env with `seed`
+ * (step counter 0).
  * cuda_stream is a cudaStream_t (NULL = default stream).  Allocates all device memory
  * the context will ever use.  Returns AHT_EINVAL, AHT_ENOMEM or AHT_ECUDA on failure
  * (*out is then NULL). */
