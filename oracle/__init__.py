@@ -21,7 +21,8 @@ import numpy as np
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _BUILD = os.path.join(_HERE, "_build")
 _SO = os.path.join(_BUILD, "liboracle.so")
-_SRC = [os.path.join(_HERE, "aht_oracle.cpp"), os.path.join(_HERE, "ppo_oracle.cpp")]
+_SRC = [os.path.join(_HERE, "aht_oracle.cpp"), os.path.join(_HERE, "ppo_oracle.cpp"),
+        os.path.join(_HERE, "s5_oracle.cpp")]
 _HDR = os.path.join(_HERE, "aht_oracle.h")
 _lock = threading.Lock()
 _lib = None
@@ -508,3 +509,77 @@ def ppo_update(net, params, m, v, t, batch: PpoBatchNp, hp, n_threads=1):
 
 def lbf_heuristic(d, state, seat, k):
     return int(lib().orc_lbf_heuristic(C.byref(d), C.byref(state), seat, k))
+
+
+# ---- S5 recurrent actor-critic (s5_oracle.cpp) ------------------------------------------
+class S5Net(C.Structure):
+    _fields_ = [("obs_dim", C.c_int32), ("n_actions", C.c_int32), ("H", C.c_int32),
+                ("P", C.c_int32), ("F", C.c_int32),
+                ("We1", _P), ("be1", _P), ("We2", _P), ("be2", _P),
+                ("lam_re", _P), ("lam_im", _P), ("log_dt", _P),
+                ("B_re", _P), ("B_im", _P), ("C_re", _P), ("C_im", _P), ("Dv", _P),
+                ("Wa", _P * 4), ("ba", _P * 4), ("Wc", _P * 4), ("bc", _P * 4)]
+
+
+S5_KEYS = ("We1", "be1", "We2", "be2", "lam_re", "lam_im", "log_dt", "B_re", "B_im",
+           "C_re", "C_im", "Dv")
+
+
+class S5:
+    """fp64 copies of an S5 actor-critic's parameters (a dict of arrays: the S5_KEYS and
+    lists Wa, ba, Wc, bc of four arrays each) and the oracle's entry points."""
+
+    def __init__(self, params):
+        self.p = {k: np.ascontiguousarray(np.asarray(params[k], np.float64)) for k in S5_KEYS}
+        for k in ("Wa", "ba", "Wc", "bc"):
+            self.p[k] = [np.ascontiguousarray(np.asarray(a, np.float64)) for a in params[k]]
+        H, K = self.p["We1"].shape
+        self.H, self.K = H, K
+        self.P = self.p["lam_re"].shape[0]
+        self.F = self.p["Wa"][0].shape[0]
+        self.A = self.p["Wa"][3].shape[0]
+        net = S5Net(obs_dim=K, n_actions=self.A, H=H, P=self.P, F=self.F)
+        for k in S5_KEYS:
+            setattr(net, k, _ptr(self.p[k]))
+        for k in ("Wa", "ba", "Wc", "bc"):
+            arr = (_P * 4)(*[_ptr(a) for a in self.p[k]])
+            setattr(net, k, arr)
+        self.net = net
+        L = lib()
+        if not getattr(L, "_s5_typed", False):
+            L.orc_s5_encode.argtypes = [C.POINTER(S5Net), _P, _P]
+            L.orc_s5_ssm_step.argtypes = [C.POINTER(S5Net), _P, C.c_int32, _P, _P]
+            L.orc_s5_heads.argtypes = [C.POINTER(S5Net), _P, _P, _P, _P]
+            L.orc_s5_step.argtypes = [C.POINTER(S5Net), _P, _P, _P, C.c_int64, _P, _P, _P, C.c_int32]
+            L._s5_typed = True
+
+    def encode(self, obs):
+        obs = np.ascontiguousarray(obs, np.uint8)
+        u = np.zeros(self.H)
+        lib().orc_s5_encode(C.byref(self.net), _ptr(obs), _ptr(u))
+        return u
+
+    def ssm_step(self, u, reset, state):
+        u = np.ascontiguousarray(u, np.float64)
+        y = np.zeros(self.H)
+        lib().orc_s5_ssm_step(C.byref(self.net), _ptr(u), int(reset), _ptr(state), _ptr(y))
+        return y
+
+    def heads(self, v, legal=None):
+        v = np.ascontiguousarray(v, np.float64)
+        logits, value = np.zeros(self.A), np.zeros(1)
+        legal = None if legal is None else np.ascontiguousarray(legal, np.uint8)
+        lib().orc_s5_heads(C.byref(self.net), _ptr(v), _ptr(legal), _ptr(logits), _ptr(value))
+        return logits, float(value[0])
+
+    def step(self, obs, reset, state, legal=None, n_threads=8):
+        """One step for n envs; state [n][2P] (float64) is updated in place."""
+        obs = np.ascontiguousarray(obs, np.uint8)
+        reset = np.ascontiguousarray(reset, np.uint8)
+        n = obs.shape[0]
+        assert state.dtype == np.float64 and state.shape == (n, 2 * self.P) and state.flags.c_contiguous
+        legal = None if legal is None else np.ascontiguousarray(legal, np.uint8)
+        logits, values = np.zeros((n, self.A)), np.zeros(n)
+        lib().orc_s5_step(C.byref(self.net), _ptr(obs), _ptr(reset), _ptr(legal), n, _ptr(state),
+                          _ptr(logits), _ptr(values), n_threads)
+        return logits, values

@@ -367,6 +367,45 @@ void orc_ppo_update(const orc_ppo_net* n, double* params, double* m, double* v, 
 /* Policy outputs z for n observations (u8 [n][obs_dim]) -> [n][n_out]. */
 void orc_policy_outputs(const orc_mlp* p, const uint8_t* obs, int64_t n, double* out);
 
+/* ---- S5 recurrent actor-critic (App. B "Training protocol", Sec. 4: recurrent S5 ego
+ * agents) ------------------------------------------------------------------------------
+ * The paper: observations go through dense layers into an S5 sequence model of model
+ * size H = 128 and SSM state size P = 128 (Smith, Warrington, Linderman, "Simplified State
+ * Space Layers for Sequence Modeling", ICLR 2023), then separate MLP heads with three
+ * hidden layers of 1024 units give a masked categorical policy and a value.  Readings
+ * (the rest is unstated):
+ *   encoder u = relu(We2 relu(We1 o + be1) + be2)   (o the u8 observation, E = H units)
+ *   SSM, P diagonal complex modes, zero-order hold with step dt_p = exp(log_dt_p):
+ *     lbar_p = exp(lambda_p dt_p),  Bbar[p][:] = (lbar_p - 1) / lambda_p * B[p][:]
+ *     x_t = lbar (.) x_{t-1} + Bbar u_t  (x_{t-1} = 0 at an episode's first step)
+ *     y_t = Re(C x_t) + D (.) u_t          (B: P x H complex, C: H x P complex, D: H real)
+ *   v_t = u_t + gelu(y_t),  gelu(a) = a Phi(a) (the exact form, Phi the normal CDF)
+ *   heads: relu MLPs H -> F -> F -> F -> n_actions (actor) and -> 1 (critic), F = 1024;
+ *   the actor's logits are masked by the legal actions when given.
+ * The state is carried per env as 2P doubles (real parts, then imaginary parts). */
+typedef struct orc_s5_net {
+  int32_t obs_dim, n_actions, H, P, F;
+  const double *We1, *be1, *We2, *be2;       /* [H][obs_dim] [H] [H][H] [H] */
+  const double *lam_re, *lam_im, *log_dt;    /* [P] each, lam_re < 0 */
+  const double *B_re, *B_im;                 /* [P][H] */
+  const double *C_re, *C_im;                 /* [H][P] */
+  const double *Dv;                          /* [H] */
+  const double *Wa[4], *ba[4];               /* actor [F][H] [F][F] [F][F] [A][F], biases */
+  const double *Wc[4], *bc[4];               /* critic [F][H] [F][F] [F][F] [1][F], biases */
+} orc_s5_net;
+/* u = encoder(o) [H]. */
+void orc_s5_encode(const orc_s5_net* n, const uint8_t* obs, double* u);
+/* One SSM step: state [2P] in/out (zeroed first when reset), y [H]. */
+void orc_s5_ssm_step(const orc_s5_net* n, const double* u, int32_t reset, double* state, double* y);
+/* Heads on v [H]: logits [n_actions] (-inf where legal[a] == 0, legal may be NULL), value. */
+void orc_s5_heads(const orc_s5_net* n, const double* v, const uint8_t* legal, double* logits,
+                  double* value);
+/* One full step for n envs: obs u8 [n][obs_dim], reset [n], legal u8 [n][A] or NULL,
+ * state [n][2P] in/out -> logits [n][A], values [n]. */
+void orc_s5_step(const orc_s5_net* net, const uint8_t* obs, const uint8_t* reset,
+                 const uint8_t* legal, int64_t n, double* state, double* logits, double* values,
+                 int32_t n_threads);
+
 #ifdef __cplusplus
 }
 #endif

@@ -206,3 +206,42 @@ def xp_matrix(seed: int, n_ego: int, n_tm: int, scale: float = 1.0,
     if quantum > 0:
         m = np.round(m / quantum) * quantum
     return m.astype(np.float32)
+
+
+def s5_params(seed: int, obs_dim: int, n_actions: int, H: int = 128, P: int = 128, F: int = 1024):
+    """Synthetic parameters of the recurrent S5 actor-critic (random init, no training).
+
+    Dense layers (encoder and both heads) are N(0, 1/fan_in) and rounded to bf16 (the
+    GPU runs them as bf16 GEMMs); the SSM's continuous-time modes have decay rates
+    exp(U(log 0.05, 0)) (lambda_re = -rate), frequencies U(-pi, pi) and log steps
+    U(log 1e-3, log 1e-1); B and C are complex N(0, 1/(2 fan_in)), D is N(0, 1); all fp32.
+    Returns a dict of float32 arrays: We1 be1 We2 be2 lam_re lam_im log_dt B_re B_im C_re
+    C_im Dv, and lists Wa ba Wc bc of the heads' four layers."""
+    rng = np.random.Generator(np.random.Philox(90000 + seed))
+    f32 = lambda a: np.asarray(a, np.float32)
+
+    def dense(rows, cols):
+        W = round_to_bf16(f32(rng.standard_normal((rows, cols)) / np.sqrt(cols)))
+        b = round_to_bf16(f32(rng.standard_normal(rows) * 0.1))
+        return W, b
+
+    p = {}
+    p["We1"], p["be1"] = dense(H, obs_dim)
+    p["We2"], p["be2"] = dense(H, H)
+    p["lam_re"] = f32(-np.exp(rng.uniform(np.log(0.05), 0.0, P)))
+    p["lam_im"] = f32(rng.uniform(-np.pi, np.pi, P))
+    p["log_dt"] = f32(rng.uniform(np.log(1e-3), np.log(1e-1), P))
+    p["B_re"] = f32(rng.standard_normal((P, H)) / np.sqrt(2 * H))
+    p["B_im"] = f32(rng.standard_normal((P, H)) / np.sqrt(2 * H))
+    p["C_re"] = f32(rng.standard_normal((H, P)) / np.sqrt(2 * P))
+    p["C_im"] = f32(rng.standard_normal((H, P)) / np.sqrt(2 * P))
+    p["Dv"] = f32(rng.standard_normal(H))
+    for head, out in (("a", n_actions), ("c", 1)):
+        dims = [H, F, F, F, out]
+        Ws, bs = [], []
+        for i in range(4):
+            W, b = dense(dims[i + 1], dims[i])
+            Ws.append(W)
+            bs.append(b)
+        p["W" + head], p["b" + head] = Ws, bs
+    return p
