@@ -358,6 +358,43 @@ aht_status aht_learner_push(aht_learner* L, aht_ctx* ctx, int32_t policy);
  * expired (the status word is then cleared). */
 aht_status aht_learner_sync(aht_learner* L);
 
+/* ---- S5 recurrent actor-critic (App. B training protocol; Sec. 4: recurrent S5 egos) ---
+ * A dense relu encoder (H units, two layers), an S5 layer (Smith et al., ICLR 2023) of
+ * model size H and P diagonal complex modes discretised by zero-order hold, a residual
+ * GELU, and two relu MLP heads of three F-unit hidden layers (actor: n_actions logits
+ * masked by the legal actions; critic: one value):
+ *   u = relu(We2 relu(We1 o + be1) + be2)
+ *   lbar = exp(lambda dt), Bbar = (lbar - 1) / lambda * B, dt = exp(log_dt)
+ *   x_t = lbar (.) x_{t-1} + Bbar u_t  (x_{t-1} = 0 where reset),  y = Re(C x_t) + D (.) u
+ *   v = u + gelu(y) (gelu(a) = a Phi(a)),  logits / value = heads(v).
+ * The paper gives H = P = 128 and F = 1024; the rest is this library's reading.  Dense
+ * layers run as bf16 GEMMs (weights rounded to bf16 at create; activations carried as
+ * two bf16, hi + lo, ~2^-17 relative, fp32 accumulate); the SSM in fp32 (lbar and Bbar
+ * computed in fp64 at create).  Parameters are host fp32 arrays, row-major [out][in]. */
+typedef struct aht_s5_params {
+  int32_t obs_dim, n_actions, H, P, F;  /* H, P multiples of 16, F of 16; n_actions <= 32 */
+  const float *We1, *be1, *We2, *be2;   /* [H][obs_dim] [H] [H][H] [H] */
+  const float *lam_re, *lam_im, *log_dt;/* [P] (lam_re < 0) */
+  const float *B_re, *B_im;             /* [P][H] */
+  const float *C_re, *C_im;             /* [H][P] */
+  const float *D;                       /* [H] */
+  const float *Wa[4], *ba[4];           /* actor [F][H] [F][F] [F][F] [n_actions][F] */
+  const float *Wc[4], *bc[4];           /* critic [F][H] [F][F] [F][F] [1][F] */
+} aht_s5_params;
+typedef struct aht_s5 aht_s5;           /* opaque, library-owned */
+/* Allocates everything a step of up to max_envs envs needs (weights, scratch, a GEMM
+ * workspace).  cuda_stream: a cudaStream_t (NULL = default). */
+aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_stream, aht_s5** out);
+void aht_s5_destroy(aht_s5* s);
+/* One policy step of n envs (device arrays): obs u8 [n][obs_dim], reset u8 [n] (1 zeroes
+ * the env's state first: the first step of an episode), legal u8 [n][n_actions] or NULL,
+ * state f32 [n][2P] in/out (real parts, then imaginary parts) -> logits f32
+ * [n][n_actions] (-inf where illegal), values f32 [n].  1 <= n <= max_envs.
+ * Asynchronous on the creation stream; aht_s5_sync reports errors. */
+aht_status aht_s5_step(aht_s5* s, const uint8_t* obs, const uint8_t* reset, const uint8_t* legal,
+                       int64_t n, float* state, float* logits, float* values);
+aht_status aht_s5_sync(aht_s5* s);
+
 /* Stateless GAE (App. C "PPO ego"), time-major [T][n_envs] device arrays:
  *   delta_t = r_t + gamma (1 - d_t) V_{t+1} - V_t,
  *   A_t = delta_t + gamma lambda (1 - d_t) A_{t+1},  V_T = v_last,  A_T = 0,

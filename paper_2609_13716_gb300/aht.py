@@ -26,7 +26,8 @@ EXPORTED = ["aht_create", "aht_destroy", "aht_reset", "aht_rollout", "aht_xplay_
             "aht_xplay_matrix_static", "aht_debug_tanh", "aht_debug_expire_wait",
             "aht_xp_stats", "aht_learner_create", "aht_learner_destroy", "aht_learner_n_params",
             "aht_ppo_update", "aht_ppo_grad", "aht_learner_get", "aht_learner_set",
-            "aht_learner_push", "aht_learner_sync", "aht_rollout_ippo", "aht_rollout_resample"]
+            "aht_learner_push", "aht_learner_sync", "aht_rollout_ippo", "aht_rollout_resample",
+            "aht_s5_create", "aht_s5_destroy", "aht_s5_step", "aht_s5_sync"]
 
 
 class AhtError(RuntimeError):
@@ -109,6 +110,14 @@ def load() -> C.CDLL:
             L.aht_reset.argtypes = [vp, u64]
             L.aht_rollout.argtypes = [vp, i32, C.POINTER(i32), i32, i32, C.POINTER(Traj)]
             L.aht_rollout_ippo.argtypes = [vp, i32, i32, i32, C.POINTER(Traj), C.POINTER(Traj)]
+            L.aht_s5_create.argtypes = [C.POINTER(S5Params), i64, vp, C.POINTER(vp)]
+            L.aht_s5_create.restype = C.c_int
+            L.aht_s5_destroy.argtypes = [vp]
+            L.aht_s5_destroy.restype = None
+            L.aht_s5_step.argtypes = [vp, vp, vp, vp, i64, vp, vp, vp]
+            L.aht_s5_step.restype = C.c_int
+            L.aht_s5_sync.argtypes = [vp]
+            L.aht_s5_sync.restype = C.c_int
             L.aht_rollout_resample.argtypes = [vp, i32, C.POINTER(i32), i32, i32, C.POINTER(Traj), vp]
             L.aht_xplay_matrix.argtypes = [vp, C.POINTER(i32), i32, C.POINTER(i32), i32, i32, i32, C.POINTER(XplayOut)]
             L.aht_gae.argtypes = [vp, vp, vp, vp, i64, i32, C.c_float, C.c_float, vp, vp, vp]
@@ -499,3 +508,76 @@ def aht_learner_push(learner: Learner, ctx: Context, policy):
 
 def aht_learner_sync(learner: Learner):
     _check(load().aht_learner_sync(learner.handle))
+
+
+# ---- S5 recurrent actor-critic ----------------------------------------------------------
+_FP = C.POINTER(C.c_float)
+
+
+class S5Params(C.Structure):
+    _fields_ = [("obs_dim", C.c_int32), ("n_actions", C.c_int32), ("H", C.c_int32),
+                ("P", C.c_int32), ("F", C.c_int32),
+                ("We1", _FP), ("be1", _FP), ("We2", _FP), ("be2", _FP),
+                ("lam_re", _FP), ("lam_im", _FP), ("log_dt", _FP),
+                ("B_re", _FP), ("B_im", _FP), ("C_re", _FP), ("C_im", _FP), ("D", _FP),
+                ("Wa", _FP * 4), ("ba", _FP * 4), ("Wc", _FP * 4), ("bc", _FP * 4)]
+
+
+class S5Policy:
+    """Owns an aht_s5 handle (aht_s5_destroy on close / garbage collection)."""
+
+    def __init__(self, handle, obs_dim, n_actions, P):
+        self.handle, self.obs_dim, self.n_actions, self.P = handle, obs_dim, n_actions, P
+
+    def close(self):
+        if self.handle:
+            load().aht_s5_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def aht_s5_create(params, max_envs, stream=None) -> S5Policy:
+    """params: dict of host float32 numpy arrays (the keys of workloads.s5_params)."""
+    import numpy as np
+    keep = {}
+
+    def fp(a):
+        a = np.ascontiguousarray(a, np.float32)
+        keep[id(a)] = a
+        return a.ctypes.data_as(_FP)
+
+    H, K = params["We1"].shape
+    P = params["lam_re"].shape[0]
+    F = params["Wa"][0].shape[0]
+    A = params["Wa"][3].shape[0]
+    sp = S5Params(obs_dim=K, n_actions=A, H=H, P=P, F=F)
+    for k, f in (("We1", "We1"), ("be1", "be1"), ("We2", "We2"), ("be2", "be2"), ("lam_re", "lam_re"),
+                 ("lam_im", "lam_im"), ("log_dt", "log_dt"), ("B_re", "B_re"), ("B_im", "B_im"),
+                 ("C_re", "C_re"), ("C_im", "C_im"), ("Dv", "D")):
+        setattr(sp, f, fp(params[k]))
+    for k in ("Wa", "ba", "Wc", "bc"):
+        setattr(sp, k, (_FP * 4)(*[fp(a) for a in params[k]]))
+    h = C.c_void_p()
+    st = None if stream is None else C.c_void_p(stream.cuda_stream)
+    _check(load().aht_s5_create(C.byref(sp), int(max_envs), st, C.byref(h)))
+    return S5Policy(h, K, A, P)
+
+
+def aht_s5_step(pol: S5Policy, obs, reset, state, logits, values, legal=None):
+    n = obs.shape[0]
+    u8, f32 = torch.uint8, torch.float32
+    _check(load().aht_s5_step(pol.handle, _ptr(obs, u8, (n, pol.obs_dim), "obs"),
+                              _ptr(reset, u8, (n,), "reset"),
+                              _ptr(legal, u8, (n, pol.n_actions), "legal"), n,
+                              _ptr(state, f32, (n, 2 * pol.P), "state"),
+                              _ptr(logits, f32, (n, pol.n_actions), "logits"),
+                              _ptr(values, f32, (n,), "values")))
+
+
+def aht_s5_sync(pol: S5Policy):
+    _check(load().aht_s5_sync(pol.handle))

@@ -588,6 +588,10 @@ int spread_rows(const aht_ctx* c, int M, int which, F tiles) {
 
 }  // namespace
 
+namespace aht {
+aht_status set_last_error(aht_status s, const char* msg) { return fail(s, msg); }
+}  // namespace aht
+
 extern "C" {
 
 const char* aht_last_error(void) { return g_err.c_str(); }

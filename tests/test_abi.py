@@ -11,7 +11,7 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 def declared_symbols():
     src = open(os.path.join(ROOT, "include", "aht.h")).read()
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-    return sorted(set(re.findall(r"\b(aht_[a-z_]+)\s*\(", src)))
+    return sorted(set(re.findall(r"\b(aht_[a-z0-9_]+)\s*\(", src)))
 
 
 @pytest.fixture(scope="module")

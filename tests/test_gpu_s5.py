@@ -1,0 +1,78 @@
+"""The recurrent S5 actor-critic step on the GPU (aht_s5_step) against the fp64 oracle,
+at the paper's sizes (H = P = 128, heads of three 1024-unit layers) over an LBF 7x7
+observation stream: a sequence of steps with episode resets and legal-action masks.
+Tolerance: logits and values |g - o| <= 1e-4 |o| + 1e-4 rms(o) (the dense layers carry
+their activations as two bf16, ~2^-17 relative, with fp32 accumulation; the SSM is fp32);
+the recurrent state 1e-4 likewise."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2609_13716_gb300 import aht
+from paper_2609_13716_gb300 import workloads as W
+
+from gpu_util import close, np_, require_gpu
+
+pytestmark = pytest.mark.gpu
+
+
+def lbf_observations(T, N, seed):
+    """Real LBF 7x7 observations of seat 0 along forced random play (with auto-resets)."""
+    d = O.env_desc(O.LBF, 7, 7, 3, 3, 8)
+    st = O.reset_all(d, seed, N)
+    rng = np.random.default_rng(seed)
+    obs, resets = [], []
+    reset = np.ones(N, np.uint8)
+    for t in range(T):
+        rc, _, _, dones, ob2 = O.step_forced(d, seed, t, st, rng.integers(0, 6, (N, 2)).astype(np.uint8))
+        obs.append(ob2[:, 0].copy())
+        resets.append(reset.copy())
+        reset = dones.astype(np.uint8)
+    return np.stack(obs), np.stack(resets)
+
+
+@pytest.mark.parametrize("N,T", [(300, 6), (1, 3)])
+def test_s5_steps_match_the_oracle(N, T):
+    require_gpu()
+    params = W.s5_params(0, 196, 6)
+    pol = aht.aht_s5_create(params, max(N, 64))
+    net = O.S5(params)
+    obs, resets = lbf_observations(T, N, 5)
+    rng = np.random.default_rng(6)
+    legal = (rng.random((T, N, 6)) < 0.8).astype(np.uint8)
+    legal[..., 0] = 1
+    state = torch.zeros(N, 2 * net.P, device="cuda")
+    state_ref = np.zeros((N, 2 * net.P))
+    logits = torch.empty(N, 6, device="cuda")
+    values = torch.empty(N, device="cuda")
+    for t in range(T):
+        aht.aht_s5_step(pol, torch.from_numpy(obs[t]).cuda(), torch.from_numpy(resets[t]).cuda(), state,
+                        logits, values, torch.from_numpy(legal[t]).cuda())
+        aht.aht_s5_sync(pol)
+        lg_ref, v_ref = net.step(obs[t], resets[t], state_ref, legal[t])
+        lg = np_(logits)
+        assert np.array_equal(np.isinf(lg), legal[t] == 0), "masked actions"
+        finite = legal[t] == 1
+        ok, worst = close(lg[finite], lg_ref[finite])
+        assert ok, f"logits at step {t}: {worst:.3g}"
+        ok, worst = close(np_(values), v_ref)
+        assert ok, f"values at step {t}: {worst:.3g}"
+        ok, worst = close(np_(state), state_ref)
+        assert ok, f"state at step {t}: {worst:.3g}"
+    pol.close()
+
+
+def test_s5_rejects_bad_sizes():
+    require_gpu()
+    params = W.s5_params(1, 196, 6, H=16, P=16, F=32)
+    bad = dict(params)
+    bad["lam_re"] = -bad["lam_re"]          # growing modes
+    with pytest.raises(aht.AhtError):
+        aht.aht_s5_create(bad, 8)
+    pol = aht.aht_s5_create(params, 8)
+    obs = torch.zeros(9, 196, dtype=torch.uint8, device="cuda")
+    with pytest.raises(aht.AhtError):       # more envs than max_envs
+        aht.aht_s5_step(pol, obs, torch.zeros(9, dtype=torch.uint8, device="cuda"),
+                        torch.zeros(9, 32, device="cuda"), torch.empty(9, 6, device="cuda"),
+                        torch.empty(9, device="cuda"))
