@@ -391,6 +391,7 @@ def run_ours(args):
         line["ippo"] = run_ippo(aht, W, torch, stream, bf16_peak)
         line["resample"] = run_resample(aht, wl, pop, torch, stream, bf16_peak)
         line["lbf12x12_ppo"] = run_lbf12_ppo(aht, W, torch, stream, bf16_peak)
+        line["s5"] = run_s5(aht, W, torch, stream, bf16_peak)
     if not args.no_ppo:
         pu = run_ppo_update(args, aht, wl, pop_np, traj, torch, bf16_peak, stream)
         if line is not None:
@@ -564,6 +565,49 @@ def run_lbf12_ppo(aht, W, torch, stream, bf16_peak):
                          "frac": achieved / bf16_peak, "flops_per_launch": flops,
                          "flops_basis": "dense-equivalent MLP FLOPs; the first layer is formed on CUDA "
                                         "cores from the observation's changed features"}}
+
+
+def run_s5(aht, W, torch, stream, bf16_peak, n=16384, K=10):
+    """The recurrent S5 actor-critic step (App. B sizes: model 128, state 128, heads of three
+    1024-unit layers) for n LBF 7x7 observations (196 features, 6 actions): encoder, the
+    diagonal recurrence with 1 % of envs resetting, both heads, masked logits.  ms per step
+    from CUDA events on the policy's stream (L2 scrubbed between steps, outside the events);
+    the roofline counts the model's FLOPs once (the GPU runs the split-activation layers
+    twice: hi and lo bf16 halves)."""
+    obs_dim, A, H, P, F = 196, 6, 128, 128, 1024
+    pol = aht.aht_s5_create(W.s5_params(0, obs_dim, A), n, stream=stream)
+    g = torch.Generator(device="cuda").manual_seed(3)
+    obs = torch.randint(0, 3, (n, obs_dim), dtype=torch.uint8, device="cuda", generator=g)
+    reset = (torch.rand(n, device="cuda", generator=g) < 0.01).to(torch.uint8)
+    legal = torch.ones(n, A, dtype=torch.uint8, device="cuda")
+    state = torch.zeros(n, 2 * P, device="cuda")
+    logits = torch.empty(n, A, device="cuda")
+    values = torch.empty(n, device="cuda")
+    scrub = torch.empty(256 * 2 ** 20, dtype=torch.uint8, device="cuda")
+    torch.cuda.synchronize()
+    for _ in range(3):
+        aht.aht_s5_step(pol, obs, reset, state, logits, values, legal)
+    aht.aht_s5_sync(pol)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    with torch.cuda.stream(stream):
+        for k in range(K):
+            scrub.fill_(k & 0xFF)
+            ev[k][0].record(stream)
+            aht.aht_s5_step(pol, obs, reset, state, logits, values, legal)
+            ev[k][1].record(stream)
+    torch.cuda.synchronize()
+    pol.close()
+    ms = sum(a.elapsed_time(b) for a, b in ev) / K
+    dense = mlp_flops([obs_dim, H, H]) + mlp_flops([H, F, F, F, A]) + mlp_flops([H, F, F, F, 1])
+    ssm = 2 * (2 * P * H) + 8 * P + 2 * (H * 2 * P)
+    flops = n * (dense + ssm)
+    achieved = flops / (ms * 1e-3) / 1e12
+    return {"workload": f"s5_actor_critic_lbf7x7_{n}", "ms_per_step": ms,
+            "env_steps_per_s": n / (ms * 1e-3), "bf16_gemm_launches": 5, "fp32_gemm_launches": 2, "own_kernel_launches": 8,
+            "roofline": {"bound": "tensor", "achieved": achieved, "peak": bf16_peak, "unit": "TFLOP/s",
+                         "frac": achieved / bf16_peak, "flops_per_step": flops,
+                         "flops_basis": "model FLOPs of the encoder, SSM and heads, counted once; "
+                                        "the split layers execute twice as many"}}
 
 
 PPO_FLOPS_PER_SAMPLE = 204032   # forward 84,736 + backward 119,296 (dW1, dW2, dh1, dW3, dh2)

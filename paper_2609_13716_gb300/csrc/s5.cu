@@ -26,17 +26,21 @@ struct aht_s5 {
   cublasHandle_t blas = nullptr;
   int K = 0, A = 0, H = 0, P = 0, F = 0;
   int64_t max_n = 0;
-  // bf16 weights [out][in]; heads stacked: layer 0 [2F][H] (actor rows, then critic),
-  // layers 1-2 [2][F][F], layer 3 actor [A][F] and critic [1][F]
-  __nv_bfloat16 *We1 = nullptr, *We2 = nullptr, *Wh0 = nullptr, *Wh1 = nullptr, *Wh2 = nullptr,
-                *Wa3 = nullptr, *Wc3 = nullptr;
+  // bf16 weights [out][in]. A layer fed with split activations holds each weight row twice,
+  // [W | W] (in = 2I), so that one product over [hi | lo] sums both halves. Heads: layer 0
+  // [2F][2H] (actor rows, then critic), layers 1-2 [2][F][2F]; the encoder's layer 1 [H][K]
+  // sees exact bf16 observations. The output layers, W3 [A + 1][F] (actor rows, then the
+  // critic's), hold the bf16-rounded weights as fp32 for the CUDA-core output kernel.
+  __nv_bfloat16 *We1 = nullptr, *We2 = nullptr, *Wh0 = nullptr, *Wh1 = nullptr, *Wh2 = nullptr;
+  float* W3 = nullptr;
   float *be1 = nullptr, *be2 = nullptr, *bh0 = nullptr, *bh1 = nullptr, *bh2 = nullptr,
         *ba3 = nullptr, *bc3 = nullptr;
   // SSM: lbar [2][P] (re, im), Bbar [2P][H] (re rows, then im rows), Cc [H][2P] (C_re | -C_im), D [H]
   float *lbar = nullptr, *Bbar = nullptr, *Cc = nullptr, *Dv = nullptr;
   // scratch
-  __nv_bfloat16 *x16 = nullptr, *hi = nullptr, *lo = nullptr;  // [n][K], [n][2F] each
-  float *acc = nullptr, *u = nullptr, *bu = nullptr, *xs = nullptr, *y = nullptr;
+  // x16 [n][K]; act: split activations, each row [group][hi | lo][I] (heads: 2 groups of F)
+  __nv_bfloat16 *x16 = nullptr, *act = nullptr;
+  float *acc = nullptr, *u = nullptr, *bu = nullptr, *y = nullptr;
   void* workspace = nullptr;
   std::vector<void*> owned;
 };
@@ -60,78 +64,196 @@ __global__ void u8_to_bf16(const uint8_t* __restrict__ in, __nv_bfloat16* __rest
   if (i < n) out[i] = __float2bfloat16_rn((float)in[i]);
 }
 
-// out = act(acc + b) as fp32 (optional) and as hi + lo bf16, rows of `cols` (ld = cols)
-__global__ void bias_act_split(const float* __restrict__ acc, const float* __restrict__ b, int cols,
-                               int64_t total, bool relu, float* __restrict__ out32,
-                               __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __restrict__ lo) {
-  const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (i >= total) return;
-  float v = acc[i] + b[i % cols];
-  if (relu) v = fmaxf(v, 0.0f);
-  if (out32) out32[i] = v;
-  const __nv_bfloat16 h = __float2bfloat16_rn(v);
-  hi[i] = h;
-  lo[i] = __float2bfloat16_rn(v - __bfloat162float(h));
+// Row-wise kernels run on 2-D blocks and grids: x covers a row's columns (four per thread;
+// the widths are multiples of 16), y strides over rows, so that column arithmetic stays
+// 32-bit.
+constexpr int kRowsPerThread = 4;  // rows a thread of bias_act_split loads before it stores
+
+__device__ __forceinline__ int64_t row0() { return (int64_t)blockIdx.y * blockDim.y + threadIdx.y; }
+__device__ __forceinline__ int64_t row_step() { return (int64_t)gridDim.y * blockDim.y; }
+
+__device__ __forceinline__ uint2 pack_bf16x4(float a, float b, float c, float d) {
+  __nv_bfloat162 lo = __floats2bfloat162_rn(a, b), hi = __floats2bfloat162_rn(c, d);
+  return make_uint2(*reinterpret_cast<uint32_t*>(&lo), *reinterpret_cast<uint32_t*>(&hi));
 }
 
-// x = lbar x (x = 0 first where reset) + Bbar u; state [n][2P], bu [n][2P], xs = state out
+// writes v (four columns) as hi at d and lo = bf16(v - hi) at d + I
+__device__ __forceinline__ void store_split4(__nv_bfloat16* d, int I, float4 v) {
+  const uint2 h = pack_bf16x4(v.x, v.y, v.z, v.w);
+  const __nv_bfloat162 h01 = *reinterpret_cast<const __nv_bfloat162*>(&h.x);
+  const __nv_bfloat162 h23 = *reinterpret_cast<const __nv_bfloat162*>(&h.y);
+  const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+  *reinterpret_cast<uint2*>(d) = h;
+  *reinterpret_cast<uint2*>(d + I) = pack_bf16x4(v.x - f01.x, v.y - f01.y, v.z - f23.x, v.w - f23.y);
+}
+
+// v = act(acc + b), acc rows of g groups of I columns (ld g I, I % 4 == 0): v as fp32
+// (optional) and as a bf16 pair hi + lo (optional) at split[row][group][0 | 1][col] (ld 2 g I)
+__global__ void bias_act_split(const float* __restrict__ acc, const float* __restrict__ b, int I, int g,
+                               int64_t n, bool relu, float* __restrict__ out32,
+                               __nv_bfloat16* __restrict__ split) {
+  const int c = 4 * (blockIdx.x * blockDim.x + threadIdx.x);
+  const int row_w = g * I;
+  if (c >= row_w) return;
+  const int gg = c / I, f = c - gg * I;
+  const float4 bb = *reinterpret_cast<const float4*>(b + c);
+  const int64_t step = row_step();
+  for (int64_t r0 = row0(); r0 < n; r0 += kRowsPerThread * step) {
+    float4 v[kRowsPerThread];
+#pragma unroll
+    for (int k = 0; k < kRowsPerThread; ++k)  // all loads first: several rows in flight
+      if (r0 + k * step < n) v[k] = __ldcs(reinterpret_cast<const float4*>(acc + (r0 + k * step) * row_w + c));
+#pragma unroll
+    for (int k = 0; k < kRowsPerThread; ++k) {
+      const int64_t r = r0 + k * step;
+      if (r >= n) break;
+      float4 x = v[k];
+      x.x += bb.x; x.y += bb.y; x.z += bb.z; x.w += bb.w;
+      if (relu) {
+        x.x = fmaxf(x.x, 0.0f); x.y = fmaxf(x.y, 0.0f); x.z = fmaxf(x.z, 0.0f); x.w = fmaxf(x.w, 0.0f);
+      }
+      if (out32) *reinterpret_cast<float4*>(out32 + r * row_w + c) = x;
+      if (split) store_split4(split + r * 2 * row_w + (int64_t)gg * 2 * I + f, I, x);
+    }
+  }
+}
+
+// x = lbar x (x = 0 first where reset) + Bbar u, in place; state [n][2P] (re, im), bu [n][2P]
 __global__ void ssm_recur(const float* __restrict__ lbar, const float* __restrict__ bu,
                           const uint8_t* __restrict__ reset, float* __restrict__ state, int P,
                           int64_t n) {
-  const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (i >= n * P) return;
-  const int64_t e = i / P;
-  const int p = (int)(i - e * P);
-  float* s = state + e * 2 * P;
-  const float xr = reset[e] ? 0.0f : s[p], xi = reset[e] ? 0.0f : s[P + p];
-  const float lr = lbar[p], li = lbar[P + p];
-  const float* b = bu + e * 2 * P;
-  s[p] = fmaf(lr, xr, fmaf(-li, xi, b[p]));
-  s[P + p] = fmaf(lr, xi, fmaf(li, xr, b[P + p]));
-}
-
-// v = u + gelu(y + D u) -> hi + lo bf16
-__global__ void residual_gelu(const float* __restrict__ y, const float* __restrict__ u,
-                              const float* __restrict__ D, int H, int64_t total,
-                              __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __restrict__ lo) {
-  const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (i >= total) return;
-  const float uu = u[i];
-  const float yy = fmaf(D[i % H], uu, y[i]);
-  const float v = uu + yy * 0.5f * erfcf(-yy * 0.70710678118654752f);
-  const __nv_bfloat16 h = __float2bfloat16_rn(v);
-  hi[i] = h;
-  lo[i] = __float2bfloat16_rn(v - __bfloat162float(h));
-}
-
-// logits = acc_a + ba (-inf where illegal), value = acc_c + bc
-__global__ void s5_outputs(const float* __restrict__ acc_a, const float* __restrict__ acc_c,
-                           const float* __restrict__ ba, const float* __restrict__ bc,
-                           const uint8_t* __restrict__ legal, int A, int64_t n,
-                           float* __restrict__ logits, float* __restrict__ values) {
-  const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (i < n * A) {
-    const int a = (int)(i % A);
-    const float z = acc_a[i] + ba[a];
-    logits[i] = (legal && !legal[i]) ? -INFINITY : z;
+  const int p = 4 * (blockIdx.x * blockDim.x + threadIdx.x);
+  if (p >= P) return;
+  const float4 lr = *reinterpret_cast<const float4*>(lbar + p);
+  const float4 li = *reinterpret_cast<const float4*>(lbar + P + p);
+  for (int64_t e = row0(); e < n; e += row_step()) {
+    float* s = state + e * 2 * P;
+    const float* bp = bu + e * 2 * P;
+    float4 xr = *reinterpret_cast<const float4*>(s + p), xi = *reinterpret_cast<const float4*>(s + P + p);
+    if (reset[e]) xr = xi = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    const float4 br = *reinterpret_cast<const float4*>(bp + p), bi = *reinterpret_cast<const float4*>(bp + P + p);
+    float4 orr, oi;
+    orr.x = fmaf(lr.x, xr.x, fmaf(-li.x, xi.x, br.x)); oi.x = fmaf(lr.x, xi.x, fmaf(li.x, xr.x, bi.x));
+    orr.y = fmaf(lr.y, xr.y, fmaf(-li.y, xi.y, br.y)); oi.y = fmaf(lr.y, xi.y, fmaf(li.y, xr.y, bi.y));
+    orr.z = fmaf(lr.z, xr.z, fmaf(-li.z, xi.z, br.z)); oi.z = fmaf(lr.z, xi.z, fmaf(li.z, xr.z, bi.z));
+    orr.w = fmaf(lr.w, xr.w, fmaf(-li.w, xi.w, br.w)); oi.w = fmaf(lr.w, xi.w, fmaf(li.w, xr.w, bi.w));
+    *reinterpret_cast<float4*>(s + p) = orr;
+    *reinterpret_cast<float4*>(s + P + p) = oi;
   }
-  if (i < n) values[i] = acc_c[i] + bc[0];
+}
+
+__device__ __forceinline__ float gelu_exact(float y) { return y * 0.5f * erfcf(-y * 0.70710678118654752f); }
+
+// v = u + gelu(y + D u) -> split[row][0 | 1][H] (hi, lo bf16)
+__global__ void residual_gelu(const float* __restrict__ y, const float* __restrict__ u,
+                              const float* __restrict__ D, int H, int64_t n,
+                              __nv_bfloat16* __restrict__ split) {
+  const int c = 4 * (blockIdx.x * blockDim.x + threadIdx.x);
+  if (c >= H) return;
+  const float4 dd = *reinterpret_cast<const float4*>(D + c);
+  for (int64_t r = row0(); r < n; r += row_step()) {
+    const float4 uu = *reinterpret_cast<const float4*>(u + r * H + c);
+    const float4 yy = *reinterpret_cast<const float4*>(y + r * H + c);
+    float4 v;
+    v.x = uu.x + gelu_exact(fmaf(dd.x, uu.x, yy.x));
+    v.y = uu.y + gelu_exact(fmaf(dd.y, uu.y, yy.y));
+    v.z = uu.z + gelu_exact(fmaf(dd.z, uu.z, yy.z));
+    v.w = uu.w + gelu_exact(fmaf(dd.w, uu.w, yy.w));
+    store_split4(split + r * 2 * H + c, H, v);
+  }
+}
+
+__device__ __forceinline__ float warp_sum(float x) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  return x;
+}
+
+// The heads' last hidden layer and both output layers, one warp per env: h = relu(acc + b)
+// in fp32 (acc [n][2F]: actor columns, then critic), logits[a] = Wa3[a] . h_actor + ba3[a]
+// (-inf where illegal), value = Wc3 . h_critic + bc3. W3 [A + 1][F] fp32 (actor rows, then
+// the critic's); AM >= A is the register width of the logit sums.
+template <int AM>
+__global__ void heads_out(const float* __restrict__ acc, const float* __restrict__ b,
+                          const float* __restrict__ W3, const float* __restrict__ ba3,
+                          const float* __restrict__ bc3, const uint8_t* __restrict__ legal, int A, int F,
+                          int64_t n, float* __restrict__ logits, float* __restrict__ values) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+  const int quads = F / 4;
+  for (int64_t e = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); e < n; e += warps) {
+    const float* row = acc + e * 2 * F;
+    float pa[AM], pv = 0.0f;
+#pragma unroll
+    for (int a = 0; a < AM; ++a) pa[a] = 0.0f;
+#pragma unroll 2
+    for (int q = lane; q < quads; q += 32) {
+      const float4 x = __ldcs(reinterpret_cast<const float4*>(row) + q);
+      const float4 bb = reinterpret_cast<const float4*>(b)[q];
+      const float4 h = make_float4(fmaxf(x.x + bb.x, 0.0f), fmaxf(x.y + bb.y, 0.0f), fmaxf(x.z + bb.z, 0.0f),
+                                   fmaxf(x.w + bb.w, 0.0f));
+#pragma unroll
+      for (int a = 0; a < AM; ++a)
+        if (a < A) {
+          const float4 w = __ldg(reinterpret_cast<const float4*>(W3 + (size_t)a * F) + q);
+          pa[a] = fmaf(h.x, w.x, fmaf(h.y, w.y, fmaf(h.z, w.z, fmaf(h.w, w.w, pa[a]))));
+        }
+      const float4 xc = __ldcs(reinterpret_cast<const float4*>(row + F) + q);
+      const float4 bc = reinterpret_cast<const float4*>(b + F)[q];
+      const float4 w = __ldg(reinterpret_cast<const float4*>(W3 + (size_t)A * F) + q);
+      pv = fmaf(fmaxf(xc.x + bc.x, 0.0f), w.x, pv);
+      pv = fmaf(fmaxf(xc.y + bc.y, 0.0f), w.y, pv);
+      pv = fmaf(fmaxf(xc.z + bc.z, 0.0f), w.z, pv);
+      pv = fmaf(fmaxf(xc.w + bc.w, 0.0f), w.w, pv);
+    }
+#pragma unroll
+    for (int a = 0; a < AM; ++a)
+      if (a < A) {
+        const float z = warp_sum(pa[a]) + ba3[a];
+        if (lane == a) logits[e * A + a] = (legal && !legal[e * A + a]) ? -INFINITY : z;
+      }
+    pv = warp_sum(pv);
+    if (lane == 0) values[e] = pv + bc3[0];
+  }
+}
+
+// launch shape of a row-wise kernel: 256 threads, x over a row's `quads` four-column groups
+// (rounded up to a warp), y over rows; at most 65535 row blocks (the kernels stride)
+struct RowsLaunch {
+  dim3 grid, block;
+};
+RowsLaunch rows_launch(int quads, int64_t n, int rows_per_thread) {
+  const int bx = std::min(256, (quads + 31) / 32 * 32), by = 256 / bx;
+  const int64_t per_block = (int64_t)by * rows_per_thread;
+  return {dim3((unsigned)((quads + bx - 1) / bx), (unsigned)std::min<int64_t>((n + per_block - 1) / per_block, 65535)),
+          dim3((unsigned)bx, (unsigned)by)};
+}
+template <typename... KArgs, typename... Args>
+void launch_rows(void (*kernel)(KArgs...), int quads, int64_t n, cudaStream_t st, Args... args) {
+  const RowsLaunch L = rows_launch(quads, n, (void*)kernel == (void*)bias_act_split ? kRowsPerThread : 1);
+  kernel<<<L.grid, L.block, 0, st>>>(args...);
 }
 
 int blocks_for(int64_t total) { return (int)((total + 255) / 256); }
 
-// C[n][O] (+)= X[n][I] W^T for row-major X (ld ldx), W [O][I] (ld I), C (ld ldc)
+// C[n][O] = X[n][I] W^T for row-major X (ld ldx), W [O][I] (ld I), C (ld ldc); `batch`
+// products at once, the b-th at W + b sW, X + b sX, C + b sC
 cublasStatus_t gemm_bf16(cublasHandle_t h, int64_t n, int O, int I, const __nv_bfloat16* W,
-                         const __nv_bfloat16* X, int ldx, float* Cm, int ldc, float beta) {
-  const float one = 1.0f;
-  return cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, O, (int)n, I, &one, W, CUDA_R_16BF, I, X, CUDA_R_16BF,
-                      ldx, &beta, Cm, CUDA_R_32F, ldc, CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
+                         const __nv_bfloat16* X, int ldx, float* Cm, int ldc, int batch = 1,
+                         int64_t sW = 0, int64_t sX = 0, int64_t sC = 0) {
+  const float one = 1.0f, zero = 0.0f;
+  if (batch == 1)
+    return cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, O, (int)n, I, &one, W, CUDA_R_16BF, I, X, CUDA_R_16BF,
+                        ldx, &zero, Cm, CUDA_R_32F, ldc, CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
+  return cublasGemmStridedBatchedEx(h, CUBLAS_OP_T, CUBLAS_OP_N, O, (int)n, I, &one, W, CUDA_R_16BF, I, sW,
+                                    X, CUDA_R_16BF, ldx, sX, &zero, Cm, CUDA_R_32F, ldc, sC, batch,
+                                    CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
 }
 cublasStatus_t gemm_f32(cublasHandle_t h, int64_t n, int O, int I, const float* W, const float* X,
                         float* Cm) {
   const float one = 1.0f, zero = 0.0f;
   return cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, O, (int)n, I, &one, W, CUDA_R_32F, I, X, CUDA_R_32F, I,
-                      &zero, Cm, CUDA_R_32F, O, CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
+                      &zero, Cm, CUDA_R_32F, O, CUBLAS_COMPUTE_32F_PEDANTIC, CUBLAS_GEMM_DEFAULT);
 }
 
 }  // namespace
@@ -186,15 +308,29 @@ aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_st
     return alloc((void**)dst, h.size() * 4) && cudaMemcpy(*dst, h.data(), h.size() * 4, cudaMemcpyHostToDevice) == cudaSuccess;
   };
   auto vec = [](const float* a, size_t n) { return std::vector<float>(a, a + n); };
+  auto bf16_rounded = [](const float* a, size_t n) {
+    std::vector<float> v(n);
+    for (size_t i = 0; i < n; ++i) v[i] = __bfloat162float(__float2bfloat16_rn(a[i]));
+    return v;
+  };
   auto cat = [](std::vector<float> a, const std::vector<float>& b) {
     a.insert(a.end(), b.begin(), b.end());
     return a;
   };
-  bool ok = up16(&s->We1, {p->We1}, {(size_t)H * K}) && up16(&s->We2, {p->We2}, {(size_t)H * H}) &&
-            up16(&s->Wh0, {p->Wa[0], p->Wc[0]}, {(size_t)F * H, (size_t)F * H}) &&
-            up16(&s->Wh1, {p->Wa[1], p->Wc[1]}, {(size_t)F * F, (size_t)F * F}) &&
-            up16(&s->Wh2, {p->Wa[2], p->Wc[2]}, {(size_t)F * F, (size_t)F * F}) &&
-            up16(&s->Wa3, {p->Wa[3]}, {(size_t)A * F}) && up16(&s->Wc3, {p->Wc[3]}, {(size_t)F}) &&
+  // [W | W] rows: each of `rows` rows of every part written twice
+  auto up16x2 = [&](__nv_bfloat16** dst, const std::vector<const float*>& parts, size_t rows, size_t cols) {
+    std::vector<__nv_bfloat16> h(parts.size() * rows * 2 * cols);
+    size_t o = 0;
+    for (const float* w : parts)
+      for (size_t r = 0; r < rows; ++r)
+        for (int rep = 0; rep < 2; ++rep)
+          for (size_t c = 0; c < cols; ++c) h[o++] = __float2bfloat16_rn(w[r * cols + c]);
+    return alloc((void**)dst, h.size() * 2) && cudaMemcpy(*dst, h.data(), h.size() * 2, cudaMemcpyHostToDevice) == cudaSuccess;
+  };
+  bool ok = up16(&s->We1, {p->We1}, {(size_t)H * K}) && up16x2(&s->We2, {p->We2}, H, H) &&
+            up16x2(&s->Wh0, {p->Wa[0], p->Wc[0]}, F, H) && up16x2(&s->Wh1, {p->Wa[1], p->Wc[1]}, F, F) &&
+            up16x2(&s->Wh2, {p->Wa[2], p->Wc[2]}, F, F) &&
+            up32(&s->W3, cat(bf16_rounded(p->Wa[3], (size_t)A * F), bf16_rounded(p->Wc[3], F))) &&
             up32(&s->be1, vec(p->be1, H)) && up32(&s->be2, vec(p->be2, H)) &&
             up32(&s->bh0, cat(vec(p->ba[0], F), vec(p->bc[0], F))) &&
             up32(&s->bh1, cat(vec(p->ba[1], F), vec(p->bc[1], F))) &&
@@ -222,15 +358,14 @@ aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_st
     }
   if (!up32(&s->lbar, lbar) || !up32(&s->Bbar, Bbar) || !up32(&s->Cc, Cc)) return bail(AHT_ENOMEM, "S5 upload failed");
   const int64_t n = max_envs;
-  const int widest = std::max(2 * F, std::max(2 * P, H));
-  ok = alloc((void**)&s->x16, (size_t)n * K * 2) && alloc((void**)&s->hi, (size_t)n * widest * 2) &&
-       alloc((void**)&s->lo, (size_t)n * widest * 2) && alloc((void**)&s->acc, (size_t)n * widest * 4) &&
-       alloc((void**)&s->u, (size_t)n * H * 4) && alloc((void**)&s->bu, (size_t)n * 2 * P * 4) &&
-       alloc((void**)&s->y, (size_t)n * (2 * F > H ? 2 * F : H) * 4) && alloc(&s->workspace, kWorkspace);
+  ok = alloc((void**)&s->x16, (size_t)n * K * 2) && alloc((void**)&s->act, (size_t)n * std::max(4 * F, 2 * H) * 2) &&
+       alloc((void**)&s->acc, (size_t)n * std::max(2 * F, H) * 4) && alloc((void**)&s->u, (size_t)n * H * 4) &&
+       alloc((void**)&s->bu, (size_t)n * 2 * P * 4) && alloc((void**)&s->y, (size_t)n * H * 4) &&
+       alloc(&s->workspace, kWorkspace);
   if (!ok) return bail(AHT_ENOMEM, "S5 scratch allocation failed");
   if (cublasCreate(&s->blas) != CUBLAS_STATUS_SUCCESS || cublasSetStream(s->blas, s->stream) != CUBLAS_STATUS_SUCCESS ||
       cublasSetWorkspace(s->blas, s->workspace, kWorkspace) != CUBLAS_STATUS_SUCCESS ||
-      cublasSetMathMode(s->blas, CUBLAS_PEDANTIC_MATH) != CUBLAS_STATUS_SUCCESS)
+      cublasSetMathMode(s->blas, CUBLAS_DEFAULT_MATH) != CUBLAS_STATUS_SUCCESS)
     return bail(AHT_ECUDA, "cuBLAS set-up failed");
   *out = s;
   return AHT_OK;
@@ -250,38 +385,36 @@ aht_status aht_s5_step(aht_s5* s, const uint8_t* obs, const uint8_t* reset, cons
   const int K = s->K, A = s->A, H = s->H, P = s->P, F = s->F;
   cudaStream_t st = s->stream;
   cublasHandle_t b = s->blas;
-  // encoder: the observation is exact in bf16, so layer 1 is one product
+  // encoder: the observation is exact in bf16, so layer 1 is one plain product; later
+  // layers take [hi | lo] against [W | W], one product with fp32 accumulation
   u8_to_bf16<<<blocks_for(n * K), 256, 0, st>>>(obs, s->x16, n * K);
-  S5_BLAS(gemm_bf16(b, n, H, K, s->We1, s->x16, K, s->acc, H, 0.0f));
-  bias_act_split<<<blocks_for(n * H), 256, 0, st>>>(s->acc, s->be1, H, n * H, true, nullptr, s->hi, s->lo);
-  S5_BLAS(gemm_bf16(b, n, H, H, s->We2, s->hi, H, s->acc, H, 0.0f));
-  S5_BLAS(gemm_bf16(b, n, H, H, s->We2, s->lo, H, s->acc, H, 1.0f));
-  bias_act_split<<<blocks_for(n * H), 256, 0, st>>>(s->acc, s->be2, H, n * H, true, s->u, s->hi, s->lo);
+  S5_BLAS(gemm_bf16(b, n, H, K, s->We1, s->x16, K, s->acc, H));
+  launch_rows(bias_act_split, H / 4, n, st, s->acc, s->be1, H, 1, n, true, (float*)nullptr, s->act);
+  S5_BLAS(gemm_bf16(b, n, H, 2 * H, s->We2, s->act, 2 * H, s->acc, H));
+  launch_rows(bias_act_split, H / 4, n, st, s->acc, s->be2, H, 1, n, true, s->u, (__nv_bfloat16*)nullptr);
   // SSM (fp32): Bbar u, the recurrence, Re(C x)
   S5_BLAS(gemm_f32(b, n, 2 * P, H, s->Bbar, s->u, s->bu));
-  ssm_recur<<<blocks_for(n * P), 256, 0, st>>>(s->lbar, s->bu, reset, state, P, n);
+  launch_rows(ssm_recur, P / 4, n, st, s->lbar, s->bu, reset, state, P, n);
   S5_BLAS(gemm_f32(b, n, H, 2 * P, s->Cc, state, s->y));
-  residual_gelu<<<blocks_for(n * H), 256, 0, st>>>(s->y, s->u, s->Dv, H, n * H, s->hi, s->lo);
-  // heads: layer 0 for both heads at once ([2F] outputs), layers 1-2 per head
-  S5_BLAS(gemm_bf16(b, n, 2 * F, H, s->Wh0, s->hi, H, s->acc, 2 * F, 0.0f));
-  S5_BLAS(gemm_bf16(b, n, 2 * F, H, s->Wh0, s->lo, H, s->acc, 2 * F, 1.0f));
-  bias_act_split<<<blocks_for(n * 2 * F), 256, 0, st>>>(s->acc, s->bh0, 2 * F, n * 2 * F, true, nullptr, s->hi, s->lo);
+  launch_rows(residual_gelu, H / 4, n, st, s->y, s->u, s->Dv, H, n, s->act);
+  // heads: layer 0 for both heads at once ([2F] outputs, split as 2 groups of F), layers
+  // 1-2 as one two-member batch (head h reads group h, writes columns h F of acc)
+  S5_BLAS(gemm_bf16(b, n, 2 * F, 2 * H, s->Wh0, s->act, 2 * H, s->acc, 2 * F));
+  launch_rows(bias_act_split, 2 * F / 4, n, st, s->acc, s->bh0, F, 2, n, true, (float*)nullptr, s->act);
   const __nv_bfloat16* Wl[2] = {s->Wh1, s->Wh2};
   const float* bl[2] = {s->bh1, s->bh2};
   for (int l = 0; l < 2; ++l) {
-    for (int head = 0; head < 2; ++head) {
-      const __nv_bfloat16* Wh = Wl[l] + (size_t)head * F * F;
-      S5_BLAS(gemm_bf16(b, n, F, F, Wh, s->hi + head * F, 2 * F, s->acc + head * F, 2 * F, 0.0f));
-      S5_BLAS(gemm_bf16(b, n, F, F, Wh, s->lo + head * F, 2 * F, s->acc + head * F, 2 * F, 1.0f));
-    }
-    bias_act_split<<<blocks_for(n * 2 * F), 256, 0, st>>>(s->acc, bl[l], 2 * F, n * 2 * F, true, nullptr, s->hi, s->lo);
+    S5_BLAS(gemm_bf16(b, n, F, 2 * F, Wl[l], s->act, 4 * F, s->acc, 2 * F, 2, (int64_t)F * 2 * F, 2 * F, F));
+    if (l == 0) launch_rows(bias_act_split, 2 * F / 4, n, st, s->acc, bl[l], F, 2, n, true, (float*)nullptr, s->act);
   }
-  // output layers: actor logits [n][A] into acc, critic value [n] into y
-  S5_BLAS(gemm_bf16(b, n, A, F, s->Wa3, s->hi, 2 * F, s->acc, A, 0.0f));
-  S5_BLAS(gemm_bf16(b, n, A, F, s->Wa3, s->lo, 2 * F, s->acc, A, 1.0f));
-  S5_BLAS(gemm_bf16(b, n, 1, F, s->Wc3, s->hi + F, 2 * F, s->y, 1, 0.0f));
-  S5_BLAS(gemm_bf16(b, n, 1, F, s->Wc3, s->lo + F, 2 * F, s->y, 1, 1.0f));
-  s5_outputs<<<blocks_for(n * A), 256, 0, st>>>(s->acc, s->y, s->ba3, s->bc3, legal, A, n, logits, values);
+  // layer 2's bias and relu, and both output layers, in fp32 (one warp per env)
+  const int out_blocks = (int)std::min<int64_t>((n + 7) / 8, 65535);
+  if (A <= 8)
+    heads_out<8><<<out_blocks, 256, 0, st>>>(s->acc, s->bh2, s->W3, s->ba3, s->bc3, legal, A, F, n, logits, values);
+  else if (A <= 16)
+    heads_out<16><<<out_blocks, 256, 0, st>>>(s->acc, s->bh2, s->W3, s->ba3, s->bc3, legal, A, F, n, logits, values);
+  else
+    heads_out<32><<<out_blocks, 256, 0, st>>>(s->acc, s->bh2, s->W3, s->ba3, s->bc3, legal, A, F, n, logits, values);
   S5_CUDA(cudaGetLastError());
   return AHT_OK;
 }
