@@ -63,6 +63,46 @@ def test_s5_steps_match_the_oracle(N, T):
     pol.close()
 
 
+@pytest.mark.parametrize("K,A,H,P,F,N,max_envs,masked", [
+    (100, 20, 32, 16, 64, 77, 128, True),     # 9-16 actions; fewer envs than max_envs
+    (37, 32, 16, 32, 48, 5, 5, False),        # 32 actions, no mask; F / 4 < 32 lanes
+    (10, 1, 16, 16, 16, 33, 40, True),        # one action
+])
+def test_s5_other_shapes(K, A, H, P, F, N, max_envs, masked):
+    """Action counts on each register width of the output kernel, the unmasked path,
+    narrow heads and ragged env counts, over four steps with resets."""
+    require_gpu()
+    params = W.s5_params(3, K, A, H=H, P=P, F=F)
+    pol = aht.aht_s5_create(params, max_envs)
+    net = O.S5(params)
+    rng = np.random.default_rng(K)
+    state = torch.zeros(N, 2 * P, device="cuda")
+    state_ref = np.zeros((N, 2 * P))
+    logits = torch.empty(N, A, device="cuda")
+    values = torch.empty(N, device="cuda")
+    for t in range(4):
+        obs = rng.integers(0, 4, (N, K)).astype(np.uint8)
+        reset = (rng.random(N) < 0.3).astype(np.uint8) if t else np.ones(N, np.uint8)
+        legal = None
+        if masked:
+            legal = (rng.random((N, A)) < 0.7).astype(np.uint8)
+            legal[:, 0] = 1
+        aht.aht_s5_step(pol, torch.from_numpy(obs).cuda(), torch.from_numpy(reset).cuda(), state, logits,
+                        values, None if legal is None else torch.from_numpy(legal).cuda())
+        aht.aht_s5_sync(pol)
+        lg_ref, v_ref = net.step(obs, reset, state_ref, legal)
+        lg = np_(logits)
+        fin = np.isfinite(lg_ref)
+        assert np.array_equal(np.isfinite(lg), fin), "masked actions"
+        ok, worst = close(lg[fin], lg_ref[fin])
+        assert ok, f"logits at step {t}: {worst:.3g}"
+        ok, worst = close(np_(values), v_ref)
+        assert ok, f"values at step {t}: {worst:.3g}"
+        ok, worst = close(np_(state), state_ref)
+        assert ok, f"state at step {t}: {worst:.3g}"
+    pol.close()
+
+
 def test_s5_rejects_bad_sizes():
     require_gpu()
     params = W.s5_params(1, 196, 6, H=16, P=16, F=32)
