@@ -369,9 +369,10 @@ aht_status aht_learner_sync(aht_learner* L);
  *   v = u + gelu(y) (gelu(a) = a Phi(a)),  logits / value = heads(v).
  * The paper gives H = P = 128 and F = 1024; the rest is this library's reading.  Weights
  * are rounded to bf16 at create.  Hidden layers run as bf16 GEMMs (activations carried
- * as two bf16, hi + lo, ~2^-17 relative, fp32 accumulate); the SSM runs in fp32 (lbar and
- * Bbar computed in fp64 at create); the output layers run in fp32 from the fp32 last
- * hidden layer.  Parameters are host fp32 arrays, row-major [out][in]. */
+ * as two bf16, hi + lo, ~2^-17 relative, fp32 accumulate); the SSM's products run as
+ * three bf16 terms (hi hi + hi lo + lo hi, ~2^-16 relative, fp32 accumulate) and its
+ * recurrence in fp32 (lbar and Bbar computed in fp64 at create); the output layers run
+ * in fp32 from the fp32 last hidden layer.  Parameters are host fp32 arrays, row-major [out][in]. */
 typedef struct aht_s5_params {
   int32_t obs_dim, n_actions, H, P, F;  /* H, P multiples of 16, F of 16; n_actions <= 32 */
   const float *We1, *be1, *We2, *be2;   /* [H][obs_dim] [H] [H][H] [H] */

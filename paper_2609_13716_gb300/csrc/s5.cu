@@ -35,8 +35,12 @@ struct aht_s5 {
   float* W3 = nullptr;
   float *be1 = nullptr, *be2 = nullptr, *bh0 = nullptr, *bh1 = nullptr, *bh2 = nullptr,
         *ba3 = nullptr, *bc3 = nullptr;
-  // SSM: lbar [2][P] (re, im), Bbar [2P][H] (re rows, then im rows), Cc [H][2P] (C_re | -C_im), D [H]
-  float *lbar = nullptr, *Bbar = nullptr, *Cc = nullptr, *Dv = nullptr;
+  // SSM: lbar [2][P] (re, im) and D [H] fp32.  Its products run as three bf16 terms: an
+  // fp32 operand a = ah + al (two bf16), activations stored [hi | lo | hi] and weights
+  // [Wh | Wh | Wl], one GEMM sums Wh hi + Wh lo + Wl hi (~2^-16 relative).  Bbar3 [2P][3H]
+  // (re rows, then im rows), Cc3 [H][3 x 2P] from Cc = (C_re | -C_im).
+  float *lbar = nullptr, *Dv = nullptr;
+  __nv_bfloat16 *Bbar3 = nullptr, *Cc3 = nullptr;
   // scratch
   // x16 [n][K]; act: split activations, each row [group][hi | lo][I] (heads: 2 groups of F)
   __nv_bfloat16 *x16 = nullptr, *act = nullptr;
@@ -77,21 +81,24 @@ __device__ __forceinline__ uint2 pack_bf16x4(float a, float b, float c, float d)
   return make_uint2(*reinterpret_cast<uint32_t*>(&lo), *reinterpret_cast<uint32_t*>(&hi));
 }
 
-// writes v (four columns) as hi at d and lo = bf16(v - hi) at d + I
-__device__ __forceinline__ void store_split4(__nv_bfloat16* d, int I, float4 v) {
+// writes v (four columns) as hi at d and lo = bf16(v - hi) at d + I (and hi again at
+// d + 2I for a three-term product)
+__device__ __forceinline__ void store_split4(__nv_bfloat16* d, int I, float4 v, bool hi_again = false) {
   const uint2 h = pack_bf16x4(v.x, v.y, v.z, v.w);
   const __nv_bfloat162 h01 = *reinterpret_cast<const __nv_bfloat162*>(&h.x);
   const __nv_bfloat162 h23 = *reinterpret_cast<const __nv_bfloat162*>(&h.y);
   const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
   *reinterpret_cast<uint2*>(d) = h;
   *reinterpret_cast<uint2*>(d + I) = pack_bf16x4(v.x - f01.x, v.y - f01.y, v.z - f23.x, v.w - f23.y);
+  if (hi_again) *reinterpret_cast<uint2*>(d + 2 * I) = h;
 }
 
 // v = act(acc + b), acc rows of g groups of I columns (ld g I, I % 4 == 0): v as fp32
-// (optional) and as a bf16 pair hi + lo (optional) at split[row][group][0 | 1][col] (ld 2 g I)
+// (optional) and split (optional) at split[row][group][part][col] (ld parts g I): parts = 2
+// stores hi, lo; parts = 3 stores hi, lo, hi
 __global__ void bias_act_split(const float* __restrict__ acc, const float* __restrict__ b, int I, int g,
                                int64_t n, bool relu, float* __restrict__ out32,
-                               __nv_bfloat16* __restrict__ split) {
+                               __nv_bfloat16* __restrict__ split, int parts) {
   const int c = 4 * (blockIdx.x * blockDim.x + threadIdx.x);
   const int row_w = g * I;
   if (c >= row_w) return;
@@ -113,15 +120,16 @@ __global__ void bias_act_split(const float* __restrict__ acc, const float* __res
         x.x = fmaxf(x.x, 0.0f); x.y = fmaxf(x.y, 0.0f); x.z = fmaxf(x.z, 0.0f); x.w = fmaxf(x.w, 0.0f);
       }
       if (out32) *reinterpret_cast<float4*>(out32 + r * row_w + c) = x;
-      if (split) store_split4(split + r * 2 * row_w + (int64_t)gg * 2 * I + f, I, x);
+      if (split) store_split4(split + r * parts * row_w + (int64_t)gg * parts * I + f, I, x, parts == 3);
     }
   }
 }
 
-// x = lbar x (x = 0 first where reset) + Bbar u, in place; state [n][2P] (re, im), bu [n][2P]
+// x = lbar x (x = 0 first where reset) + Bbar u, in place; state [n][2P] (re, im), bu [n][2P];
+// x also as [hi | lo | hi] bf16 rows of 2P each (ld 6P) for the three-term C product
 __global__ void ssm_recur(const float* __restrict__ lbar, const float* __restrict__ bu,
                           const uint8_t* __restrict__ reset, float* __restrict__ state, int P,
-                          int64_t n) {
+                          int64_t n, __nv_bfloat16* __restrict__ xsplit) {
   const int p = 4 * (blockIdx.x * blockDim.x + threadIdx.x);
   if (p >= P) return;
   const float4 lr = *reinterpret_cast<const float4*>(lbar + p);
@@ -139,6 +147,8 @@ __global__ void ssm_recur(const float* __restrict__ lbar, const float* __restric
     orr.w = fmaf(lr.w, xr.w, fmaf(-li.w, xi.w, br.w)); oi.w = fmaf(lr.w, xi.w, fmaf(li.w, xr.w, bi.w));
     *reinterpret_cast<float4*>(s + p) = orr;
     *reinterpret_cast<float4*>(s + P + p) = oi;
+    store_split4(xsplit + e * 6 * P + p, 2 * P, orr, true);
+    store_split4(xsplit + e * 6 * P + P + p, 2 * P, oi, true);
   }
 }
 
@@ -249,12 +259,6 @@ cublasStatus_t gemm_bf16(cublasHandle_t h, int64_t n, int O, int I, const __nv_b
                                     X, CUDA_R_16BF, ldx, sX, &zero, Cm, CUDA_R_32F, ldc, sC, batch,
                                     CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
 }
-cublasStatus_t gemm_f32(cublasHandle_t h, int64_t n, int O, int I, const float* W, const float* X,
-                        float* Cm) {
-  const float one = 1.0f, zero = 0.0f;
-  return cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, O, (int)n, I, &one, W, CUDA_R_32F, I, X, CUDA_R_32F, I,
-                      &zero, Cm, CUDA_R_32F, O, CUBLAS_COMPUTE_32F_PEDANTIC, CUBLAS_GEMM_DEFAULT);
-}
 
 }  // namespace
 
@@ -356,9 +360,23 @@ aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_st
       Cc[(size_t)h * 2 * P + q] = p->C_re[(size_t)h * P + q];
       Cc[(size_t)h * 2 * P + P + q] = -p->C_im[(size_t)h * P + q];
     }
-  if (!up32(&s->lbar, lbar) || !up32(&s->Bbar, Bbar) || !up32(&s->Cc, Cc)) return bail(AHT_ENOMEM, "S5 upload failed");
+  // three-term bf16 rows [Wh | Wh | Wl] of an fp32 matrix [rows][cols]
+  auto up_three = [&](__nv_bfloat16** dst, const std::vector<float>& w, size_t rows, size_t cols) {
+    std::vector<__nv_bfloat16> h(rows * 3 * cols);
+    for (size_t r = 0; r < rows; ++r)
+      for (size_t c = 0; c < cols; ++c) {
+        const float x = w[r * cols + c];
+        const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+        h[r * 3 * cols + c] = hi;
+        h[r * 3 * cols + cols + c] = hi;
+        h[r * 3 * cols + 2 * cols + c] = __float2bfloat16_rn(x - __bfloat162float(hi));
+      }
+    return alloc((void**)dst, h.size() * 2) && cudaMemcpy(*dst, h.data(), h.size() * 2, cudaMemcpyHostToDevice) == cudaSuccess;
+  };
+  if (!up32(&s->lbar, lbar) || !up_three(&s->Bbar3, Bbar, 2 * P, H) || !up_three(&s->Cc3, Cc, H, 2 * P))
+    return bail(AHT_ENOMEM, "S5 upload failed");
   const int64_t n = max_envs;
-  ok = alloc((void**)&s->x16, (size_t)n * K * 2) && alloc((void**)&s->act, (size_t)n * std::max(4 * F, 2 * H) * 2) &&
+  ok = alloc((void**)&s->x16, (size_t)n * K * 2) && alloc((void**)&s->act, (size_t)n * std::max({4 * F, 3 * H, 6 * P}) * 2) &&
        alloc((void**)&s->acc, (size_t)n * std::max(2 * F, H) * 4) && alloc((void**)&s->u, (size_t)n * H * 4) &&
        alloc((void**)&s->bu, (size_t)n * 2 * P * 4) && alloc((void**)&s->y, (size_t)n * H * 4) &&
        alloc(&s->workspace, kWorkspace);
@@ -389,23 +407,23 @@ aht_status aht_s5_step(aht_s5* s, const uint8_t* obs, const uint8_t* reset, cons
   // layers take [hi | lo] against [W | W], one product with fp32 accumulation
   u8_to_bf16<<<blocks_for(n * K), 256, 0, st>>>(obs, s->x16, n * K);
   S5_BLAS(gemm_bf16(b, n, H, K, s->We1, s->x16, K, s->acc, H));
-  launch_rows(bias_act_split, H / 4, n, st, s->acc, s->be1, H, 1, n, true, (float*)nullptr, s->act);
+  launch_rows(bias_act_split, H / 4, n, st, s->acc, s->be1, H, 1, n, true, (float*)nullptr, s->act, 2);
   S5_BLAS(gemm_bf16(b, n, H, 2 * H, s->We2, s->act, 2 * H, s->acc, H));
-  launch_rows(bias_act_split, H / 4, n, st, s->acc, s->be2, H, 1, n, true, s->u, (__nv_bfloat16*)nullptr);
-  // SSM (fp32): Bbar u, the recurrence, Re(C x)
-  S5_BLAS(gemm_f32(b, n, 2 * P, H, s->Bbar, s->u, s->bu));
-  launch_rows(ssm_recur, P / 4, n, st, s->lbar, s->bu, reset, state, P, n);
-  S5_BLAS(gemm_f32(b, n, H, 2 * P, s->Cc, state, s->y));
+  launch_rows(bias_act_split, H / 4, n, st, s->acc, s->be2, H, 1, n, true, s->u, s->act, 3);
+  // SSM: Bbar u and Re(C x) as three-term bf16 products, the recurrence in fp32
+  S5_BLAS(gemm_bf16(b, n, 2 * P, 3 * H, s->Bbar3, s->act, 3 * H, s->bu, 2 * P));
+  launch_rows(ssm_recur, P / 4, n, st, s->lbar, s->bu, reset, state, P, n, s->act);
+  S5_BLAS(gemm_bf16(b, n, H, 6 * P, s->Cc3, s->act, 6 * P, s->y, H));
   launch_rows(residual_gelu, H / 4, n, st, s->y, s->u, s->Dv, H, n, s->act);
   // heads: layer 0 for both heads at once ([2F] outputs, split as 2 groups of F), layers
   // 1-2 as one two-member batch (head h reads group h, writes columns h F of acc)
   S5_BLAS(gemm_bf16(b, n, 2 * F, 2 * H, s->Wh0, s->act, 2 * H, s->acc, 2 * F));
-  launch_rows(bias_act_split, 2 * F / 4, n, st, s->acc, s->bh0, F, 2, n, true, (float*)nullptr, s->act);
+  launch_rows(bias_act_split, 2 * F / 4, n, st, s->acc, s->bh0, F, 2, n, true, (float*)nullptr, s->act, 2);
   const __nv_bfloat16* Wl[2] = {s->Wh1, s->Wh2};
   const float* bl[2] = {s->bh1, s->bh2};
   for (int l = 0; l < 2; ++l) {
     S5_BLAS(gemm_bf16(b, n, F, 2 * F, Wl[l], s->act, 4 * F, s->acc, 2 * F, 2, (int64_t)F * 2 * F, 2 * F, F));
-    if (l == 0) launch_rows(bias_act_split, 2 * F / 4, n, st, s->acc, bl[l], F, 2, n, true, (float*)nullptr, s->act);
+    if (l == 0) launch_rows(bias_act_split, 2 * F / 4, n, st, s->acc, bl[l], F, 2, n, true, (float*)nullptr, s->act, 2);
   }
   // layer 2's bias and relu, and both output layers, in fp32 (one warp per env)
   const int out_blocks = (int)std::min<int64_t>((n + 7) / 8, 65535);
