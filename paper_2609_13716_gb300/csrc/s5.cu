@@ -25,6 +25,7 @@ struct aht_s5 {
   cudaStream_t stream = nullptr;
   cublasHandle_t blas = nullptr;
   int K = 0, A = 0, H = 0, P = 0, F = 0;
+  int Kp = 0;  // K rounded up to 16: observation rows and We1 rows padded with zeros
   int64_t max_n = 0;
   // bf16 weights [out][in]. A layer fed with split activations holds each weight row twice,
   // [W | W] (in = 2I), so that one product over [hi | lo] sums both halves. Heads: layer 0
@@ -42,7 +43,7 @@ struct aht_s5 {
   float *lbar = nullptr, *Dv = nullptr;
   __nv_bfloat16 *Bbar3 = nullptr, *Cc3 = nullptr;
   // scratch
-  // x16 [n][K]; act: split activations, each row [group][hi | lo][I] (heads: 2 groups of F)
+  // x16 [n][Kp]; act: split activations, each row [group][hi | lo][I] (heads: 2 groups of F)
   __nv_bfloat16 *x16 = nullptr, *act = nullptr;
   float *acc = nullptr, *u = nullptr, *bu = nullptr, *y = nullptr;
   void* workspace = nullptr;
@@ -63,9 +64,21 @@ namespace {
 
 constexpr size_t kWorkspace = 32u << 20;
 
-__global__ void u8_to_bf16(const uint8_t* __restrict__ in, __nv_bfloat16* __restrict__ out, int64_t n) {
-  const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (i < n) out[i] = __float2bfloat16_rn((float)in[i]);
+// out[r][c] = obs[r][c] as bf16 for c < K, 0 for K <= c < Kp (Kp % 4 == 0); four columns
+// a thread
+__global__ void u8_to_bf16(const uint8_t* __restrict__ in, __nv_bfloat16* __restrict__ out, int K, int Kp,
+                           int64_t n) {
+  const int c = 4 * (blockIdx.x * blockDim.x + threadIdx.x);
+  if (c >= Kp) return;
+  for (int64_t r = (int64_t)blockIdx.y * blockDim.y + threadIdx.y; r < n; r += (int64_t)gridDim.y * blockDim.y) {
+    const uint8_t* row = in + r * K;
+    float v[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) v[k] = c + k < K ? (float)row[c + k] : 0.0f;
+    __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]), b = __floats2bfloat162_rn(v[2], v[3]);
+    *reinterpret_cast<uint2*>(out + r * Kp + c) =
+        make_uint2(*reinterpret_cast<uint32_t*>(&a), *reinterpret_cast<uint32_t*>(&b));
+  }
 }
 
 // Row-wise kernels run on 2-D blocks and grids: x covers a row's columns (four per thread;
@@ -244,7 +257,6 @@ void launch_rows(void (*kernel)(KArgs...), int quads, int64_t n, cudaStream_t st
   kernel<<<L.grid, L.block, 0, st>>>(args...);
 }
 
-int blocks_for(int64_t total) { return (int)((total + 255) / 256); }
 
 // C[n][O] = X[n][I] W^T for row-major X (ld ldx), W [O][I] (ld I), C (ld ldc); `batch`
 // products at once, the b-th at W + b sW, X + b sX, C + b sC
@@ -284,6 +296,7 @@ aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_st
   aht_s5* s = new aht_s5();
   const int K = p->obs_dim, A = p->n_actions, H = p->H, P = p->P, F = p->F;
   s->K = K; s->A = A; s->H = H; s->P = P; s->F = F;
+  s->Kp = (K + 15) / 16 * 16;
   s->max_n = max_envs;
   s->stream = static_cast<cudaStream_t>(cuda_stream);
   cudaGetDevice(&s->device);
@@ -331,7 +344,9 @@ aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_st
           for (size_t c = 0; c < cols; ++c) h[o++] = __float2bfloat16_rn(w[r * cols + c]);
     return alloc((void**)dst, h.size() * 2) && cudaMemcpy(*dst, h.data(), h.size() * 2, cudaMemcpyHostToDevice) == cudaSuccess;
   };
-  bool ok = up16(&s->We1, {p->We1}, {(size_t)H * K}) && up16x2(&s->We2, {p->We2}, H, H) &&
+  std::vector<float> We1p((size_t)H * s->Kp, 0.0f);
+  for (int h = 0; h < H; ++h) std::copy(p->We1 + (size_t)h * K, p->We1 + (size_t)(h + 1) * K, We1p.begin() + (size_t)h * s->Kp);
+  bool ok = up16(&s->We1, {We1p.data()}, {We1p.size()}) && up16x2(&s->We2, {p->We2}, H, H) &&
             up16x2(&s->Wh0, {p->Wa[0], p->Wc[0]}, F, H) && up16x2(&s->Wh1, {p->Wa[1], p->Wc[1]}, F, F) &&
             up16x2(&s->Wh2, {p->Wa[2], p->Wc[2]}, F, F) &&
             up32(&s->W3, cat(bf16_rounded(p->Wa[3], (size_t)A * F), bf16_rounded(p->Wc[3], F))) &&
@@ -376,7 +391,7 @@ aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_st
   if (!up32(&s->lbar, lbar) || !up_three(&s->Bbar3, Bbar, 2 * P, H) || !up_three(&s->Cc3, Cc, H, 2 * P))
     return bail(AHT_ENOMEM, "S5 upload failed");
   const int64_t n = max_envs;
-  ok = alloc((void**)&s->x16, (size_t)n * K * 2) && alloc((void**)&s->act, (size_t)n * std::max({4 * F, 3 * H, 6 * P}) * 2) &&
+  ok = alloc((void**)&s->x16, (size_t)n * s->Kp * 2) && alloc((void**)&s->act, (size_t)n * std::max({4 * F, 3 * H, 6 * P}) * 2) &&
        alloc((void**)&s->acc, (size_t)n * std::max(2 * F, H) * 4) && alloc((void**)&s->u, (size_t)n * H * 4) &&
        alloc((void**)&s->bu, (size_t)n * 2 * P * 4) && alloc((void**)&s->y, (size_t)n * H * 4) &&
        alloc(&s->workspace, kWorkspace);
@@ -405,8 +420,8 @@ aht_status aht_s5_step(aht_s5* s, const uint8_t* obs, const uint8_t* reset, cons
   cublasHandle_t b = s->blas;
   // encoder: the observation is exact in bf16, so layer 1 is one plain product; later
   // layers take [hi | lo] against [W | W], one product with fp32 accumulation
-  u8_to_bf16<<<blocks_for(n * K), 256, 0, st>>>(obs, s->x16, n * K);
-  S5_BLAS(gemm_bf16(b, n, H, K, s->We1, s->x16, K, s->acc, H));
+  launch_rows(u8_to_bf16, s->Kp / 4, n, st, obs, s->x16, K, s->Kp, n);
+  S5_BLAS(gemm_bf16(b, n, H, s->Kp, s->We1, s->x16, s->Kp, s->acc, H));
   launch_rows(bias_act_split, H / 4, n, st, s->acc, s->be1, H, 1, n, true, (float*)nullptr, s->act, 2);
   S5_BLAS(gemm_bf16(b, n, H, 2 * H, s->We2, s->act, 2 * H, s->acc, H));
   launch_rows(bias_act_split, H / 4, n, st, s->acc, s->be2, H, 1, n, true, s->u, s->act, 3);
