@@ -1242,15 +1242,14 @@ extern "C" int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32
   std::vector<int> status(N, 0);
   parallel_for(N, io->n_threads, [&](int64_t e) {
     const uint32_t env = (uint32_t)(io->env_ids ? io->env_ids[e] : e);
-    // Teammate: one uniform pool draw per block of ORC_TEAMMATE_BLOCK consecutive envs
-    // and call, taken from the block's first env (counter (first env, step0, stream 3)).
-    // Per-episode mode: the teammate of the episode that began at step s.
+    // Teammate (Sec. 3): per call, one uniform pool draw per env at the call's first
+    // step (counter (env, step0, stream 3)), kept for the whole call; per episode, the
+    // draw of the step the current episode began (counter (env, s, stream 5)).
     auto episode_teammate = [&](uint32_t s) {
       const uint32_t x = orc_draw(io->seed, env, s, ORC_STREAM_EPISODE_TEAMMATE, 0);
       return io->pool[orc_uniform_int(x, (uint32_t)io->pool_size)];
     };
-    const uint32_t first = env - env % ORC_TEAMMATE_BLOCK;
-    const uint32_t x = orc_draw(io->seed, first, (uint32_t)io->step0, ORC_STREAM_TEAMMATE, 0);
+    const uint32_t x = orc_draw(io->seed, env, (uint32_t)io->step0, ORC_STREAM_TEAMMATE, 0);
     int tm_id = io->resample ? episode_teammate(io->ep_step[e])
                              : io->pool[orc_uniform_int(x, (uint32_t)io->pool_size)];
     if (io->teammate) io->teammate[e] = tm_id;

@@ -207,14 +207,15 @@ void orc_gae(const float* r, const float* v, const uint8_t* d, const float* v_la
              double* adv, double* targets);
 
 /* ---- PPO rollout collection (simultaneous-move envs) ---------------------------- */
-/* Teammates (Sec. 3: the ego meets teammates drawn from the training set).  Block mode:
- * envs 128k .. 128k+127 share for the whole call the teammate drawn for env 128k at the
- * call's first step.  Per-episode mode (resample = 1): each episode draws its own
- * teammate when it begins -- env e whose current episode began at step s plays
- * pool[uniform_int(x, pool_size)], x = word 0 of counter (e, s, stream 5); the step an
- * episode began is carried per env in ep_step (0 after a reset of the whole batch), and
- * every auto-reset at step s' sets it to s'. */
-enum { ORC_TEAMMATE_BLOCK = 128 };
+/* Teammates (Sec. 3: the ego meets teammates drawn from the training set).  Per-call
+ * mode: every env draws its own teammate once per call, at the call's first step --
+ * env e plays pool[uniform_int(x, pool_size)], x = word 0 of counter (e, step0,
+ * stream 3) -- and keeps it for the whole call, auto-reset episodes included.
+ * Per-episode mode (resample = 1): each episode draws its own teammate when it begins --
+ * env e whose current episode began at step s plays pool[uniform_int(x, pool_size)],
+ * x = word 0 of counter (e, s, stream 5); the step an episode began is carried per env
+ * in ep_step (0 after a reset of the whole batch), and every auto-reset at step s' sets
+ * it to s'. */
 typedef struct orc_rollout_io {
   /* inputs */
   uint64_t seed;
@@ -246,8 +247,8 @@ typedef struct orc_rollout_io {
   double* values_tm;           /* [T][N] teammate value (0 without a value row) */
   double* last_value_tm;       /* [N] teammate value of the state after the last step */
   /* per-episode teammates */
-  int32_t resample;            /* 0: block mode, 1: per-episode mode (ep_step required) */
-  uint32_t* ep_step;           /* [N] in/out, or NULL in block mode */
+  int32_t resample;            /* 0: per-call mode, 1: per-episode mode (ep_step required) */
+  uint32_t* ep_step;           /* [N] in/out, or NULL in per-call mode */
   int32_t* teammates_t;        /* [T][N] teammate policy id at each step, or NULL */
 } orc_rollout_io;
 int32_t orc_rollout(const orc_env_desc* d, const orc_mlp* pols, int32_t n_pols,

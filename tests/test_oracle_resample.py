@@ -76,7 +76,7 @@ def test_teammate_network_is_the_recorded_one():
         assert np.allclose(out["values_tm"][sel], x[:, K].numpy(), atol=1e-12)
 
 
-def test_single_member_pool_matches_block_mode():
+def test_single_member_pool_matches_per_call_mode():
     d, pols, K, N = setup(N=300)
     P = O.Policies(pols)
     a = O.rollout(d, P, 5, O.reset_all(d, 5, N), 0, 30, 0, [2],
