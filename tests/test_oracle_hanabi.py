@@ -195,3 +195,129 @@ def test_losing_all_lives_zeroes_return(orc):
             assert sum(rets) == 0.0 and rets[-1] == -float(sum(1 for x in rets if x == 1.0))
             return
     pytest.fail("no scoring game that lost all lives")
+
+
+# Observation offsets of the 660-bit Hanabi encoding (partner hand 125, own knowledge
+# 125, partner knowledge 125, fireworks 25, info 8, lives 3, deck 40, discards 50, last
+# action 53 = actor 2 | type 4 | colour 5 | rank 5 | slot 5 | card 25 | hinted 5 |
+# success 1 | bomb 1, own hints 50, partner hints 50, own slots 5, final round 1).
+PH, OK, PK, FW, INFO, LIFE, DECK, DISC, LA, OH, PHH, SLOTS, FR = (
+    0, 125, 250, 375, 400, 408, 411, 451, 501, 554, 604, 654, 659)
+R, Y, G, Wc, B = range(5)
+RANK1 = sum(1 << (c * 5) for c in range(5))       # knowledge bits of every rank-1 card
+
+
+def card(c, r):
+    return c * 5 + r - 1
+
+
+def scripted_state(orc):
+    """Seat 0: R1 G2 B1 Y4 W5; seat 1: G1 R1 Y3 B2 W1; the next draws R3, B4, Y1; the
+    rest of the deck in canonical order (the 50 cards are conserved)."""
+    s = reset(orc, 0)
+    hands = [[card(R, 1), card(G, 2), card(B, 1), card(Y, 4), card(Wc, 5)],
+             [card(G, 1), card(R, 1), card(Y, 3), card(B, 2), card(Wc, 1)]]
+    head = hands[0] + hands[1] + [card(R, 3), card(B, 4), card(Y, 1)]
+    rest = [c * 5 + r - 1 for c in range(5) for r in (1, 1, 1, 2, 2, 3, 3, 4, 4, 5)]
+    for x in head:
+        rest.remove(x)
+    for k, x in enumerate(head + rest):
+        s.deck[k] = x
+    for p in range(2):
+        for k in range(5):
+            s.hand[p][k] = hands[p][k]
+    assert conserved(s)
+    return s
+
+
+def therm(o, a, n, ones):
+    return o[a:a + ones].all() and not o[a + ones:a + n].any()
+
+
+def last_action(o, *bits):
+    want = np.zeros(53, np.uint8)
+    want[list(bits)] = 1
+    return np.array_equal(o[LA:LA + 53], want)
+
+
+def test_observation_sections_through_play_hint_discard_and_bomb(orc):
+    s = scripted_state(orc)
+    full = (1 << 25) - 1
+    # turn 0, seat 0 plays R1 from slot 0: a success, then draws R3 into slot 4
+    assert step(orc, s, 0) == (0, 1.0)
+    o = obs(orc, s, 1)
+    partner = [card(G, 2), card(B, 1), card(Y, 4), card(Wc, 5), card(R, 3)]
+    assert o[PH:OK].sum() == 5 and all(o[PH + 25 * k + x] for k, x in enumerate(partner))
+    assert o[OK:PK].all() and o[PK:FW].all()
+    assert o[FW:INFO].sum() == 1 and o[FW + 5 * R + 0] == 1           # red firework at 1
+    assert therm(o, INFO, 8, 8) and therm(o, LIFE, 3, 3) and therm(o, DECK, 40, 39)
+    assert not o[DISC:LA].any()
+    # actor = partner, type play, colour R, rank 1, slot 0, card R1, success
+    assert last_action(o, 1, 2 + 0, 6 + R, 11 + 0, 16 + 0, 21 + card(R, 1), 51)
+    assert not o[OH:SLOTS].any() and o[SLOTS:FR].all() and o[FR] == 0
+    assert o.sum() == 5 + 125 + 125 + 1 + 8 + 3 + 39 + 7 + 5
+    # the actor's own view: actor = self
+    assert last_action(obs(orc, s, 0), 0, 2 + 0, 6 + R, 11 + 0, 16 + 0, 21 + card(R, 1), 51)
+
+    # turn 1, seat 1 hints rank 1: only seat 0's slot 1 (B1) matches
+    assert step(orc, s, 15 + 0) == (0, 0.0)
+    o = obs(orc, s, 0)
+    for k in range(5):
+        bits = sum(int(b) << i for i, b in enumerate(o[OK + 25 * k:OK + 25 * k + 25]))
+        assert bits == (RANK1 if k == 1 else full & ~RANK1), k
+    assert o[OH:PHH].sum() == 1 and o[OH + 10 * 1 + 5 + 0] == 1        # own slot 1: rank 1
+    assert not o[PHH:SLOTS].any()
+    assert therm(o, INFO, 8, 7)
+    assert last_action(o, 1, 2 + 3, 11 + 0, 46 + 1)                   # hint rank 1, slot 1
+    o1 = obs(orc, s, 1)                                                # the hinter's view
+    assert np.array_equal(o1[PK:FW], o[OK:PK])
+    assert o1[PHH:SLOTS].sum() == 1 and o1[PHH + 10 * 1 + 5] == 1
+    assert last_action(o1, 0, 2 + 3, 11 + 0, 46 + 1)
+
+    # turn 2, seat 0 discards W5 from slot 3 and draws B4
+    assert step(orc, s, 5 + 3) == (0, 0.0)
+    o = obs(orc, s, 1)
+    assert o[DISC:LA].sum() == 1 and o[DISC + 10 * Wc + 9] == 1        # the single W5 copy
+    assert therm(o, INFO, 8, 8) and therm(o, DECK, 40, 38)
+    assert last_action(o, 1, 2 + 1, 6 + Wc, 11 + 4, 16 + 3, 21 + card(Wc, 5))
+    # seat 0's hand is now G2 B1 Y4 R3 B4: the hint moved with B1, the new card knows all
+    know = [full & ~RANK1, RANK1, full & ~RANK1, full & ~RANK1, full]
+    for k in range(5):
+        bits = sum(int(b) << i for i, b in enumerate(o[PK + 25 * k:PK + 25 * k + 25]))
+        assert bits == know[k], k
+    assert o[PHH:SLOTS].sum() == 1 and o[PHH + 10 + 5] == 1
+
+    # turn 3, seat 1 plays B2 from slot 3 on an empty blue firework: a bomb
+    assert step(orc, s, 3) == (0, 0.0)
+    o = obs(orc, s, 0)
+    assert therm(o, LIFE, 3, 2)
+    assert o[DISC:LA].sum() == 2 and o[DISC + 10 * Wc + 9] and o[DISC + 10 * B + 3]
+    assert last_action(o, 1, 2 + 0, 6 + B, 11 + 1, 16 + 3, 21 + card(B, 2), 52)
+    assert o[FW:INFO].sum() == 1 and o[FW + 5 * R] == 1                # score unchanged
+
+    # turn 4, seat 0 hints green: seat 1's hand is G1 R1 Y3 W1 Y1, slot 0 matches
+    assert step(orc, s, 10 + G) == (0, 0.0)
+    o = obs(orc, s, 1)
+    assert o[OH:PHH].sum() == 1 and o[OH + G] == 1                     # own slot 0: green
+    bits = sum(int(b) << i for i, b in enumerate(o[OK:OK + 25]))
+    assert bits == 0x1F << (5 * G)
+    assert last_action(o, 1, 2 + 2, 6 + G, 46 + 0)
+
+    # turn 5, seat 1 discards R1 from slot 1: the first red rank-1 copy
+    assert step(orc, s, 5 + 1) == (0, 0.0)
+    o = obs(orc, s, 0)
+    assert o[DISC:LA].sum() == 3 and o[DISC + 10 * R + 0] == 1 and o[DISC + 10 * R + 1] == 0
+    s.disc[card(R, 1)] = 2                                             # a second copy
+    o = obs(orc, s, 0)
+    assert o[DISC + 10 * R + 0] == 1 and o[DISC + 10 * R + 1] == 1 and o[DISC + 10 * R + 2] == 0
+    assert o[DISC + 10 * R + 3] == 0                                   # rank 2 starts at 3
+
+
+def test_final_round_flag_and_empty_deck_bits(orc):
+    s = reset(orc, 21)
+    while s.ptr < 50:
+        m = legal(orc, s)
+        step(orc, s, 5 if m[5] else int(np.flatnonzero(m[10:])[0]) + 10)
+    o = obs(orc, s, s.turn % 2)
+    assert o[FR] == 1 and not o[DECK:DISC].any()
+    assert o[SLOTS:FR].sum() == s.n_hand[s.turn % 2]

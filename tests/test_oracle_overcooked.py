@@ -142,3 +142,71 @@ def test_random_play_invariants(orc):
             assert (s.ax[0], s.ay[0]) != (s.ax[1], s.ay[1])
             assert done == (t == 399)
         assert s.ret % 20 == 0
+
+
+def test_item_pot_and_holding_channels_along_the_soup_script(orc):
+    """Channels 15-24 at hand-worked points of the scripted soup (index (y*5 + x)*26 + c;
+    15/16/17 onion/dish/soup on a counter or in a hand at the holder's cell, 18/19/20 pot
+    with 1/2/3 onions, 21 cooking, 22 ready, 23 self holding, 24 other holding).  Agent 0
+    starts at (1,1), the pot is at (3,0), agent 1 waits at (2,2)."""
+    d = desc(orc)
+    s = fresh(orc, d)
+    POT = (0, 3)                                      # (y, x)
+
+    def ch(seat):
+        return obs(orc, d, s, seat)[:, :, 15:25]      # channels 15..24 as [..., 0..9]
+
+    def only(o, *cells):
+        """the 10 channels are zero except at the listed (y, x, c) entries"""
+        want = np.zeros_like(o)
+        for y, x, c in cells:
+            want[y, x, c - 15] = 1
+        return np.array_equal(o, want)
+
+    t = 0
+
+    def run(a0):
+        nonlocal t
+        step(orc, d, s, a0, W if t == 0 else NOOP)
+        t += 1
+
+    assert only(ch(0)) and only(ch(1))               # empty kitchen
+    run(SCRIPT[0])                                    # t0: agent 0 takes an onion at (1,1)
+    assert s.held[0] == ONION
+    assert only(ch(0), (1, 1, 15), (1, 1, 23))        # onion in own hand, self holding
+    assert only(ch(1), (1, 1, 15), (1, 1, 24))        # seen by the other: other holding
+    for a in SCRIPT[1:5]:                             # t1..t4: first onion into the pot
+        run(a)
+    assert s.pot_n == 1
+    assert only(ch(0), (*POT, 18)) and only(ch(1), (*POT, 18))
+    for a in SCRIPT[5:13]:                            # second onion (t12)
+        run(a)
+    assert s.pot_n == 2 and only(ch(0), (*POT, 19))
+    for a in SCRIPT[13:21]:                           # third onion (t20): cooking starts
+        run(a)
+    assert (s.pot_n, s.pot_timer) == (3, 20)
+    assert only(ch(0), (*POT, 20), (*POT, 21))
+    for a in SCRIPT[21:]:                             # to the dish dispenser and back
+        run(a)
+        if s.held[0] == DISH:
+            y, x = s.ay[0], s.ax[0]
+            assert only(ch(0), (*POT, 20), (*POT, 21), (y, x, 16), (y, x, 23))
+            assert only(ch(1), (*POT, 20), (*POT, 21), (y, x, 16), (y, x, 24))
+    assert s.held[0] == DISH and (s.ax[0], s.ay[0]) == (3, 1)
+    while t < 41:                                     # still cooking through t40
+        assert ch(0)[POT[0], POT[1], 21 - 15] == 1
+        run(INTERACT)
+    assert s.pot_timer == 0                           # ready after t40
+    assert only(ch(0), (*POT, 20), (*POT, 22), (1, 3, 16), (1, 3, 23))
+    run(INTERACT)                                     # t41: soup into the dish, pot empties
+    assert s.held[0] == SOUP
+    assert only(ch(0), (1, 3, 17), (1, 3, 23)) and only(ch(1), (1, 3, 17), (1, 3, 24))
+    run(E)                                            # (4,1) is a counter: turn east
+    run(INTERACT)                                     # soup placed on the counter at (4,1)
+    assert s.held[0] == NONE and s.counter_item[1 * 5 + 4] == SOUP
+    assert only(ch(0), (1, 4, 17)) and only(ch(1), (1, 4, 17))
+    s.counter_item[0 * 5 + 0] = DISH                  # a dish on the corner counter (0,0)
+    assert only(ch(0), (1, 4, 17), (0, 0, 16))
+    s.held[1] = ONION                                 # the other agent holds an onion at (2,2)
+    assert only(ch(0), (1, 4, 17), (0, 0, 16), (2, 2, 15), (2, 2, 24))
+    assert only(ch(1), (1, 4, 17), (0, 0, 16), (2, 2, 15), (2, 2, 23))
