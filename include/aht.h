@@ -158,17 +158,20 @@ typedef struct aht_traj {
 } aht_traj;
 
 /* PPO rollout collection (App. C "PPO ego"; Sec. 3 ego vs teammates from T_train).
- * Teammates are assigned per block of AHT_TEAMMATE_BLOCK (128) consecutive envs, once per
- * call: block k plays pool[floor(x * pool_size / 2^32)] with x the first draw of counter
- * (128 k, step0, stream 3), so each env meets a uniformly drawn pool member and every
- * block runs one teammate policy (one tensor-core tile).  Then for t in 0..T-1 (step
- * step0+t): both seats observe, the ego and the teammate MLPs run, actions are
- * sampled by inverse CDF with u from stream 0/1, the env steps, and an env whose
- * episode ended is reset at step step0+t+1 (stream 2).  Finally V_T is computed and
- * GAE (advantages, targets) is formed when `advantages` is non-NULL.  The step counter
+ * Every env draws its teammate once per call: env e plays pool[floor(x * pool_size /
+ * 2^32)] with x the first draw of counter (e, step0, stream 3), and keeps it for the
+ * whole call, auto-reset episodes included, so each env meets a uniformly drawn pool
+ * member, independently of its neighbours.  The envs are grouped by their draw so that a
+ * tensor-core tile runs one teammate policy (the tiles of a group are not contiguous env
+ * ranges; a pool of p members makes at most ceil(n_envs / 128) + p tiles).  Then for t in
+ * 0..T-1 (step step0+t): both seats observe, the ego and the teammate MLPs run, actions
+ * are sampled by inverse CDF with u from stream 0/1, the env steps, and an env whose
+ * episode ended is reset at step step0+t+1 (stream 2).  Finally V_T is computed and GAE
+ * (advantages, targets) is formed when `advantages` is non-NULL.  The step counter
  * advances by T.  Simultaneous-move envs only (LBF, Overcooked): AHT_EINVAL for Hanabi.
- * pool: host [pool_size] policy ids, 1 <= pool_size <= 256.  T >= 1. */
-#define AHT_TEAMMATE_BLOCK 128
+ * pool: host [pool_size] policy ids, 1 <= pool_size <= 256 (ids may repeat; each entry is
+ * drawn with probability 1 / pool_size).  out->obs must be 4-byte aligned when
+ * pool_size > 1.  T >= 1. */
 aht_status aht_rollout(aht_ctx* ctx, int32_t ego_id, const int32_t* pool, int32_t pool_size,
                        int32_t T, const aht_traj* out);
 
@@ -239,7 +242,9 @@ aht_status aht_xplay_matrix(aht_ctx* ctx, const int32_t* ego_ids, int32_t n_ego,
  *     device current) and caches it; make that first call before any stream capture.
  *   - All calls, on every context and stream of a device, share the one array; each
  *     call writes every entry it reads before reading it, so nothing needs clearing, but
- *     calls that overlap on the GPU race and must be serialised by the caller. */
+ *     calls that overlap on the GPU race and must be serialised by the caller.
+ *   - When aht_sync reports AHT_ETIMEOUT for the call, the cells of the pairs whose
+ *     tiles gave up hold NaN (their returns are written as NaN, never left stale). */
 #define AHT_XPLAY_STATIC_MAX_ENVS 65536
 aht_status aht_xplay_matrix_static(aht_ctx* ctx, const int32_t* ego_ids, int32_t n_ego,
                                    const int32_t* tm_ids, int32_t n_tm, int32_t envs_per_pair,

@@ -835,6 +835,8 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
   if (T < 1) return fail(AHT_EINVAL, "T must be >= 1");
   if (c->step + T + 1 > (int64_t)UINT32_MAX) return fail(AHT_EINVAL, "step counter would exceed 2^32");
   if (aht_status e = check_traj_out(out)) return e;
+  if (pool_size > 1 && (reinterpret_cast<uintptr_t>(out->obs) & 3u))
+    return fail(AHT_EINVAL, "out->obs must be 4-byte aligned when pool_size > 1");
   if (out1) {
     if (aht_status e = check_traj_out(out1)) return e;
     if (reinterpret_cast<uintptr_t>(out1->obs) & 3u)
@@ -845,14 +847,23 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
   // the sparse-first-layer tensor-core kernel does plain collection; IPPO there runs on
   // the CUDA-core kernel
   const bool use_tc = c->tc && !(c->tcd.sparse && out1);
+  // Sec. 3: every env draws its teammate from the pool (once per call); with more than
+  // one member the envs are grouped by their draw, so a tile runs one teammate policy
+  const bool grouped = pool_size > 1;
+  auto n_tiles = [&](int m) -> int64_t {
+    return grouped ? resample_tiles(Nall, m, pool_size) : group_tiles(Nall, m);
+  };
   int M = 128;
   if (use_tc) {
     // a tensor-core tile's step takes about as long for 32 rows as for 128: while the
-    // batch would leave SMs idle, cut the teammate blocks into smaller tiles
-    while (M > 32 && group_tiles(Nall, M / 2) <= c->n_sms) M /= 2;
+    // batch would leave SMs idle, cut the teammate groups into smaller tiles
+    while (M > 32 && n_tiles(M / 2) <= c->n_sms) M /= 2;
   } else {
-    M = spread_rows(c, fit_rows(c, 128), 0, [&](int m) { return (int64_t)group_tiles(Nall, m); });
+    M = spread_rows(c, fit_rows(c, 128), 0, n_tiles);
   }
+  const size_t tc_smem = c->tc_smem + (grouped ? kTcGatherScratch : 0);
+  if (use_tc && tc_smem > c->smem_optin) return fail(AHT_EINVAL, "no shared memory left for the teammate grouping");
+  const int grid = (int)n_tiles(M);
 
   GroupArgs ga{};
   ga.key = batch_of(c).key;
@@ -861,11 +872,32 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
   ga.pool_size = pool_size;
   for (int k = 0; k < pool_size; ++k) ga.pool[k] = pool[k];
   ga.M = M;
-  ga.max_tiles = group_tiles(c->n_envs, M);
+  ga.max_tiles = grid;
   ga.perm = c->perm;
   ga.tiles = c->tiles;
   ga.teammate = out->teammate;
-  AHT_CUDA(launch_group(ga, c->stream));
+  if (!grouped) {
+    AHT_CUDA(launch_group(ga, c->stream));
+  } else if (use_tc) {
+    ga.kidx = c->rs_kidx;
+    ga.hist = c->rs_hist;
+    AHT_CUDA(cudaMemsetAsync(c->rs_hist, 0, (size_t)pool_size * 4, c->stream));
+    AHT_CUDA(launch_teammate_draw(ga, c->stream));
+  } else {
+    ResampleGroupArgs rg{};
+    rg.key = ga.key;
+    rg.n_envs = Nall;
+    rg.step0 = ga.step0;
+    rg.ep_step = nullptr;  // per-call draw
+    rg.pool_size = pool_size;
+    for (int k = 0; k < pool_size; ++k) rg.pool[k] = pool[k];
+    rg.M = M;
+    rg.max_tiles = grid;
+    rg.perm = c->perm;
+    rg.tiles = c->tiles;
+    rg.teammate = out->teammate;
+    AHT_CUDA(launch_resample_group(rg, c->stream));
+  }
 
   PpoArgs a{};
   a.b = batch_of(c);
@@ -900,13 +932,23 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
     ta.traj = a.traj;
     ta.traj1 = a.traj1;
     ta.ep_step = c->ep_step;
+    if (grouped) {
+      ta.gather = 1;
+      ta.g.kidx_cur = c->rs_kidx;
+      ta.g.hist_cur = c->rs_hist;
+      ta.g.scratch_off = (uint32_t)c->tc_smem;
+      ta.g.resample = 0;
+      ta.g.M = M;
+      ta.g.pool_size = pool_size;
+      for (int k = 0; k < pool_size; ++k) ta.g.pool[k] = pool[k];
+    }
     const int tk = timer_begin(c);
-    AHT_CUDA(lbf_ppo_tc(ta, ga.max_tiles, c->tc_smem, c->stream));
+    AHT_CUDA(lbf_ppo_tc(ta, grid, tc_smem, c->stream));
     timer_end(c, tk);
   } else {
     const size_t smem = smem_layout(M, c->mlp, c->ops.bytes()).total;
     const int tk = timer_begin(c);
-    AHT_CUDA(c->ops.ppo(a, ga.max_tiles, smem, c->stream));
+    AHT_CUDA(c->ops.ppo(a, grid, smem, c->stream));
     timer_end(c, tk);
   }
   if (out->advantages)
@@ -970,6 +1012,8 @@ aht_status aht_rollout_resample(aht_ctx* c, int32_t ego_id, const int32_t* pool,
     ta.ep_step = c->ep_step;
     ta.gather = 1;
     ta.g.scratch_off = (uint32_t)c->tc_smem;
+    ta.g.resample = 1;
+    ta.g.M = 128;
     ta.g.pool_size = pool_size;
     for (int k = 0; k < pool_size; ++k) ta.g.pool[k] = pool[k];
     for (int t = 0; t < T; ++t) {
@@ -1001,6 +1045,7 @@ aht_status aht_rollout_resample(aht_ctx* c, int32_t ego_id, const int32_t* pool,
   ResampleGroupArgs ga{};
   ga.key = batch_of(c).key;
   ga.n_envs = N;
+  ga.step0 = (uint32_t)c->step;
   ga.ep_step = c->ep_step;
   ga.pool_size = pool_size;
   for (int k = 0; k < pool_size; ++k) ga.pool[k] = pool[k];

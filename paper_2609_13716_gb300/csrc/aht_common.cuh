@@ -11,7 +11,6 @@ namespace aht {
 constexpr int kThreads = 256;       // threads per CTA of the rollout kernels
 constexpr int kMaxPool = 256;       // teammate pool entries passed by value
 constexpr int kMaxXpIds = 64;       // ego / teammate ids per cross-play call
-constexpr int kTeammateBlock = 128; // envs per teammate draw (AHT_TEAMMATE_BLOCK)
 
 // Device status word bits (latched with atomicOr, read by aht_sync).
 enum : uint32_t {

@@ -77,22 +77,28 @@ struct TcXp {
   uint8_t* actions;        // optional [max_steps][n_total][2], pre-filled with 255
 };
 
-// Per-episode teammates on the tensor-core rollout, one launch per step.  Each env
-// carries the pool index of its episode's teammate (kidx, double-buffered by step) and
-// the launch carries the envs per index (hist, triple-buffered).  CTA j takes tile j of
-// the groups laid out in pool-index order (each group cut into tiles of up to 128 envs
-// in env order), finds its envs by a rank scan of kidx, steps them, writes each env's
-// index for the next step (a new draw after an auto-reset) and adds the next step's
-// counts; CTA 0 zeroes the buffer the step after next will count into.
+// Gathered tiles of the tensor-core rollout: the envs of one tile share a teammate's
+// pool index but are not a contiguous range.  Each env carries its pool index (kidx) and
+// the launch the envs per index (hist).  CTA j takes tile j of the groups laid out in
+// pool-index order (each group cut into tiles of up to M envs in env order) and finds
+// its envs by a rank scan of kidx.
+//   Per call (resample = 0): kidx / hist of the call's draw; the tile keeps its envs for
+//   all T steps of the launch.
+//   Per episode (resample = 1, one launch per step): kidx double-buffered and hist
+//   triple-buffered by step; the launch writes each env's index for the next step (a new
+//   draw after an auto-reset) and adds the next step's counts; CTA 0 zeroes the buffer
+//   the step after next will count into.
 struct TcGather {
   const uint8_t* kidx_cur;  // [N] pool index per env at this step (16-byte aligned)
-  uint8_t* kidx_next;       // [N] at the next step
+  uint8_t* kidx_next;       // [N] at the next step (per episode)
   const int32_t* hist_cur;  // [pool_size] envs per index at this step
-  int32_t* hist_next;       // [pool_size] accumulated for the next step (zero on entry)
-  int32_t* hist_zero;       // [pool_size] zeroed by CTA 0
-  int32_t* teammate;        // optional [N]: policy of each env at this step
-  int32_t* teammate2;       // optional second copy
+  int32_t* hist_next;       // [pool_size] accumulated for the next step (per episode; zero on entry)
+  int32_t* hist_zero;       // [pool_size] zeroed by CTA 0 (per episode)
+  int32_t* teammate;        // optional [N]: policy of each env at this step (per episode)
+  int32_t* teammate2;       // optional second copy (per episode)
   uint32_t scratch_off;     // dynamic shared-memory offset of the scan scratch
+  int32_t resample;         // 1: per-episode mode
+  int32_t M;                // rows per tile (32, 64 or 128)
   int32_t pool_size;
   int32_t pool[kMaxPool];
 };
@@ -109,7 +115,7 @@ struct PpoTcArgs {
   uint32_t step0;
   int32_t T;
   uint32_t* ep_step;     // as in PpoArgs
-  int32_t gather;        // per-episode teammates, one step per launch (see TcGather)
+  int32_t gather;        // gathered tiles (see TcGather)
   TrajPtrs traj;
   TrajPtrs traj1;        // as in PpoArgs
   TcXp xp;               // cross-play launches only
@@ -158,6 +164,7 @@ struct XpTcArgs {
   uint8_t* actions;        // optional [max_steps][n_total][2]
 };
 
+// Teammate assignment of one collection call (per-call draw, counter (e, step0, stream 3)).
 struct GroupArgs {
   Key key;
   int64_t n_envs;
@@ -166,17 +173,21 @@ struct GroupArgs {
   int32_t pool[kMaxPool];
   int32_t M;
   int32_t max_tiles;
-  int32_t* perm;
-  int4* tiles;
+  int32_t* perm;         // group_kernel (one-member pool): identity
+  int4* tiles;           // group_kernel: contiguous tiles of up to M envs
   int32_t* teammate;     // optional [n_envs]
+  uint8_t* kidx;         // teammate_draw_kernel: [n_envs] pool index per env
+  int32_t* hist;         // teammate_draw_kernel: [pool_size] += envs per index (zeroed before)
 };
 
-// Per-episode teammates: env e plays pool[uniform_int(x, pool_size)] with x the first
-// draw of counter (e, ep_step[e], stream 5); perm lists the envs grouped by pool index,
+// Teammates grouped for the CUDA-core rollout: env e plays pool[uniform_int(x, pool_size)]
+// with x the first draw of counter (e, ep_step[e], stream 5) per episode, or of (e, step0,
+// stream 3) per call when ep_step is NULL; perm lists the envs grouped by pool index,
 // tiles (perm offset, count, policy, -) cover each group in tiles of up to M envs.
 struct ResampleGroupArgs {
   Key key;
   int64_t n_envs;
+  uint32_t step0;
   const uint32_t* ep_step;
   int32_t pool_size;
   int32_t pool[kMaxPool];
@@ -263,12 +274,13 @@ cudaError_t minihanabi_xplay_tc_smem_limit(size_t smem);
 size_t xp_tc_smem_bytes(const WideDims& w);
 
 // misc.cu
-cudaError_t launch_group(const GroupArgs&, cudaStream_t);
+cudaError_t launch_group(const GroupArgs&, cudaStream_t);          // one-member pool
+cudaError_t launch_teammate_draw(const GroupArgs&, cudaStream_t);  // kidx, hist, teammate
 cudaError_t launch_policy(const PolicyArgs&, int grid, size_t smem, cudaStream_t);
 cudaError_t policy_set_smem_limit(size_t bytes);
 cudaError_t launch_tanh_probe(const float* x, float* y, int64_t n, cudaStream_t);
 cudaError_t launch_expire_wait(uint32_t* status, uint64_t limit_ns, cudaStream_t);
-int group_tiles(int64_t n_envs, int M);  // tile-table entries of a launch
+int group_tiles(int64_t n_envs, int M);  // tile-table entries of a one-member-pool launch
 cudaError_t launch_resample_group(const ResampleGroupArgs&, cudaStream_t);
 int resample_tiles(int64_t n_envs, int M, int pool_size);  // tile-table entries, per-episode mode
 // kidx[e] = pool index of env e's episode teammate, hist[k] += envs with index k

@@ -9,30 +9,46 @@
 
 namespace aht {
 
-// ---- teammate assignment: one pool draw per block of kTeammateBlock envs ---------------
-// Block k (envs 128k .. 128k+127) plays pool[floor(x * pool_size / 2^32)], x = first draw
-// of (128k, step0, stream 3).  Tiles of up to M rows never cross a block, so each tile
-// runs one teammate policy; the env order is the identity (perm[e] = e).
+// ---- teammate assignment (Sec. 3: teammates drawn uniformly from the training pool) ----
+// Per call, env e plays pool[floor(x * pool_size / 2^32)], x = first draw of (e, step0,
+// stream 3), for the whole call.  With a one-member pool every env plays pool[0] (the
+// draw is 0 whatever x is): group_kernel cuts the envs into contiguous tiles of up to M
+// (perm[e] = e).  With a larger pool, teammate_draw_kernel writes each env's pool index
+// and the envs per index; the tensor-core rollout then finds each tile's envs by a rank
+// scan, and the CUDA-core path groups them with resample_group_kernel (per-call draw).
 __global__ void group_kernel(const GroupArgs a) {
   const int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (e >= a.n_envs) return;
-  const int64_t blk = e / kTeammateBlock, first = blk * kTeammateBlock;
-  const uint32_t b = uniform_int(draw0(a.key, (uint32_t)first, a.step0, kStreamTeammate), (uint32_t)a.pool_size);
-  const int tm = a.pool[b];
+  const int tm = a.pool[0];
   a.perm[e] = (int32_t)e;
   if (a.teammate) a.teammate[e] = tm;
-  if (e == first) {
-    const int n_blk = (int)min((int64_t)kTeammateBlock, a.n_envs - first);
-    const int tpb = (kTeammateBlock + a.M - 1) / a.M;
-    for (int j = 0; j < tpb; ++j) {
-      const int r0 = j * a.M, cnt = max(0, min(a.M, n_blk - r0));
-      a.tiles[blk * tpb + j] = make_int4((int)first + r0, cnt, tm, 0);
-    }
-  }
+  if (e % a.M == 0) a.tiles[e / a.M] = make_int4((int)e, (int)min((int64_t)a.M, a.n_envs - e), tm, 0);
 }
 
-int group_tiles(int64_t n_envs, int M) {
-  return (int)(((n_envs + kTeammateBlock - 1) / kTeammateBlock) * ((kTeammateBlock + M - 1) / M));
+int group_tiles(int64_t n_envs, int M) { return (int)((n_envs + M - 1) / M); }
+
+__global__ void teammate_draw_kernel(const GroupArgs a) {
+  __shared__ int cnt[kMaxPool];
+  const uint32_t P = (uint32_t)a.pool_size;
+  for (int k = threadIdx.x; k < (int)P; k += blockDim.x) cnt[k] = 0;
+  __syncthreads();
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < a.n_envs;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const uint32_t k = uniform_int(draw0(a.key, (uint32_t)e, a.step0, kStreamTeammate), P);
+    a.kidx[e] = (uint8_t)k;
+    if (a.teammate) a.teammate[e] = a.pool[k];
+    atomicAdd(&cnt[k], 1);
+  }
+  __syncthreads();
+  for (int k = threadIdx.x; k < (int)P; k += blockDim.x)
+    if (cnt[k]) atomicAdd(&a.hist[k], cnt[k]);
+}
+
+cudaError_t launch_teammate_draw(const GroupArgs& a, cudaStream_t s) {
+  int64_t blocks = (a.n_envs + 255) / 256;
+  if (blocks > 148) blocks = 148;
+  teammate_draw_kernel<<<(unsigned)blocks, 256, 0, s>>>(a);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_group(const GroupArgs& a, cudaStream_t s) {
@@ -40,7 +56,7 @@ cudaError_t launch_group(const GroupArgs& a, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-// ---- per-episode teammates: group the envs by their episode's pool index ----------------
+// ---- group the envs by their teammate's pool index (per episode, or per call) ----------
 // One CTA: count the envs per pool index (shared-memory atomics), lay the groups out
 // back to back in perm and cut each into tiles of up to M envs, then scatter the env ids.
 // The order of the envs inside a group is not fixed (atomic slots); every row's result
@@ -50,8 +66,12 @@ __global__ void __launch_bounds__(1024) resample_group_kernel(const ResampleGrou
   __shared__ int n_tiles;
   const int tid = threadIdx.x;
   const uint32_t P = (uint32_t)a.pool_size;
+  // per episode: the draw of the step the env's episode began; per call (ep_step NULL):
+  // the draw of the call's first step on the teammate stream
   auto index_of = [&](int64_t e) {
-    return (int)uniform_int(draw0(a.key, (uint32_t)e, a.ep_step[e], kStreamEpisodeTeammate), P);
+    return (int)uniform_int(a.ep_step ? draw0(a.key, (uint32_t)e, a.ep_step[e], kStreamEpisodeTeammate)
+                                      : draw0(a.key, (uint32_t)e, a.step0, kStreamTeammate),
+                            P);
   };
   for (int k = tid; k < a.pool_size; k += blockDim.x) cnt[k] = 0;
   __syncthreads();

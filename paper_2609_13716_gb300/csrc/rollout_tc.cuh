@@ -1,7 +1,9 @@
 // rollout_tc.cuh -- fused PPO rollout with the policy MLPs on tcgen05 tensor cores.
 //
-// One CTA owns a tile of up to 128 envs that share one teammate policy, for all T steps
-// (per-episode teammates: for one step, the tile's envs found by a rank scan, kGather).
+// One CTA owns a tile of up to 128 envs that share one teammate policy, for all T steps:
+// a contiguous env range (one-member pools, cross-play), or the envs of one teammate's
+// group found by a rank scan of the per-env pool indices (kGather; per-episode
+// teammates: one step per launch).
 // Per step and agent (ego = seat 0, teammate = seat 1):
 //   obs (u8, shared memory, a constant 1 after the last feature) -> A operand in tensor
 //       memory as bf16 (exact: small integers)
@@ -16,9 +18,12 @@
 //
 // Warp roles: warps 0-7 ("compute", 256 threads) build observations, run the epilogues
 // (thread r and r + 128 own env row r, tensor-memory lane r; the halves split the
-// columns), sample and step the envs; warp 8 issues every MMA.  They meet only through
-// mbarriers: operand-ready (256 arrivals from the compute threads) and accumulator-ready
-// (a tcgen05.commit).  Each of these barriers completes once per step, so its phase
+// columns), sample and step the envs; warp 8 issues every MMA; warps 9-12 store the
+// ego's observation rows of gathered tiles (scattered rows, a quarter each, one warp per
+// SM sub-partition) while the compute warps go on.  They meet only through mbarriers:
+// operand-ready (256 arrivals from the compute threads) and accumulator-ready (a
+// tcgen05.commit); observation rows ready (256 arrivals) and observation buffer free
+// (one arrival per store warp).  Each of these barriers completes once per step, so its phase
 // parity is the step's parity.  Compute warps synchronise among themselves with a named
 // barrier that also ORs an error flag.  Weights are bulk-copied (TMA) into shared memory
 // once per CTA.  Every wait is bounded: on expiry the CTA records kStatusTimeout, stops,
@@ -34,7 +39,8 @@
 namespace aht {
 
 constexpr int kTcCompute = 256;          // compute threads
-constexpr int kTcThreads = 288;          // + one MMA warp
+constexpr int kTcThreads = 416;          // + one MMA warp + four observation-store warps
+constexpr int kTcStoreWarps = 4;         // warps 9-12: one per SM sub-partition
 constexpr int kTcComputeBar = 1;         // named barrier id of the compute warps
 constexpr int kTcPairBar = 2;            // ids 2..5: warps q and q + 4 (rows 32q .. 32q + 31)
 
@@ -43,9 +49,10 @@ constexpr int kTcPairBar = 2;            // ids 2..5: warps q and q + 4 (rows 32
 // of PPO collection.  kSplit: fp32 weights held as bf16 pairs W = W_hi + W_lo, L1 =
 // X W1_hi + X W1_lo and L2 = b2 + hi W2_hi + lo W2_hi + hi W2_lo (lo W2_lo is below
 // 2^-16 of the sum and left out).  kIppo (PPO collection only): seat 1 learns too, and
-// its trajectory goes to a.traj1.  kGather (PPO collection, one step per launch): the
-// tile's rows are the envs perm[tile.x + r] (a group of envs whose episodes drew the
-// same teammate) instead of a contiguous range.  kSparse (observations wider than the
+// its trajectory goes to a.traj1.  kGather (PPO collection): the tile's rows are envs of
+// one teammate group found by a rank scan of the per-env pool indices (the call's draw
+// for all T steps, or, per episode, one step per launch) instead of a contiguous range.
+// kSparse (observations wider than the
 // 256 tensor-memory columns of an agent's A operand; Env::sparse_obs required): no first
 // layer on the tensor cores -- each thread forms its half of h1 = tanh(c + sum over the
 // observation's changed features of delta W1[:, f]) on CUDA cores from the fp32 W1^T and
@@ -54,13 +61,15 @@ template <class Env, bool kXp, bool kSplit, bool kIppo, bool kGather, bool kSpar
 __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a) {
   static_assert(!(kXp && kIppo), "seat-1 trajectories belong to PPO collection");
   static_assert(!(kGather && (kXp || kIppo)), "gathered tiles are plain PPO collection");
-  static_assert(!(kSparse && (kIppo || kGather)), "the sparse first layer serves plain collection and cross-play");
+  static_assert(!(kSparse && kIppo), "the sparse first layer serves plain collection and cross-play");
+  static_assert(kTcThreads / 32 + 3 <= 16, "gather scratch: one total per warp and 3 selection words");
   using State = typename Env::State;
   constexpr int NA = Env::kNumActions;
   extern __shared__ __align__(16) uint8_t smem[];  // no-swizzle operands need 16 B
   __shared__ __align__(8) uint64_t acc_bar[4];     // [2*agent + layer], tcgen05.commit
   __shared__ __align__(8) uint64_t opnd_bar[4];    // [2*agent + layer], 256 arrivals
   __shared__ __align__(8) uint64_t wload_bar, drain_bar;
+  __shared__ __align__(8) uint64_t obs_full, obs_free;  // gathered observation rows: warps 9-12
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
   __shared__ volatile int stop_flag;               // cross-play: every env of the tile is done
@@ -77,33 +86,34 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     tm_pol = a.xp.tm_ids[pair % a.xp.n_tm];
   } else if constexpr (kGather) {
     // Tile blockIdx.x of the groups in pool-index order: group k holds hist_cur[k] envs,
-    // cut into tiles of up to 128 in env order.  Rows are found by a rank scan of kidx:
+    // cut into tiles of up to M in env order.  Rows are found by a rank scan of kidx:
     // each thread counts its contiguous chunk's envs of group k, an exclusive scan gives
     // the chunk's first rank, and the envs of ranks [r0, r0 + count) become rows.
-    int* wsum = reinterpret_cast<int*>(rowenv + 128);  // [0, 9) warp totals, [10, 13) selection
+    int* wsum = reinterpret_cast<int*>(rowenv + 128);  // [0, 13) warp totals, [13, 16) selection
     const int t0 = threadIdx.x, w0 = t0 >> 5, l0 = t0 & 31;
-    if (blockIdx.x == 0)
+    if (blockIdx.x == 0 && a.g.resample)
       for (int k = t0; k < a.g.pool_size; k += blockDim.x) a.g.hist_zero[k] = 0;
     if (t0 < 128) rowenv[t0] = -1;
     if (t0 == 0) {
+      const int M = a.g.M;
       int cum = 0, ks = -1, r0 = 0, cnt = 0;
       for (int k = 0; k < a.g.pool_size; ++k) {
-        const int h = a.g.hist_cur[k], nt = (h + 127) >> 7;
+        const int h = a.g.hist_cur[k], nt = (h + M - 1) / M;
         if (ks < 0 && (int)blockIdx.x < cum + nt) {
           ks = k;
-          r0 = ((int)blockIdx.x - cum) * 128;
-          cnt = min(128, h - r0);
+          r0 = ((int)blockIdx.x - cum) * M;
+          cnt = min(M, h - r0);
         }
         cum += nt;
       }
-      wsum[10] = ks;
-      wsum[11] = r0;
-      wsum[12] = ks < 0 ? 0 : cnt;
+      wsum[13] = ks;
+      wsum[14] = r0;
+      wsum[15] = ks < 0 ? 0 : cnt;
     }
     __syncthreads();
-    g_k = wsum[10];
-    const int r0 = wsum[11];
-    count = wsum[12];
+    g_k = wsum[13];
+    const int r0 = wsum[14];
+    count = wsum[15];
     env0 = 0;
     ego_pol = a.ego;
     tm_pol = g_k < 0 ? 0 : a.g.pool[g_k];
@@ -195,6 +205,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   // V_T after the last step: the ego's, and seat 1's when it learns too (IPPO)
   const bool boot1 = kIppo && !tm_rule && a.traj1.last_value != nullptr;
   const bool with_boot = !kXp && (a.traj.last_value != nullptr || boot1);
+  // gathered tiles: warps 9-12 store the ego's observation rows of every step
+  const bool obs_warp = kGather && a.traj.obs != nullptr;
 
   // The tile is the contiguous env range [tile.x, tile.x + count); observation rows are
   // packed at obs_dim bytes (an odd number of words: no bank conflicts per thread row),
@@ -212,6 +224,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     }
     tc::mbar_init(&wload_bar, 1);
     tc::mbar_init(&drain_bar, 1);
+    tc::mbar_init(&obs_full, kTcCompute);
+    tc::mbar_init(&obs_free, kTcStoreWarps);
     tc::mbar_init_fence();
     abort_flag = 0;
     stop_flag = 0;
@@ -293,6 +307,46 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         if (ok) issue(0, 1, par);
       }
       if (!ok) abort_flag = 1;
+    }
+  } else if (warp > 8) {
+    // ======================= observation-store warps (gathered) =====================
+    // Step t's ego rows (built by the compute warps, obs_full phase t) go to their envs'
+    // trajectory rows with consecutive words, warp 9 + q taking rows q, q + 4, ...;
+    // obs_free (one arrival per warp) tells the compute warps that the buffer may be
+    // rebuilt.
+    const int q = warp - 9;
+    for (int t = 0; obs_warp && t < a.T; ++t) {
+      int ok = 0;
+      if (lane == 0)
+        for (int tries = 0; tries < 1000 && !ok && !abort_flag; ++tries)
+          ok = tc::mbar_wait(&obs_full, (uint32_t)t & 1u, 2000000ull);
+      ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
+      __syncwarp();
+      if (!ok) break;  // the compute warps gave up
+      // lane l moves word w0 + l of 8 rows per iteration: 8 independent shared-memory
+      // loads in flight, then 8 stores (each row's words leave as consecutive words)
+      uint32_t* const base = reinterpret_cast<uint32_t*>(a.traj.obs + (int64_t)t * N * od);
+      const uint32_t* const src = reinterpret_cast<const uint32_t*>(sObs);
+      for (int w0 = 0; w0 < cells; w0 += 32) {
+        const int w = w0 + lane;
+        const bool wok = w < cells;
+#pragma unroll 1
+        for (int r0 = q; r0 < count; r0 += 4 * 8) {
+          uint32_t v[8];
+          int64_t dst[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int r = min(r0 + 4 * j, count - 1);
+            dst[j] = (int64_t)rowenv[r] * cells + w;
+            v[j] = wok ? src[r * cells + w] : 0u;
+          }
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            if (wok && r0 + 4 * j < count) base[dst[j]] = v[j];
+        }
+      }
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&obs_free);
     }
   } else {
     // ============================== compute warps ===================================
@@ -458,20 +512,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     };
     // the tile's ego observation rows -> trajectory [t][env0 .. env0+count): one contiguous
     // block, written by one bulk (TMA) store when 16-byte aligned, else by all threads
+    // (gathered tiles: warp 9)
     const bool bulk_obs = !kXp && !kGather && a.traj.obs && (count * od) % 16 == 0;
     auto copy_obs = [&](int t) {
-      if constexpr (kGather) {
-        // scattered rows: warps q and q + 4 store rows 32q .. 32q + 31, one row at a time
-        // with consecutive words; lane i of either warp holds the env of row 32q + i
-        const int q = warp & 3, pt = half * 32 + lane, n = min(32, count - 32 * q);
-        for (int i = 0; i < n; ++i) {
-          const int env = __shfl_sync(0xFFFFFFFFu, (int)my_env, i);
-          uint32_t* d32 = reinterpret_cast<uint32_t*>(a.traj.obs + ((int64_t)t * N + env) * od);
-          const uint32_t* s32 = reinterpret_cast<const uint32_t*>(sObs + (32 * q + i) * od);
-          for (int w = pt; w < cells; w += 64) d32[w] = s32[w];
-        }
-        return;
-      }
       uint8_t* dst = a.traj.obs + ((int64_t)t * N + env0) * od;
       const uint32_t bytes = (uint32_t)(count * od);
       if (bulk_obs && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
@@ -503,6 +546,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
           break;
         }
       }
+      // gathered tiles: the previous step's ego rows must have left the buffer
+      if (obs_warp && t >= 1) {
+        if (!bad && !tc::mbar_wait(&obs_free, (uint32_t)(t - 1) & 1u)) bad = true;
+        bad = __any_sync(0xFFFFFFFFu, bad);
+      }
       // teammate first: the ego's rows stay for the copy
       const int first = (boot && !boot1) || tm_rule ? 0 : 1;
       const uint32_t par = (uint32_t)t & 1u, gt = a.step0 + (uint32_t)t;
@@ -515,10 +563,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
           // the ego's u8 row is the trajectory's observation; no first layer to feed
           if (!kXp && i == 0 && !boot && a.traj.obs && row < count)
             Env::obs_words(a.b.env, s, 0, reinterpret_cast<uint32_t*>(sObs + row * od), my_w0, my_w1);
+          if (obs_warp && i == 0 && !boot) tc::mbar_arrive(&obs_full);
           if (!bad) sparse_h1(i, s);
           continue;
         }
         obs_x(i, s);
+        if (obs_warp && i == 0 && !boot) tc::mbar_arrive(&obs_full);
         if (kIppo && i == 1 && !boot && a.traj1.obs) {
           // seat 1's rows -> its trajectory before the ego's overwrite them: warps q and
           // q + 4 built rows 32q .. 32q + 31, a contiguous block in shared and in global
@@ -539,7 +589,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         wait_acc(i, 0, par);
         if (!bad) epilogue1(i);
       }
-      if (!kXp && !boot && a.traj.obs) {  // overlaps L2 on the tensor cores
+      if (!kXp && !kGather && !boot && a.traj.obs) {  // overlaps L2 on the tensor cores
         tc::fence_proxy_async();       // the rows were written by ordinary stores
         if (sync_or()) break;
         copy_obs(t);
@@ -629,7 +679,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
           Env::reset(a.b.env, a.b.key, (uint32_t)env, gt + 1, s);
           if (a.ep_step) a.ep_step[env] = gt + 1;
         }
-        if constexpr (kGather) {  // the next step's pool index: a new episode draws again
+        if (kGather && a.g.resample) {  // the next step's pool index: a new episode draws again
           int kn = g_k;
           if (done > 0) {
             kn = (int)uniform_int(draw0(a.b.key, (uint32_t)env, gt + 1, kStreamEpisodeTeammate),
@@ -641,7 +691,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         }
         st[row] = s;
       }
-      if constexpr (kGather) {
+      if (kGather && a.g.resample) {
         if (half == 0) {  // warps 0-3: one count per warp of the rows that keep the teammate
           const unsigned m = __ballot_sync(0xFFFFFFFFu, stayed);
           if (lane == 0 && m) atomicAdd(&a.g.hist_next[g_k], __popc(m));
@@ -653,6 +703,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     if (tid == 0 && bulk_obs) tc::bulk_wait_all();
     if (bad || abort_flag) {
       abort_flag = 1;
+      // cross-play: the tile gave up, so its returns are undefined; NaN (not a stale
+      // entry of an earlier call) makes every mean over them NaN
+      if (kXp && tid < count) a.xp.returns[env0 + tid] = __int_as_float(0x7FC00000);
     } else if (tid < count) {
       if constexpr (kXp) {
         a.xp.returns[env0 + tid] = Env::ret(st[tid]);
@@ -694,7 +747,10 @@ struct LaunchTc {
     const bool ippo = u.obs || u.actions || u.tm_actions || u.logp || u.values || u.rewards ||
                       u.dones || u.last_value;
     if (a.tc.sparse) {  // plain collection only (the host keeps the others on CUDA cores)
-      if (ippo || a.gather) return cudaErrorNotSupported;
+      if (ippo || (a.gather && a.g.resample)) return cudaErrorNotSupported;
+      if (a.gather)
+        return a.tc.split ? run<false, true, false, true, true>(a, grid, smem, s)
+                          : run<false, false, false, true, true>(a, grid, smem, s);
       return a.tc.split ? run<false, true, false, false, true>(a, grid, smem, s)
                         : run<false, false, false, false, true>(a, grid, smem, s);
     }

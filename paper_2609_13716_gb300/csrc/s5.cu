@@ -20,6 +20,20 @@ aht_status set_last_error(aht_status s, const char* msg);  // the message of aht
 
 using namespace aht;
 
+namespace {
+// Makes the S5 context's device current for the call (and restores the caller's).
+struct S5DeviceGuard {
+  int prev = -1;
+  explicit S5DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) cudaSetDevice(dev);
+    else prev = -1;
+  }
+  ~S5DeviceGuard() {
+    if (prev >= 0) cudaSetDevice(prev);
+  }
+};
+}  // namespace
+
 struct aht_s5 {
   int device = 0;
   cudaStream_t stream = nullptr;
@@ -406,6 +420,7 @@ aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_st
 
 void aht_s5_destroy(aht_s5* s) {
   if (!s) return;
+  S5DeviceGuard g(s->device);
   if (s->blas) cublasDestroy(s->blas);
   for (void* q : s->owned) cudaFree(q);
   delete s;
@@ -415,6 +430,7 @@ aht_status aht_s5_step(aht_s5* s, const uint8_t* obs, const uint8_t* reset, cons
                        int64_t n, float* state, float* logits, float* values) {
   if (!s || !obs || !reset || !state || !logits || !values) return set_last_error(AHT_EINVAL, "NULL argument");
   if (n < 1 || n > s->max_n) return set_last_error(AHT_EINVAL, "n must be in 1..max_envs");
+  S5DeviceGuard g(s->device);
   const int K = s->K, A = s->A, H = s->H, P = s->P, F = s->F;
   cudaStream_t st = s->stream;
   cublasHandle_t b = s->blas;
@@ -454,6 +470,7 @@ aht_status aht_s5_step(aht_s5* s, const uint8_t* obs, const uint8_t* reset, cons
 
 aht_status aht_s5_sync(aht_s5* s) {
   if (!s) return set_last_error(AHT_EINVAL, "NULL argument");
+  S5DeviceGuard g(s->device);
   S5_CUDA(cudaStreamSynchronize(s->stream));
   return AHT_OK;
 }

@@ -5,7 +5,7 @@ first step, exact), and the trajectory follows the usual rollout protocol (obser
 rewards, dones exact; sampled actions equal away from CDF edges; logp / values / V_T
 within the rollout tolerance; GAE teacher-forced).  Cases: the bf16 tensor-core kernel
 with network and rule teammates, fp32-split weights, the CUDA-core kernel, calls that
-carry episodes across, a block-mode call before a per-episode one, the checkpoint, and
+carry episodes across, a per-call aht_rollout before a per-episode one, the checkpoint, and
 the full 16384 x 128 launch on sampled envs."""
 import dataclasses
 
@@ -76,8 +76,8 @@ def test_cuda_core_kernel():
     run_and_check(wl, ctx, pop_np, st, np.zeros(N, np.uint32), 0, T, 2, [9, 10, 11])
 
 
-def test_block_mode_call_then_per_episode_call():
-    """A block-mode aht_rollout also records where episodes begin, so a per-episode call
+def test_per_call_rollout_then_per_episode_call():
+    """A per-call aht_rollout also records where episodes begin, so a per-episode call
     after it draws from the right steps."""
     require_gpu()
     wl = short_lbf(W.WORKLOADS["lbf7x7_ppo_16384x128"], 11)

@@ -133,7 +133,33 @@ def test_full_size_16384x128_sampled_envs():
     d, _ = oracle_of(wl.env, pop_np)
     st = O.reset_envs(d, wl.env_seed, ids)
     check_rollout(wl, pop_np, traj, st, wl.env_seed, 0, wl.T, wl.ego_id, list(wl.pool), env_ids=ids)
+    # every env's teammate draw, bit-exact against the oracle's (one step of all envs)
+    ref = O.rollout(d, O.Policies(pop_np), wl.env_seed, O.reset_all(d, wl.env_seed, wl.n_envs), 0, 1,
+                    wl.ego_id, list(wl.pool), n_threads=8)
+    assert ref["rc"] == 0
+    assert np.array_equal(np_(traj["teammate"]), ref["teammate"]), "teammate draws"
     # properties over all envs: dones at most every 50 steps, rewards in [0, 1]
     r = np_(traj["rewards"])
     assert (r >= 0).all() and (r <= 1.0 + 1e-6).all()
     assert (np_(traj["dones"]).sum(0) >= 2).all()
+
+
+@pytest.mark.parametrize("N,pool", [
+    (1, list(range(1, 33)) * 8),             # one env, a 256-entry pool: one tile
+    (300, list(range(1, 33)) * 8),           # most of 256 groups empty or single-env
+    (517, [5, 5, 5, 7]),                     # repeated ids: entries are drawn, not ids
+    (2000, [-1, 3, -12, 4, -6]),             # rule teammates among networks
+])
+def test_per_call_teammate_groups_edge_cases(N, pool):
+    """Per-call teammate draws grouped into gathered tensor-core tiles: a single env,
+    empty and single-env groups, repeated pool ids and rule teammates."""
+    require_gpu()
+    wl = W.WORKLOADS["lbf7x7_ppo_16384x128"]
+    T = 12
+    ctx, pop_np = make_ctx(wl, N)
+    d, _ = oracle_of(wl.env, pop_np)
+    st = O.reset_all(d, wl.env_seed, N)
+    traj = aht.traj_buffers(ctx, T)
+    aht.aht_rollout(ctx, 0, pool, T, traj)
+    aht.aht_sync(ctx)
+    check_rollout(wl, pop_np, traj, st, wl.env_seed, 0, T, 0, pool)
