@@ -102,7 +102,7 @@ struct TcGather {
   int32_t pool_size;
   int32_t pool[kMaxPool];
 };
-constexpr uint32_t kTcGatherScratch = 128 * 4 + 16 * 4;  // row envs, warp totals, selection
+constexpr uint32_t kTcGatherScratch = 128 * 4 + 32 * 4;  // row envs, warp totals, selection
 
 struct PpoTcArgs {
   Batch b;
@@ -261,6 +261,8 @@ AHT_DECLARE_ENV_LAUNCHERS(minihanabi)
 // columns of tensor memory; PPO collection (grid = tile table entries) and cross-play
 // (grid = pairs x tpp).  a.tc.split selects the fp32 (split-weight) variant.
 cudaError_t lbf_ppo_tc(const PpoTcArgs&, int grid, size_t smem, cudaStream_t);
+// plain collection with a dense first layer, one warp group per agent (rollout_lbf2.cu)
+cudaError_t lbf_ppo_tc2(const PpoTcArgs&, int grid, size_t smem, cudaStream_t);
 cudaError_t lbf_xplay_tc(const PpoTcArgs&, int grid, size_t smem, cudaStream_t);
 
 // Streamed tensor-core cross-play step (rollout_overcooked.cu, rollout_hanabi.cu).

@@ -1,0 +1,9 @@
+// rollout_lbf2.cu -- the LBF PPO collection kernel with one warp group per agent.
+#include "env_lbf.cuh"
+#include "rollout_tc2.cuh"
+
+namespace aht {
+cudaError_t lbf_ppo_tc2(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
+  return LaunchTc2<EnvLbf>::ppo(a, grid, smem, s);
+}
+}  // namespace aht

@@ -44,40 +44,22 @@ constexpr int kTcStoreWarps = 4;         // warps 9-12: one per SM sub-partition
 constexpr int kTcComputeBar = 1;         // named barrier id of the compute warps
 constexpr int kTcPairBar = 2;            // ids 2..5: warps q and q + 4 (rows 32q .. 32q + 31)
 
-// kXp: cross-play (each tile is a chunk of one pair's envs, reset at the call's first
-// step, frozen once done; the per-env return and episode length are the outputs) instead
-// of PPO collection.  kSplit: fp32 weights held as bf16 pairs W = W_hi + W_lo, L1 =
-// X W1_hi + X W1_lo and L2 = b2 + hi W2_hi + lo W2_hi + hi W2_lo (lo W2_lo is below
-// 2^-16 of the sum and left out).  kIppo (PPO collection only): seat 1 learns too, and
-// its trajectory goes to a.traj1.  kGather (PPO collection): the tile's rows are envs of
-// one teammate group found by a rank scan of the per-env pool indices (the call's draw
-// for all T steps, or, per episode, one step per launch) instead of a contiguous range.
-// kSparse (observations wider than the
-// 256 tensor-memory columns of an agent's A operand; Env::sparse_obs required): no first
-// layer on the tensor cores -- each thread forms its half of h1 = tanh(c + sum over the
-// observation's changed features of delta W1[:, f]) on CUDA cores from the fp32 W1^T and
-// c of the CUDA-core population, and writes it as the A operand of L2 directly.
-template <class Env, bool kXp, bool kSplit, bool kIppo, bool kGather, bool kSparse>
-__global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a) {
-  static_assert(!(kXp && kIppo), "seat-1 trajectories belong to PPO collection");
-  static_assert(!(kGather && (kXp || kIppo)), "gathered tiles are plain PPO collection");
-  static_assert(!(kSparse && kIppo), "the sparse first layer serves plain collection and cross-play");
-  static_assert(kTcThreads / 32 + 3 <= 16, "gather scratch: one total per warp and 3 selection words");
-  using State = typename Env::State;
-  constexpr int NA = Env::kNumActions;
-  extern __shared__ __align__(16) uint8_t smem[];  // no-swizzle operands need 16 B
-  __shared__ __align__(8) uint64_t acc_bar[4];     // [2*agent + layer], tcgen05.commit
-  __shared__ __align__(8) uint64_t opnd_bar[4];    // [2*agent + layer], 256 arrivals
-  __shared__ __align__(8) uint64_t wload_bar, drain_bar;
-  __shared__ __align__(8) uint64_t obs_full, obs_free;  // gathered observation rows: warps 9-12
-  __shared__ uint32_t tmem_slot;
-  __shared__ volatile int abort_flag;
-  __shared__ volatile int stop_flag;               // cross-play: every env of the tile is done
-
+// The tile of CTA blockIdx.x: cross-play (kXp) chunk `blockIdx.x % tpp` of pair
+// `blockIdx.x / tpp`; gathered (kGather) tile blockIdx.x of the teammate groups, its envs
+// found by a rank scan of the per-env pool indices into rowenv[0 .. count); otherwise
+// entry blockIdx.x of the contiguous tile table.  Every thread of the block calls it (it
+// synchronises the block); blockDim.x <= 24 warps.
+struct TcTile {
+  int64_t env0;   // first env (contiguous tiles)
+  int count;      // rows (0: nothing to do)
+  int ego_pol, tm_pol;
+  int g_k;        // gathered: the tile's pool index
+};
+template <bool kXp, bool kGather>
+__device__ __forceinline__ TcTile tc_find_tile(const PpoTcArgs& a, int32_t* rowenv) {
   int64_t env0;
   int count, ego_pol, tm_pol;
   int g_k = 0;                                      // gather: the tile's pool index
-  int32_t* const rowenv = kGather ? reinterpret_cast<int32_t*>(smem + a.g.scratch_off) : nullptr;
   if constexpr (kXp) {
     const int pair = blockIdx.x / a.xp.tpp, chunk = blockIdx.x - pair * a.xp.tpp;
     env0 = (int64_t)pair * a.xp.P + 128 * chunk;
@@ -89,7 +71,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     // cut into tiles of up to M in env order.  Rows are found by a rank scan of kidx:
     // each thread counts its contiguous chunk's envs of group k, an exclusive scan gives
     // the chunk's first rank, and the envs of ranks [r0, r0 + count) become rows.
-    int* wsum = reinterpret_cast<int*>(rowenv + 128);  // [0, 13) warp totals, [13, 16) selection
+    int* wsum = reinterpret_cast<int*>(rowenv + 128);  // [0, 24) warp totals, [28, 31) selection
     const int t0 = threadIdx.x, w0 = t0 >> 5, l0 = t0 & 31;
     if (blockIdx.x == 0 && a.g.resample)
       for (int k = t0; k < a.g.pool_size; k += blockDim.x) a.g.hist_zero[k] = 0;
@@ -106,14 +88,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         }
         cum += nt;
       }
-      wsum[13] = ks;
-      wsum[14] = r0;
-      wsum[15] = ks < 0 ? 0 : cnt;
+      wsum[28] = ks;
+      wsum[29] = r0;
+      wsum[30] = ks < 0 ? 0 : cnt;
     }
     __syncthreads();
-    g_k = wsum[13];
-    const int r0 = wsum[14];
-    count = wsum[15];
+    g_k = wsum[28];
+    const int r0 = wsum[29];
+    count = wsum[30];
     env0 = 0;
     ego_pol = a.ego;
     tm_pol = g_k < 0 ? 0 : a.g.pool[g_k];
@@ -186,6 +168,43 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     ego_pol = a.ego;
     tm_pol = tile.z;
   }
+  return TcTile{env0, count, ego_pol, tm_pol, g_k};
+}
+
+// kXp: cross-play (each tile is a chunk of one pair's envs, reset at the call's first
+// step, frozen once done; the per-env return and episode length are the outputs) instead
+// of PPO collection.  kSplit: fp32 weights held as bf16 pairs W = W_hi + W_lo, L1 =
+// X W1_hi + X W1_lo and L2 = b2 + hi W2_hi + lo W2_hi + hi W2_lo (lo W2_lo is below
+// 2^-16 of the sum and left out).  kIppo (PPO collection only): seat 1 learns too, and
+// its trajectory goes to a.traj1.  kGather (PPO collection): the tile's rows are envs of
+// one teammate group found by a rank scan of the per-env pool indices (the call's draw
+// for all T steps, or, per episode, one step per launch) instead of a contiguous range.
+// kSparse (observations wider than the
+// 256 tensor-memory columns of an agent's A operand; Env::sparse_obs required): no first
+// layer on the tensor cores -- each thread forms its half of h1 = tanh(c + sum over the
+// observation's changed features of delta W1[:, f]) on CUDA cores from the fp32 W1^T and
+// c of the CUDA-core population, and writes it as the A operand of L2 directly.
+template <class Env, bool kXp, bool kSplit, bool kIppo, bool kGather, bool kSparse>
+__global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a) {
+  static_assert(!(kXp && kIppo), "seat-1 trajectories belong to PPO collection");
+  static_assert(!(kGather && (kXp || kIppo)), "gathered tiles are plain PPO collection");
+  static_assert(!(kSparse && kIppo), "the sparse first layer serves plain collection and cross-play");
+  static_assert(kTcThreads / 32 <= 24, "gather scratch: one total per warp");
+  using State = typename Env::State;
+  constexpr int NA = Env::kNumActions;
+  extern __shared__ __align__(16) uint8_t smem[];  // no-swizzle operands need 16 B
+  __shared__ __align__(8) uint64_t acc_bar[4];     // [2*agent + layer], tcgen05.commit
+  __shared__ __align__(8) uint64_t opnd_bar[4];    // [2*agent + layer], 256 arrivals
+  __shared__ __align__(8) uint64_t wload_bar, drain_bar;
+  __shared__ __align__(8) uint64_t obs_full, obs_free;  // gathered observation rows: warps 9-12
+  __shared__ uint32_t tmem_slot;
+  __shared__ volatile int abort_flag;
+  __shared__ volatile int stop_flag;               // cross-play: every env of the tile is done
+
+  int32_t* const rowenv = kGather ? reinterpret_cast<int32_t*>(smem + a.g.scratch_off) : nullptr;
+  const TcTile tile = tc_find_tile<kXp, kGather>(a, rowenv);
+  const int64_t env0 = tile.env0;
+  const int count = tile.count, ego_pol = tile.ego_pol, tm_pol = tile.tm_pol, g_k = tile.g_k;
   if (count <= 0) return;
   // a negative teammate id is LBF heuristic -1 - id: no teammate network, its rule acts
   const bool tm_rule = tm_pol < 0;
@@ -505,8 +524,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       const float* p0 = zpart + ((ag * 2 + 0) * 128 + row) * 8;
       const float* p1 = zpart + ((ag * 2 + 1) * 128 + row) * 8;
       const float* b3 = reinterpret_cast<const float*>(pol_block(ag) + d.ob3);
+      // two 16-byte loads per half (a row's 8 partial sums; 8-byte-strided scalar loads
+      // would hit the same banks 8 ways)
+      const float4 a0 = *reinterpret_cast<const float4*>(p0), a1 = *reinterpret_cast<const float4*>(p0 + 4);
+      const float4 c0 = *reinterpret_cast<const float4*>(p1), c1 = *reinterpret_cast<const float4*>(p1 + 4);
+      const float pa[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+      const float pc[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
 #pragma unroll
-      for (int o = 0; o < 8; ++o) z[o] = (p0[o] + p1[o]) + b3[o];
+      for (int o = 0; o < 8; ++o) z[o] = (pa[o] + pc[o]) + b3[o];
 #pragma unroll
       for (int o = 8; o < 16; ++o) z[o] = 0.0f;
     };
