@@ -476,6 +476,20 @@ aht_status aht_sync(aht_ctx* ctx);
  * timeout bit, so the next aht_sync returns AHT_ETIMEOUT.  No fault, no hang. */
 aht_status aht_debug_expire_wait(aht_ctx* ctx, int64_t limit_ns);
 
+/* Parity hook (no paper counterpart): the policy outputs of the tensor-core kernels,
+ * element by element.  While buf (device fp32, `floats` floats, caller-owned) is set,
+ * every aht_rollout, aht_rollout_resample and aht_xplay_matrix call that runs on a
+ * tensor-core kernel also writes, for each policy evaluation it makes, the evaluated
+ * policy's output vector (its logits, then its value row if it has one, then zeros; 8
+ * entries for LBF, the padded action count for Overcooked and Hanabi) at
+ * buf[((step * rows + env) * 2 + seat) * AHT_DEBUG_STRIDE ..], rows = n_envs for
+ * collection and n_ego * n_tm * envs_per_pair for cross-play (whose frozen envs are
+ * evaluated too); entries of seats that did not act are left as they were.  A call that
+ * would write past `floats` floats returns AHT_EINVAL before it launches anything.  The
+ * CUDA-core kernels do not write it.  buf == NULL turns the hook off. */
+#define AHT_DEBUG_STRIDE 32
+aht_status aht_debug_logits(aht_ctx* ctx, float* buf, int64_t floats);
+
 const char* aht_last_error(void);
 const char* aht_status_string(aht_status s);
 

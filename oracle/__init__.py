@@ -147,7 +147,8 @@ class XplayIO(C.Structure):
                 ("n_ego", C.c_int32), ("tm_ids", _P), ("n_tm", C.c_int32),
                 ("envs_per_pair", C.c_int32), ("max_steps", C.c_int32), ("forced", _P),
                 ("env_ids", _P), ("n_sel", C.c_int64), ("n_threads", C.c_int32), ("returns", _P), ("steps", _P), ("actions", _P),
-                ("own_actions", _P), ("margin", _P), ("matrix", _P)]
+                ("own_actions", _P), ("margin", _P), ("matrix", _P), ("logits", _P),
+                ("logit_stride", C.c_int32)]
 
 
 def lib() -> C.CDLL:
@@ -370,8 +371,10 @@ def rollout(d, pols: Policies, seed, states, step0, T, ego_id, pool, forced=None
 
 
 def xplay(d, pols: Policies, seed, step0, ego_ids, tm_ids, P, max_steps, forced=None,
-          n_threads=1, record=True, env_ids=None):
-    """Cross-play.  env_ids: run only these global env indices (rows of the outputs)."""
+          n_threads=1, record=True, env_ids=None, logit_stride=0):
+    """Cross-play.  env_ids: run only these global env indices (rows of the outputs).
+    logit_stride > 0: also the acting seats' policy outputs, [max_steps][rows][2][stride]
+    (NaN where a seat did not act)."""
     ego_ids = np.ascontiguousarray(ego_ids, np.int32)
     tm_ids = np.ascontiguousarray(tm_ids, np.int32)
     N = len(ego_ids) * len(tm_ids) * P
@@ -384,13 +387,15 @@ def xplay(d, pols: Policies, seed, step0, ego_ids, tm_ids, P, max_steps, forced=
         out.update(actions=np.zeros((max_steps, N, 2), np.uint8),
                    own_actions=np.zeros((max_steps, N, 2), np.uint8),
                    margin=np.zeros((max_steps, N, 2), np.float64))
+    if logit_stride:
+        out["logits"] = np.full((max_steps, N, 2, logit_stride), np.nan)
     if forced is not None:
         forced = np.ascontiguousarray(forced, np.uint8)
     io = XplayIO(seed=seed, step0=step0, ego_ids=_ptr(ego_ids), n_ego=len(ego_ids),
                  tm_ids=_ptr(tm_ids), n_tm=len(tm_ids), envs_per_pair=P, max_steps=max_steps,
                  forced=_ptr(forced), env_ids=_ptr(env_ids),
                  n_sel=0 if env_ids is None else len(env_ids), n_threads=n_threads,
-                 **{k: _ptr(v) for k, v in out.items()})
+                 logit_stride=logit_stride, **{k: _ptr(v) for k, v in out.items()})
     rc = lib().orc_xplay(C.byref(d), pols.arr, pols.n, C.byref(io))
     out["rc"] = rc
     return out

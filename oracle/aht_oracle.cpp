@@ -1379,6 +1379,9 @@ extern "C" int32_t orc_xplay(const orc_env_desc* d, const orc_mlp* pols, int32_t
         env_obs(d, &st, seat, o.data());
         env_legal(d, &st, legal.data());
         orc_mlp_forward(pol[seat], obs_to_double(o.data(), od).data(), z.data());
+        if (io->logits)
+          for (int k = 0; k < pol[seat]->n_out && k < io->logit_stride; ++k)
+            io->logits[(i * 2 + seat) * io->logit_stride + k] = z[k];
         int own;
         double lp, mg;
         orc_sample(z.data(), legal.data(), K,

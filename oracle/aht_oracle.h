@@ -288,6 +288,9 @@ typedef struct orc_xplay_io {
   uint8_t* own_actions;    /* [max_steps][n_envs][2] */
   double* margin;          /* [max_steps][n_envs][2] (2 = no sample) */
   float* matrix;           /* [n_ego][n_tm] mean return, fp64 sum (all envs only) */
+  double* logits;          /* [max_steps][n_envs][2][logit_stride]: the acting seats'
+                              policy outputs (untouched where a seat did not act) */
+  int32_t logit_stride;
 } orc_xplay_io;
 int32_t orc_xplay(const orc_env_desc* d, const orc_mlp* pols, int32_t n_pols,
                   orc_xplay_io* io);

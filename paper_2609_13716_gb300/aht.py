@@ -141,6 +141,8 @@ def load() -> C.CDLL:
             L.aht_set_policy.argtypes = [vp, i32, C.POINTER(vp), C.POINTER(vp), i32, i32]
             L.aht_set_timing.argtypes = [vp, i32]
             L.aht_get_timing.argtypes = [vp, C.POINTER(C.c_double), C.POINTER(i64)]
+            L.aht_debug_logits.argtypes = [vp, vp, i64]
+            L.aht_debug_logits.restype = C.c_int
             L.aht_step_counter.argtypes = [vp]
             L.aht_step_counter.restype = i64
             L.aht_sync.argtypes = [vp]
@@ -413,6 +415,19 @@ def aht_step_counter(ctx: Context) -> int:
 
 def aht_sync(ctx: Context):
     _check(load().aht_sync(ctx.handle))
+
+
+AHT_DEBUG_STRIDE = 32
+
+
+def aht_debug_logits(ctx: Context, buf):
+    """Parity hook: while ``buf`` (a contiguous CUDA fp32 tensor) is set, the tensor-core
+    kernels of the next calls write every policy output vector into it, at
+    [step][row][seat][AHT_DEBUG_STRIDE]; ``None`` turns it off."""
+    if buf is None:
+        _check(load().aht_debug_logits(ctx.handle, None, 0))
+        return
+    _check(load().aht_debug_logits(ctx.handle, _ptr(buf, torch.float32, name="buf"), buf.numel()))
 
 
 def aht_debug_expire_wait(ctx: Context, limit_ns: int):

@@ -109,6 +109,9 @@ struct aht_ctx {
   uint8_t* rs_kidx = nullptr;   // [2][align_up(n_envs, 16)] per-episode pool index by step parity
   int32_t* rs_hist = nullptr;   // [3][kMaxPool] envs per pool index, by step mod 3
   uint32_t* status = nullptr;
+  // test hook (aht_debug_logits): caller-owned output buffer of the tensor-core kernels
+  float* dbg_logits = nullptr;
+  int64_t dbg_floats = 0;
   // tensor-core path (bf16 LBF populations that fit shared and tensor memory)
   int32_t weight_dtype = AHT_BF16;
   bool tc = false;
@@ -487,6 +490,19 @@ void timer_end(aht_ctx* c, int i) {
   if (i >= 0) cudaEventRecord(c->ev[2 * i + 1], c->stream);
 }
 
+// The test hook's buffer for a call of `steps` steps over `rows` rows: NULL when unset;
+// false (and the error set) when it is too small.
+bool dbg_buffer(aht_ctx* c, int64_t steps, int64_t rows, float** out) {
+  *out = nullptr;
+  if (!c->dbg_logits) return true;
+  if (steps * rows * 2 * kDbgStride > c->dbg_floats) {
+    fail(AHT_EINVAL, "the aht_debug_logits buffer is too small for this call");
+    return false;
+  }
+  *out = c->dbg_logits;
+  return true;
+}
+
 // Cross-play on the streamed tensor-core kernel: max_steps + 1 launches, one per step
 // (the last applies the final transition), then the exact pair means.
 aht_status xplay_wide(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego, const int32_t* tm_ids,
@@ -507,6 +523,7 @@ aht_status xplay_wide(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego, const i
   a.returns = out->returns ? out->returns : c->xp_returns;
   a.steps = out->steps;
   a.actions = out->actions;
+  if (!dbg_buffer(c, max_steps, a.n_total, &a.dbg_logits)) return AHT_EINVAL;
   const int64_t T0 = ((int64_t)n_tm * P + 127) / 128, T1 = ((int64_t)n_ego * P + 127) / 128;
   const int64_t tiles0 = n_ego * T0, tiles1 = n_tm * T1;
   if (tiles0 + tiles1 > INT32_MAX) return fail(AHT_EINVAL, "too many tiles");
@@ -555,6 +572,7 @@ aht_status xplay_lbf_tc(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego, const
   ta.xp.returns = returns;
   ta.xp.steps = steps;
   ta.xp.actions = actions;
+  if (!dbg_buffer(c, max_steps, ta.xp.n_total, &ta.dbg_logits)) return AHT_EINVAL;
   const int64_t n_pairs = (int64_t)n_ego * n_tm;
   const int64_t grid = n_pairs * ta.xp.tpp;
   if (grid > INT32_MAX) return fail(AHT_EINVAL, "too many tiles");
@@ -863,6 +881,8 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
   }
   const size_t tc_smem = c->tc_smem + (grouped ? kTcGatherScratch : 0);
   if (use_tc && tc_smem > c->smem_optin) return fail(AHT_EINVAL, "no shared memory left for the teammate grouping");
+  float* dbg = nullptr;
+  if (use_tc && !dbg_buffer(c, T, Nall, &dbg)) return AHT_EINVAL;
   const int grid = (int)n_tiles(M);
 
   GroupArgs ga{};
@@ -932,6 +952,7 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
     ta.traj = a.traj;
     ta.traj1 = a.traj1;
     ta.ep_step = c->ep_step;
+    ta.dbg_logits = dbg;
     if (grouped) {
       ta.gather = 1;
       ta.g.kidx_cur = c->rs_kidx;
@@ -997,6 +1018,8 @@ aht_status aht_rollout_resample(aht_ctx* c, int32_t ego_id, const int32_t* pool,
     // Tensor-core path: each step's launch groups its own rows (TcGather).
     const size_t smem = c->tc_smem + kTcGatherScratch;
     if (smem > c->smem_optin) return fail(AHT_EINVAL, "no shared memory left for the per-episode grouping");
+    float* dbg = nullptr;
+    if (!dbg_buffer(c, T, N, &dbg)) return AHT_EINVAL;
     const size_t ks = (size_t)align_up(N, 16);
     AHT_CUDA(cudaMemsetAsync(c->rs_hist, 0, 3 * (size_t)kMaxPool * 4, c->stream));
     AHT_CUDA(launch_resample_init(batch_of(c).key, N, c->ep_step, pool_size, c->rs_kidx, c->rs_hist,
@@ -1030,6 +1053,7 @@ aht_status aht_rollout_resample(aht_ctx* c, int32_t ego_id, const int32_t* pool,
       ta.g.hist_zero = c->rs_hist + ((t + 2) % 3) * kMaxPool;
       ta.g.teammate = teammates ? teammates + o : nullptr;
       ta.g.teammate2 = t == 0 ? out->teammate : nullptr;
+      ta.dbg_logits = dbg ? dbg + o * 2 * kDbgStride : nullptr;  // this step's slice
       const int tk = timer_begin(c);
       AHT_CUDA(lbf_ppo_tc(ta, resample_tiles(N, 128, pool_size), smem, c->stream));
       timer_end(c, tk);
@@ -1407,6 +1431,14 @@ aht_status aht_sync(aht_ctx* c) {
                             " (1 illegal action, 2 actor mismatch, 4 bad policy, 8 a bounded wait expired)";
     return fail(s == kStatusTimeout ? AHT_ETIMEOUT : AHT_EDEVICE, msg);
   }
+  return AHT_OK;
+}
+
+aht_status aht_debug_logits(aht_ctx* c, float* buf, int64_t floats) {
+  if (!c) return fail(AHT_EINVAL, "ctx is NULL");
+  if (buf && floats < 1) return fail(AHT_EINVAL, "floats must be >= 1");
+  c->dbg_logits = buf;
+  c->dbg_floats = buf ? floats : 0;
   return AHT_OK;
 }
 

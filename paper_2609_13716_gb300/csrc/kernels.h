@@ -120,6 +120,7 @@ struct PpoTcArgs {
   TrajPtrs traj1;        // as in PpoArgs
   TcXp xp;               // cross-play launches only
   TcGather g;            // gather launches only
+  float* dbg_logits;     // test hook, or NULL: [steps][rows][2 seats][kDbgStride] outputs
 };
 
 // Per-policy block of the streamed tensor-core path (binary observations, hidden width H
@@ -162,7 +163,13 @@ struct XpTcArgs {
   float* returns;          // [n_total]
   int32_t* steps;          // optional [n_total]
   uint8_t* actions;        // optional [max_steps][n_total][2]
+  float* dbg_logits;       // test hook, or NULL: [max_steps][n_total][2 seats][kDbgStride]
 };
+
+// Test hook layout: every policy evaluation of a tensor-core kernel may write its output
+// vector (logits, then the value where the policy has one, then zeros) at
+// [step][row][seat][0 .. kDbgStride).
+constexpr int kDbgStride = 32;
 
 // Teammate assignment of one collection call (per-call draw, counter (e, step0, stream 3)).
 struct GroupArgs {

@@ -644,6 +644,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       } else if (row < count) {
         const int ag = half == 0 ? 0 : 1;
         logits(ag, z);
+        if (a.dbg_logits) {  // test hook: this row's outputs of step t (frozen rows too)
+          const int64_t rows = kXp ? a.xp.n_total : N;
+          float* p = a.dbg_logits + (((int64_t)t * rows + my_env) * 2 + ag) * kDbgStride;
+#pragma unroll
+          for (int o = 0; o < 8; ++o) p[o] = z[o];
+        }
         float lp;
         const int act = sample_k<NA>(z, 0xFFFFFFFFu >> (32 - NA), u_act, lp);
         if (ag == 1) {

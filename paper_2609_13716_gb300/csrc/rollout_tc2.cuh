@@ -257,6 +257,13 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
 #pragma unroll
       for (int o = 8; o < 16; ++o) z[o] = 0.0f;
     };
+    // test hook: this row's outputs of step t
+    auto dbg_store = [&](int t, const float (&z)[16]) {
+      if (!a.dbg_logits) return;
+      float* p = a.dbg_logits + (((int64_t)t * N + my_env) * 2 + ag) * kDbgStride;
+#pragma unroll
+      for (int o = 0; o < 8; ++o) p[o] = z[o];
+    };
     // contiguous tiles: the ego's rows -> trajectory [t][env0 .. env0 + count) as one
     // contiguous block, by one bulk (TMA) store when 16-byte aligned, else by the group
     const bool bulk_obs = !kGather && a.traj.obs && (count * od) % 16 == 0;
@@ -331,6 +338,7 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
             act1s[row] = (uint8_t)Env::heuristic(a.b.env, s, -1 - tm_pol);
           } else {
             logits(z);
+            dbg_store(t, z);
             float lp;
             act1s[row] = (uint8_t)sample_k<NA>(z, 0xFFFFFFFFu >> (32 - NA), u_act, lp);
           }
@@ -363,6 +371,7 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
           }
         } else if (sampler) {
           logits(z);
+          dbg_store(t, z);
           act0 = sample_k<NA>(z, 0xFFFFFFFFu >> (32 - NA), u_act, lp0);
           val0 = z[NA];
         }

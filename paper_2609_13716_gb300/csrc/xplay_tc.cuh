@@ -547,6 +547,11 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
 #pragma unroll
       for (int o = 0; o < NAP; ++o)
         z[o] = (zpart[row * NAP + o] + zpart[(128 + row) * NAP + o]) + b3[o];
+      if (a.dbg_logits) {  // test hook: this row's outputs of step s
+        float* p = a.dbg_logits + (((int64_t)a.s * a.n_total + e) * 2 + seat) * kDbgStride;
+#pragma unroll
+        for (int o = 0; o < NAP; ++o) p[o] = z[o];
+      }
       float lp;
       const int act = sample_k<NA>(z, legal, u_act, lp);
       a.act_out[2 * e + seat] = (uint8_t)act;

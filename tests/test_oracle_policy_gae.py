@@ -1,4 +1,6 @@
 """Pins for the oracle's policy forward, masked categorical sampling, GAE and drivers."""
+import ctypes as C
+
 import numpy as np
 import pytest
 import torch
@@ -191,3 +193,45 @@ def test_xplay_matrix_is_pair_mean(orc):
         live = acts[s, :, 0] != 255
         assert (acts[s, :, 1 - s % 2] == 255).all()
         assert ((acts[s, :, s % 2] != 255) == (out["steps"] > s)).all()
+
+
+def test_xplay_logits_output_is_what_the_sampler_used(orc):
+    """The cross-play logits output (a parity-test record) is the forward the oracle
+    sampled from: re-sampling it with the same draw gives the recorded own action, and an
+    independent torch fp64 forward of the seat-0 reset observation gives the same values."""
+    wl = W.WORKLOADS["hanabi_xplay_16x16x32"]
+    d = orc.env_desc(*wl.env.astuple())
+    layers = W.population(wl)[:4]
+    pols = orc.Policies(layers)
+    out = orc.xplay(d, pols, 4, 0, [0, 1], [2, 3], 3, 100, n_threads=4, logit_stride=32)
+    assert out["rc"] == 0
+    L, own = out["logits"], out["own_actions"]
+    n = 0
+    for s in range(6):
+        for e in range(12):
+            seat = s % 2
+            if own[s, e, seat] == 255:
+                assert np.isnan(L[s, e, seat]).all()
+                continue
+            assert np.isnan(L[s, e, 1 - seat]).all()      # only the acting seat runs
+            z = L[s, e, seat, :20]
+            assert np.isnan(L[s, e, seat, 20:]).all()
+            u = (int(orc.draw(4, e, s, seat, 0)) >> 8) * 2.0 ** -24
+            if s == 0:
+                st = orc.reset_envs(d, 4, [e])
+                legal = np.zeros(20, np.uint8)
+                hs = orc.HanabiState.from_buffer(st)
+                orc.lib().orc_hanabi_legal(C.byref(hs), legal.ctypes.data_as(C.c_void_p))
+                o = np.zeros(660, np.uint8)
+                orc.lib().orc_hanabi_obs(C.byref(hs), 0, o.ctypes.data_as(C.c_void_p))
+                pid = [0, 1][e // 6]
+                x = torch.from_numpy(o.astype(np.float64))
+                for k, (Wt, b) in enumerate(layers[pid]):
+                    x = torch.from_numpy(np.asarray(Wt, np.float64)) @ x + torch.from_numpy(np.asarray(b, np.float64))
+                    if k < 2:
+                        x = torch.tanh(x)
+                assert np.allclose(z, x.numpy(), rtol=1e-12, atol=1e-12)
+                a, _, _ = orc.sample(z, legal, u)
+                assert a == own[s, e, seat]
+                n += 1
+    assert n == 12

@@ -7,7 +7,9 @@ without more device memory.  The static variant keeps that scratch in one file-s
 device array of the library instead.  Here it runs on a context of capacity 16 and must
 reproduce, on two calls in a row, the matrices that aht_xplay_matrix computes on a
 context sized for the whole batch (both contexts start from the same seed and step, so
-their draws coincide).  This file is collected last on purpose.
+their draws coincide).  On bf16 Overcooked and Hanabi contexts, whose static matrix runs
+the CUDA-core kernel, each pair without a close call at a sampling-CDF edge must have the
+fp64 oracle's cell exactly.  This file is collected last on purpose.
 """
 import pytest
 import torch
@@ -52,3 +54,36 @@ def test_static_scratch_rejects_batches_above_its_size():
         aht.aht_xplay_matrix_static(ctx, ids, ids, 32, 100, m)
     assert e.value.status == aht.AHT_EINVAL
     assert aht.aht_step_counter(ctx) == 0
+
+
+@pytest.mark.parametrize("name,ego,tm,P,S", [
+    ("overcooked5x4_xplay_8x8x64", [0, 1, 2, 3], [8, 9, 10, 11], 2, 400),
+    ("hanabi_xplay_16x16x32", [0, 5, 9], [16, 30], 40, 100),
+])
+def test_static_scratch_matrix_on_bf16_overcooked_and_hanabi(name, ego, tm, P, S):
+    """bf16 Overcooked and Hanabi contexts: the static variant runs the CUDA-core
+    cross-play kernel.  The oracle plays the same episodes free-running in fp64; an env
+    whose every sample lies at least 1e-5 from a CDF edge plays the oracle's episode
+    exactly, so each pair with no such close call has exactly the oracle's cell, on two
+    calls in a row (the second from the advanced step counter)."""
+    import numpy as np
+    import oracle as O
+    from gpu_util import CDF_MARGIN, oracle_of
+    require_gpu()
+    wl = W.WORKLOADS[name]
+    ctx, pop_np = make_ctx(wl, 16)
+    d, pols = oracle_of(wl.env, pop_np)
+    checked = 0
+    for call in range(2):
+        got = torch.full((len(ego), len(tm)), float("nan"), device="cuda")
+        aht.aht_xplay_matrix_static(ctx, ego, tm, P, S, got)
+        aht.aht_sync(ctx)
+        ref = O.xplay(d, pols, wl.env_seed, call * S, ego, tm, P, S, n_threads=8)
+        assert ref["rc"] == 0
+        close_call = (ref["margin"] < CDF_MARGIN).any(axis=(0, 2)).reshape(len(ego), len(tm), P).any(-1)
+        g = got.cpu().numpy()
+        assert np.isfinite(g).all()
+        assert np.array_equal(g[~close_call], ref["matrix"][~close_call]), call
+        checked += int((~close_call).sum())
+        assert aht.aht_step_counter(ctx) == (call + 1) * S
+    assert checked >= len(ego) * len(tm)   # most pairs have no close call
