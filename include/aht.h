@@ -476,6 +476,20 @@ aht_status aht_sync(aht_ctx* ctx);
  * timeout bit, so the next aht_sync returns AHT_ETIMEOUT.  No fault, no hang. */
 aht_status aht_debug_expire_wait(aht_ctx* ctx, int64_t limit_ns);
 
+/* Failure-detection hook for the real kernels (no paper counterpart).  The next call of
+ * aht_rollout, aht_rollout_resample, aht_rollout_ippo or aht_xplay_matrix that runs on a
+ * tensor-core kernel makes its compute threads, at the call's step `step` (cross-play
+ * on the streamed Overcooked / Hanabi kernel: at its launch for step `step`), wait on an
+ * mbarrier nothing arrives on, in place of an accumulator wait, with the kernels' bounded
+ * wait limited to limit_ns (1 .. 10^9).  The wait expires and the kernel takes its abort
+ * path: it latches the timeout bit, stops, waits (bounded) for the MMAs and copies it has
+ * in flight, frees its tensor memory and exits; its env state is not stored (the context
+ * keeps the state from before the call; the step counter still advances by the call's
+ * length) and cross-play cells of aborted tiles are NaN (LBF) or hold the returns
+ * reached so far (the streamed kernel stops those envs).  The next aht_sync returns
+ * AHT_ETIMEOUT.  The hook fires once; step < 0 clears it.  No fault, no hang. */
+aht_status aht_debug_expire_at(aht_ctx* ctx, int32_t step, int64_t limit_ns);
+
 /* Parity hook (no paper counterpart): the policy outputs of the tensor-core kernels,
  * element by element.  While buf (device fp32, `floats` floats, caller-owned) is set,
  * every aht_rollout, aht_rollout_resample and aht_xplay_matrix call that runs on a

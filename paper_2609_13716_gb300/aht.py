@@ -141,6 +141,8 @@ def load() -> C.CDLL:
             L.aht_set_policy.argtypes = [vp, i32, C.POINTER(vp), C.POINTER(vp), i32, i32]
             L.aht_set_timing.argtypes = [vp, i32]
             L.aht_get_timing.argtypes = [vp, C.POINTER(C.c_double), C.POINTER(i64)]
+            L.aht_debug_expire_at.argtypes = [vp, i32, i64]
+            L.aht_debug_expire_at.restype = C.c_int
             L.aht_debug_logits.argtypes = [vp, vp, i64]
             L.aht_debug_logits.restype = C.c_int
             L.aht_step_counter.argtypes = [vp]
@@ -418,6 +420,12 @@ def aht_sync(ctx: Context):
 
 
 AHT_DEBUG_STRIDE = 32
+
+
+def aht_debug_expire_at(ctx: Context, step: int, limit_ns: int):
+    """Failure-detection hook: the next tensor-core call waits in vain (bounded by
+    limit_ns) at its step ``step`` and aborts; ``step < 0`` clears the hook."""
+    _check(load().aht_debug_expire_at(ctx.handle, step, limit_ns))
 
 
 def aht_debug_logits(ctx: Context, buf):

@@ -112,6 +112,9 @@ struct aht_ctx {
   // test hook (aht_debug_logits): caller-owned output buffer of the tensor-core kernels
   float* dbg_logits = nullptr;
   int64_t dbg_floats = 0;
+  // failure-detection hook (aht_debug_expire_at): one tensor-core call waits in vain
+  int32_t dbg_expire_step = -1;
+  uint64_t dbg_expire_ns = 0;
   // tensor-core path (bf16 LBF populations that fit shared and tensor memory)
   int32_t weight_dtype = AHT_BF16;
   bool tc = false;
@@ -490,6 +493,13 @@ void timer_end(aht_ctx* c, int i) {
   if (i >= 0) cudaEventRecord(c->ev[2 * i + 1], c->stream);
 }
 
+// The failure-detection hook for the tensor-core call about to launch (it fires once).
+void take_expire(aht_ctx* c, int32_t* step, uint64_t* ns) {
+  *step = c->dbg_expire_step;
+  *ns = c->dbg_expire_ns;
+  c->dbg_expire_step = -1;
+}
+
 // The test hook's buffer for a call of `steps` steps over `rows` rows: NULL when unset;
 // false (and the error set) when it is too small.
 bool dbg_buffer(aht_ctx* c, int64_t steps, int64_t rows, float** out) {
@@ -525,6 +535,7 @@ aht_status xplay_wide(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego, const i
   a.actions = out->actions;
   if (!dbg_buffer(c, max_steps, a.n_total, &a.dbg_logits)) return AHT_EINVAL;
   const int64_t T0 = ((int64_t)n_tm * P + 127) / 128, T1 = ((int64_t)n_ego * P + 127) / 128;
+  take_expire(c, &a.dbg_expire_step, &a.dbg_expire_ns);
   const int64_t tiles0 = n_ego * T0, tiles1 = n_tm * T1;
   if (tiles0 + tiles1 > INT32_MAX) return fail(AHT_EINVAL, "too many tiles");
   const bool turn = c->env.kind == AHT_HANABI || c->env.kind == AHT_MINI_HANABI;
@@ -576,6 +587,7 @@ aht_status xplay_lbf_tc(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego, const
   const int64_t n_pairs = (int64_t)n_ego * n_tm;
   const int64_t grid = n_pairs * ta.xp.tpp;
   if (grid > INT32_MAX) return fail(AHT_EINVAL, "too many tiles");
+  take_expire(c, &ta.dbg_expire_step, &ta.dbg_expire_ns);
   const int tk = timer_begin(c);
   AHT_CUDA(lbf_xplay_tc(ta, (int)grid, c->tc_smem, c->stream));
   timer_end(c, tk);
@@ -953,6 +965,7 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
     ta.traj1 = a.traj1;
     ta.ep_step = c->ep_step;
     ta.dbg_logits = dbg;
+    take_expire(c, &ta.dbg_expire_step, &ta.dbg_expire_ns);
     if (grouped) {
       ta.gather = 1;
       ta.g.kidx_cur = c->rs_kidx;
@@ -1020,6 +1033,9 @@ aht_status aht_rollout_resample(aht_ctx* c, int32_t ego_id, const int32_t* pool,
     if (smem > c->smem_optin) return fail(AHT_EINVAL, "no shared memory left for the per-episode grouping");
     float* dbg = nullptr;
     if (!dbg_buffer(c, T, N, &dbg)) return AHT_EINVAL;
+    int32_t expire_step;
+    uint64_t expire_ns;
+    take_expire(c, &expire_step, &expire_ns);
     const size_t ks = (size_t)align_up(N, 16);
     AHT_CUDA(cudaMemsetAsync(c->rs_hist, 0, 3 * (size_t)kMaxPool * 4, c->stream));
     AHT_CUDA(launch_resample_init(batch_of(c).key, N, c->ep_step, pool_size, c->rs_kidx, c->rs_hist,
@@ -1054,6 +1070,8 @@ aht_status aht_rollout_resample(aht_ctx* c, int32_t ego_id, const int32_t* pool,
       ta.g.teammate = teammates ? teammates + o : nullptr;
       ta.g.teammate2 = t == 0 ? out->teammate : nullptr;
       ta.dbg_logits = dbg ? dbg + o * 2 * kDbgStride : nullptr;  // this step's slice
+      ta.dbg_expire_step = t == expire_step ? 0 : -1;             // this launch's step 0
+      ta.dbg_expire_ns = expire_ns;
       const int tk = timer_begin(c);
       AHT_CUDA(lbf_ppo_tc(ta, resample_tiles(N, 128, pool_size), smem, c->stream));
       timer_end(c, tk);
@@ -1439,6 +1457,14 @@ aht_status aht_debug_logits(aht_ctx* c, float* buf, int64_t floats) {
   if (buf && floats < 1) return fail(AHT_EINVAL, "floats must be >= 1");
   c->dbg_logits = buf;
   c->dbg_floats = buf ? floats : 0;
+  return AHT_OK;
+}
+
+aht_status aht_debug_expire_at(aht_ctx* c, int32_t step, int64_t limit_ns) {
+  if (!c) return fail(AHT_EINVAL, "ctx is NULL");
+  if (step >= 0 && (limit_ns < 1 || limit_ns > 1000000000)) return fail(AHT_EINVAL, "limit_ns must be in 1..1e9");
+  c->dbg_expire_step = step < 0 ? -1 : step;
+  c->dbg_expire_ns = (uint64_t)limit_ns;
   return AHT_OK;
 }
 

@@ -121,6 +121,8 @@ struct PpoTcArgs {
   TcXp xp;               // cross-play launches only
   TcGather g;            // gather launches only
   float* dbg_logits;     // test hook, or NULL: [steps][rows][2 seats][kDbgStride] outputs
+  int32_t dbg_expire_step;   // test hook: at this step the compute threads wait, bounded by
+  uint64_t dbg_expire_ns;    // dbg_expire_ns, on an mbarrier nothing arrives on (-1: never)
 };
 
 // Per-policy block of the streamed tensor-core path (binary observations, hidden width H
@@ -164,6 +166,8 @@ struct XpTcArgs {
   int32_t* steps;          // optional [n_total]
   uint8_t* actions;        // optional [max_steps][n_total][2]
   float* dbg_logits;       // test hook, or NULL: [max_steps][n_total][2 seats][kDbgStride]
+  int32_t dbg_expire_step; // test hook: launch s == this waits on an mbarrier nothing
+  uint64_t dbg_expire_ns;  // arrives on, bounded by dbg_expire_ns (-1: never)
 };
 
 // Test hook layout: every policy evaluation of a tensor-core kernel may write its output

@@ -197,6 +197,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   __shared__ __align__(8) uint64_t opnd_bar[4];    // [2*agent + layer], 256 arrivals
   __shared__ __align__(8) uint64_t wload_bar, drain_bar;
   __shared__ __align__(8) uint64_t obs_full, obs_free;  // gathered observation rows: warps 9-12
+  __shared__ __align__(8) uint64_t never_bar;           // test hook: nothing arrives on it
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
   __shared__ volatile int stop_flag;               // cross-play: every env of the tile is done
@@ -245,6 +246,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     tc::mbar_init(&drain_bar, 1);
     tc::mbar_init(&obs_full, kTcCompute);
     tc::mbar_init(&obs_free, kTcStoreWarps);
+    tc::mbar_init(&never_bar, 1);
     tc::mbar_init_fence();
     abort_flag = 0;
     stop_flag = 0;
@@ -608,6 +610,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
           }
           tc::bar_sync(kTcPairBar + q, 64);
         }
+      }
+      if (t == a.dbg_expire_step) {  // test hook: an accumulator wait that never completes
+        if (!bad && !tc::mbar_wait(&never_bar, 0, a.dbg_expire_ns)) bad = true;
+        bad = __any_sync(0xFFFFFFFFu, bad);
       }
 #pragma unroll 1
       for (int i = first; i >= 0 && !kSparse; --i) {

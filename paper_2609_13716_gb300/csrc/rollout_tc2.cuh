@@ -41,6 +41,7 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
   __shared__ __align__(8) uint64_t wload_bar[2], drain_bar[2];  // per agent
   __shared__ __align__(8) uint64_t buf_free;       // teammate rows in tensor memory (256)
   __shared__ __align__(8) uint64_t rows_ready;     // ego rows built (256; gathered copy)
+  __shared__ __align__(8) uint64_t never_bar;      // test hook: nothing arrives on it
   __shared__ uint32_t tmem_slot;
 
   int32_t* const rowenv = kGather ? reinterpret_cast<int32_t*>(smem + a.g.scratch_off) : nullptr;
@@ -80,6 +81,7 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
     }
     tc::mbar_init(&buf_free, kT2Group);
     tc::mbar_init(&rows_ready, kT2Group);
+    tc::mbar_init(&never_bar, 1);
     tc::mbar_init_fence();
   }
   if (warp == 0) tc::tmem_alloc(&tmem_slot, 512);
@@ -357,6 +359,10 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
         if (!boot && a.traj.obs) {
           if constexpr (kGather) tc::mbar_arrive(&rows_ready);
           else copy_rows_contiguous(t);
+        }
+        if (t == a.dbg_expire_step) {  // test hook: an accumulator wait that never completes
+          if (!bad && !tc::mbar_wait(&never_bar, 0, a.dbg_expire_ns)) bad = true;
+          bad = __any_sync(0xFFFFFFFFu, bad);
         }
         wait_acc(0, par);
         if (!bad) epilogue1();

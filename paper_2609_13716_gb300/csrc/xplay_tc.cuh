@@ -112,6 +112,7 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
   extern __shared__ __align__(16) uint8_t smem[];  // the no-swizzle operands need 16 B
   __shared__ __align__(8) uint64_t full_bar[kXpMaxStages], empty_bar[kXpMaxStages];
   __shared__ __align__(8) uint64_t obs_bar, acc_bar[3], epi1_bar, epi2_bar, w3_bar, drain_bar;
+  __shared__ __align__(8) uint64_t never_bar;  // test hook: nothing arrives on it
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
   bool w3_issued = false;  // (MMA lane) the W3 copy is in flight or done
@@ -166,6 +167,7 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
     tc::mbar_init(&epi2_bar, kXpCompute);
     tc::mbar_init(&w3_bar, 1);
     tc::mbar_init(&drain_bar, 1);
+    tc::mbar_init(&never_bar, 1);
     tc::mbar_init_fence();
     abort_flag = 0;
   }
@@ -411,6 +413,10 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
     }
 
     // 4. epilogue 1
+    if (a.s == a.dbg_expire_step) {  // test hook: an accumulator wait that never completes
+      if (!bad && !tc::mbar_wait(&never_bar, 0, a.dbg_expire_ns)) bad = true;
+      bad = __any_sync(0xFFFFFFFFu, bad);
+    }
     wait_acc(&acc_bar[0]);
     if (!bad && w.H == 256) {
       for (int c0 = 128 * half; c0 < 128 * half + 128; c0 += 32) {
@@ -556,6 +562,9 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
       const int act = sample_k<NA>(z, legal, u_act, lp);
       a.act_out[2 * e + seat] = (uint8_t)act;
     }
+    // a tile that gave up wrote no action: its envs stop here, so that no later step of
+    // the call applies a stale one (their returns stay those of the state before)
+    if (bad && tid < 128 && e >= 0 && owner) a.alive_out[e] = 0;
     if (bad) abort_flag = 1;
   }
 
