@@ -104,6 +104,32 @@ def oracle_rate(wl, target_s, seed_offset=0):
     return n * wl.T / dt, threads, sample, dt
 
 
+def oracle_rate_1thread(wl, target_s):
+    """The oracle's free-running PPO collection (rollout + GAE) on one host thread, on a
+    bounded env sample sized for about target_s seconds.  Returns (env-steps/s, sample)."""
+    import numpy as np
+    import oracle as O
+    from paper_2609_13716_gb300 import workloads as W
+    d = O.env_desc(*wl.env.astuple())
+    pols = O.Policies(W.population(wl))
+    n = 4
+    for _ in range(2):  # the first pilot also pays one-time costs
+        t0 = time.perf_counter()
+        O.rollout(d, pols, wl.env_seed, O.reset_all(d, wl.env_seed, n), 0, wl.T, wl.ego_id,
+                  list(wl.pool), n_threads=1)
+        rate = n * wl.T / (time.perf_counter() - t0)
+    n = int(min(wl.n_envs, max(4, rate * target_s / wl.T)))
+    ids = np.arange(n, dtype=np.int64) * (wl.n_envs // n)
+    st = O.reset_envs(d, wl.env_seed, ids)
+    t0 = time.perf_counter()
+    out = O.rollout(d, pols, wl.env_seed, st, 0, wl.T, wl.ego_id, list(wl.pool), n_threads=1,
+                    env_ids=ids)
+    O.gae(out["rewards"], out["values"].astype(np.float32), out["dones"],
+          out["last_value"].astype(np.float32), wl.gamma, wl.lam)
+    dt = time.perf_counter() - t0
+    return n * wl.T / dt, f"{n} of {wl.n_envs} envs x {wl.T} steps (rollout + GAE) on 1 thread"
+
+
 def run_reference(args):
     rank, _, world = dist_env()
     if rank != 0:
@@ -402,8 +428,9 @@ def run_ours(args):
             line["xplay"] = xp
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         v, cores, sample, _ = oracle_rate(wl, args.cpu_seconds)
+        v1, sample1 = oracle_rate_1thread(wl, min(4.0, args.cpu_seconds / 3))
         line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
-                                "sample": sample}
+                                "sample": sample, "value_1_thread": v1, "sample_1_thread": sample1}
     if line is not None:
         print(json.dumps(line), flush=True)
     ctx.close()

@@ -11,8 +11,9 @@
  *   - PPO rollout collection with GAE targets (App. C, "PPO ego");
  *   - the ego-by-teammate cross-play (XP) return matrix (App. B, "Cross-play matrix
  *     construction"); its row mean over held-out teammates is J_AHT of Sec. 3.
- * The paper does not state the game rules; the rules implemented are the readings
- * listed in the design doc.
+ * The paper does not state the game rules; the library implements readings of the
+ * workload descriptions, stated rule by rule in the env sources (csrc/env_*.cuh) and in
+ * the test oracle's header.
  *
  * Conventions (all entry points):
  *   - Bulk tensors are DEVICE pointers owned by the caller, laid out as documented,
@@ -475,6 +476,15 @@ aht_status aht_sync(aht_ctx* ctx);
  * (1 .. 10^9), on an mbarrier nothing arrives on; the wait expires and latches the
  * timeout bit, so the next aht_sync returns AHT_ETIMEOUT.  No fault, no hang. */
 aht_status aht_debug_expire_wait(aht_ctx* ctx, int64_t limit_ns);
+
+/* Allocation-failure hook (no paper counterpart), process-wide: with n >= 1 the n-th
+ * device or pinned-host allocation that aht_create makes from now on fails as if the
+ * device were out of memory (nothing is allocated for it), so that aht_create's unwinding
+ * can be checked: it returns AHT_ENOMEM and frees everything it had allocated.  n <= 0
+ * switches the hook off.  aht_debug_live_allocs returns the number of device and pinned
+ * blocks that contexts hold right now (each aht_destroy returns its context's). */
+aht_status aht_debug_fail_alloc(int64_t n);
+int64_t aht_debug_live_allocs(void);
 
 /* Failure-detection hook for the real kernels (no paper counterpart).  The next call of
  * aht_rollout, aht_rollout_resample, aht_rollout_ippo or aht_xplay_matrix that runs on a

@@ -1,6 +1,6 @@
 // aht_oracle.cpp -- plain, slow CPU oracle (TEST INFRASTRUCTURE ONLY; see aht_oracle.h).
 //
-// Written to be read against the paper and the readings in the design doc, not to be fast:
+// Written to be read against the paper and the readings stated in aht_oracle.h, not to be fast:
 // one env at a time, plain loops, fp64 for every policy, sampling and GAE quantity,
 // fp32 exactly where the method's own rewards and returns are fp32.  Built with
 // -ffp-contract=off so no multiply-add is fused on any host.

@@ -11,8 +11,7 @@
  *     observation, one shared team reward) for three games: Level-Based Foraging,
  *     a 5x4 Overcooked-style kitchen and 2-player Hanabi (Sec. 4, Table
  *     "JaxAHT Environments").  The paper gives no game rules; the rules here are
- *     the readings listed in DESIGN.md ("Readings"), written from the workload
- *     descriptions;
+ *     readings of the workload descriptions, stated with each game's functions below;
  *   - the decentralised MLP policy pi_i(a | o_i) (Sec. 3) in fp64 from exact weights,
  *     masked categorical sampling (App. B, masked categorical) in fp64;
  *   - PPO's generalised advantage estimate (App. C, "PPO ego") in fp64;
@@ -87,7 +86,7 @@ void orc_lbf_obs(const orc_env_desc* d, const orc_lbf_state* s, int32_t seat, ui
 
 /* Rule-based LBF teammates (App. F, LBF heuristic suite: Greedy picks the next uneaten
  * food online by a criterion, Sequential plans a food order before the episode).  The
- * paper names the criteria and orderings only; the rules are the readings in the design doc:
+ * paper names the criteria and orderings only; the rules are these readings:
  *   k = 0..4  Greedy: argmin over uneaten foods of dist(self) | dist(teammate) |
  *             dist(self) + dist(teammate) | level | -level (ties: lower food index);
  *   k = 5..10 Sequential: the first uneaten food in the order of row-major cell index
@@ -151,7 +150,7 @@ int32_t orc_hanabi_step(orc_hanabi_state* s, int32_t a, float* team);
 void orc_hanabi_obs(const orc_hanabi_state* s, int32_t seat, uint8_t* out);
 
 /* ---- Mini Hanabi, 2 players (Sec. 4 Table "JaxAHT Environments": 3 colours x 3 ranks).
- * The paper gives only the colour and rank counts; the rest is the reading in the design doc:
+ * The paper gives only the colour and rank counts; the rest is this reading:
  * 18-card deck (ranks 1,1,1,2,2,3 per colour), 2-card hands, 3 info and 1 life tokens,
  * 10 actions (play slot 0-1, discard slot 0-1, hint colour 0-2, hint rank 1-3), card type
  * = colour*3 + rank-1, and the full game's rules and observation sections at this size
@@ -321,7 +320,10 @@ void orc_xp_stats(const float* xp, int32_t n_ego, int32_t n_tm, double* upper, d
 /* ---- PPO ego update (fp64; ppo_oracle.cpp) -------------------------------------- */
 /* App. C "PPO ego": PPO (Schulman et al. 2017) with the clipped surrogate, a clipped
  * value loss and an entropy bonus, per-minibatch advantage normalisation, global-norm
- * gradient clipping and Adam (Kingma & Ba 2015).  Readings in DESIGN.md "PPO update".
+ * gradient clipping and Adam (Kingma & Ba 2015); the paper states neither the loss nor
+ * the hyperparameters, so the settings are those orc_ppo_hp carries (defaults: 4 epochs x
+ * 4 minibatches, clip 0.2, value 0.5, entropy 0.01, gradient norm 0.5, Adam 0.9 / 0.999 /
+ * 1e-5, lr 2.5e-4).
  * Parameters are one flat array: W1 [h0][obs_dim], b1 [h0], W2 [h1][h0], b2 [h1],
  * W3 [n_act + 1][h1], b3 [n_act + 1] (the last output row is the value estimate). */
 enum { ORC_STREAM_PERMUTE = 4 };

@@ -4,7 +4,7 @@
 // distribution; the paper states no loss details or hyperparameters, so the update here
 // is the clipped-surrogate PPO of that paper (policy term, clipped value term, entropy
 // bonus), with per-minibatch advantage normalisation, global-norm gradient clipping and
-// Adam (Kingma & Ba 2015).  The readings are listed in DESIGN.md ("PPO update").  The
+// Adam (Kingma & Ba 2015), with the settings stated at orc_ppo_update in aht_oracle.h.  The
 // forward and backward use bf16-rounded copies of W1 and W2 (the weights the bf16
 // rollout runs), fp64 everywhere else; the gradient is taken at the rounded weights and
 // applied to the fp64 master copy.  Plain loops in the order of the definitions.

@@ -141,6 +141,10 @@ def load() -> C.CDLL:
             L.aht_set_policy.argtypes = [vp, i32, C.POINTER(vp), C.POINTER(vp), i32, i32]
             L.aht_set_timing.argtypes = [vp, i32]
             L.aht_get_timing.argtypes = [vp, C.POINTER(C.c_double), C.POINTER(i64)]
+            L.aht_debug_fail_alloc.argtypes = [i64]
+            L.aht_debug_fail_alloc.restype = C.c_int
+            L.aht_debug_live_allocs.argtypes = []
+            L.aht_debug_live_allocs.restype = i64
             L.aht_debug_expire_at.argtypes = [vp, i32, i64]
             L.aht_debug_expire_at.restype = C.c_int
             L.aht_debug_logits.argtypes = [vp, vp, i64]
@@ -420,6 +424,17 @@ def aht_sync(ctx: Context):
 
 
 AHT_DEBUG_STRIDE = 32
+
+
+def aht_debug_fail_alloc(n: int):
+    """Allocation-failure hook: the n-th allocation aht_create makes from now on fails
+    (n <= 0: off)."""
+    _check(load().aht_debug_fail_alloc(n))
+
+
+def aht_debug_live_allocs() -> int:
+    """Device and pinned blocks that contexts hold now."""
+    return int(load().aht_debug_live_allocs())
 
 
 def aht_debug_expire_at(ctx: Context, step: int, limit_ns: int):

@@ -2,6 +2,7 @@
 // context memory, weight packing and kernel launches.  No compute happens on the host
 // except packing the population once in aht_create.
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -30,6 +31,36 @@ aht_status fail(aht_status s, const std::string& msg) {
     if (e_ != cudaSuccess)                                                               \
       return fail(AHT_ECUDA, std::string(#call) + ": " + cudaGetErrorString(e_));        \
   } while (0)
+
+// Device and pinned allocations of contexts go through these: they count the blocks a
+// context holds (aht_debug_live_allocs) and let a test make the n-th allocation fail
+// (aht_debug_fail_alloc) without touching the device.
+std::atomic<int64_t> g_fail_countdown{0};  // > 0: the allocation that brings it to 0 fails
+std::atomic<int64_t> g_live_allocs{0};
+bool alloc_hook_fires() {
+  int64_t n = g_fail_countdown.load();
+  while (n > 0 && !g_fail_countdown.compare_exchange_weak(n, n - 1)) {
+  }
+  return n == 1;
+}
+cudaError_t ctx_malloc(void** p, size_t bytes) {
+  if (alloc_hook_fires()) return cudaErrorMemoryAllocation;
+  const cudaError_t e = cudaMalloc(p, bytes);
+  if (e == cudaSuccess) ++g_live_allocs;
+  return e;
+}
+cudaError_t ctx_malloc_host(void** p, size_t bytes) {
+  if (alloc_hook_fires()) return cudaErrorMemoryAllocation;
+  const cudaError_t e = cudaMallocHost(p, bytes);
+  if (e == cudaSuccess) ++g_live_allocs;
+  return e;
+}
+void ctx_free(void* p) {
+  if (p && cudaFree(p) == cudaSuccess) --g_live_allocs;
+}
+void ctx_free_host(void* p) {
+  if (p && cudaFreeHost(p) == cudaSuccess) --g_live_allocs;
+}
 
 struct DeviceGuard {
   int prev = -1;
@@ -642,27 +673,27 @@ void aht_destroy(aht_ctx* c) {
   if (!c) return;
   DeviceGuard g(c->device);
   cudaStreamSynchronize(c->stream);
-  cudaFree(c->state);
-  cudaFree(c->ep_step);
-  cudaFree(c->rs_kidx);
-  cudaFree(c->rs_hist);
-  cudaFree(c->weights);
-  cudaFree(c->perm);
-  cudaFree(c->tiles);
-  cudaFree(c->xp_returns);
-  cudaFree(c->last_value);
-  cudaFree(c->status);
-  if (c->staging) cudaFreeHost(c->staging);
-  if (c->tc_staging) cudaFreeHost(c->tc_staging);
-  if (c->wide_staging) cudaFreeHost(c->wide_staging);
-  cudaFree(c->tcw);
-  cudaFree(c->wtcw);
+  ctx_free(c->state);
+  ctx_free(c->ep_step);
+  ctx_free(c->rs_kidx);
+  ctx_free(c->rs_hist);
+  ctx_free(c->weights);
+  ctx_free(c->perm);
+  ctx_free(c->tiles);
+  ctx_free(c->xp_returns);
+  ctx_free(c->last_value);
+  ctx_free(c->status);
+  if (c->staging) ctx_free_host(c->staging);
+  if (c->tc_staging) ctx_free_host(c->tc_staging);
+  if (c->wide_staging) ctx_free_host(c->wide_staging);
+  ctx_free(c->tcw);
+  ctx_free(c->wtcw);
   for (int i = 0; i < 2; ++i) {
-    cudaFree(c->xp_st[i]);
-    cudaFree(c->xp_act[i]);
-    cudaFree(c->xp_alive[i]);
+    ctx_free(c->xp_st[i]);
+    ctx_free(c->xp_act[i]);
+    ctx_free(c->xp_alive[i]);
   }
-  cudaFree(c->xp_nsteps);
+  ctx_free(c->xp_nsteps);
   if (c->upload_done) cudaEventDestroy(c->upload_done);
   for (auto& e : c->ev)
     if (e) cudaEventDestroy(e);
@@ -737,7 +768,7 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
       {(void**)&c->status, 4},
   };
   for (auto& a : allocs)
-    if (cudaMalloc(a.p, a.bytes) != cudaSuccess) {
+    if (ctx_malloc(a.p, a.bytes) != cudaSuccess) {
       cudaGetLastError();
       return bail(AHT_ENOMEM, "cudaMalloc of " + std::to_string(a.bytes) + " bytes failed");
     }
@@ -746,7 +777,7 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
     return bail(AHT_ECUDA, "uploading the population failed");
   if (c->ops.smem_limit(c->smem_optin) != cudaSuccess || policy_set_smem_limit(c->smem_optin) != cudaSuccess)
     return bail(AHT_ECUDA, "setting the shared-memory limit failed");
-  if (cudaMallocHost((void**)&c->staging, (size_t)m.stride * 4) != cudaSuccess)
+  if (ctx_malloc_host((void**)&c->staging, (size_t)m.stride * 4) != cudaSuccess)
     return bail(AHT_ENOMEM, "pinned staging allocation failed");
   if (cudaEventCreateWithFlags(&c->upload_done, cudaEventDisableTiming) != cudaSuccess)
     return bail(AHT_ECUDA, "cudaEventCreate failed");
@@ -766,13 +797,13 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
         return bail(ps, msg);
       }
     }
-    if (cudaMalloc((void**)&c->tcw, blocks.size()) != cudaSuccess) {
+    if (ctx_malloc((void**)&c->tcw, blocks.size()) != cudaSuccess) {
       cudaGetLastError();
       return bail(AHT_ENOMEM, "cudaMalloc of the tensor-core population failed");
     }
     if (cudaMemcpy(c->tcw, blocks.data(), blocks.size(), cudaMemcpyHostToDevice) != cudaSuccess)
       return bail(AHT_ECUDA, "uploading the tensor-core population failed");
-    if (cudaMallocHost((void**)&c->tc_staging, c->tcd.pol_bytes) != cudaSuccess)
+    if (ctx_malloc_host((void**)&c->tc_staging, c->tcd.pol_bytes) != cudaSuccess)
       return bail(AHT_ENOMEM, "pinned staging allocation failed");
     c->tc = true;
   }
@@ -800,7 +831,7 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
         {(void**)&c->xp_nsteps, (size_t)n_envs * 4},
     };
     for (auto& x : wa)
-      if (cudaMalloc(x.p, x.bytes) != cudaSuccess) {
+      if (ctx_malloc(x.p, x.bytes) != cudaSuccess) {
         cudaGetLastError();
         return bail(AHT_ENOMEM, "cudaMalloc of " + std::to_string(x.bytes) + " bytes failed");
       }
@@ -810,7 +841,7 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
                            : env.kind == AHT_HANABI    ? hanabi_xplay_tc_smem_limit(c->wide_smem)
                                                   : overcooked_xplay_tc_smem_limit(c->wide_smem);
     if (se != cudaSuccess) return bail(AHT_ECUDA, "setting the shared-memory limit failed");
-    if (cudaMallocHost((void**)&c->wide_staging, c->wd.pol_bytes) != cudaSuccess)
+    if (ctx_malloc_host((void**)&c->wide_staging, c->wd.pol_bytes) != cudaSuccess)
       return bail(AHT_ENOMEM, "pinned staging allocation failed");
     c->wide = true;
   }
@@ -1459,6 +1490,13 @@ aht_status aht_debug_logits(aht_ctx* c, float* buf, int64_t floats) {
   c->dbg_floats = buf ? floats : 0;
   return AHT_OK;
 }
+
+aht_status aht_debug_fail_alloc(int64_t n) {
+  g_fail_countdown.store(n > 0 ? n : 0);
+  return AHT_OK;
+}
+
+int64_t aht_debug_live_allocs(void) { return g_live_allocs.load(); }
 
 aht_status aht_debug_expire_at(aht_ctx* c, int32_t step, int64_t limit_ns) {
   if (!c) return fail(AHT_EINVAL, "ctx is NULL");

@@ -2,8 +2,12 @@
 //
 // 50-card deck (5 colours x ranks 1,1,1,2,2,3,3,4,4,5), 5-card hands, 8 info and 3 life
 // tokens, 20 actions (play slot 0-4, discard slot 0-4, hint colour 0-4, hint rank 1-5),
-// seat 0 first.  Card type = colour*5 + rank-1.  Rules and the 660-bit observation as
-// read in DESIGN.md "Readings".
+// seat 0 first.  Card type = colour*5 + rank-1.  Play is legal for an occupied slot,
+// discard also needs info < 8, a hint needs info > 0 and a matching partner card; a
+// successful play pays +1 (a completed 5 returns an info token), losing the last life
+// zeroes the return; the game ends at 0 lives, score 25, or two turns after the draw that
+// empties the deck.  The 660-bit observation (Sec. 4 Table, Hanabi; layout ours) is laid
+// out section by section in obs_into.
 #pragma once
 #include "aht_common.cuh"
 

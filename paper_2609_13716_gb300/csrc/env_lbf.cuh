@@ -1,6 +1,6 @@
 // env_lbf.cuh -- Level-Based Foraging on the device (one thread per env).
 //
-// Rules (the workload's statement): two agents with levels in
+// Rules (the workload's statement; the paper fixes none, Sec. 4 Table): two agents with levels in
 // 1..max_level, n_food foods with levels in 1..(sum of agent levels); actions
 // {noop, N, S, W, E, load}; a food is eaten when the summed levels of the 4-adjacent
 // loading agents reach its level, each loader receiving food_level*agent_level /

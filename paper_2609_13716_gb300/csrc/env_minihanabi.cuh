@@ -2,8 +2,9 @@
 //
 // 3 colours x ranks 1,1,1,2,2,3 (18 cards), 2-card hands, 3 info and 1 life tokens, 10
 // actions (play slot 0-1, discard slot 0-1, hint colour 0-2, hint rank 1-3), seat 0
-// first.  Card type = colour*3 + rank-1.  The full game's rules at this size; the
-// 156-feature observation (153 + 3 zero) as read in DESIGN.md "Readings".
+// first.  Card type = colour*3 + rank-1.  The full game's rules at this size (Sec. 4
+// Table: "Mini (3 colors x 3 ranks)"); the observation is the full game's sections at
+// this size, 153 features, then 3 zero features (156).
 #pragma once
 #include "aht_common.cuh"
 

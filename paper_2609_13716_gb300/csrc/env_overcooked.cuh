@@ -3,7 +3,10 @@
 // Layout (x right, y down):  row 0 "#O#P#", row 1 "#...#", row 2 "D...S", row 3 "##O##"
 // (# counter, O onion dispenser, P pot, D dish dispenser, S serving cell, . floor).
 // Actions {noop, N, S, E, W, interact}; a full pot (3 onions) cooks for cook_time steps;
-// a served soup pays soup_reward to the team.  Rules as read in DESIGN.md "Readings".
+// a served soup pays soup_reward to the team.  A move sets the facing and enters floor
+// only (equal targets or a swap: both stay); interact acts on the faced cell, agent 0
+// first; a pot cooking at the start of a step counts down at its end; episodes have a
+// fixed length and a shared reward only.
 #pragma once
 #include "aht_common.cuh"
 

@@ -134,3 +134,45 @@ def test_expire_at_validates_its_limit():
             aht.aht_debug_expire_at(ctx, 3, bad)
         assert e.value.status == aht.AHT_EINVAL
     aht.aht_debug_expire_at(ctx, -1, 0)     # clearing needs no limit
+
+
+@pytest.mark.parametrize("name,n_envs", [
+    ("lbf7x7_ppo_16384x128", 500),      # bf16 LBF: tensor-core blocks too
+    ("lbf7x7_64x50_fp32", 64),          # fp32 LBF: split-weight blocks
+    ("hanabi_xplay_16x16x32", 300),     # streamed cross-play buffers too
+])
+def test_create_unwinds_every_failed_allocation(name, n_envs):
+    """aht_create with its k-th allocation failing, for every k: AHT_ENOMEM, no context,
+    and every block it had allocated is freed (the library's live-block count and the
+    device's free memory are back where they were); then a normal create succeeds."""
+    require_gpu()
+    wl = W.WORKLOADS[name]
+    import gc
+    ctx, _ = make_ctx(wl, n_envs)            # loads the kernels once
+    ctx.close()
+    gc.collect()                             # contexts of earlier tests go now, not mid-loop
+    gc.disable()
+    torch.cuda.synchronize()
+    base = aht.aht_debug_live_allocs()
+    free0 = torch.cuda.mem_get_info()[0]
+    k, failed = 1, 0
+    while True:
+        aht.aht_debug_fail_alloc(k)
+        try:
+            ctx, _ = make_ctx(wl, n_envs)
+        except aht.AhtError as e:
+            assert e.status == aht.AHT_ENOMEM, (k, e)
+            assert aht.aht_debug_live_allocs() == base, k
+            failed += 1
+            k += 1
+            continue
+        finally:
+            aht.aht_debug_fail_alloc(0)
+        break                                # k exceeds the allocations of one create
+    assert failed >= 10                      # every allocation of a create was tried
+    assert aht.aht_debug_live_allocs() == base + failed
+    ctx.close()
+    gc.enable()
+    assert aht.aht_debug_live_allocs() == base
+    torch.cuda.synchronize()
+    assert abs(torch.cuda.mem_get_info()[0] - free0) <= 4 << 20
