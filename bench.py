@@ -630,7 +630,8 @@ def run_s5(aht, W, torch, stream, bf16_peak, n=16384, K=10):
     flops = n * (dense + ssm)
     achieved = flops / (ms * 1e-3) / 1e12
     return {"workload": f"s5_actor_critic_lbf7x7_{n}", "ms_per_step": ms,
-            "env_steps_per_s": n / (ms * 1e-3), "bf16_gemm_launches": 7, "own_kernel_launches": 8,
+            "env_steps_per_s": n / (ms * 1e-3), "tcgen05_gemm_launches": 7, "own_kernel_launches": 9,
+            "library_gemm_launches": 0,
             "roofline": {"bound": "tensor", "achieved": achieved, "peak": bf16_peak, "unit": "TFLOP/s",
                          "frac": achieved / bf16_peak, "flops_per_step": flops,
                          "flops_basis": "model FLOPs of the encoder, SSM and heads, counted once; "

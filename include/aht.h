@@ -380,7 +380,8 @@ aht_status aht_learner_sync(aht_learner* L);
  * recurrence in fp32 (lbar and Bbar computed in fp64 at create); the output layers run
  * in fp32 from the fp32 last hidden layer.  Parameters are host fp32 arrays, row-major [out][in]. */
 typedef struct aht_s5_params {
-  int32_t obs_dim, n_actions, H, P, F;  /* H, P multiples of 16, F of 16; n_actions <= 32 */
+  int32_t obs_dim, n_actions, H, P, F;  /* obs_dim <= 2048; H, P, F multiples of 32, P <= 128;
+                                           n_actions <= 32 */
   const float *We1, *be1, *We2, *be2;   /* [H][obs_dim] [H] [H][H] [H] */
   const float *lam_re, *lam_im, *log_dt;/* [P] (lam_re < 0) */
   const float *B_re, *B_im;             /* [P][H] */
@@ -390,15 +391,17 @@ typedef struct aht_s5_params {
   const float *Wc[4], *bc[4];           /* critic [F][H] [F][F] [F][F] [1][F] */
 } aht_s5_params;
 typedef struct aht_s5 aht_s5;           /* opaque, library-owned */
-/* Allocates everything a step of up to max_envs envs needs (weights, scratch, a GEMM
- * workspace).  cuda_stream: a cudaStream_t (NULL = default). */
+/* Allocates everything a step of up to max_envs envs needs (weights packed as tiled bf16
+ * operands of the library's tensor-core GEMM, scratch activations).  cuda_stream: a
+ * cudaStream_t (NULL = default). */
 aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_stream, aht_s5** out);
 void aht_s5_destroy(aht_s5* s);
 /* One policy step of n envs (device arrays): obs u8 [n][obs_dim], reset u8 [n] (1 zeroes
  * the env's state first: the first step of an episode), legal u8 [n][n_actions] or NULL,
  * state f32 [n][2P] in/out (real parts, then imaginary parts) -> logits f32
  * [n][n_actions] (-inf where illegal), values f32 [n].  1 <= n <= max_envs.
- * Asynchronous on the creation stream; aht_s5_sync reports errors. */
+ * Asynchronous on the creation stream; aht_s5_sync reports errors (AHT_ETIMEOUT if a
+ * product's bounded wait expired). */
 aht_status aht_s5_step(aht_s5* s, const uint8_t* obs, const uint8_t* reset, const uint8_t* legal,
                        int64_t n, float* state, float* logits, float* values);
 aht_status aht_s5_sync(aht_s5* s);

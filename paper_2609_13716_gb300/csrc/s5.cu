@@ -1,9 +1,9 @@
 // s5.cu -- one step of the recurrent S5 actor-critic for a batch of envs (the model and
-// its readings are stated in include/aht.h).  The dense layers are plain GEMMs over the
-// batch (cuBLAS, bf16 operands, fp32 accumulate) with the activations carried as two bf16
-// halves; the elementwise parts (bias, relu, the split, the SSM recurrence, GELU, masking)
-// are this file's kernels.
-#include <cublas_v2.h>
+// its readings are stated in include/aht.h).  The dense layers and the SSM's products run
+// on this library's tcgen05 GEMM (s5_gemm.cuh) with bf16 operands and fp32 accumulation;
+// activations are carried as bf16 terms (hi | lo, or hi | lo | hi against weights
+// [Wh | Wh | Wl] for the SSM's fp32 operands) written by each product's epilogue straight
+// into the next product's tiled operand, so no fp32 accumulator goes through memory.
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -13,6 +13,7 @@
 #include <vector>
 
 #include "kernels.h"
+#include "s5_gemm.cuh"
 
 namespace aht {
 aht_status set_last_error(aht_status s, const char* msg);  // the message of aht_last_error
@@ -37,30 +38,29 @@ struct S5DeviceGuard {
 struct aht_s5 {
   int device = 0;
   cudaStream_t stream = nullptr;
-  cublasHandle_t blas = nullptr;
   int K = 0, A = 0, H = 0, P = 0, F = 0;
-  int Kp = 0;  // K rounded up to 16: observation rows and We1 rows padded with zeros
+  int K0 = 0;  // K rounded up to 64: observation columns (and We1 columns) padded with zeros
   int64_t max_n = 0;
-  // bf16 weights [out][in]. A layer fed with split activations holds each weight row twice,
-  // [W | W] (in = 2I), so that one product over [hi | lo] sums both halves. Heads: layer 0
-  // [2F][2H] (actor rows, then critic), layers 1-2 [2][F][2F]; the encoder's layer 1 [H][K]
-  // sees exact bf16 observations. The output layers, W3 [A + 1][F] (actor rows, then the
-  // critic's), hold the bf16-rounded weights as fp32 for the CUDA-core output kernel.
-  __nv_bfloat16 *We1 = nullptr, *We2 = nullptr, *Wh0 = nullptr, *Wh1 = nullptr, *Wh2 = nullptr;
-  float* W3 = nullptr;
+  int m_tiles = 0;  // 128-row tiles of max_n
+  int n_sms = 0;
+  // weights as tiled bf16 GEMM operands (see s5_gemm.cuh).  A layer fed with split
+  // activations holds each weight row twice, [W | W] (in = 2I), so that one product over
+  // [hi | lo] sums both halves: encoder We1 [H][K0], We2 [H][2H]; SSM Bbar3 [2P][3H]
+  // (re rows, then im rows) and Cc3 [H][6P] from Cc = (C_re | -C_im) as [Wh | Wh | Wl];
+  // heads Wh0 [2F][2H] (actor rows, then critic), Wh1 and Wh2 [2][F][2F].  The output
+  // layers W3a [A][F], W3c [1][F] hold the bf16-rounded weights as fp32.
+  uint8_t *We1 = nullptr, *We2 = nullptr, *Bbar3 = nullptr, *Cc3 = nullptr, *Wh0 = nullptr, *Wh1 = nullptr,
+          *Wh2 = nullptr;
+  float *W3a = nullptr, *W3c = nullptr;
   float *be1 = nullptr, *be2 = nullptr, *bh0 = nullptr, *bh1 = nullptr, *bh2 = nullptr,
         *ba3 = nullptr, *bc3 = nullptr;
-  // SSM: lbar [2][P] (re, im) and D [H] fp32.  Its products run as three bf16 terms: an
-  // fp32 operand a = ah + al (two bf16), activations stored [hi | lo | hi] and weights
-  // [Wh | Wh | Wl], one GEMM sums Wh hi + Wh lo + Wl hi (~2^-16 relative).  Bbar3 [2P][3H]
-  // (re rows, then im rows), Cc3 [H][3 x 2P] from Cc = (C_re | -C_im).
-  float *lbar = nullptr, *Dv = nullptr;
-  __nv_bfloat16 *Bbar3 = nullptr, *Cc3 = nullptr;
-  // scratch
-  // x16 [n][Kp]; act: split activations, each row [group][hi | lo][I] (heads: 2 groups of F)
-  __nv_bfloat16 *x16 = nullptr, *act = nullptr;
-  float *acc = nullptr, *u = nullptr, *bu = nullptr, *y = nullptr;
-  void* workspace = nullptr;
+  float *lbar = nullptr, *Dv = nullptr;  // lbar [2][P] (re, im), D [H]
+  // scratch: tiled activations (x0: the observation; a1..a4: encoder, SSM input and
+  // output, residual; a5, a6: [2 heads] of [hi | lo] of F), u fp32 [n][H], head partials
+  uint8_t *x0 = nullptr, *a1 = nullptr, *a2 = nullptr, *a3 = nullptr, *a4 = nullptr, *a5 = nullptr,
+          *a6 = nullptr;
+  float *u = nullptr, *partial = nullptr;
+  uint32_t* status = nullptr;
   std::vector<void*> owned;
 };
 
@@ -71,219 +71,87 @@ namespace {
     cudaError_t e_ = (call);                                                                   \
     if (e_ != cudaSuccess) return set_last_error(AHT_ECUDA, cudaGetErrorString(e_));          \
   } while (0)
-#define S5_BLAS(call)                                                                          \
-  do {                                                                                         \
-    if ((call) != CUBLAS_STATUS_SUCCESS) return set_last_error(AHT_ECUDA, "cuBLAS call failed"); \
-  } while (0)
 
-constexpr size_t kWorkspace = 32u << 20;
-
-// out[r][c] = obs[r][c] as bf16 for c < K, 0 for K <= c < Kp (Kp % 4 == 0); four columns
-// a thread
-__global__ void u8_to_bf16(const uint8_t* __restrict__ in, __nv_bfloat16* __restrict__ out, int K, int Kp,
-                           int64_t n) {
-  const int c = 4 * (blockIdx.x * blockDim.x + threadIdx.x);
-  if (c >= Kp) return;
-  for (int64_t r = (int64_t)blockIdx.y * blockDim.y + threadIdx.y; r < n; r += (int64_t)gridDim.y * blockDim.y) {
-    const uint8_t* row = in + r * K;
-    float v[4];
+// The observation u8 [n][K] -> the first product's tiled bf16 operand [m_tiles][K0 / 64]
+// (exact: small integers), columns K..K0-1 zero; one thread per 8 columns of a row
+// (x over a row's chunks, y over rows).
+__global__ void obs_tiles(const uint8_t* __restrict__ obs, int K, int K0, int64_t n, uint8_t* __restrict__ x0) {
+  const int kc = threadIdx.x;  // 8-column chunk
+  if (kc >= K0 / 8) return;
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.y + threadIdx.y; r < n; r += (int64_t)gridDim.x * blockDim.y) {
+    const uint8_t* row = obs + r * K;
+    uint32_t w[4];
 #pragma unroll
-    for (int k = 0; k < 4; ++k) v[k] = c + k < K ? (float)row[c + k] : 0.0f;
-    __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]), b = __floats2bfloat162_rn(v[2], v[3]);
-    *reinterpret_cast<uint2*>(out + r * Kp + c) =
-        make_uint2(*reinterpret_cast<uint32_t*>(&a), *reinterpret_cast<uint32_t*>(&b));
-  }
-}
-
-// Row-wise kernels run on 2-D blocks and grids: x covers a row's columns (four per thread;
-// the widths are multiples of 16), y strides over rows, so that column arithmetic stays
-// 32-bit.
-constexpr int kRowsPerThread = 4;  // rows a thread of bias_act_split loads before it stores
-
-__device__ __forceinline__ int64_t row0() { return (int64_t)blockIdx.y * blockDim.y + threadIdx.y; }
-__device__ __forceinline__ int64_t row_step() { return (int64_t)gridDim.y * blockDim.y; }
-
-__device__ __forceinline__ uint2 pack_bf16x4(float a, float b, float c, float d) {
-  __nv_bfloat162 lo = __floats2bfloat162_rn(a, b), hi = __floats2bfloat162_rn(c, d);
-  return make_uint2(*reinterpret_cast<uint32_t*>(&lo), *reinterpret_cast<uint32_t*>(&hi));
-}
-
-// writes v (four columns) as hi at d and lo = bf16(v - hi) at d + I (and hi again at
-// d + 2I for a three-term product)
-__device__ __forceinline__ void store_split4(__nv_bfloat16* d, int I, float4 v, bool hi_again = false) {
-  const uint2 h = pack_bf16x4(v.x, v.y, v.z, v.w);
-  const __nv_bfloat162 h01 = *reinterpret_cast<const __nv_bfloat162*>(&h.x);
-  const __nv_bfloat162 h23 = *reinterpret_cast<const __nv_bfloat162*>(&h.y);
-  const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
-  *reinterpret_cast<uint2*>(d) = h;
-  *reinterpret_cast<uint2*>(d + I) = pack_bf16x4(v.x - f01.x, v.y - f01.y, v.z - f23.x, v.w - f23.y);
-  if (hi_again) *reinterpret_cast<uint2*>(d + 2 * I) = h;
-}
-
-// v = act(acc + b), acc rows of g groups of I columns (ld g I, I % 4 == 0): v as fp32
-// (optional) and split (optional) at split[row][group][part][col] (ld parts g I): parts = 2
-// stores hi, lo; parts = 3 stores hi, lo, hi
-__global__ void bias_act_split(const float* __restrict__ acc, const float* __restrict__ b, int I, int g,
-                               int64_t n, bool relu, float* __restrict__ out32,
-                               __nv_bfloat16* __restrict__ split, int parts) {
-  const int c = 4 * (blockIdx.x * blockDim.x + threadIdx.x);
-  const int row_w = g * I;
-  if (c >= row_w) return;
-  const int gg = c / I, f = c - gg * I;
-  const float4 bb = *reinterpret_cast<const float4*>(b + c);
-  const int64_t step = row_step();
-  for (int64_t r0 = row0(); r0 < n; r0 += kRowsPerThread * step) {
-    float4 v[kRowsPerThread];
-#pragma unroll
-    for (int k = 0; k < kRowsPerThread; ++k)  // all loads first: several rows in flight
-      if (r0 + k * step < n) v[k] = __ldcs(reinterpret_cast<const float4*>(acc + (r0 + k * step) * row_w + c));
-#pragma unroll
-    for (int k = 0; k < kRowsPerThread; ++k) {
-      const int64_t r = r0 + k * step;
-      if (r >= n) break;
-      float4 x = v[k];
-      x.x += bb.x; x.y += bb.y; x.z += bb.z; x.w += bb.w;
-      if (relu) {
-        x.x = fmaxf(x.x, 0.0f); x.y = fmaxf(x.y, 0.0f); x.z = fmaxf(x.z, 0.0f); x.w = fmaxf(x.w, 0.0f);
-      }
-      if (out32) *reinterpret_cast<float4*>(out32 + r * row_w + c) = x;
-      if (split) store_split4(split + r * parts * row_w + (int64_t)gg * parts * I + f, I, x, parts == 3);
+    for (int j = 0; j < 4; ++j) {
+      const int c = 8 * kc + 2 * j;
+      const float f0 = c < K ? (float)row[c] : 0.0f, f1 = c + 1 < K ? (float)row[c + 1] : 0.0f;
+      w[j] = tc::pack_bf16(f0, f1);
     }
+    const int64_t mt = r >> 7;
+    const int rr = (int)(r & 127), kt = kc >> 3, kb = kc & 7;
+    *reinterpret_cast<uint4*>(x0 + s5g::chunk_off(mt, K0 / 64, kt, rr, kb)) = make_uint4(w[0], w[1], w[2], w[3]);
   }
 }
 
-// x = lbar x (x = 0 first where reset) + Bbar u, in place; state [n][2P] (re, im), bu [n][2P];
-// x also as [hi | lo | hi] bf16 rows of 2P each (ld 6P) for the three-term C product
-__global__ void ssm_recur(const float* __restrict__ lbar, const float* __restrict__ bu,
-                          const uint8_t* __restrict__ reset, float* __restrict__ state, int P,
-                          int64_t n, __nv_bfloat16* __restrict__ xsplit) {
-  const int p = 4 * (blockIdx.x * blockDim.x + threadIdx.x);
-  if (p >= P) return;
-  const float4 lr = *reinterpret_cast<const float4*>(lbar + p);
-  const float4 li = *reinterpret_cast<const float4*>(lbar + P + p);
-  for (int64_t e = row0(); e < n; e += row_step()) {
-    float* s = state + e * 2 * P;
-    const float* bp = bu + e * 2 * P;
-    float4 xr = *reinterpret_cast<const float4*>(s + p), xi = *reinterpret_cast<const float4*>(s + P + p);
-    if (reset[e]) xr = xi = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-    const float4 br = *reinterpret_cast<const float4*>(bp + p), bi = *reinterpret_cast<const float4*>(bp + P + p);
-    float4 orr, oi;
-    orr.x = fmaf(lr.x, xr.x, fmaf(-li.x, xi.x, br.x)); oi.x = fmaf(lr.x, xi.x, fmaf(li.x, xr.x, bi.x));
-    orr.y = fmaf(lr.y, xr.y, fmaf(-li.y, xi.y, br.y)); oi.y = fmaf(lr.y, xi.y, fmaf(li.y, xr.y, bi.y));
-    orr.z = fmaf(lr.z, xr.z, fmaf(-li.z, xi.z, br.z)); oi.z = fmaf(lr.z, xi.z, fmaf(li.z, xr.z, bi.z));
-    orr.w = fmaf(lr.w, xr.w, fmaf(-li.w, xi.w, br.w)); oi.w = fmaf(lr.w, xi.w, fmaf(li.w, xr.w, bi.w));
-    *reinterpret_cast<float4*>(s + p) = orr;
-    *reinterpret_cast<float4*>(s + P + p) = oi;
-    store_split4(xsplit + e * 6 * P + p, 2 * P, orr, true);
-    store_split4(xsplit + e * 6 * P + P + p, 2 * P, oi, true);
+// logits[e][a] = sum over n-tiles and column halves (in order) of the actor's partial sums
+// + ba3[a] (-inf where illegal); values[e] likewise from the critic's
+// (slots: the partial sums per (row, head, n-tile, column half): 8, or 32 for A > 8)
+__global__ void heads_final(const float* __restrict__ partial, int n_tiles, int slots, const float* __restrict__ ba3,
+                            const float* __restrict__ bc3, const uint8_t* __restrict__ legal, int A, int64_t n,
+                            float* __restrict__ logits, float* __restrict__ values) {
+  const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= n) return;
+  const int parts = 2 * n_tiles;  // (n-tile, column half) pairs
+  const float* pa = partial + (e * 2 + 0) * (int64_t)parts * slots;
+  const float* pc = partial + (e * 2 + 1) * (int64_t)parts * slots;
+  for (int a = 0; a < A; ++a) {
+    float z = 0.0f;
+    for (int t = 0; t < parts; ++t) z += pa[t * slots + a];
+    z += ba3[a];
+    logits[e * A + a] = (legal && !legal[e * A + a]) ? -INFINITY : z;
   }
+  float v = 0.0f;
+  for (int t = 0; t < parts; ++t) v += pc[t * slots];
+  values[e] = v + bc3[0];
 }
 
-__device__ __forceinline__ float gelu_exact(float y) { return y * 0.5f * erfcf(-y * 0.70710678118654752f); }
-
-// v = u + gelu(y + D u) -> split[row][0 | 1][H] (hi, lo bf16)
-__global__ void residual_gelu(const float* __restrict__ y, const float* __restrict__ u,
-                              const float* __restrict__ D, int H, int64_t n,
-                              __nv_bfloat16* __restrict__ split) {
-  const int c = 4 * (blockIdx.x * blockDim.x + threadIdx.x);
-  if (c >= H) return;
-  const float4 dd = *reinterpret_cast<const float4*>(D + c);
-  for (int64_t r = row0(); r < n; r += row_step()) {
-    const float4 uu = *reinterpret_cast<const float4*>(u + r * H + c);
-    const float4 yy = *reinterpret_cast<const float4*>(y + r * H + c);
-    float4 v;
-    v.x = uu.x + gelu_exact(fmaf(dd.x, uu.x, yy.x));
-    v.y = uu.y + gelu_exact(fmaf(dd.y, uu.y, yy.y));
-    v.z = uu.z + gelu_exact(fmaf(dd.z, uu.z, yy.z));
-    v.w = uu.w + gelu_exact(fmaf(dd.w, uu.w, yy.w));
-    store_split4(split + r * 2 * H + c, H, v);
-  }
+// Output columns per GEMM tile for an N-column product: the widest multiple of 32 up to
+// 256 that divides N (N is a multiple of 32).
+int bn_for(int N) {
+  for (int b = 256; b >= 32; b -= 32)
+    if (N % b == 0) return b;
+  return 32;
 }
 
-__device__ __forceinline__ float warp_sum(float x) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-  return x;
-}
-
-// The heads' last hidden layer and both output layers, one warp per env: h = relu(acc + b)
-// in fp32 (acc [n][2F]: actor columns, then critic), logits[a] = Wa3[a] . h_actor + ba3[a]
-// (-inf where illegal), value = Wc3 . h_critic + bc3. W3 [A + 1][F] fp32 (actor rows, then
-// the critic's); AM >= A is the register width of the logit sums.
-template <int AM>
-__global__ void heads_out(const float* __restrict__ acc, const float* __restrict__ b,
-                          const float* __restrict__ W3, const float* __restrict__ ba3,
-                          const float* __restrict__ bc3, const uint8_t* __restrict__ legal, int A, int F,
-                          int64_t n, float* __restrict__ logits, float* __restrict__ values) {
-  const int lane = threadIdx.x & 31;
-  const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
-  const int quads = F / 4;
-  for (int64_t e = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); e < n; e += warps) {
-    const float* row = acc + e * 2 * F;
-    float pa[AM], pv = 0.0f;
-#pragma unroll
-    for (int a = 0; a < AM; ++a) pa[a] = 0.0f;
-#pragma unroll 2
-    for (int q = lane; q < quads; q += 32) {
-      const float4 x = __ldcs(reinterpret_cast<const float4*>(row) + q);
-      const float4 bb = reinterpret_cast<const float4*>(b)[q];
-      const float4 h = make_float4(fmaxf(x.x + bb.x, 0.0f), fmaxf(x.y + bb.y, 0.0f), fmaxf(x.z + bb.z, 0.0f),
-                                   fmaxf(x.w + bb.w, 0.0f));
-#pragma unroll
-      for (int a = 0; a < AM; ++a)
-        if (a < A) {
-          const float4 w = __ldg(reinterpret_cast<const float4*>(W3 + (size_t)a * F) + q);
-          pa[a] = fmaf(h.x, w.x, fmaf(h.y, w.y, fmaf(h.z, w.z, fmaf(h.w, w.w, pa[a]))));
-        }
-      const float4 xc = __ldcs(reinterpret_cast<const float4*>(row + F) + q);
-      const float4 bc = reinterpret_cast<const float4*>(b + F)[q];
-      const float4 w = __ldg(reinterpret_cast<const float4*>(W3 + (size_t)A * F) + q);
-      pv = fmaf(fmaxf(xc.x + bc.x, 0.0f), w.x, pv);
-      pv = fmaf(fmaxf(xc.y + bc.y, 0.0f), w.y, pv);
-      pv = fmaf(fmaxf(xc.z + bc.z, 0.0f), w.z, pv);
-      pv = fmaf(fmaxf(xc.w + bc.w, 0.0f), w.w, pv);
+// Tiles of a bf16 matrix [rows][cols] (row-major, cols padded with zeros to a multiple of
+// 64) for the GEMM: n-tiles of BN rows (rows a multiple of BN), k-tiles of 64.
+std::vector<__nv_bfloat16> tile_matrix(const std::vector<__nv_bfloat16>& w, int rows, int cols, int BN) {
+  const int KT = (cols + 63) / 64, NT = rows / BN;
+  std::vector<__nv_bfloat16> t((size_t)NT * KT * BN * 64, __float2bfloat16_rn(0.0f));
+  for (int r = 0; r < rows; ++r)
+    for (int c = 0; c < cols; ++c) {
+      const int nt = r / BN, rr = r % BN, kt = c / 64, kk = c % 64;
+      const size_t tile = ((size_t)nt * KT + kt) * BN * 64;
+      const size_t off = (size_t)((rr >> 3) * 8 + (kk >> 3)) * 64 + (rr & 7) * 8 + (kk & 7);
+      t[tile + off] = w[(size_t)r * cols + c];
     }
-#pragma unroll
-    for (int a = 0; a < AM; ++a)
-      if (a < A) {
-        const float z = warp_sum(pa[a]) + ba3[a];
-        if (lane == a) logits[e * A + a] = (legal && !legal[e * A + a]) ? -INFINITY : z;
-      }
-    pv = warp_sum(pv);
-    if (lane == 0) values[e] = pv + bc3[0];
-  }
+  return t;
 }
 
-// launch shape of a row-wise kernel: 256 threads, x over a row's `quads` four-column groups
-// (rounded up to a warp), y over rows; at most 65535 row blocks (the kernels stride)
-struct RowsLaunch {
-  dim3 grid, block;
-};
-RowsLaunch rows_launch(int quads, int64_t n, int rows_per_thread) {
-  const int bx = std::min(256, (quads + 31) / 32 * 32), by = 256 / bx;
-  const int64_t per_block = (int64_t)by * rows_per_thread;
-  return {dim3((unsigned)((quads + bx - 1) / bx), (unsigned)std::min<int64_t>((n + per_block - 1) / per_block, 65535)),
-          dim3((unsigned)bx, (unsigned)by)};
-}
-template <typename... KArgs, typename... Args>
-void launch_rows(void (*kernel)(KArgs...), int quads, int64_t n, cudaStream_t st, Args... args) {
-  const RowsLaunch L = rows_launch(quads, n, (void*)kernel == (void*)bias_act_split ? kRowsPerThread : 1);
-  kernel<<<L.grid, L.block, 0, st>>>(args...);
-}
-
-
-// C[n][O] = X[n][I] W^T for row-major X (ld ldx), W [O][I] (ld I), C (ld ldc); `batch`
-// products at once, the b-th at W + b sW, X + b sX, C + b sC
-cublasStatus_t gemm_bf16(cublasHandle_t h, int64_t n, int O, int I, const __nv_bfloat16* W,
-                         const __nv_bfloat16* X, int ldx, float* Cm, int ldc, int batch = 1,
-                         int64_t sW = 0, int64_t sX = 0, int64_t sC = 0) {
-  const float one = 1.0f, zero = 0.0f;
-  if (batch == 1)
-    return cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, O, (int)n, I, &one, W, CUDA_R_16BF, I, X, CUDA_R_16BF,
-                        ldx, &zero, Cm, CUDA_R_32F, ldc, CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
-  return cublasGemmStridedBatchedEx(h, CUBLAS_OP_T, CUBLAS_OP_N, O, (int)n, I, &one, W, CUDA_R_16BF, I, sW,
-                                    X, CUDA_R_16BF, ldx, sX, &zero, Cm, CUDA_R_32F, ldc, sC, batch,
-                                    CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
+aht_status run_gemm(aht_s5* s, const s5g::GemmArgs& g0, int64_t n) {
+  s5g::GemmArgs g = g0;
+  g.n = n;
+  g.m_tiles = (int)((n + s5g::kBM - 1) / s5g::kBM);
+  g.status = s->status;
+  const int tiles = g.m_tiles * g.n_tiles * g.batch;
+  const int grid = std::min(tiles, s->n_sms);
+  const size_t smem = s5g::gemm_smem_bytes(g.BN);
+  if (g.epi == s5g::kHeads && (g.n_out[0] > 8 || g.n_out[1] > 8))
+    s5g::gemm_kernel<s5g::kMaxOut><<<grid, s5g::kThreads, smem, s->stream>>>(g);
+  else
+    s5g::gemm_kernel<8><<<grid, s5g::kThreads, smem, s->stream>>>(g);
+  S5_CUDA(cudaGetLastError());
+  return AHT_OK;
 }
 
 }  // namespace
@@ -294,9 +162,10 @@ aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_st
   if (!out) return set_last_error(AHT_EINVAL, "out is NULL");
   *out = nullptr;
   if (!p) return set_last_error(AHT_EINVAL, "params is NULL");
-  if (p->obs_dim < 1 || p->n_actions < 1 || p->n_actions > 32 || p->H < 16 || p->H % 16 || p->P < 16 ||
-      p->P % 16 || p->F < 16 || p->F % 16)
-    return set_last_error(AHT_EINVAL, "S5 sizes: obs_dim >= 1, 1 <= n_actions <= 32, H, P, F multiples of 16");
+  if (p->obs_dim < 1 || p->obs_dim > 2048 || p->n_actions < 1 || p->n_actions > 32 || p->H < 32 ||
+      p->H % 32 || p->P < 32 || p->P % 32 || p->P > 128 || p->F < 32 || p->F % 32)
+    return set_last_error(AHT_EINVAL,
+                          "S5 sizes: 1 <= obs_dim <= 2048, 1 <= n_actions <= 32, H, P, F multiples of 32, P <= 128");
   if (max_envs < 1 || max_envs > (1 << 20)) return set_last_error(AHT_EINVAL, "max_envs must be in 1..2^20");
   const float* req[] = {p->We1, p->be1, p->We2, p->be2, p->lam_re, p->lam_im, p->log_dt, p->B_re,
                         p->B_im, p->C_re, p->C_im, p->D};
@@ -310,10 +179,12 @@ aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_st
   aht_s5* s = new aht_s5();
   const int K = p->obs_dim, A = p->n_actions, H = p->H, P = p->P, F = p->F;
   s->K = K; s->A = A; s->H = H; s->P = P; s->F = F;
-  s->Kp = (K + 15) / 16 * 16;
+  s->K0 = (K + 63) / 64 * 64;
   s->max_n = max_envs;
+  s->m_tiles = (int)((max_envs + s5g::kBM - 1) / s5g::kBM);
   s->stream = static_cast<cudaStream_t>(cuda_stream);
   cudaGetDevice(&s->device);
+  cudaDeviceGetAttribute(&s->n_sms, cudaDevAttrMultiProcessorCount, s->device);
   auto bail = [&](aht_status st, const char* msg) {
     aht_s5_destroy(s);
     return set_last_error(st, msg);
@@ -326,17 +197,33 @@ aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_st
     s->owned.push_back(*ptr);
     return true;
   };
-  auto up16 = [&](__nv_bfloat16** dst, const std::vector<const float*>& parts, const std::vector<size_t>& counts) {
-    size_t total = 0;
-    for (size_t c : counts) total += c;
-    std::vector<__nv_bfloat16> h(total);
-    size_t o = 0;
-    for (size_t k = 0; k < parts.size(); ++k)
-      for (size_t i = 0; i < counts[k]; ++i) h[o++] = __float2bfloat16_rn(parts[k][i]);
-    return alloc((void**)dst, total * 2) && cudaMemcpy(*dst, h.data(), total * 2, cudaMemcpyHostToDevice) == cudaSuccess;
+  auto up = [&](void** dst, const void* h, size_t bytes) {
+    return alloc(dst, bytes) && cudaMemcpy(*dst, h, bytes, cudaMemcpyHostToDevice) == cudaSuccess;
   };
-  auto up32 = [&](float** dst, const std::vector<float>& h) {
-    return alloc((void**)dst, h.size() * 4) && cudaMemcpy(*dst, h.data(), h.size() * 4, cudaMemcpyHostToDevice) == cudaSuccess;
+  auto bf = [](float x) { return __float2bfloat16_rn(x); };
+  // a tiled GEMM operand from an fp32 matrix [rows][cols] given by parts of columns:
+  // each part (pointer, its column count, 0: as is, 1: its bf16 remainder w - bf16(w))
+  struct Part { const float* w; int cols; int lo; };
+  auto tiles_of = [&](int rows, const std::vector<Part>& parts, int row_stride_of_parts) {
+    int cols = 0;
+    for (const Part& q : parts) cols += q.cols;
+    std::vector<__nv_bfloat16> m((size_t)rows * cols);
+    for (int r = 0; r < rows; ++r) {
+      int c0 = 0;
+      for (const Part& q : parts) {
+        for (int c = 0; c < q.cols; ++c) {
+          const float x = q.w[(size_t)r * row_stride_of_parts + c];
+          const __nv_bfloat16 hi = bf(x);
+          m[(size_t)r * cols + c0 + c] = q.lo ? bf(x - __bfloat162float(hi)) : hi;
+        }
+        c0 += q.cols;
+      }
+    }
+    return tile_matrix(m, rows, cols, bn_for(rows));
+  };
+  auto up_tiled = [&](uint8_t** dst, int rows, const std::vector<Part>& parts, int row_stride_of_parts) {
+    const std::vector<__nv_bfloat16> t = tiles_of(rows, parts, row_stride_of_parts);
+    return up((void**)dst, t.data(), t.size() * 2);
   };
   auto vec = [](const float* a, size_t n) { return std::vector<float>(a, a + n); };
   auto bf16_rounded = [](const float* a, size_t n) {
@@ -348,27 +235,34 @@ aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_st
     a.insert(a.end(), b.begin(), b.end());
     return a;
   };
-  // [W | W] rows: each of `rows` rows of every part written twice
-  auto up16x2 = [&](__nv_bfloat16** dst, const std::vector<const float*>& parts, size_t rows, size_t cols) {
-    std::vector<__nv_bfloat16> h(parts.size() * rows * 2 * cols);
-    size_t o = 0;
-    for (const float* w : parts)
-      for (size_t r = 0; r < rows; ++r)
-        for (int rep = 0; rep < 2; ++rep)
-          for (size_t c = 0; c < cols; ++c) h[o++] = __float2bfloat16_rn(w[r * cols + c]);
-    return alloc((void**)dst, h.size() * 2) && cudaMemcpy(*dst, h.data(), h.size() * 2, cudaMemcpyHostToDevice) == cudaSuccess;
+  auto up32 = [&](float** dst, const std::vector<float>& h) { return up((void**)dst, h.data(), h.size() * 4); };
+  // heads: actor rows, then critic rows, of one layer [F][I] as one matrix [2F][I]
+  auto stack = [](const float* a, const float* c, size_t n) {
+    std::vector<float> v(a, a + n);
+    v.insert(v.end(), c, c + n);
+    return v;
   };
-  std::vector<float> We1p((size_t)H * s->Kp, 0.0f);
-  for (int h = 0; h < H; ++h) std::copy(p->We1 + (size_t)h * K, p->We1 + (size_t)(h + 1) * K, We1p.begin() + (size_t)h * s->Kp);
-  bool ok = up16(&s->We1, {We1p.data()}, {We1p.size()}) && up16x2(&s->We2, {p->We2}, H, H) &&
-            up16x2(&s->Wh0, {p->Wa[0], p->Wc[0]}, F, H) && up16x2(&s->Wh1, {p->Wa[1], p->Wc[1]}, F, F) &&
-            up16x2(&s->Wh2, {p->Wa[2], p->Wc[2]}, F, F) &&
-            up32(&s->W3, cat(bf16_rounded(p->Wa[3], (size_t)A * F), bf16_rounded(p->Wc[3], F))) &&
-            up32(&s->be1, vec(p->be1, H)) && up32(&s->be2, vec(p->be2, H)) &&
-            up32(&s->bh0, cat(vec(p->ba[0], F), vec(p->bc[0], F))) &&
-            up32(&s->bh1, cat(vec(p->ba[1], F), vec(p->bc[1], F))) &&
-            up32(&s->bh2, cat(vec(p->ba[2], F), vec(p->bc[2], F))) && up32(&s->ba3, vec(p->ba[3], A)) &&
-            up32(&s->bc3, vec(p->bc[3], 1)) && up32(&s->Dv, vec(p->D, H));
+  const std::vector<float> h0 = stack(p->Wa[0], p->Wc[0], (size_t)F * H);
+  bool ok = up_tiled(&s->We1, H, {{p->We1, K, 0}}, K) &&
+            up_tiled(&s->We2, H, {{p->We2, H, 0}, {p->We2, H, 0}}, H) &&
+            up_tiled(&s->Wh0, 2 * F, {{h0.data(), H, 0}, {h0.data(), H, 0}}, H);
+  // the two heads' layers 1 and 2, each a two-member batch: actor tiles, then critic's
+  for (int l = 1; ok && l <= 2; ++l) {
+    std::vector<__nv_bfloat16> both;
+    for (int h = 0; h < 2; ++h) {
+      const float* w = h ? p->Wc[l] : p->Wa[l];
+      const std::vector<__nv_bfloat16> t = tiles_of(F, {{w, F, 0}, {w, F, 0}}, F);
+      both.insert(both.end(), t.begin(), t.end());
+    }
+    ok = up((void**)(l == 1 ? &s->Wh1 : &s->Wh2), both.data(), both.size() * 2);
+  }
+  if (!ok) return bail(AHT_ENOMEM, "S5 weight upload failed");
+  ok = up32(&s->W3a, bf16_rounded(p->Wa[3], (size_t)A * F)) && up32(&s->W3c, bf16_rounded(p->Wc[3], F)) &&
+       up32(&s->be1, vec(p->be1, H)) && up32(&s->be2, vec(p->be2, H)) &&
+       up32(&s->bh0, cat(vec(p->ba[0], F), vec(p->bc[0], F))) &&
+       up32(&s->bh1, cat(vec(p->ba[1], F), vec(p->bc[1], F))) &&
+       up32(&s->bh2, cat(vec(p->ba[2], F), vec(p->bc[2], F))) && up32(&s->ba3, vec(p->ba[3], A)) &&
+       up32(&s->bc3, vec(p->bc[3], 1)) && up32(&s->Dv, vec(p->D, H));
   if (!ok) return bail(AHT_ENOMEM, "S5 weight upload failed");
   // zero-order hold in fp64
   std::vector<float> lbar(2 * P), Bbar((size_t)2 * P * H), Cc((size_t)H * 2 * P);
@@ -389,31 +283,32 @@ aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_st
       Cc[(size_t)h * 2 * P + q] = p->C_re[(size_t)h * P + q];
       Cc[(size_t)h * 2 * P + P + q] = -p->C_im[(size_t)h * P + q];
     }
-  // three-term bf16 rows [Wh | Wh | Wl] of an fp32 matrix [rows][cols]
-  auto up_three = [&](__nv_bfloat16** dst, const std::vector<float>& w, size_t rows, size_t cols) {
-    std::vector<__nv_bfloat16> h(rows * 3 * cols);
-    for (size_t r = 0; r < rows; ++r)
-      for (size_t c = 0; c < cols; ++c) {
-        const float x = w[r * cols + c];
-        const __nv_bfloat16 hi = __float2bfloat16_rn(x);
-        h[r * 3 * cols + c] = hi;
-        h[r * 3 * cols + cols + c] = hi;
-        h[r * 3 * cols + 2 * cols + c] = __float2bfloat16_rn(x - __bfloat162float(hi));
-      }
-    return alloc((void**)dst, h.size() * 2) && cudaMemcpy(*dst, h.data(), h.size() * 2, cudaMemcpyHostToDevice) == cudaSuccess;
-  };
-  if (!up32(&s->lbar, lbar) || !up_three(&s->Bbar3, Bbar, 2 * P, H) || !up_three(&s->Cc3, Cc, H, 2 * P))
+  // three-term rows [Wh | Wh | Wl] of the SSM's fp32 matrices
+  if (!up32(&s->lbar, lbar) ||
+      !up_tiled(&s->Bbar3, 2 * P, {{Bbar.data(), H, 0}, {Bbar.data(), H, 0}, {Bbar.data(), H, 1}}, H) ||
+      !up_tiled(&s->Cc3, H, {{Cc.data(), 2 * P, 0}, {Cc.data(), 2 * P, 0}, {Cc.data(), 2 * P, 1}}, 2 * P))
     return bail(AHT_ENOMEM, "S5 upload failed");
-  const int64_t n = max_envs;
-  ok = alloc((void**)&s->x16, (size_t)n * s->Kp * 2) && alloc((void**)&s->act, (size_t)n * std::max({4 * F, 3 * H, 6 * P}) * 2) &&
-       alloc((void**)&s->acc, (size_t)n * std::max(2 * F, H) * 4) && alloc((void**)&s->u, (size_t)n * H * 4) &&
-       alloc((void**)&s->bu, (size_t)n * 2 * P * 4) && alloc((void**)&s->y, (size_t)n * H * 4) &&
-       alloc(&s->workspace, kWorkspace);
-  if (!ok) return bail(AHT_ENOMEM, "S5 scratch allocation failed");
-  if (cublasCreate(&s->blas) != CUBLAS_STATUS_SUCCESS || cublasSetStream(s->blas, s->stream) != CUBLAS_STATUS_SUCCESS ||
-      cublasSetWorkspace(s->blas, s->workspace, kWorkspace) != CUBLAS_STATUS_SUCCESS ||
-      cublasSetMathMode(s->blas, CUBLAS_DEFAULT_MATH) != CUBLAS_STATUS_SUCCESS)
-    return bail(AHT_ECUDA, "cuBLAS set-up failed");
+  // scratch: tiled activations, zeroed once (their padding columns are never written)
+  const int64_t rows = (int64_t)s->m_tiles * s5g::kBM;
+  auto kp = [](int k) { return (size_t)((k + 63) / 64 * 64); };
+  struct Act { uint8_t** p; size_t bytes; };
+  const Act acts[] = {{&s->x0, rows * kp(K) * 2},      {&s->a1, rows * kp(2 * H) * 2},
+                      {&s->a2, rows * kp(3 * H) * 2},  {&s->a3, rows * kp(6 * P) * 2},
+                      {&s->a4, rows * kp(2 * H) * 2},  {&s->a5, 2 * rows * kp(2 * F) * 2},
+                      {&s->a6, 2 * rows * kp(2 * F) * 2}};
+  for (const Act& x : acts)
+    if (!alloc((void**)x.p, x.bytes) || cudaMemset(*x.p, 0, x.bytes) != cudaSuccess)
+      return bail(AHT_ENOMEM, "S5 scratch allocation failed");
+  const int n_tiles_f = F / bn_for(F);
+  if (!alloc((void**)&s->u, (size_t)rows * H * 4) ||
+      !alloc((void**)&s->partial, (size_t)rows * 2 * n_tiles_f * 2 * s5g::kMaxOut * 4) ||
+      !alloc((void**)&s->status, 4) || cudaMemset(s->status, 0, 4) != cudaSuccess)
+    return bail(AHT_ENOMEM, "S5 scratch allocation failed");
+  if (cudaFuncSetAttribute(s5g::gemm_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)s5g::gemm_smem_bytes(256)) != cudaSuccess ||
+      cudaFuncSetAttribute(s5g::gemm_kernel<s5g::kMaxOut>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)s5g::gemm_smem_bytes(256)) != cudaSuccess)
+    return bail(AHT_ECUDA, "setting the GEMM's shared-memory limit failed");
   *out = s;
   return AHT_OK;
 }
@@ -421,7 +316,6 @@ aht_status aht_s5_create(const aht_s5_params* p, int64_t max_envs, void* cuda_st
 void aht_s5_destroy(aht_s5* s) {
   if (!s) return;
   S5DeviceGuard g(s->device);
-  if (s->blas) cublasDestroy(s->blas);
   for (void* q : s->owned) cudaFree(q);
   delete s;
 }
@@ -430,40 +324,64 @@ aht_status aht_s5_step(aht_s5* s, const uint8_t* obs, const uint8_t* reset, cons
                        int64_t n, float* state, float* logits, float* values) {
   if (!s || !obs || !reset || !state || !logits || !values) return set_last_error(AHT_EINVAL, "NULL argument");
   if (n < 1 || n > s->max_n) return set_last_error(AHT_EINVAL, "n must be in 1..max_envs");
-  S5DeviceGuard g(s->device);
+  S5DeviceGuard dg(s->device);
   const int K = s->K, A = s->A, H = s->H, P = s->P, F = s->F;
-  cudaStream_t st = s->stream;
-  cublasHandle_t b = s->blas;
-  // encoder: the observation is exact in bf16, so layer 1 is one plain product; later
-  // layers take [hi | lo] against [W | W], one product with fp32 accumulation
-  launch_rows(u8_to_bf16, s->Kp / 4, n, st, obs, s->x16, K, s->Kp, n);
-  S5_BLAS(gemm_bf16(b, n, H, s->Kp, s->We1, s->x16, s->Kp, s->acc, H));
-  launch_rows(bias_act_split, H / 4, n, st, s->acc, s->be1, H, 1, n, true, (float*)nullptr, s->act, 2);
-  S5_BLAS(gemm_bf16(b, n, H, 2 * H, s->We2, s->act, 2 * H, s->acc, H));
-  launch_rows(bias_act_split, H / 4, n, st, s->acc, s->be2, H, 1, n, true, s->u, s->act, 3);
-  // SSM: Bbar u and Re(C x) as three-term bf16 products, the recurrence in fp32
-  S5_BLAS(gemm_bf16(b, n, 2 * P, 3 * H, s->Bbar3, s->act, 3 * H, s->bu, 2 * P));
-  launch_rows(ssm_recur, P / 4, n, st, s->lbar, s->bu, reset, state, P, n, s->act);
-  S5_BLAS(gemm_bf16(b, n, H, 6 * P, s->Cc3, s->act, 6 * P, s->y, H));
-  launch_rows(residual_gelu, H / 4, n, st, s->y, s->u, s->Dv, H, n, s->act);
-  // heads: layer 0 for both heads at once ([2F] outputs, split as 2 groups of F), layers
-  // 1-2 as one two-member batch (head h reads group h, writes columns h F of acc)
-  S5_BLAS(gemm_bf16(b, n, 2 * F, 2 * H, s->Wh0, s->act, 2 * H, s->acc, 2 * F));
-  launch_rows(bias_act_split, 2 * F / 4, n, st, s->acc, s->bh0, F, 2, n, true, (float*)nullptr, s->act, 2);
-  const __nv_bfloat16* Wl[2] = {s->Wh1, s->Wh2};
-  const float* bl[2] = {s->bh1, s->bh2};
-  for (int l = 0; l < 2; ++l) {
-    S5_BLAS(gemm_bf16(b, n, F, 2 * F, Wl[l], s->act, 4 * F, s->acc, 2 * F, 2, (int64_t)F * 2 * F, 2 * F, F));
-    if (l == 0) launch_rows(bias_act_split, 2 * F / 4, n, st, s->acc, bl[l], F, 2, n, true, (float*)nullptr, s->act, 2);
+  const int64_t rows = (int64_t)s->m_tiles * s5g::kBM;
+  auto kt = [](int k) { return (k + 63) / 64; };
+  // the observation -> tiled bf16
+  {
+    const int bx = s->K0 / 8, by = std::max(1, 256 / bx);  // K0 <= 2048 keeps bx <= 256
+    const int64_t blocks = std::min<int64_t>((n + by - 1) / by, 65535);
+    obs_tiles<<<(unsigned)blocks, dim3((unsigned)bx, (unsigned)by), 0, s->stream>>>(obs, K, s->K0, n, s->x0);
+    S5_CUDA(cudaGetLastError());
   }
-  // layer 2's bias and relu, and both output layers, in fp32 (one warp per env)
-  const int out_blocks = (int)std::min<int64_t>((n + 7) / 8, 65535);
-  if (A <= 8)
-    heads_out<8><<<out_blocks, 256, 0, st>>>(s->acc, s->bh2, s->W3, s->ba3, s->bc3, legal, A, F, n, logits, values);
-  else if (A <= 16)
-    heads_out<16><<<out_blocks, 256, 0, st>>>(s->acc, s->bh2, s->W3, s->ba3, s->bc3, legal, A, F, n, logits, values);
-  else
-    heads_out<32><<<out_blocks, 256, 0, st>>>(s->acc, s->bh2, s->W3, s->ba3, s->bc3, legal, A, F, n, logits, values);
+  auto layer = [&](const uint8_t* A_, int k_in, const uint8_t* B_, int N, int epi) {
+    s5g::GemmArgs g{};
+    g.A = A_;
+    g.B = B_;
+    g.k_tiles = kt(k_in);
+    g.BN = bn_for(N);
+    g.n_tiles = N / g.BN;
+    g.batch = 1;
+    g.epi = epi;
+    return g;
+  };
+  // encoder layer 1 (exact bf16 observation): relu, hi | lo
+  s5g::GemmArgs g = layer(s->x0, K, s->We1, H, s5g::kSplit);
+  g.bias = s->be1; g.relu = 1; g.parts = 2; g.I = H; g.out = s->a1; g.out_k_tiles = kt(2 * H);
+  if (aht_status e = run_gemm(s, g, n)) return e;
+  // encoder layer 2: relu; u (fp32) and its hi | lo | hi for the three-term SSM product
+  g = layer(s->a1, 2 * H, s->We2, H, s5g::kSplit);
+  g.bias = s->be2; g.relu = 1; g.parts = 3; g.I = H; g.out = s->a2; g.out_k_tiles = kt(3 * H); g.out32 = s->u;
+  if (aht_status e = run_gemm(s, g, n)) return e;
+  // SSM: Bbar u, the recurrence and x's hi | lo | hi
+  g = layer(s->a2, 3 * H, s->Bbar3, 2 * P, s5g::kSsm);
+  g.lbar = s->lbar; g.state = state; g.reset = reset; g.P = P; g.out = s->a3; g.out_k_tiles = kt(6 * P);
+  if (aht_status e = run_gemm(s, g, n)) return e;
+  // Re(C x), then v = u + gelu(y + D u) as hi | lo
+  g = layer(s->a3, 6 * P, s->Cc3, H, s5g::kGelu);
+  g.u = s->u; g.D = s->Dv; g.I = H; g.out = s->a4; g.out_k_tiles = kt(2 * H);
+  if (aht_status e = run_gemm(s, g, n)) return e;
+  // heads layer 0, both heads at once: relu, hi | lo of each head's F units
+  const int64_t head_act = rows * kt(2 * F) * 64 * 2;  // bytes of one head's activation
+  g = layer(s->a4, 2 * H, s->Wh0, 2 * F, s5g::kSplit);
+  g.bias = s->bh0; g.relu = 1; g.parts = 2; g.I = F; g.out = s->a5; g.out_stride = head_act;
+  g.out_k_tiles = kt(2 * F);
+  if (aht_status e = run_gemm(s, g, n)) return e;
+  // heads layer 1 (two-member batch)
+  const int64_t wh_bytes = (int64_t)F * 2 * F * 2;
+  g = layer(s->a5, 2 * F, s->Wh1, F, s5g::kSplit);
+  g.batch = 2; g.a_stride = head_act; g.b_stride = wh_bytes;
+  g.bias = s->bh1; g.relu = 1; g.parts = 2; g.I = F; g.out = s->a6; g.out_stride = head_act;
+  g.out_k_tiles = kt(2 * F);
+  if (aht_status e = run_gemm(s, g, n)) return e;
+  // heads layer 2 with both output layers: per-tile partial sums
+  g = layer(s->a6, 2 * F, s->Wh2, F, s5g::kHeads);
+  g.batch = 2; g.a_stride = head_act; g.b_stride = wh_bytes;
+  g.bias = s->bh2; g.W3[0] = s->W3a; g.W3[1] = s->W3c; g.n_out[0] = A; g.n_out[1] = 1; g.partial = s->partial;
+  if (aht_status e = run_gemm(s, g, n)) return e;
+  heads_final<<<(unsigned)((n + 255) / 256), 256, 0, s->stream>>>(s->partial, F / bn_for(F), A > 8 ? s5g::kMaxOut : 8,
+                                                                  s->ba3, s->bc3, legal, A, n, logits, values);
   S5_CUDA(cudaGetLastError());
   return AHT_OK;
 }
@@ -472,6 +390,12 @@ aht_status aht_s5_sync(aht_s5* s) {
   if (!s) return set_last_error(AHT_EINVAL, "NULL argument");
   S5DeviceGuard g(s->device);
   S5_CUDA(cudaStreamSynchronize(s->stream));
+  uint32_t st = 0;
+  S5_CUDA(cudaMemcpy(&st, s->status, 4, cudaMemcpyDeviceToHost));
+  if (st) {
+    cudaMemset(s->status, 0, 4);
+    return set_last_error(AHT_ETIMEOUT, "an S5 GEMM's bounded wait expired");
+  }
   return AHT_OK;
 }
 

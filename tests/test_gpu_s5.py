@@ -64,9 +64,9 @@ def test_s5_steps_match_the_oracle(N, T):
 
 
 @pytest.mark.parametrize("K,A,H,P,F,N,max_envs,masked", [
-    (100, 20, 32, 16, 64, 77, 128, True),     # 9-16 actions; fewer envs than max_envs
-    (37, 32, 16, 32, 48, 5, 5, False),        # 32 actions, no mask; F / 4 < 32 lanes
-    (10, 1, 16, 16, 16, 33, 40, True),        # one action
+    (100, 20, 64, 32, 64, 77, 128, True),     # 20 actions; fewer envs than max_envs
+    (37, 32, 32, 96, 288, 5, 5, False),       # 32 actions, no mask; 3 n-tiles of 96 per head
+    (10, 1, 32, 32, 32, 300, 300, True),      # one action; 3 row tiles, the last ragged
 ])
 def test_s5_other_shapes(K, A, H, P, F, N, max_envs, masked):
     """Action counts on each register width of the output kernel, the unmasked path,
@@ -105,7 +105,7 @@ def test_s5_other_shapes(K, A, H, P, F, N, max_envs, masked):
 
 def test_s5_rejects_bad_sizes():
     require_gpu()
-    params = W.s5_params(1, 196, 6, H=16, P=16, F=32)
+    params = W.s5_params(1, 196, 6, H=32, P=32, F=32)
     bad = dict(params)
     bad["lam_re"] = -bad["lam_re"]          # growing modes
     with pytest.raises(aht.AhtError):
@@ -114,5 +114,5 @@ def test_s5_rejects_bad_sizes():
     obs = torch.zeros(9, 196, dtype=torch.uint8, device="cuda")
     with pytest.raises(aht.AhtError):       # more envs than max_envs
         aht.aht_s5_step(pol, obs, torch.zeros(9, dtype=torch.uint8, device="cuda"),
-                        torch.zeros(9, 32, device="cuda"), torch.empty(9, 6, device="cuda"),
+                        torch.zeros(9, 64, device="cuda"), torch.empty(9, 6, device="cuda"),
                         torch.empty(9, device="cuda"))
