@@ -223,8 +223,8 @@ class ClockSampler:
 
 
 # the sources the fused rollout kernel is compiled from
-ROLLOUT_SOURCES = ("rollout_tc.cuh", "tc_common.cuh", "env_lbf.cuh", "aht_common.cuh", "mlp_simt.cuh",
-                   "rollout_impl.cuh", "kernels.h", "rollout_lbf.cu")
+ROLLOUT_SOURCES = ("rollout_tc2.cuh", "rollout_tc.cuh", "tc_common.cuh", "env_lbf.cuh", "aht_common.cuh",
+                   "mlp_simt.cuh", "rollout_impl.cuh", "kernels.h", "rollout_lbf.cu", "rollout_lbf2.cu")
 
 
 def csrc_hash():
@@ -382,7 +382,7 @@ def run_ours(args):
     kern_ms = kernel_ms / max(1, kernel_launches)
     achieved_tflops = flops_launch / (kern_ms * 1e-3) / 1e12
     achieved_gbs = env_steps * bytes_per_env_step / (kern_ms * 1e-3) / 1e9
-    traffic = recorded_traffic("ppo_tc_kernel")
+    traffic = recorded_traffic("ppo2_tc_kernel")
 
     line = None
     if rank == 0:
@@ -399,7 +399,7 @@ def run_ours(args):
                        "parallelism": f"{world} independent replicas" if world > 1 else "1 GPU"},
             "roofline": {"bound": "tensor", "achieved": achieved_tflops, "peak": bf16_peak,
                          "unit": "TFLOP/s", "frac": achieved_tflops / bf16_peak,
-                         "traffic": traffic, "kernel": "ppo_tc_kernel<EnvLbf>",
+                         "traffic": traffic, "kernel": "ppo2_tc_kernel<EnvLbf, bf16, gathered tiles>",
                          "kernel_ms": kern_ms, "flops_per_launch": flops_launch,
                          "peak_source": f"{peak_src} bf16 burst",
                          "frac_of_sustained": achieved_tflops / bf16_sustained,
