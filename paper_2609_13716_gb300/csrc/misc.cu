@@ -138,32 +138,51 @@ cudaError_t launch_resample_group(const ResampleGroupArgs& a, cudaStream_t s) {
 }
 
 // ---- GAE: one thread per env, reverse scan over T (time-major, coalesced across envs) --
-__global__ void gae_kernel(const float* __restrict__ r, const float* __restrict__ v,
-                           const uint8_t* __restrict__ d, const float* __restrict__ v_last,
-                           int64_t n, int32_t T, float gamma, float lambda,
-                           float* __restrict__ adv, float* __restrict__ tgt) {
+// The scan carries only two floats from step to step, so each thread loads the rewards,
+// values and done flags of kGaeChunk steps at once (independent loads in flight together)
+// and then runs the recurrence over them in the same order as a step-by-step scan.
+constexpr int kGaeChunk = 16;
+
+__global__ void __launch_bounds__(128) gae_kernel(const float* __restrict__ r, const float* __restrict__ v,
+                                                  const uint8_t* __restrict__ d, const float* __restrict__ v_last,
+                                                  int64_t n, int32_t T, float gamma, float lambda,
+                                                  float* __restrict__ adv, float* __restrict__ tgt) {
   const int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (e >= n) return;
   float next_v = v_last[e];
   float next_a = 0.0f;
   const float gl = gamma * lambda;
-  for (int t = T - 1; t >= 0; --t) {
-    const int64_t i = (int64_t)t * n + e;
-    const float vt = v[i];
-    const float nonterminal = d[i] ? 0.0f : 1.0f;
-    const float delta = r[i] + gamma * nonterminal * next_v - vt;
-    const float at = delta + gl * nonterminal * next_a;
-    adv[i] = at;
-    if (tgt) tgt[i] = at + vt;
-    next_a = at;
-    next_v = vt;
+  for (int t0 = T - 1; t0 >= 0; t0 -= kGaeChunk) {
+    const int c = t0 + 1 < kGaeChunk ? t0 + 1 : kGaeChunk;  // steps t0, t0 - 1, ..., t0 - c + 1
+    float rv[kGaeChunk], vv[kGaeChunk];
+    uint8_t dv[kGaeChunk];
+#pragma unroll
+    for (int j = 0; j < kGaeChunk; ++j)
+      if (j < c) {
+        const int64_t i = (int64_t)(t0 - j) * n + e;
+        rv[j] = r[i];
+        vv[j] = v[i];
+        dv[j] = d[i];
+      }
+#pragma unroll
+    for (int j = 0; j < kGaeChunk; ++j)
+      if (j < c) {
+        const int64_t i = (int64_t)(t0 - j) * n + e;
+        const float nonterminal = dv[j] ? 0.0f : 1.0f;
+        const float delta = rv[j] + gamma * nonterminal * next_v - vv[j];
+        const float at = delta + gl * nonterminal * next_a;
+        adv[i] = at;
+        if (tgt) tgt[i] = at + vv[j];
+        next_a = at;
+        next_v = vv[j];
+      }
   }
 }
 
 cudaError_t launch_gae(const float* r, const float* v, const uint8_t* d, const float* v_last,
                        int64_t n, int32_t T, float gamma, float lambda, float* adv, float* tgt,
                        cudaStream_t s) {
-  const int threads = 256;
+  const int threads = 128;  // 16384 envs -> 128 CTAs, spread over the SMs
   const int blocks = (int)((n + threads - 1) / threads);
   gae_kernel<<<blocks, threads, 0, s>>>(r, v, d, v_last, n, T, gamma, lambda, adv, tgt);
   return cudaGetLastError();
