@@ -1103,6 +1103,7 @@ aht_status aht_rollout_resample(aht_ctx* c, int32_t ego_id, const int32_t* pool,
       ta.dbg_logits = dbg ? dbg + o * 2 * kDbgStride : nullptr;  // this step's slice
       ta.dbg_expire_step = t == expire_step ? 0 : -1;             // this launch's step 0
       ta.dbg_expire_ns = expire_ns;
+      ta.pdl = t > 0;  // step 0 follows the grouping launch in plain stream order
       const int tk = timer_begin(c);
       AHT_CUDA(lbf_ppo_tc(ta, resample_tiles(N, 128, pool_size), smem, c->stream));
       timer_end(c, tk);

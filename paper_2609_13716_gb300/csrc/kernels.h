@@ -123,6 +123,8 @@ struct PpoTcArgs {
   float* dbg_logits;     // test hook, or NULL: [steps][rows][2 seats][kDbgStride] outputs
   int32_t dbg_expire_step;   // test hook: at this step the compute threads wait, bounded by
   uint64_t dbg_expire_ns;    // dbg_expire_ns, on an mbarrier nothing arrives on (-1: never)
+  int32_t pdl;               // launch as a programmatic dependent of the stream's previous
+                             // kernel (the two-group kernel only; its setup overlaps that kernel)
 };
 
 // Per-policy block of the streamed tensor-core path (binary observations, hidden width H

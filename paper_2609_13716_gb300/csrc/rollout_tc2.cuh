@@ -43,15 +43,51 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
   __shared__ __align__(8) uint64_t rows_ready;     // ego rows built (256; gathered copy)
   __shared__ __align__(8) uint64_t never_bar;      // test hook: nothing arrives on it
   __shared__ uint32_t tmem_slot;
+  const TcDims& d = a.tc;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, row = tid & 127;
+
+  // A per-episode call launches its steps after the first as programmatic dependents of
+  // the step before: everything up to griddepcontrol.wait touches nothing that step
+  // writes -- the barriers, tensor memory and the ego's weights (the ego is the same for
+  // the whole call).  (Without that launch attribute the wait returns at once.)
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  if (tid == 0) {
+    for (int i = 0; i < 4; ++i) tc::mbar_init(&acc_bar[i], 1);
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&wload_bar[i], 1);
+      tc::mbar_init(&drain_bar[i], 1);
+    }
+    tc::mbar_init(&buf_free, kT2Group);
+    tc::mbar_init(&rows_ready, kT2Group);
+    tc::mbar_init(&never_bar, 1);
+    tc::mbar_init_fence();
+    // the ego's policy block -> shared memory, waited for by the ego group
+    const uint8_t* src = a.tcw + (int64_t)a.ego * d.pol_bytes;
+    tc::mbar_expect_tx(&wload_bar[0], d.pol_bytes);
+    for (uint32_t off = 0; off < d.pol_bytes; off += 32768u)
+      tc::bulk_g2s(smem + off, src + off, min(32768u, d.pol_bytes - off), &wload_bar[0]);
+  }
+  if (warp == 0) tc::tmem_alloc(&tmem_slot, 512);
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 
   int32_t* const rowenv = kGather ? reinterpret_cast<int32_t*>(smem + a.g.scratch_off) : nullptr;
   const TcTile tile = tc_find_tile<false, kGather>(a, rowenv);
   const int64_t env0 = tile.env0;
-  const int count = tile.count, ego_pol = tile.ego_pol, tm_pol = tile.tm_pol, g_k = tile.g_k;
-  if (count <= 0) return;
+  const int count = tile.count, tm_pol = tile.tm_pol, g_k = tile.g_k;
+  if (count <= 0) {  // no rows: the ego's copy lands, then tensor memory is freed
+    if (tid == 0) tc::mbar_wait(&wload_bar[0], 0);
+    tc::fence_before_sync();
+    __syncthreads();
+    if (warp == 0) {
+      tc::fence_after_sync();
+      tc::tmem_dealloc(tmem_slot, 512);
+    }
+    return;
+  }
   const bool tm_rule = tm_pol < 0;  // LBF heuristic -1 - id: no teammate network
-  const TcDims& d = a.tc;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, row = tid & 127;
   const int grp = warp >> 3;                 // 0 ego, 1 teammate
   const int half = (warp >> 2) & 1;          // which half of the agent's columns
   auto env_of = [&](int r) -> int64_t { return kGather ? (int64_t)rowenv[r] : env0 + r; };
@@ -73,18 +109,6 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
   uint8_t* act1s = reinterpret_cast<uint8_t*>(st) + align_up(128 * sizeof(State), 16);  // [128]
   float* zpart = reinterpret_cast<float*>(act1s + 128);                     // [2][2][128][8]
 
-  if (tid == 0) {
-    for (int i = 0; i < 4; ++i) tc::mbar_init(&acc_bar[i], 1);
-    for (int i = 0; i < 2; ++i) {
-      tc::mbar_init(&wload_bar[i], 1);
-      tc::mbar_init(&drain_bar[i], 1);
-    }
-    tc::mbar_init(&buf_free, kT2Group);
-    tc::mbar_init(&rows_ready, kT2Group);
-    tc::mbar_init(&never_bar, 1);
-    tc::mbar_init_fence();
-  }
-  if (warp == 0) tc::tmem_alloc(&tmem_slot, 512);
   for (int i = tid; i < 32 * od; i += blockDim.x) reinterpret_cast<uint32_t*>(sObs)[i] = 0u;
   if (tid < count) load_state(a.state, N, env_of(tid), st[tid]);
   tc::fence_before_sync();
@@ -97,9 +121,10 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
     const bool leader = (tid & (kT2Group - 1)) == 0;  // issues the group's copies and MMAs
     const bool net = ag == 0 || !tm_rule;              // the group runs a network
     bool bad = false;
-    // this agent's policy block -> shared memory (its leader), waited for by the group
-    if (leader && net) {
-      const uint8_t* src = a.tcw + (int64_t)(ag == 0 ? ego_pol : tm_pol) * d.pol_bytes;
+    // the teammate's policy block -> shared memory (its leader; the ego's is on its way),
+    // waited for by the group
+    if (leader && net && ag == 1) {
+      const uint8_t* src = a.tcw + (int64_t)tm_pol * d.pol_bytes;
       uint8_t* dst = sW0 + (size_t)ag * d.pol_bytes;
       tc::mbar_expect_tx(&wload_bar[ag], d.pol_bytes);
       for (uint32_t off = 0; off < d.pol_bytes; off += 32768u)
@@ -453,8 +478,17 @@ struct LaunchTc2 {
     cudaError_t e = cudaFuncSetAttribute(ppo2_tc_kernel<Env, kSplit, kGather>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    ppo2_tc_kernel<Env, kSplit, kGather><<<grid, kT2Threads, smem, s>>>(a);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kT2Threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = a.pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, ppo2_tc_kernel<Env, kSplit, kGather>, a);
   }
   // plain PPO collection (no IPPO, dense first layer)
   static cudaError_t ppo(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
