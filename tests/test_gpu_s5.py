@@ -116,3 +116,33 @@ def test_s5_rejects_bad_sizes():
         aht.aht_s5_step(pol, obs, torch.zeros(9, dtype=torch.uint8, device="cuda"),
                         torch.zeros(9, 64, device="cuda"), torch.empty(9, 6, device="cuda"),
                         torch.empty(9, device="cuda"))
+
+
+def test_s5_step_with_another_device_current():
+    """A policy created on GPU 0 steps, syncs and is destroyed correctly while another
+    device is current: the library makes the policy's device current for each call.
+    Needs two GPUs."""
+    require_gpu()
+    if torch.cuda.device_count() < 2:
+        pytest.skip("needs two GPUs")
+    N = 64
+    params = W.s5_params(0, 196, 6)
+    obs, resets = lbf_observations(2, N, 5)
+    legal = torch.ones(N, 6, dtype=torch.uint8, device="cuda:0")
+    out = []
+    for other in (False, True):
+        torch.cuda.set_device(0)
+        pol = aht.aht_s5_create(params, N)
+        state = torch.zeros(N, 2 * O.S5(params).P, device="cuda:0")
+        logits = torch.empty(N, 6, device="cuda:0")
+        values = torch.empty(N, device="cuda:0")
+        if other:
+            torch.cuda.set_device(1)
+        for t in range(2):
+            aht.aht_s5_step(pol, torch.from_numpy(obs[t]).to("cuda:0"), torch.from_numpy(resets[t]).to("cuda:0"),
+                            state, logits, values, legal)
+        aht.aht_s5_sync(pol)
+        pol.close()
+        torch.cuda.set_device(0)
+        out.append((logits.cpu(), values.cpu()))
+    assert torch.equal(out[0][0], out[1][0]) and torch.equal(out[0][1], out[1][1])
