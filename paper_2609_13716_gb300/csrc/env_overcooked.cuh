@@ -12,11 +12,42 @@
 
 namespace aht {
 
-// Cell types: 0 floor, 1 counter, 2 onion dispenser, 3 pot, 4 dish dispenser, 5 serving.
-__constant__ uint8_t kKitchenCell[20] = {1, 2, 1, 3, 1,   //
-                                         1, 0, 0, 0, 1,   //
-                                         4, 0, 0, 0, 5,   //
-                                         1, 1, 2, 1, 1};
+// Cell types: 0 floor, 1 counter, 2 onion dispenser, 3 pot, 4 dish dispenser, 5 serving;
+// cell c = y * 5 + x of the layout above.
+__host__ __device__ constexpr int kitchen_type(int c) {
+  return (c == 1 || c == 17) ? 2
+         : c == 3            ? 3
+         : c == 10           ? 4
+         : c == 14           ? 5
+         : (c == 6 || c == 7 || c == 8 || c == 11 || c == 12 || c == 13) ? 0
+                                                                          : 1;
+}
+// the same table in constant memory, for cells indexed at run time
+__constant__ uint8_t kKitchenCell[20] = {
+    kitchen_type(0),  kitchen_type(1),  kitchen_type(2),  kitchen_type(3),  kitchen_type(4),
+    kitchen_type(5),  kitchen_type(6),  kitchen_type(7),  kitchen_type(8),  kitchen_type(9),
+    kitchen_type(10), kitchen_type(11), kitchen_type(12), kitchen_type(13), kitchen_type(14),
+    kitchen_type(15), kitchen_type(16), kitchen_type(17), kitchen_type(18), kitchen_type(19)};
+
+// The observation bits that depend only on the layout (each cell's type channel) and on
+// the urgency flag (channel 25 of every cell), as 32-bit words (bit k % 32 of word k / 32).
+constexpr int kOcObsBits = 20 * 26;
+constexpr int kOcObsWords = (kOcObsBits + 31) / 32;
+struct OcObsMasks {
+  uint32_t layout[kOcObsWords], urgent[kOcObsWords];
+};
+__host__ __device__ constexpr int oc_type_channel(int t) {
+  return t == 1 ? 10 : t == 2 ? 12 : t == 3 ? 11 : t == 4 ? 13 : t == 5 ? 14 : -1;
+}
+__host__ __device__ constexpr OcObsMasks oc_obs_masks() {
+  OcObsMasks m{};
+  for (int c = 0; c < 20; ++c) {
+    const int ch = oc_type_channel(kitchen_type(c));
+    if (ch >= 0) m.layout[(c * 26 + ch) >> 5] |= 1u << ((c * 26 + ch) & 31);
+    m.urgent[(c * 26 + 25) >> 5] |= 1u << ((c * 26 + 25) & 31);
+  }
+  return m;
+}
 
 struct EnvOvercooked {
   static constexpr bool kTurnBased = false;
@@ -128,28 +159,20 @@ struct EnvOvercooked {
   }
 
   // 26 binary channels per cell, index (y*5 + x)*26 + c.
+  __device__ static bool urgent(const DevEnv& d, const State& s) { return d.episode_len - (int)s.ep_t <= 40; }
+  // the channels that change with the state: items on counters, the pot, the agents
   template <class Row>
-  __device__ static void obs_into(const DevEnv& d, const State& s, int seat, Row& row) {
-    row.clear();
-    const bool urgent = d.episode_len - (int)s.ep_t <= 40;
+  __device__ static void obs_state_bits(const State& s, int seat, Row& row) {
+#pragma unroll
     for (int c = 0; c < 20; ++c) {
       const int o = c * 26;
-      const int t = kKitchenCell[c];
+      const int t = kitchen_type(c);
       if (t == 1) {
-        row.set(o + 10, 1);
         if (s.item[c] != kNone) row.set(o + 14 + s.item[c], 1);
-      } else if (t == 2) {
-        row.set(o + 12, 1);
       } else if (t == 3) {
-        row.set(o + 11, 1);
         if (s.pot_n >= 1) row.set(o + 17 + s.pot_n, 1);
         if (s.pot_n == 3) row.set(o + (s.pot_timer > 0 ? 21 : 22), 1);
-      } else if (t == 4) {
-        row.set(o + 13, 1);
-      } else if (t == 5) {
-        row.set(o + 14, 1);
       }
-      if (urgent) row.set(o + 25, 1);
     }
     for (int who = 0; who < 2; ++who) {
       const int i = who == 0 ? seat : 1 - seat;
@@ -161,6 +184,27 @@ struct EnvOvercooked {
         row.set(o + 14 + s.held[i], 1);
       }
     }
+  }
+  template <class Row>
+  __device__ static void obs_into(const DevEnv& d, const State& s, int seat, Row& row) {
+    row.clear();
+    const bool urg = urgent(d, s);
+    for (int c = 0; c < 20; ++c) {
+      const int ch = oc_type_channel(kKitchenCell[c]);
+      if (ch >= 0) row.set(c * 26 + ch, 1);
+      if (urg) row.set(c * 26 + 25, 1);
+    }
+    obs_state_bits(s, seat, row);
+  }
+  // The same bits into a word row (the streamed cross-play kernel): the layout and urgency
+  // channels as whole words, then the state's channels bit by bit.
+  __device__ static void obs_into(const DevEnv& d, const State& s, int seat, ObsBits& row) {
+    constexpr OcObsMasks M = oc_obs_masks();
+    const uint32_t u = urgent(d, s) ? 0xFFFFFFFFu : 0u;
+#pragma unroll
+    for (int i = 0; i < kOcObsWords; ++i) row.w[i] = M.layout[i] | (M.urgent[i] & u);
+    for (int i = kOcObsWords; i < row.words; ++i) row.w[i] = 0u;
+    obs_state_bits(s, seat, row);
   }
   __device__ static void obs(const DevEnv& d, const State& s, int seat, uint8_t* row) {
     ObsBytes w{row, 130};

@@ -98,9 +98,11 @@ __host__ __device__ inline XpTcSmem xp_tc_layout(const WideDims& w) {
   return L;
 }
 
-// Two binary features (bits 0, 1 of x) as a bf16 pair: 0 or 1.0 (0x3F80) each.
+// Two binary features (bits 0, 1 of x) as a bf16 pair: 0 or 1.0 (0x3F80) each.  Bit 0
+// times 0x8001 stays at bit 0 and bit 1 lands on bit 16 (the mask drops the cross terms),
+// so one multiply by 0x3F80 writes both halves.
 __device__ __forceinline__ uint32_t bits_to_bf16x2(uint32_t x) {
-  return ((x & 1u) * 0x3F80u) | ((x & 2u) * 0x1FC00000u);
+  return (((x & 3u) * 0x8001u) & 0x00010001u) * 0x3F80u;
 }
 
 template <class Env>
@@ -399,14 +401,18 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
       const uint32_t* bits = sBits + row * L.bit_words;
       const int nkb = w.KP / 8, split = (nkb + 1) / 2;
       const int kb0 = half ? split : 0, kb1 = half ? nkb : split;
-      for (int kb = kb0; kb < kb1; ++kb) {
-        const uint32_t byte = (bits[kb >> 2] >> (8 * (kb & 3))) & 0xFFu;
+      // the 16-byte core-matrix rows of consecutive 8-feature blocks are 128 bytes apart
+      uint8_t* dst = sA + tc::canon_offset(row, 8 * kb0, w.KP);
+      uint32_t word = kb0 < kb1 ? bits[kb0 >> 2] : 0u;
+      for (int kb = kb0; kb < kb1; ++kb, dst += 128) {
+        if ((kb & 3) == 0) word = bits[kb >> 2];
+        const uint32_t byte = (word >> (8 * (kb & 3))) & 0xFFu;
         uint4 v;
         v.x = bits_to_bf16x2(byte);
         v.y = bits_to_bf16x2(byte >> 2);
         v.z = bits_to_bf16x2(byte >> 4);
         v.w = bits_to_bf16x2(byte >> 6);
-        *reinterpret_cast<uint4*>(sA + tc::canon_offset(row, 8 * kb, w.KP)) = v;
+        *reinterpret_cast<uint4*>(dst) = v;
       }
       tc::fence_proxy_async();
       tc::mbar_arrive(&obs_bar);
