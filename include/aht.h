@@ -181,10 +181,11 @@ aht_status aht_rollout(aht_ctx* ctx, int32_t ego_id, const int32_t* pool, int32_
  * plays pool[floor(x * pool_size / 2^32)], x the first draw of counter (e, s, stream 5);
  * the context carries per env the step its current episode began (aht_reset: 0; every
  * auto-reset at step s' -- in any collection call or aht_step_forced -- sets s'; part of
- * the checkpoint).  Each step regroups the envs by teammate (a grouping kernel, then one
- * launch of the fused rollout over the groups' tiles), so this call runs 2T launches
- * instead of 1; otherwise the step, the draws and the trajectory layout are those of
- * aht_rollout.  out->teammate receives the teammate of the call's first step; teammates
+ * the checkpoint).  Each step regroups the envs by teammate, so this call runs one launch
+ * per step instead of one per call (on the tensor-core path each step's launch groups
+ * its own rows and starts while the step before finishes; on the CUDA-core path a
+ * grouping launch precedes each step's launch); otherwise the step, the draws and the
+ * trajectory layout are those of aht_rollout.  out->teammate receives the teammate of the call's first step; teammates
  * (device int32 [T][N], or NULL) the teammate of every step.  out->obs must be 4-byte
  * aligned.  Same pool rules as aht_rollout (rule teammates on LBF tensor-core contexts). */
 aht_status aht_rollout_resample(aht_ctx* ctx, int32_t ego_id, const int32_t* pool,
@@ -516,6 +517,15 @@ aht_status aht_debug_expire_at(aht_ctx* ctx, int32_t step, int64_t limit_ns);
  * CUDA-core kernels do not write it.  buf == NULL turns the hook off. */
 #define AHT_DEBUG_STRIDE 32
 aht_status aht_debug_logits(aht_ctx* ctx, float* buf, int64_t floats);
+
+/* Parity hook (no paper counterpart): the observation rows the streamed cross-play kernel
+ * builds for Overcooked, Hanabi and Mini Hanabi contexts, for seat `seat` (0 or 1) of
+ * every env's current state (Sec. 3, Omega: each agent's observation).  out: device
+ * uint32 [n_envs][(obs_dim + 32) / 32], caller-owned; feature k of env e is bit k % 32 of
+ * out[e][k / 32], then bit obs_dim is the constant 1 input that carries layer 1's bias,
+ * and every later bit is 0.  Runs on the context's stream (aht_sync to wait).  LBF
+ * contexts: AHT_EINVAL (their observations are bytes). */
+aht_status aht_debug_obs_words(aht_ctx* ctx, int32_t seat, uint32_t* out);
 
 const char* aht_last_error(void);
 const char* aht_status_string(aht_status s);

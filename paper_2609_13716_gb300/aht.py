@@ -149,6 +149,8 @@ def load() -> C.CDLL:
             L.aht_debug_expire_at.restype = C.c_int
             L.aht_debug_logits.argtypes = [vp, vp, i64]
             L.aht_debug_logits.restype = C.c_int
+            L.aht_debug_obs_words.argtypes = [vp, i32, vp]
+            L.aht_debug_obs_words.restype = C.c_int
             L.aht_step_counter.argtypes = [vp]
             L.aht_step_counter.restype = i64
             L.aht_sync.argtypes = [vp]
@@ -451,6 +453,14 @@ def aht_debug_logits(ctx: Context, buf):
         _check(load().aht_debug_logits(ctx.handle, None, 0))
         return
     _check(load().aht_debug_logits(ctx.handle, _ptr(buf, torch.float32, name="buf"), buf.numel()))
+
+
+def aht_debug_obs_words(ctx: Context, seat: int, out):
+    """Parity hook: the streamed cross-play kernel's observation rows of seat ``seat`` of
+    every env's current state, into ``out`` (CUDA int32 [n_envs][(obs_dim + 32) // 32],
+    the bits of uint32 words); Overcooked, Hanabi and Mini Hanabi contexts."""
+    words = (ctx.obs_dim + 32) // 32
+    _check(load().aht_debug_obs_words(ctx.handle, seat, _ptr(out, torch.int32, (ctx.n_envs, words), "out")))
 
 
 def aht_debug_expire_wait(ctx: Context, limit_ns: int):

@@ -1492,6 +1492,20 @@ aht_status aht_debug_logits(aht_ctx* c, float* buf, int64_t floats) {
   return AHT_OK;
 }
 
+aht_status aht_debug_obs_words(aht_ctx* c, int32_t seat, uint32_t* out) {
+  if (!c || !out) return fail(AHT_EINVAL, "ctx or out is NULL");
+  if (seat != 0 && seat != 1) return fail(AHT_EINVAL, "seat must be 0 or 1");
+  auto launch = c->env.kind == AHT_HANABI        ? hanabi_obs_words
+                : c->env.kind == AHT_MINI_HANABI ? minihanabi_obs_words
+                : c->env.kind == AHT_OVERCOOKED  ? overcooked_obs_words
+                                                 : nullptr;
+  if (!launch) return fail(AHT_EINVAL, "LBF observations are not bit rows (LBF cross-play reads bytes)");
+  DeviceGuard g(c->device);
+  const int words = (c->env.obs_dim + 32) / 32;
+  AHT_CUDA(launch(c->state, c->n_envs, batch_of(c).env, seat, words, out, c->stream));
+  return AHT_OK;
+}
+
 aht_status aht_debug_fail_alloc(int64_t n) {
   g_fail_countdown.store(n > 0 ? n : 0);
   return AHT_OK;

@@ -237,6 +237,68 @@ struct EnvHanabi {
     row.set_run(654, s.n_hand[me]);                                            // [654,659)
     if (s.fr >= 0) row.set(659, 1);                                            // [659]
   }
+  // The same bits into a word row (the streamed cross-play kernel): every section is a
+  // field of at most 64 bits at a fixed position, ORed into registers, one store per word.
+  static constexpr int kObsWords = (660 + 31) / 32;
+  __device__ static void obs_into(const DevEnv&, const State& s, int seat, ObsBits& row) {
+    uint32_t wd[kObsWords];
+#pragma unroll
+    for (int i = 0; i < kObsWords; ++i) wd[i] = 0u;
+    auto put = [&](int pos, int nbits, uint64_t v) {  // v < 2^nbits, nbits <= 64
+      const int w = pos >> 5, sh = pos & 31;
+      wd[w] |= (uint32_t)(v << sh);
+      if (sh + nbits > 32) wd[w + 1] |= (uint32_t)((v << sh) >> 32);
+      if (sh + nbits > 64) wd[w + 2] |= (uint32_t)(v >> (64 - sh));
+    };
+    const int me = seat, pa = seat ^ 1;
+#pragma unroll
+    for (int k = 0; k < 5; ++k)  // [0,125) the partner's cards, one-hot
+      put(25 * k, 25, k < s.n_hand[pa] ? 1ull << s.hand[pa][k] : 0ull);
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {  // [125,375) card knowledge, own then the partner's
+      const int who = q == 0 ? me : pa;
+#pragma unroll
+      for (int k = 0; k < 5; ++k)
+        put(125 + 125 * q + 25 * k, 25, k < s.n_hand[who] ? (uint64_t)(s.know[who][k] & 0x1FFFFFFu) : 0ull);
+    }
+    uint32_t fw = 0;  // [375,400) fireworks
+#pragma unroll
+    for (int c = 0; c < 5; ++c)
+      if (s.fw[c]) fw |= 1u << (5 * c + s.fw[c] - 1);
+    put(375, 25, fw);
+    // [400,451) information tokens, life tokens, cards left in the deck (thermometers)
+    put(400, 51, ((1ull << s.info) - 1) | (((1ull << s.lives) - 1) << 8) | (((1ull << (50 - s.ptr)) - 1) << 11));
+    uint64_t disc = 0;  // [451,501) discards: a thermometer per card type (3, 2, 2, 2, 1 copies)
+#pragma unroll
+    for (int t = 0; t < 25; ++t) {
+      const int base = (t % 5) == 0 ? 0 : (t % 5) == 1 ? 3 : (t % 5) == 2 ? 5 : (t % 5) == 3 ? 7 : 9;
+      disc |= ((1ull << s.disc[t]) - 1) << ((t / 5) * 10 + base);
+    }
+    put(451, 50, disc);
+    if (s.la_flags & 1u) {  // [501,554) the last action
+      uint64_t la = 1ull << ((((s.la_flags >> 1) & 1u) == (uint32_t)me) ? 0 : 1);
+      la |= 1ull << (2 + s.la_type);
+      if (s.la_colour != 255) la |= 1ull << (6 + s.la_colour);
+      if (s.la_rank) la |= 1ull << (11 + s.la_rank - 1);
+      if (s.la_slot != 255) la |= 1ull << (16 + s.la_slot);
+      if (s.la_card != 255) la |= 1ull << (21 + s.la_card);
+      la |= (uint64_t)(s.la_hinted & 0x1Fu) << 46;
+      if (s.la_flags & 4u) la |= 1ull << 51;
+      if (s.la_flags & 8u) la |= 1ull << 52;
+      put(501, 53, la);
+    }
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {  // [554,654) explicit hints, own then the partner's
+      const int who = q == 0 ? me : pa;
+#pragma unroll
+      for (int k = 0; k < 5; ++k) put(554 + 50 * q + 10 * k, 10, s.hints[who][k] & 0x3FFu);
+    }
+    // [654,659) own hand size (thermometer), [659] the final round
+    put(654, 6, ((1ull << s.n_hand[me]) - 1) | (s.fr >= 0 ? 1ull << 5 : 0ull));
+#pragma unroll
+    for (int i = 0; i < kObsWords; ++i) row.w[i] = wd[i];
+    for (int i = kObsWords; i < row.words; ++i) row.w[i] = 0u;
+  }
   __device__ static void obs(const DevEnv& d, const State& s, int seat, uint8_t* row) {
     ObsBytes w{row, 165};
     obs_into(d, s, seat, w);

@@ -285,6 +285,13 @@ cudaError_t hanabi_xplay_tc(const XpTcArgs&, int grid, size_t smem, cudaStream_t
 cudaError_t overcooked_xplay_tc_smem_limit(size_t smem);  // once per device, before launches
 cudaError_t hanabi_xplay_tc_smem_limit(size_t smem);
 cudaError_t minihanabi_xplay_tc(const XpTcArgs&, int grid, size_t smem, cudaStream_t);
+// test hook: the cross-play kernel's observation rows of a state array (see xplay_tc.cuh)
+cudaError_t hanabi_obs_words(const uint32_t* state, int64_t n, const DevEnv& env, int seat, int words,
+                             uint32_t* out, cudaStream_t s);
+cudaError_t minihanabi_obs_words(const uint32_t* state, int64_t n, const DevEnv& env, int seat, int words,
+                                 uint32_t* out, cudaStream_t s);
+cudaError_t overcooked_obs_words(const uint32_t* state, int64_t n, const DevEnv& env, int seat, int words,
+                                 uint32_t* out, cudaStream_t s);
 cudaError_t minihanabi_xplay_tc_smem_limit(size_t smem);
 size_t xp_tc_smem_bytes(const WideDims& w);
 

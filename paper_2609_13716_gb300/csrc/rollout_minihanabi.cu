@@ -10,4 +10,8 @@ cudaError_t minihanabi_xplay_tc(const XpTcArgs& a, int grid, size_t smem, cudaSt
   return launch_xp_tc<EnvMiniHanabi>(a, grid, smem, s);
 }
 cudaError_t minihanabi_xplay_tc_smem_limit(size_t smem) { return xp_tc_smem_limit<EnvMiniHanabi>(smem); }
+cudaError_t minihanabi_obs_words(const uint32_t* state, int64_t n, const DevEnv& env, int seat, int words,
+                             uint32_t* out, cudaStream_t s) {
+  return launch_obs_words<EnvMiniHanabi>(state, n, env, seat, words, out, s);
+}
 }  // namespace aht

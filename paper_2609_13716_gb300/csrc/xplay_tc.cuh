@@ -597,6 +597,26 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
   }
 }
 
+// Test hook: the observation rows this kernel builds (the env's bit-row writer, then the
+// constant-1 input at bit obs_dim) for `seat` of every env of a state array (SoA, n envs).
+template <class Env>
+__global__ void obs_words_kernel(const uint32_t* __restrict__ state, int64_t n, const DevEnv env, int seat,
+                                 int words, uint32_t* __restrict__ out) {
+  const int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (e >= n) return;
+  typename Env::State s;
+  load_state(state, n, e, s);
+  ObsBits wr{out + e * words, words};
+  Env::obs_into(env, s, seat, wr);
+  wr.set(env.obs_dim, 1);
+}
+template <class Env>
+cudaError_t launch_obs_words(const uint32_t* state, int64_t n, const DevEnv& env, int seat, int words,
+                             uint32_t* out, cudaStream_t s) {
+  obs_words_kernel<Env><<<(unsigned)((n + 127) / 128), 128, 0, s>>>(state, n, env, seat, words, out);
+  return cudaGetLastError();
+}
+
 // Steps after the first are launched with programmatic stream serialization: their CTAs
 // may start while the previous step finishes, and the kernel waits (griddepcontrol.wait)
 // before it reads or writes anything the previous step touches.  Step 0 follows

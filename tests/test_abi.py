@@ -55,6 +55,7 @@ def test_host_validation_needs_no_gpu(lib):
     assert L.aht_gae(None, None, None, None, 1, 1, 0.9, 0.9, None, None, None) == aht.AHT_EINVAL
     L.aht_debug_expire_wait.argtypes = [C.c_void_p, C.c_int64]
     assert L.aht_debug_expire_wait(None, 1000) == aht.AHT_EINVAL
+    assert L.aht_debug_obs_words(None, 0, None) == aht.AHT_EINVAL
 
     out = aht.XpStatsOut()
     fake = C.c_void_p(16)  # never dereferenced: every case below fails a host check
