@@ -233,6 +233,65 @@ struct EnvMiniHanabi {
     row.set_run(150, s.n_hand[me]);                                          // [150,152)
     if (s.fr >= 0) row.set(152, 1);                                          // [152]
   }
+  // The same bits into a word row (the streamed cross-play kernel): each section a field
+  // at its fixed position, ORed into register words, one store per word.
+  static constexpr int kObsWords = (156 + 31) / 32;
+  __device__ static void obs_into(const DevEnv&, const State& s, int seat, ObsBits& row) {
+    uint32_t wd[kObsWords];
+#pragma unroll
+    for (int i = 0; i < kObsWords; ++i) wd[i] = 0u;
+    auto put = [&](int pos, int nbits, uint64_t v) {  // v < 2^nbits, nbits <= 64
+      const int w = pos >> 5, sh = pos & 31;
+      wd[w] |= (uint32_t)(v << sh);
+      if (sh + nbits > 32) wd[w + 1] |= (uint32_t)((v << sh) >> 32);
+      if (sh + nbits > 64) wd[w + 2] |= (uint32_t)(v >> (64 - sh));
+    };
+    const int me = seat, pa = seat ^ 1;
+#pragma unroll
+    for (int k = 0; k < 2; ++k)  // [0,18) the partner's cards, one-hot
+      put(9 * k, 9, k < s.n_hand[pa] ? 1ull << s.hand[pa][k] : 0ull);
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {  // [18,54) card knowledge, own then the partner's
+      const int who = q == 0 ? me : pa;
+#pragma unroll
+      for (int k = 0; k < 2; ++k) put(18 + 18 * q + 9 * k, 9, k < s.n_hand[who] ? (uint64_t)(s.know[who][k] & 0x1FFu) : 0ull);
+    }
+    uint32_t fw = 0;  // [54,63) fireworks
+#pragma unroll
+    for (int c = 0; c < 3; ++c)
+      if (s.fw[c]) fw |= 1u << (3 * c + s.fw[c] - 1);
+    put(54, 9, fw);
+    // [63,81) information tokens, life token, cards left in the deck (thermometers)
+    put(63, 18, ((1ull << s.info) - 1) | (((1ull << s.lives) - 1) << 3) | (((1ull << (18 - s.ptr)) - 1) << 4));
+    uint64_t disc = 0;  // [81,99) discards: a thermometer per card type (3, 2, 1 copies)
+#pragma unroll
+    for (int t = 0; t < 9; ++t)
+      disc |= ((1ull << s.disc[t]) - 1) << ((t / 3) * 6 + ((t % 3) == 0 ? 0 : ((t % 3) == 1 ? 3 : 5)));
+    put(81, 18, disc);
+    if (s.la_flags & 1u) {  // [99,126) the last action
+      uint64_t la = 1ull << ((((s.la_flags >> 1) & 1u) == (uint32_t)me) ? 0 : 1);
+      la |= 1ull << (2 + s.la_type);
+      if (s.la_colour != 255) la |= 1ull << (6 + s.la_colour);
+      if (s.la_rank) la |= 1ull << (9 + s.la_rank - 1);
+      if (s.la_slot != 255) la |= 1ull << (12 + s.la_slot);
+      if (s.la_card != 255) la |= 1ull << (14 + s.la_card);
+      la |= (uint64_t)(s.la_hinted & 0x3u) << 23;
+      if (s.la_flags & 4u) la |= 1ull << 25;
+      if (s.la_flags & 8u) la |= 1ull << 26;
+      put(99, 27, la);
+    }
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {  // [126,150) explicit hints, own then the partner's
+      const int who = q == 0 ? me : pa;
+#pragma unroll
+      for (int k = 0; k < 2; ++k) put(126 + 12 * q + 6 * k, 6, s.hints[who][k] & 0x3Fu);
+    }
+    // [150,152) own hand size (thermometer), [152] the final round
+    put(150, 3, ((1ull << s.n_hand[me]) - 1) | (s.fr >= 0 ? 1ull << 2 : 0ull));
+#pragma unroll
+    for (int i = 0; i < kObsWords; ++i) row.w[i] = wd[i];
+    for (int i = kObsWords; i < row.words; ++i) row.w[i] = 0u;
+  }
   __device__ static void obs(const DevEnv& d, const State& s, int seat, uint8_t* row) {
     ObsBytes w{row, 39};
     obs_into(d, s, seat, w);
