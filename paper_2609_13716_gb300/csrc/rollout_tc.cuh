@@ -3,7 +3,9 @@
 // One CTA owns a tile of up to 128 envs that share one teammate policy, for all T steps:
 // a contiguous env range (one-member pools, cross-play), or the envs of one teammate's
 // group found by a rank scan of the per-env pool indices (kGather; per-episode
-// teammates: one step per launch).
+// teammates: one step per launch).  This kernel runs cross-play, IPPO and the sparse
+// first layer; plain collection with a dense first layer runs on the two-group kernel of
+// rollout_tc2.cuh, which shares this file's tile finder.
 // Per step and agent (ego = seat 0, teammate = seat 1):
 //   obs (u8, shared memory, a constant 1 after the last feature) -> A operand in tensor
 //       memory as bf16 (exact: small integers)
@@ -791,12 +793,11 @@ struct LaunchTc {
       return a.tc.split ? run<false, true, false, false, true>(a, grid, smem, s)
                         : run<false, false, false, false, true>(a, grid, smem, s);
     }
-    if (a.gather)
-      return a.tc.split ? run<false, true, false, true>(a, grid, smem, s)
-                        : run<false, false, false, true>(a, grid, smem, s);
-    if (ippo)
+    // with a dense first layer this kernel runs IPPO only: plain collection, with contiguous
+    // or gathered tiles, runs on the two-group kernel (rollout_tc2.cuh)
+    if (ippo && !a.gather)
       return a.tc.split ? run<false, true, true>(a, grid, smem, s) : run<false, false, true>(a, grid, smem, s);
-    return a.tc.split ? run<false, true, false>(a, grid, smem, s) : run<false, false, false>(a, grid, smem, s);
+    return cudaErrorNotSupported;
   }
   static cudaError_t xplay(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
     if (a.tc.sparse)
