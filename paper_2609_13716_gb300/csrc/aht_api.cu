@@ -161,6 +161,7 @@ struct aht_ctx {
   size_t wide_smem = 0;
   uint32_t* xp_st[2] = {};
   uint8_t* xp_act[2] = {};
+  float* xp_zp[2] = {};
   uint8_t* xp_alive[2] = {};
   int32_t* xp_nsteps = nullptr;
   // pinned host staging for aht_set_policy, and the event pool of the kernel timer
@@ -568,7 +569,9 @@ aht_status xplay_wide(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego, const i
   const int64_t T0 = ((int64_t)n_tm * P + 127) / 128, T1 = ((int64_t)n_ego * P + 127) / 128;
   take_expire(c, &a.dbg_expire_step, &a.dbg_expire_ns);
   const int64_t tiles0 = n_ego * T0, tiles1 = n_tm * T1;
-  if (tiles0 + tiles1 > INT32_MAX) return fail(AHT_EINVAL, "too many tiles");
+  // H = 512: two CTAs per tile, each computing one N = 256 block of layer 2
+  a.parts = c->wd.H == 512 ? 2 : 1;
+  if ((tiles0 + tiles1) * a.parts > INT32_MAX) return fail(AHT_EINVAL, "too many tiles");
   const bool turn = c->env.kind == AHT_HANABI || c->env.kind == AHT_MINI_HANABI;
   auto launch = c->env.kind == AHT_HANABI        ? hanabi_xplay_tc
                 : c->env.kind == AHT_MINI_HANABI ? minihanabi_xplay_tc
@@ -582,10 +585,12 @@ aht_status xplay_wide(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego, const i
     a.alive_out = c->xp_alive[(s + 1) & 1];
     a.act_in = c->xp_act[(s + 1) & 1];
     a.act_out = c->xp_act[s & 1];
+    a.zp_in = c->xp_zp[(s + 1) & 1];
+    a.zp_out = c->xp_zp[s & 1];
     int64_t grid;
     if (turn) grid = (s & 1) ? tiles1 : tiles0;
     else grid = s < max_steps ? tiles0 + tiles1 : tiles0;
-    AHT_CUDA(launch(a, (int)grid, c->wide_smem, c->stream));
+    AHT_CUDA(launch(a, (int)(grid * a.parts), c->wide_smem, c->stream));
   }
   timer_end(c, tk);
   const int64_t n_pairs = (int64_t)n_ego * n_tm;
@@ -691,6 +696,7 @@ void aht_destroy(aht_ctx* c) {
   for (int i = 0; i < 2; ++i) {
     ctx_free(c->xp_st[i]);
     ctx_free(c->xp_act[i]);
+    ctx_free(c->xp_zp[i]);
     ctx_free(c->xp_alive[i]);
   }
   ctx_free(c->xp_nsteps);
@@ -826,6 +832,8 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
         {(void**)&c->xp_st[1], (size_t)words * n_envs * 4},
         {(void**)&c->xp_act[0], (size_t)n_envs * 2},
         {(void**)&c->xp_act[1], (size_t)n_envs * 2},
+        {(void**)&c->xp_zp[0], (size_t)n_envs * 2 * 2 * c->wd.NAP * 4},
+        {(void**)&c->xp_zp[1], (size_t)n_envs * 2 * 2 * c->wd.NAP * 4},
         {(void**)&c->xp_alive[0], (size_t)n_envs},
         {(void**)&c->xp_alive[1], (size_t)n_envs},
         {(void**)&c->xp_nsteps, (size_t)n_envs * 4},

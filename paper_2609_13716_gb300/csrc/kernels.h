@@ -159,8 +159,11 @@ struct XpTcArgs {
   int64_t n_total;         // n_ego * n_tm * P
   const uint32_t* st_in;   // SoA state [words][n_total]: after step s - 1
   uint32_t* st_out;        // after step s (written by the owning tiles)
-  const uint8_t* act_in;   // [n_total][2] actions of step s - 1
-  uint8_t* act_out;        // [n_total][2] actions of step s
+  int32_t parts;           // CTAs per tile: 2 split layer 2 by N = 256 block (H = 512), else 1
+  const uint8_t* act_in;   // one part: [n_total][2] actions of step s - 1
+  uint8_t* act_out;        // one part: [n_total][2] actions of step s
+  const float* zp_in;      // two parts: [n_total][2 seats][2 parts][NAP] outputs of step s - 1,
+  float* zp_out;           //   without b3; those of step s (each part writes its slot)
   const uint8_t* alive_in; // [n_total]
   uint8_t* alive_out;
   int32_t* nsteps;         // [n_total] steps taken

@@ -6,20 +6,26 @@
 // teammate j).  One launch is one step s of every env (J_AHT of Sec. 3 estimated per
 // pair, XP matrix of App. B).  A tile is up to 128 envs whose acting agent in seat
 // `seat` runs the same policy: seat 0 groups the envs of ego i (pairs (i, 0..n_tm-1),
-// contiguous), seat 1 those of teammate j (pairs (0..n_ego-1, j)).  The envs of a tile
-// change with the seat, so the env state goes through L2 between launches (the SoA
-// state, alive flag and actions are double-buffered by step parity):
-//   1. transition: the tile's envs take step s - 1 with the actions chosen by the
-//      previous launch (step 0: reset).  Each env has one owning tile that writes the
-//      new state, alive flag, step count and return (turn-based games: the tile of the
-//      seat acting at s; simultaneous games: the seat-0 tile; a seat-1 tile of a
-//      simultaneous game computes the same transition for its own use);
+// contiguous), seat 1 those of teammate j (pairs (0..n_ego-1, j)).  For H = 512 a tile
+// has two CTAs ("parts"): both run the transition, the observation, L1 and epilogue 1,
+// and part p computes the N = 256 block p of L2, its epilogue and that block's share of
+// the output layer, so each streams only its half of W2 and runs half of L2.  The envs
+// of a tile change with the seat, so the env state goes through L2 between launches (the
+// SoA state, alive flag and actions or output shares are double-buffered by step parity):
+//   1. transition: the tile's envs take step s - 1 with the actions the previous launch
+//      chose (step 0: reset); with two parts the action is sampled here, from the previous
+//      launch's output shares (their sum + b3, masked inverse CDF, Philox stream = seat).
+//      Each env has one owning CTA (part 0 of the tile of the seat acting at s, or of the
+//      seat-0 tile in simultaneous games) that writes the new state, alive flag, step
+//      count and return; the other CTAs compute the same transition for their own use;
 //   2. the acting seat's binary observation -> bf16 A operand in shared memory (exact);
 //   3. L1 = [o 1] W1^T on tensor cores (N = 256 per instruction, b1 folded into W1);
 //   4. epilogue 1: h1 = tanh(L1), split h1 = hi + lo (two bf16) -> A operands of L2;
 //   5. L2 = hi W2^T + lo W2^T on tensor cores (fp32 accumulate in tensor memory);
-//   6. epilogue 2: h2 = tanh(L2 + b2) and z = W3 h2 + b3 on CUDA cores (fp32);
-//   7. masked inverse-CDF sample of the acting seat's action (Philox stream = seat).
+//   6. epilogue 2: h2 = tanh(L2 + b2) and this CTA's share of W3 h2 (mma.sync);
+//   7. one part: z = W3 h2 + b3 and the masked inverse-CDF sample of the acting seat's
+//      action (Philox stream = seat); two parts: the shares go to global memory for the
+//      next launch, which adds them and samples.
 // Launch max_steps only applies the last transition.
 //
 // Warp roles (320 threads): warps 0-7 compute (thread r and r + 128 own env row r,
@@ -129,7 +135,9 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
   // ---- the tile: seat, acting policy, rows ------------------------------------------
   const int G0 = a.n_tm * a.P, G1 = a.n_ego * a.P;
   const int T0 = (G0 + 127) / 128, T1 = (G1 + 127) / 128;
-  int seat, t = blockIdx.x;
+  // a.parts CTAs per tile: part p computes layer 2's N = 256 block p (H = 512, two parts)
+  int seat, t = (int)blockIdx.x / a.parts;
+  const int part = (int)blockIdx.x - t * a.parts;
   if (kTurn) {
     seat = a.s & 1;
   } else {
@@ -140,7 +148,7 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
   const int group = t / Tn, q0 = (t - group * Tn) * 128;
   const int count = min(128, G - q0);
   const int pol = seat ? a.tm_ids[group] : a.ego_ids[group];
-  const bool owner = kTurn || seat == 0;
+  const bool owner = (kTurn || seat == 0) && part == 0;  // writes the envs' state and records
   auto env_of = [&](int r) -> int64_t {
     const int q = q0 + r;
     if (seat == 0) return (int64_t)group * G0 + q;
@@ -177,9 +185,24 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
-  const int n_chunks = w.n_l1 + w.n_l2;
+  // the chunks this CTA streams: W1's, then W2's (only block `part` when there are two
+  // parts); chunk c of the stream is chunk src(c) of the policy block
+  const int n_l2_own = w.n_l2 / a.parts;
+  const int n_chunks = w.n_l1 + n_l2_own;
   const int SPC = L.spc, n_stages = (n_chunks + SPC - 1) / SPC;
   const uint32_t stage_bytes = (uint32_t)SPC * kWideChunk;
+  const int l2_shift = part * n_l2_own;  // W2 chunks skipped ahead of this part's block
+  // stage k -> one bulk copy, or two where it straddles the W1 / W2 boundary
+  auto copy_stage = [&](int k, uint8_t* dst, uint64_t* bar, uint64_t policy) {
+    const int c0 = k * SPC, c1 = min(c0 + SPC, n_chunks);
+    tc::mbar_expect_tx(bar, (uint32_t)(c1 - c0) * kWideChunk);
+    const int cut = c0 < w.n_l1 && c1 > w.n_l1 ? w.n_l1 : c1;  // end of the first piece
+    const int s0 = c0 < w.n_l1 ? c0 : c0 + l2_shift;
+    tc::bulk_g2s_hint(dst, pblk + (int64_t)s0 * kWideChunk, (uint32_t)(cut - c0) * kWideChunk, bar, policy);
+    if (cut < c1)
+      tc::bulk_g2s_hint(dst + (size_t)(cut - c0) * kWideChunk, pblk + (int64_t)(cut + l2_shift) * kWideChunk,
+                        (uint32_t)(c1 - cut) * kWideChunk, bar, policy);
+  };
   // producer state (warp 9, lane 0): next stage, its ring slot, uses of that slot so far
   int pk = 0, pslot = 0;
   uint32_t puse = 0;
@@ -187,11 +210,8 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
   const int free_slots = (int)((L.bits_off - L.stage_off) / stage_bytes);
   if (warp == 9 && lane == 0) {  // the first stages: the population is read-only
     const uint64_t keep = tc::l2_evict_last();
-    for (; pk < n_stages && pk < NST && pk < free_slots; ++pk, ++pslot) {
-      const uint32_t bytes = (uint32_t)min(SPC, n_chunks - pk * SPC) * kWideChunk;
-      tc::mbar_expect_tx(&full_bar[pslot], bytes);
-      tc::bulk_g2s_hint(sStage + pslot * stage_bytes, pblk + (int64_t)pk * stage_bytes, bytes, &full_bar[pslot], keep);
-    }
+    for (; pk < n_stages && pk < NST && pk < free_slots; ++pk, ++pslot)
+      copy_stage(pk, sStage + pslot * stage_bytes, &full_bar[pslot], keep);
     if (pslot == NST) {
       pslot = 0;
       puse = 1;
@@ -202,9 +222,44 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
 
   // ---- 1. transition of step s - 1, and this step's observation bits -----------------
   bool alive = false;
-  float u_act = 0.0f;
-  uint32_t legal = 0xFFFFFFFFu >> (32 - NA);
   int64_t e = -1;
+  float u_act = 0.0f;                           // one part: this step's sampling happens here
+  uint32_t legal = 0xFFFFFFFFu >> (32 - NA);
+  // Two parts: the action seat q of env e chose at step s - 1 comes from the outputs of the
+  // previous launch -- the two parts' shares plus b3 of seat q's policy -- sampled as in
+  // every other kernel (masked inverse CDF, Philox stream q at step s - 1).  The shares
+  // and b3 are loaded (16-byte vectors) before the state, so their latency overlaps it.
+  constexpr int kActing = kTurn ? 1 : 2;  // seats that act in a step
+  auto gather_z = [&](int q, int64_t env, float (&z)[NAP]) {  // false if a part gave up (NaN)
+    const float4* zp = reinterpret_cast<const float4*>(a.zp_in + ((env * 2 + q) * 2) * NAP);
+    const int64_t pair = env / a.P;
+    const int i = (int)(pair / a.n_tm), j = (int)(pair - (int64_t)i * a.n_tm);
+    const int pq = q == 0 ? a.ego_ids[i] : a.tm_ids[j];
+    const float4* b3 = reinterpret_cast<const float4*>(a.tcw + (int64_t)pq * w.pol_bytes + w.ob3);
+#pragma unroll
+    for (int v = 0; v < NAP / 4; ++v) {
+      const float4 p0 = zp[v], p1 = zp[NAP / 4 + v], bb = b3[v];
+      z[4 * v] = (p0.x + p1.x) + bb.x;
+      z[4 * v + 1] = (p0.y + p1.y) + bb.y;
+      z[4 * v + 2] = (p0.z + p1.z) + bb.z;
+      z[4 * v + 3] = (p0.w + p1.w) + bb.w;
+    }
+  };
+  auto pick = [&](int q, const State& st, int64_t env, const float (&z)[NAP]) -> int {
+    bool finite = true;
+#pragma unroll
+    for (int o = 0; o < NAP; ++o) finite = finite && z[o] == z[o];
+    if (!finite) return -1;
+    if (owner && a.dbg_logits) {  // test hook: the outputs of step s - 1
+      float* p = a.dbg_logits + (((int64_t)(a.s - 1) * a.n_total + env) * 2 + q) * kDbgStride;
+#pragma unroll
+      for (int o = 0; o < NAP; ++o) p[o] = z[o];
+    }
+    const uint32_t lg = kTurn ? Env::legal(st) : 0xFFFFFFFFu >> (32 - NA);
+    const float u = u01(draw0(a.b.key, (uint32_t)env, gt - 1u, kStreamAct0 + q));
+    float lp;
+    return sample_k<NA>(z, lg, u, lp);
+  };
   if (tid < 128) {
     uint32_t* bits = sBits + row * L.bit_words;
     if (row < count) {
@@ -214,6 +269,13 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
       // this kernel's shared memory
       State& s = reinterpret_cast<State*>(sA)[row];
       int nst = 0;
+      const int actor = kTurn ? ((a.s - 1) & 1) : -1;  // the seat that acted at s - 1
+      float zq[kActing][NAP];
+      const bool two = a.parts == 2 && a.s > 0;
+      if (two) {
+#pragma unroll
+        for (int k = 0; k < kActing; ++k) gather_z(kTurn ? actor : k, e, zq[k]);
+      }
       if (a.s == 0) {
         Env::reset(a.b.env, a.b.key, (uint32_t)e, a.step0, s);
         alive = true;
@@ -222,22 +284,37 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
         alive = a.alive_in[e] != 0;
         if (owner) nst = a.nsteps[e];
         if (alive) {
-          const int actor = kTurn ? ((a.s - 1) & 1) : -1;
-          const int a0 = (actor < 0 || actor == 0) ? a.act_in[2 * e] : 0;
-          const int a1 = (actor < 0 || actor == 1) ? a.act_in[2 * e + 1] : 0;
-          if (owner && a.actions) {
-            uint8_t* rec = a.actions + ((int64_t)(a.s - 1) * a.n_total + e) * 2;
-            rec[0] = (actor < 0 || actor == 0) ? (uint8_t)a0 : 255;
-            rec[1] = (actor < 0 || actor == 1) ? (uint8_t)a1 : 255;
-          }
-          float r0, r1, team;
-          const int done = Env::step(a.b.env, s, a0, a1, r0, r1, team);
-          if (done < 0) {
-            if (owner) atomicOr(a.b.status, kStatusIllegalAction);
-            alive = false;
+          int a0 = 0, a1 = 0;
+          if (two) {
+            if (kTurn) {
+              const int act = pick(actor, s, e, zq[0]);
+              (actor == 0 ? a0 : a1) = act;
+              if (act < 0) a0 = -1;
+            } else {
+              a0 = pick(0, s, e, zq[0]);
+              a1 = pick(1, s, e, zq[kActing - 1]);
+            }
           } else {
-            nst += 1;
-            if (done) alive = false;
+            if (actor < 0 || actor == 0) a0 = a.act_in[2 * e];
+            if (actor < 0 || actor == 1) a1 = a.act_in[2 * e + 1];
+          }
+          if (a0 < 0 || a1 < 0) {
+            alive = false;  // a part of the previous launch gave up: the env stops
+          } else {
+            if (owner && a.actions) {
+              uint8_t* rec = a.actions + ((int64_t)(a.s - 1) * a.n_total + e) * 2;
+              rec[0] = (actor < 0 || actor == 0) ? (uint8_t)a0 : 255;
+              rec[1] = (actor < 0 || actor == 1) ? (uint8_t)a1 : 255;
+            }
+            float r0, r1, team;
+            const int done = Env::step(a.b.env, s, a0, a1, r0, r1, team);
+            if (done < 0) {
+              if (owner) atomicOr(a.b.status, kStatusIllegalAction);
+              alive = false;
+            } else {
+              nst += 1;
+              if (done) alive = false;
+            }
           }
         }
       }
@@ -256,7 +333,7 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
           legal = Env::legal(s);
           if (Env::actor(s) != seat) atomicOr(a.b.status, kStatusActorMismatch);
         }
-        u_act = u01(draw0(a.b.key, (uint32_t)e, gt, kStreamAct0 + seat));
+        if (a.parts == 1) u_act = u01(draw0(a.b.key, (uint32_t)e, gt, kStreamAct0 + seat));
       } else {
         for (int i = 0; i < L.bit_words; ++i) bits[i] = 0u;
       }
@@ -295,9 +372,7 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
             ok = tc::mbar_wait(&empty_bar[slot], (use - 1) & 1u, 2000000ull);
           if (!ok) break;
         }
-        const uint32_t bytes = (uint32_t)min(SPC, n_chunks - k * SPC) * kWideChunk;
-        tc::mbar_expect_tx(&full_bar[slot], bytes);
-        tc::bulk_g2s_hint(sStage + slot * stage_bytes, pblk + (int64_t)k * stage_bytes, bytes, &full_bar[slot], keep);
+        copy_stage(k, sStage + slot * stage_bytes, &full_bar[slot], keep);
         if (++slot == NST) {
           slot = 0;
           ++use;
@@ -369,8 +444,10 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
         if (ok) tc::commit(&acc_bar[1]);
       } else if (ok) {
         const uint32_t ahi = tc::smem_u32(sA);
-        for (int nh = 0; ok && nh < 2; ++nh) {
-          if (nh == 1 && !(ok = wait_for(&epi2_bar, 0))) break;
+        // this CTA's blocks of L2: both, or its part's (then into acc_bar[1])
+        const int nh0 = a.parts == 2 ? part : 0, nh1 = a.parts == 2 ? part + 1 : 2;
+        for (int nh = nh0; ok && nh < nh1; ++nh) {
+          if (nh > nh0 && !(ok = wait_for(&epi2_bar, 0))) break;
           for (int ks = 0; ok && ks < 32; ++ks) {
             uint64_t bd;
             if (!(ok = chunk(bd))) break;
@@ -378,7 +455,7 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
             tc::mma_ts(tmem + 256u, tmem + 8u * ks, bd, idesc, 1u);
             release();
           }
-          if (ok) tc::commit(&acc_bar[1 + nh]);
+          if (ok) tc::commit(&acc_bar[1 + nh - nh0]);
         }
       }
       if (!ok) abort_flag = 1;
@@ -496,10 +573,11 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
       for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
         for (int i = 0; i < 4; ++i) zacc[rg][nt][i] = 0.0f;
-    const int n_blocks = w.H / 256;
+    // the N = 256 blocks of L2 this CTA computes: all, or its part's
+    const int nb0 = a.parts == 2 ? part : 0, nb1 = a.parts == 2 ? part + 1 : w.H / 256;
     const uint32_t R1q = tmem + 256u + ((uint32_t)((warp & 3) * 32) << 16);  // this warp's rows
-    for (int nh = 0; nh < n_blocks; ++nh) {
-      wait_acc(&acc_bar[1 + nh]);
+    for (int nh = nb0; nh < nb1; ++nh) {
+      wait_acc(&acc_bar[1 + nh - nb0]);
       if (bad) break;
 #pragma unroll 1
       for (int kc = 0; kc < 8; ++kc) {
@@ -531,7 +609,7 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
           }
         }
       }
-      if (nh == 0 && n_blocks == 2) {
+      if (nh + 1 < nb1) {
         tc::fence_before_sync();
         tc::mbar_arrive(&epi2_bar);  // R1 may take the second half
       }
@@ -553,23 +631,40 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
     }
     bad = sync_or();
 
-    // 7. sample the acting seat's action (half 0 threads, live rows)
-    if (!bad && tid < 128 && alive) {
-      float z[NAP];
+    // 7. one part: sample the acting seat's action (half 0 threads, live rows).  Two parts:
+    //    this CTA's share of the outputs (the sum over its units of W3 h2) goes to global
+    //    memory, and the next launch adds the shares and b3 and samples.
+    if (a.parts == 1) {
+      if (!bad && tid < 128 && alive) {
+        float z[NAP];
 #pragma unroll
-      for (int o = 0; o < NAP; ++o)
-        z[o] = (zpart[row * NAP + o] + zpart[(128 + row) * NAP + o]) + b3[o];
-      if (a.dbg_logits) {  // test hook: this row's outputs of step s
-        float* p = a.dbg_logits + (((int64_t)a.s * a.n_total + e) * 2 + seat) * kDbgStride;
+        for (int o = 0; o < NAP; ++o)
+          z[o] = (zpart[row * NAP + o] + zpart[(128 + row) * NAP + o]) + b3[o];
+        if (a.dbg_logits) {  // test hook: this row's outputs of step s
+          float* p = a.dbg_logits + (((int64_t)a.s * a.n_total + e) * 2 + seat) * kDbgStride;
 #pragma unroll
-        for (int o = 0; o < NAP; ++o) p[o] = z[o];
+          for (int o = 0; o < NAP; ++o) p[o] = z[o];
+        }
+        float lp;
+        const int act = sample_k<NA>(z, legal, u_act, lp);
+        a.act_out[2 * e + seat] = (uint8_t)act;
       }
-      float lp;
-      const int act = sample_k<NA>(z, legal, u_act, lp);
-      a.act_out[2 * e + seat] = (uint8_t)act;
+    } else {
+      if (!bad && tid < 128 && row < count) {
+        float* zo = a.zp_out + ((e * 2 + seat) * 2 + part) * NAP;
+#pragma unroll
+        for (int o = 0; o < NAP; ++o) zo[o] = zpart[row * NAP + o] + zpart[(128 + row) * NAP + o];
+      }
+      // a CTA that gave up leaves NaN shares: the next launch stops those envs rather
+      // than sample from stale ones (their returns stay those of the state before)
+      if (bad && tid < 128 && e >= 0) {
+        float* zo = a.zp_out + ((e * 2 + seat) * 2 + part) * NAP;
+#pragma unroll
+        for (int o = 0; o < NAP; ++o) zo[o] = __int_as_float(0x7FC00000);
+      }
     }
     // a tile that gave up wrote no action: its envs stop here, so that no later step of
-    // the call applies a stale one (their returns stay those of the state before)
+    // the call applies a stale one
     if (bad && tid < 128 && e >= 0 && owner) a.alive_out[e] = 0;
     if (bad) abort_flag = 1;
   }
