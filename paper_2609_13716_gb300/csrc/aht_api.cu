@@ -378,6 +378,8 @@ bool wide_eligible(const aht_ctx* c, int dtype) {
   const MlpDims& m = c->mlp;
   if (dtype != AHT_BF16 || c->env.kind == AHT_LBF) return false;
   if (m.H0 != m.H1 || (m.H0 != 256 && m.H0 != 512)) return false;
+  // the 128 env states of a tile live at the start of the operand region during the transition
+  if (128 * (size_t)c->ops.bytes() > xp_tc_state_bytes(make_wide_dims(m))) return false;
   return xp_tc_smem_bytes(make_wide_dims(m)) <= c->smem_optin;
 }
 

@@ -297,6 +297,7 @@ cudaError_t overcooked_obs_words(const uint32_t* state, int64_t n, const DevEnv&
                                  uint32_t* out, cudaStream_t s);
 cudaError_t minihanabi_xplay_tc_smem_limit(size_t smem);
 size_t xp_tc_smem_bytes(const WideDims& w);
+size_t xp_tc_state_bytes(const WideDims& w);  // room for the tile's env states (operand region)
 
 // misc.cu
 cudaError_t launch_group(const GroupArgs&, cudaStream_t);          // one-member pool

@@ -12,6 +12,7 @@ cudaError_t overcooked_xplay_tc(const XpTcArgs& a, int grid, size_t smem, cudaSt
 cudaError_t overcooked_xplay_tc_smem_limit(size_t smem) { return xp_tc_smem_limit<EnvOvercooked>(smem); }
 
 size_t xp_tc_smem_bytes(const WideDims& w) { return xp_tc_layout(w).total; }
+size_t xp_tc_state_bytes(const WideDims& w) { return xp_tc_layout(w).a_bytes; }
 cudaError_t overcooked_obs_words(const uint32_t* state, int64_t n, const DevEnv& env, int seat, int words,
                              uint32_t* out, cudaStream_t s) {
   return launch_obs_words<EnvOvercooked>(state, n, env, seat, words, out, s);

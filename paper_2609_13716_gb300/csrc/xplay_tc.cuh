@@ -54,7 +54,7 @@ constexpr int kXpCompute = 256;
 constexpr int kXpThreads = 320;
 constexpr int kXpComputeBar = 1;
 constexpr int kXpMaxStages = 3;
-constexpr int kXpMaxChunksPerStage = 5;
+constexpr int kXpMaxChunksPerStage = 12;  // a bulk copy's rate grows with its size (to ~100 KB)
 constexpr uint32_t kXpSmemBudget = 231424;  // opt-in maximum minus a margin for static data
 
 struct XpTcSmem {
@@ -68,12 +68,17 @@ struct XpTcSmem {
   int nst;             // stages
   int spc;             // 8 KB chunks per stage (one bulk copy, one full / empty barrier pair)
   int bit_words;       // 32-bit words per observation bit row
+  int k_tm;            // H = 256: the first k_tm observation inputs form L1's A operand in
+                       // tensor memory (columns [256, 256 + k_tm / 2), free until L2);
+                       // the rest (KP - k_tm) sit in shared memory.  H = 512: 0.
 };
 
 __host__ __device__ inline XpTcSmem xp_tc_layout(const WideDims& w) {
   XpTcSmem L;
-  // L1: observation tile.  L2 and after: hi (H = 512) or the output partials, then W3.
-  const uint32_t obs = 128u * (uint32_t)w.KP * 2u;
+  // L1: observation tile (H = 256: only its part beyond the tensor-memory columns).  L2
+  // and after: hi (H = 512) or the output partials, then W3.
+  L.k_tm = w.H == 256 ? (w.KP < 512 ? w.KP : 512) : 0;
+  const uint32_t obs = 128u * (uint32_t)(w.KP - L.k_tm) * 2u;
   const uint32_t hi = w.H == 512 ? 128u * 512u * 2u : 0u;
   const uint32_t zp = 2u * 128u * (uint32_t)w.NAP * 4u;
   L.w3_off = (uint32_t)align_up(hi > zp ? hi : zp, 1024);
@@ -415,14 +420,29 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
         ++c;
       };
       bool ok = wait_for(&obs_bar, 0);
-      const uint32_t aobs = tc::smem_u32(sA), sbo_obs = (uint32_t)(w.KP / 8) * 128u;
-      for (int nh = 0; ok && nh < w.H / 256; ++nh)
+      // the observation operand: inputs [0, k_tm) in tensor memory (H = 256), the rest in
+      // shared memory as a canonical [128][KP - k_tm] matrix
+      const int ks_tm = L.k_tm / 16;
+      const uint32_t aobs = tc::smem_u32(sA), sbo_obs = (uint32_t)((w.KP - L.k_tm) / 8) * 128u;
+      if (ks_tm == 0) {  // all in shared memory (H = 512)
+        for (int nh = 0; ok && nh < w.H / 256; ++nh)
+          for (int ks = 0; ok && ks < w.KP / 16; ++ks) {
+            uint64_t bd;
+            if (!(ok = chunk(bd))) break;
+            tc::mma_ss(tmem + 256u * nh, tc::smem_desc(aobs + 256u * ks, 128u, sbo_obs), bd, idesc, ks > 0);
+            release();
+          }
+      } else {  // H = 256: one N = 256 block
         for (int ks = 0; ok && ks < w.KP / 16; ++ks) {
           uint64_t bd;
           if (!(ok = chunk(bd))) break;
-          tc::mma_ss(tmem + 256u * nh, tc::smem_desc(aobs + 256u * ks, 128u, sbo_obs), bd, idesc, ks > 0);
+          if (ks < ks_tm)
+            tc::mma_ts(tmem, tmem + 256u + 8u * ks, bd, idesc, ks > 0);
+          else
+            tc::mma_ss(tmem, tc::smem_desc(aobs + 256u * (ks - ks_tm), 128u, sbo_obs), bd, idesc, ks > 0);
           release();
         }
+      }
       if (ok) tc::commit(&acc_bar[0]);
       // once L1 has read the observation tile, W3 b2 b3 go to the A region's tail
       if (ok) ok = wait_for(&acc_bar[0], 0);
@@ -472,26 +492,53 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
     };
     auto sync_or = [&]() { return tc::bar_or(kXpComputeBar, kXpCompute, bad || abort_flag); };
 
-    // 2. observation bits -> bf16 A operand (canonical K-major [128][KP]); each half of
-    //    the threads expands half of the row's 8-feature chunks
+    // 2. observation bits -> bf16 A operand.  H = 512: all in shared memory (canonical
+    //    K-major [128][KP]).  H = 256: 8-feature blocks [0, k_tm / 8) into tensor memory
+    //    (this warp's rows, 4 columns per block, two blocks per store), the rest into
+    //    shared memory ([128][KP - k_tm]).  Each half of the threads expands an even-sized
+    //    half of the row's blocks.
     {
       const uint32_t* bits = sBits + row * L.bit_words;
-      const int nkb = w.KP / 8, split = (nkb + 1) / 2;
+      const int nkb = w.KP / 8, split = (nkb / 2) & ~1, kb_tm = L.k_tm / 8;
       const int kb0 = half ? split : 0, kb1 = half ? nkb : split;
-      // the 16-byte core-matrix rows of consecutive 8-feature blocks are 128 bytes apart
-      uint8_t* dst = sA + tc::canon_offset(row, 8 * kb0, w.KP);
-      uint32_t word = kb0 < kb1 ? bits[kb0 >> 2] : 0u;
-      for (int kb = kb0; kb < kb1; ++kb, dst += 128) {
+      auto block = [&](uint32_t word, int kb, uint32_t (&v)[4]) {  // block kb's bf16 pairs
+        const uint32_t byte = (word >> (8 * (kb & 3))) & 0xFFu;  // word = bits[kb / 4]
+        v[0] = bits_to_bf16x2(byte);
+        v[1] = bits_to_bf16x2(byte >> 2);
+        v[2] = bits_to_bf16x2(byte >> 4);
+        v[3] = bits_to_bf16x2(byte >> 6);
+      };
+      int kb = kb0;
+      if (kb_tm > 0) {
+        // KP and k_tm are multiples of 16 and `split` is even, so each half's blocks in
+        // tensor memory come in pairs (kb even: column 256 + 4 kb is a multiple of 8)
+        const int t1 = kb1 < kb_tm ? kb1 : kb_tm;
+        for (; kb < t1; kb += 2) {
+          const uint32_t word = bits[kb >> 2];  // kb even: kb + 1 is in the same word
+          uint32_t v[8], u[4];
+          block(word, kb, u);
+          v[0] = u[0], v[1] = u[1], v[2] = u[2], v[3] = u[3];
+          block(word, kb + 1, u);
+          v[4] = u[0], v[5] = u[1], v[6] = u[2], v[7] = u[3];
+          tc::st_x8(tmem + lane_base + 256u + 4u * (uint32_t)kb, v);
+        }
+        tc::wait_st();
+        if (kb < kb_tm) kb = kb_tm;
+      }
+      // the shared-memory part: 16-byte core-matrix rows of consecutive blocks 128 bytes apart
+      uint8_t* dst = sA + tc::canon_offset(row, 8 * (kb - kb_tm), w.KP - L.k_tm);
+      uint32_t word = kb < kb1 ? bits[kb >> 2] : 0u;
+      for (; kb < kb1; ++kb, dst += 128) {
         if ((kb & 3) == 0) word = bits[kb >> 2];
-        const uint32_t byte = (word >> (8 * (kb & 3))) & 0xFFu;
         uint4 v;
-        v.x = bits_to_bf16x2(byte);
-        v.y = bits_to_bf16x2(byte >> 2);
-        v.z = bits_to_bf16x2(byte >> 4);
-        v.w = bits_to_bf16x2(byte >> 6);
+        v.x = bits_to_bf16x2(word >> (8 * (kb & 3)));
+        v.y = bits_to_bf16x2(word >> (8 * (kb & 3) + 2));
+        v.z = bits_to_bf16x2(word >> (8 * (kb & 3) + 4));
+        v.w = bits_to_bf16x2(word >> (8 * (kb & 3) + 6));
         *reinterpret_cast<uint4*>(dst) = v;
       }
       tc::fence_proxy_async();
+      if (kb_tm > 0) tc::fence_before_sync();
       tc::mbar_arrive(&obs_bar);
     }
 
