@@ -237,8 +237,8 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
   constexpr int kActing = kTurn ? 1 : 2;  // seats that act in a step
   auto gather_z = [&](int q, int64_t env, float (&z)[NAP]) {  // false if a part gave up (NaN)
     const float4* zp = reinterpret_cast<const float4*>(a.zp_in + ((env * 2 + q) * 2) * NAP);
-    const int64_t pair = env / a.P;
-    const int i = (int)(pair / a.n_tm), j = (int)(pair - (int64_t)i * a.n_tm);
+    const uint32_t pair = (uint32_t)env / (uint32_t)a.P;  // 32-bit: n_total < 2^31
+    const int i = (int)(pair / (uint32_t)a.n_tm), j = (int)(pair - (uint32_t)i * (uint32_t)a.n_tm);
     const int pq = q == 0 ? a.ego_ids[i] : a.tm_ids[j];
     const float4* b3 = reinterpret_cast<const float4*>(a.tcw + (int64_t)pq * w.pol_bytes + w.ob3);
 #pragma unroll
