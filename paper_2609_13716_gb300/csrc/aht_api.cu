@@ -1017,6 +1017,10 @@ static aht_status rollout_common(aht_ctx* c, int32_t ego_id, const int32_t* pool
       ta.g.pool_size = pool_size;
       for (int k = 0; k < pool_size; ++k) ta.g.pool[k] = pool[k];
     }
+    // a programmatic dependent of the grouping kernel just launched: its CTAs set up and
+    // copy the ego's weights while that kernel finishes (the two-group kernel; the others
+    // launch in plain stream order)
+    ta.pdl = 1;
     const int tk = timer_begin(c);
     AHT_CUDA(lbf_ppo_tc(ta, grid, tc_smem, c->stream));
     timer_end(c, tk);

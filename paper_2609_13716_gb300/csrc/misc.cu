@@ -147,6 +147,9 @@ __global__ void __launch_bounds__(128) gae_kernel(const float* __restrict__ r, c
                                                   const uint8_t* __restrict__ d, const float* __restrict__ v_last,
                                                   int64_t n, int32_t T, float gamma, float lambda,
                                                   float* __restrict__ adv, float* __restrict__ tgt) {
+  // launched as a programmatic dependent of the stream's previous kernel (the rollout
+  // that wrote the trajectory): wait until it is complete
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (e >= n) return;
   float next_v = v_last[e];
@@ -183,9 +186,16 @@ cudaError_t launch_gae(const float* r, const float* v, const uint8_t* d, const f
                        int64_t n, int32_t T, float gamma, float lambda, float* adv, float* tgt,
                        cudaStream_t s) {
   const int threads = 128;  // 16384 envs -> 128 CTAs, spread over the SMs
-  const int blocks = (int)((n + threads - 1) / threads);
-  gae_kernel<<<blocks, threads, 0, s>>>(r, v, d, v_last, n, T, gamma, lambda, adv, tgt);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)((n + threads - 1) / threads));
+  cfg.blockDim = dim3(threads);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, gae_kernel, r, v, d, v_last, n, T, gamma, lambda, adv, tgt);
 }
 
 // ---- cross-play cell means: exact fp64 sum of each pair's P returns, divided by P -------
