@@ -411,7 +411,11 @@ float bf16_val(uint16_t h) {
 
 // Packs one policy into its tensor-core block (dst: t.pol_bytes bytes).  bf16 weights go
 // in as they are; fp32 weights w as hi = bf16(w) and lo = bf16(w - hi) (w - hi is exact
-// in fp32).
+// in fp32).  The kernels hand each hidden layer on as its logistic r = 1 / (1 + exp(2x))
+// instead of tanh(x) = 1 - 2 r, so the layers above it hold W' = -2 W (exact: a sign and
+// an exponent) and b' = b + sum_k W[n][k] (summed in fp64 from the given weights and
+// rounded once): W' r + b' = W tanh(x) + b.  L2's b' is stored times 2 / ln 2, the scale
+// its epilogue applies to the accumulator (one fused multiply-add).
 aht_status pack_policy_tc(const MlpDims& m, const TcDims& t, const void* const* W,
                           const void* const* b, int vh, int dtype, uint8_t* dst) {
   if ((dtype == AHT_FP32) != (t.split != 0)) return fail(AHT_EINVAL, "weight dtype differs from the context's population");
@@ -428,14 +432,19 @@ aht_status pack_policy_tc(const MlpDims& m, const TcDims& t, const void* const* 
       std::memcpy(dst + o_lo + off, &lo, 2);
     }
   };
+  const double two_over_ln2 = 2.0 / std::log(2.0);
+  std::vector<double> rowsum;
   for (int l = 0; l < 3; ++l) {
     const void* src = nullptr;
     if (!W[l] || !b[l]) return fail(AHT_EINVAL, "NULL weight pointer");
     if (!read_host(W[l], (size_t)outs[l] * ins[l] * esz, tmp, &src)) return fail(AHT_ECUDA, "copying weights failed");
+    rowsum.assign((size_t)outs[l], 0.0);
     for (int n = 0; n < outs[l]; ++n)
       for (int k = 0; k < ins[l]; ++k) {
         const int64_t i = (int64_t)n * ins[l] + k;
-        const float f = to_f32(src, i, dtype);
+        const float f0 = to_f32(src, i, dtype);
+        rowsum[n] += (double)f0;
+        const float f = l == 0 ? f0 : -2.0f * f0;  // layers fed by a logistic
         if (l == 0 && !t.sparse) put(t.oW1, t.oW1lo, tc::canon_offset(n, k, t.KP), f);
         if (l == 1) put(t.oW2, t.oW2lo, tc::canon_offset(n, k, m.H0), f);
         if (l == 2) {  // B fragment of chunk k / 16 (see TcDims), remainders for split blocks
@@ -449,8 +458,14 @@ aht_status pack_policy_tc(const MlpDims& m, const TcDims& t, const void* const* 
       const float f = to_f32(src, n, dtype);
       if (l == 0 && !t.sparse)  // b1: weight of the constant-1 input
         put(t.oW1, t.oW1lo, tc::canon_offset(n, m.K, t.KP), f);
-      if (l == 1) std::memcpy(dst + t.ob2 + 4 * n, &f, 4);
-      if (l == 2) std::memcpy(dst + t.ob3 + 4 * n, &f, 4);
+      if (l == 1) {
+        const float bk = (float)(((double)f + rowsum[n]) * two_over_ln2);
+        std::memcpy(dst + t.ob2 + 4 * n, &bk, 4);
+      }
+      if (l == 2) {
+        const float bf = (float)((double)f + rowsum[n]);
+        std::memcpy(dst + t.ob3 + 4 * n, &bf, 4);
+      }
     }
   }
   return AHT_OK;

@@ -28,9 +28,12 @@ struct EnvLbf {
     s.al[1] = (uint8_t)(1 + uniform_int(r.next(), (uint32_t)d.max_level));
     const uint32_t lsum = s.al[0] + s.al[1];
     uint32_t F = 0;
-    for (int k = 0; k < d.n_food; ++k) {
-      s.fl[k] = (uint8_t)(1 + uniform_int(r.next(), lsum));
-      F += s.fl[k];
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {  // fixed trip count: the state stays in registers
+      if (k < d.n_food) {
+        s.fl[k] = (uint8_t)(1 + uniform_int(r.next(), lsum));
+        F += s.fl[k];
+      }
     }
     s.F = (uint8_t)F;
     // n_food + 2 steps of a Fisher-Yates shuffle of the cell indices (identity at the
@@ -60,11 +63,16 @@ struct EnvLbf {
         wval[i] = 0;
       }
     }
+    // cell -> (x, y): one division for the grid's reciprocal, then y = floor(c * m / 2^32)
+    // with m = ceil(2^32 / width), exact for c, width < 2^16
+    const uint32_t wd = (uint32_t)d.width, m = 0xFFFFFFFFu / wd + 1u;
+    auto cell_y = [&](int c) { return __umulhi((uint32_t)c, m); };
     s.eaten = 0;
     for (int k = 0; k < 3; ++k) {
       if (k < d.n_food) {
-        s.fx[k] = (uint8_t)(placed[k] % d.width);
-        s.fy[k] = (uint8_t)(placed[k] / d.width);
+        const uint32_t y = cell_y(placed[k]);
+        s.fx[k] = (uint8_t)((uint32_t)placed[k] - y * wd);
+        s.fy[k] = (uint8_t)y;
       } else {
         s.fx[k] = s.fy[k] = s.fl[k] = 0;
         s.eaten |= (uint8_t)(1u << k);
@@ -72,8 +80,13 @@ struct EnvLbf {
     }
     s.fl[3] = 0;
     for (int i = 0; i < 2; ++i) {
-      s.ax[i] = (uint8_t)(placed[d.n_food + i] % d.width);
-      s.ay[i] = (uint8_t)(placed[d.n_food + i] / d.width);
+      int c = 0;  // placed[n_food + i], selected without a runtime register index
+#pragma unroll
+      for (int j = 0; j < 5; ++j)
+        if (j == d.n_food + i) c = placed[j];
+      const uint32_t y = cell_y(c);
+      s.ax[i] = (uint8_t)((uint32_t)c - y * wd);
+      s.ay[i] = (uint8_t)y;
     }
     s.fx[3] = s.ax[1];  // the start position a Sequential teammate plans from
     s.fy[3] = s.ay[1];

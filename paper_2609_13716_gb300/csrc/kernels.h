@@ -51,6 +51,10 @@ struct PpoArgs {
 //      value row when absent, are zero); split blocks follow with the bf16 remainders
 //      W3 - bf16(W3) in the same layout at + H1 * 16 bytes,
 //   b2 fp32 [H1], b3 fp32 [8],
+// where the layers above a hidden layer hold the affine map of its logistic activation
+// r = 1 / (1 + exp(2x)) = (1 - tanh(x)) / 2 (the kernels' activation): W2 and W3 are
+// stored as -2 W (exact), b3 as b3 + W3 1 and b2 as (b2 + W2 1) 2 / ln 2 (the scale of
+// epilogue 2's exponent; sums in fp64, rounded once),
 // and for fp32 populations ("split" blocks) W1lo and W2lo, the bf16 remainders
 // W - bf16(W) in the same layouts as W1 and W2: W = W1 + W1lo to about 2^-17 relative
 // (the weight of the constant-1 input likewise carries b1 as two parts).

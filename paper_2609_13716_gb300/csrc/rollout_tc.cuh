@@ -10,10 +10,12 @@
 //   obs (u8, shared memory, a constant 1 after the last feature) -> A operand in tensor
 //       memory as bf16 (exact: small integers)
 //   L1 (tensor cores): D = [o 1] [W1 b1]^T      (M = 128 envs, N = hidden0, K = KP)
-//   epilogue 1: h1 = tanh(D) split h1 = hi + lo (two bf16) into tensor memory
-//   L2 (tensor cores): D = hi W2^T + lo W2^T  (the split keeps ~2^-17 relative precision
-//       of h1 with bf16 operands and fp32 accumulate)
-//   epilogue 2: h2 = tanh(D + b2), split again, and z = W3 h2 + b3 by mma.sync m16n8k16
+//   epilogue 1: r1 = 1 / (1 + exp(2 D)) split r1 = hi + lo (two bf16) into tensor memory;
+//       tanh(D) = 1 - 2 r1, and the block's W2, b2 hold -2 W2 and b2 + W2 1, so L2 sees
+//       exactly the tanh layer (the same for r2 and W3, b3 below)
+//   L2 (tensor cores): D = hi W2'^T + lo W2'^T  (the split keeps ~2^-17 relative precision
+//       of r1 with bf16 operands and fp32 accumulate)
+//   epilogue 2: r2 = 1 / (1 + exp(2 (D + b2))), split again, and z = W3' r2 + b3' by mma.sync m16n8k16
 //       from registers (16x256b accumulator loads are its fragment layout; a handful of
 //       outputs would waste an N = 16 tcgen05 instruction's round trip)
 //   sampling (ego in warps 0-3, teammate in warps 4-7), env step, trajectory write.
@@ -410,7 +412,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       tc::wait_st();
       operand_ready(ag, 0);
     };
-    // epilogue 1: h1 = tanh(D) -> hi | lo bf16 A operand of L2 (b2 is added in epilogue 2)
+    // epilogue 1: r1 = 1 / (1 + exp(2 D)) -> hi | lo bf16 A operand of L2 (b2 is added in
+    // epilogue 2)
     auto epilogue1 = [&](int ag) {
       const int H = d.H0;
       const uint32_t P = tmem + (uint32_t)(ag * 256) + lane_base, Q = P + 128;
@@ -421,7 +424,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         uint32_t hi[16], lo[16];
 #pragma unroll
         for (int j = 0; j < 16; ++j)
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]))),
+          tc::split_bf16x2_p(tc::logistic2(tc::f2_mul(tc::f2_pack(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1])), tc::kTwoOverLn2x2)),
                              hi[j], lo[j]);
         tc::st_x16(P + c0 / 2, hi);
         tc::st_x16(P + H / 2 + c0 / 2, lo);
@@ -429,7 +432,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       tc::wait_st();
       operand_ready(ag, 1);
     };
-    // kSparse: h1 = tanh(c + sum over the changed features f of delta W1[:, f]) for this
+    // kSparse: r1 = 1 / (1 + exp(2 (c + sum over the changed features f of delta W1[:, f]))) for this
     // thread's half of the units, written like epilogue 1 (hi | lo operand of L2); rows
     // past count take c alone
     auto sparse_h1 = [&](int ag, const State& s) {
@@ -464,19 +467,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         uint32_t hi[16], lo[16];
 #pragma unroll
         for (int j = 0; j < 16; ++j)
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(v[2 * j], v[2 * j + 1])), hi[j], lo[j]);
+          tc::split_bf16x2_p(tc::logistic2(tc::f2_mul(tc::f2_pack(v[2 * j], v[2 * j + 1]), tc::kTwoOverLn2x2)), hi[j], lo[j]);
         tc::st_x16(P + c0 / 2, hi);
         tc::st_x16(P + H / 2 + c0 / 2, lo);
       }
       tc::wait_st();
       operand_ready(ag, 1);
     };
-    // epilogue 2: h2 = tanh(D) and this half's partial z = sum_k W3[:, k] h2[k] on the
+    // epilogue 2: r2 = 1 / (1 + exp(2 (D + b2))) and this half's partial z = sum_k W3'[:, k] r2[k] on the
     // tensor cores from registers (mma.sync m16n8k16, one n-tile of 8 outputs): the warp
     // takes its 32 rows as two groups of 16 and its half's units as chunks of 16; two
     // 16x256b loads of the accumulator give the thread its A fragment (rows g, g + 8 with
     // g = lane / 4; units 2c, 2c + 1 and 2c + 8, 2c + 9 of the chunk, c = lane % 4);
-    // h2 = tanh(D + b2) = hi + lo (two bf16) and z += hi W3^T + lo W3^T (+ hi W3lo^T for
+    // r2 = hi + lo (two bf16) and z += hi W3'^T + lo W3'^T (+ hi W3lo'^T for
     // split blocks), fp32 accumulate.  The partial sums go to shared memory for the
     // sampling half.
     auto epilogue2 = [&](int ag) {
@@ -502,13 +505,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
           tc::ld_16x256b(Qq + ((uint32_t)(16 * rg) << 16) + (uint32_t)(c0 + 8), t1);
           tc::wait_ld();
           uint32_t ahi[4], alo[4];
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t0[0]), __uint_as_float(t0[1])), bA)),
+          tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t0[0]), __uint_as_float(t0[1])), tc::kTwoOverLn2x2, bA)),
                              ahi[0], alo[0]);
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t0[2]), __uint_as_float(t0[3])), bA)),
+          tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t0[2]), __uint_as_float(t0[3])), tc::kTwoOverLn2x2, bA)),
                              ahi[1], alo[1]);
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t1[0]), __uint_as_float(t1[1])), bB)),
+          tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t1[0]), __uint_as_float(t1[1])), tc::kTwoOverLn2x2, bB)),
                              ahi[2], alo[2]);
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t1[2]), __uint_as_float(t1[3])), bB)),
+          tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t1[2]), __uint_as_float(t1[3])), tc::kTwoOverLn2x2, bB)),
                              ahi[3], alo[3]);
           tc::mma_m16n8k16_bf16(zacc[rg], ahi, bw.x, bw.y);
           tc::mma_m16n8k16_bf16(zacc[rg], alo, bw.x, bw.y);

@@ -204,7 +204,8 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
       }
       tc::wait_st();
     };
-    // epilogue 1: h1 = tanh(D) -> hi | lo bf16 A operand of L2, 16 units at a time
+    // epilogue 1: r1 = 1 / (1 + exp(2 D)) -> hi | lo bf16 A operand of L2, 16 units at a
+    // time (tanh(D) = 1 - 2 r1: the block's W2, b2 absorb the affine map, as W3, b3 do for r2)
     auto epilogue1 = [&]() {
       const int H = d.H0;
 #pragma unroll 1
@@ -215,14 +216,14 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
         uint32_t hi[8], lo[8];
 #pragma unroll
         for (int j = 0; j < 8; ++j)
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]))),
+          tc::split_bf16x2_p(tc::logistic2(tc::f2_mul(tc::f2_pack(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1])), tc::kTwoOverLn2x2)),
                              hi[j], lo[j]);
         tc::st_x8(P + c0 / 2, hi);
         tc::st_x8(P + H / 2 + c0 / 2, lo);
       }
       tc::wait_st();
     };
-    // epilogue 2: h2 = tanh(D + b2) split hi + lo, and this half's partial z = W3 h2 by
+    // epilogue 2: r2 = 1 / (1 + exp(2 (D + b2))) split hi + lo, and this half's partial z = W3' r2 by
     // mma.sync m16n8k16 from the 16x256b accumulator fragments (see ppo_tc_kernel)
     auto epilogue2 = [&]() {
       const int H = d.H1;
@@ -247,13 +248,13 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
           tc::ld_16x256b(Qq + ((uint32_t)(16 * rg) << 16) + (uint32_t)(c0 + 8), t1);
           tc::wait_ld();
           uint32_t ahi[4], alo[4];
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t0[0]), __uint_as_float(t0[1])), bA)),
+          tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t0[0]), __uint_as_float(t0[1])), tc::kTwoOverLn2x2, bA)),
                              ahi[0], alo[0]);
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t0[2]), __uint_as_float(t0[3])), bA)),
+          tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t0[2]), __uint_as_float(t0[3])), tc::kTwoOverLn2x2, bA)),
                              ahi[1], alo[1]);
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t1[0]), __uint_as_float(t1[1])), bB)),
+          tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t1[0]), __uint_as_float(t1[1])), tc::kTwoOverLn2x2, bB)),
                              ahi[2], alo[2]);
-          tc::split_bf16x2_p(tc::tanh2(tc::f2_add(tc::f2_pack(__uint_as_float(t1[2]), __uint_as_float(t1[3])), bB)),
+          tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t1[2]), __uint_as_float(t1[3])), tc::kTwoOverLn2x2, bB)),
                              ahi[3], alo[3]);
           tc::mma_m16n8k16_bf16(zacc[rg], ahi, bw.x, bw.y);
           tc::mma_m16n8k16_bf16(zacc[rg], alo, bw.x, bw.y);

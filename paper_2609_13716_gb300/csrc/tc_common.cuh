@@ -275,15 +275,6 @@ __device__ __forceinline__ float rcp_approx(float x) {
   return y;
 }
 
-// Bytes b0, b1 of a 32-bit word (unsigned 0..255) as a packed bf16x2 (b0 low), without
-// integer-to-float conversion instructions: 0x4B000000 | b is the float 2^23 + b, so
-// subtracting 2^23 gives b exactly; a value below 2^8 is exact in bf16, whose bits are
-// the float's upper 16 bits.
-__device__ __forceinline__ uint32_t bytes_to_bf16x2(uint32_t w, int first) {
-  const float f0 = __uint_as_float(__byte_perm(w, 0x4B000000u, 0x7440 + first)) - 8388608.0f;
-  const float f1 = __uint_as_float(__byte_perm(w, 0x4B000000u, 0x7441 + first)) - 8388608.0f;
-  return __byte_perm(__float_as_uint(f0), __float_as_uint(f1), 0x7632);
-}
 
 // ---- packed fp32 pairs (sm_100+ f32x2 arithmetic; each lane is IEEE fp32) -------------
 __device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
@@ -314,6 +305,37 @@ __device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
   uint64_t d;
   asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
+}
+
+// Bytes b0, b1 of a 32-bit word (unsigned 0..255; b0 = byte `first`) as a packed bf16x2
+// (b0 low), without integer-to-float conversion instructions: 0x4B000000 | b is the float
+// 2^23 + b, so subtracting 2^23 (one packed subtraction for both) gives b exactly; a value
+// below 2^8 is exact in bf16, whose bits are the float's upper 16 bits.
+__device__ __forceinline__ uint32_t bytes_to_bf16x2(uint32_t w, int first) {
+  const uint64_t two23 = 0x4B0000004B000000ull;  // 2^23 in each half
+  float f0, f1;
+  f2_unpack(f2_sub(f2_pack(__uint_as_float(__byte_perm(w, 0x4B000000u, 0x7440 + first)),
+                           __uint_as_float(__byte_perm(w, 0x4B000000u, 0x7441 + first))),
+                   two23),
+            f0, f1);
+  return __byte_perm(__float_as_uint(f0), __float_as_uint(f1), 0x7632);
+}
+
+// 2 / ln 2 in each half of a pair: x (2 / ln 2) is the exponent of 2 that gives exp(2x).
+constexpr uint64_t kTwoOverLn2x2 = 0x4038AA3B4038AA3Bull;
+
+// The logistic half of tanh for a pair y = (2 / ln 2) x: r = 1 / (1 + 2^y) = 1 / (1 +
+// exp(2x)), so tanh(x) = 1 - 2 r.  The LBF tensor-core kernels pass r on as the hidden
+// activation and fold the affine map into the next layer instead (weights -2 W, exact in
+// bf16; bias b + W 1): W tanh(x) + b = (-2 W) r + (b + W 1).  The hardware exp2 and
+// reciprocal approximations on each value; r saturates to 0 (y = inf) and 1 (y = -inf).
+__device__ __forceinline__ uint64_t logistic2(uint64_t y) {
+  const uint64_t one = 0x3F8000003F800000ull;  // 1.0f, 1.0f
+  float a, b;
+  f2_unpack(y, a, b);
+  const float ea = ex2_approx(a), eb = ex2_approx(b);
+  f2_unpack(f2_add(f2_pack(ea, eb), one), a, b);
+  return f2_pack(rcp_approx(a), rcp_approx(b));
 }
 
 // tanh of a pair from tanh(x) = 1 - 2 / (1 + e), e = exp(2x) = 2^(2x / ln 2): the
