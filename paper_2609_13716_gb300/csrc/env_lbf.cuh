@@ -44,6 +44,7 @@ struct EnvLbf {
     const int cells = d.width * d.height;
     const int n_obj = d.n_food + 2;
     int wpos[5], wval[5], placed[5];
+    int c0 = 0, c1 = 0;  // the agents' cells, placed[n_food] and placed[n_food + 1]
 #pragma unroll
     for (int i = 0; i < 5; ++i) {
       if (i < n_obj) {
@@ -57,6 +58,8 @@ struct EnvLbf {
         placed[i] = vj;  // position i now holds the old value at j
         wpos[i] = j;     // and position j the old value at i
         wval[i] = vi;
+        if (i == n_obj - 2) c0 = vj;  // taken as they are placed: a runtime index into
+        if (i == n_obj - 1) c1 = vj;  // placed[] would move it out of registers
       } else {
         placed[i] = 0;
         wpos[i] = -1;
@@ -68,6 +71,7 @@ struct EnvLbf {
     const uint32_t wd = (uint32_t)d.width, m = 0xFFFFFFFFu / wd + 1u;
     auto cell_y = [&](int c) { return __umulhi((uint32_t)c, m); };
     s.eaten = 0;
+#pragma unroll
     for (int k = 0; k < 3; ++k) {
       if (k < d.n_food) {
         const uint32_t y = cell_y(placed[k]);
@@ -79,15 +83,11 @@ struct EnvLbf {
       }
     }
     s.fl[3] = 0;
-    for (int i = 0; i < 2; ++i) {
-      int c = 0;  // placed[n_food + i], selected without a runtime register index
-#pragma unroll
-      for (int j = 0; j < 5; ++j)
-        if (j == d.n_food + i) c = placed[j];
-      const uint32_t y = cell_y(c);
-      s.ax[i] = (uint8_t)((uint32_t)c - y * wd);
-      s.ay[i] = (uint8_t)y;
-    }
+    const uint32_t y0 = cell_y(c0), y1 = cell_y(c1);
+    s.ax[0] = (uint8_t)((uint32_t)c0 - y0 * wd);
+    s.ay[0] = (uint8_t)y0;
+    s.ax[1] = (uint8_t)((uint32_t)c1 - y1 * wd);
+    s.ay[1] = (uint8_t)y1;
     s.fx[3] = s.ax[1];  // the start position a Sequential teammate plans from
     s.fy[3] = s.ay[1];
     s.ep_t = 0;
@@ -192,9 +192,11 @@ struct EnvLbf {
 #pragma unroll
     for (int k = 0; k < 3; ++k)  // absent foods are marked eaten
       if (!((s.eaten >> k) & 1u)) put(s.fx[k], s.fy[k], (uint32_t)s.fl[k] << 16);
-    const int o = 1 - seat;
-    put(s.ax[o], s.ay[o], (uint32_t)s.al[o] << 8);
-    put(s.ax[seat], s.ay[seat], (uint32_t)s.al[seat]);
+    // the agents by selection, not by a runtime index (which would move the state copy
+    // out of registers)
+    const bool s1 = seat != 0;
+    put(s1 ? s.ax[0] : s.ax[1], s1 ? s.ay[0] : s.ay[1], (uint32_t)(s1 ? s.al[0] : s.al[1]) << 8);
+    put(s1 ? s.ax[1] : s.ax[0], s1 ? s.ay[1] : s.ay[0], (uint32_t)(s1 ? s.al[1] : s.al[0]));
   }
 
   // Rule-based teammate k in seat 1 (the LBF heuristic suite: Greedy criteria 0..4,

@@ -363,7 +363,7 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
         pair_sync();
         if (sampler) {
           if (tm_rule) {
-            act1s[row] = (uint8_t)Env::heuristic(a.b.env, s, -1 - tm_pol);
+            act1s[row] = (uint8_t)Env::heuristic(a.b.env, st[row], -1 - tm_pol);  // st[row] == s
           } else {
             logits(z);
             dbg_store(t, z);
