@@ -204,22 +204,23 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
       }
       tc::wait_st();
     };
-    // epilogue 1: r1 = 1 / (1 + exp(2 D)) -> hi | lo bf16 A operand of L2, 16 units at a
-    // time (tanh(D) = 1 - 2 r1: the block's W2, b2 absorb the affine map, as W3, b3 do for r2)
+    // epilogue 1: r1 = 1 / (1 + exp(2 D)) -> hi | lo bf16 A operand of L2, 32 units per
+    // tensor-memory load (16 independent pairs between waits; tanh(D) = 1 - 2 r1: the
+    // block's W2, b2 absorb the affine map, as W3, b3 do for r2)
     auto epilogue1 = [&]() {
       const int H = d.H0;
 #pragma unroll 1
-      for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 16) {
-        uint32_t v[16];
-        tc::ld_x16(Q + c0, v);
+      for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 32) {
+        uint32_t v[32];
+        tc::ld_x32(Q + c0, v);
         tc::wait_ld();
-        uint32_t hi[8], lo[8];
+        uint32_t hi[16], lo[16];
 #pragma unroll
-        for (int j = 0; j < 8; ++j)
+        for (int j = 0; j < 16; ++j)
           tc::split_bf16x2_p(tc::logistic2(tc::f2_mul(tc::f2_pack(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1])), tc::kTwoOverLn2x2)),
                              hi[j], lo[j]);
-        tc::st_x8(P + c0 / 2, hi);
-        tc::st_x8(P + H / 2 + c0 / 2, lo);
+        tc::st_x16(P + c0 / 2, hi);
+        tc::st_x16(P + H / 2 + c0 / 2, lo);
       }
       tc::wait_st();
     };
@@ -241,12 +242,18 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
         const uint64_t bB = *reinterpret_cast<const uint64_t*>(b2 + c0 + 8 + 2 * c4);
         uint2 bl = make_uint2(0u, 0u);
         if constexpr (kSplit) bl = *reinterpret_cast<const uint2*>(W3l + (j * 32 + lane) * 2);
+        // both row groups' fragments under one wait: 8 independent pairs
+        uint32_t tt[2][2][4];
 #pragma unroll
         for (int rg = 0; rg < 2; ++rg) {
-          uint32_t t0[4], t1[4];
-          tc::ld_16x256b(Qq + ((uint32_t)(16 * rg) << 16) + (uint32_t)c0, t0);
-          tc::ld_16x256b(Qq + ((uint32_t)(16 * rg) << 16) + (uint32_t)(c0 + 8), t1);
-          tc::wait_ld();
+          tc::ld_16x256b(Qq + ((uint32_t)(16 * rg) << 16) + (uint32_t)c0, tt[rg][0]);
+          tc::ld_16x256b(Qq + ((uint32_t)(16 * rg) << 16) + (uint32_t)(c0 + 8), tt[rg][1]);
+        }
+        tc::wait_ld();
+#pragma unroll
+        for (int rg = 0; rg < 2; ++rg) {
+          const uint32_t (&t0)[4] = tt[rg][0];
+          const uint32_t (&t1)[4] = tt[rg][1];
           uint32_t ahi[4], alo[4];
           tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t0[0]), __uint_as_float(t0[1])), tc::kTwoOverLn2x2, bA)),
                              ahi[0], alo[0]);
