@@ -164,6 +164,11 @@ struct aht_ctx {
   float* xp_zp[2] = {};
   uint8_t* xp_alive[2] = {};
   int32_t* xp_nsteps = nullptr;
+  // two-part tiles (H = 512): the parts' exchange slots and flags, and the launch stamp
+  uint8_t* xp_xch = nullptr;
+  uint32_t* xp_xflag = nullptr;
+  int64_t xp_slots = 0;
+  uint32_t xp_stamp = 0;
   // pinned host staging for aht_set_policy, and the event pool of the kernel timer
   float* staging = nullptr;
   cudaEvent_t upload_done = nullptr;
@@ -586,9 +591,13 @@ aht_status xplay_wide(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego, const i
   const int64_t T0 = ((int64_t)n_tm * P + 127) / 128, T1 = ((int64_t)n_ego * P + 127) / 128;
   take_expire(c, &a.dbg_expire_step, &a.dbg_expire_ns);
   const int64_t tiles0 = n_ego * T0, tiles1 = n_tm * T1;
-  // H = 512: two CTAs per tile, each computing one N = 256 block of layer 2
+  // H = 512: two CTAs per tile, each computing one N = 256 block of layers 1 and 2
   a.parts = c->wd.H == 512 ? 2 : 1;
   if ((tiles0 + tiles1) * a.parts > INT32_MAX) return fail(AHT_EINVAL, "too many tiles");
+  if (a.parts == 2 && std::max(tiles0, tiles1) * 2 > c->xp_slots)
+    return fail(AHT_EINVAL, "more two-part tiles than exchange slots");
+  a.xch = c->xp_xch;
+  a.xflag = c->xp_xflag;
   const bool turn = c->env.kind == AHT_HANABI || c->env.kind == AHT_MINI_HANABI;
   auto launch = c->env.kind == AHT_HANABI        ? hanabi_xplay_tc
                 : c->env.kind == AHT_MINI_HANABI ? minihanabi_xplay_tc
@@ -607,6 +616,9 @@ aht_status xplay_wide(aht_ctx* c, const int32_t* ego_ids, int32_t n_ego, const i
     int64_t grid;
     if (turn) grid = (s & 1) ? tiles1 : tiles0;
     else grid = s < max_steps ? tiles0 + tiles1 : tiles0;
+    // a stamp no earlier launch of this context used (0 is the flags' initial value)
+    if (++c->xp_stamp >= 0x7FFFFFFFu) c->xp_stamp = 1;
+    a.xstamp = c->xp_stamp;
     AHT_CUDA(launch(a, (int)(grid * a.parts), c->wide_smem, c->stream));
   }
   timer_end(c, tk);
@@ -717,6 +729,8 @@ void aht_destroy(aht_ctx* c) {
     ctx_free(c->xp_alive[i]);
   }
   ctx_free(c->xp_nsteps);
+  ctx_free(c->xp_xch);
+  ctx_free(c->xp_xflag);
   if (c->upload_done) cudaEventDestroy(c->upload_done);
   for (auto& e : c->ev)
     if (e) cudaEventDestroy(e);
@@ -868,6 +882,17 @@ aht_status aht_create(const aht_env_desc* envd, const aht_pop_desc* pop, int64_t
     if (se != cudaSuccess) return bail(AHT_ECUDA, "setting the shared-memory limit failed");
     if (ctx_malloc_host((void**)&c->wide_staging, c->wd.pol_bytes) != cudaSuccess)
       return bail(AHT_ENOMEM, "pinned staging allocation failed");
+    if (c->wd.H == 512) {
+      // a call's tiles of one seat: at most n_total / 128 + n_ego (or n_tm) <= n_envs / 128 + 64
+      c->xp_slots = 2 * ((n_envs + 127) / 128 + kMaxXpIds);
+      if (ctx_malloc((void**)&c->xp_xch, (size_t)c->xp_slots * kXchSlot) != cudaSuccess ||
+          ctx_malloc((void**)&c->xp_xflag, (size_t)c->xp_slots * 4) != cudaSuccess) {
+        cudaGetLastError();
+        return bail(AHT_ENOMEM, "cudaMalloc of the cross-play exchange slots failed");
+      }
+      if (cudaMemset(c->xp_xflag, 0, (size_t)c->xp_slots * 4) != cudaSuccess)
+        return bail(AHT_ECUDA, "clearing the cross-play exchange flags failed");
+    }
     c->wide = true;
   }
   *out = c;

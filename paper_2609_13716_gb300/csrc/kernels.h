@@ -177,7 +177,17 @@ struct XpTcArgs {
   float* dbg_logits;       // test hook, or NULL: [max_steps][n_total][2 seats][kDbgStride]
   int32_t dbg_expire_step; // test hook: launch s == this waits on an mbarrier nothing
   uint64_t dbg_expire_ns;  // arrives on, bounded by dbg_expire_ns (-1: never)
+  // Two parts (H = 512): each computes one N = 256 block of L1 and the parts swap their
+  // hidden units' bf16 halves through L2-resident memory: CTA b's slot of kXchSlot bytes
+  // at xch + b kXchSlot, published by xflag[b] = 2 xstamp (2 xstamp + 1: the CTA gave up).
+  // xstamp is unique per launch of a context, so no flag needs clearing between launches.
+  uint8_t* xch;
+  uint32_t* xflag;
+  uint32_t xstamp;
 };
+// One part's exchange slot: hi and lo of 256 hidden units x 128 rows, bf16, as 16-byte
+// chunks of 8 units, [hi 32 | lo 32 chunks][128 rows].
+constexpr size_t kXchSlot = 2 * 32 * 128 * 16;
 
 // Test hook layout: every policy evaluation of a tensor-core kernel may write its output
 // vector (logits, then the value where the policy has one, then zeros) at

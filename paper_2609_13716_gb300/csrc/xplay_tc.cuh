@@ -7,9 +7,12 @@
 // pair, XP matrix of App. B).  A tile is up to 128 envs whose acting agent in seat
 // `seat` runs the same policy: seat 0 groups the envs of ego i (pairs (i, 0..n_tm-1),
 // contiguous), seat 1 those of teammate j (pairs (0..n_ego-1, j)).  For H = 512 a tile
-// has two CTAs ("parts"): both run the transition, the observation, L1 and epilogue 1,
-// and part p computes the N = 256 block p of L2, its epilogue and that block's share of
-// the output layer, so each streams only its half of W2 and runs half of L2.  The envs
+// has two CTAs ("parts", launched as a cluster of two so that they are co-resident): both
+// run the transition and the observation; part p computes the N = 256 block p of L1 and
+// its epilogue, the parts swap their hidden units' bf16 halves through L2-resident
+// exchange slots (a release flag per slot, bounded acquire waits), and part p computes
+// block p of L2, its epilogue and that block's share of the output layer -- so each part
+// streams half of W1 and half of W2 and runs half of every layer.  The envs
 // of a tile change with the seat, so the env state goes through L2 between launches (the
 // SoA state, alive flag and actions or output shares are double-buffered by step parity):
 //   1. transition: the tile's envs take step s - 1 with the actions the previous launch
@@ -18,9 +21,11 @@
 //      Each env has one owning CTA (part 0 of the tile of the seat acting at s, or of the
 //      seat-0 tile in simultaneous games) that writes the new state, alive flag, step
 //      count and return; the other CTAs compute the same transition for their own use;
-//   2. the acting seat's binary observation -> bf16 A operand in shared memory (exact);
-//   3. L1 = [o 1] W1^T on tensor cores (N = 256 per instruction, b1 folded into W1);
-//   4. epilogue 1: h1 = tanh(L1), split h1 = hi + lo (two bf16) -> A operands of L2;
+//   2. the acting seat's binary observation -> bf16 A operand (exact): its first 512
+//      inputs in tensor memory, the rest in shared memory;
+//   3. L1 = [o 1] W1^T on tensor cores (one N = 256 block, b1 folded into W1);
+//   4. epilogue 1: h1 = tanh(L1), split h1 = hi + lo (two bf16) -> A operands of L2
+//      (two parts: each its block's units, then the exchange);
 //   5. L2 = hi W2^T + lo W2^T on tensor cores (fp32 accumulate in tensor memory);
 //   6. epilogue 2: h2 = tanh(L2 + b2) and this CTA's share of W3 h2 (mma.sync);
 //   7. one part: z = W3 h2 + b3 and the masked inverse-CDF sample of the acting seat's
@@ -35,13 +40,13 @@
 // and one full / empty mbarrier pair per stage).  Every wait is bounded; on expiry the CTA records kStatusTimeout, stops,
 // drains its MMAs and copies, frees tensor memory and exits.
 //
-// Tensor memory (512 columns), R0 = [0, 256), R1 = [256, 512):
+// Tensor memory (512 columns), R0 = [0, 256), R1 = [256, 512); the observation's first
+// 512 inputs sit in R1 until L1 is done:
 //   H = 256: L1 -> R0; epilogue 1 rewrites each 32-column block of R0 in place as
 //            16 columns hi | 16 columns lo; L2 -> R1.
-//   H = 512: L1 units [0, 256) -> R0, [256, 512) -> R1; epilogue 1 writes hi to shared
-//            memory (a [128][512] canonical A operand over the dead observation tile)
-//            and packs lo of all 512 units into R0; L2 runs as two N = 256 halves, each
-//            into R1 (the second after epilogue 2 has read the first).
+//   H = 512: L1 block `part` -> R0; epilogue 1 writes hi to shared memory (a [128][512]
+//            canonical A operand over the dead observation tile) and, after the
+//            exchange, lo of all 512 units packed into R0; L2 block `part` -> R1.
 #pragma once
 #include "kernels.h"
 #include "mlp_simt.cuh"
@@ -68,16 +73,17 @@ struct XpTcSmem {
   int nst;             // stages
   int spc;             // 8 KB chunks per stage (one bulk copy, one full / empty barrier pair)
   int bit_words;       // 32-bit words per observation bit row
-  int k_tm;            // H = 256: the first k_tm observation inputs form L1's A operand in
-                       // tensor memory (columns [256, 256 + k_tm / 2), free until L2);
-                       // the rest (KP - k_tm) sit in shared memory.  H = 512: 0.
+  int k_tm;            // the first k_tm observation inputs form L1's A operand in tensor
+                       // memory (columns [256, 256 + k_tm / 2), free until L2); the rest
+                       // (KP - k_tm) sit in shared memory
 };
 
 __host__ __device__ inline XpTcSmem xp_tc_layout(const WideDims& w) {
   XpTcSmem L;
-  // L1: observation tile (H = 256: only its part beyond the tensor-memory columns).  L2
-  // and after: hi (H = 512) or the output partials, then W3.
-  L.k_tm = w.H == 256 ? (w.KP < 512 ? w.KP : 512) : 0;
+  // L1: observation tile, only its part beyond the tensor-memory columns (L1's accumulator
+  // takes 256 columns: all units for H = 256, this part's block for H = 512).  L2 and
+  // after: hi (H = 512) or the output partials, then W3.
+  L.k_tm = w.KP < 512 ? w.KP : 512;
   const uint32_t obs = 128u * (uint32_t)(w.KP - L.k_tm) * 2u;
   const uint32_t hi = w.H == 512 ? 128u * 512u * 2u : 0u;
   const uint32_t zp = 2u * 128u * (uint32_t)w.NAP * 4u;
@@ -114,6 +120,25 @@ __host__ __device__ inline XpTcSmem xp_tc_layout(const WideDims& w) {
 // so one multiply by 0x3F80 writes both halves.
 __device__ __forceinline__ uint32_t bits_to_bf16x2(uint32_t x) {
   return (((x & 3u) * 0x8001u) & 0x00010001u) * 0x3F80u;
+}
+
+// The parts of a tile publish their exchange slot with a release store of the flag after
+// a barrier of the writing threads (one thread, after a gpu-scope fence), and the reader
+// polls it with acquire loads and then releases its threads with a barrier.
+__device__ __forceinline__ void xch_publish(uint32_t* flag, uint32_t v) {
+  asm volatile("fence.acq_rel.gpu;\nst.relaxed.gpu.global.u32 [%0], %1;" ::"l"(flag), "r"(v) : "memory");
+}
+// Until *flag is `ok` (true) or ok + 1 (the writer gave up: false); false as well after 2 s.
+__device__ __forceinline__ bool xch_wait(const uint32_t* flag, uint32_t ok) {
+  const uint64_t t0 = tc::globaltimer_ns();
+  for (uint32_t i = 0; i < (1u << 30); ++i) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(flag) : "memory");
+    if (v == ok) return true;
+    if (v == ok + 1u) return false;
+    if ((i & 63u) == 63u && tc::globaltimer_ns() - t0 > 2000000000ull) return false;
+  }
+  return false;
 }
 
 template <class Env>
@@ -190,22 +215,25 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
-  // the chunks this CTA streams: W1's, then W2's (only block `part` when there are two
-  // parts); chunk c of the stream is chunk src(c) of the policy block
-  const int n_l2_own = w.n_l2 / a.parts;
-  const int n_chunks = w.n_l1 + n_l2_own;
+  // the chunks this CTA streams: W1's, then W2's -- with two parts only block `part` of
+  // each (N = 256 rows of W1 and of W2); chunk c of the stream is chunk src(c) of the
+  // policy block
+  const int n_l1_own = w.n_l1 / a.parts, n_l2_own = w.n_l2 / a.parts;
+  const int n_chunks = n_l1_own + n_l2_own;
   const int SPC = L.spc, n_stages = (n_chunks + SPC - 1) / SPC;
   const uint32_t stage_bytes = (uint32_t)SPC * kWideChunk;
-  const int l2_shift = part * n_l2_own;  // W2 chunks skipped ahead of this part's block
+  auto src_chunk = [&](int c) {  // W1 block `part`, then W2 block `part`
+    return c < n_l1_own ? part * n_l1_own + c : w.n_l1 + part * n_l2_own + (c - n_l1_own);
+  };
   // stage k -> one bulk copy, or two where it straddles the W1 / W2 boundary
   auto copy_stage = [&](int k, uint8_t* dst, uint64_t* bar, uint64_t policy) {
     const int c0 = k * SPC, c1 = min(c0 + SPC, n_chunks);
     tc::mbar_expect_tx(bar, (uint32_t)(c1 - c0) * kWideChunk);
-    const int cut = c0 < w.n_l1 && c1 > w.n_l1 ? w.n_l1 : c1;  // end of the first piece
-    const int s0 = c0 < w.n_l1 ? c0 : c0 + l2_shift;
-    tc::bulk_g2s_hint(dst, pblk + (int64_t)s0 * kWideChunk, (uint32_t)(cut - c0) * kWideChunk, bar, policy);
+    const int cut = c0 < n_l1_own && c1 > n_l1_own ? n_l1_own : c1;  // end of the first piece
+    tc::bulk_g2s_hint(dst, pblk + (int64_t)src_chunk(c0) * kWideChunk, (uint32_t)(cut - c0) * kWideChunk, bar,
+                      policy);
     if (cut < c1)
-      tc::bulk_g2s_hint(dst + (size_t)(cut - c0) * kWideChunk, pblk + (int64_t)(cut + l2_shift) * kWideChunk,
+      tc::bulk_g2s_hint(dst + (size_t)(cut - c0) * kWideChunk, pblk + (int64_t)src_chunk(cut) * kWideChunk,
                         (uint32_t)(c1 - cut) * kWideChunk, bar, policy);
   };
   // producer state (warp 9, lane 0): next stage, its ring slot, uses of that slot so far
@@ -420,28 +448,19 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
         ++c;
       };
       bool ok = wait_for(&obs_bar, 0);
-      // the observation operand: inputs [0, k_tm) in tensor memory (H = 256), the rest in
-      // shared memory as a canonical [128][KP - k_tm] matrix
+      // L1: one N = 256 block (all units for H = 256, block `part` for H = 512) into
+      // columns [0, 256); the observation operand has inputs [0, k_tm) in tensor memory,
+      // the rest in shared memory as a canonical [128][KP - k_tm] matrix
       const int ks_tm = L.k_tm / 16;
       const uint32_t aobs = tc::smem_u32(sA), sbo_obs = (uint32_t)((w.KP - L.k_tm) / 8) * 128u;
-      if (ks_tm == 0) {  // all in shared memory (H = 512)
-        for (int nh = 0; ok && nh < w.H / 256; ++nh)
-          for (int ks = 0; ok && ks < w.KP / 16; ++ks) {
-            uint64_t bd;
-            if (!(ok = chunk(bd))) break;
-            tc::mma_ss(tmem + 256u * nh, tc::smem_desc(aobs + 256u * ks, 128u, sbo_obs), bd, idesc, ks > 0);
-            release();
-          }
-      } else {  // H = 256: one N = 256 block
-        for (int ks = 0; ok && ks < w.KP / 16; ++ks) {
-          uint64_t bd;
-          if (!(ok = chunk(bd))) break;
-          if (ks < ks_tm)
-            tc::mma_ts(tmem, tmem + 256u + 8u * ks, bd, idesc, ks > 0);
-          else
-            tc::mma_ss(tmem, tc::smem_desc(aobs + 256u * (ks - ks_tm), 128u, sbo_obs), bd, idesc, ks > 0);
-          release();
-        }
+      for (int ks = 0; ok && ks < w.KP / 16; ++ks) {
+        uint64_t bd;
+        if (!(ok = chunk(bd))) break;
+        if (ks < ks_tm)
+          tc::mma_ts(tmem, tmem + 256u + 8u * ks, bd, idesc, ks > 0);
+        else
+          tc::mma_ss(tmem, tc::smem_desc(aobs + 256u * (ks - ks_tm), 128u, sbo_obs), bd, idesc, ks > 0);
+        release();
       }
       if (ok) tc::commit(&acc_bar[0]);
       // once L1 has read the observation tile, W3 b2 b3 go to the A region's tail
@@ -484,7 +503,7 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
     // ============================== compute warps ===================================
     bool bad = false;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
-    const uint32_t R0 = tmem + lane_base, R1 = tmem + 256u + lane_base;
+    const uint32_t R0 = tmem + lane_base;
     auto wait_acc = [&](uint64_t* bar) {
       if (!bad && !tc::mbar_wait(bar, 0)) bad = true;
       bad = __any_sync(0xFFFFFFFFu, bad);
@@ -562,34 +581,67 @@ __global__ void __launch_bounds__(kXpThreads, 1) xp_tc_kernel(const XpTcArgs a) 
       }
       tc::wait_st();
     } else if (w.H == 512) {
-      // half 0: units [0, 256) from R0; half 1: units [256, 512) from R1.  hi -> shared
-      // memory; lo -> packed in place at the start of the region read
-      const uint32_t src = half ? R1 : R0;
-      for (int cb = 0; cb < 8 && !bad; ++cb) {
-        uint32_t v[32], hi[16], lo[16];
-        tc::ld_x32(src + 32u * cb, v);
+      // This part's block of L1, units [256 part, 256 part + 256) in R0 [0, 256); half h
+      // takes [128 h, 128 h + 128) of it.  hi -> shared memory (the canonical [128][512]
+      // A operand of L2) and this CTA's exchange slot; lo -> the slot and registers.  Then
+      // the two parts of the tile swap halves through L2-resident memory: each takes the
+      // other's hi into shared memory, and every unit's lo goes to R0 packed (unit u at
+      // column u / 2) once all of R0 has been read.
+      uint32_t lo_keep[64];
+      uint4* const mine = reinterpret_cast<uint4*>(a.xch + (size_t)blockIdx.x * kXchSlot);
+      for (int cb = 0; cb < 4; ++cb) {
+        if (bad) break;
+        uint32_t v[32], hi[16];
+        tc::ld_x32(R0 + 128u * half + 32u * cb, v);
         tc::wait_ld();
 #pragma unroll
         for (int j = 0; j < 16; ++j)
           tc::split_bf16x2_p(tc::tanh2(tc::f2_pack(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]))),
-                             hi[j], lo[j]);
-        const int u0 = 256 * half + 32 * cb;
+                             hi[j], lo_keep[16 * cb + j]);
+        const int ub = 128 * half + 32 * cb;  // unit within the block
 #pragma unroll
-        for (int q = 0; q < 4; ++q)
-          *reinterpret_cast<uint4*>(sA + tc::canon_offset(row, u0 + 8 * q, 512)) =
-              make_uint4(hi[4 * q], hi[4 * q + 1], hi[4 * q + 2], hi[4 * q + 3]);
-        tc::st_x16(src + 16u * cb, lo);
+        for (int q = 0; q < 4; ++q) {
+          const uint4 h4 = make_uint4(hi[4 * q], hi[4 * q + 1], hi[4 * q + 2], hi[4 * q + 3]);
+          *reinterpret_cast<uint4*>(sA + tc::canon_offset(row, 256 * part + ub + 8 * q, 512)) = h4;
+          const int ch = ub / 8 + q;  // 8-unit chunk of the block
+          __stcg(mine + ch * 128 + row, h4);
+          __stcg(mine + (32 + ch) * 128 + row,
+                 make_uint4(lo_keep[16 * cb + 4 * q], lo_keep[16 * cb + 4 * q + 1], lo_keep[16 * cb + 4 * q + 2],
+                            lo_keep[16 * cb + 4 * q + 3]));
+        }
       }
-      tc::wait_st();
+      // publish this part's slot (2 stamp, or 2 stamp + 1 when it gave up), then take the
+      // partner's (bounded wait; a partner that gave up makes this part give up too)
       tc::fence_before_sync();
-      bad = sync_or();  // half 0 has read R0 [128, 256) before half 1 writes there
+      bad = sync_or();  // also: every thread has read its columns of R0
       tc::fence_after_sync();
-      if (!bad && half) {
-        for (int cb = 0; cb < 4; ++cb) {
+      const uint32_t partner = blockIdx.x ^ 1u;
+      if (tid == 0) {
+        xch_publish(a.xflag + blockIdx.x, 2u * a.xstamp + (bad ? 1u : 0u));
+        if (!bad && !xch_wait(a.xflag + partner, 2u * a.xstamp)) bad = true;
+      }
+      bad = sync_or();
+      if (!bad) {
+        const uint4* const theirs = reinterpret_cast<const uint4*>(a.xch + (size_t)partner * kXchSlot);
+        const int op = 1 - part;
+        // the partner's hi for units [256 op + 128 h, + 128) of this row
+#pragma unroll 4
+        for (int q = 0; q < 16; ++q)
+          *reinterpret_cast<uint4*>(sA + tc::canon_offset(row, 256 * op + 128 * half + 8 * q, 512)) =
+              __ldcg(theirs + (16 * half + q) * 128 + row);
+        // lo: this thread's own units -> columns [128 part + 64 h, + 64), the partner's
+        // units [256 op + 128 h, + 128) -> columns [128 op + 64 h, + 64)
+        tc::st_x32(R0 + 128u * part + 64u * half, *reinterpret_cast<const uint32_t(*)[32]>(lo_keep));
+        tc::st_x32(R0 + 128u * part + 64u * half + 32u, *reinterpret_cast<const uint32_t(*)[32]>(lo_keep + 32));
+#pragma unroll
+        for (int g2 = 0; g2 < 2; ++g2) {
           uint32_t v[32];
-          tc::ld_x32(R1 + 32u * cb, v);
-          tc::wait_ld();
-          tc::st_x32(R0 + 128u + 32u * cb, v);
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const uint4 l4 = __ldcg(theirs + (32 + 16 * half + 8 * g2 + q) * 128 + row);
+            v[4 * q] = l4.x, v[4 * q + 1] = l4.y, v[4 * q + 2] = l4.z, v[4 * q + 3] = l4.w;
+          }
+          tc::st_x32(R0 + 128u * op + 64u * half + 32u * g2, v);
         }
         tc::wait_st();
       }
@@ -770,11 +822,23 @@ cudaError_t launch_xp_tc(const XpTcArgs& a, int grid, size_t smem, cudaStream_t 
   cfg.blockDim = dim3(kXpThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  // the two parts of a tile wait on each other: a cluster of two makes them co-resident
+  cudaLaunchAttribute attr[2];
+  int n = 0;
+  if (a.parts == 2) {
+    attr[n].id = cudaLaunchAttributeClusterDimension;
+    attr[n].val.clusterDim.x = 2;
+    attr[n].val.clusterDim.y = 1;
+    attr[n].val.clusterDim.z = 1;
+    ++n;
+  }
+  if (a.s > 0) {
+    attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = a.s > 0 ? 1 : 0;
+  cfg.numAttrs = n;
   return cudaLaunchKernelEx(&cfg, xp_tc_kernel<Env>, a);
 }
 
