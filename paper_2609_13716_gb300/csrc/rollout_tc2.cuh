@@ -14,10 +14,10 @@
 // barrier), its first thread issues the layer's MMAs and commits them to the group's
 // accumulator barrier.  The groups share one observation buffer: the teammate's rows are
 // built first, and once they are in tensor memory the buffer passes to the ego (an
-// mbarrier); for gathered tiles the teammate group then writes the ego's rows to the
-// trajectory while the ego finishes its chain.  Both groups meet twice per step on a
-// named barrier that also ORs their error flags: once both actions exist (then the ego
-// group steps the envs) and once the new state is in shared memory.  Every mbarrier wait
+// mbarrier).  Both groups meet twice per step on a named barrier that also ORs their
+// error flags: once both actions exist (then the ego group's first half steps the envs
+// while, for gathered tiles, the teammate group and the ego's second half write the ego's
+// rows to the trajectory) and once the new state is in shared memory.  Every mbarrier wait
 // is bounded (2 s): on expiry the CTA records kStatusTimeout, stops, waits (bounded) for
 // its own MMAs, frees tensor memory and exits.
 #pragma once
@@ -40,7 +40,6 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
   __shared__ __align__(8) uint64_t acc_bar[4];     // [2*agent + layer], tcgen05.commit
   __shared__ __align__(8) uint64_t wload_bar[2], drain_bar[2];  // per agent
   __shared__ __align__(8) uint64_t buf_free;       // teammate rows in tensor memory (256)
-  __shared__ __align__(8) uint64_t rows_ready;     // ego rows built (256; gathered copy)
   __shared__ __align__(8) uint64_t never_bar;      // test hook: nothing arrives on it
   __shared__ uint32_t tmem_slot;
   const TcDims& d = a.tc;
@@ -58,7 +57,6 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
       tc::mbar_init(&drain_bar[i], 1);
     }
     tc::mbar_init(&buf_free, kT2Group);
-    tc::mbar_init(&rows_ready, kT2Group);
     tc::mbar_init(&never_bar, 1);
     tc::mbar_init_fence();
     // the ego's policy block -> shared memory, waited for by the ego group
@@ -101,7 +99,7 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
   const int my_c0 = half ? split : 0, my_c1 = half ? chunks : split;
   const int my_w0 = min(4 * my_c0, cells), my_w1 = min(4 * my_c1, cells);
   const bool with_boot = a.traj.last_value != nullptr;
-  const bool obs_copy = kGather && a.traj.obs != nullptr;  // the teammate group stores the rows
+  const bool obs_copy = kGather && a.traj.obs != nullptr;  // 12 warps store the rows during the step
 
   uint8_t* const sW0 = smem;                                                // policy blocks
   uint8_t* const sObs = smem + 2 * d.pol_bytes;                             // [128][obs_dim] u8
@@ -316,29 +314,21 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
         for (uint32_t w = tid; w < bytes / 4; w += kT2Group) d32[w] = src[w];
       }
     };
-    // gathered tiles: the ego's rows -> their envs' trajectory rows, by the teammate group
-    // (warp 8 + q takes rows q, q + 8, ...; lane l word w0 + l; 4 rows in flight)
-    auto copy_rows_gathered = [&](int t) {
-      const int q = warp - 8;
+    // gathered tiles: the ego's rows -> their envs' trajectory rows, while the ego group's
+    // first half steps the envs: the 12 warps of the teammate group and of the ego's
+    // second half take the tile's count x cells words in turn (consecutive lanes,
+    // consecutive words of a row; row = word / cells by a reciprocal multiply, exact for
+    // fewer than 2^16 words)
+    const uint32_t cells_rcp = 0xFFFFFFFFu / (uint32_t)cells + 1u;
+    auto copy_rows_gathered = [&](int t, int cw) {
+      constexpr int kCopyWarps = 12;
       uint32_t* const base = reinterpret_cast<uint32_t*>(a.traj.obs + (int64_t)t * N * od);
       const uint32_t* const src = reinterpret_cast<const uint32_t*>(sObs);
-      for (int w0 = 0; w0 < cells; w0 += 32) {
-        const int w = w0 + lane;
-        const bool wok = w < cells;
-#pragma unroll 1
-        for (int r0 = q; r0 < count; r0 += 8 * 4) {
-          uint32_t v[4];
-          int64_t dst[4];
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const int r = min(r0 + 8 * j, count - 1);
-            dst[j] = (int64_t)rowenv[r] * cells + w;
-            v[j] = wok ? src[r * cells + w] : 0u;
-          }
-#pragma unroll
-          for (int j = 0; j < 4; ++j)
-            if (wok && r0 + 8 * j < count) base[dst[j]] = v[j];
-        }
+      const int total = count * cells;
+#pragma unroll 4
+      for (int f = cw * 32 + lane; f < total; f += kCopyWarps * 32) {
+        const int r = (int)__umulhi((uint32_t)f, cells_rcp);
+        base[(int64_t)rowenv[r] * cells + (f - r * cells)] = src[f];
       }
     };
 
@@ -378,10 +368,6 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
             act1s[row] = (uint8_t)sample_k<NA>(z, 0xFFFFFFFFu >> (32 - NA), u_act, lp);
           }
         }
-        if (obs_copy && !boot) {
-          wait_bar(&rows_ready, par);
-          if (!bad) copy_rows_gathered(t);
-        }
       } else {
         // ------------------------------- ego group ---------------------------------
         wait_bar(&buf_free, par);
@@ -389,10 +375,7 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
         // contiguous tiles: the rows (ordinary stores) are read by the bulk copy engine
         if (!kGather && !boot && a.traj.obs) tc::fence_proxy_async();
         issue(0);  // (its group barrier also orders the rows before the copy)
-        if (!boot && a.traj.obs) {
-          if constexpr (kGather) tc::mbar_arrive(&rows_ready);
-          else copy_rows_contiguous(t);
-        }
+        if (!kGather && !boot && a.traj.obs) copy_rows_contiguous(t);
         if (t == a.dbg_expire_step) {  // test hook: an accumulator wait that never completes
           if (!bad && !tc::mbar_wait(&never_bar, 0, a.dbg_expire_ns)) bad = true;
           bad = __any_sync(0xFFFFFFFFu, bad);
@@ -454,6 +437,7 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
         const unsigned m = __ballot_sync(0xFFFFFFFFu, stayed);
         if (lane == 0 && m) atomicAdd(&a.g.hist_next[g_k], __popc(m));
       }
+      if (obs_copy && (ag == 1 || half == 1)) copy_rows_gathered(t, ag == 1 ? warp - 8 : warp + 4);
       if (tid == 0 && bulk_obs) tc::bulk_wait_read();  // the rows may be rebuilt
       if (sync_all()) break;                            // the new state is in place
     }
