@@ -232,39 +232,49 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
       const uint32_t* W3l = W3f + H * 4;
       const int g = lane >> 2, c4 = lane & 3;
       float zacc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+      // two 16-unit chunks (both row groups of each) under one wait: 16 independent pairs;
+      // each row group accumulates chunk by chunk, hi then lo, as in ppo_tc_kernel
 #pragma unroll 1
-      for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 16) {
-        const int j = c0 >> 4;
-        const uint2 bw = *reinterpret_cast<const uint2*>(W3f + (j * 32 + lane) * 2);
-        const uint64_t bA = *reinterpret_cast<const uint64_t*>(b2 + c0 + 2 * c4);
-        const uint64_t bB = *reinterpret_cast<const uint64_t*>(b2 + c0 + 8 + 2 * c4);
-        uint2 bl = make_uint2(0u, 0u);
-        if constexpr (kSplit) bl = *reinterpret_cast<const uint2*>(W3l + (j * 32 + lane) * 2);
-        // both row groups' fragments under one wait: 8 independent pairs
-        uint32_t tt[2][2][4];
+      for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 32) {
+        uint32_t tt[2][2][2][4];  // [chunk][row group][column half][fragment]
 #pragma unroll
-        for (int rg = 0; rg < 2; ++rg) {
-          tc::ld_16x256b(Qq + ((uint32_t)(16 * rg) << 16) + (uint32_t)c0, tt[rg][0]);
-          tc::ld_16x256b(Qq + ((uint32_t)(16 * rg) << 16) + (uint32_t)(c0 + 8), tt[rg][1]);
+        for (int cc = 0; cc < 2; ++cc)
+#pragma unroll
+          for (int rg = 0; rg < 2; ++rg) {
+            tc::ld_16x256b(Qq + ((uint32_t)(16 * rg) << 16) + (uint32_t)(c0 + 16 * cc), tt[cc][rg][0]);
+            tc::ld_16x256b(Qq + ((uint32_t)(16 * rg) << 16) + (uint32_t)(c0 + 16 * cc + 8), tt[cc][rg][1]);
+          }
+        uint2 bw[2], bl[2];
+        uint64_t bA[2], bB[2];
+#pragma unroll
+        for (int cc = 0; cc < 2; ++cc) {
+          const int j = (c0 >> 4) + cc, u0 = c0 + 16 * cc;
+          bw[cc] = *reinterpret_cast<const uint2*>(W3f + (j * 32 + lane) * 2);
+          bl[cc] = make_uint2(0u, 0u);
+          if constexpr (kSplit) bl[cc] = *reinterpret_cast<const uint2*>(W3l + (j * 32 + lane) * 2);
+          bA[cc] = *reinterpret_cast<const uint64_t*>(b2 + u0 + 2 * c4);
+          bB[cc] = *reinterpret_cast<const uint64_t*>(b2 + u0 + 8 + 2 * c4);
         }
         tc::wait_ld();
 #pragma unroll
-        for (int rg = 0; rg < 2; ++rg) {
-          const uint32_t (&t0)[4] = tt[rg][0];
-          const uint32_t (&t1)[4] = tt[rg][1];
-          uint32_t ahi[4], alo[4];
-          tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t0[0]), __uint_as_float(t0[1])), tc::kTwoOverLn2x2, bA)),
-                             ahi[0], alo[0]);
-          tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t0[2]), __uint_as_float(t0[3])), tc::kTwoOverLn2x2, bA)),
-                             ahi[1], alo[1]);
-          tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t1[0]), __uint_as_float(t1[1])), tc::kTwoOverLn2x2, bB)),
-                             ahi[2], alo[2]);
-          tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t1[2]), __uint_as_float(t1[3])), tc::kTwoOverLn2x2, bB)),
-                             ahi[3], alo[3]);
-          tc::mma_m16n8k16_bf16(zacc[rg], ahi, bw.x, bw.y);
-          tc::mma_m16n8k16_bf16(zacc[rg], alo, bw.x, bw.y);
-          if constexpr (kSplit) tc::mma_m16n8k16_bf16(zacc[rg], ahi, bl.x, bl.y);
-        }
+        for (int cc = 0; cc < 2; ++cc)
+#pragma unroll
+          for (int rg = 0; rg < 2; ++rg) {
+            const uint32_t (&t0)[4] = tt[cc][rg][0];
+            const uint32_t (&t1)[4] = tt[cc][rg][1];
+            uint32_t ahi[4], alo[4];
+            tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t0[0]), __uint_as_float(t0[1])), tc::kTwoOverLn2x2, bA[cc])),
+                               ahi[0], alo[0]);
+            tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t0[2]), __uint_as_float(t0[3])), tc::kTwoOverLn2x2, bA[cc])),
+                               ahi[1], alo[1]);
+            tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t1[0]), __uint_as_float(t1[1])), tc::kTwoOverLn2x2, bB[cc])),
+                               ahi[2], alo[2]);
+            tc::split_bf16x2_p(tc::logistic2(tc::f2_fma(tc::f2_pack(__uint_as_float(t1[2]), __uint_as_float(t1[3])), tc::kTwoOverLn2x2, bB[cc])),
+                               ahi[3], alo[3]);
+            tc::mma_m16n8k16_bf16(zacc[rg], ahi, bw[cc].x, bw[cc].y);
+            tc::mma_m16n8k16_bf16(zacc[rg], alo, bw[cc].x, bw[cc].y);
+            if constexpr (kSplit) tc::mma_m16n8k16_bf16(zacc[rg], ahi, bl[cc].x, bl[cc].y);
+          }
       }
       float* zp = zpart + (ag * 2 + half) * 128 * 8;
 #pragma unroll
@@ -339,7 +349,11 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
       if (boot && !with_boot) break;
       const uint32_t par = (uint32_t)t & 1u, gt = a.step0 + (uint32_t)t;
       const bool sampler = half == 0 && row < count && !boot;
-      const float u_act = sampler ? u01(draw0(a.b.key, (uint32_t)my_env, gt, kStreamAct0 + ag)) : 0.0f;
+      // this step's action draw (Philox), computed while L1 runs on the tensor cores
+      float u_act = 0.0f;
+      auto draw_action = [&]() {
+        if (sampler) u_act = u01(draw0(a.b.key, (uint32_t)my_env, gt, kStreamAct0 + ag));
+      };
       const State s = st[row];  // register copy for this step (rows past count are never used)
       float z[16];
       int act0 = 0;
@@ -351,6 +365,7 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
         tc::mbar_arrive(&buf_free);  // its rows are in tensor memory: the buffer is the ego's
         if (run) {
           issue(0);
+          draw_action();
           wait_acc(0, par);
           if (!bad) epilogue1();
           issue(1);
@@ -375,6 +390,7 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
         // contiguous tiles: the rows (ordinary stores) are read by the bulk copy engine
         if (!kGather && !boot && a.traj.obs) tc::fence_proxy_async();
         issue(0);  // (its group barrier also orders the rows before the copy)
+        draw_action();
         if (!kGather && !boot && a.traj.obs) copy_rows_contiguous(t);
         if (t == a.dbg_expire_step) {  // test hook: an accumulator wait that never completes
           if (!bad && !tc::mbar_wait(&never_bar, 0, a.dbg_expire_ns)) bad = true;
