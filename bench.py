@@ -329,10 +329,11 @@ def run_ours(args):
     aht.aht_sync(ctx)
 
     # ---- end to end: ego weights from pinned host memory in, whole trajectory out ------
-    # Two trajectory buffers, as a user would double-buffer: step k's trajectory is copied
-    # to pinned host memory on a copy stream while step k + 1 runs on the library's
-    # stream.  Every step's upload and download lies inside the timed region, which ends
-    # when the last download has landed.
+    # Through the library's API: aht_set_policy uploads the ego's weights, aht_rollout
+    # collects, aht_traj_copy downloads.  Two trajectory buffers, as a user would
+    # double-buffer: step k's trajectory is copied to pinned host memory on a copy stream
+    # while step k + 1 runs on the library's stream.  Every step's upload and download
+    # lies inside the timed region, which ends when the last download has landed.
     ego_host = [(W_.to(torch.bfloat16).cpu().pin_memory(), b.to(torch.bfloat16).cpu().pin_memory())
                 for W_, b in [(torch.from_numpy(a), torch.from_numpy(c)) for a, c in pop_np[wl.ego_id]]]
     e2e_ms = []
@@ -353,9 +354,7 @@ def run_ours(args):
             aht.aht_rollout(ctx, wl.ego_id, wl.pool, T, trajs[b], wl.gamma, wl.lam)
             rolled[b].record(stream)
             copy_stream.wait_event(rolled[b])
-            with torch.cuda.stream(copy_stream):
-                for key, hv in hosts[b].items():
-                    hv.copy_(trajs[b][key], non_blocking=True)
+            aht.aht_traj_copy(trajs[b], hosts[b], N, T, wl.env.obs_dim, copy_stream)
             copied[b].record(copy_stream)
 
         for k in range(2):

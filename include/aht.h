@@ -416,6 +416,21 @@ aht_status aht_gae(const float* rewards, const float* values, const uint8_t* don
                    const float* v_last, int64_t n_envs, int32_t T, float gamma, float lambda,
                    float* advantages, float* targets, void* cuda_stream);
 
+/* Copies a collected trajectory from one set of caller-owned buffers to another: from the
+ * device buffers aht_rollout wrote to pinned host buffers for a learner or a logger on
+ * the host, or between device buffers (not in the paper: a transfer helper of this
+ * library).  Every field that is non-NULL in both src and dst is copied in full: obs
+ * [T][n_envs][obs_dim] u8, actions / tm_actions / dones [T][n_envs] u8, logp / values /
+ * rewards / advantages / targets [T][n_envs] fp32, last_value [n_envs] fp32, teammate
+ * [n_envs] int32; gamma and lambda are not read.  One cudaMemcpyAsync per field, in
+ * this order, enqueued on cuda_stream (a cudaStream_t, NULL = default; the direction
+ * follows from the pointers, and pageable host memory makes a copy synchronous); the
+ * caller orders the copies after the call that wrote src (same stream, or an event).
+ * AHT_EINVAL for NULL src / dst or sizes below 1, AHT_ECUDA if an enqueue fails.
+ * Allocates nothing. */
+aht_status aht_traj_copy(const aht_traj* src, const aht_traj* dst, int64_t n_envs, int32_t T,
+                         int32_t obs_dim, void* cuda_stream);
+
 /* Replaces the weights of one policy (App. C: PPO updates the ego between rollout
  * collections).  W[l] / b[l] (l = 0..2) have the shapes of aht_pop_desc for this policy,
  * in host or device memory of weight_dtype; has_value_head as in aht_pop_desc.  The

@@ -27,7 +27,7 @@ EXPORTED = ["aht_create", "aht_destroy", "aht_reset", "aht_rollout", "aht_xplay_
             "aht_xp_stats", "aht_learner_create", "aht_learner_destroy", "aht_learner_n_params",
             "aht_ppo_update", "aht_ppo_grad", "aht_learner_get", "aht_learner_set",
             "aht_learner_push", "aht_learner_sync", "aht_rollout_ippo", "aht_rollout_resample",
-            "aht_s5_create", "aht_s5_destroy", "aht_s5_step", "aht_s5_sync"]
+            "aht_s5_create", "aht_s5_destroy", "aht_s5_step", "aht_s5_sync", "aht_traj_copy"]
 
 
 class AhtError(RuntimeError):
@@ -121,6 +121,7 @@ def load() -> C.CDLL:
             L.aht_rollout_resample.argtypes = [vp, i32, C.POINTER(i32), i32, i32, C.POINTER(Traj), vp]
             L.aht_xplay_matrix.argtypes = [vp, C.POINTER(i32), i32, C.POINTER(i32), i32, i32, i32, C.POINTER(XplayOut)]
             L.aht_gae.argtypes = [vp, vp, vp, vp, i64, i32, C.c_float, C.c_float, vp, vp, vp]
+            L.aht_traj_copy.argtypes = [C.POINTER(Traj), C.POINTER(Traj), i64, i32, i32, vp]
             L.aht_xp_stats.argtypes = [vp, i32, i32, vp, C.POINTER(XpStatsOut), vp]
             L.aht_step_forced.argtypes = [vp, vp, C.POINTER(StepOut)]
             L.aht_learner_create.argtypes = [i32, i32, C.POINTER(vp), C.POINTER(vp), C.POINTER(PpoConfig),
@@ -348,6 +349,37 @@ def aht_gae(rewards, values, dones, v_last, gamma, lam, advantages, targets=None
                           _ptr(dones, torch.uint8, (T, N), "dones"), _ptr(v_last, f32, (N,), "v_last"),
                           N, T, gamma, lam, _ptr(advantages, f32, (T, N), "advantages"),
                           _ptr(targets, f32, (T, N), "targets"), _stream(stream)))
+
+
+def _ptr_pinned_or_cuda(t, dtype, shape, name):
+    """A CUDA tensor, or a pinned host tensor (the trajectory copy's host side)."""
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor) or not (t.is_cuda or t.is_pinned()):
+        raise TypeError(f"{name} must be a CUDA tensor or a pinned host tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+    return t.data_ptr()
+
+
+def aht_traj_copy(src: dict, dst: dict, n_envs: int, T: int, obs_dim: int, stream=None):
+    """Copies every trajectory field present in both ``src`` and ``dst`` (dicts as from
+    traj_buffers; CUDA or pinned host tensors), enqueued on ``stream``."""
+    f32, u8 = torch.float32, torch.uint8
+    shapes = dict(obs=((T, n_envs, obs_dim), u8), actions=((T, n_envs), u8), tm_actions=((T, n_envs), u8),
+                  logp=((T, n_envs), f32), values=((T, n_envs), f32), rewards=((T, n_envs), f32),
+                  dones=((T, n_envs), u8), advantages=((T, n_envs), f32), targets=((T, n_envs), f32),
+                  last_value=((n_envs,), f32), teammate=((n_envs,), torch.int32))
+
+    def side(d):
+        return Traj(*[_ptr_pinned_or_cuda(d.get(k), dt, sh, k) for k, (sh, dt) in shapes.items()], 0.0, 0.0)
+
+    a, b = side(src), side(dst)
+    _check(load().aht_traj_copy(C.byref(a), C.byref(b), n_envs, T, obs_dim, _stream(stream)))
 
 
 def aht_xp_stats(xp, upper, norm=None, regret=None, j_aht=None, j_norm=None, max_regret=None,

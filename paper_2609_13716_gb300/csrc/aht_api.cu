@@ -1380,6 +1380,30 @@ aht_status aht_xplay_matrix_static(aht_ctx* c, const int32_t* ego_ids, int32_t n
   return AHT_OK;
 }
 
+aht_status aht_traj_copy(const aht_traj* src, const aht_traj* dst, int64_t n_envs, int32_t T,
+                         int32_t obs_dim, void* cuda_stream) {
+  if (!src || !dst) return fail(AHT_EINVAL, "src or dst is NULL");
+  if (n_envs < 1 || T < 1 || obs_dim < 1) return fail(AHT_EINVAL, "n_envs, T and obs_dim must be >= 1");
+  const cudaStream_t st = (cudaStream_t)cuda_stream;
+  const size_t steps = (size_t)T * (size_t)n_envs;
+  auto copy = [&](void* to, const void* from, size_t bytes) -> bool {
+    if (!to || !from) return true;
+    return cudaMemcpyAsync(to, from, bytes, cudaMemcpyDefault, st) == cudaSuccess;
+  };
+  const bool ok = copy(dst->obs, src->obs, steps * (size_t)obs_dim) &&
+                  copy(dst->actions, src->actions, steps) && copy(dst->tm_actions, src->tm_actions, steps) &&
+                  copy(dst->logp, src->logp, steps * 4) && copy(dst->values, src->values, steps * 4) &&
+                  copy(dst->rewards, src->rewards, steps * 4) && copy(dst->dones, src->dones, steps) &&
+                  copy(dst->advantages, src->advantages, steps * 4) && copy(dst->targets, src->targets, steps * 4) &&
+                  copy(dst->last_value, src->last_value, (size_t)n_envs * 4) &&
+                  copy(dst->teammate, src->teammate, (size_t)n_envs * 4);
+  if (!ok) {
+    const cudaError_t e = cudaGetLastError();
+    return fail(AHT_ECUDA, std::string("cudaMemcpyAsync: ") + cudaGetErrorString(e));
+  }
+  return AHT_OK;
+}
+
 aht_status aht_gae(const float* r, const float* v, const uint8_t* d, const float* v_last,
                    int64_t n_envs, int32_t T, float gamma, float lambda, float* adv,
                    float* tgt, void* cuda_stream) {

@@ -53,6 +53,9 @@ def test_host_validation_needs_no_gpu(lib):
     assert L.aht_create(C.byref(bad), None, 4, 0, None, C.byref(h)) == aht.AHT_EINVAL
     assert b"width" in L.aht_last_error()
     assert L.aht_gae(None, None, None, None, 1, 1, 0.9, 0.9, None, None, None) == aht.AHT_EINVAL
+    t = aht.Traj()
+    assert L.aht_traj_copy(None, C.byref(t), 1, 1, 1, None) == aht.AHT_EINVAL
+    assert L.aht_traj_copy(C.byref(t), C.byref(t), 0, 1, 1, None) == aht.AHT_EINVAL
     L.aht_debug_expire_wait.argtypes = [C.c_void_p, C.c_int64]
     assert L.aht_debug_expire_wait(None, 1000) == aht.AHT_EINVAL
     assert L.aht_debug_obs_words(None, 0, None) == aht.AHT_EINVAL

@@ -163,3 +163,30 @@ def test_per_call_teammate_groups_edge_cases(N, pool):
     aht.aht_rollout(ctx, 0, pool, T, traj)
     aht.aht_sync(ctx)
     check_rollout(wl, pop_np, traj, st, wl.env_seed, 0, T, 0, pool)
+
+
+def test_traj_copy_to_pinned_host_and_device():
+    # aht_traj_copy (the API's trajectory download) delivers every field bit for bit, to
+    # pinned host buffers and to another set of device buffers; a field missing on either
+    # side is skipped.
+    require_gpu()
+    wl = W.WORKLOADS["lbf7x7_ppo_16384x128"]
+    N, T = 300, 12
+    ctx, _ = make_ctx(wl, N)
+    traj = aht.traj_buffers(ctx, T)
+    aht.aht_rollout(ctx, 0, wl.pool, T, traj, 0.99, 0.95)
+    host = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in traj.items()}
+    host["targets"] = None
+    dev = aht.traj_buffers(ctx, T)
+    stream = torch.cuda.Stream()
+    stream.wait_stream(torch.cuda.current_stream())
+    aht.aht_sync(ctx)
+    aht.aht_traj_copy(traj, host, N, T, ctx.obs_dim, stream)
+    aht.aht_traj_copy(traj, dev, N, T, ctx.obs_dim, stream)
+    stream.synchronize()
+    for k, v in traj.items():
+        if host[k] is not None:
+            assert torch.equal(host[k], v.cpu()), k
+        assert torch.equal(dev[k].cpu(), v.cpu()), k
+    with pytest.raises(ValueError):  # the binding checks the shapes (the C call: test_abi)
+        aht.aht_traj_copy(traj, host, 0, T, ctx.obs_dim, stream)
