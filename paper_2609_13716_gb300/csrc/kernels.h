@@ -293,6 +293,7 @@ AHT_DECLARE_ENV_LAUNCHERS(minihanabi)
 cudaError_t lbf_ppo_tc(const PpoTcArgs&, int grid, size_t smem, cudaStream_t);
 // plain collection with a dense first layer, one warp group per agent (rollout_lbf2.cu)
 cudaError_t lbf_ppo_tc2(const PpoTcArgs&, int grid, size_t smem, cudaStream_t);
+cudaError_t lbf_xplay_tc2(const PpoTcArgs&, int grid, size_t smem, cudaStream_t);
 cudaError_t lbf_xplay_tc(const PpoTcArgs&, int grid, size_t smem, cudaStream_t);
 
 // Streamed tensor-core cross-play step (rollout_overcooked.cu, rollout_hanabi.cu).

@@ -16,6 +16,8 @@ cudaError_t lbf_ppo_tc(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s
 }
 
 cudaError_t lbf_xplay_tc(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
+  // a dense first layer: one warp group per agent (rollout_tc2.cuh)
+  if (!a.tc.sparse) return lbf_xplay_tc2(a, grid, smem, s);
   return LaunchTc<EnvLbf>::xplay(a, grid, smem, s);
 }
 }  // namespace aht

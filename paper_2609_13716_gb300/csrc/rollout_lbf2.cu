@@ -6,4 +6,7 @@ namespace aht {
 cudaError_t lbf_ppo_tc2(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
   return LaunchTc2<EnvLbf>::ppo(a, grid, smem, s);
 }
+cudaError_t lbf_xplay_tc2(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
+  return LaunchTc2<EnvLbf>::xplay(a, grid, smem, s);
+}
 }  // namespace aht

@@ -31,7 +31,11 @@ constexpr int kT2AllBar = 1;      // named barrier ids: both groups (OR of the e
 constexpr int kT2GroupBar = 2;    // 2 + g: group g
 constexpr int kT2PairBar = 4;     // 4 + 4 g + q: warps 8 g + q and 8 g + q + 4 (rows 32 q ..)
 
-template <class Env, bool kSplit, bool kGather>
+// kXp: cross-play instead of collection -- a tile is up to 128 envs of one pair (ego i,
+// teammate j), reset at the call's first step and frozen once its first episode ends; the
+// CTA stops when every env of the tile is done and writes each env's return and length
+// (NaN returns if it gave up); no trajectory.
+template <class Env, bool kSplit, bool kGather, bool kXp>
 __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs a) {
   using State = typename Env::State;
   constexpr int NA = Env::kNumActions;
@@ -59,11 +63,14 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
     tc::mbar_init(&buf_free, kT2Group);
     tc::mbar_init(&never_bar, 1);
     tc::mbar_init_fence();
-    // the ego's policy block -> shared memory, waited for by the ego group
-    const uint8_t* src = a.tcw + (int64_t)a.ego * d.pol_bytes;
-    tc::mbar_expect_tx(&wload_bar[0], d.pol_bytes);
-    for (uint32_t off = 0; off < d.pol_bytes; off += 32768u)
-      tc::bulk_g2s(smem + off, src + off, min(32768u, d.pol_bytes - off), &wload_bar[0]);
+    // the ego's policy block -> shared memory, waited for by the ego group (collection:
+    // the same ego for every tile; cross-play: once the tile is known, below)
+    if (!kXp) {
+      const uint8_t* src = a.tcw + (int64_t)a.ego * d.pol_bytes;
+      tc::mbar_expect_tx(&wload_bar[0], d.pol_bytes);
+      for (uint32_t off = 0; off < d.pol_bytes; off += 32768u)
+        tc::bulk_g2s(smem + off, src + off, min(32768u, d.pol_bytes - off), &wload_bar[0]);
+    }
   }
   if (warp == 0) tc::tmem_alloc(&tmem_slot, 512);
   tc::fence_before_sync();
@@ -72,9 +79,16 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
   asm volatile("griddepcontrol.wait;" ::: "memory");
 
   int32_t* const rowenv = kGather ? reinterpret_cast<int32_t*>(smem + a.g.scratch_off) : nullptr;
-  const TcTile tile = tc_find_tile<false, kGather>(a, rowenv);
+  static_assert(!(kXp && kGather), "cross-play tiles are contiguous");
+  const TcTile tile = tc_find_tile<kXp, kGather>(a, rowenv);
   const int64_t env0 = tile.env0;
   const int count = tile.count, tm_pol = tile.tm_pol, g_k = tile.g_k;
+  if (kXp && tid == 0) {  // cross-play: this tile's ego
+    const uint8_t* src = a.tcw + (int64_t)tile.ego_pol * d.pol_bytes;
+    tc::mbar_expect_tx(&wload_bar[0], d.pol_bytes);
+    for (uint32_t off = 0; off < d.pol_bytes; off += 32768u)
+      tc::bulk_g2s(smem + off, src + off, min(32768u, d.pol_bytes - off), &wload_bar[0]);
+  }
   if (count <= 0) {  // no rows: the ego's copy lands, then tensor memory is freed
     if (tid == 0) tc::mbar_wait(&wload_bar[0], 0);
     tc::fence_before_sync();
@@ -98,7 +112,7 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
   const int split = (chunks + 1) / 2;
   const int my_c0 = half ? split : 0, my_c1 = half ? chunks : split;
   const int my_w0 = min(4 * my_c0, cells), my_w1 = min(4 * my_c1, cells);
-  const bool with_boot = a.traj.last_value != nullptr;
+  const bool with_boot = !kXp && a.traj.last_value != nullptr;
   const bool obs_copy = kGather && a.traj.obs != nullptr;  // 12 warps store the rows during the step
 
   uint8_t* const sW0 = smem;                                                // policy blocks
@@ -108,7 +122,10 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
   float* zpart = reinterpret_cast<float*>(act1s + 128);                     // [2][2][128][8]
 
   for (int i = tid; i < 32 * od; i += blockDim.x) reinterpret_cast<uint32_t*>(sObs)[i] = 0u;
-  if (tid < count) load_state(a.state, N, env_of(tid), st[tid]);
+  if (tid < count) {
+    if constexpr (kXp) Env::reset(a.b.env, a.b.key, (uint32_t)(env0 + tid), a.step0, st[tid]);
+    else load_state(a.state, N, env_of(tid), st[tid]);
+  }
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
@@ -303,7 +320,8 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
     // test hook: this row's outputs of step t
     auto dbg_store = [&](int t, const float (&z)[16]) {
       if (!a.dbg_logits) return;
-      float* p = a.dbg_logits + (((int64_t)t * N + my_env) * 2 + ag) * kDbgStride;
+      const int64_t rows = kXp ? a.xp.n_total : N;
+      float* p = a.dbg_logits + (((int64_t)t * rows + my_env) * 2 + ag) * kDbgStride;
 #pragma unroll
       for (int o = 0; o < 8; ++o) p[o] = z[o];
     };
@@ -343,10 +361,15 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
     };
 
     // Steps 0..T-1, then (if requested) the ego's V_T of the state after the last step.
-    const int n_steps = a.T;
+    const int n_steps = kXp ? a.xp.max_steps : a.T;
+    bool alive = true;  // cross-play: the row's episode is running (ego group, first half)
+    int nsteps = 0;
     for (int t = 0; t <= n_steps; ++t) {
       const bool boot = t == n_steps;
       if (boot && !with_boot) break;
+      if constexpr (kXp) {  // every env of the tile is done: stop (no MMA is in flight)
+        if (!tc::bar_or(kT2AllBar, kT2Threads, ag == 0 && half == 0 && row < count && alive)) break;
+      }
       const uint32_t par = (uint32_t)t & 1u, gt = a.step0 + (uint32_t)t;
       const bool sampler = half == 0 && row < count && !boot;
       // this step's action draw (Philox), computed while L1 runs on the tensor cores
@@ -416,7 +439,25 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
       }
       if (sync_all() || boot) break;  // both actions exist
       bool stayed = false;            // per-episode gather: the env keeps its teammate
-      if (ag == 0 && half == 0 && row < count) {
+      if (kXp && ag == 0 && half == 0 && row < count && alive) {
+        State s2 = s;
+        const int act1 = act1s[row];
+        if (a.xp.actions) {
+          uint8_t* rec = a.xp.actions + ((int64_t)t * a.xp.n_total + my_env) * 2;
+          rec[0] = (uint8_t)act0;
+          rec[1] = (uint8_t)act1;
+        }
+        float r0, r1, team;
+        const int done = Env::step(a.b.env, s2, act0, act1, r0, r1, team);
+        if (done < 0) {
+          atomicOr(a.b.status, kStatusIllegalAction);
+          alive = false;
+        } else {
+          nsteps += 1;
+          if (done) alive = false;
+        }
+        st[row] = s2;
+      } else if (!kXp && ag == 0 && half == 0 && row < count) {
         State s2 = s;
         const int act1 = act1s[row];
         const int64_t env = my_env;
@@ -460,9 +501,17 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
     if (tid == 0 && bulk_obs) tc::bulk_wait_all();
     if (bad) {
       atomicOr(a.b.status, kStatusTimeout);
+      // cross-play: the tile gave up, so its returns are undefined; NaN (not a stale entry
+      // of an earlier call) makes every mean over them NaN
+      if (kXp && tid < count) a.xp.returns[env0 + tid] = __int_as_float(0x7FC00000);
     } else if (tid < count) {
-      store_state(a.state, N, env_of(tid), st[tid]);
+      if constexpr (kXp) {
+        a.xp.returns[env0 + tid] = Env::ret(st[tid]);
+      } else {
+        store_state(a.state, N, env_of(tid), st[tid]);
+      }
     }
+    if (kXp && a.xp.steps && !bad && ag == 0 && half == 0 && row < count) a.xp.steps[env0 + row] = nsteps;
     // ---- drain: every MMA this thread issued completes (bounded) ----
     if (leader && n_issued > 0) {
       tc::commit(&drain_bar[ag]);
@@ -481,9 +530,9 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
 
 template <class Env>
 struct LaunchTc2 {
-  template <bool kSplit, bool kGather>
+  template <bool kSplit, bool kGather, bool kXp = false>
   static cudaError_t run(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
-    cudaError_t e = cudaFuncSetAttribute(ppo2_tc_kernel<Env, kSplit, kGather>,
+    cudaError_t e = cudaFuncSetAttribute(ppo2_tc_kernel<Env, kSplit, kGather, kXp>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
@@ -496,7 +545,11 @@ struct LaunchTc2 {
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = a.pdl ? 1 : 0;
-    return cudaLaunchKernelEx(&cfg, ppo2_tc_kernel<Env, kSplit, kGather>, a);
+    return cudaLaunchKernelEx(&cfg, ppo2_tc_kernel<Env, kSplit, kGather, kXp>, a);
+  }
+  // cross-play (dense first layer)
+  static cudaError_t xplay(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
+    return a.tc.split ? run<true, false, true>(a, grid, smem, s) : run<false, false, true>(a, grid, smem, s);
   }
   // plain PPO collection (no IPPO, dense first layer)
   static cudaError_t ppo(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
