@@ -181,6 +181,11 @@ struct EnvLbf {
     return mask;
   }
 
+  // The other seat's view of one cell word of the observation: channels 0 (the observing
+  // agent's level) and 1 (the other agent's level) trade places; the food and empty
+  // channels do not depend on the seat.
+  __device__ static uint32_t other_seat_word(uint32_t w) { return __byte_perm(w, 0u, 0x3201); }
+
   // Words [w0, w1) of the same row (w1 <= cells): one cell per word.
   __device__ static void obs_words(const DevEnv& d, const State& s, int seat, uint32_t* w, int w0,
                                    int w1) {

@@ -10,8 +10,9 @@ cudaError_t lbf_ppo_tc(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s
   const TrajPtrs& u = a.traj1;
   const bool ippo = u.obs || u.actions || u.tm_actions || u.logp || u.values || u.rewards ||
                     u.dones || u.last_value;
-  // plain collection with a dense first layer: one warp group per agent (rollout_tc2.cuh)
-  if (!ippo && !a.tc.sparse) return lbf_ppo_tc2(a, grid, smem, s);
+  // collection with a dense first layer (plain, or IPPO on contiguous tiles): one warp
+  // group per agent (rollout_tc2.cuh)
+  if (!a.tc.sparse && (!ippo || !a.gather)) return lbf_ppo_tc2(a, grid, smem, s);
   return LaunchTc<EnvLbf>::ppo(a, grid, smem, s);
 }
 

@@ -35,7 +35,11 @@ constexpr int kT2PairBar = 4;     // 4 + 4 g + q: warps 8 g + q and 8 g + q + 4 
 // teammate j), reset at the call's first step and frozen once its first episode ends; the
 // CTA stops when every env of the tile is done and writes each env's return and length
 // (NaN returns if it gave up); no trajectory.
-template <class Env, bool kSplit, bool kGather, bool kXp>
+// kIppo (collection, contiguous tiles): seat 1 learns too, and its trajectory goes to
+// a.traj1 -- its log-probabilities and values from its sampling threads, its actions,
+// rewards and dones from the env step, its observation rows (the ego's with the seats'
+// channels swapped, Env::other_seat_word) by the row-copy warps, and its V_T.
+template <class Env, bool kSplit, bool kGather, bool kXp, bool kIppo = false>
 __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs a) {
   using State = typename Env::State;
   constexpr int NA = Env::kNumActions;
@@ -80,6 +84,7 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
 
   int32_t* const rowenv = kGather ? reinterpret_cast<int32_t*>(smem + a.g.scratch_off) : nullptr;
   static_assert(!(kXp && kGather), "cross-play tiles are contiguous");
+  static_assert(!(kIppo && (kXp || kGather)), "IPPO is collection on contiguous tiles");
   const TcTile tile = tc_find_tile<kXp, kGather>(a, rowenv);
   const int64_t env0 = tile.env0;
   const int count = tile.count, tm_pol = tile.tm_pol, g_k = tile.g_k;
@@ -112,7 +117,8 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
   const int split = (chunks + 1) / 2;
   const int my_c0 = half ? split : 0, my_c1 = half ? chunks : split;
   const int my_w0 = min(4 * my_c0, cells), my_w1 = min(4 * my_c1, cells);
-  const bool with_boot = !kXp && a.traj.last_value != nullptr;
+  const bool boot1 = kIppo && tm_pol >= 0 && a.traj1.last_value != nullptr;  // seat 1's V_T
+  const bool with_boot = !kXp && (a.traj.last_value != nullptr || boot1);
   const bool obs_copy = kGather && a.traj.obs != nullptr;  // 12 warps store the rows during the step
 
   uint8_t* const sW0 = smem;                                                // policy blocks
@@ -383,7 +389,7 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
       float lp0 = 0.f, val0 = 0.f;
       if (ag == 1) {
         // ---------------------------- teammate group -------------------------------
-        const bool run = !boot && !tm_rule;
+        const bool run = (!boot || boot1) && !tm_rule;
         if (run) obs_x(s);
         tc::mbar_arrive(&buf_free);  // its rows are in tensor memory: the buffer is the ego's
         if (run) {
@@ -404,7 +410,15 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
             dbg_store(t, z);
             float lp;
             act1s[row] = (uint8_t)sample_k<NA>(z, 0xFFFFFFFFu >> (32 - NA), u_act, lp);
+            if constexpr (kIppo) {  // seat 1's learner fields
+              const int64_t o = (int64_t)t * N + my_env;
+              if (a.traj1.logp) a.traj1.logp[o] = lp;
+              if (a.traj1.values) a.traj1.values[o] = z[NA];
+            }
           }
+        } else if (boot1 && boot && half == 0 && row < count) {  // seat 1's V_T
+          logits(z);
+          a.traj1.last_value[my_env] = z[NA];
         }
       } else {
         // ------------------------------- ego group ---------------------------------
@@ -426,7 +440,7 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
         if (!bad) epilogue2();
         pair_sync();
         if (boot) {
-          if (half == 0 && row < count) {
+          if (half == 0 && row < count && a.traj.last_value) {
             logits(z);
             a.traj.last_value[my_env] = z[NA];
           }
@@ -474,6 +488,12 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
         if (a.traj.values) a.traj.values[o] = val0;
         if (a.traj.rewards) a.traj.rewards[o] = team;
         if (a.traj.dones) a.traj.dones[o] = (uint8_t)(done > 0);
+        if constexpr (kIppo) {  // seat 1's learner fields
+          if (a.traj1.actions) a.traj1.actions[o] = (uint8_t)act1;
+          if (a.traj1.tm_actions) a.traj1.tm_actions[o] = (uint8_t)act0;
+          if (a.traj1.rewards) a.traj1.rewards[o] = team;
+          if (a.traj1.dones) a.traj1.dones[o] = (uint8_t)(done > 0);
+        }
         if (done > 0) {
           Env::reset(a.b.env, a.b.key, (uint32_t)env, gt + 1, s2);
           if (a.ep_step) a.ep_step[env] = gt + 1;
@@ -495,6 +515,12 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
         if (lane == 0 && m) atomicAdd(&a.g.hist_next[g_k], __popc(m));
       }
       if (obs_copy && (ag == 1 || half == 1)) copy_rows_gathered(t, ag == 1 ? warp - 8 : warp + 4);
+      if (kIppo && a.traj1.obs && (ag == 1 || half == 1)) {  // seat 1's rows, a contiguous block
+        const int cw = ag == 1 ? warp - 8 : warp + 4;
+        const uint32_t* const src = reinterpret_cast<const uint32_t*>(sObs);
+        uint32_t* const dst = reinterpret_cast<uint32_t*>(a.traj1.obs + ((int64_t)t * N + env0) * od);
+        for (int f = cw * 32 + lane; f < count * cells; f += 12 * 32) dst[f] = Env::other_seat_word(src[f]);
+      }
       if (tid == 0 && bulk_obs) tc::bulk_wait_read();  // the rows may be rebuilt
       if (sync_all()) break;                            // the new state is in place
     }
@@ -530,9 +556,9 @@ __global__ void __launch_bounds__(kT2Threads, 1) ppo2_tc_kernel(const PpoTcArgs 
 
 template <class Env>
 struct LaunchTc2 {
-  template <bool kSplit, bool kGather, bool kXp = false>
+  template <bool kSplit, bool kGather, bool kXp = false, bool kIppo = false>
   static cudaError_t run(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
-    cudaError_t e = cudaFuncSetAttribute(ppo2_tc_kernel<Env, kSplit, kGather, kXp>,
+    cudaError_t e = cudaFuncSetAttribute(ppo2_tc_kernel<Env, kSplit, kGather, kXp, kIppo>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
@@ -545,7 +571,11 @@ struct LaunchTc2 {
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = a.pdl ? 1 : 0;
-    return cudaLaunchKernelEx(&cfg, ppo2_tc_kernel<Env, kSplit, kGather, kXp>, a);
+    return cudaLaunchKernelEx(&cfg, ppo2_tc_kernel<Env, kSplit, kGather, kXp, kIppo>, a);
+  }
+  // IPPO collection (dense first layer, contiguous tiles)
+  static cudaError_t ippo(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
+    return a.tc.split ? run<true, false, false, true>(a, grid, smem, s) : run<false, false, false, true>(a, grid, smem, s);
   }
   // cross-play (dense first layer)
   static cudaError_t xplay(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
