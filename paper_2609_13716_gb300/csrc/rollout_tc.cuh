@@ -434,42 +434,54 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
     };
     // kSparse: r1 = 1 / (1 + exp(2 (c + sum over the changed features f of delta W1[:, f]))) for this
     // thread's half of the units, written like epilogue 1 (hi | lo operand of L2); rows
-    // past count take c alone
+    // past count take c alone.  The W1 rows are gathered 8 units at a time with all ten
+    // features' loads issued before their multiply-adds (one L2 round trip per 8 units,
+    // not one per feature); an absent feature reads row 0 and adds 0 x W1 (exact)
     auto sparse_h1 = [&](int ag, const State& s) {
       const int H = d.H0;
-      const uint32_t P = tmem + (uint32_t)(ag * 256) + lane_base, Q = P + 128;
+      const uint32_t P = tmem + (uint32_t)(ag * 256) + lane_base;
       const float* pw = a.b.weights + (int64_t)(ag == 0 ? ego_pol : tm_pol) * a.b.mlp.stride;
       const float* W1t = pw + a.b.mlp.oW1;
       const float* cvec = pw + a.b.mlp.oC;
       uint32_t e[10];
       const uint32_t mask = row < count ? Env::sparse_obs(a.b.env, s, ag, e) : 0u;
-      for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 32) {
-        float v[32];
+#pragma unroll 1
+      for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 16) {
+        float v[16];
 #pragma unroll
-        for (int j = 0; j < 32; j += 4) {
+        for (int j = 0; j < 16; j += 4) {
           const float4 cc = __ldg(reinterpret_cast<const float4*>(cvec + c0 + j));
           v[j] = cc.x; v[j + 1] = cc.y; v[j + 2] = cc.z; v[j + 3] = cc.w;
         }
 #pragma unroll
-        for (int q = 0; q < 10; ++q) {
-          if (!((mask >> q) & 1u)) continue;
-          const float dv = (float)(int8_t)(e[q] & 0xFFu);
-          const float* wr = W1t + (int64_t)(e[q] >> 8) * H + c0;
+        for (int j8 = 0; j8 < 16; j8 += 8) {
+          float4 w4[10][2];
 #pragma unroll
-          for (int j = 0; j < 32; j += 4) {
-            const float4 w4 = __ldg(reinterpret_cast<const float4*>(wr + j));
-            v[j] = fmaf(dv, w4.x, v[j]);
-            v[j + 1] = fmaf(dv, w4.y, v[j + 1]);
-            v[j + 2] = fmaf(dv, w4.z, v[j + 2]);
-            v[j + 3] = fmaf(dv, w4.w, v[j + 3]);
+          for (int q = 0; q < 10; ++q) {
+            const uint32_t f = (mask >> q) & 1u ? e[q] >> 8 : 0u;
+            const float* wr = W1t + (int64_t)f * H + c0 + j8;
+            w4[q][0] = __ldg(reinterpret_cast<const float4*>(wr));
+            w4[q][1] = __ldg(reinterpret_cast<const float4*>(wr + 4));
+          }
+#pragma unroll
+          for (int q = 0; q < 10; ++q) {
+            const float dv = (mask >> q) & 1u ? (float)(int8_t)(e[q] & 0xFFu) : 0.0f;
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+              float* vv = v + j8 + 4 * k;
+              vv[0] = fmaf(dv, w4[q][k].x, vv[0]);
+              vv[1] = fmaf(dv, w4[q][k].y, vv[1]);
+              vv[2] = fmaf(dv, w4[q][k].z, vv[2]);
+              vv[3] = fmaf(dv, w4[q][k].w, vv[3]);
+            }
           }
         }
-        uint32_t hi[16], lo[16];
+        uint32_t hi[8], lo[8];
 #pragma unroll
-        for (int j = 0; j < 16; ++j)
+        for (int j = 0; j < 8; ++j)
           tc::split_bf16x2_p(tc::logistic2(tc::f2_mul(tc::f2_pack(v[2 * j], v[2 * j + 1]), tc::kTwoOverLn2x2)), hi[j], lo[j]);
-        tc::st_x16(P + c0 / 2, hi);
-        tc::st_x16(P + H / 2 + c0 / 2, lo);
+        tc::st_x8(P + c0 / 2, hi);
+        tc::st_x8(P + H / 2 + c0 / 2, lo);
       }
       tc::wait_st();
       operand_ready(ag, 1);
