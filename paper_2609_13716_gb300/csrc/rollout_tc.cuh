@@ -1,40 +1,40 @@
-// rollout_tc.cuh -- fused PPO rollout with the policy MLPs on tcgen05 tensor cores.
+// rollout_tc.cuh -- fused LBF rollout with a sparse first layer and the rest of the policy
+// MLPs on tcgen05 tensor cores.
 //
-// One CTA owns a tile of up to 128 envs that share one teammate policy, for all T steps:
-// a contiguous env range (one-member pools, cross-play), or the envs of one teammate's
-// group found by a rank scan of the per-env pool indices (kGather; per-episode
-// teammates: one step per launch).  This kernel runs cross-play, IPPO and the sparse
-// first layer; plain collection with a dense first layer runs on the two-group kernel of
-// rollout_tc2.cuh, which shares this file's tile finder.
-// Per step and agent (ego = seat 0, teammate = seat 1):
-//   obs (u8, shared memory, a constant 1 after the last feature) -> A operand in tensor
-//       memory as bf16 (exact: small integers)
-//   L1 (tensor cores): D = [o 1] [W1 b1]^T      (M = 128 envs, N = hidden0, K = KP)
-//   epilogue 1: r1 = 1 / (1 + exp(2 D)) split r1 = hi + lo (two bf16) into tensor memory;
-//       tanh(D) = 1 - 2 r1, and the block's W2, b2 hold -2 W2 and b2 + W2 1, so L2 sees
-//       exactly the tanh layer (the same for r2 and W3, b3 below)
+// The kernel serves LBF observations wider than the 256 tensor-memory columns of an
+// agent's A operand (the 12x12 grid's 576 features): PPO collection (a contiguous env
+// range for a one-member pool, else the envs of one teammate's group found by a rank
+// scan of the per-env pool indices, kGather) and cross-play (kXp).  Every LBF launch with
+// a dense first layer runs on the two-group kernel of rollout_tc2.cuh, which shares this
+// file's tile finder.  One CTA owns a tile of up to 128 envs that share one teammate
+// policy, for all T steps.  Per step and agent (teammate first, then the ego = seat 0):
+//   h1 on CUDA cores: the observation is a fixed pattern plus at most ten changed
+//       features, so r1 = 1 / (1 + exp(2 (c + sum over them of delta W1[:, f]))), c = b1 +
+//       W1 x_pattern; r1 is split r1 = hi + lo (two bf16) into tensor memory.  tanh(x) =
+//       1 - 2 r1, and the block's W2, b2 hold -2 W2 and b2 + W2 1, so L2 sees exactly the
+//       tanh layer (the same for r2 and W3, b3 below)
 //   L2 (tensor cores): D = hi W2'^T + lo W2'^T  (the split keeps ~2^-17 relative precision
 //       of r1 with bf16 operands and fp32 accumulate)
 //   epilogue 2: r2 = 1 / (1 + exp(2 (D + b2))), split again, and z = W3' r2 + b3' by mma.sync m16n8k16
-//       from registers (16x256b accumulator loads are its fragment layout; a handful of
-//       outputs would waste an N = 16 tcgen05 instruction's round trip)
+//       from registers (16x256b accumulator loads are its fragment layout)
 //   sampling (ego in warps 0-3, teammate in warps 4-7), env step, trajectory write.
 //
-// Warp roles: warps 0-7 ("compute", 256 threads) build observations, run the epilogues
-// (thread r and r + 128 own env row r, tensor-memory lane r; the halves split the
-// columns), sample and step the envs; warp 8 issues every MMA; warps 9-12 store the
-// ego's observation rows of gathered tiles (scattered rows, a quarter each, one warp per
-// SM sub-partition) while the compute warps go on.  They meet only through mbarriers:
-// operand-ready (256 arrivals from the compute threads) and accumulator-ready (a
-// tcgen05.commit); observation rows ready (256 arrivals) and observation buffer free
-// (one arrival per store warp).  Each of these barriers completes once per step, so its phase
-// parity is the step's parity.  Compute warps synchronise among themselves with a named
-// barrier that also ORs an error flag.  Weights are bulk-copied (TMA) into shared memory
-// once per CTA.  Every wait is bounded: on expiry the CTA records kStatusTimeout, stops,
-// drains its own MMAs (bounded), frees tensor memory and exits.
+// Warp roles: warps 0-7 ("compute", 256 threads) build the ego's observation rows for the
+// trajectory, form h1, run epilogue 2 (thread r and r + 128 own env row r, tensor-memory
+// lane r; the halves split the columns), sample and step the envs; warp 8 issues every
+// MMA; warps 9-12 store the ego's observation rows of gathered tiles (scattered rows, a
+// quarter each, one warp per SM sub-partition) while the compute warps go on.  They meet
+// only through mbarriers: operand-ready (256 arrivals from the compute threads) and
+// accumulator-ready (a tcgen05.commit); observation rows ready (256 arrivals) and
+// observation buffer free (one arrival per store warp).  Each of these barriers completes
+// once per step, so its phase parity is the step's parity.  Compute warps synchronise
+// among themselves with a named barrier that also ORs an error flag.  Weights (all but
+// W1) are bulk-copied (TMA) into shared memory once per CTA; W1^T and c are read from
+// the L2-resident fp32 population.  Every wait is bounded: on expiry the CTA records
+// kStatusTimeout, stops, drains its own MMAs (bounded), frees tensor memory and exits.
 //
 // Tensor memory (512 columns): agent a uses columns [256a, 256a + 128) for its A operand
-// (X, then hi|lo of h1) and [256a + 128, 256a + 256) for its fp32 accumulator.
+// (hi|lo of h1) and [256a + 128, 256a + 256) for its fp32 accumulator.
 #pragma once
 #include "kernels.h"
 #include "rollout_impl.cuh"
@@ -46,7 +46,6 @@ constexpr int kTcCompute = 256;          // compute threads
 constexpr int kTcThreads = 416;          // + one MMA warp + four observation-store warps
 constexpr int kTcStoreWarps = 4;         // warps 9-12: one per SM sub-partition
 constexpr int kTcComputeBar = 1;         // named barrier id of the compute warps
-constexpr int kTcPairBar = 2;            // ids 2..5: warps q and q + 4 (rows 32q .. 32q + 31)
 
 // The tile of CTA blockIdx.x: cross-play (kXp) chunk `blockIdx.x % tpp` of pair
 // `blockIdx.x / tpp`; gathered (kGather) tile blockIdx.x of the teammate groups, its envs
@@ -177,28 +176,21 @@ __device__ __forceinline__ TcTile tc_find_tile(const PpoTcArgs& a, int32_t* rowe
 
 // kXp: cross-play (each tile is a chunk of one pair's envs, reset at the call's first
 // step, frozen once done; the per-env return and episode length are the outputs) instead
-// of PPO collection.  kSplit: fp32 weights held as bf16 pairs W = W_hi + W_lo, L1 =
-// X W1_hi + X W1_lo and L2 = b2 + hi W2_hi + lo W2_hi + hi W2_lo (lo W2_lo is below
-// 2^-16 of the sum and left out).  kIppo (PPO collection only): seat 1 learns too, and
-// its trajectory goes to a.traj1.  kGather (PPO collection): the tile's rows are envs of
-// one teammate group found by a rank scan of the per-env pool indices (the call's draw
-// for all T steps, or, per episode, one step per launch) instead of a contiguous range.
-// kSparse (observations wider than the
-// 256 tensor-memory columns of an agent's A operand; Env::sparse_obs required): no first
-// layer on the tensor cores -- each thread forms its half of h1 = tanh(c + sum over the
-// observation's changed features of delta W1[:, f]) on CUDA cores from the fp32 W1^T and
-// c of the CUDA-core population, and writes it as the A operand of L2 directly.
-template <class Env, bool kXp, bool kSplit, bool kIppo, bool kGather, bool kSparse>
+// of PPO collection.  kSplit: fp32 weights held as bf16 pairs W = W_hi + W_lo and L2 = b2
+// + hi W2_hi + lo W2_hi + hi W2_lo (lo W2_lo is below 2^-16 of the sum and left out).
+// kGather (PPO collection): the tile's rows are envs of one teammate group found by a rank
+// scan of the per-env pool indices (the call's draw, held for all T steps) instead of a
+// contiguous range.  Env::sparse_obs lists the changed features; W1^T and c are the fp32
+// copies of the CUDA-core population.
+template <class Env, bool kXp, bool kSplit, bool kGather>
 __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a) {
-  static_assert(!(kXp && kIppo), "seat-1 trajectories belong to PPO collection");
-  static_assert(!(kGather && (kXp || kIppo)), "gathered tiles are plain PPO collection");
-  static_assert(!(kSparse && kIppo), "the sparse first layer serves plain collection and cross-play");
+  static_assert(!(kGather && kXp), "gathered tiles are PPO collection");
   static_assert(kTcThreads / 32 <= 24, "gather scratch: one total per warp");
   using State = typename Env::State;
   constexpr int NA = Env::kNumActions;
   extern __shared__ __align__(16) uint8_t smem[];  // no-swizzle operands need 16 B
-  __shared__ __align__(8) uint64_t acc_bar[4];     // [2*agent + layer], tcgen05.commit
-  __shared__ __align__(8) uint64_t opnd_bar[4];    // [2*agent + layer], 256 arrivals
+  __shared__ __align__(8) uint64_t acc_bar[2];     // [agent], L2 committed (tcgen05.commit)
+  __shared__ __align__(8) uint64_t opnd_bar[2];    // [agent], h1 in tensor memory (256 arrivals)
   __shared__ __align__(8) uint64_t wload_bar, drain_bar;
   __shared__ __align__(8) uint64_t obs_full, obs_free;  // gathered observation rows: warps 9-12
   __shared__ __align__(8) uint64_t never_bar;           // test hook: nothing arrives on it
@@ -209,7 +201,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   int32_t* const rowenv = kGather ? reinterpret_cast<int32_t*>(smem + a.g.scratch_off) : nullptr;
   const TcTile tile = tc_find_tile<kXp, kGather>(a, rowenv);
   const int64_t env0 = tile.env0;
-  const int count = tile.count, ego_pol = tile.ego_pol, tm_pol = tile.tm_pol, g_k = tile.g_k;
+  const int count = tile.count, ego_pol = tile.ego_pol, tm_pol = tile.tm_pol;
   if (count <= 0) return;
   // a negative teammate id is LBF heuristic -1 - id: no teammate network, its rule acts
   const bool tm_rule = tm_pol < 0;
@@ -224,11 +216,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   const int cells = od / 4;          // observation words per row
   const int chunks = d.KP / 16;      // 16-byte chunks per observation row
   const int split = (chunks + 1) / 2;
-  const int my_c0 = half ? split : 0, my_c1 = half ? chunks : split;
-  const int my_w0 = min(4 * my_c0, cells), my_w1 = min(4 * my_c1, cells);
-  // V_T after the last step: the ego's, and seat 1's when it learns too (IPPO)
-  const bool boot1 = kIppo && !tm_rule && a.traj1.last_value != nullptr;
-  const bool with_boot = !kXp && (a.traj.last_value != nullptr || boot1);
+  // the halves build words [my_w0, my_w1) of the ego's row
+  const int my_w0 = min(4 * (half ? split : 0), cells), my_w1 = min(4 * (half ? chunks : split), cells);
+  const bool with_boot = !kXp && a.traj.last_value != nullptr;  // the ego's V_T after the last step
   // gathered tiles: warps 9-12 store the ego's observation rows of every step
   const bool obs_warp = kGather && a.traj.obs != nullptr;
 
@@ -242,7 +232,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   float* zpart = reinterpret_cast<float*>(act1s + 128);                     // [2][2][128][8]
 
   if (tid == 0) {
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < 2; ++i) {
       tc::mbar_init(&acc_bar[i], 1);
       tc::mbar_init(&opnd_bar[i], kTcCompute);
     }
@@ -278,14 +268,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
           tc::bulk_g2s(sW0 + p * d.pol_bytes + off, src + off, min(32768u, d.pol_bytes - off), &wload_bar);
       }
       bool ok = tc::mbar_wait(&wload_bar, 0);
-      const uint32_t idesc1 = tc::idesc_bf16(128, d.H0), idesc2 = tc::idesc_bf16(128, d.H1);
-      const uint32_t sbo1 = (uint32_t)(d.KP / 8) * 128u, sbo2 = (uint32_t)(d.H0 / 8) * 128u;
+      const uint32_t idesc2 = tc::idesc_bf16(128, d.H1);
+      const uint32_t sbo2 = (uint32_t)(d.H0 / 8) * 128u;
       // agents in the order the compute warps release them: teammate, then ego
       bool stopped = false;
-      auto issue = [&](int ag, int layer, uint32_t parity) {
+      auto issue = [&](int ag, uint32_t parity) {  // L2 of agent ag
         ok = false;
         for (int tries = 0; tries < 1000 && !ok && !abort_flag; ++tries)
-          ok = tc::mbar_wait(&opnd_bar[2 * ag + layer], parity, 2000000ull);
+          ok = tc::mbar_wait(&opnd_bar[ag], parity, 2000000ull);
         if (!ok) return;
         if (kXp && stop_flag) {  // released without operands: the tile is finished
           stopped = true;
@@ -294,43 +284,22 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         tc::fence_after_sync();
         const uint32_t wbase = tc::smem_u32(sW0) + (uint32_t)ag * d.pol_bytes;
         const uint32_t P = tmem + (uint32_t)(ag * 256), Q = P + 128;
-        if (layer == 0) {
-          const uint64_t w0 = tc::smem_desc(wbase + d.oW1, 128u, sbo1);
-          for (int ks = 0; ks < d.KP / 16; ++ks) tc::mma_ts(Q, P + 8 * ks, w0 + 16u * ks, idesc1, ks > 0);
-          if constexpr (kSplit) {
-            const uint64_t w1 = tc::smem_desc(wbase + d.oW1lo, 128u, sbo1);
-            for (int ks = 0; ks < d.KP / 16; ++ks) tc::mma_ts(Q, P + 8 * ks, w1 + 16u * ks, idesc1, 1u);
-          }
-        } else {
-          const uint64_t w0 = tc::smem_desc(wbase + d.oW2, 128u, sbo2);
-          for (int ks = 0; ks < d.H0 / 16; ++ks) tc::mma_ts(Q, P + 8 * ks, w0 + 16u * ks, idesc2, ks > 0);
-          for (int ks = 0; ks < d.H0 / 16; ++ks) tc::mma_ts(Q, P + d.H0 / 2 + 8 * ks, w0 + 16u * ks, idesc2, 1u);
-          if constexpr (kSplit) {
-            const uint64_t w1 = tc::smem_desc(wbase + d.oW2lo, 128u, sbo2);
-            for (int ks = 0; ks < d.H0 / 16; ++ks) tc::mma_ts(Q, P + 8 * ks, w1 + 16u * ks, idesc2, 1u);
-          }
+        const uint64_t w0 = tc::smem_desc(wbase + d.oW2, 128u, sbo2);
+        for (int ks = 0; ks < d.H0 / 16; ++ks) tc::mma_ts(Q, P + 8 * ks, w0 + 16u * ks, idesc2, ks > 0);
+        for (int ks = 0; ks < d.H0 / 16; ++ks) tc::mma_ts(Q, P + d.H0 / 2 + 8 * ks, w0 + 16u * ks, idesc2, 1u);
+        if constexpr (kSplit) {
+          const uint64_t w1 = tc::smem_desc(wbase + d.oW2lo, 128u, sbo2);
+          for (int ks = 0; ks < d.H0 / 16; ++ks) tc::mma_ts(Q, P + 8 * ks, w1 + 16u * ks, idesc2, 1u);
         }
-        tc::commit(&acc_bar[2 * ag + layer]);
+        tc::commit(&acc_bar[ag]);
       };
       const int n_steps = kXp ? a.xp.max_steps : a.T;
       for (int t = 0; ok && !stopped && t < n_steps; ++t) {
         const uint32_t par = (uint32_t)t & 1u;
-        if (!kSparse) {
-          if (!tm_rule) issue(1, 0, par);
-          if (ok && !stopped) issue(0, 0, par);
-        }
-        if (ok && !stopped && !tm_rule) issue(1, 1, par);
-        if (ok && !stopped) issue(0, 1, par);
+        if (!tm_rule) issue(1, par);
+        if (ok && !stopped) issue(0, par);
       }
-      if (ok && with_boot) {
-        const uint32_t par = (uint32_t)a.T & 1u;
-        if (!kSparse) {
-          if (boot1) issue(1, 0, par);
-          if (ok) issue(0, 0, par);
-        }
-        if (ok && boot1) issue(1, 1, par);
-        if (ok) issue(0, 1, par);
-      }
+      if (ok && with_boot) issue(0, (uint32_t)a.T & 1u);
       if (!ok) abort_flag = 1;
     }
   } else if (warp > 8) {
@@ -376,65 +345,21 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
   } else {
     // ============================== compute warps ===================================
     bool bad = false;
-    auto wait_acc = [&](int ag, int layer, uint32_t parity) {
-      if (!bad && !tc::mbar_wait(&acc_bar[2 * ag + layer], parity)) bad = true;
+    auto wait_acc = [&](int ag, uint32_t parity) {
+      if (!bad && !tc::mbar_wait(&acc_bar[ag], parity)) bad = true;
       bad = __any_sync(0xFFFFFFFFu, bad);  // warp-uniform: tensor-memory loads are collective
       tc::fence_after_sync();
     };
-    auto operand_ready = [&](int ag, int layer) {  // this thread's tensor-memory traffic is done
+    auto operand_ready = [&](int ag) {  // this thread's tensor-memory traffic is done
       tc::fence_before_sync();
-      tc::mbar_arrive(&opnd_bar[2 * ag + layer]);
+      tc::mbar_arrive(&opnd_bar[ag]);
     };
     auto sync_or = [&]() { return tc::bar_or(kTcComputeBar, kTcCompute, bad || abort_flag); };
     auto pol_block = [&](int ag) { return sW0 + (size_t)ag * d.pol_bytes; };
 
-    // observation (built into this thread's half row) -> bf16 A operand of L1; feature
-    // obs_dim is the constant 1 that carries b1, the rest of the padding is 0
-    auto obs_x = [&](int ag, const State& s) {
-      uint32_t* roww = reinterpret_cast<uint32_t*>(sObs + row * od);
-      if (row < count) Env::obs_words(a.b.env, s, ag, roww, my_w0, my_w1);
-      const uint32_t P = tmem + (uint32_t)(ag * 256) + lane_base;
-      for (int c = my_c0; c < my_c1; ++c) {
-        uint32_t w4[4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int w = 4 * c + j;
-          w4[j] = w < cells ? roww[w] : (w == cells ? 1u : 0u);
-        }
-        uint32_t v[8];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          v[2 * j] = tc::bytes_to_bf16x2(w4[j], 0);
-          v[2 * j + 1] = tc::bytes_to_bf16x2(w4[j], 2);
-        }
-        tc::st_x8(P + 8 * c, v);
-      }
-      tc::wait_st();
-      operand_ready(ag, 0);
-    };
-    // epilogue 1: r1 = 1 / (1 + exp(2 D)) -> hi | lo bf16 A operand of L2 (b2 is added in
-    // epilogue 2)
-    auto epilogue1 = [&](int ag) {
-      const int H = d.H0;
-      const uint32_t P = tmem + (uint32_t)(ag * 256) + lane_base, Q = P + 128;
-      for (int c0 = half * (H / 2); c0 < (half + 1) * (H / 2); c0 += 32) {
-        uint32_t v[32];
-        tc::ld_x32(Q + c0, v);
-        tc::wait_ld();
-        uint32_t hi[16], lo[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j)
-          tc::split_bf16x2_p(tc::logistic2(tc::f2_mul(tc::f2_pack(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1])), tc::kTwoOverLn2x2)),
-                             hi[j], lo[j]);
-        tc::st_x16(P + c0 / 2, hi);
-        tc::st_x16(P + H / 2 + c0 / 2, lo);
-      }
-      tc::wait_st();
-      operand_ready(ag, 1);
-    };
-    // kSparse: r1 = 1 / (1 + exp(2 (c + sum over the changed features f of delta W1[:, f]))) for this
-    // thread's half of the units, written like epilogue 1 (hi | lo operand of L2); rows
-    // past count take c alone.  The W1 rows are gathered 8 units at a time with all ten
+    // h1: r1 = 1 / (1 + exp(2 (c + sum over the changed features f of delta W1[:, f]))) for this
+    // thread's half of the units, split hi | lo into the A operand of L2; rows past count
+    // take c alone.  The W1 rows are gathered 8 units at a time with all ten
     // features' loads issued before their multiply-adds (one L2 round trip per 8 units,
     // not one per feature); an absent feature reads row 0 and adds 0 x W1 (exact)
     auto sparse_h1 = [&](int ag, const State& s) {
@@ -484,7 +409,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         tc::st_x8(P + H / 2 + c0 / 2, lo);
       }
       tc::wait_st();
-      operand_ready(ag, 1);
+      operand_ready(ag);
     };
     // epilogue 2: r2 = 1 / (1 + exp(2 (D + b2))) and this half's partial z = sum_k W3'[:, k] r2[k] on the
     // tensor cores from registers (mma.sync m16n8k16, one n-tile of 8 outputs): the warp
@@ -585,8 +510,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         // every env of the tile is done: release the MMA warp without operands and stop
         if (!tc::bar_or(kTcComputeBar, kTcCompute, half == 0 && row < count && alive)) {
           if (tid == 0) stop_flag = 1;
-          // the first barrier it waits on: L1 of the first agent (L2 without a first layer)
-          tc::mbar_arrive(&opnd_bar[(tm_rule ? 0 : 2) + (kSparse ? 1 : 0)]);
+          tc::mbar_arrive(&opnd_bar[tm_rule ? 0 : 1]);  // the first barrier it waits on
           break;
         }
       }
@@ -595,47 +519,23 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         if (!bad && !tc::mbar_wait(&obs_free, (uint32_t)(t - 1) & 1u)) bad = true;
         bad = __any_sync(0xFFFFFFFFu, bad);
       }
-      // teammate first: the ego's rows stay for the copy
-      const int first = (boot && !boot1) || tm_rule ? 0 : 1;
+      // teammate first (its network runs in every step but the bootstrap)
+      const int first = boot || tm_rule ? 0 : 1;
       const uint32_t par = (uint32_t)t & 1u, gt = a.step0 + (uint32_t)t;
       // this half's action draw (ego: warps 0-3, teammate: warps 4-7), ahead of its use
       const float u_act = boot ? 0.0f : u01(draw0(a.b.key, (uint32_t)my_env, gt, kStreamAct0 + half));
       State s = st[row];  // register copy for this step (rows past count are never used)
 #pragma unroll 1
       for (int i = first; i >= 0; --i) {
-        if constexpr (kSparse) {
-          // the ego's u8 row is the trajectory's observation; no first layer to feed
-          if (!kXp && i == 0 && !boot && a.traj.obs && row < count)
-            Env::obs_words(a.b.env, s, 0, reinterpret_cast<uint32_t*>(sObs + row * od), my_w0, my_w1);
-          if (obs_warp && i == 0 && !boot) tc::mbar_arrive(&obs_full);
-          if (!bad) sparse_h1(i, s);
-          continue;
-        }
-        obs_x(i, s);
+        // the ego's u8 row is the trajectory's observation; no first layer to feed
+        if (!kXp && i == 0 && !boot && a.traj.obs && row < count)
+          Env::obs_words(a.b.env, s, 0, reinterpret_cast<uint32_t*>(sObs + row * od), my_w0, my_w1);
         if (obs_warp && i == 0 && !boot) tc::mbar_arrive(&obs_full);
-        if (kIppo && i == 1 && !boot && a.traj1.obs) {
-          // seat 1's rows -> its trajectory before the ego's overwrite them: warps q and
-          // q + 4 built rows 32q .. 32q + 31, a contiguous block in shared and in global
-          // memory, which they store with consecutive words
-          const int q = warp & 3, pt = half * 32 + lane;
-          tc::bar_sync(kTcPairBar + q, 64);
-          const int rows = min(32, count - 32 * q);
-          if (rows > 0) {
-            const uint32_t* src = reinterpret_cast<const uint32_t*>(sObs + 32 * q * od);
-            uint32_t* dst = reinterpret_cast<uint32_t*>(a.traj1.obs + ((int64_t)t * N + env0 + 32 * q) * od);
-            for (int w = pt; w < rows * cells; w += 64) dst[w] = src[w];
-          }
-          tc::bar_sync(kTcPairBar + q, 64);
-        }
+        if (!bad) sparse_h1(i, s);
       }
       if (t == a.dbg_expire_step) {  // test hook: an accumulator wait that never completes
         if (!bad && !tc::mbar_wait(&never_bar, 0, a.dbg_expire_ns)) bad = true;
         bad = __any_sync(0xFFFFFFFFu, bad);
-      }
-#pragma unroll 1
-      for (int i = first; i >= 0 && !kSparse; --i) {
-        wait_acc(i, 0, par);
-        if (!bad) epilogue1(i);
       }
       if (!kXp && !kGather && !boot && a.traj.obs) {  // overlaps L2 on the tensor cores
         tc::fence_proxy_async();       // the rows were written by ordinary stores
@@ -644,23 +544,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
       }
 #pragma unroll 1
       for (int i = first; i >= 0; --i) {
-        wait_acc(i, 1, par);
+        wait_acc(i, par);
         if (!bad) epilogue2(i);
       }
       if (sync_or()) break;
       float z[16];
       if (boot) {
-        if (half == 0 && row < count && a.traj.last_value) {
+        if (half == 0 && row < count) {
           logits(0, z);
           a.traj.last_value[my_env] = z[NA];
-        } else if (kIppo && half == 1 && row < count && boot1) {
-          logits(1, z);
-          a.traj1.last_value[my_env] = z[NA];
         }
         break;
       }
       int act0 = 0;
-      bool stayed = false;  // gather: the row's env keeps its teammate for the next step
       float lp0 = 0.f, val0 = 0.f;
       if (row < count && half == 1 && tm_rule) {
         act1s[row] = (uint8_t)Env::heuristic(a.b.env, st[row], -1 - tm_pol);  // st[row] == s here
@@ -677,11 +573,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         const int act = sample_k<NA>(z, 0xFFFFFFFFu >> (32 - NA), u_act, lp);
         if (ag == 1) {
           act1s[row] = (uint8_t)act;
-          if constexpr (kIppo) {
-            const int64_t o = (int64_t)t * N + my_env;
-            if (a.traj1.logp) a.traj1.logp[o] = lp;
-            if (a.traj1.values) a.traj1.values[o] = z[NA];
-          }
         } else {
           act0 = act;
           lp0 = lp;
@@ -723,33 +614,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
         if (a.traj.values) a.traj.values[o] = val0;
         if (a.traj.rewards) a.traj.rewards[o] = team;
         if (a.traj.dones) a.traj.dones[o] = (uint8_t)(done > 0);
-        if constexpr (kIppo) {
-          if (a.traj1.actions) a.traj1.actions[o] = (uint8_t)act1;
-          if (a.traj1.tm_actions) a.traj1.tm_actions[o] = (uint8_t)act0;
-          if (a.traj1.rewards) a.traj1.rewards[o] = team;
-          if (a.traj1.dones) a.traj1.dones[o] = (uint8_t)(done > 0);
-        }
         if (done > 0) {
           Env::reset(a.b.env, a.b.key, (uint32_t)env, gt + 1, s);
           if (a.ep_step) a.ep_step[env] = gt + 1;
         }
-        if (kGather && a.g.resample) {  // the next step's pool index: a new episode draws again
-          int kn = g_k;
-          if (done > 0) {
-            kn = (int)uniform_int(draw0(a.b.key, (uint32_t)env, gt + 1, kStreamEpisodeTeammate),
-                                  (uint32_t)a.g.pool_size);
-            atomicAdd(&a.g.hist_next[kn], 1);
-          }
-          a.g.kidx_next[env] = (uint8_t)kn;
-          stayed = done <= 0;
-        }
         st[row] = s;
-      }
-      if (kGather && a.g.resample) {
-        if (half == 0) {  // warps 0-3: one count per warp of the rows that keep the teammate
-          const unsigned m = __ballot_sync(0xFFFFFFFFu, stayed);
-          if (lane == 0 && m) atomicAdd(&a.g.hist_next[g_k], __popc(m));
-        }
       }
       if (tid == 0 && bulk_obs) tc::bulk_wait_read();  // the rows may be rebuilt
       if (sync_or()) break;
@@ -788,36 +657,26 @@ __global__ void __launch_bounds__(kTcThreads, 1) ppo_tc_kernel(const PpoTcArgs a
 
 template <class Env>
 struct LaunchTc {
-  template <bool kXp, bool kSplit, bool kIppo, bool kGather = false, bool kSparse = false>
+  template <bool kXp, bool kSplit, bool kGather>
   static cudaError_t run(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
-    cudaError_t e = cudaFuncSetAttribute(ppo_tc_kernel<Env, kXp, kSplit, kIppo, kGather, kSparse>,
+    cudaError_t e = cudaFuncSetAttribute(ppo_tc_kernel<Env, kXp, kSplit, kGather>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    ppo_tc_kernel<Env, kXp, kSplit, kIppo, kGather, kSparse><<<grid, kTcThreads, smem, s>>>(a);
+    ppo_tc_kernel<Env, kXp, kSplit, kGather><<<grid, kTcThreads, smem, s>>>(a);
     return cudaGetLastError();
   }
+  // PPO collection with the call's draw (the host keeps IPPO and per-episode teammates of
+  // such contexts on CUDA cores)
   static cudaError_t ppo(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
     const TrajPtrs& u = a.traj1;
     const bool ippo = u.obs || u.actions || u.tm_actions || u.logp || u.values || u.rewards ||
                       u.dones || u.last_value;
-    if (a.tc.sparse) {  // plain collection only (the host keeps the others on CUDA cores)
-      if (ippo || (a.gather && a.g.resample)) return cudaErrorNotSupported;
-      if (a.gather)
-        return a.tc.split ? run<false, true, false, true, true>(a, grid, smem, s)
-                          : run<false, false, false, true, true>(a, grid, smem, s);
-      return a.tc.split ? run<false, true, false, false, true>(a, grid, smem, s)
-                        : run<false, false, false, false, true>(a, grid, smem, s);
-    }
-    // with a dense first layer this kernel runs IPPO only: plain collection, with contiguous
-    // or gathered tiles, runs on the two-group kernel (rollout_tc2.cuh)
-    if (ippo && !a.gather)
-      return a.tc.split ? run<false, true, true>(a, grid, smem, s) : run<false, false, true>(a, grid, smem, s);
-    return cudaErrorNotSupported;
+    if (!a.tc.sparse || ippo || (a.gather && a.g.resample)) return cudaErrorNotSupported;
+    if (a.gather) return a.tc.split ? run<false, true, true>(a, grid, smem, s) : run<false, false, true>(a, grid, smem, s);
+    return a.tc.split ? run<false, true, false>(a, grid, smem, s) : run<false, false, false>(a, grid, smem, s);
   }
   static cudaError_t xplay(const PpoTcArgs& a, int grid, size_t smem, cudaStream_t s) {
-    if (a.tc.sparse)
-      return a.tc.split ? run<true, true, false, false, true>(a, grid, smem, s)
-                        : run<true, false, false, false, true>(a, grid, smem, s);
+    if (!a.tc.sparse) return cudaErrorNotSupported;
     return a.tc.split ? run<true, true, false>(a, grid, smem, s) : run<true, false, false>(a, grid, smem, s);
   }
 };

@@ -1,25 +1,39 @@
-// rollout_tc2.cuh -- PPO collection with the ego and the teammate on separate warp groups.
+// rollout_tc2.cuh -- LBF rollouts with a dense first layer (PPO collection, IPPO and
+// cross-play), with the ego and the teammate on separate warp groups.
 //
-// The same step as ppo_tc_kernel's plain collection (one CTA owns a tile of up to 128 envs
-// that share a teammate policy, for all T steps; the MLPs on tcgen05 with split-bf16
-// activations, the output layer on mma.sync from the accumulator fragments, sampling, the
-// env step, the trajectory write), but each agent has its own eight warps:
+// One CTA owns a tile of up to 128 envs that share a teammate policy, for all T steps.
+// Per step and agent (ego = seat 0, teammate = seat 1):
+//   obs (u8, shared memory, a constant 1 after the last feature) -> A operand in tensor
+//       memory as bf16 (exact: small integers)
+//   L1 (tensor cores): D = [o 1] [W1 b1]^T      (M = 128 envs, N = hidden0, K = KP)
+//   epilogue 1: r1 = 1 / (1 + exp(2 D)) split r1 = hi + lo (two bf16) into tensor memory;
+//       tanh(D) = 1 - 2 r1, and the block's W2, b2 hold -2 W2 and b2 + W2 1, so L2 sees
+//       exactly the tanh layer (the same for r2 and W3, b3 below)
+//   L2 (tensor cores): D = hi W2'^T + lo W2'^T  (the split keeps ~2^-17 relative precision
+//       of r1 with bf16 operands and fp32 accumulate)
+//   epilogue 2: r2 = 1 / (1 + exp(2 (D + b2))), split again, and z = W3' r2 + b3' by
+//       mma.sync m16n8k16 from registers (16x256b accumulator loads are its fragment
+//       layout; a handful of outputs would waste an N = 16 tcgen05 instruction's round trip)
+//   sampling, env step, trajectory write.
+// Each agent has its own eight warps:
 //   warps 0-7   ego group: thread r and r + 128 own env row r (tensor-memory lane r) and
 //               split the ego's columns; they also step the envs and write the trajectory;
 //   warps 8-15  teammate group: the same for the teammate (or its rule).
 // The two agents' dependent chains (observation -> L1 -> epilogue 1 -> L2 -> epilogue 2 ->
-// sampling) run concurrently, four warps per SM sub-partition, instead of one chain of
-// eight warps that alternates between the agents.  There is no MMA warp (sixteen warps
-// keep 128 registers a thread): once a group's operand is in tensor memory (a group
-// barrier), its first thread issues the layer's MMAs and commits them to the group's
-// accumulator barrier.  The groups share one observation buffer: the teammate's rows are
-// built first, and once they are in tensor memory the buffer passes to the ego (an
-// mbarrier).  Both groups meet twice per step on a named barrier that also ORs their
+// sampling) run concurrently, four warps per SM sub-partition.  There is no MMA warp
+// (sixteen warps keep 128 registers a thread): once a group's operand is in tensor memory
+// (a group barrier), its first thread issues the layer's MMAs and commits them to the
+// group's accumulator barrier.  The groups share one observation buffer: the teammate's
+// rows are built first, and once they are in tensor memory the buffer passes to the ego
+// (an mbarrier).  Both groups meet twice per step on a named barrier that also ORs their
 // error flags: once both actions exist (then the ego group's first half steps the envs
 // while, for gathered tiles, the teammate group and the ego's second half write the ego's
 // rows to the trajectory) and once the new state is in shared memory.  Every mbarrier wait
 // is bounded (2 s): on expiry the CTA records kStatusTimeout, stops, waits (bounded) for
 // its own MMAs, frees tensor memory and exits.
+//
+// Tensor memory (512 columns): agent a uses columns [256a, 256a + 128) for its A operand
+// (X, then hi|lo of h1) and [256a + 128, 256a + 256) for its fp32 accumulator.
 #pragma once
 #include "rollout_tc.cuh"
 
