@@ -68,7 +68,8 @@ def expire_then(ctx, call):
 @pytest.mark.parametrize("wl_name,pool,ippo", [
     ("lbf7x7_ppo_16384x128", [1, 2, 3, 4], False),   # two-group kernel, gathered tiles
     ("lbf7x7_ppo_16384x128", [2], False),            # two-group kernel, contiguous tiles
-    ("lbf7x7_ippo_16384x128", [1], True),            # one-group kernel (IPPO)
+    ("lbf7x7_ippo_16384x128", [1], True),            # two-group kernel, IPPO
+    ("lbf12x12_ppo_4096x128", [1, 2, 3], False),     # sparse first layer, gathered tiles
 ])
 def test_collection_kernel_wait_expires_mid_rollout(wl_name, pool, ippo):
     """The real collection kernels: a wait made to expire at step 5 of 12 takes the abort
