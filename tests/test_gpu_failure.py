@@ -5,8 +5,9 @@ Every wait of the tensor-core kernels on another warp's progress is bounded by
 returns.  Here a wait is made to expire on purpose (an mbarrier nothing arrives on, a
 1 ms limit): the host must read the timeout from aht_sync, and the context must stay
 usable for the next call.  First in a one-thread probe, then inside the real kernels
-(aht_debug_expire_at): the two-warp-group and one-group collection kernels and the
-LBF and streamed cross-play kernels, each mid-call with MMAs in flight.
+(aht_debug_expire_at): the two-warp-group kernel (collection, IPPO and LBF cross-play),
+the sparse-first-layer kernel and the streamed cross-play kernel, each mid-call with MMAs
+in flight.
 """
 import numpy as np
 import pytest

@@ -6,13 +6,13 @@ evaluation's whole output vector -- every logit, and the value row where the pol
 one -- and each element is compared with the oracle's forward of the same observation
 (protocol M3: |g - o| <= 1e-4 |o| + 1e-4 rms(o) over the tensor), for every MLP shape the
 tensor-core kernels run:
-  - PPO collection on the two-warp-group kernel: bf16 196-128-128-7 ego and 196-128-128-6
-    teammates (gathered tiles, contiguous tiles), fp32 196-64-64-6 (split weights);
-  - IPPO collection on the one-group kernel (both seats' networks);
+  - the two-warp-group kernel: PPO collection with bf16 196-128-128-7 ego and
+    196-128-128-6 teammates (gathered tiles, contiguous tiles) and fp32 196-64-64-6
+    (split weights); IPPO collection (both seats' networks); LBF cross-play with fp32
+    196-64-64-6 (split weights, frozen envs evaluated too);
   - LBF 12x12 PPO collection with the sparse first layer (576-128-128);
-  - cross-play: LBF fp32 196-64-64-6 (split weights, frozen envs evaluated too),
-    Overcooked 520-256-256-6, Hanabi 660-512-512-20 and Mini Hanabi 156-256-256-10 on the
-    streamed kernel.
+  - cross-play on the streamed kernel: Overcooked 520-256-256-6, Hanabi 660-512-512-20
+    and Mini Hanabi 156-256-256-10.
 Every case has at least 1200 evaluated rows per seat and step range."""
 import numpy as np
 import pytest

@@ -95,3 +95,23 @@ def test_seat_swap_on_a_symmetric_start():
     lsm = torch.log_softmax(torch.from_numpy(z[:, :K]), -1).numpy()
     a1 = ab["actions"][0, :, 1].astype(np.int64)
     assert np.allclose(ab["logp_tm"][0], lsm[np.arange(N), a1], atol=1e-12)
+
+
+def test_seat1_rows_are_seat0_rows_with_the_level_channels_swapped():
+    """Seat 1's LBF observation differs from seat 0's only in which agent fills the
+    observer's and the other agent's level channels (0 and 1); food and empty cells are
+    the same for both.  The tensor-core IPPO collection writes seat 1's trajectory rows
+    from seat 0's by that swap, so it is checked here on the oracle's own rows, along
+    rollouts with auto-resets on the 7x7 and 12x12 grids."""
+    rng = np.random.default_rng(5)
+    for w, h in [(7, 7), (12, 12)]:
+        d = O.env_desc(O.LBF, w, h, 3, 3, 20)
+        od = 4 * w * h
+        pols = [rand_policy(rng, [od, 16, 16, 7]), rand_policy(rng, [od, 16, 16, 7])]
+        st = O.reset_all(d, 3, 64)
+        out = O.rollout(d, O.Policies(pols), 3, st, 0, 45, 0, [1])
+        assert out["rc"] == 0 and out["dones"].any()
+        rows0 = out["obs"].reshape(45, 64, w * h, 4)
+        rows1 = out["obs_tm"].reshape(45, 64, w * h, 4)
+        assert np.array_equal(rows1, rows0[..., [1, 0, 2, 3]])
+        assert (rows0[..., 0] > 0).sum(-1).min() == 1   # each row shows its observer once
