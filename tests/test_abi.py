@@ -79,3 +79,102 @@ def test_host_validation_needs_no_gpu(lib):
     assert L.aht_learner_create(196, 6, ptrs, ptrs, C.byref(bad_cfg), None, C.byref(out_l)) == aht.AHT_EINVAL
     assert L.aht_ppo_update(None, None, 64, 1, None) == aht.AHT_EINVAL
     assert L.aht_learner_n_params(None) == -1
+
+
+def test_null_handles_and_arguments_are_rejected_before_any_cuda_call(lib):
+    # Every entry point that takes a context, learner or S5 handle checks it (and its
+    # output pointers) on the host first: AHT_EINVAL and a message, no CUDA call, so
+    # none of this needs a GPU.  The destroy calls accept NULL.
+    import ctypes as C
+    from paper_2609_13716_gb300 import aht
+    L = aht.load()
+    E = aht.AHT_EINVAL
+    fake = C.c_void_p(16)  # never dereferenced: each call fails a host check first
+    t = aht.Traj()
+    i32 = C.c_int32
+    ids = (i32 * 2)(0, 1)
+    calls = {
+        "aht_sync": lambda: L.aht_sync(None),
+        "aht_set_timing": lambda: L.aht_set_timing(None, 1),
+        "aht_get_timing": lambda: L.aht_get_timing(None, None, None),
+        "aht_get_state": lambda: L.aht_get_state(None, None, None),
+        "aht_set_state": lambda: L.aht_set_state(None, None, 0),
+        "aht_set_policy": lambda: L.aht_set_policy(None, 0, None, None, 0, 0),
+        "aht_step_forced": lambda: L.aht_step_forced(None, None, None),
+        "aht_policy_forward": lambda: L.aht_policy_forward(None, 0, None, 1, None),
+        "aht_rollout_ippo": lambda: L.aht_rollout_ippo(None, 0, 1, 4, C.byref(t), C.byref(t)),
+        "aht_rollout_resample": lambda: L.aht_rollout_resample(None, 0, ids, 2, 4, C.byref(t), None),
+        "aht_debug_expire_at": lambda: L.aht_debug_expire_at(None, 1, 1000),
+        "aht_debug_logits": lambda: L.aht_debug_logits(None, None, 0),
+        "aht_learner_get": lambda: L.aht_learner_get(None, None, None, None, None, None),
+        "aht_learner_set": lambda: L.aht_learner_set(None, None, None, None, 0, 0),
+        "aht_learner_push": lambda: L.aht_learner_push(None, None, 0),
+        "aht_learner_sync": lambda: L.aht_learner_sync(None),
+        "aht_ppo_grad": lambda: L.aht_ppo_grad(None, C.byref(t), 1, 1, 0, 0, None, None),
+        "aht_s5_step": lambda: L.aht_s5_step(None, fake, fake, fake, 1, fake, fake, fake),
+        "aht_s5_sync": lambda: L.aht_s5_sync(None),
+    }
+    L.aht_xplay_matrix_static.argtypes = [C.c_void_p, C.POINTER(i32), i32, C.POINTER(i32), i32, i32,
+                                          i32, C.c_void_p]
+    L.aht_xplay_matrix_static.restype = C.c_int
+    calls["aht_xplay_matrix_static"] = lambda: L.aht_xplay_matrix_static(None, ids, 1, ids, 1, 4, 4, fake)
+    L.aht_debug_tanh.argtypes = [C.c_void_p, C.c_void_p, C.c_int64, C.c_void_p]
+    L.aht_debug_tanh.restype = C.c_int
+    calls["aht_debug_tanh"] = lambda: L.aht_debug_tanh(None, None, 4, None)
+    out = C.c_void_p(16)
+    calls["aht_s5_create (NULL params)"] = lambda: L.aht_s5_create(None, 16, None, C.byref(out))
+    calls["aht_s5_create (NULL out)"] = lambda: L.aht_s5_create(None, 16, None, None)
+    for name, call in calls.items():
+        assert call() == E, name
+        assert L.aht_last_error(), name
+    assert out.value is None  # aht_s5_create clears *out before it fails
+    L.aht_destroy(None)
+    L.aht_learner_destroy(None)
+    L.aht_s5_destroy(None)
+
+
+def test_s5_create_checks_its_sizes_and_arrays_on_the_host(lib):
+    # aht_s5_create validates the model sizes, max_envs, every parameter array and the
+    # sign of Re(lambda) (the S5 recurrence must decay) before it allocates or touches
+    # the device.
+    import ctypes as C
+    import numpy as np
+    from paper_2609_13716_gb300 import aht
+    L = aht.load()
+    keep = []
+
+    def arr(n, v=0.1):
+        a = np.full(n, v, np.float32)
+        keep.append(a)
+        return a.ctypes.data_as(C.POINTER(C.c_float))
+
+    def params(**kw):
+        p = aht.S5Params()
+        p.obs_dim, p.n_actions, p.H, p.P, p.F = 196, 6, 128, 128, 1024
+        for f in ("We1", "be1", "We2", "be2", "lam_im", "log_dt", "B_re", "B_im", "C_re", "C_im", "D"):
+            setattr(p, f, arr(4))
+        p.lam_re = arr(128, -0.5)
+        for l in range(4):
+            p.Wa[l], p.ba[l], p.Wc[l], p.bc[l] = arr(4), arr(4), arr(4), arr(4)
+        for k, v in kw.items():
+            setattr(p, k, v)
+        return p
+
+    out = C.c_void_p()
+    cases = [
+        (params(H=100), 16, b"multiples of 32"),
+        (params(P=160), 16, b"P <= 128"),
+        (params(n_actions=33), 16, b"n_actions"),
+        (params(obs_dim=0), 16, b"obs_dim"),
+        (params(), 0, b"max_envs"),
+        (params(), (1 << 20) + 1, b"max_envs"),
+        (params(D=None), 16, b"NULL parameter array"),
+        (params(lam_re=arr(128, 0.0)), 16, b"negative"),
+    ]
+    p = params()
+    p.Wc[3] = None
+    cases.append((p, 16, b"NULL head array"))
+    for prm, n, msg in cases:
+        assert L.aht_s5_create(C.byref(prm), n, None, C.byref(out)) == aht.AHT_EINVAL, msg
+        assert msg in L.aht_last_error(), (msg, L.aht_last_error())
+        assert out.value is None
